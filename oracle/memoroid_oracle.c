@@ -1,0 +1,419 @@
+/*
+ * memoroid_oracle.c -- plain fp64 CPU oracle for the resettable memoroid scans.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing on the product path links, loads or calls
+ * this file: only the test suite, the smoke check and the benchmark's CPU
+ * baseline use it.  It shares no code, header or constant with the CUDA path.
+ *
+ * Every routine is a direct, unblocked transcription of a definition from
+ * "Recurrent Reinforcement Learning with Memoroids" (arXiv 2402.09900):
+ *
+ *   - the memoroid state sequence h_t = e_I . f(P_0) . ... . f(P_t)
+ *     (Definition 3.1, the equation giving h_t and s_t);
+ *   - the resettable monoid transform (A,b) o (A',b') =
+ *     ((A (1-b') + e_I b') . A', b or b') with identity (e_I, 0) (Theorem 3.2),
+ *     read as a select: when b' = 1 the left operand is replaced by e_I;
+ *   - the S5 / LRU monoid (X,x) . (X',x') = (X'X, X'x + x') with e_I = (I, 0),
+ *     here with diagonal X (Appendix "Simplified State Space Models" and
+ *     "Linear Recurrent Unit");
+ *   - the Linear Transformer sum monoid (X + X') (Appendix "Linear
+ *     Transformer"), generalised with a per-step decay gamma_t that multiplies
+ *     the carried state, read out as y_t = S_t^T q_t.
+ *
+ * Conventions (readings of the paper, listed in the design notes):
+ *   - b_t = 1 on the first step of an episode (Section 2.1).
+ *   - Diagonal scan: within an episode h_t = lambda_t * h_{t-1} + u_t and the
+ *     head step keeps its own f(P): h_s = u_s.  A tape whose row begins with
+ *     b_0 = 0 continues an earlier episode from h0 (h0 = NULL means e_I = 0).
+ *   - Backward passes use PyTorch's complex-gradient convention
+ *     (grad = dL/dRe + i dL/dIm), for which the holomorphic chain rule of
+ *     z = a*w reads grad_w = conj(a) * grad_z.
+ *
+ * All routines return 0 on success and a negative value on a bad argument.
+ * Arrays are row-major; complex arrays are interleaved (re, im) doubles,
+ * i.e. C99 double complex.
+ */
+#include <complex.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+typedef double complex cplx;
+
+/* Thread count used by the parallel loops over independent channels, heads
+ * and tapes (1 when built without OpenMP). */
+void oracle_set_threads(int n)
+{
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+
+int oracle_max_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+/* ------------------------------------------------------------------------ */
+/* The resettable S5/LRU monoid for one diagonal channel (Theorem 3.2 applied
+ * to the diagonal S5/LRU monoid).  An element is ((a, x), b): a is the
+ * product of the lambdas, x the state, b the begin flag.                    */
+/* ------------------------------------------------------------------------ */
+
+void oracle_diag_combine(const double *left, int b_left, const double *right, int b_right,
+                         double *out, int *b_out)
+{
+    /* left, right, out: [a_re, a_im, x_re, x_im] */
+    cplx a = left[0] + I * left[1], x = left[2] + I * left[3];
+    cplx a2 = right[0] + I * right[1], x2 = right[2] + I * right[3];
+    cplx ra, rx;
+    if (b_right) {
+        /* (A,b) o (A',1) = (e_I . A', 1) = A'  (first row of the b'=1 cases) */
+        ra = a2;
+        rx = x2;
+    } else {
+        /* (A,b) o (A',0) = (A . A', b);  (a,x).(a',x') = (a' a, a' x + x') */
+        ra = a2 * a;
+        rx = a2 * x + x2;
+    }
+    out[0] = creal(ra); out[1] = cimag(ra);
+    out[2] = creal(rx); out[3] = cimag(rx);
+    *b_out = (b_left || b_right) ? 1 : 0;
+}
+
+/* lambda for tape b, step t, channel d */
+static inline cplx lam_at(const cplx *lambda, int per_step, int64_t b, int64_t t, int64_t L,
+                          int64_t D, int64_t d)
+{
+    return per_step ? lambda[(b * L + t) * D + d] : lambda[d];
+}
+
+/*
+ * Diagonal scan, forward: the definition, episode by episode.
+ * lambda: [D] or [B,L,D]; u, h: [B,L,D]; start: [B,L]; h0, h_last: [B,D] or NULL.
+ */
+int oracle_diag_fwd(int64_t B, int64_t L, int64_t D, const cplx *lambda, int lambda_per_step,
+                    const cplx *u, const uint8_t *start, const cplx *h0, cplx *h, cplx *h_last)
+{
+    if (B < 0 || L < 0 || D < 0) return -1;
+    if (L > 0 && (!lambda || !u || !start || !h)) return -1;
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int64_t b = 0; b < B; ++b) {
+        for (int64_t d = 0; d < D; ++d) {
+            int64_t s = 0;
+            while (s < L) {
+                /* episode [s, e): next begin flag after s, or the tape end */
+                int64_t e = s + 1;
+                while (e < L && !start[b * L + e]) ++e;
+                cplx prev;
+                if (start[b * L + s]) {
+                    prev = 0.0; /* e_I; unused: the head keeps its own f(P) */
+                } else {
+                    /* only possible at s = 0: a row that continues an episode */
+                    prev = h0 ? h0[b * D + d] : 0.0;
+                }
+                for (int64_t t = s; t < e; ++t) {
+                    cplx ut = u[(b * L + t) * D + d];
+                    cplx ht = (t == s && start[b * L + s])
+                                  ? ut
+                                  : lam_at(lambda, lambda_per_step, b, t, L, D, d) * prev + ut;
+                    h[(b * L + t) * D + d] = ht;
+                    prev = ht;
+                }
+                s = e;
+            }
+            if (h_last) {
+                h_last[b * D + d] = (L > 0) ? h[(b * L + L - 1) * D + d] : (h0 ? h0[b * D + d] : 0.0);
+            }
+        }
+    }
+    return 0;
+}
+
+/*
+ * Diagonal scan, forward, by folding the resettable combine from the identity
+ * g_I = (e_I, 0) (Definition 3.1 with Theorem 3.2).  The element lifted from
+ * step t is ((lambda_t, u_t), b_t).  A row that starts with b_0 = 0 folds from
+ * ((1, h0), 0) instead of g_I.
+ */
+int oracle_diag_fold(int64_t B, int64_t L, int64_t D, const cplx *lambda, int lambda_per_step,
+                     const cplx *u, const uint8_t *start, const cplx *h0, cplx *h)
+{
+    if (B < 0 || L < 0 || D < 0) return -1;
+    for (int64_t b = 0; b < B; ++b) {
+        for (int64_t d = 0; d < D; ++d) {
+            double acc[4] = {1.0, 0.0, h0 ? creal(h0[b * D + d]) : 0.0, h0 ? cimag(h0[b * D + d]) : 0.0};
+            int acc_b = 0;
+            for (int64_t t = 0; t < L; ++t) {
+                cplx l = lam_at(lambda, lambda_per_step, b, t, L, D, d);
+                cplx x = u[(b * L + t) * D + d];
+                double el[4] = {creal(l), cimag(l), creal(x), cimag(x)};
+                double out[4];
+                int ob;
+                oracle_diag_combine(acc, acc_b, el, start[b * L + t], out, &ob);
+                memcpy(acc, out, sizeof(acc));
+                acc_b = ob;
+                h[(b * L + t) * D + d] = acc[2] + I * acc[3];
+            }
+        }
+    }
+    return 0;
+}
+
+/*
+ * Diagonal scan, backward (reverse-mode of the forward definition).
+ * Inputs: the forward's h [B,L,D], upstream g = dL/dh [B,L,D], g_last =
+ * dL/dh_last [B,D] or NULL.  The adjoint of h_t is
+ *     delta_t = g_t + [b_{t+1} = 0] conj(lambda_{t+1}) delta_{t+1},
+ *     delta_{L-1} = g_{L-1} + g_last,
+ * and grad_u_t = delta_t, grad_lambda_t = [b_t = 0] delta_t conj(h_{t-1})
+ * (h_{-1} = h0, or 0 when h0 is NULL), grad_h0 = [b_0 = 0] conj(lambda_0) delta_0.
+ * grad_lambda is [D] (summed over B and L) for a per-channel lambda and
+ * [B,L,D] for a per-step lambda.  Any output may be NULL to skip it.
+ */
+int oracle_diag_bwd(int64_t B, int64_t L, int64_t D, const cplx *lambda, int lambda_per_step,
+                    const uint8_t *start, const cplx *h0, const cplx *h, const cplx *g,
+                    const cplx *g_last, cplx *grad_u, cplx *grad_lambda, cplx *grad_h0)
+{
+    if (B < 0 || L < 0 || D < 0) return -1;
+    if (grad_lambda && !lambda_per_step) {
+        for (int64_t d = 0; d < D; ++d) grad_lambda[d] = 0.0;
+    }
+#pragma omp parallel for schedule(static)
+    for (int64_t d = 0; d < D; ++d) {
+        cplx lam_sum = 0.0;
+        for (int64_t b = 0; b < B; ++b) {
+            cplx delta_next = 0.0; /* delta_{t+1} */
+            for (int64_t t = L - 1; t >= 0; --t) {
+                cplx delta = g[(b * L + t) * D + d];
+                if (t == L - 1) {
+                    if (g_last) delta += g_last[b * D + d];
+                } else if (!start[b * L + t + 1]) {
+                    delta += conj(lam_at(lambda, lambda_per_step, b, t + 1, L, D, d)) * delta_next;
+                }
+                if (grad_u) grad_u[(b * L + t) * D + d] = delta;
+                if (grad_lambda) {
+                    cplx gl = 0.0;
+                    if (!start[b * L + t]) {
+                        cplx hprev = (t > 0) ? h[(b * L + t - 1) * D + d] : (h0 ? h0[b * D + d] : 0.0);
+                        gl = delta * conj(hprev);
+                    }
+                    if (lambda_per_step) grad_lambda[(b * L + t) * D + d] = gl;
+                    else lam_sum += gl;
+                }
+                delta_next = delta;
+            }
+            if (grad_h0) {
+                grad_h0[b * D + d] = (L > 0 && !start[b * L])
+                                         ? conj(lam_at(lambda, lambda_per_step, b, 0, L, D, d)) * delta_next
+                                         : (L == 0 && g_last ? g_last[b * D + d] : 0.0);
+            }
+        }
+        if (grad_lambda && !lambda_per_step) grad_lambda[d] = lam_sum;
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Decayed linear-attention memoroid.                                        */
+/*   S_t = [b_t = 0] gamma_t S_{t-1} + k_t v_t^T,   y_t = S_t^T q_t           */
+/* (sum monoid of the Linear Transformer with a multiplicative decay on the  */
+/* carried state; the head step of an episode starts from e_I = 0).          */
+/* ------------------------------------------------------------------------ */
+
+static inline double gam_at(const double *gamma, int per_step, int64_t b, int64_t t, int64_t L,
+                            int64_t H, int64_t hh)
+{
+    return per_step ? gamma[(b * L + t) * H + hh] : gamma[hh];
+}
+
+/*
+ * q, k: [B,L,H,dk]; v: [B,L,H,dv]; gamma: [H] or [B,L,H]; start: [B,L];
+ * S0, S_last: [B,H,dk,dv] or NULL; y: [B,L,H,dv].
+ */
+int oracle_linattn_fwd(int64_t B, int64_t L, int64_t H, int64_t dk, int64_t dv, const double *q,
+                       const double *k, const double *v, const double *gamma, int gamma_per_step,
+                       const uint8_t *start, const double *S0, double *y, double *S_last)
+{
+    if (B < 0 || L < 0 || H < 0 || dk <= 0 || dv <= 0) return -1;
+#pragma omp parallel for collapse(2) schedule(dynamic)
+    for (int64_t b = 0; b < B; ++b) {
+        for (int64_t hh = 0; hh < H; ++hh) {
+            double *S = (double *)calloc((size_t)(dk * dv), sizeof(double));
+            if (S0) memcpy(S, S0 + (b * H + hh) * dk * dv, sizeof(double) * dk * dv);
+            for (int64_t t = 0; t < L; ++t) {
+                const double *kt = k + ((b * L + t) * H + hh) * dk;
+                const double *vt = v + ((b * L + t) * H + hh) * dv;
+                const double *qt = q + ((b * L + t) * H + hh) * dk;
+                double gt = start[b * L + t] ? 0.0 : gam_at(gamma, gamma_per_step, b, t, L, H, hh);
+                for (int64_t i = 0; i < dk; ++i)
+                    for (int64_t j = 0; j < dv; ++j)
+                        S[i * dv + j] = (start[b * L + t] ? 0.0 : gt * S[i * dv + j]) + kt[i] * vt[j];
+                double *yt = y + ((b * L + t) * H + hh) * dv;
+                for (int64_t j = 0; j < dv; ++j) {
+                    double acc = 0.0;
+                    for (int64_t i = 0; i < dk; ++i) acc += S[i * dv + j] * qt[i];
+                    yt[j] = acc;
+                }
+            }
+            if (S_last) memcpy(S_last + (b * H + hh) * dk * dv, S, sizeof(double) * dk * dv);
+            free(S);
+        }
+    }
+    return 0;
+}
+
+/*
+ * Backward of oracle_linattn_fwd, by the transposed recurrence:
+ *   dS_t = q_t dy_t^T + [b_{t+1} = 0] gamma_{t+1} dS_{t+1}   (dS_{L-1} += dS_last)
+ *   dq_t = S_t dy_t,  dk_t = dS_t v_t,  dv_t = dS_t^T k_t,
+ *   dgamma_t = [b_t = 0] <dS_t, S_{t-1}>_F,  dS0 = [b_0 = 0] gamma_0 dS_0.
+ * The forward states of each episode are recomputed and kept for the reverse
+ * sweep.  dgamma is [H] (summed over B, L) or [B,L,H] for a per-step gamma.
+ * Any output may be NULL.
+ */
+int oracle_linattn_bwd(int64_t B, int64_t L, int64_t H, int64_t dk, int64_t dv, const double *q,
+                       const double *k, const double *v, const double *gamma, int gamma_per_step,
+                       const uint8_t *start, const double *S0, const double *dy,
+                       const double *dS_last, double *dq, double *dkk, double *dvv, double *dgamma,
+                       double *dS0)
+{
+    if (B < 0 || L < 0 || H < 0 || dk <= 0 || dv <= 0) return -1;
+    const int64_t M = dk * dv;
+    double *gsum = NULL;
+    if (dgamma && !gamma_per_step) {
+        gsum = (double *)calloc((size_t)(B * H > 0 ? B * H : 1), sizeof(double));
+    }
+    int bad = 0;
+#pragma omp parallel for collapse(2) schedule(dynamic)
+    for (int64_t b = 0; b < B; ++b) {
+        for (int64_t hh = 0; hh < H; ++hh) {
+            double *dS = (double *)calloc((size_t)M, sizeof(double));
+            double gacc = 0.0;
+            /* episodes in reverse order; [s, e) */
+            int64_t e = L;
+            while (e > 0) {
+                int64_t s = e - 1;
+                while (s > 0 && !start[b * L + s]) --s;
+                const int64_t n = e - s;
+                /* states S_{s-1} .. S_{e-1}: slot 0 holds the incoming state */
+                double *St = (double *)calloc((size_t)((n + 1) * M), sizeof(double));
+                if (!St) { bad = 1; break; }
+                if (!start[b * L + s] && S0) memcpy(St, S0 + (b * H + hh) * M, sizeof(double) * M);
+                for (int64_t t = s; t < e; ++t) {
+                    const double *kt = k + ((b * L + t) * H + hh) * dk;
+                    const double *vt = v + ((b * L + t) * H + hh) * dv;
+                    double gt = start[b * L + t] ? 0.0 : gam_at(gamma, gamma_per_step, b, t, L, H, hh);
+                    double *prev = St + (t - s) * M, *cur = St + (t - s + 1) * M;
+                    for (int64_t i = 0; i < dk; ++i)
+                        for (int64_t j = 0; j < dv; ++j)
+                            cur[i * dv + j] = (start[b * L + t] ? 0.0 : gt * prev[i * dv + j]) + kt[i] * vt[j];
+                }
+                /* reverse sweep */
+                for (int64_t t = e - 1; t >= s; --t) {
+                    const double *kt = k + ((b * L + t) * H + hh) * dk;
+                    const double *vt = v + ((b * L + t) * H + hh) * dv;
+                    const double *qt = q + ((b * L + t) * H + hh) * dk;
+                    const double *dyt = dy + ((b * L + t) * H + hh) * dv;
+                    if (t == e - 1) {
+                        /* the step after e-1 starts a new episode (or is past the tape) */
+                        for (int64_t x = 0; x < M; ++x) dS[x] = 0.0;
+                        if (e == L && dS_last) memcpy(dS, dS_last + (b * H + hh) * M, sizeof(double) * M);
+                    } else {
+                        double gn = gam_at(gamma, gamma_per_step, b, t + 1, L, H, hh);
+                        for (int64_t x = 0; x < M; ++x) dS[x] *= gn;
+                    }
+                    for (int64_t i = 0; i < dk; ++i)
+                        for (int64_t j = 0; j < dv; ++j) dS[i * dv + j] += qt[i] * dyt[j];
+                    const double *Scur = St + (t - s + 1) * M, *Sprev = St + (t - s) * M;
+                    if (dq) {
+                        double *o = dq + ((b * L + t) * H + hh) * dk;
+                        for (int64_t i = 0; i < dk; ++i) {
+                            double acc = 0.0;
+                            for (int64_t j = 0; j < dv; ++j) acc += Scur[i * dv + j] * dyt[j];
+                            o[i] = acc;
+                        }
+                    }
+                    if (dkk) {
+                        double *o = dkk + ((b * L + t) * H + hh) * dk;
+                        for (int64_t i = 0; i < dk; ++i) {
+                            double acc = 0.0;
+                            for (int64_t j = 0; j < dv; ++j) acc += dS[i * dv + j] * vt[j];
+                            o[i] = acc;
+                        }
+                    }
+                    if (dvv) {
+                        double *o = dvv + ((b * L + t) * H + hh) * dv;
+                        for (int64_t j = 0; j < dv; ++j) {
+                            double acc = 0.0;
+                            for (int64_t i = 0; i < dk; ++i) acc += dS[i * dv + j] * kt[i];
+                            o[j] = acc;
+                        }
+                    }
+                    double dg = 0.0;
+                    if (!start[b * L + t]) {
+                        for (int64_t x = 0; x < M; ++x) dg += dS[x] * Sprev[x];
+                    }
+                    if (dgamma) {
+                        if (gamma_per_step) dgamma[(b * L + t) * H + hh] = dg;
+                        else gacc += dg;
+                    }
+                }
+                if (s == 0 && dS0) {
+                    double *o = dS0 + (b * H + hh) * M;
+                    double g0 = gam_at(gamma, gamma_per_step, b, 0, L, H, hh);
+                    for (int64_t x = 0; x < M; ++x) o[x] = start[b * L] ? 0.0 : g0 * dS[x];
+                }
+                free(St);
+                e = s;
+            }
+            if (L == 0 && dS0) {
+                double *o = dS0 + (b * H + hh) * M;
+                for (int64_t x = 0; x < M; ++x) o[x] = dS_last ? dS_last[(b * H + hh) * M + x] : 0.0;
+            }
+            if (gsum) gsum[b * H + hh] = gacc;
+            free(dS);
+        }
+    }
+    if (gsum) {
+        for (int64_t hh = 0; hh < H; ++hh) {
+            double acc = 0.0;
+            for (int64_t b = 0; b < B; ++b) acc += gsum[b * H + hh];
+            dgamma[hh] = acc;
+        }
+        free(gsum);
+    }
+    return bad ? -2 : 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Episode index list I <-> begin flags (Algorithm 1: I = where(b)).         */
+/* ------------------------------------------------------------------------ */
+
+int oracle_starts_from_offsets(const int64_t *offsets, int64_t E, int64_t L, uint8_t *start)
+{
+    if (E < 0 || L < 0) return -1;
+    for (int64_t t = 0; t < L; ++t) start[t] = 0;
+    for (int64_t i = 0; i < E; ++i) {
+        if (offsets[i] >= 0 && offsets[i] < L) start[offsets[i]] = 1;
+    }
+    return 0;
+}
+
+int64_t oracle_offsets_from_starts(const uint8_t *start, int64_t L, int64_t *offsets)
+{
+    int64_t n = 0;
+    for (int64_t t = 0; t < L; ++t) {
+        if (start[t]) offsets[n++] = t;
+    }
+    return n;
+}

@@ -1,0 +1,519 @@
+"""Pins of the fp64 oracle against facts that do not come from the oracle.
+
+Each test checks the oracle against something the paper or mathematics fixes:
+the case table of Theorem 3.2's proof, hand-worked examples, closed forms,
+library routines (scipy.signal.lfilter, numpy.cumsum, numpy matmul), brute
+force, torch.autograd in float64 through an independent loop, and central
+finite differences.
+"""
+import os
+
+import numpy as np
+import pytest
+import scipy.signal
+
+import oracle
+import tapegen
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rng(seed=0):
+    return np.random.default_rng(seed)
+
+
+def _rand_c(rng, *shape):
+    return rng.standard_normal(shape) + 1j * rng.standard_normal(shape)
+
+
+def _rand_lam(rng, *shape):
+    return rng.uniform(0.3, 0.99, shape) * np.exp(1j * rng.uniform(0, 2 * np.pi, shape))
+
+
+def _random_starts(rng, B, L, p=0.15, first=True):
+    s = (rng.random((B, L)) < p).astype(np.uint8)
+    if first and L:
+        s[:, 0] = 1
+    return s
+
+
+# ---------------------------------------------------------------------------
+# the resettable combine (Theorem 3.2)
+# ---------------------------------------------------------------------------
+
+def _s5(e1, e2):
+    # S5/LRU monoid with diagonal X (Appendix "Simplified State Space Models"):
+    # (X, x) . (X', x') = (X' X, X' x + x'), applied to one channel.
+    return (e2[0] * e1[0], e2[0] * e1[1] + e2[1])
+
+
+def _read_table():
+    rows = []
+    with open(os.path.join(GOLDEN, "resettable_cases.txt")) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                rows.append(line.split())
+    return rows
+
+
+def test_combine_case_table():
+    rng = _rng(1)
+    table = _read_table()
+    assert sum(r[0] == "pair" for r in table) == 4 and sum(r[0] == "triple" for r in table) == 8
+    for _ in range(5):
+        A, A1, A2 = [(complex(*rng.standard_normal(2)), complex(*rng.standard_normal(2))) for _ in range(3)]
+        eI = (1.0 + 0j, 0j)
+        expect_elems = {
+            "AA'": _s5(A, A1), "eA'": _s5(eI, A1),
+            "AA'A''": _s5(_s5(A, A1), A2), "eA'A''": _s5(_s5(eI, A1), A2), "eA''": _s5(eI, A2),
+        }
+        for row in table:
+            if row[0] == "pair":
+                b, b1 = int(row[1]), int(row[2])
+                got, gb = oracle.diag_combine(A, b, A1, b1)
+                res, flag = row[3], int(row[4])
+            else:
+                b, b1, b2 = int(row[1]), int(row[2]), int(row[3])
+                left, lb = oracle.diag_combine(A, b, A1, b1)
+                got, gb = oracle.diag_combine(left, lb, A2, b2)
+                res, flag = row[4], int(row[5])
+            assert gb == flag
+            np.testing.assert_allclose(np.array(got), np.array(expect_elems[res]), rtol=1e-13, atol=1e-13)
+
+
+def test_combine_associative_all_flag_patterns():
+    rng = _rng(2)
+    for trial in range(200):
+        els = [(complex(*rng.standard_normal(2)), complex(*rng.standard_normal(2))) for _ in range(3)]
+        for pattern in range(8):
+            fl = [(pattern >> i) & 1 for i in range(3)]
+            l1, lb1 = oracle.diag_combine(els[0], fl[0], els[1], fl[1])
+            left, lb = oracle.diag_combine(l1, lb1, els[2], fl[2])
+            r1, rb1 = oracle.diag_combine(els[1], fl[1], els[2], fl[2])
+            right, rb = oracle.diag_combine(els[0], fl[0], r1, rb1)
+            assert lb == rb
+            scale = max(1.0, max(abs(z) for z in left + right))
+            assert max(abs(a - b) for a, b in zip(left, right)) <= 1e-12 * scale
+
+
+def test_combine_identity_exact():
+    rng = _rng(3)
+    gI = ((1.0 + 0j, 0j), 0)
+    for _ in range(50):
+        e = (complex(*rng.standard_normal(2)), complex(*rng.standard_normal(2)))
+        for b in (0, 1):
+            got, gb = oracle.diag_combine(gI[0], gI[1], e, b)
+            assert got == e and gb == b
+            got, gb = oracle.diag_combine(e, b, gI[0], gI[1])
+            assert got == e and gb == b
+
+
+# ---------------------------------------------------------------------------
+# diagonal scan, forward
+# ---------------------------------------------------------------------------
+
+def test_diag_worked_example():
+    vals = {}
+    with open(os.path.join(GOLDEN, "diag_worked_example.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                k, *v = line.split()
+                vals[k] = [float(x) for x in v]
+    lam = np.array([vals["lambda"][0]], dtype=np.complex128)
+    u = np.array(vals["u"], dtype=np.complex128).reshape(1, -1, 1)
+    start = np.array(vals["start"], dtype=np.uint8).reshape(1, -1)
+    h, h_last = oracle.diag_fwd(lam, u, start)
+    np.testing.assert_array_equal(h.reshape(-1).real, np.array(vals["h"]))
+    assert h_last[0, 0] == vals["h"][-1]
+
+
+def _closed_form(lam, u, start, h0=None):
+    # h_t = sum_{r=s}^{t} (prod_{j=r+1}^{t} lambda_j) u_r over t's episode [s, ..],
+    # plus (prod_{j=0}^{t} lambda_j) h0 for a row that continues an episode.
+    B, L, D = u.shape
+    per_step = lam.ndim == 3
+    out = np.zeros((B, L, D), dtype=np.complex128)
+    for b in range(B):
+        for t in range(L):
+            s = t
+            while s > 0 and not start[b, s]:
+                s -= 1
+            for d in range(D):
+                lams = lam[b, :, d] if per_step else np.full(L, lam[d])
+                acc = 0j
+                for r in range(s, t + 1):
+                    acc += np.prod(lams[r + 1:t + 1]) * u[b, r, d]
+                if s == 0 and not start[b, 0] and h0 is not None:
+                    acc += np.prod(lams[0:t + 1]) * h0[b, d]
+                out[b, t, d] = acc
+    return out
+
+
+@pytest.mark.parametrize("per_step", [False, True])
+@pytest.mark.parametrize("first", [True, False])
+def test_diag_fwd_closed_form(per_step, first):
+    rng = _rng(4)
+    B, L, D = 2, 40, 3
+    lam = _rand_lam(rng, B, L, D) if per_step else _rand_lam(rng, D)
+    u = _rand_c(rng, B, L, D)
+    start = _random_starts(rng, B, L, 0.12, first=first)
+    h0 = _rand_c(rng, B, D)
+    h, h_last = oracle.diag_fwd(lam, u, start, h0)
+    ref = _closed_form(lam, u, start, h0)
+    np.testing.assert_allclose(h, ref, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(h_last, ref[:, -1], rtol=1e-12, atol=1e-12)
+
+
+def test_diag_lambda_zero_is_identity_map():
+    rng = _rng(5)
+    u = _rand_c(rng, 2, 50, 4)
+    start = _random_starts(rng, 2, 50)
+    h, _ = oracle.diag_fwd(np.zeros(4, np.complex128), u, start)
+    np.testing.assert_array_equal(h, u)
+
+
+def test_diag_lambda_one_is_segmented_cumsum():
+    rng = _rng(6)
+    B, L, D = 3, 200, 5
+    u = _rand_c(rng, B, L, D)
+    start = _random_starts(rng, B, L, 0.05)
+    h, _ = oracle.diag_fwd(np.ones(D, np.complex128), u, start)
+    for b in range(B):
+        for s, e in tapegen.episode_bounds(start[b]):
+            np.testing.assert_allclose(h[b, s:e], np.cumsum(u[b, s:e], axis=0), rtol=1e-12, atol=1e-12)
+
+
+def test_diag_matches_lfilter_per_episode():
+    # h_t = lambda h_{t-1} + u_t is the IIR filter b = [1], a = [1, -lambda].
+    rng = _rng(7)
+    B, L, D = 2, 3000, 6
+    lam = _rand_lam(rng, D)
+    u = _rand_c(rng, B, L, D)
+    start = _random_starts(rng, B, L, 0.01)
+    h, _ = oracle.diag_fwd(lam, u, start)
+    for b in range(B):
+        for s, e in tapegen.episode_bounds(start[b]):
+            for d in range(D):
+                ref = scipy.signal.lfilter([1.0], [1.0, -lam[d]], u[b, s:e, d])
+                np.testing.assert_allclose(h[b, s:e, d], ref, rtol=1e-11, atol=1e-11)
+
+
+def test_diag_fold_matches_definition():
+    rng = _rng(8)
+    for per_step in (False, True):
+        B, L, D = 2, 300, 4
+        lam = _rand_lam(rng, B, L, D) if per_step else _rand_lam(rng, D)
+        u = _rand_c(rng, B, L, D)
+        start = _random_starts(rng, B, L, 0.05, first=False)
+        h0 = _rand_c(rng, B, D)
+        h, _ = oracle.diag_fwd(lam, u, start, h0)
+        hf = oracle.diag_fold(lam, u, start, h0)
+        np.testing.assert_allclose(hf, h, rtol=1e-12, atol=1e-12)
+
+
+def test_diag_all_start_and_reset_invariant():
+    rng = _rng(9)
+    B, L, D = 2, 64, 4
+    lam = _rand_lam(rng, D)
+    u = _rand_c(rng, B, L, D)
+    h, _ = oracle.diag_fwd(lam, u, np.ones((B, L), np.uint8))
+    np.testing.assert_array_equal(h, u)
+    # tape over many episodes == each episode scanned on its own
+    start = _random_starts(rng, B, L, 0.2)
+    h, _ = oracle.diag_fwd(lam, u, start)
+    for b in range(B):
+        for s, e in tapegen.episode_bounds(start[b]):
+            one, _ = oracle.diag_fwd(lam, u[b:b + 1, s:e], np.eye(1, e - s, dtype=np.uint8))
+            np.testing.assert_array_equal(one[0], h[b, s:e])
+
+
+def test_diag_tbb_equals_sbb_for_equal_lengths():
+    # With every episode exactly L_ep long, the tape equals a [E, L_ep] batch
+    # of independent segments (Section 5, TBB vs SBB).
+    rng = _rng(10)
+    E, Lep, D = 7, 13, 3
+    lam = _rand_lam(rng, D)
+    u = _rand_c(rng, 1, E * Lep, D)
+    start = np.zeros((1, E * Lep), np.uint8)
+    start[0, ::Lep] = 1
+    h_tape, _ = oracle.diag_fwd(lam, u, start)
+    sb = np.zeros((E, Lep), np.uint8)
+    sb[:, 0] = 1
+    h_seg, _ = oracle.diag_fwd(lam, u.reshape(E, Lep, D), sb)
+    np.testing.assert_array_equal(h_tape.reshape(E, Lep, D), h_seg)
+
+
+def test_diag_split_resume():
+    rng = _rng(11)
+    B, L, D = 2, 100, 3
+    lam = _rand_lam(rng, D)
+    u = _rand_c(rng, B, L, D)
+    start = _random_starts(rng, B, L, 0.05)
+    start[:, 50] = 0
+    h, h_last = oracle.diag_fwd(lam, u, start)
+    h1, hl1 = oracle.diag_fwd(lam, u[:, :50], start[:, :50])
+    h2, hl2 = oracle.diag_fwd(lam, u[:, 50:], start[:, 50:], h0=hl1)
+    np.testing.assert_allclose(np.concatenate([h1, h2], 1), h, rtol=1e-13, atol=1e-13)
+    np.testing.assert_allclose(hl2, h_last, rtol=1e-13, atol=1e-13)
+
+
+# ---------------------------------------------------------------------------
+# diagonal scan, backward
+# ---------------------------------------------------------------------------
+
+def _torch_diag_loss(torch, lam, u, start, h0, g, g_last, per_step):
+    # An independent forward loop in torch (complex128): h_t = lambda h_{t-1} + u_t,
+    # h_t = u_t at begin flags; loss = sum Re(conj(g) h) + Re(conj(g_last) h_last),
+    # whose torch-convention gradient w.r.t. h is g.
+    B, L, D = u.shape
+    loss = 0.0
+    for b in range(B):
+        prev = h0[b] if h0 is not None else torch.zeros(D, dtype=torch.complex128)
+        for t in range(L):
+            lt = lam[b, t] if per_step else lam
+            cur = u[b, t] if start[b, t] else lt * prev + u[b, t]
+            loss = loss + (torch.conj(g[b, t]) * cur).real.sum()
+            prev = cur
+        loss = loss + (torch.conj(g_last[b]) * prev).real.sum()
+    return loss
+
+
+@pytest.mark.parametrize("per_step", [False, True])
+@pytest.mark.parametrize("first", [True, False])
+def test_diag_bwd_vs_torch_autograd(per_step, first):
+    torch = pytest.importorskip("torch")
+    rng = _rng(12)
+    B, L, D = 2, 24, 3
+    lam = _rand_lam(rng, B, L, D) if per_step else _rand_lam(rng, D)
+    u = _rand_c(rng, B, L, D)
+    start = _random_starts(rng, B, L, 0.2, first=first)
+    start[0, 5] = 1
+    start[0, 6] = 1
+    h0 = _rand_c(rng, B, D)
+    g = _rand_c(rng, B, L, D)
+    g_last = _rand_c(rng, B, D)
+    tl = torch.tensor(lam, requires_grad=True)
+    tu = torch.tensor(u, requires_grad=True)
+    th0 = torch.tensor(h0, requires_grad=True)
+    loss = _torch_diag_loss(torch, tl, tu, start, th0, torch.tensor(g), torch.tensor(g_last), per_step)
+    loss.backward()
+    h, _ = oracle.diag_fwd(lam, u, start, h0)
+    gu, glam, gh0 = oracle.diag_bwd(lam, start, h, g, g_last, h0)
+    np.testing.assert_allclose(gu, tu.grad.numpy(), rtol=1e-11, atol=1e-11)
+    np.testing.assert_allclose(glam, tl.grad.numpy(), rtol=1e-11, atol=1e-11)
+    ref_h0 = np.zeros_like(gh0) if th0.grad is None else th0.grad.numpy()
+    np.testing.assert_allclose(gh0, ref_h0, rtol=1e-11, atol=1e-11)
+
+
+def test_diag_bwd_finite_differences():
+    rng = _rng(13)
+    B, L, D = 1, 12, 2
+    lam = _rand_lam(rng, D)
+    u = _rand_c(rng, B, L, D)
+    start = np.zeros((B, L), np.uint8)
+    start[0, [4, 9]] = 1  # row continues an episode from h0, then two resets
+    h0 = _rand_c(rng, B, D)
+    g = _rand_c(rng, B, L, D)
+    g_last = _rand_c(rng, B, D)
+
+    def loss(lam_, u_, h0_):
+        h, hl = oracle.diag_fwd(lam_, u_, start, h0_)
+        return float(np.sum((np.conj(g) * h).real) + np.sum((np.conj(g_last) * hl).real))
+
+    h, _ = oracle.diag_fwd(lam, u, start, h0)
+    gu, glam, gh0 = oracle.diag_bwd(lam, start, h, g, g_last, h0)
+    eps = 1e-6
+
+    def fd(arr, idx, f):
+        out = 0j
+        for part, unit in ((0, 1.0), (1, 1j)):
+            a1, a2 = arr.copy(), arr.copy()
+            a1[idx] += eps * unit
+            a2[idx] -= eps * unit
+            d = (f(a1) - f(a2)) / (2 * eps)
+            out += d if part == 0 else 1j * d
+        return out
+
+    for idx in [(0, 0, 0), (0, 3, 1), (0, 4, 0), (0, 8, 1), (0, 11, 0)]:
+        assert abs(fd(u, idx, lambda a: loss(lam, a, h0)) - gu[idx]) < 1e-6
+    for d in range(D):
+        assert abs(fd(lam, (d,), lambda a: loss(a, u, h0)) - glam[d]) < 1e-6
+        assert abs(fd(h0, (0, d), lambda a: loss(lam, u, a)) - gh0[0, d]) < 1e-6
+
+
+# ---------------------------------------------------------------------------
+# linear attention, forward
+# ---------------------------------------------------------------------------
+
+def _la_inputs(rng, B, L, H, dk, dv, per_step, p=0.1, first=True):
+    q = rng.standard_normal((B, L, H, dk)) * 0.5
+    k = rng.standard_normal((B, L, H, dk)) * 0.5
+    v = rng.standard_normal((B, L, H, dv)) * 0.5
+    gamma = rng.uniform(0.5, 1.0, (B, L, H)) if per_step else rng.uniform(0.5, 1.0, H)
+    start = _random_starts(rng, B, L, p, first=first)
+    return q, k, v, gamma, start
+
+
+def _la_brute(q, k, v, gamma, start, S0=None):
+    # y_t = sum_{r in ep(t), r <= t} (prod_{j=r+1}^{t} gamma_j) (q_t . k_r) v_r
+    #       (+ (prod_{j=0}^{t} gamma_j) S0^T q_t for a row continuing an episode)
+    B, L, H, dk = q.shape
+    per_step = gamma.ndim == 3
+    y = np.zeros(v.shape)
+    for b in range(B):
+        for h in range(H):
+            gam = gamma[b, :, h] if per_step else np.full(L, gamma[h])
+            for t in range(L):
+                s = t
+                while s > 0 and not start[b, s]:
+                    s -= 1
+                for r in range(s, t + 1):
+                    y[b, t, h] += np.prod(gam[r + 1:t + 1]) * (q[b, t, h] @ k[b, r, h]) * v[b, r, h]
+                if s == 0 and not start[b, 0] and S0 is not None:
+                    y[b, t, h] += np.prod(gam[0:t + 1]) * (S0[b, h].T @ q[b, t, h])
+    return y
+
+
+@pytest.mark.parametrize("per_step", [False, True])
+@pytest.mark.parametrize("first", [True, False])
+def test_linattn_fwd_brute_force(per_step, first):
+    rng = _rng(20)
+    B, L, H, dk, dv = 2, 30, 2, 3, 4
+    q, k, v, gamma, start = _la_inputs(rng, B, L, H, dk, dv, per_step, first=first)
+    S0 = rng.standard_normal((B, H, dk, dv))
+    y, S_last = oracle.linattn_fwd(q, k, v, gamma, start, S0)
+    np.testing.assert_allclose(y, _la_brute(q, k, v, gamma, start, S0), rtol=1e-11, atol=1e-11)
+    # S_last: the decayed sum of outer products of the last episode
+    for b in range(B):
+        for h in range(H):
+            s = L - 1
+            while s > 0 and not start[b, s]:
+                s -= 1
+            gam = gamma[b, :, h] if per_step else np.full(L, gamma[h])
+            ref = sum(np.prod(gam[r + 1:L]) * np.outer(k[b, r, h], v[b, r, h]) for r in range(s, L))
+            if s == 0 and not start[b, 0]:
+                ref = ref + np.prod(gam[0:L]) * S0[b, h]
+            np.testing.assert_allclose(S_last[b, h], ref, rtol=1e-11, atol=1e-11)
+
+
+def test_linattn_gamma_one_is_causal_attention():
+    rng = _rng(21)
+    B, L, H, d = 1, 300, 2, 8
+    q, k, v, _, start = _la_inputs(rng, B, L, H, d, d, False, p=0.02)
+    y, _ = oracle.linattn_fwd(q, k, v, np.ones(H), start)
+    for s, e in tapegen.episode_bounds(start[0]):
+        for h in range(H):
+            Q, K, V = q[0, s:e, h], k[0, s:e, h], v[0, s:e, h]
+            ref = np.tril(Q @ K.T) @ V
+            np.testing.assert_allclose(y[0, s:e, h], ref, rtol=1e-10, atol=1e-10)
+
+
+def test_linattn_all_start():
+    rng = _rng(22)
+    q, k, v, gamma, _ = _la_inputs(rng, 2, 20, 2, 4, 3, True)
+    y, _ = oracle.linattn_fwd(q, k, v, gamma, np.ones((2, 20), np.uint8))
+    ref = np.einsum("blhi,blhi->blh", q, k)[..., None] * v
+    np.testing.assert_allclose(y, ref, rtol=1e-13, atol=1e-13)
+
+
+# ---------------------------------------------------------------------------
+# linear attention, backward
+# ---------------------------------------------------------------------------
+
+def _torch_la_loss(torch, q, k, v, gamma, start, S0, dy, dS_last, per_step):
+    B, L, H, dk = q.shape
+    dv = v.shape[-1]
+    loss = 0.0
+    for b in range(B):
+        for h in range(H):
+            S = S0[b, h] if S0 is not None else torch.zeros(dk, dv, dtype=torch.float64)
+            for t in range(L):
+                g = gamma[b, t, h] if per_step else gamma[h]
+                kv = torch.outer(k[b, t, h], v[b, t, h])
+                S = kv if start[b, t] else g * S + kv
+                loss = loss + (dy[b, t, h] * (S.T @ q[b, t, h])).sum()
+            loss = loss + (dS_last[b, h] * S).sum()
+    return loss
+
+
+@pytest.mark.parametrize("per_step", [False, True])
+@pytest.mark.parametrize("first", [True, False])
+def test_linattn_bwd_vs_torch_autograd(per_step, first):
+    torch = pytest.importorskip("torch")
+    rng = _rng(23)
+    B, L, H, dk, dv = 2, 16, 2, 3, 2
+    q, k, v, gamma, start = _la_inputs(rng, B, L, H, dk, dv, per_step, p=0.2, first=first)
+    start[0, 7] = 1
+    start[0, 8] = 1
+    S0 = rng.standard_normal((B, H, dk, dv))
+    dy = rng.standard_normal((B, L, H, dv))
+    dS_last = rng.standard_normal((B, H, dk, dv))
+    t = {n: torch.tensor(a, requires_grad=True) for n, a in
+         dict(q=q, k=k, v=v, gamma=gamma, S0=S0).items()}
+    loss = _torch_la_loss(torch, t["q"], t["k"], t["v"], t["gamma"], start, t["S0"],
+                          torch.tensor(dy), torch.tensor(dS_last), per_step)
+    loss.backward()
+    dq, dk_, dv_, dg, dS0 = oracle.linattn_bwd(q, k, v, gamma, start, dy, dS_last, S0)
+    for name, got in dict(q=dq, k=dk_, v=dv_, gamma=dg, S0=dS0).items():
+        ref = t[name].grad
+        ref = np.zeros_like(got) if ref is None else ref.numpy()
+        np.testing.assert_allclose(got, ref, rtol=1e-11, atol=1e-11, err_msg=name)
+
+
+def test_linattn_bwd_finite_differences():
+    rng = _rng(24)
+    B, L, H, dk, dv = 1, 10, 1, 2, 3
+    q, k, v, gamma, start = _la_inputs(rng, B, L, H, dk, dv, True, first=False)
+    start[0, :] = 0
+    start[0, 6] = 1
+    S0 = rng.standard_normal((B, H, dk, dv))
+    dy = rng.standard_normal((B, L, H, dv))
+    dS_last = rng.standard_normal((B, H, dk, dv))
+
+    def loss(q_, k_, v_, g_, S0_):
+        y, Sl = oracle.linattn_fwd(q_, k_, v_, g_, start, S0_)
+        return float(np.sum(dy * y) + np.sum(dS_last * Sl))
+
+    dq, dk_, dv_, dg, dS0 = oracle.linattn_bwd(q, k, v, gamma, start, dy, dS_last, S0)
+    eps = 1e-6
+    args = [q, k, v, gamma, S0]
+    grads = [dq, dk_, dv_, dg, dS0]
+    for ai in range(5):
+        arr = args[ai]
+        for _ in range(6):
+            idx = tuple(rng.integers(0, n) for n in arr.shape)
+            a1, a2 = arr.copy(), arr.copy()
+            a1[idx] += eps
+            a2[idx] -= eps
+            f1 = loss(*[a1 if j == ai else args[j] for j in range(5)])
+            f2 = loss(*[a2 if j == ai else args[j] for j in range(5)])
+            assert abs((f1 - f2) / (2 * eps) - grads[ai][idx]) < 1e-6, (ai, idx)
+
+
+# ---------------------------------------------------------------------------
+# episode index list <-> begin flags
+# ---------------------------------------------------------------------------
+
+def test_figure2_tape_indices():
+    vals = {}
+    with open(os.path.join(GOLDEN, "tbb_figure2.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                k, *v = line.split()
+                vals[k] = [int(x) for x in v]
+    start = oracle.starts_from_offsets(vals["I"], len(vals["episode"]))
+    np.testing.assert_array_equal(start, vals["start"])
+    np.testing.assert_array_equal(oracle.offsets_from_starts(start), vals["I"])
+    # the episode labels change exactly at the begin indices
+    ep = np.array(vals["episode"])
+    np.testing.assert_array_equal(np.flatnonzero(np.r_[1, np.diff(ep) != 0]), vals["I"])
+
+
+def test_offsets_round_trip_random():
+    rng = _rng(30)
+    for L in (1, 7, 1000):
+        start = (rng.random(L) < 0.1).astype(np.uint8)
+        offs = oracle.offsets_from_starts(start)
+        np.testing.assert_array_equal(offs, np.flatnonzero(start))
+        np.testing.assert_array_equal(oracle.starts_from_offsets(offs, L), start)
