@@ -1,0 +1,151 @@
+/*
+ * memoroid.h -- C ABI of the GB300 (sm_103a) resettable memoroid scans.
+ *
+ * The library evaluates memoroid memory models over one flat "tape" of
+ * concatenated episodes ("Recurrent Reinforcement Learning with Memoroids",
+ * arXiv 2402.09900): a begin flag b_t = 1 on the first step of each episode
+ * (Section 2.1) drives the resettable monoid transform of Theorem 3.2, so
+ * that no information crosses an episode boundary.  States are the inclusive
+ * scan h_t = e_I . f(P_0) . ... . f(P_t) of Definition 3.1.
+ *
+ * Conventions shared by every entry point:
+ *   - Every tensor argument is caller-owned DEVICE memory, row-major and
+ *     contiguous.  The library never allocates or frees device memory; scratch
+ *     space ("workspace") comes from the caller, sized by the *_workspace_bytes
+ *     query, 256-byte aligned.
+ *   - Complex tensors are interleaved (re, im) fp32 pairs (the memory layout
+ *     of torch.complex64).  Complex arrays must be 16-byte aligned.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Calls
+ *     only enqueue work and return at once.  Argument errors are reported
+ *     synchronously by the return value; launch failures map to
+ *     MEMOROID_ERR_CUDA.  Kernels never trap: a bounded wait that runs out
+ *     records MEMOROID_ERR_TIMEOUT in the workspace, read back by
+ *     memoroid_get_device_error().
+ *   - B independent tapes are scanned in one call.  start[b, 0] = 1, or a NULL
+ *     initial state, means the tape starts from the monoid identity e_I.
+ *   - Gradients of complex inputs follow PyTorch's convention
+ *     (grad = dL/dRe + i dL/dIm).
+ */
+#ifndef MEMOROID_H
+#define MEMOROID_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    MEMOROID_OK = 0,
+    MEMOROID_ERR_INVALID_ARG = 1, /* null, misaligned or out-of-range argument */
+    MEMOROID_ERR_UNSUPPORTED = 2, /* a shape or mode this build does not implement */
+    MEMOROID_ERR_WORKSPACE = 3,   /* workspace missing, misaligned or too small */
+    MEMOROID_ERR_CUDA = 4,        /* a CUDA runtime call or launch failed */
+    MEMOROID_ERR_TIMEOUT = 5      /* a bounded device-side wait ran out */
+} memoroid_status_t;
+
+typedef enum { MEMOROID_F32 = 0, MEMOROID_BF16 = 1 } memoroid_dtype_t;
+
+/* Human-readable name of a status code (static string). */
+const char *memoroid_status_string(memoroid_status_t status);
+
+/* Library version as major*10000 + minor*100 + patch. */
+int memoroid_version(void);
+
+/* ======================================================================== */
+/* Diagonal complex scan (S5 / LRU memoroid, Appendix "Simplified State     */
+/* Space Models" and "Linear Recurrent Unit", with diagonal X; reset per    */
+/* Theorem 3.2):                                                            */
+/*     h_t = u_t                          if b_t = 1                        */
+/*     h_t = lambda_t * h_{t-1} + u_t     otherwise (h_{-1} = h0, or 0)     */
+/* element-wise over D complex channels.                                    */
+/* ======================================================================== */
+
+/* Bytes of workspace needed by memoroid_scan_diag_fwd and _bwd for this
+ * shape (one size serves both).  Returns 0 for an invalid shape. */
+size_t memoroid_scan_diag_workspace_bytes(int64_t B, int64_t L, int64_t D);
+
+/*
+ * Forward diagonal scan.
+ *   lambda          complex [D] (lambda_per_step = 0) or [B,L,D] (= 1)
+ *   u               complex [B,L,D]: the lifted inputs f(P_t)
+ *   start           uint8 [B,L]: begin flags, 0 or 1 (any non-zero is 1)
+ *   h0              complex [B,D] or NULL (identity): state before step 0,
+ *                   used only where start[b,0] = 0
+ *   h               complex [B,L,D] output; may alias u
+ *   h_last          complex [B,D] output (h at step L-1) or NULL
+ *   D must be even (two complex channels per 16-byte access).
+ * Errors: INVALID_ARG (null/misaligned pointer, negative size, odd D),
+ * WORKSPACE, CUDA.
+ */
+memoroid_status_t memoroid_scan_diag_fwd(const void *lambda, int lambda_per_step, const void *u,
+                                         const uint8_t *start, const void *h0, void *h,
+                                         void *h_last, int64_t B, int64_t L, int64_t D,
+                                         void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * Backward diagonal scan (reverse-mode of the forward; no truncation across
+ * the tape, cf. the full-BPTT gradient of Section 3).  With delta_t = dL/dh_t
+ * accumulated through the recurrence,
+ *     delta_t = grad_h_t + [b_{t+1} = 0] conj(lambda_{t+1}) delta_{t+1},
+ *     delta_{L-1} = grad_h_{L-1} + grad_h_last,
+ * outputs grad_u_t = delta_t, grad_lambda = sum_{t: b_t=0} delta_t conj(h_{t-1})
+ * (over B and L for a per-channel lambda -> [D]; per step -> [B,L,D]) and
+ * grad_h0 = [b_0 = 0] conj(lambda_0) delta_0.
+ *   h               complex [B,L,D]: the forward output (must not alias grad_u)
+ *   grad_h          complex [B,L,D]
+ *   grad_h_last     complex [B,D] or NULL
+ *   grad_u          complex [B,L,D] output; may alias grad_h
+ *   grad_lambda     complex [D] or [B,L,D] output, or NULL to skip
+ *   grad_h0         complex [B,D] output or NULL
+ * grad_lambda for a per-channel lambda is reduced in a fixed order, so
+ * repeated calls are bit-identical.
+ */
+memoroid_status_t memoroid_scan_diag_bwd(const void *lambda, int lambda_per_step,
+                                         const uint8_t *start, const void *h0, const void *h,
+                                         const void *grad_h, const void *grad_h_last, void *grad_u,
+                                         void *grad_lambda, void *grad_h0, int64_t B, int64_t L,
+                                         int64_t D, void *workspace, size_t workspace_bytes,
+                                         void *stream);
+
+/* ======================================================================== */
+/* Episode index list <-> begin flags (Algorithm 1 keeps I = where(b)).     */
+/* ======================================================================== */
+
+/* start[t] = 1 for t in offsets[0..E), 0 elsewhere, t in [0, L).  Offsets
+ * outside [0, L) are ignored.  offsets: int64 device array; start: uint8 [L]. */
+memoroid_status_t memoroid_starts_from_offsets(const int64_t *offsets, int64_t E, int64_t L,
+                                               uint8_t *start, void *stream);
+
+/* Workspace bytes for memoroid_offsets_from_starts. */
+size_t memoroid_offsets_workspace_bytes(int64_t L);
+
+/* offsets[0..n) = increasing indices t with start[t] != 0; *count = n (int64,
+ * device memory).  offsets must hold L entries. */
+memoroid_status_t memoroid_offsets_from_starts(const uint8_t *start, int64_t L, int64_t *offsets,
+                                               int64_t *count, void *workspace,
+                                               size_t workspace_bytes, void *stream);
+
+/* ======================================================================== */
+/* Device-side error reporting and debug knobs.                             */
+/* ======================================================================== */
+
+/* Synchronises `stream`, then reads the error word that the last call using
+ * `workspace` left there: MEMOROID_OK or MEMOROID_ERR_TIMEOUT. */
+memoroid_status_t memoroid_get_device_error(const void *workspace, void *stream);
+
+/* Process-wide limit for every bounded device-side wait, in nanoseconds
+ * (0 restores the default of 1 s).  Applies to later calls. */
+void memoroid_debug_set_wait_limit_ns(uint64_t ns);
+
+/* Fault injection for tests: the tile with this scheduling ticket skips
+ * publishing its look-back status, so its successor's wait runs out
+ * (-1 = off, the default).  Applies to later scan calls. */
+void memoroid_debug_withhold_tile(int64_t ticket);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MEMOROID_H */

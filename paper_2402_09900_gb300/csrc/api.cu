@@ -1,0 +1,196 @@
+// api.cu -- the C ABI (include/memoroid.h): argument validation, workspace
+// checks, launches and device-error read-back.
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cstdint>
+
+#include "internal.cuh"
+
+namespace memoroid {
+
+namespace {
+constexpr uint64_t kDefaultWaitNs = 1000000000ull;  // 1 s
+std::atomic<uint64_t> g_wait_ns{kDefaultWaitNs};
+std::atomic<int64_t> g_withhold{-1};
+
+inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+inline cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
+}  // namespace
+
+DebugKnobs debug_knobs() { return DebugKnobs{g_wait_ns.load(), g_withhold.load()}; }
+
+}  // namespace memoroid
+
+using namespace memoroid;
+
+extern "C" {
+
+const char* memoroid_status_string(memoroid_status_t s) {
+    switch (s) {
+        case MEMOROID_OK: return "ok";
+        case MEMOROID_ERR_INVALID_ARG: return "invalid argument";
+        case MEMOROID_ERR_UNSUPPORTED: return "unsupported shape or mode";
+        case MEMOROID_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+        case MEMOROID_ERR_CUDA: return "CUDA error";
+        case MEMOROID_ERR_TIMEOUT: return "device-side wait timed out";
+    }
+    return "unknown status";
+}
+
+int memoroid_version(void) { return 100; }
+
+void memoroid_debug_set_wait_limit_ns(uint64_t ns) { g_wait_ns.store(ns == 0 ? kDefaultWaitNs : ns); }
+
+void memoroid_debug_withhold_tile(int64_t ticket) { g_withhold.store(ticket); }
+
+memoroid_status_t memoroid_get_device_error(const void* workspace, void* stream) {
+    if (workspace == nullptr) return MEMOROID_ERR_INVALID_ARG;
+    uint32_t code = 0;
+    cudaStream_t s = as_stream(stream);
+    if (cudaMemcpyAsync(&code, workspace, sizeof(code), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return MEMOROID_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    return code == DEV_OK ? MEMOROID_OK : MEMOROID_ERR_TIMEOUT;
+}
+
+// ---------------------------------------------------------------------------
+// diagonal scan
+// ---------------------------------------------------------------------------
+
+size_t memoroid_scan_diag_workspace_bytes(int64_t B, int64_t L, int64_t D) {
+    if (B < 0 || L < 0 || D < 0 || (D % 2) != 0) return 0;
+    return diag::workspace_bytes(B, L, D);
+}
+
+static memoroid_status_t check_ws(int64_t B, int64_t L, int64_t D, const void* ws, size_t bytes) {
+    if (ws == nullptr || !aligned(ws, 256)) return MEMOROID_ERR_WORKSPACE;
+    if (bytes < diag::workspace_bytes(B, L, D)) return MEMOROID_ERR_WORKSPACE;
+    return MEMOROID_OK;
+}
+
+memoroid_status_t memoroid_scan_diag_fwd(const void* lambda, int lambda_per_step, const void* u,
+                                         const uint8_t* start, const void* h0, void* h,
+                                         void* h_last, int64_t B, int64_t L, int64_t D,
+                                         void* workspace, size_t workspace_bytes, void* stream) {
+    if (B < 0 || L < 0 || D < 0 || (D % 2) != 0) return MEMOROID_ERR_INVALID_ARG;
+    if (lambda_per_step != 0 && lambda_per_step != 1) return MEMOROID_ERR_INVALID_ARG;
+    const bool work = B > 0 && L > 0 && D > 0;
+    if (work) {
+        if (!lambda || !u || !start || !h) return MEMOROID_ERR_INVALID_ARG;
+        if (!aligned(lambda, 16) || !aligned(u, 16) || !aligned(h, 16)) return MEMOROID_ERR_INVALID_ARG;
+    }
+    if ((h0 && !aligned(h0, 16)) || (h_last && !aligned(h_last, 16))) return MEMOROID_ERR_INVALID_ARG;
+    cudaStream_t s = as_stream(stream);
+    if (!work) {
+        // empty tape: h_last = h0 (or the identity)
+        if (h_last && B > 0 && D > 0) {
+            const size_t bytes = static_cast<size_t>(B) * D * 8;
+            const cudaError_t e = h0 ? cudaMemcpyAsync(h_last, h0, bytes, cudaMemcpyDeviceToDevice, s)
+                                     : cudaMemsetAsync(h_last, 0, bytes, s);
+            if (e != cudaSuccess) return MEMOROID_ERR_CUDA;
+        }
+        return MEMOROID_OK;
+    }
+    const memoroid_status_t w = check_ws(B, L, D, workspace, workspace_bytes);
+    if (w != MEMOROID_OK) return w;
+    diag::Args a{};
+    a.lambda = lambda;
+    a.lambda_per_step = lambda_per_step;
+    a.u = u;
+    a.start = start;
+    a.h0 = h0;
+    a.out = h;
+    a.out_last = h_last;
+    a.B = B;
+    a.L = L;
+    a.D = D;
+    a.workspace = workspace;
+    a.workspace_bytes = workspace_bytes;
+    return diag::launch_fwd(a, s);
+}
+
+memoroid_status_t memoroid_scan_diag_bwd(const void* lambda, int lambda_per_step,
+                                         const uint8_t* start, const void* h0, const void* h,
+                                         const void* grad_h, const void* grad_h_last, void* grad_u,
+                                         void* grad_lambda, void* grad_h0, int64_t B, int64_t L,
+                                         int64_t D, void* workspace, size_t workspace_bytes,
+                                         void* stream) {
+    if (B < 0 || L < 0 || D < 0 || (D % 2) != 0) return MEMOROID_ERR_INVALID_ARG;
+    if (lambda_per_step != 0 && lambda_per_step != 1) return MEMOROID_ERR_INVALID_ARG;
+    const bool work = B > 0 && L > 0 && D > 0;
+    cudaStream_t s = as_stream(stream);
+    if ((h0 && !aligned(h0, 16)) || (grad_h_last && !aligned(grad_h_last, 16)) ||
+        (grad_lambda && !aligned(grad_lambda, 16)) || (grad_h0 && !aligned(grad_h0, 16)))
+        return MEMOROID_ERR_INVALID_ARG;
+    if (work) {
+        if (!lambda || !start || !h || !grad_h || !grad_u) return MEMOROID_ERR_INVALID_ARG;
+        if (!aligned(lambda, 16) || !aligned(h, 16) || !aligned(grad_h, 16) || !aligned(grad_u, 16))
+            return MEMOROID_ERR_INVALID_ARG;
+        if (grad_u == h) return MEMOROID_ERR_INVALID_ARG;
+    }
+    if (!work) {
+        if (D > 0 && grad_lambda && !lambda_per_step &&
+            cudaMemsetAsync(grad_lambda, 0, static_cast<size_t>(D) * 8, s) != cudaSuccess)
+            return MEMOROID_ERR_CUDA;
+        if (grad_h0 && B > 0 && D > 0) {
+            const size_t bytes = static_cast<size_t>(B) * D * 8;
+            const cudaError_t e = grad_h_last
+                                      ? cudaMemcpyAsync(grad_h0, grad_h_last, bytes, cudaMemcpyDeviceToDevice, s)
+                                      : cudaMemsetAsync(grad_h0, 0, bytes, s);
+            if (e != cudaSuccess) return MEMOROID_ERR_CUDA;
+        }
+        return MEMOROID_OK;
+    }
+    const memoroid_status_t w = check_ws(B, L, D, workspace, workspace_bytes);
+    if (w != MEMOROID_OK) return w;
+    diag::Args a{};
+    a.lambda = lambda;
+    a.lambda_per_step = lambda_per_step;
+    a.u = grad_h;
+    a.start = start;
+    a.h0 = h0;
+    a.out = grad_u;
+    a.h = h;
+    a.g_last = grad_h_last;
+    a.grad_lambda = grad_lambda;
+    a.grad_h0 = grad_h0;
+    a.B = B;
+    a.L = L;
+    a.D = D;
+    a.workspace = workspace;
+    a.workspace_bytes = workspace_bytes;
+    return diag::launch_bwd(a, s);
+}
+
+// ---------------------------------------------------------------------------
+// episode index list <-> begin flags
+// ---------------------------------------------------------------------------
+
+memoroid_status_t memoroid_starts_from_offsets(const int64_t* offsets, int64_t E, int64_t L,
+                                               uint8_t* start, void* stream) {
+    if (E < 0 || L < 0) return MEMOROID_ERR_INVALID_ARG;
+    if ((L > 0 && !start) || (E > 0 && !offsets)) return MEMOROID_ERR_INVALID_ARG;
+    return tape::launch_starts_from_offsets(offsets, E, L, start, as_stream(stream));
+}
+
+size_t memoroid_offsets_workspace_bytes(int64_t L) {
+    if (L < 0) return 0;
+    return tape::offsets_workspace_bytes(L);
+}
+
+memoroid_status_t memoroid_offsets_from_starts(const uint8_t* start, int64_t L, int64_t* offsets,
+                                               int64_t* count, void* workspace,
+                                               size_t workspace_bytes, void* stream) {
+    if (L < 0 || !count) return MEMOROID_ERR_INVALID_ARG;
+    if (L > 0 && (!start || !offsets)) return MEMOROID_ERR_INVALID_ARG;
+    if (!aligned(count, 8) || (offsets && !aligned(offsets, 8))) return MEMOROID_ERR_INVALID_ARG;
+    if (L > 0) {
+        if (!workspace || !aligned(workspace, 256)) return MEMOROID_ERR_WORKSPACE;
+        if (workspace_bytes < tape::offsets_workspace_bytes(L)) return MEMOROID_ERR_WORKSPACE;
+    }
+    return tape::launch_offsets_from_starts(start, L, offsets, count, workspace, workspace_bytes,
+                                            as_stream(stream));
+}
+
+}  // extern "C"

@@ -1,0 +1,66 @@
+// internal.cuh -- declarations shared by the C-ABI layer and the kernel files.
+#pragma once
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "memoroid.h"
+
+namespace memoroid {
+
+// Device-side error codes written to the first word of a workspace header.
+enum DeviceError : uint32_t {
+    DEV_OK = 0,
+    DEV_LOOKBACK_TIMEOUT = 1,  // a look-back wait on a predecessor ran out
+    DEV_TMA_TIMEOUT = 2,       // a TMA completion wait ran out
+};
+
+// Workspace header (256 bytes): [0] error code, [1] tile ticket counter,
+// [2..3] ticket of the tile that recorded the error (u64).
+constexpr size_t kHeaderBytes = 256;
+
+// Process-wide debug knobs (set through memoroid_debug_*).
+struct DebugKnobs {
+    uint64_t wait_ns;
+    int64_t withhold_ticket;
+};
+DebugKnobs debug_knobs();
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+namespace diag {
+
+struct Args {
+    const void* lambda;
+    int lambda_per_step;
+    const void* u;  // fwd: u; bwd: grad_h
+    const uint8_t* start;
+    const void* h0;
+    void* out;       // fwd: h; bwd: grad_u
+    void* out_last;  // fwd: h_last
+    const void* h;   // bwd: forward output
+    const void* g_last;
+    void* grad_lambda;
+    void* grad_h0;
+    int64_t B, L, D;
+    void* workspace;
+    size_t workspace_bytes;
+};
+
+size_t workspace_bytes(int64_t B, int64_t L, int64_t D);
+memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream);
+memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream);
+
+}  // namespace diag
+
+namespace tape {
+size_t offsets_workspace_bytes(int64_t L);
+memoroid_status_t launch_starts_from_offsets(const int64_t* offsets, int64_t E, int64_t L,
+                                             uint8_t* start, cudaStream_t stream);
+memoroid_status_t launch_offsets_from_starts(const uint8_t* start, int64_t L, int64_t* offsets,
+                                             int64_t* count, void* workspace, size_t ws_bytes,
+                                             cudaStream_t stream);
+}  // namespace tape
+
+}  // namespace memoroid

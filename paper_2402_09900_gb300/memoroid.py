@@ -1,0 +1,242 @@
+"""ctypes binding of the C ABI in include/memoroid.h.
+
+Argument marshalling only: every step of every scan runs in the CUDA kernels
+of libmemoroid.so.  PyTorch supplies device memory (outputs and workspace are
+torch tensors) and the current CUDA stream.  There is no fallback: if the
+library is missing or no GPU is present, the calls raise.
+
+The raw entry points keep the C names (memoroid_scan_diag_fwd, ...) and take
+torch tensors (or None) where the C call takes a pointer; the short helpers
+(diag_fwd, diag_bwd, ...) allocate outputs and workspace and return tensors.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+MEMOROID_OK = 0
+MEMOROID_ERR_INVALID_ARG = 1
+MEMOROID_ERR_UNSUPPORTED = 2
+MEMOROID_ERR_WORKSPACE = 3
+MEMOROID_ERR_CUDA = 4
+MEMOROID_ERR_TIMEOUT = 5
+MEMOROID_F32 = 0
+MEMOROID_BF16 = 1
+
+_lock = threading.Lock()
+_lib = None
+
+_p = ctypes.c_void_p
+_i64 = ctypes.c_int64
+_int = ctypes.c_int
+_sz = ctypes.c_size_t
+
+# name -> (restype, argtypes); mirrors include/memoroid.h
+SIGNATURES = {
+    "memoroid_status_string": (ctypes.c_char_p, [_int]),
+    "memoroid_version": (_int, []),
+    "memoroid_scan_diag_workspace_bytes": (_sz, [_i64, _i64, _i64]),
+    "memoroid_scan_diag_fwd": (_int, [_p, _int, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p, _sz, _p]),
+    "memoroid_scan_diag_bwd": (_int, [_p, _int, _p, _p, _p, _p, _p, _p, _p, _p, _i64, _i64, _i64,
+                                      _p, _sz, _p]),
+    "memoroid_starts_from_offsets": (_int, [_p, _i64, _i64, _p, _p]),
+    "memoroid_offsets_workspace_bytes": (_sz, [_i64]),
+    "memoroid_offsets_from_starts": (_int, [_p, _i64, _p, _p, _p, _sz, _p]),
+    "memoroid_get_device_error": (_int, [_p, _p]),
+    "memoroid_debug_set_wait_limit_ns": (None, [ctypes.c_uint64]),
+    "memoroid_debug_withhold_tile": (None, [_i64]),
+}
+
+
+class MemoroidError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+
+
+def lib_path() -> str:
+    return _build.lib_path()
+
+
+def load():
+    """Loads libmemoroid.so (it must have been built: __graft_entry__.build()
+    or paper_2402_09900_gb300.build.build())."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = lib_path()
+            if not os.path.exists(path):
+                raise RuntimeError(f"{path} is missing: build the CUDA library first")
+            L = ctypes.CDLL(path)
+            for name, (res, args) in SIGNATURES.items():
+                fn = getattr(L, name)
+                fn.restype = res
+                fn.argtypes = args
+            _lib = L
+    return _lib
+
+
+def status_string(status: int) -> str:
+    return load().memoroid_status_string(int(status)).decode()
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(status, where):
+    if status != MEMOROID_OK:
+        raise MemoroidError(status, where)
+
+
+def _need_cuda(*ts):
+    for t in ts:
+        if t is not None:
+            if not t.is_cuda:
+                raise ValueError("memoroid kernels take CUDA tensors only")
+            if not t.is_contiguous():
+                raise ValueError("memoroid kernels take contiguous tensors only")
+
+
+# ---------------------------------------------------------------------------
+# raw entry points (same names as the C ABI)
+# ---------------------------------------------------------------------------
+
+def memoroid_scan_diag_workspace_bytes(B, L, D) -> int:
+    return int(load().memoroid_scan_diag_workspace_bytes(B, L, D))
+
+
+def memoroid_scan_diag_fwd(lam, lambda_per_step, u, start, h0, h, h_last, B, L, D, workspace,
+                           stream=None):
+    _need_cuda(lam, u, start, h0, h, h_last, workspace)
+    st = load().memoroid_scan_diag_fwd(_ptr(lam), int(lambda_per_step), _ptr(u), _ptr(start), _ptr(h0),
+                                       _ptr(h), _ptr(h_last), B, L, D, _ptr(workspace),
+                                       workspace.numel() if workspace is not None else 0, _stream(stream))
+    _check(st, "memoroid_scan_diag_fwd")
+
+
+def memoroid_scan_diag_bwd(lam, lambda_per_step, start, h0, h, grad_h, grad_h_last, grad_u, grad_lambda,
+                           grad_h0, B, L, D, workspace, stream=None):
+    _need_cuda(lam, start, h0, h, grad_h, grad_h_last, grad_u, grad_lambda, grad_h0, workspace)
+    st = load().memoroid_scan_diag_bwd(_ptr(lam), int(lambda_per_step), _ptr(start), _ptr(h0), _ptr(h),
+                                       _ptr(grad_h), _ptr(grad_h_last), _ptr(grad_u), _ptr(grad_lambda),
+                                       _ptr(grad_h0), B, L, D, _ptr(workspace),
+                                       workspace.numel() if workspace is not None else 0, _stream(stream))
+    _check(st, "memoroid_scan_diag_bwd")
+
+
+def memoroid_starts_from_offsets(offsets, E, L, start, stream=None):
+    _need_cuda(offsets, start)
+    _check(load().memoroid_starts_from_offsets(_ptr(offsets), E, L, _ptr(start), _stream(stream)),
+           "memoroid_starts_from_offsets")
+
+
+def memoroid_offsets_workspace_bytes(L) -> int:
+    return int(load().memoroid_offsets_workspace_bytes(L))
+
+
+def memoroid_offsets_from_starts(start, L, offsets, count, workspace, stream=None):
+    _need_cuda(start, offsets, count, workspace)
+    _check(load().memoroid_offsets_from_starts(_ptr(start), L, _ptr(offsets), _ptr(count), _ptr(workspace),
+                                               workspace.numel() if workspace is not None else 0,
+                                               _stream(stream)),
+           "memoroid_offsets_from_starts")
+
+
+def memoroid_get_device_error(workspace, stream=None) -> int:
+    return int(load().memoroid_get_device_error(_ptr(workspace), _stream(stream)))
+
+
+def memoroid_debug_set_wait_limit_ns(ns: int) -> None:
+    load().memoroid_debug_set_wait_limit_ns(int(ns))
+
+
+def memoroid_debug_withhold_tile(ticket: int) -> None:
+    load().memoroid_debug_withhold_tile(int(ticket))
+
+
+# ---------------------------------------------------------------------------
+# allocating helpers
+# ---------------------------------------------------------------------------
+
+def workspace(nbytes: int, device) -> torch.Tensor:
+    # torch's caching allocator returns 512-byte aligned blocks
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+def diag_workspace(B, L, D, device) -> torch.Tensor:
+    return workspace(memoroid_scan_diag_workspace_bytes(B, L, D), device)
+
+
+def diag_fwd(lam, u, start, h0=None, want_last=True, ws=None, out=None, stream=None):
+    """h, h_last = scan of u ([B,L,D] complex64) with lambda ([D] or [B,L,D])."""
+    B, L, D = u.shape
+    per_step = lam.dim() == 3
+    if ws is None:
+        ws = diag_workspace(B, L, D, u.device)
+    h = torch.empty_like(u) if out is None else out
+    h_last = torch.empty((B, D), dtype=u.dtype, device=u.device) if want_last else None
+    memoroid_scan_diag_fwd(lam, per_step, u, start, h0, h, h_last, B, L, D, ws, stream)
+    return h, h_last
+
+
+def diag_bwd(lam, start, h, grad_h, grad_h_last=None, h0=None, want_lambda=True, want_h0=False,
+             ws=None, out=None, stream=None):
+    """grad_u, grad_lambda, grad_h0 of the diagonal scan."""
+    B, L, D = grad_h.shape
+    per_step = lam.dim() == 3
+    if ws is None:
+        ws = diag_workspace(B, L, D, grad_h.device)
+    grad_u = torch.empty_like(grad_h) if out is None else out
+    grad_lambda = torch.empty_like(lam) if want_lambda else None
+    grad_h0 = torch.empty((B, D), dtype=grad_h.dtype, device=grad_h.device) if want_h0 else None
+    memoroid_scan_diag_bwd(lam, per_step, start, h0, h, grad_h, grad_h_last, grad_u, grad_lambda, grad_h0,
+                           B, L, D, ws, stream)
+    return grad_u, grad_lambda, grad_h0
+
+
+def starts_from_offsets(offsets, L, stream=None):
+    start = torch.empty(L, dtype=torch.uint8, device=offsets.device)
+    memoroid_starts_from_offsets(offsets, offsets.numel(), L, start, stream)
+    return start
+
+
+def offsets_from_starts(start, stream=None):
+    L = start.numel()
+    offsets = torch.empty(max(L, 1), dtype=torch.int64, device=start.device)
+    count = torch.empty(1, dtype=torch.int64, device=start.device)
+    ws = workspace(memoroid_offsets_workspace_bytes(L), start.device)
+    memoroid_offsets_from_starts(start, L, offsets, count, ws, stream)
+    return offsets, count
+
+
+class DiagScan(torch.autograd.Function):
+    """Autograd wrapper: h = DiagScan.apply(lam, u, start, h0)."""
+
+    @staticmethod
+    def forward(ctx, lam, u, start, h0):
+        h, _ = diag_fwd(lam, u, start, h0, want_last=False)
+        ctx.save_for_backward(lam, start, h0 if h0 is not None else torch.empty(0), h)
+        ctx.has_h0 = h0 is not None
+        return h
+
+    @staticmethod
+    def backward(ctx, grad_h):
+        lam, start, h0, h = ctx.saved_tensors
+        h0 = h0 if ctx.has_h0 else None
+        gu, gl, gh0 = diag_bwd(lam, start, h, grad_h.contiguous(), None, h0,
+                               want_lambda=ctx.needs_input_grad[0], want_h0=ctx.has_h0)
+        return gl, gu, None, gh0
