@@ -1,0 +1,398 @@
+"""Benchmark: resettable diagonal memoroid scan, forward + backward, on one
+synthetic tape of L = 2^20 steps x D = 256 complex64 channels with
+Geometric(500) episodes clipped to [1, 10000] (the tape-based batch of
+Section 4.1 at GPU scale).
+
+One step = memoroid_scan_diag_fwd + memoroid_scan_diag_bwd (with grad_lambda)
+over the whole tape.  Prints one JSON line.
+
+  python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+
+--impl reference times the fp64 CPU oracle (the plain sequential definition)
+on the host cores on a bounded sample of the same workload.
+Under torchrun each rank scans its own tape (independent tapes are plain data
+parallelism: no collective on the data path); rank 0 reports the max time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import tapegen  # noqa: E402
+
+METRIC = "tape transitions/sec (fwd+bwd) and % of HBM / tensor roofline on 1 GB300"
+UNIT = "transitions/s"
+CFG = 2
+WORKLOAD = ("diag scan fwd+bwd (grad_u, grad_lambda): B=1 tape, L=2^20 steps, D=256 complex64 "
+            "channels, per-channel lambda, Geometric(500) episodes clipped to [1,10000]")
+# algorithmic bytes per (step, channel): fwd reads u, writes h; bwd reads grad_h and h, writes grad_u
+FWD_BYTES_PER_STEP_CH = 16
+BWD_BYTES_PER_STEP_CH = 24
+PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "diag_bwd_traffic.txt")
+KERNEL_SRC = os.path.join(ROOT, "paper_2402_09900_gb300", "csrc", "diag_scan.cu")
+
+
+def _dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def _traffic_record():
+    """(bytes per launch at the bench size, note) from the committed ncu
+    summary, or (None, why) if the kernel source changed since."""
+    try:
+        rec = {}
+        with open(PROFILE_TRAFFIC) as f:
+            for line in f:
+                if ":" in line and not line.startswith("#"):
+                    k, v = line.split(":", 1)
+                    rec[k.strip()] = v.strip()
+        src = hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()
+        if rec.get("source_sha256") != src:
+            return None, "kernel changed since the ncu capture"
+        return float(rec["traffic_bytes_per_launch_at_bench_size"]), rec.get("note", "")
+    except Exception as e:  # no capture yet
+        return None, f"no ncu capture ({type(e).__name__})"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-i", str(self.gpu), "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline and the reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_sample(t, steps):
+    """A bounded sample of the workload: the first `steps` steps of the tape."""
+    return {"lam": t["lam"], "u": t["u"][:, :steps], "start": t["start"][:, :steps],
+            "grad_h": t["grad_h"][:, :steps]}
+
+
+def time_oracle_step(sample):
+    import oracle
+    t0 = time.perf_counter()
+    h, _ = oracle.diag_fwd(sample["lam"], sample["u"], sample["start"])
+    oracle.diag_bwd(sample["lam"], sample["start"], h, sample["grad_h"])
+    return time.perf_counter() - t0
+
+
+def _calibrate(t):
+    """Seconds per transition of the oracle (fwd+bwd), from a short warm run."""
+    probe = min(t["L"], 32768)
+    time_oracle_step(oracle_sample(t, 1024))  # page-in, thread pool start
+    return time_oracle_step(oracle_sample(t, probe)) / probe
+
+
+def cpu_baseline(t, target_s):
+    """The oracle timed on about `target_s` seconds of the workload's first steps."""
+    import oracle
+    oracle.build()
+    per = _calibrate(t)
+    steps = int(min(t["L"], max(4096, target_s / per)))
+    s = oracle_sample(t, steps)
+    dt = time_oracle_step(s)
+    B = s["u"].shape[0]
+    return {"value": B * steps / dt, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+            "sample": f"first {steps} steps of the tape (x {s['u'].shape[2]} channels), fwd+bwd incl. "
+                      f"grad_lambda, fp64 C oracle with OpenMP over channels; {dt:.2f} s"}
+
+
+def run_reference(args):
+    """The reference arm: the oracle on the host cores, each step a bounded
+    sample of the tape sized so that all steps take about --ref-seconds."""
+    ws, rank, _ = _dist_env()
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    t = tapegen.diag_config(CFG)
+    per = _calibrate(t)
+    steps = int(min(t["L"], max(1024, args.ref_seconds / max(args.steps, 1) / per)))
+    s = oracle_sample(t, steps)
+    for _ in range(args.warmup):
+        time_oracle_step(oracle_sample(t, min(steps, 1024)))
+    times = [time_oracle_step(s) for _ in range(args.steps)]
+    dt = sum(times) / len(times)
+    value = t["B"] * steps / dt
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "B": t["B"], "L": t["L"], "D": t["D"],
+                   "sample_steps_per_step": steps},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+                         "sample": f"first {steps} steps x {t['D']} channels per step, fwd+bwd incl. "
+                                   f"grad_lambda, fp64 C oracle"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# the GPU arm
+# ---------------------------------------------------------------------------
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    ws, rank, local = _dist_env()
+    if ws > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    from paper_2402_09900_gb300 import build as native_build
+    native_build.build()
+    from paper_2402_09900_gb300 import memoroid as m
+    m.load()
+
+    t = tapegen.diag_config(CFG)
+    if args.tape_steps:
+        # a shorter tape of the same workload (used for profiler captures)
+        t = {k: (v[:, :args.tape_steps] if k in ("u", "start", "grad_h") else v) for k, v in t.items()}
+        t["L"] = args.tape_steps
+    B, L, D = t["B"], t["L"], t["D"]
+    lam = torch.from_numpy(t["lam"]).to(dev)
+    u = torch.from_numpy(t["u"]).to(dev)
+    start = torch.from_numpy(t["start"]).to(dev)
+    grad_h = torch.from_numpy(t["grad_h"]).to(dev)
+    h = torch.empty_like(u)
+    grad_u = torch.empty_like(u)
+    grad_lam = torch.empty_like(lam)
+    wsb = m.memoroid_scan_diag_workspace_bytes(B, L, D)
+    work = m.workspace(wsb, dev)
+    stream = torch.cuda.current_stream()
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        m.memoroid_scan_diag_fwd(lam, 0, u, start, None, h, None, B, L, D, work, stream)
+        if ev is not None:
+            ev[1].record(stream)
+        m.memoroid_scan_diag_bwd(lam, 0, start, None, h, grad_h, None, grad_u, grad_lam, None, B, L, D,
+                                 work, stream)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if m.memoroid_get_device_error(work) != m.MEMOROID_OK:
+        raise RuntimeError("device-side error during warm-up")
+
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    ids = [x for x in vis.split(",") if x.strip()]
+    smi_index = int(ids[local]) if len(ids) > local and ids[local].strip().isdigit() else local
+    sampler = ClockSampler(smi_index)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    t_begin = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.3)  # let the sampler attach
+    t_begin.record(stream)
+    for i in range(args.steps):
+        step(evs[i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    if ws > 1:
+        dist.barrier()
+    if m.memoroid_get_device_error(work) != m.MEMOROID_OK:
+        raise RuntimeError("device-side error during the timed region")
+    elapsed_ms = t_begin.elapsed_time(t_end)
+    fwd_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    bwd_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    if ws > 1:
+        tt = torch.tensor([elapsed_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(tt.item())
+    ms_per_step = elapsed_ms / args.steps
+    value = ws * B * L / (ms_per_step / 1e3)
+
+    # ---- end to end through the C ABI with pinned host buffers ----
+    e2e = None
+    if args.e2e_steps > 0:
+        hu = torch.from_numpy(t["u"]).pin_memory()
+        hg = torch.from_numpy(t["grad_h"]).pin_memory()
+        hs = torch.from_numpy(t["start"]).pin_memory()
+        hl = torch.from_numpy(t["lam"]).pin_memory()
+        oh = torch.empty(h.shape, dtype=h.dtype).pin_memory()
+        ogu = torch.empty(grad_u.shape, dtype=grad_u.dtype).pin_memory()
+        ogl = torch.empty(grad_lam.shape, dtype=grad_lam.dtype).pin_memory()
+        h2d = sum(x.numel() * x.element_size() for x in (hu, hg, hs, hl))
+        d2h = sum(x.numel() * x.element_size() for x in (oh, ogu, ogl))
+
+        def e2e_step():
+            u.copy_(hu, non_blocking=True)
+            grad_h.copy_(hg, non_blocking=True)
+            start.copy_(hs, non_blocking=True)
+            lam.copy_(hl, non_blocking=True)
+            step()
+            oh.copy_(h, non_blocking=True)
+            ogu.copy_(grad_u, non_blocking=True)
+            ogl.copy_(grad_lam, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        if ws > 1:
+            dist.barrier()
+        e0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        torch.cuda.synchronize()
+        e_ms = (time.perf_counter() - e0) * 1e3 / args.e2e_steps
+        if ws > 1:
+            tt = torch.tensor([e_ms], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            e_ms = float(tt.item())
+        e2e = {"value": ws * B * L / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "steps": args.e2e_steps, "ms_per_step": e_ms}
+
+    if rank != 0:
+        if ws > 1:
+            dist.destroy_process_group()
+        return
+
+    peak, peak_kind = _peaks()
+    fwd_bytes = B * L * D * FWD_BYTES_PER_STEP_CH + B * L
+    bwd_bytes = B * L * D * BWD_BYTES_PER_STEP_CH + B * L
+    fwd_avg = sum(fwd_ms) / len(fwd_ms)
+    bwd_avg = sum(bwd_ms) / len(bwd_ms)
+    traffic, traffic_note = _traffic_record()
+    bwd_gbs = bwd_bytes / (bwd_avg * 1e-3) / 1e9
+    fwd_gbs = fwd_bytes / (fwd_avg * 1e-3) / 1e9
+    roofline = {"bound": "hbm", "achieved": bwd_gbs, "peak": peak, "unit": "GB/s",
+                "frac": bwd_gbs / peak, "traffic": traffic,
+                "kernel": "memoroid_scan_diag_bwd (reverse scan + grad_lambda reduction)",
+                "algorithmic_bytes_per_launch": bwd_bytes, "avg_launch_ms": bwd_avg,
+                "peak_kind": f"{peak_kind} (copy bandwidth)", "traffic_note": traffic_note,
+                "fwd": {"achieved": fwd_gbs, "frac": fwd_gbs / peak, "avg_launch_ms": fwd_avg,
+                        "algorithmic_bytes_per_launch": fwd_bytes},
+                "step_frac": (fwd_bytes + bwd_bytes) / (ms_per_step * 1e-3) / 1e9 / peak}
+    cpu = None
+    if ws == 1 and not args.skip_cpu_baseline:
+        cpu = cpu_baseline(t, args.cpu_seconds)
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "B": B, "L": L, "D": D, "episodes": int(t["start"].sum()),
+                   "l2": "inputs larger than L2 (each tensor 2 GiB vs 129 MB L2); no flush needed",
+                   "parallelism": f"independent tape per GPU x{ws}"},
+        "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+        "gpu_launches": 4 * args.steps, "clocks": clocks,
+    }
+    print(json.dumps(out), flush=True)
+    if ws > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="approximate CPU time of the cpu_baseline oracle sample")
+    ap.add_argument("--ref-seconds", type=float, default=90.0,
+                    help="approximate total oracle time of the --impl reference steps")
+    ap.add_argument("--skip-cpu-baseline", action="store_true")
+    ap.add_argument("--tape-steps", type=int, default=0,
+                    help="use only the first N steps of the tape (profiler captures); 0 = full workload")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 
 #include <atomic>
+#include <chrono>
 #include <cstdint>
 
 #include "internal.cuh"
@@ -13,12 +14,22 @@ namespace {
 constexpr uint64_t kDefaultWaitNs = 1000000000ull;  // 1 s
 std::atomic<uint64_t> g_wait_ns{kDefaultWaitNs};
 std::atomic<int64_t> g_withhold{-1};
+// seeded from the clock so that two processes sharing a workspace are
+// unlikely to reuse each other's tags
+std::atomic<uint32_t> g_epoch{static_cast<uint32_t>(
+    std::chrono::steady_clock::now().time_since_epoch().count() * 2654435761ull)};
 
 inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 inline cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
 }  // namespace
 
 DebugKnobs debug_knobs() { return DebugKnobs{g_wait_ns.load(), g_withhold.load()}; }
+
+uint32_t next_epoch() {
+    uint32_t e = 0;
+    while (e == 0) e = g_epoch.fetch_add(1u) & 0x7fffffffu;
+    return e;
+}
 
 }  // namespace memoroid
 

@@ -7,44 +7,52 @@
 // made resettable by Theorem 3.2: an element whose begin flag is set discards
 // everything to its left, (A, b) o (A', 1) = (A', 1).  Per step the lifted
 // element is ((lambda_t, u_t), b_t), so h_t = b_t ? u_t : lambda_t h_{t-1} + u_t.
+// The backward pass is the same scan run right to left over
+//     delta_t = grad_h_t + [b_{t+1} = 0] conj(lambda_{t+1}) delta_{t+1},
+// i.e. the element of step t is (conj(lambda_{t+1}), grad_h_t, b_{t+1}), plus
+// grad_lambda = sum_{b_t = 0} delta_t conj(h_{t-1}).
 //
 // Design (GB300-first; the paper itself ships no kernels):
 //   * The tape [B, L, D] is cut into tiles of T steps x 64 complex channels
-//     (a 512-byte row slab).  A "chain" is one (tape, slab) pair; its tiles
-//     are scanned left to right in a single pass with a look-back over
-//     already-published tile summaries.
-//   * One CTA per tile.  Tiles are handed out by an atomic ticket so that a
-//     CTA only ever waits on tiles whose CTAs are already resident.
+//     (a 512-byte row slab).  A "chain" is one (tape, slab) pair.  Tiles are
+//     handed out in order by an atomic ticket, so a tile only ever waits on
+//     tiles whose tickets were taken earlier by running CTAs.
+//   * One CTA per tile, several CTAs resident per SM.  A CTA has W scan
+//     warps and two look-back warps.  Each scan warp owns R consecutive steps
+//     and each lane two complex channels (one 16-byte vector): a lane scans
+//     its steps serially from the identity, then rescans them from its carry
+//     and streams the outputs out with 16-byte stores.  HBM traffic is one
+//     read of the inputs and one write of the outputs.
+//   * Look-back warp 1 stages the tile into shared memory (one TMA bulk copy
+//     per row), folds the summaries it needs from earlier tiles while the
+//     copies are in flight, and publishes the tile's own summary as soon as
+//     the scan warps' partial aggregates are in; look-back warp 2 derives the
+//     carry into the tile from earlier tiles' summaries, also starting at
+//     once.  A summary never waits on a carry: if it did, every tile of a
+//     chain would wait on the one before it.
 //   * The look-back is deterministic: tile j publishes the aggregate of the
 //     fixed range of tiles covered by Fenwick-tree node j+1, folded from its
 //     Fenwick children in a fixed order, and its carry is the fixed
 //     right-to-left fold of the Fenwick prefix nodes of position j.  Every
-//     value is therefore a function of the inputs alone, not of the order in
-//     which CTAs happen to run: repeated calls are bit-identical, and changing
-//     one episode leaves every other episode's outputs bit-identical.  Each
-//     tile reads at most ~2 log2(#tiles) summaries.
-//   * The tile is staged into shared memory with one TMA bulk copy per row;
-//     each warp owns R consecutive steps, each lane two complex channels
-//     (one 16-byte vector).  A lane scans its R steps serially, warps are
-//     combined through shared memory, and tiles through the look-back.
+//     value is a function of the inputs alone, not of the order in which
+//     CTAs happen to run: repeated calls are bit-identical, and changing one
+//     episode leaves every other episode's outputs bit-identical.
+//   * A summary is self-validating: each fp32 value is stored in a 64-bit
+//     word next to a per-launch tag (and the summary's begin-flag bit), and
+//     64-bit accesses are single-copy atomic, so a reader needs no separate
+//     status flag and a writer no fence: a summary is complete once every
+//     word carries this launch's tag.  Under a saturated memory system each
+//     dependent round trip costs microseconds, so this halves the look-back
+//     latency.
 //   * A begin flag inside a summary's range discards everything to its left,
-//     so folds stop at the first such summary (episode boundaries cut the
-//     look-back short); a tile whose first step is a begin flag needs no
-//     carry at all.
-//   * Outputs are recomputed from the carry with the plain recurrence and
-//     written with streaming 16-byte stores; HBM traffic is one read of the
-//     inputs and one write of the outputs.
-//   * Every wait (TMA completion, look-back) is bounded by the global timer;
-//     on expiry the kernel records an error in the workspace and returns.
-//
-// The backward pass is the same machinery run right to left over
-//     delta_t = grad_h_t + [b_{t+1} = 0] conj(lambda_{t+1}) delta_{t+1},
-// i.e. the element of step t is (conj(lambda_{t+1}), grad_h_t, b_{t+1}), plus
-// grad_lambda = sum_{b_t = 0} delta_t conj(h_{t-1}) (per-tile partials reduced
-// in a fixed order by a second kernel, so results are deterministic).
+//     so folds stop at the first such summary; a tile whose first step is a
+//     begin flag needs no carry at all.
+//   * Every wait (TMA completion, look-back flags) is bounded by the global
+//     timer; on expiry the kernel records an error in the workspace and
+//     returns.
+// grad_lambda (per-channel lambda) is accumulated per tile and reduced in a
+// fixed order by two small kernels, so it is deterministic as well.
 #include <cuda_runtime.h>
-
-#include <algorithm>
 
 #include "internal.cuh"
 #include "ptx.cuh"
@@ -52,18 +60,18 @@
 namespace memoroid {
 namespace diag {
 
-constexpr int SLAB = 64;                    // complex channels per slab
-// look-back status words: empty, Fenwick node published (its range holds no
-// begin flag / holds one), error
-constexpr uint32_t ST_EMPTY = 0, ST_NODE = 1, ST_NODE_RESET = 2, ST_ERROR = 3;
-constexpr int RED_PARTS = 64;               // first-stage parts of the grad_lambda reduction
-constexpr int MIN_T = 32;                   // smallest tile used (sizes the workspace)
+constexpr int SLAB = 64;  // complex channels per slab
+constexpr int NODE_WORDS = 8;  // 64-bit words per lane in a summary: a (4 floats), x (4 floats)
+#ifndef MEMOROID_NODE_BATCH
+#define MEMOROID_NODE_BATCH 2  // summaries read per round trip in a look-back fold
+#endif
+constexpr int NB_READ = MEMOROID_NODE_BATCH;
+constexpr int RED_PARTS = 64;  // first-stage parts of the grad_lambda reduction
+#ifndef MEMOROID_POLL_SLEEP_NS
+#define MEMOROID_POLL_SLEEP_NS 0  // longest back-off between flag polls
+#endif
 
-// tile shapes: W warps x R steps per warp
-constexpr int FWD_W = 8, FWD_R = 16;        // per-channel lambda: T = 128, 64 KB smem
-constexpr int FWDS_W = 8, FWDS_R = 8;       // per-step lambda:    T = 64, 64 KB smem
-constexpr int BWD_W = 8, BWD_R = 8;         // per-channel lambda: T = 64, 64 KB smem
-constexpr int BWDS_W = 4, BWDS_R = 8;       // per-step lambda:    T = 32, 48 KB smem
+constexpr int MIN_T = 16;      // smallest tile used (sizes the workspace)
 
 struct Params {
     const float4* lambda;  // [D/2] or [B, L, D/2]; one float4 = two complex channels
@@ -76,14 +84,13 @@ struct Params {
     const float4* g_last;  // bwd: grad_h_last or null
     float4* grad_lambda;   // bwd, per-step lambda: [B, L, D/2] or null
     float4* grad_h0;       // bwd: [B, D/2] or null
-    int64_t B, L, D2, n_slabs, n_tt, n_chains;
-    int64_t D;
-    uint32_t* hdr;         // workspace header
-    uint32_t* flags;       // [n_chains * n_tt]
-    float4* node;          // [n_chains * n_tt * 32 * 2]  Fenwick node (a, x) per lane
-    float4* gpart;         // [n_chains * n_tt * 32]      per-tile grad_lambda
+    int64_t B, L, D2, n_slabs, n_tt, n_chains, n_tiles;
+    uint32_t* hdr;               // workspace header: [0] error, [1] ticket counter
+    unsigned long long* node;    // [n_chains * n_tt * 32 * NODE_WORDS] tagged Fenwick nodes
+    float4* gpart;               // [n_chains * n_tt * 32]      per-tile grad_lambda
     uint64_t wait_ns;
     int64_t withhold;
+    uint32_t epoch;              // this launch's tag (31 bits, non-zero)
 };
 
 __host__ __device__ __forceinline__ int64_t lmin(int64_t a, int64_t b) { return a < b ? a : b; }
@@ -106,6 +113,79 @@ __device__ __forceinline__ float4 add2(float4 a, float4 b) {
     return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
 }
 
+// ---- tile shapes -------------------------------------------------------------
+// W warps x R steps per warp; REV = backward; PS = per-step lambda.
+template <int W_, int R_, bool REV_, bool PS_>
+struct Cfg {
+    static constexpr int W = W_, R = R_, T = W_ * R_;
+    static constexpr bool REV = REV_, PS = PS_;
+    // arrays staged per tile: input [, h (backward)] [, lambda (per step)]
+    static constexpr int NB = 1 + (REV_ ? 1 : 0) + (PS_ ? 1 : 0);
+    static constexpr int BUF_F4 = T * 32;  // float4 per staged array
+    static constexpr int THREADS = (W_ + 2) * 32;  // W scan warps + 2 look-back warps
+    static constexpr int NSYNC = (W_ + 1) * 32;    // scan warps + one look-back warp
+    // shared memory layout (bytes)
+    static constexpr size_t OFF_WA = size_t(NB) * BUF_F4 * 16;
+    static constexpr size_t OFF_WX = OFF_WA + W_ * 32 * 16;
+    static constexpr size_t OFF_CARRY = OFF_WX + W_ * 32 * 16;
+    static constexpr size_t OFF_ACC = OFF_CARRY + 32 * 16;
+    static constexpr size_t OFF_WR = OFF_ACC + ((REV_ && !PS_) ? W_ * 32 * 16 : 0);
+    static constexpr size_t OFF_MISC = (OFF_WR + W_ * 4 + 15) / 16 * 16;  // bar, ticket, abort
+    static constexpr size_t SMEM = OFF_MISC + 32;
+    static_assert(R_ < 32, "R + 1 begin flags are read by one warp");
+};
+
+struct Tile {
+    int64_t tk;      // ticket (-1: no more work)
+    int64_t b, c2;   // tape, first float4 column of the slab
+    int64_t pos;     // position in the chain (left-to-right forward, right-to-left backward)
+    int64_t t0;      // first step
+    int64_t fbase;   // chain * n_tt
+    int width2;      // float4 columns in the slab
+    int nrows;       // steps in the tile
+};
+
+template <class C>
+__device__ __forceinline__ Tile decode(const Params& p, int64_t tk) {
+    Tile t{};
+    t.tk = tk;
+    if (tk < 0) return t;
+    const int64_t q = tk / p.n_chains;
+    const int64_t chain = tk - q * p.n_chains;
+    t.pos = q;
+    const int64_t j = C::REV ? p.n_tt - 1 - q : q;
+    t.b = chain / p.n_slabs;
+    t.c2 = (chain - t.b * p.n_slabs) * (SLAB / 2);
+    t.width2 = static_cast<int>(lmin(SLAB / 2, p.D2 - t.c2));
+    t.t0 = j * C::T;
+    t.nrows = static_cast<int>(lmin(C::T, p.L - t.t0));
+    t.fbase = chain * p.n_tt;
+    return t;
+}
+
+// ---- optional per-tile timeline (tuning builds only) ---------------------------
+#ifdef MEMOROID_TRACE
+__device__ unsigned long long* g_trace;  // [ticket][16] global-timer stamps
+#define TRACE_TK(ticket, slot)                                                                   \
+    do {                                                                                         \
+        if (g_trace != nullptr && (threadIdx.x & 31) == 0 && (slot) >= 0)                        \
+            g_trace[(ticket) * 16 + (slot)] = static_cast<unsigned long long>(ptx::globaltimer()); \
+    } while (0)
+#else
+#define TRACE_TK(ticket, slot) (void)0
+#endif
+#define TRACE(slot) TRACE_TK(tk, slot)
+
+// ---- optional wait profiling (tuning builds only) -----------------------------
+#ifdef MEMOROID_PROFILE_WAITS
+#define PROF_T0() const uint64_t _pt0 = ptx::globaltimer()
+#define PROF_ADD(slot) atomicAdd(reinterpret_cast<unsigned long long*>(p.hdr + 32) + (slot), \
+                                 static_cast<unsigned long long>(ptx::globaltimer() - _pt0))
+#else
+#define PROF_T0() (void)0
+#define PROF_ADD(slot) (void)0
+#endif
+
 // ---- errors and bounded waits -------------------------------------------------
 __device__ __forceinline__ void record_error(const Params& p, uint32_t code, int64_t ticket) {
     if (atomicCAS(p.hdr, 0u, code) == 0u) {
@@ -114,191 +194,195 @@ __device__ __forceinline__ void record_error(const Params& p, uint32_t code, int
     }
 }
 
-// Lane-0 wait on a look-back flag; returns the published status, or
-// ST_ERROR after recording a timeout (or seeing another tile's error).
-__device__ uint32_t wait_flag(const Params& p, const uint32_t* f, uint64_t t_begin,
-                              int64_t ticket) {
-    uint32_t v = ptx::ld_acquire(f);
-    unsigned ns = 32;
-    while (v == ST_EMPTY) {
-        if (ptx::ld_relaxed(p.hdr) != 0u) return ST_ERROR;
-        if (ptx::globaltimer() - t_begin > p.wait_ns) {
-            record_error(p, DEV_LOOKBACK_TIMEOUT, ticket);
-            return ST_ERROR;
-        }
-        __nanosleep(ns);
-        if (ns < 1024) ns <<= 1;
-        v = ptx::ld_acquire(f);
-    }
-    return v;
-}
-
-// Bounded wait on the TMA mbarrier (all threads).
-__device__ bool wait_tma(const Params& p, uint64_t* bar, uint64_t t_begin, int64_t ticket) {
-    while (!ptx::mbar_try_wait(bar, 0)) {
-        if (ptx::globaltimer() - t_begin > p.wait_ns) {
-            record_error(p, DEV_TMA_TIMEOUT, ticket);
-            return false;
-        }
-    }
-    return true;
-}
-
-// Publishes a status word after this warp's payload stores (all lanes call).
-__device__ __forceinline__ void publish(uint32_t* f, uint32_t status, bool skip) {
-    __threadfence();
-    __syncwarp();
-    if (!skip && (threadIdx.x & 31) == 0) ptx::st_release(f, status);
-}
-
-// Waits for the Fenwick node of chain position `pos` (1-based; stored at
-// tile index pos-1) and folds it onto the left of (Ra, Rx, Rb), which must
-// hold no begin flag yet:  node o R = (R.a * node.a, R.a * node.x + R.x, node.b).
-// Warp-wide; returns false on timeout / error.
-__device__ bool fold_node(const Params& p, int64_t fbase, int64_t pos, float4& Ra, float4& Rx,
-                          bool& Rb, uint64_t t_begin, int64_t ticket) {
+// Publishes this lane's part of a Fenwick node (tile index idx): a, x and
+// the begin-flag bit, each value tagged with the launch's epoch.
+__device__ __forceinline__ void store_node(const Params& p, int64_t idx, float4 a, float4 x, bool b) {
     const int lane = threadIdx.x & 31;
-    const uint32_t* f = p.flags + fbase + pos - 1;
-    uint32_t st = 0;
-    if (lane == 0) st = wait_flag(p, f, t_begin, ticket);
-    st = __shfl_sync(0xffffffffu, st, 0);
-    if (st == ST_ERROR) return false;
-    (void)ptx::ld_acquire(f);  // every lane acquires before reading the payload
-    const int64_t idx = (fbase + pos - 1) * 32 + lane;
-    const float4 a = __ldcg(p.node + 2 * idx);
-    const float4 x = __ldcg(p.node + 2 * idx + 1);
-    Rx = cfma2(Ra, x, Rx);
-    Ra = cmul2(Ra, a);
-    Rb = (st == ST_NODE_RESET);
-    return true;
+    unsigned long long* dst = p.node + (idx * 32 + lane) * NODE_WORDS;
+    const unsigned long long hi = static_cast<unsigned long long>((p.epoch << 1) | (b ? 1u : 0u)) << 32;
+    auto w = [&](float v) { return hi | static_cast<unsigned long long>(__float_as_uint(v)); };
+    ptx::st_relaxed_v2u64(dst + 0, w(a.x), w(a.y));
+    ptx::st_relaxed_v2u64(dst + 2, w(a.z), w(a.w));
+    ptx::st_relaxed_v2u64(dst + 4, w(x.x), w(x.y));
+    ptx::st_relaxed_v2u64(dst + 6, w(x.z), w(x.w));
 }
 
-// Look-back of chain position j (0-based) for a tile whose aggregate is
-// (Ta, Tx, Tb) (warp-wide, warp 0).
-//  1. Publishes Fenwick node j+1, the aggregate of tiles [j+1-lowbit(j+1), j]:
-//     its children j, j-1, j-3, ... (positions j+1-k, k = 1, 2, 4, .. <
-//     lowbit) folded right to left onto the tile's own aggregate.
-//  2. If need_carry, returns the state entering tile j: the Fenwick prefix
-//     nodes of position j folded right to left, applied to `base` (the state
-//     before the chain's first step) unless a begin flag intervenes.
-// Folds stop early at a begin flag: everything to its left is discarded by
-// the select of Theorem 3.2, so stopping changes no bit of the result.
-__device__ bool fenwick_lookback(const Params& p, int64_t fbase, int64_t j, float4 Ta, float4 Tx,
-                                 bool Tb, bool need_carry, float4 base, float4& carry,
-                                 uint64_t t_begin, int64_t ticket, bool skip) {
+// Reads this lane's part of a Fenwick node.  Returns true if all of its
+// words carry this launch's tag (then b holds the node's begin-flag bit).
+__device__ __forceinline__ bool load_node(const Params& p, int64_t idx, float4& a, float4& x, bool& b) {
     const int lane = threadIdx.x & 31;
-    const int64_t pos = j + 1;
-    const int64_t lb = pos & (-pos);
+    const unsigned long long* src = p.node + (idx * 32 + lane) * NODE_WORDS;
+    unsigned long long w[NODE_WORDS];
+    ptx::ld_relaxed_v2u64(src + 0, w[0], w[1]);
+    ptx::ld_relaxed_v2u64(src + 2, w[2], w[3]);
+    ptx::ld_relaxed_v2u64(src + 4, w[4], w[5]);
+    ptx::ld_relaxed_v2u64(src + 6, w[6], w[7]);
     bool ok = true;
-    float4 Na = Ta, Nx = Tx;
-    bool Nb = Tb;
-    for (int64_t k = 1; k < lb && !Nb; k <<= 1) {
-        if (!fold_node(p, fbase, pos - k, Na, Nx, Nb, t_begin, ticket)) {
-            ok = false;
-            break;
+#pragma unroll
+    for (int i = 0; i < NODE_WORDS; ++i) ok = ok && static_cast<uint32_t>(w[i] >> 33) == p.epoch;
+    b = (w[0] >> 32) & 1u;
+    a = make_float4(__uint_as_float(static_cast<uint32_t>(w[0])), __uint_as_float(static_cast<uint32_t>(w[1])),
+                    __uint_as_float(static_cast<uint32_t>(w[2])), __uint_as_float(static_cast<uint32_t>(w[3])));
+    x = make_float4(__uint_as_float(static_cast<uint32_t>(w[4])), __uint_as_float(static_cast<uint32_t>(w[5])),
+                    __uint_as_float(static_cast<uint32_t>(w[6])), __uint_as_float(static_cast<uint32_t>(w[7])));
+    return ok;
+}
+
+// Folds the Fenwick nodes whose positions lanes 0..n-1 hold in `mypos`
+// (lane 0 the right-most) onto the left of (Ra, Rx, Rb) in that order:
+// node o R = (R.a * node.a, R.a * node.x + R.x, node.b) while R holds no begin
+// flag.  The fold stops after the first node whose range holds one (every
+// node further left would be discarded by the select of Theorem 3.2, so
+// stopping changes no bit).  Nodes are read four at a time and re-read until
+// every lane sees them complete.  Warp-wide; false on timeout / error.
+__device__ bool fold_nodes(const Params& p, int64_t fbase, int64_t mypos, int n, float4& Ra,
+                           float4& Rx, bool& Rb, int64_t ticket, int trace_slot = -1) {
+    for (int m0 = 0; m0 < n && !Rb; m0 += NB_READ) {
+        int64_t pk[NB_READ];
+#pragma unroll
+        for (int k = 0; k < NB_READ; ++k) pk[k] = __shfl_sync(0xffffffffu, mypos, (m0 + k) & 31);
+        const int cnt = n - m0 < NB_READ ? n - m0 : NB_READ;
+        uint32_t pending = (1u << cnt) - 1u;
+        float4 a[NB_READ], x[NB_READ];
+        bool rb[NB_READ];
+        uint64_t t0 = 0;
+        for (uint32_t it = 0; pending != 0u; ++it) {
+#pragma unroll
+            for (int k = 0; k < NB_READ; ++k) {
+                if ((pending >> k) & 1u) {
+                    const bool ok = load_node(p, fbase + pk[k] - 1, a[k], x[k], rb[k]);
+                    if (__all_sync(0xffffffffu, ok)) pending &= ~(1u << k);
+                }
+            }
+            if (pending == 0u) break;
+            if (it == 0) t0 = ptx::globaltimer();
+            if ((it & 15u) == 15u) {
+                if (ptx::ld_relaxed(p.hdr) != 0u) return false;
+                if (ptx::globaltimer() - t0 > p.wait_ns) {
+                    if ((threadIdx.x & 31) == 0) record_error(p, DEV_LOOKBACK_TIMEOUT, ticket);
+                    return false;
+                }
+            }
+            if (MEMOROID_POLL_SLEEP_NS > 0) __nanosleep(MEMOROID_POLL_SLEEP_NS);
+        }
+#pragma unroll
+        for (int k = 0; k < NB_READ; ++k) {
+            if (k < cnt && !Rb) {
+                Rx = cfma2(Ra, x[k], Rx);
+                Ra = cmul2(Ra, a[k]);
+                Rb = rb[k];
+            }
         }
     }
-    uint32_t* myflag = p.flags + fbase + j;
-    if (ok) {
-        const int64_t idx = (fbase + j) * 32 + lane;
-        __stcg(p.node + 2 * idx, Na);
-        __stcg(p.node + 2 * idx + 1, Nx);
-        publish(myflag, Nb ? ST_NODE_RESET : ST_NODE, skip);
-    } else {
-        if (lane == 0 && !skip) ptx::st_release(myflag, ST_ERROR);
-        return false;
-    }
-    carry = base;
-    if (!need_carry) return true;
+    TRACE_TK(ticket, trace_slot);
+    return true;
+}
+
+// Fenwick node pos (1-based; tile pos-1 of the chain) covers tiles
+// [pos - lowbit(pos), pos - 1].  Its children are the nodes pos - k for
+// k = 1, 2, 4, .. < lowbit(pos); they cover the same range minus tile pos-1.
+// Returns the children folded right to left, C = child(pos - lowbit/2) o ...
+// o child(pos - 1) (the identity if there are none).
+__device__ bool fenwick_children(const Params& p, int64_t fbase, int64_t pos, float4& Ca, float4& Cx,
+                                 bool& Cb, int64_t ticket) {
+    const int lane = threadIdx.x & 31;
+    const int64_t lb = pos & (-pos);
+    const int nc = 63 - __clzll(static_cast<long long>(lb));  // log2(lowbit(pos))
+    Ca = one2();
+    Cx = zero2();
+    Cb = false;
+    if (nc == 0) return true;
+    const int64_t child = pos - (int64_t(1) << (lane < nc ? lane : 0));
+    return fold_nodes(p, fbase, child, nc, Ca, Cx, Cb, ticket, 9);
+}
+
+// Publishes node j+1 = C o T (T: the tile's own aggregate) unless !ok or the
+// debug knob withholds it.  Warp-wide.
+__device__ void fenwick_publish(const Params& p, int64_t fbase, int64_t j, float4 Ca, float4 Cx, bool Cb,
+                                float4 Ta, float4 Tx, bool Tb, bool ok, bool skip) {
+    if (!ok || skip) return;
+    const float4 Na = Tb ? Ta : cmul2(Ta, Ca);
+    const float4 Nx = Tb ? Tx : cfma2(Ta, Cx, Tx);
+    store_node(p, fbase + j, Na, Nx, Tb || Cb);
+}
+
+// State entering chain position j > 0: the Fenwick prefix nodes of position j
+// (j, j - lowbit(j), ...) folded right to left, applied to `base` (the state
+// before the chain's first step) unless a begin flag intervenes.  Warp-wide.
+__device__ bool fenwick_carry(const Params& p, int64_t fbase, int64_t j, float4 base, float4& carry,
+                              int64_t ticket) {
+    const int lane = threadIdx.x & 31;
+    int64_t q = j;  // lane i holds the i-th prefix node position
+    for (int k = 0; k < lane && q > 0; ++k) q -= q & (-q);
+    const int nq = __popcll(static_cast<unsigned long long>(j));
     float4 Ra = one2(), Rx = zero2();
     bool Rb = false;
-    for (int64_t q = j; q > 0 && !Rb; q -= (q & (-q))) {
-        if (!fold_node(p, fbase, q, Ra, Rx, Rb, t_begin, ticket)) return false;
-    }
+    if (!fold_nodes(p, fbase, q, nq, Ra, Rx, Rb, ticket, 8)) return false;
     carry = Rb ? Rx : cfma2(Ra, base, Rx);
     return true;
 }
 
 // ============================================================================
-// forward
+// the scan kernel (forward: REV = false; backward: REV = true), one tile per CTA
 // ============================================================================
-template <int W, int R, bool PER_STEP>
-__global__ void __launch_bounds__(W * 32) diag_fwd_kernel(const Params p) {
-    constexpr int T = W * R;
-    extern __shared__ __align__(128) unsigned char smem_raw[];
-    float4* s_u = reinterpret_cast<float4*>(smem_raw);  // [T][32]
-    float4* s_l = s_u + T * 32;                         // [T][32] (per-step lambda)
-    __shared__ float4 s_wa[W][32], s_wx[W][32];
-    __shared__ uint32_t s_wr[W];
-    __shared__ float4 s_carry[32];
-    __shared__ __align__(8) uint64_t s_bar;
-    __shared__ long long s_ticket;
-    __shared__ int s_abort;
+template <class C>
+__global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
+    constexpr int W = C::W, R = C::R;
+    constexpr int LB_PUBLISH = W, LB_CARRY = W + 1;  // the two look-back warps
+    // named barriers: 1 aggregates ready (scan warps -> publisher),
+    // 2 carry ready (carry warp <-> scan warps), 3 grad_lambda parts ready
+    constexpr int BAR_AGG = 1, BAR_CARRY = 2, BAR_ACC = 3;
+    extern __shared__ __align__(128) unsigned char smem[];
+    float4* s_in = reinterpret_cast<float4*>(smem);                     // [T][32] input rows
+    float4* s_h = s_in + C::BUF_F4;                                       // [T][32] h_{t-1} (backward)
+    float4* s_l = s_in + (C::NB - 1) * C::BUF_F4;                         // [T][32] lambda (per step)
+    float4* s_wa = reinterpret_cast<float4*>(smem + C::OFF_WA);          // [W][32] warp aggregate a
+    float4* s_wx = reinterpret_cast<float4*>(smem + C::OFF_WX);          // [W][32] warp aggregate x
+    float4* s_carry = reinterpret_cast<float4*>(smem + C::OFF_CARRY);    // [32] carry into the tile
+    float4* s_acc = reinterpret_cast<float4*>(smem + C::OFF_ACC);        // [W][32] grad_lambda parts
+    uint32_t* s_wr = reinterpret_cast<uint32_t*>(smem + C::OFF_WR);      // [W] warp holds a reset
+    uint64_t* bar = reinterpret_cast<uint64_t*>(smem + C::OFF_MISC);
+    long long* s_tk = reinterpret_cast<long long*>(smem + C::OFF_MISC + 8);
+    volatile int* s_abort = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 16);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
-        s_ticket = static_cast<long long>(atomicAdd(p.hdr + 1, 1u));
-        s_abort = 0;
-        ptx::mbar_init(&s_bar, 1);
+        *s_tk = static_cast<long long>(atomicAdd(p.hdr + 1, 1u));
+        *s_abort = 0;
+        ptx::mbar_init(bar, 1);
         ptx::fence_mbar_init();
     }
     __syncthreads();
-    const int64_t ticket = s_ticket;
-    const int64_t j = ticket / p.n_chains;       // position in chain = time tile
-    const int64_t chain = ticket - j * p.n_chains;
-    const int64_t b = chain / p.n_slabs;
-    const int64_t slab = chain - b * p.n_slabs;
-    const int64_t t0 = j * T;
-    const int64_t c2 = slab * (SLAB / 2);        // first float4 column of the slab
-    const int width2 = static_cast<int>(lmin(SLAB / 2, p.D2 - c2));  // float4 columns
-    const int nrows = static_cast<int>(lmin(T, p.L - t0));
-    const uint64_t t_begin = ptx::globaltimer();
+    const int64_t tk = *s_tk;
+    const Tile t = decode<C>(p, tk);
+    const bool lane_ok = lane < t.width2;
+    if (warp == 0) TRACE(0);
 
-    if (warp == 0) {
-        const uint32_t rb = static_cast<uint32_t>(width2) * 16u;
-        if (lane == 0) ptx::mbar_arrive_expect_tx(&s_bar, rb * nrows * (PER_STEP ? 2u : 1u));
+    if (warp == LB_PUBLISH) {
+        // ----------------------------------------- stage the tile, publish its summary
+        const uint32_t rb = static_cast<uint32_t>(t.width2) * 16u;
+        const int h_rows = C::REV ? t.nrows - (t.t0 == 0 ? 1 : 0) : 0;  // rows t0-1 ..
+        const int l_rows = !C::PS ? 0 : (C::REV ? static_cast<int>(lmin(t.nrows, p.L - 1 - t.t0)) : t.nrows);
+        if (lane == 0) ptx::mbar_arrive_expect_tx(bar, rb * (t.nrows + h_rows + l_rows));
         __syncwarp();
-        for (int r = lane; r < nrows; r += 32) {
-            const int64_t g = (b * p.L + t0 + r) * p.D2 + c2;
-            ptx::bulk_g2s(s_u + r * 32, p.in + g, rb, &s_bar);
-            if (PER_STEP) ptx::bulk_g2s(s_l + r * 32, p.lambda + g, rb, &s_bar);
+        for (int r = lane; r < t.nrows; r += 32) {
+            const int64_t g = (t.b * p.L + t.t0 + r) * p.D2 + t.c2;
+            ptx::bulk_g2s(s_in + r * 32, p.in + g, rb, bar);
+            if (C::REV && t.t0 + r >= 1) ptx::bulk_g2s(s_h + r * 32, p.h + g - p.D2, rb, bar);
+            if (C::PS && r < l_rows) ptx::bulk_g2s(s_l + r * 32, p.lambda + g + (C::REV ? p.D2 : 0), rb, bar);
         }
-    }
-
-    // begin flags of this warp's steps (overlaps the copies)
-    const int64_t ts = t0 + static_cast<int64_t>(warp) * R;
-    const int nv = static_cast<int>(lmax(0, lmin(R, p.L - ts)));
-    const uint32_t bit = (lane < nv) ? (p.start[b * p.L + ts + lane] != 0) : 0u;
-    const uint32_t rmask = __ballot_sync(0xffffffffu, bit);
-    const bool lane_ok = lane < width2;
-    const float4 lam = (!PER_STEP && lane_ok) ? p.lambda[c2 + lane] : one2();
-
-    if (!wait_tma(p, &s_bar, t_begin, ticket)) return;
-
-    // phase 1: aggregate of this warp's R steps (from the identity)
-    float4 a = one2(), x = zero2();
-    for (int i = 0; i < nv; ++i) {
-        const float4 uu = s_u[(warp * R + i) * 32 + lane];
-        const float4 ll = PER_STEP ? s_l[(warp * R + i) * 32 + lane] : lam;
-        if ((rmask >> i) & 1u) {
-            a = ll;
-            x = uu;
-        } else {
-            x = cfma2(ll, x, uu);
-            a = cmul2(ll, a);
-        }
-    }
-    s_wa[warp][lane] = a;
-    s_wx[warp][lane] = x;
-    if (lane == 0) s_wr[warp] = (rmask != 0u);
-    __syncthreads();
-
-    // phase 2: tile aggregate, publish, look back (warp 0)
-    if (warp == 0) {
+        float4 Ca, Cx;
+        bool Cb;
+        bool ok = fenwick_children(p, t.fbase, t.pos + 1, Ca, Cx, Cb, tk);
+        TRACE(1);
+        ptx::named_sync(BAR_AGG, C::NSYNC);
+        TRACE(2);
+        // the tile's aggregate: the scan warps' aggregates folded in processing order
         float4 Ta = one2(), Tx = zero2();
         bool Tb = false;
-        for (int v = 0; v < W; ++v) {
-            const float4 wa = s_wa[v][lane], wx = s_wx[v][lane];
+        for (int k = 0; k < W; ++k) {
+            const int v = C::REV ? W - 1 - k : k;
+            const float4 wa = s_wa[v * 32 + lane], wx = s_wx[v * 32 + lane];
             if (s_wr[v]) {
                 Ta = wa;
                 Tx = wx;
@@ -308,214 +392,177 @@ __global__ void __launch_bounds__(W * 32) diag_fwd_kernel(const Params p) {
                 Ta = cmul2(wa, Ta);
             }
         }
-        const int64_t fbase = chain * p.n_tt;
-        const bool skip = (ticket == p.withhold);
-        const bool first_is_start = (rmask & 1u) != 0u;
-        // state before the chain's first step: h0 (or the identity's 0)
-        const float4 base = (p.h0 != nullptr && lane_ok) ? p.h0[b * p.D2 + c2 + lane] : zero2();
-        float4 carry = zero2();
-        const bool ok = fenwick_lookback(p, fbase, j, Ta, Tx, Tb, !first_is_start, base, carry,
-                                         t_begin, ticket, skip);
+        ok = ok && (*s_abort == 0);
+        fenwick_publish(p, t.fbase, t.pos, Ca, Cx, Cb, Ta, Tx, Tb, ok, tk == p.withhold);
+        TRACE(3);
+        return;
+    }
+
+    if (warp == LB_CARRY) {
+        // ------------------------------------------------- carry into the tile
+        bool need_carry;
+        float4 base = zero2();
+        if (!C::REV) {
+            need_carry = p.start[t.b * p.L + t.t0] == 0;
+            if (p.h0 != nullptr && lane_ok) base = p.h0[t.b * p.D2 + t.c2 + lane];
+        } else {
+            // the first step processed is t0 + nrows - 1; its carry is cut if b_{t0+nrows} = 1
+            const int64_t tn = t.t0 + t.nrows;
+            need_carry = !(tn < p.L && p.start[t.b * p.L + tn] != 0);
+            if (p.g_last != nullptr && lane_ok) base = p.g_last[t.b * p.D2 + t.c2 + lane];
+        }
+        float4 carry = base;
+        bool ok = true;
+        if (need_carry && t.pos > 0) ok = fenwick_carry(p, t.fbase, t.pos, base, carry, tk);
+        TRACE(4);
         s_carry[lane] = carry;
-        if (lane == 0 && !ok) s_abort = 1;
-    }
-    __syncthreads();
-    if (s_abort) return;
-
-    // phase 3: carry into this warp, recompute and store
-    float4 Ea = one2(), Ex = zero2();
-    bool Eb = false;
-    for (int v = 0; v < warp; ++v) {
-        const float4 wa = s_wa[v][lane], wx = s_wx[v][lane];
-        if (s_wr[v]) {
-            Ea = wa;
-            Ex = wx;
-            Eb = true;
-        } else {
-            Ex = cfma2(wa, Ex, wx);
-            Ea = cmul2(wa, Ea);
+        if (!ok && lane == 0) *s_abort = 1;
+        ptx::named_sync(BAR_CARRY, C::NSYNC);
+        if (C::REV && !C::PS && *s_abort == 0) {
+            // grad_lambda partial of this tile, summed over warps in a fixed order
+            ptx::named_sync(BAR_ACC, C::NSYNC);
+            float4 sum = zero2();
+            for (int v = 0; v < W; ++v) sum = add2(sum, s_acc[v * 32 + lane]);
+            const int64_t jt = p.n_tt - 1 - t.pos;
+            p.gpart[(t.fbase + jt) * 32 + lane] = sum;
         }
-    }
-    float4 hc = Eb ? Ex : cfma2(Ea, s_carry[lane], Ex);
-    if (lane_ok) {
-        float4* dst = p.out + (b * p.L + ts) * p.D2 + c2 + lane;
-        for (int i = 0; i < nv; ++i) {
-            const float4 uu = s_u[(warp * R + i) * 32 + lane];
-            const float4 ll = PER_STEP ? s_l[(warp * R + i) * 32 + lane] : lam;
-            hc = ((rmask >> i) & 1u) ? uu : cfma2(ll, hc, uu);
-            __stcs(dst + static_cast<int64_t>(i) * p.D2, hc);
-        }
-        if (p.out_last != nullptr && nv > 0 && ts + nv == p.L) p.out_last[b * p.D2 + c2 + lane] = hc;
-    }
-}
-
-// ============================================================================
-// backward (right-to-left)
-// ============================================================================
-template <int W, int R, bool PER_STEP>
-__global__ void __launch_bounds__(W * 32) diag_bwd_kernel(const Params p) {
-    static_assert(R < 32, "R + 1 begin flags are read by one warp");
-    constexpr int T = W * R;
-    extern __shared__ __align__(128) unsigned char smem_raw[];
-    float4* s_g = reinterpret_cast<float4*>(smem_raw);  // row i: grad_h_{t0+i}
-    float4* s_h = s_g + T * 32;                          // row i: h_{t0+i-1}
-    float4* s_l = s_h + T * 32;                          // row i: lambda_{t0+i+1} (per step)
-    __shared__ float4 s_wa[W][32], s_wx[W][32];
-    __shared__ uint32_t s_wr[W];
-    __shared__ float4 s_carry[32];
-    __shared__ float4 s_acc[W][32];
-    __shared__ __align__(8) uint64_t s_bar;
-    __shared__ long long s_ticket;
-    __shared__ int s_abort;
-
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (threadIdx.x == 0) {
-        s_ticket = static_cast<long long>(atomicAdd(p.hdr + 1, 1u));
-        s_abort = 0;
-        ptx::mbar_init(&s_bar, 1);
-        ptx::fence_mbar_init();
-    }
-    __syncthreads();
-    const int64_t ticket = s_ticket;
-    const int64_t jr = ticket / p.n_chains;  // position in chain (right to left)
-    const int64_t chain = ticket - jr * p.n_chains;
-    const int64_t j = p.n_tt - 1 - jr;       // time tile
-    const int64_t b = chain / p.n_slabs;
-    const int64_t slab = chain - b * p.n_slabs;
-    const int64_t t0 = j * T;
-    const int64_t c2 = slab * (SLAB / 2);
-    const int width2 = static_cast<int>(lmin(SLAB / 2, p.D2 - c2));
-    const int nrows = static_cast<int>(lmin(T, p.L - t0));
-    const uint64_t t_begin = ptx::globaltimer();
-
-    if (warp == 0) {
-        const uint32_t rb = static_cast<uint32_t>(width2) * 16u;
-        const int h_rows = nrows - (t0 == 0 ? 1 : 0);                               // rows t0-1 .. t0+nrows-2
-        const int l_rows = PER_STEP ? static_cast<int>(lmin(nrows, p.L - 1 - t0)) : 0;  // rows t0+1 ..
-        if (lane == 0) ptx::mbar_arrive_expect_tx(&s_bar, rb * (nrows + h_rows + l_rows));
-        __syncwarp();
-        for (int r = lane; r < nrows; r += 32) {
-            const int64_t g = (b * p.L + t0 + r) * p.D2 + c2;
-            ptx::bulk_g2s(s_g + r * 32, p.in + g, rb, &s_bar);
-            if (t0 + r >= 1) ptx::bulk_g2s(s_h + r * 32, p.h + g - p.D2, rb, &s_bar);
-            if (PER_STEP && r < l_rows) ptx::bulk_g2s(s_l + r * 32, p.lambda + g + p.D2, rb, &s_bar);
-        }
+        return;
     }
 
-    const int64_t ts = t0 + static_cast<int64_t>(warp) * R;
+    // ----------------------------------------------------------------- scan warps
+    const int64_t ts = t.t0 + static_cast<int64_t>(warp) * R;
     const int nv = static_cast<int>(lmax(0, lmin(R, p.L - ts)));
-    // bit i of bmask: b_{ts+i} for i <= R (0 past the tape end)
-    const uint32_t bit = (lane <= R && ts + lane < p.L) ? (p.start[b * p.L + ts + lane] != 0) : 0u;
-    const uint32_t bmask = __ballot_sync(0xffffffffu, bit);
-    const uint32_t rmask = bmask >> 1;  // bit i: b_{ts+i+1}, the reset of the reverse element
-    const bool lane_ok = lane < width2;
-    const float4 lam = (!PER_STEP && lane_ok) ? p.lambda[c2 + lane] : one2();
+    uint32_t rmask, bmask;
+    if (!C::REV) {
+        const uint32_t bit = (lane < nv) ? (p.start[t.b * p.L + ts + lane] != 0) : 0u;
+        rmask = bmask = __ballot_sync(0xffffffffu, bit);
+    } else {
+        // bit k of bmask: b_{ts+k} for k <= R (0 past the tape end);
+        // bit k of rmask: b_{ts+k+1}, the reset of the reverse element of step ts+k
+        const uint32_t bit = (lane <= R && ts + lane < p.L) ? (p.start[t.b * p.L + ts + lane] != 0) : 0u;
+        bmask = __ballot_sync(0xffffffffu, bit);
+        rmask = bmask >> 1;
+    }
+    const float4 lam = (!C::PS && lane_ok) ? p.lambda[t.c2 + lane] : one2();
     const float4 mlam = conj2(lam);
+    const float4* sin = s_in + warp * R * 32 + lane;
+    const float4* sl = s_l + warp * R * 32 + lane;
 
-    if (!wait_tma(p, &s_bar, t_begin, ticket)) return;
+    bool landed = true;
+    {
+        const uint64_t w0 = ptx::globaltimer();
+        while (!ptx::mbar_try_wait(bar, 0)) {
+            if (ptx::globaltimer() - w0 > p.wait_ns) {
+                record_error(p, DEV_TMA_TIMEOUT, tk);
+                landed = false;
+                break;
+            }
+        }
+    }
+    if (!landed && lane == 0) *s_abort = 1;
+    if (warp == 0) TRACE(5);
 
-    // phase 1: aggregate over this warp's steps, right to left
+    // phase 1: aggregate of this warp's steps, from the identity, in processing order
     float4 a = one2(), x = zero2();
-    for (int i = nv - 1; i >= 0; --i) {
-        const int64_t t = ts + i;
-        const float4 gg = s_g[(warp * R + i) * 32 + lane];
-        const float4 m = (t == p.L - 1) ? one2() : (PER_STEP ? conj2(s_l[(warp * R + i) * 32 + lane]) : mlam);
-        if ((rmask >> i) & 1u) {
-            a = m;
-            x = gg;
+    if (landed) {
+        if (!C::REV) {
+            for (int k = 0; k < nv; ++k) {
+                const float4 uu = sin[k * 32];
+                const float4 ll = C::PS ? sl[k * 32] : lam;
+                if ((rmask >> k) & 1u) {
+                    a = ll;
+                    x = uu;
+                } else {
+                    x = cfma2(ll, x, uu);
+                    a = cmul2(ll, a);
+                }
+            }
         } else {
-            x = cfma2(m, x, gg);
-            a = cmul2(m, a);
+            for (int k = nv - 1; k >= 0; --k) {
+                const float4 gg = sin[k * 32];
+                const float4 m = (ts + k == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
+                if ((rmask >> k) & 1u) {
+                    a = m;
+                    x = gg;
+                } else {
+                    x = cfma2(m, x, gg);
+                    a = cmul2(m, a);
+                }
+            }
         }
     }
     const uint32_t vmask = (nv >= 32) ? 0xffffffffu : ((1u << nv) - 1u);
-    s_wa[warp][lane] = a;
-    s_wx[warp][lane] = x;
+    s_wa[warp * 32 + lane] = a;
+    s_wx[warp * 32 + lane] = x;
     if (lane == 0) s_wr[warp] = ((rmask & vmask) != 0u);
-    __syncthreads();
+    ptx::named_arrive(BAR_AGG, C::NSYNC);
+    ptx::named_sync(BAR_CARRY, C::NSYNC);
+    if (*s_abort) return;
 
-    if (warp == 0) {
-        float4 Ta = one2(), Tx = zero2();
-        bool Tb = false;
-        for (int v = W - 1; v >= 0; --v) {
-            const float4 wa = s_wa[v][lane], wx = s_wx[v][lane];
-            if (s_wr[v]) {
-                Ta = wa;
-                Tx = wx;
-                Tb = true;
-            } else {
-                Tx = cfma2(wa, Tx, wx);
-                Ta = cmul2(wa, Ta);
-            }
-        }
-        const int64_t fbase = chain * p.n_tt;
-        const bool skip = (ticket == p.withhold);
-        // the first step processed is t0 + nrows - 1; its carry is cut if b_{t0+nrows} = 1
-        const int64_t tn = t0 + nrows;
-        const bool first_cut = (tn < p.L) && (p.start[b * p.L + tn] != 0);
-        // adjoint entering the chain's first (right-most) step: grad_h_last (or 0)
-        const float4 base = (p.g_last != nullptr && lane_ok) ? p.g_last[b * p.D2 + c2 + lane] : zero2();
-        float4 carry = zero2();
-        const bool ok = fenwick_lookback(p, fbase, jr, Ta, Tx, Tb, !first_cut, base, carry,
-                                         t_begin, ticket, skip);
-        s_carry[lane] = carry;
-        if (lane == 0 && !ok) s_abort = 1;
+    // carry into this warp: the tile's carry through the warps before it (in processing order)
+    float4 c = s_carry[lane];
+    for (int k = 0; k < W; ++k) {
+        const int v = C::REV ? W - 1 - k : k;
+        if (v == warp) break;
+        const float4 wa = s_wa[v * 32 + lane], wx = s_wx[v * 32 + lane];
+        c = s_wr[v] ? wx : cfma2(wa, c, wx);
     }
-    __syncthreads();
-    if (s_abort) return;
 
-    // carry into this warp from the warps to its right
-    float4 Ea = one2(), Ex = zero2();
-    bool Eb = false;
-    for (int v = W - 1; v > warp; --v) {
-        const float4 wa = s_wa[v][lane], wx = s_wx[v][lane];
-        if (s_wr[v]) {
-            Ea = wa;
-            Ex = wx;
-            Eb = true;
-        } else {
-            Ex = cfma2(wa, Ex, wx);
-            Ea = cmul2(wa, Ea);
-        }
-    }
-    float4 delta = Eb ? Ex : cfma2(Ea, s_carry[lane], Ex);
-    float4 acc = zero2();
-    if (lane_ok) {
-        float4* dst = p.out + (b * p.L + ts) * p.D2 + c2 + lane;
-        for (int i = nv - 1; i >= 0; --i) {
-            const int64_t t = ts + i;
-            const float4 gg = s_g[(warp * R + i) * 32 + lane];
-            const float4 m = (t == p.L - 1) ? one2() : (PER_STEP ? conj2(s_l[(warp * R + i) * 32 + lane]) : mlam);
-            delta = ((rmask >> i) & 1u) ? gg : cfma2(m, delta, gg);
-            __stcs(dst + static_cast<int64_t>(i) * p.D2, delta);
-            float4 gl = zero2();
-            if (!((bmask >> i) & 1u)) {
-                float4 hp;
-                if (t > 0) hp = s_h[(warp * R + i) * 32 + lane];
-                else hp = (p.h0 != nullptr) ? p.h0[b * p.D2 + c2 + lane] : zero2();
-                gl = cmul2(delta, conj2(hp));
+    // phase 3: rescan from the carry and stream the outputs
+    if (!C::REV) {
+        if (lane_ok) {
+            float4* dst = p.out + (t.b * p.L + ts) * p.D2 + t.c2 + lane;
+            for (int k = 0; k < nv; ++k) {
+                const float4 uu = sin[k * 32];
+                const float4 ll = C::PS ? sl[k * 32] : lam;
+                c = ((rmask >> k) & 1u) ? uu : cfma2(ll, c, uu);
+                __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
             }
-            if (PER_STEP) {
-                if (p.grad_lambda != nullptr) __stcs(p.grad_lambda + (b * p.L + t) * p.D2 + c2 + lane, gl);
-            } else {
-                acc = add2(acc, gl);
-            }
-            if (t == 0 && p.grad_h0 != nullptr) {
-                float4 l0 = lam;
-                if (PER_STEP) l0 = p.lambda[(b * p.L) * p.D2 + c2 + lane];
-                p.grad_h0[b * p.D2 + c2 + lane] = (bmask & 1u) ? zero2() : cmul2(conj2(l0), delta);
+            if (p.out_last != nullptr && nv > 0 && ts + nv == p.L) p.out_last[t.b * p.D2 + t.c2 + lane] = c;
+        }
+        if (warp == 0) TRACE(6);
+    } else {
+        const float4* sh = s_h + warp * R * 32 + lane;
+        float4 acc = zero2();
+        if (lane_ok) {
+            float4* dst = p.out + (t.b * p.L + ts) * p.D2 + t.c2 + lane;
+            for (int k = nv - 1; k >= 0; --k) {
+                const int64_t tt = ts + k;
+                const float4 gg = sin[k * 32];
+                const float4 m = (tt == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
+                c = ((rmask >> k) & 1u) ? gg : cfma2(m, c, gg);
+                __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
+                float4 gl = zero2();
+                if (!((bmask >> k) & 1u)) {
+                    float4 hp;
+                    if (tt > 0) hp = sh[k * 32];
+                    else hp = (p.h0 != nullptr) ? p.h0[t.b * p.D2 + t.c2 + lane] : zero2();
+                    gl = cmul2(c, conj2(hp));
+                }
+                if (C::PS) {
+                    if (p.grad_lambda != nullptr) __stcs(p.grad_lambda + (t.b * p.L + tt) * p.D2 + t.c2 + lane, gl);
+                } else {
+                    acc = add2(acc, gl);
+                }
+                if (tt == 0 && p.grad_h0 != nullptr) {
+                    const float4 l0 = C::PS ? p.lambda[(t.b * p.L) * p.D2 + t.c2 + lane] : lam;
+                    p.grad_h0[t.b * p.D2 + t.c2 + lane] = (bmask & 1u) ? zero2() : cmul2(conj2(l0), c);
+                }
             }
         }
-    }
-    if (!PER_STEP) {
-        s_acc[warp][lane] = acc;
-        __syncthreads();
-        if (warp == 0) {
-            float4 s = zero2();
-            for (int v = 0; v < W; ++v) s = add2(s, s_acc[v][lane]);
-            p.gpart[(chain * p.n_tt + j) * 32 + lane] = s;
+        if (!C::PS) {
+            s_acc[warp * 32 + lane] = acc;
+            ptx::named_arrive(BAR_ACC, C::NSYNC);
         }
+        if (warp == 0) TRACE(6);
     }
+#ifdef MEMOROID_TRACE
+    if (warp == 0 && lane == 0 && g_trace != nullptr) {
+        unsigned smid;
+        asm volatile("mov.u32 %0, %%smid;" : "=r"(smid));
+        g_trace[tk * 16 + 7] = smid;
+    }
+#endif
 }
 
 // ============================================================================
@@ -569,9 +616,25 @@ __global__ void reduce_final_kernel(const double* __restrict__ rpart, float4* __
 // ============================================================================
 namespace {
 
+// Tile shapes (warps, steps per warp).  The defaults are the measured best on
+// GB300; the macros exist for tuning sweeps.
+#ifndef MEMOROID_FWD_W
+#define MEMOROID_FWD_W 2
+#define MEMOROID_FWD_R 24
+#endif
+#ifndef MEMOROID_BWD_W
+#define MEMOROID_BWD_W 3
+#define MEMOROID_BWD_R 16
+#endif
+using FwdC = Cfg<MEMOROID_FWD_W, MEMOROID_FWD_R, false, false>;
+using FwdS = Cfg<4, 8, false, true>;
+using BwdC = Cfg<MEMOROID_BWD_W, MEMOROID_BWD_R, true, false>;
+using BwdS = Cfg<4, 8, true, true>;
+static_assert(FwdC::T >= MIN_T && FwdS::T >= MIN_T && BwdC::T >= MIN_T && BwdS::T >= MIN_T, "tile");
+
 struct Layout {
     int64_t n_slabs, n_tt_max, n_chains;
-    size_t flags_off, node_off, gpart_off, rpart_off, total;
+    size_t node_off, gpart_off, rpart_off, total;
 };
 
 Layout layout(int64_t B, int64_t L, int64_t D) {
@@ -580,17 +643,11 @@ Layout layout(int64_t B, int64_t L, int64_t D) {
     l.n_tt_max = (L + MIN_T - 1) / MIN_T;
     l.n_chains = B * l.n_slabs;
     const size_t tiles = static_cast<size_t>(l.n_chains) * static_cast<size_t>(l.n_tt_max);
-    l.flags_off = kHeaderBytes;
-    l.node_off = align_up(l.flags_off + tiles * 4, 256);
-    l.gpart_off = align_up(l.node_off + tiles * 32 * 32, 256);
+    l.node_off = kHeaderBytes;
+    l.gpart_off = align_up(l.node_off + tiles * 32 * NODE_WORDS * 8, 256);
     l.rpart_off = align_up(l.gpart_off + tiles * 32 * 16, 256);
     l.total = align_up(l.rpart_off + static_cast<size_t>(l.n_slabs) * RED_PARTS * 32 * 32, 256);
     return l;
-}
-
-template <typename K>
-cudaError_t set_smem(K kernel, int bytes) {
-    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
 Params make_params(const Args& a, const Layout& l, int64_t n_tt) {
@@ -607,85 +664,69 @@ Params make_params(const Args& a, const Layout& l, int64_t n_tt) {
     p.grad_h0 = static_cast<float4*>(a.grad_h0);
     p.B = a.B;
     p.L = a.L;
-    p.D = a.D;
     p.D2 = a.D / 2;
     p.n_slabs = l.n_slabs;
     p.n_tt = n_tt;
     p.n_chains = l.n_chains;
+    p.n_tiles = n_tt * l.n_chains;
     unsigned char* ws = static_cast<unsigned char*>(a.workspace);
     p.hdr = reinterpret_cast<uint32_t*>(ws);
-    p.flags = reinterpret_cast<uint32_t*>(ws + l.flags_off);
-    p.node = reinterpret_cast<float4*>(ws + l.node_off);
+    p.node = reinterpret_cast<unsigned long long*>(ws + l.node_off);
     p.gpart = reinterpret_cast<float4*>(ws + l.gpart_off);
     const DebugKnobs k = debug_knobs();
     p.wait_ns = k.wait_ns;
     p.withhold = k.withhold_ticket;
+    p.epoch = next_epoch();
     return p;
 }
 
-cudaError_t clear_status(const Args& a, const Layout& l, int64_t n_tt, cudaStream_t s) {
-    const size_t bytes = l.flags_off + static_cast<size_t>(l.n_chains) * n_tt * 4;
-    return cudaMemsetAsync(a.workspace, 0, bytes, s);
+// One CTA per tile; tiles are claimed in ticket order by the CTAs as they start.
+template <class C>
+memoroid_status_t launch(const Args& a, const Layout& l, cudaStream_t s) {
+    const int64_t n_tt = (a.L + C::T - 1) / C::T;
+    const int64_t n_tiles = n_tt * l.n_chains;
+    if (n_tiles >= 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;
+    if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, s) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    auto kernel = diag_scan_kernel<C>;
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(C::SMEM)) != cudaSuccess)
+        return MEMOROID_ERR_CUDA;
+    const Params p = make_params(a, l, n_tt);
+    kernel<<<static_cast<unsigned>(n_tiles), C::THREADS, C::SMEM, s>>>(p);
+    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    return MEMOROID_OK;
 }
 
 }  // namespace
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t D) { return layout(B, L, D).total; }
 
+#ifdef MEMOROID_TRACE
+extern "C" int memoroid_trace_set_buffer(void* dev_ptr) {
+    unsigned long long* ptr = static_cast<unsigned long long*>(dev_ptr);
+    return static_cast<int>(cudaMemcpyToSymbol(g_trace, &ptr, sizeof(ptr)));
+}
+#endif
+
 memoroid_status_t launch_fwd(const Args& a, cudaStream_t s) {
     const Layout l = layout(a.B, a.L, a.D);
-    const bool ps = a.lambda_per_step != 0;
-    const int T = ps ? FWDS_W * FWDS_R : FWD_W * FWD_R;
-    const int64_t n_tt = (a.L + T - 1) / T;
-    const int64_t n_tiles = n_tt * l.n_chains;
-    if (n_tiles > 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;
-    if (clear_status(a, l, n_tt, s) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    const Params p = make_params(a, l, n_tt);
-    cudaError_t e;
-    if (ps) {
-        const int smem = 2 * T * 32 * 16;
-        auto k = diag_fwd_kernel<FWDS_W, FWDS_R, true>;
-        e = set_smem(k, smem);
-        if (e == cudaSuccess) k<<<static_cast<unsigned>(n_tiles), FWDS_W * 32, smem, s>>>(p);
-    } else {
-        const int smem = T * 32 * 16;
-        auto k = diag_fwd_kernel<FWD_W, FWD_R, false>;
-        e = set_smem(k, smem);
-        if (e == cudaSuccess) k<<<static_cast<unsigned>(n_tiles), FWD_W * 32, smem, s>>>(p);
-    }
-    if (e != cudaSuccess || cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
-    return MEMOROID_OK;
+    return a.lambda_per_step ? launch<FwdS>(a, l, s) : launch<FwdC>(a, l, s);
 }
 
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t s) {
     const Layout l = layout(a.B, a.L, a.D);
     const bool ps = a.lambda_per_step != 0;
-    const int T = ps ? BWDS_W * BWDS_R : BWD_W * BWD_R;
-    const int64_t n_tt = (a.L + T - 1) / T;
-    const int64_t n_tiles = n_tt * l.n_chains;
-    if (n_tiles > 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;
-    if (clear_status(a, l, n_tt, s) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    const Params p = make_params(a, l, n_tt);
-    cudaError_t e;
-    if (ps) {
-        const int smem = 3 * T * 32 * 16;
-        auto k = diag_bwd_kernel<BWDS_W, BWDS_R, true>;
-        e = set_smem(k, smem);
-        if (e == cudaSuccess) k<<<static_cast<unsigned>(n_tiles), BWDS_W * 32, smem, s>>>(p);
-    } else {
-        const int smem = 2 * T * 32 * 16;
-        auto k = diag_bwd_kernel<BWD_W, BWD_R, false>;
-        e = set_smem(k, smem);
-        if (e == cudaSuccess) k<<<static_cast<unsigned>(n_tiles), BWD_W * 32, smem, s>>>(p);
-    }
-    if (e != cudaSuccess || cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    const memoroid_status_t st = ps ? launch<BwdS>(a, l, s) : launch<BwdC>(a, l, s);
+    if (st != MEMOROID_OK) return st;
     if (!ps && a.grad_lambda != nullptr) {
+        const int64_t n_tt = (a.L + BwdC::T - 1) / BwdC::T;
         unsigned char* ws = static_cast<unsigned char*>(a.workspace);
+        const float4* gpart = reinterpret_cast<const float4*>(ws + l.gpart_off);
         double* rpart = reinterpret_cast<double*>(ws + l.rpart_off);
         reduce_parts_kernel<<<dim3(static_cast<unsigned>(l.n_slabs), RED_PARTS), 256, 0, s>>>(
-            p.gpart, rpart, a.B, l.n_slabs, n_tt);
+            gpart, rpart, a.B, l.n_slabs, n_tt);
         reduce_final_kernel<<<static_cast<unsigned>(l.n_slabs), 32, 0, s>>>(
-            rpart, static_cast<float4*>(a.grad_lambda), p.D2);
+            rpart, static_cast<float4*>(a.grad_lambda), a.D / 2);
         if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     }
     return MEMOROID_OK;

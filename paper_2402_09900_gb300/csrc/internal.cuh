@@ -12,8 +12,13 @@ namespace memoroid {
 // Device-side error codes written to the first word of a workspace header.
 enum DeviceError : uint32_t {
     DEV_OK = 0,
-    DEV_LOOKBACK_TIMEOUT = 1,  // a look-back wait on a predecessor ran out
-    DEV_TMA_TIMEOUT = 2,       // a TMA completion wait ran out
+    DEV_LOOKBACK_TIMEOUT = 1,  // a look-back wait on a predecessor's summary ran out
+    DEV_TMA_TIMEOUT = 2,       // a wait for staged data (TMA completion) ran out
+    DEV_STAGE_TIMEOUT = 3,     // the producer's wait for a free stage ran out
+    DEV_AGG_TIMEOUT = 4,       // the look-back warp's wait for warp aggregates ran out
+    DEV_CARRY_TIMEOUT = 5,     // a compute warp's wait for its carry ran out
+    DEV_ACC_TIMEOUT = 6,       // the wait for grad_lambda partials ran out
+    DEV_DRAIN_TIMEOUT = 7,     // the final wait for in-flight copies ran out
 };
 
 // Workspace header (256 bytes): [0] error code, [1] tile ticket counter,
@@ -26,6 +31,11 @@ struct DebugKnobs {
     int64_t withhold_ticket;
 };
 DebugKnobs debug_knobs();
+
+// A fresh 31-bit, non-zero tag per launch.  Look-back summaries carry it, so
+// that words left in a workspace by an earlier launch are never mistaken for
+// this launch's.
+uint32_t next_epoch();
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 

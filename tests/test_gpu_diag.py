@@ -37,11 +37,15 @@ def dev(a):
 def run_gpu(t, h0=None, g_last=None, want_h0=False):
     m = _m()
     lam, u, start = dev(t["lam"]), dev(t["u"]), dev(t["start"])
+    B, L, D = t["u"].shape
+    ws = m.diag_workspace(B, L, D, "cuda")
     h0d = dev(h0)
-    h, h_last = m.diag_fwd(lam, u, start, h0d)
+    h, h_last = m.diag_fwd(lam, u, start, h0d, ws=ws)
+    assert m.memoroid_get_device_error(ws) == m.MEMOROID_OK
     out = dict(h=h, h_last=h_last)
     if "grad_h" in t:
-        gu, gl, gh0 = m.diag_bwd(lam, start, h, dev(t["grad_h"]), dev(g_last), h0d, want_h0=want_h0)
+        gu, gl, gh0 = m.diag_bwd(lam, start, h, dev(t["grad_h"]), dev(g_last), h0d, want_h0=want_h0, ws=ws)
+        assert m.memoroid_get_device_error(ws) == m.MEMOROID_OK
         out.update(grad_u=gu, grad_lambda=gl, grad_h0=gh0)
     torch.cuda.synchronize()
     return {k: (None if v is None else v.cpu().numpy()) for k, v in out.items()}
