@@ -41,7 +41,7 @@ WORKLOAD = ("diag scan fwd+bwd (grad_u, grad_lambda): B=1 tape, L=2^20 steps, D=
 # algorithmic bytes per (step, channel): fwd reads u, writes h; bwd reads grad_h and h, writes grad_u
 FWD_BYTES_PER_STEP_CH = 16
 BWD_BYTES_PER_STEP_CH = 24
-PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "diag_bwd_traffic.txt")
+PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "diag_scan_traffic_L1M_D256.md")
 KERNEL_SRC = os.path.join(ROOT, "paper_2402_09900_gb300", "csrc", "diag_scan.cu")
 
 
@@ -69,7 +69,7 @@ def _traffic_record():
         rec = {}
         with open(PROFILE_TRAFFIC) as f:
             for line in f:
-                if ":" in line and not line.startswith("#"):
+                if ":" in line and not line.startswith(("#", "|", " ")):
                     k, v = line.split(":", 1)
                     rec[k.strip()] = v.strip()
         src = hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()
@@ -364,7 +364,9 @@ def run_ours(args):
                    "l2": "inputs larger than L2 (each tensor 2 GiB vs 129 MB L2); no flush needed",
                    "parallelism": f"independent tape per GPU x{ws}"},
         "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
-        "gpu_launches": 4 * args.steps, "clocks": clocks,
+        "gpu_launches": args.steps * (m.memoroid_scan_diag_kernels_per_call(B, L, D, 0, 0, 0)
+                                      + m.memoroid_scan_diag_kernels_per_call(B, L, D, 0, 1, 1)),
+        "clocks": clocks,
     }
     print(json.dumps(out), flush=True)
     if ws > 1:

@@ -66,6 +66,12 @@ int memoroid_version(void);
  * shape (one size serves both).  Returns 0 for an invalid shape. */
 size_t memoroid_scan_diag_workspace_bytes(int64_t B, int64_t L, int64_t D);
 
+/* Number of GPU kernels one memoroid_scan_diag_fwd (backward = 0) or
+ * memoroid_scan_diag_bwd (backward = 1) call launches for this shape, not
+ * counting the small workspace-header memset (-1 for an invalid shape). */
+int memoroid_scan_diag_kernels_per_call(int64_t B, int64_t L, int64_t D, int lambda_per_step,
+                                        int backward, int with_grad_lambda);
+
 /*
  * Forward diagonal scan.
  *   lambda          complex [D] (lambda_per_step = 0) or [B,L,D] (= 1)

@@ -74,6 +74,12 @@ size_t memoroid_scan_diag_workspace_bytes(int64_t B, int64_t L, int64_t D) {
     return diag::workspace_bytes(B, L, D);
 }
 
+int memoroid_scan_diag_kernels_per_call(int64_t B, int64_t L, int64_t D, int lambda_per_step,
+                                        int backward, int with_grad_lambda) {
+    if (B < 0 || L < 0 || D < 0 || (D % 2) != 0) return -1;
+    return diag::kernels_per_call(B, L, D, lambda_per_step != 0, backward != 0, with_grad_lambda != 0);
+}
+
 static memoroid_status_t check_ws(int64_t B, int64_t L, int64_t D, const void* ws, size_t bytes) {
     if (ws == nullptr || !aligned(ws, 256)) return MEMOROID_ERR_WORKSPACE;
     if (bytes < diag::workspace_bytes(B, L, D)) return MEMOROID_ERR_WORKSPACE;

@@ -44,6 +44,16 @@
 //     word carries this launch's tag.  Under a saturated memory system each
 //     dependent round trip costs microseconds, so this halves the look-back
 //     latency.
+//   * Each chain is cut into G segments that are scanned as independent
+//     chains from the identity, and tiles are handed out position-major over
+//     all segments: the tile before a given tile in its chain was handed out
+//     (chains x G) tickets earlier, long enough for its summary to be visible
+//     when it is needed.  A small second pass then adds the true state
+//     entering each segment to the steps of that segment before its first
+//     begin flag (only those depend on it): for the step-t output the
+//     correction is (product of the multipliers from the segment start to t)
+//     times that state.  With episodes much shorter than a segment this
+//     touches a few percent of the tape.
 //   * A begin flag inside a summary's range discards everything to its left,
 //     so folds stop at the first such summary; a tile whose first step is a
 //     begin flag needs no carry at all.
@@ -61,17 +71,27 @@ namespace memoroid {
 namespace diag {
 
 constexpr int SLAB = 64;  // complex channels per slab
-constexpr int NODE_WORDS = 8;  // 64-bit words per lane in a summary: a (4 floats), x (4 floats)
+// 64-bit words per lane in a summary: (a, x) = 8 floats with a per-step lambda;
+// x alone (4 floats) with a per-channel lambda, whose a is lambda^(steps in
+// the summary's range) and is recomputed by the reader.
+constexpr int NODE_WORDS = 8;
 #ifndef MEMOROID_NODE_BATCH
 #define MEMOROID_NODE_BATCH 2  // summaries read per round trip in a look-back fold
 #endif
 constexpr int NB_READ = MEMOROID_NODE_BATCH;
-constexpr int RED_PARTS = 64;  // first-stage parts of the grad_lambda reduction
+// Unroll factors of the per-step loops (measured: unrolling helps the
+// backward scan and slows the forward one).
+#ifndef MEMOROID_UNROLL_FWD
+#define MEMOROID_UNROLL_FWD 1
+#endif
+#ifndef MEMOROID_UNROLL_BWD
+#define MEMOROID_UNROLL_BWD 32
+#endif
+constexpr int RED_PARTS = 128;  // first-stage parts of the grad_lambda reduction
 #ifndef MEMOROID_POLL_SLEEP_NS
 #define MEMOROID_POLL_SLEEP_NS 0  // longest back-off between flag polls
 #endif
 
-constexpr int MIN_T = 16;      // smallest tile used (sizes the workspace)
 
 struct Params {
     const float4* lambda;  // [D/2] or [B, L, D/2]; one float4 = two complex channels
@@ -85,12 +105,21 @@ struct Params {
     float4* grad_lambda;   // bwd, per-step lambda: [B, L, D/2] or null
     float4* grad_h0;       // bwd: [B, D/2] or null
     int64_t B, L, D2, n_slabs, n_tt, n_chains, n_tiles;
+    int64_t n_seg, q_seg, n_sc;  // segments per chain, tiles per segment, segment chains
     uint32_t* hdr;               // workspace header: [0] error, [1] ticket counter
-    unsigned long long* node;    // [n_chains * n_tt * 32 * NODE_WORDS] tagged Fenwick nodes
+    unsigned long long* node;    // [n_sc * q_seg * 32 * NODE_WORDS] tagged Fenwick nodes
     float4* gpart;               // [n_chains * n_tt * 32]      per-tile grad_lambda
+    uint32_t* fix;               // [n_chains * n_tt] tile needs its segment's carry added (n_seg > 1)
+    float4* pin;                 // [n_chains * n_tt * 32] product of multipliers from the segment start
+    float4* segc;                // [n_chains * n_seg * 32] true state entering each segment
+    float4* sega;                // [n_chains * n_seg * 32 * 2] each segment's aggregate (a, x)
+    uint32_t* segb;              // [n_chains * n_seg] each segment holds a begin flag
     uint64_t wait_ns;
     int64_t withhold;
     uint32_t epoch;              // this launch's tag (31 bits, non-zero)
+    int full_nodes;              // summaries store a (per-step lambda) or only x
+    int T;                       // steps per tile
+    int rag;                     // steps missing from the chain's first tile in processing order
 };
 
 __host__ __device__ __forceinline__ int64_t lmin(int64_t a, int64_t b) { return a < b ? a : b; }
@@ -119,6 +148,7 @@ template <int W_, int R_, bool REV_, bool PS_>
 struct Cfg {
     static constexpr int W = W_, R = R_, T = W_ * R_;
     static constexpr bool REV = REV_, PS = PS_;
+    static constexpr int UNROLL = REV_ ? MEMOROID_UNROLL_BWD : MEMOROID_UNROLL_FWD;
     // arrays staged per tile: input [, h (backward)] [, lambda (per step)]
     static constexpr int NB = 1 + (REV_ ? 1 : 0) + (PS_ ? 1 : 0);
     static constexpr int BUF_F4 = T * 32;  // float4 per staged array
@@ -136,30 +166,45 @@ struct Cfg {
 };
 
 struct Tile {
-    int64_t tk;      // ticket (-1: no more work)
+    int64_t tk;      // ticket
     int64_t b, c2;   // tape, first float4 column of the slab
-    int64_t pos;     // position in the chain (left-to-right forward, right-to-left backward)
+    int64_t chain;   // tape * n_slabs + slab
+    int64_t g;       // segment of the chain
+    int64_t pos;     // position in the segment (left-to-right forward, right-to-left backward)
+    int64_t jt;      // time tile
     int64_t t0;      // first step
-    int64_t fbase;   // chain * n_tt
+    int64_t fbase;   // first node of the segment chain
     int width2;      // float4 columns in the slab
     int nrows;       // steps in the tile
+    bool valid;      // the ticket maps to a tile (the last segment may be shorter)
 };
 
+// Tickets are position-major over the segment chains: ticket = pos * n_sc + sc,
+// sc = g * n_chains + chain, so the slabs of the same steps are handed out
+// together (their rows share DRAM pages).
 template <class C>
 __device__ __forceinline__ Tile decode(const Params& p, int64_t tk) {
     Tile t{};
     t.tk = tk;
-    if (tk < 0) return t;
-    const int64_t q = tk / p.n_chains;
-    const int64_t chain = tk - q * p.n_chains;
+    const int64_t q = tk / p.n_sc;
+    const int64_t sc = tk - q * p.n_sc;
+#ifndef MEMOROID_CHAIN_MAJOR
+    t.g = sc / p.n_chains;
+    t.chain = sc - t.g * p.n_chains;
+#else
+    t.chain = sc / p.n_seg;
+    t.g = sc - t.chain * p.n_seg;
+#endif
     t.pos = q;
-    const int64_t j = C::REV ? p.n_tt - 1 - q : q;
-    t.b = chain / p.n_slabs;
-    t.c2 = (chain - t.b * p.n_slabs) * (SLAB / 2);
+    const int64_t jg = t.g * p.q_seg + q;  // position in the whole chain
+    t.valid = (q < p.q_seg) && (jg < p.n_tt);
+    t.jt = C::REV ? p.n_tt - 1 - jg : jg;
+    t.b = t.chain / p.n_slabs;
+    t.c2 = (t.chain - t.b * p.n_slabs) * (SLAB / 2);
     t.width2 = static_cast<int>(lmin(SLAB / 2, p.D2 - t.c2));
-    t.t0 = j * C::T;
+    t.t0 = t.jt * C::T;
     t.nrows = static_cast<int>(lmin(C::T, p.L - t.t0));
-    t.fbase = chain * p.n_tt;
+    t.fbase = sc * p.q_seg;
     return t;
 }
 
@@ -194,37 +239,61 @@ __device__ __forceinline__ void record_error(const Params& p, uint32_t code, int
     }
 }
 
-// Publishes this lane's part of a Fenwick node (tile index idx): a, x and
+// Publishes this lane's part of a Fenwick node (tile index idx): [a,] x and
 // the begin-flag bit, each value tagged with the launch's epoch.
 __device__ __forceinline__ void store_node(const Params& p, int64_t idx, float4 a, float4 x, bool b) {
     const int lane = threadIdx.x & 31;
     unsigned long long* dst = p.node + (idx * 32 + lane) * NODE_WORDS;
     const unsigned long long hi = static_cast<unsigned long long>((p.epoch << 1) | (b ? 1u : 0u)) << 32;
     auto w = [&](float v) { return hi | static_cast<unsigned long long>(__float_as_uint(v)); };
-    ptx::st_relaxed_v2u64(dst + 0, w(a.x), w(a.y));
-    ptx::st_relaxed_v2u64(dst + 2, w(a.z), w(a.w));
-    ptx::st_relaxed_v2u64(dst + 4, w(x.x), w(x.y));
-    ptx::st_relaxed_v2u64(dst + 6, w(x.z), w(x.w));
+    ptx::st_relaxed_v2u64(dst + 0, w(x.x), w(x.y));
+    ptx::st_relaxed_v2u64(dst + 2, w(x.z), w(x.w));
+    if (p.full_nodes) {
+        ptx::st_relaxed_v2u64(dst + 4, w(a.x), w(a.y));
+        ptx::st_relaxed_v2u64(dst + 6, w(a.z), w(a.w));
+    }
 }
 
-// Reads this lane's part of a Fenwick node.  Returns true if all of its
-// words carry this launch's tag (then b holds the node's begin-flag bit).
-__device__ __forceinline__ bool load_node(const Params& p, int64_t idx, float4& a, float4& x, bool& b) {
+// m^n for the two complex numbers of a float4, by repeated squaring.
+__device__ __forceinline__ float4 cpow2(float4 m, int64_t n) {
+    float4 r = one2();
+    while (n > 0) {
+        if (n & 1) r = cmul2(r, m);
+        m = cmul2(m, m);
+        n >>= 1;
+    }
+    return r;
+}
+
+// Reads this lane's part of Fenwick node `pos` (1-based) of a segment chain.
+// Returns true if all of its words carry this launch's tag (then b holds the
+// node's begin-flag bit).  Without stored a, a = mul^(steps in the node's
+// range); rag = steps missing from the segment chain's first tile.
+__device__ __forceinline__ bool load_node(const Params& p, int64_t fbase, int64_t pos, float4 mul,
+                                          int rag, float4& a, float4& x, bool& b) {
     const int lane = threadIdx.x & 31;
-    const unsigned long long* src = p.node + (idx * 32 + lane) * NODE_WORDS;
+    const unsigned long long* src = p.node + ((fbase + pos - 1) * 32 + lane) * NODE_WORDS;
     unsigned long long w[NODE_WORDS];
     ptx::ld_relaxed_v2u64(src + 0, w[0], w[1]);
     ptx::ld_relaxed_v2u64(src + 2, w[2], w[3]);
-    ptx::ld_relaxed_v2u64(src + 4, w[4], w[5]);
-    ptx::ld_relaxed_v2u64(src + 6, w[6], w[7]);
+    const int nw = p.full_nodes ? 8 : 4;
+    if (p.full_nodes) {
+        ptx::ld_relaxed_v2u64(src + 4, w[4], w[5]);
+        ptx::ld_relaxed_v2u64(src + 6, w[6], w[7]);
+    }
     bool ok = true;
 #pragma unroll
-    for (int i = 0; i < NODE_WORDS; ++i) ok = ok && static_cast<uint32_t>(w[i] >> 33) == p.epoch;
+    for (int i = 0; i < NODE_WORDS; ++i) ok = ok && (i >= nw || static_cast<uint32_t>(w[i] >> 33) == p.epoch);
     b = (w[0] >> 32) & 1u;
-    a = make_float4(__uint_as_float(static_cast<uint32_t>(w[0])), __uint_as_float(static_cast<uint32_t>(w[1])),
-                    __uint_as_float(static_cast<uint32_t>(w[2])), __uint_as_float(static_cast<uint32_t>(w[3])));
-    x = make_float4(__uint_as_float(static_cast<uint32_t>(w[4])), __uint_as_float(static_cast<uint32_t>(w[5])),
-                    __uint_as_float(static_cast<uint32_t>(w[6])), __uint_as_float(static_cast<uint32_t>(w[7])));
+    auto f = [&](int i) { return __uint_as_float(static_cast<uint32_t>(w[i])); };
+    x = make_float4(f(0), f(1), f(2), f(3));
+    if (p.full_nodes) {
+        a = make_float4(f(4), f(5), f(6), f(7));
+    } else {
+        const int64_t lb = pos & (-pos);
+        const int64_t steps = lb * p.T - ((pos == lb) ? rag : 0);
+        a = b ? one2() : cpow2(mul, steps);  // a of a range holding a begin flag is never used
+    }
     return ok;
 }
 
@@ -235,8 +304,8 @@ __device__ __forceinline__ bool load_node(const Params& p, int64_t idx, float4& 
 // node further left would be discarded by the select of Theorem 3.2, so
 // stopping changes no bit).  Nodes are read four at a time and re-read until
 // every lane sees them complete.  Warp-wide; false on timeout / error.
-__device__ bool fold_nodes(const Params& p, int64_t fbase, int64_t mypos, int n, float4& Ra,
-                           float4& Rx, bool& Rb, int64_t ticket, int trace_slot = -1) {
+__device__ bool fold_nodes(const Params& p, int64_t fbase, int64_t mypos, int n, float4 mul, int rag,
+                           float4& Ra, float4& Rx, bool& Rb, int64_t ticket, int trace_slot = -1) {
     for (int m0 = 0; m0 < n && !Rb; m0 += NB_READ) {
         int64_t pk[NB_READ];
 #pragma unroll
@@ -250,7 +319,7 @@ __device__ bool fold_nodes(const Params& p, int64_t fbase, int64_t mypos, int n,
 #pragma unroll
             for (int k = 0; k < NB_READ; ++k) {
                 if ((pending >> k) & 1u) {
-                    const bool ok = load_node(p, fbase + pk[k] - 1, a[k], x[k], rb[k]);
+                    const bool ok = load_node(p, fbase, pk[k], mul, rag, a[k], x[k], rb[k]);
                     if (__all_sync(0xffffffffu, ok)) pending &= ~(1u << k);
                 }
             }
@@ -283,8 +352,8 @@ __device__ bool fold_nodes(const Params& p, int64_t fbase, int64_t mypos, int n,
 // k = 1, 2, 4, .. < lowbit(pos); they cover the same range minus tile pos-1.
 // Returns the children folded right to left, C = child(pos - lowbit/2) o ...
 // o child(pos - 1) (the identity if there are none).
-__device__ bool fenwick_children(const Params& p, int64_t fbase, int64_t pos, float4& Ca, float4& Cx,
-                                 bool& Cb, int64_t ticket) {
+__device__ bool fenwick_children(const Params& p, int64_t fbase, int64_t pos, float4 mul, int rag,
+                                 float4& Ca, float4& Cx, bool& Cb, int64_t ticket) {
     const int lane = threadIdx.x & 31;
     const int64_t lb = pos & (-pos);
     const int nc = 63 - __clzll(static_cast<long long>(lb));  // log2(lowbit(pos))
@@ -293,7 +362,7 @@ __device__ bool fenwick_children(const Params& p, int64_t fbase, int64_t pos, fl
     Cb = false;
     if (nc == 0) return true;
     const int64_t child = pos - (int64_t(1) << (lane < nc ? lane : 0));
-    return fold_nodes(p, fbase, child, nc, Ca, Cx, Cb, ticket, 9);
+    return fold_nodes(p, fbase, child, nc, mul, rag, Ca, Cx, Cb, ticket, 9);
 }
 
 // Publishes node j+1 = C o T (T: the tile's own aggregate) unless !ok or the
@@ -306,18 +375,20 @@ __device__ void fenwick_publish(const Params& p, int64_t fbase, int64_t j, float
     store_node(p, fbase + j, Na, Nx, Tb || Cb);
 }
 
-// State entering chain position j > 0: the Fenwick prefix nodes of position j
-// (j, j - lowbit(j), ...) folded right to left, applied to `base` (the state
-// before the chain's first step) unless a begin flag intervenes.  Warp-wide.
-__device__ bool fenwick_carry(const Params& p, int64_t fbase, int64_t j, float4 base, float4& carry,
-                              int64_t ticket) {
+// State entering segment position j > 0: the Fenwick prefix nodes of
+// position j (j, j - lowbit(j), ...) folded right to left into (Ra, Rx, Rb)
+// and applied to `base` (the state before the segment's first step) unless a
+// begin flag intervenes.  Warp-wide.
+__device__ bool fenwick_carry(const Params& p, int64_t fbase, int64_t j, float4 mul, int rag, float4 base,
+                              float4& carry, float4& Ra, float4& Rx, bool& Rb, int64_t ticket) {
     const int lane = threadIdx.x & 31;
     int64_t q = j;  // lane i holds the i-th prefix node position
     for (int k = 0; k < lane && q > 0; ++k) q -= q & (-q);
     const int nq = __popcll(static_cast<unsigned long long>(j));
-    float4 Ra = one2(), Rx = zero2();
-    bool Rb = false;
-    if (!fold_nodes(p, fbase, q, nq, Ra, Rx, Rb, ticket, 8)) return false;
+    Rx = zero2();
+    Ra = one2();
+    Rb = false;
+    if (!fold_nodes(p, fbase, q, nq, mul, rag, Ra, Rx, Rb, ticket, 8)) return false;
     carry = Rb ? Rx : cfma2(Ra, base, Rx);
     return true;
 }
@@ -355,7 +426,12 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
     __syncthreads();
     const int64_t tk = *s_tk;
     const Tile t = decode<C>(p, tk);
+    if (!t.valid) return;  // uniform over the CTA: the ticket has no tile
     const bool lane_ok = lane < t.width2;
+    // multiplier whose powers rebuild the a of summaries stored without it
+    float4 node_mul = one2();
+    if (!C::PS && lane_ok) node_mul = C::REV ? conj2(p.lambda[t.c2 + lane]) : p.lambda[t.c2 + lane];
+    const int node_rag = (t.g == 0) ? p.rag : 0;
     if (warp == 0) TRACE(0);
 
     if (warp == LB_PUBLISH) {
@@ -373,7 +449,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
         }
         float4 Ca, Cx;
         bool Cb;
-        bool ok = fenwick_children(p, t.fbase, t.pos + 1, Ca, Cx, Cb, tk);
+        bool ok = fenwick_children(p, t.fbase, t.pos + 1, node_mul, node_rag, Ca, Cx, Cb, tk);
         TRACE(1);
         ptx::named_sync(BAR_AGG, C::NSYNC);
         TRACE(2);
@@ -411,20 +487,50 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
             need_carry = !(tn < p.L && p.start[t.b * p.L + tn] != 0);
             if (p.g_last != nullptr && lane_ok) base = p.g_last[t.b * p.D2 + t.c2 + lane];
         }
-        float4 carry = base;
-        bool ok = true;
-        if (need_carry && t.pos > 0) ok = fenwick_carry(p, t.fbase, t.pos, base, carry, tk);
+        if (t.g > 0) base = zero2();  // later segments start from the identity; fixed up afterwards
+        float4 carry = base, Ra = one2(), Rx = zero2();
+        bool Rb = false, ok = true;
+        if (need_carry && t.pos > 0)
+            ok = fenwick_carry(p, t.fbase, t.pos, node_mul, node_rag, base, carry, Ra, Rx, Rb, tk);
         TRACE(4);
+        if (p.fix != nullptr) {
+            // steps of this tile before its first begin flag miss the state entering the segment
+            const int64_t tid = t.chain * p.n_tt + t.jt;
+            const bool partial = (t.g > 0) && need_carry && !Rb;
+            if (partial) p.pin[tid * 32 + lane] = Ra;
+            if (lane == 0) p.fix[tid] = partial ? 1u : 0u;
+        }
         s_carry[lane] = carry;
         if (!ok && lane == 0) *s_abort = 1;
         ptx::named_sync(BAR_CARRY, C::NSYNC);
+        if (p.fix != nullptr && *s_abort == 0 && t.pos == lmin(p.q_seg, p.n_tt - t.g * p.q_seg) - 1) {
+            // last tile of its segment: the segment's aggregate, T o R, for the carry pass
+            // (the scan warps' aggregates are visible here: they were written before BAR_CARRY)
+            float4 Ta = one2(), Tx = zero2();
+            bool Tb = false;
+            for (int k = 0; k < W; ++k) {
+                const int v = C::REV ? W - 1 - k : k;
+                const float4 wa = s_wa[v * 32 + lane], wx = s_wx[v * 32 + lane];
+                if (s_wr[v]) {
+                    Ta = wa;
+                    Tx = wx;
+                    Tb = true;
+                } else {
+                    Tx = cfma2(wa, Tx, wx);
+                    Ta = cmul2(wa, Ta);
+                }
+            }
+            const int64_t si = t.chain * p.n_seg + t.g;
+            p.sega[si * 64 + lane] = Tb ? Ta : cmul2(Ta, Ra);
+            p.sega[si * 64 + 32 + lane] = Tb ? Tx : cfma2(Ta, Rx, Tx);
+            if (lane == 0) p.segb[si] = (Tb || Rb) ? 1u : 0u;
+        }
         if (C::REV && !C::PS && *s_abort == 0) {
             // grad_lambda partial of this tile, summed over warps in a fixed order
             ptx::named_sync(BAR_ACC, C::NSYNC);
             float4 sum = zero2();
             for (int v = 0; v < W; ++v) sum = add2(sum, s_acc[v * 32 + lane]);
-            const int64_t jt = p.n_tt - 1 - t.pos;
-            p.gpart[(t.fbase + jt) * 32 + lane] = sum;
+            p.gpart[(t.chain * p.n_tt + t.jt) * 32 + lane] = sum;
         }
         return;
     }
@@ -466,27 +572,34 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
     float4 a = one2(), x = zero2();
     if (landed) {
         if (!C::REV) {
-            for (int k = 0; k < nv; ++k) {
-                const float4 uu = sin[k * 32];
-                const float4 ll = C::PS ? sl[k * 32] : lam;
-                if ((rmask >> k) & 1u) {
-                    a = ll;
-                    x = uu;
-                } else {
-                    x = cfma2(ll, x, uu);
-                    a = cmul2(ll, a);
+#pragma unroll C::UNROLL
+            for (int k = 0; k < R; ++k) {
+                if (k < nv) {
+                    const float4 uu = sin[k * 32];
+                    const float4 ll = C::PS ? sl[k * 32] : lam;
+                    if ((rmask >> k) & 1u) {
+                        a = ll;
+                        x = uu;
+                    } else {
+                        x = cfma2(ll, x, uu);
+                        a = cmul2(ll, a);
+                    }
                 }
             }
         } else {
-            for (int k = nv - 1; k >= 0; --k) {
-                const float4 gg = sin[k * 32];
-                const float4 m = (ts + k == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
-                if ((rmask >> k) & 1u) {
-                    a = m;
-                    x = gg;
-                } else {
-                    x = cfma2(m, x, gg);
-                    a = cmul2(m, a);
+#pragma unroll C::UNROLL
+            for (int kk = 0; kk < R; ++kk) {
+                const int k = R - 1 - kk;
+                if (k < nv) {
+                    const float4 gg = sin[k * 32];
+                    const float4 m = (ts + k == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
+                    if ((rmask >> k) & 1u) {
+                        a = m;
+                        x = gg;
+                    } else {
+                        x = cfma2(m, x, gg);
+                        a = cmul2(m, a);
+                    }
                 }
             }
         }
@@ -512,11 +625,14 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
     if (!C::REV) {
         if (lane_ok) {
             float4* dst = p.out + (t.b * p.L + ts) * p.D2 + t.c2 + lane;
-            for (int k = 0; k < nv; ++k) {
-                const float4 uu = sin[k * 32];
-                const float4 ll = C::PS ? sl[k * 32] : lam;
-                c = ((rmask >> k) & 1u) ? uu : cfma2(ll, c, uu);
-                __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
+#pragma unroll C::UNROLL
+            for (int k = 0; k < R; ++k) {
+                if (k < nv) {
+                    const float4 uu = sin[k * 32];
+                    const float4 ll = C::PS ? sl[k * 32] : lam;
+                    c = ((rmask >> k) & 1u) ? uu : cfma2(ll, c, uu);
+                    __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
+                }
             }
             if (p.out_last != nullptr && nv > 0 && ts + nv == p.L) p.out_last[t.b * p.D2 + t.c2 + lane] = c;
         }
@@ -526,7 +642,10 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
         float4 acc = zero2();
         if (lane_ok) {
             float4* dst = p.out + (t.b * p.L + ts) * p.D2 + t.c2 + lane;
-            for (int k = nv - 1; k >= 0; --k) {
+#pragma unroll C::UNROLL
+            for (int kk = 0; kk < R; ++kk) {
+                const int k = R - 1 - kk;
+                if (k >= nv) continue;
                 const int64_t tt = ts + k;
                 const float4 gg = sin[k * 32];
                 const float4 m = (tt == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
@@ -566,6 +685,138 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
 }
 
 // ============================================================================
+// segment fix-up
+// ============================================================================
+// State entering each segment (one warp per chain): the segments' aggregates,
+// published by their last tiles, folded left to right from the chain's
+// initial state.
+__global__ void __launch_bounds__(256) segment_carry_kernel(const Params p, bool rev) {
+    const int lane = threadIdx.x & 31;
+    const int64_t chain = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+    if (chain >= p.n_chains || ptx::ld_relaxed(p.hdr) != 0u) return;
+    const int64_t G = p.n_seg;
+    const int64_t b = chain / p.n_slabs;
+    const int64_t c2 = (chain - b * p.n_slabs) * (SLAB / 2);
+    const bool lane_ok = lane < lmin(SLAB / 2, p.D2 - c2);
+    const float4* base_src = rev ? p.g_last : p.h0;
+    float4 c = (base_src != nullptr && lane_ok) ? base_src[b * p.D2 + c2 + lane] : zero2();
+    for (int64_t g0 = 0; g0 < G; g0 += 8) {
+        float4 a[8], x[8];
+        uint32_t bb[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int64_t si = chain * G + g0 + k;
+            if (g0 + k < G) {
+                a[k] = p.sega[si * 64 + lane];
+                x[k] = p.sega[si * 64 + 32 + lane];
+                bb[k] = p.segb[si];
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            if (g0 + k < G) {
+                p.segc[(chain * G + g0 + k) * 32 + lane] = c;
+                c = bb[k] ? x[k] : cfma2(a[k], c, x[k]);
+            }
+        }
+    }
+}
+
+// Adds the state entering its segment to the outputs of a tile that the
+// scan computed from the identity, up to the tile's first begin flag (one warp
+// per tile; tiles that need nothing return at once).  The rows to fix are
+// counted first, so their loads can be issued in batches.
+template <class C>
+__global__ void __launch_bounds__(128) segment_fix_kernel(const Params p) {
+    constexpr int BATCH = 8;
+    const int lane = threadIdx.x & 31;
+    const int64_t tid = static_cast<int64_t>(blockIdx.x) * 4 + (threadIdx.x >> 5);
+    if (tid >= static_cast<int64_t>(p.n_chains) * p.n_tt) return;
+    if (p.fix[tid] == 0u || ptx::ld_relaxed(p.hdr) != 0u) return;
+    const int64_t chain = tid / p.n_tt, jt = tid - chain * p.n_tt;
+    const int64_t b = chain / p.n_slabs;
+    const int64_t c2 = (chain - b * p.n_slabs) * (SLAB / 2);
+    const int64_t jg = C::REV ? p.n_tt - 1 - jt : jt;
+    const int64_t g = jg / p.q_seg;
+    const int64_t t0 = jt * C::T;
+    const int nrows = static_cast<int>(lmin(C::T, p.L - t0));
+    // steps to fix, in processing order, before the first begin flag that cuts the carry
+    int nfix = nrows;
+    for (int r0 = 0; r0 < nrows; r0 += 32) {
+        const int r = r0 + lane;
+        bool cut = false;
+        if (r < nrows) {
+            if (!C::REV) {
+                cut = p.start[b * p.L + t0 + r] != 0;
+            } else {
+                const int64_t t = t0 + nrows - 1 - r;  // r-th step processed
+                cut = (t + 1 < p.L) && p.start[b * p.L + t + 1] != 0;
+            }
+        }
+        const uint32_t m = __ballot_sync(0xffffffffu, cut);
+        if (m != 0u) {
+            nfix = r0 + __ffs(m) - 1;
+            break;
+        }
+    }
+    if (lane >= lmin(SLAB / 2, p.D2 - c2)) return;
+    const int64_t col = c2 + lane;
+    float4 corr = cmul2(p.pin[tid * 32 + lane], p.segc[(chain * p.n_seg + g) * 32 + lane]);
+    const float4 lam = C::PS ? one2() : p.lambda[col];
+    float4 gl = zero2();
+    for (int k0 = 0; k0 < nfix; k0 += BATCH) {
+        float4 v[BATCH], aux[BATCH];
+#pragma unroll
+        for (int k = 0; k < BATCH; ++k) {
+            if (k0 + k < nfix) {
+                const int64_t t = C::REV ? t0 + nrows - 1 - (k0 + k) : t0 + k0 + k;
+                v[k] = p.out[(b * p.L + t) * p.D2 + col];
+                if (C::REV) {
+                    aux[k] = (t > 0) ? p.h[(b * p.L + t - 1) * p.D2 + col]
+                                     : ((p.h0 != nullptr) ? p.h0[b * p.D2 + col] : zero2());
+                }
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < BATCH; ++k) {
+            if (k0 + k >= nfix) break;
+            const int64_t t = C::REV ? t0 + nrows - 1 - (k0 + k) : t0 + k0 + k;
+            if (!C::REV) {
+                const float4 l = C::PS ? p.lambda[(b * p.L + t) * p.D2 + col] : lam;
+                corr = cmul2(l, corr);
+            } else {
+                const float4 m = (t == p.L - 1) ? one2()
+                                                : conj2(C::PS ? p.lambda[(b * p.L + t + 1) * p.D2 + col] : lam);
+                corr = cmul2(m, corr);
+            }
+            p.out[(b * p.L + t) * p.D2 + col] = add2(v[k], corr);
+            if (!C::REV) {
+                if (t == p.L - 1 && p.out_last != nullptr) {
+                    float4* ol = p.out_last + b * p.D2 + col;
+                    *ol = add2(*ol, corr);
+                }
+            } else if (p.start[b * p.L + t] == 0) {
+                const float4 d = cmul2(corr, conj2(aux[k]));
+                if (C::PS) {
+                    if (p.grad_lambda != nullptr) {
+                        float4* gp = p.grad_lambda + (b * p.L + t) * p.D2 + col;
+                        *gp = add2(*gp, d);
+                    }
+                } else {
+                    gl = add2(gl, d);
+                }
+                if (t == 0 && p.grad_h0 != nullptr) {
+                    const float4 l0 = C::PS ? p.lambda[(b * p.L) * p.D2 + col] : lam;
+                    float4* g0 = p.grad_h0 + b * p.D2 + col;
+                    *g0 = add2(*g0, cmul2(conj2(l0), corr));
+                }
+            }
+        }
+    }
+    if (C::REV && !C::PS) p.gpart[tid * 32 + lane] = add2(p.gpart[tid * 32 + lane], gl);
+}
+
+// ============================================================================
 // grad_lambda reduction (per-channel lambda): fixed-order fp64 sums
 // ============================================================================
 __global__ void __launch_bounds__(256) reduce_parts_kernel(const float4* __restrict__ gpart,
@@ -578,9 +829,15 @@ __global__ void __launch_bounds__(256) reduce_parts_kernel(const float4* __restr
     const int64_t per = (total + RED_PARTS - 1) / RED_PARTS;
     const int64_t k0 = part * per, k1 = lmin(total, k0 + per);
     double acc[4] = {0.0, 0.0, 0.0, 0.0};
+    int64_t bb = (k0 + grp) / n_tt, jj = (k0 + grp) - bb * n_tt;
+#pragma unroll 8
     for (int64_t k = k0 + grp; k < k1; k += 8) {
-        const int64_t bb = k / n_tt, jj = k - bb * n_tt;
         const float4 v = gpart[((bb * n_slabs + slab) * n_tt + jj) * 32 + lane];
+        jj += 8;
+        while (jj >= n_tt) {
+            jj -= n_tt;
+            ++bb;
+        }
         acc[0] += v.x;
         acc[1] += v.y;
         acc[2] += v.z;
@@ -601,9 +858,15 @@ __global__ void reduce_final_kernel(const double* __restrict__ rpart, float4* __
                                     int64_t D2) {
     const int slab = blockIdx.x, lane = threadIdx.x;
     double r[4] = {0.0, 0.0, 0.0, 0.0};
+#pragma unroll 16
     for (int part = 0; part < RED_PARTS; ++part) {
-        const double* o = rpart + ((static_cast<int64_t>(slab) * RED_PARTS + part) * 32 + lane) * 4;
-        for (int c = 0; c < 4; ++c) r[c] += o[c];
+        const double2* o = reinterpret_cast<const double2*>(
+            rpart + ((static_cast<int64_t>(slab) * RED_PARTS + part) * 32 + lane) * 4);
+        const double2 v0 = o[0], v1 = o[1];
+        r[0] += v0.x;
+        r[1] += v0.y;
+        r[2] += v1.x;
+        r[3] += v1.y;
     }
     const int64_t col = static_cast<int64_t>(slab) * 32 + lane;
     if (col < D2)
@@ -619,38 +882,68 @@ namespace {
 // Tile shapes (warps, steps per warp).  The defaults are the measured best on
 // GB300; the macros exist for tuning sweeps.
 #ifndef MEMOROID_FWD_W
-#define MEMOROID_FWD_W 2
+#define MEMOROID_FWD_W 4
 #define MEMOROID_FWD_R 24
 #endif
 #ifndef MEMOROID_BWD_W
-#define MEMOROID_BWD_W 3
-#define MEMOROID_BWD_R 16
+#define MEMOROID_BWD_W 4
+#define MEMOROID_BWD_R 12
 #endif
 using FwdC = Cfg<MEMOROID_FWD_W, MEMOROID_FWD_R, false, false>;
 using FwdS = Cfg<4, 8, false, true>;
 using BwdC = Cfg<MEMOROID_BWD_W, MEMOROID_BWD_R, true, false>;
 using BwdS = Cfg<4, 8, true, true>;
-static_assert(FwdC::T >= MIN_T && FwdS::T >= MIN_T && BwdC::T >= MIN_T && BwdS::T >= MIN_T, "tile");
+
+// Segments per chain: enough segment chains that a tile's predecessor was
+// handed out long before it (target), at least MIN_SEG_TILES tiles each.
+#ifndef MEMOROID_TARGET_SC
+#define MEMOROID_TARGET_SC 512
+#endif
+constexpr int64_t MAX_SEG = 192;
+constexpr int64_t MIN_SEG_TILES = 8;
+
+struct Segs {
+    int64_t G, Q;
+};
+Segs choose_segments(int64_t n_chains, int64_t n_tt) {
+    int64_t G = (MEMOROID_TARGET_SC + n_chains - 1) / n_chains;
+    G = lmin(G, lmin(MAX_SEG, n_tt / MIN_SEG_TILES));
+    if (G < 1) G = 1;
+    const int64_t Q = (n_tt + G - 1) / G;
+    return Segs{(n_tt + Q - 1) / Q, Q};
+}
 
 struct Layout {
-    int64_t n_slabs, n_tt_max, n_chains;
-    size_t node_off, gpart_off, rpart_off, total;
+    int64_t n_slabs, n_chains, n_tt;
+    Segs sg;
+    size_t node_off, gpart_off, fix_off, pin_off, segc_off, sega_off, segb_off, rpart_off, total;
 };
 
-Layout layout(int64_t B, int64_t L, int64_t D) {
+// Workspace layout for tiles of T steps.
+Layout layout(int64_t B, int64_t L, int64_t D, int T) {
     Layout l{};
     l.n_slabs = (D + SLAB - 1) / SLAB;
-    l.n_tt_max = (L + MIN_T - 1) / MIN_T;
     l.n_chains = B * l.n_slabs;
-    const size_t tiles = static_cast<size_t>(l.n_chains) * static_cast<size_t>(l.n_tt_max);
+    l.n_tt = (L + T - 1) / T;
+    l.sg = choose_segments(l.n_chains, l.n_tt);
+    const size_t tiles = static_cast<size_t>(l.n_chains) * static_cast<size_t>(l.n_tt);
+    const size_t nodes = static_cast<size_t>(l.n_chains) * static_cast<size_t>(l.sg.G * l.sg.Q);
     l.node_off = kHeaderBytes;
-    l.gpart_off = align_up(l.node_off + tiles * 32 * NODE_WORDS * 8, 256);
-    l.rpart_off = align_up(l.gpart_off + tiles * 32 * 16, 256);
+    l.gpart_off = align_up(l.node_off + nodes * 32 * NODE_WORDS * 8, 256);
+    l.fix_off = align_up(l.gpart_off + tiles * 32 * 16, 256);
+    l.pin_off = align_up(l.fix_off + tiles * 4, 256);
+    l.segc_off = align_up(l.pin_off + tiles * 32 * 16, 256);
+    const size_t nseg = static_cast<size_t>(l.n_chains * l.sg.G);
+    l.sega_off = align_up(l.segc_off + nseg * 32 * 16, 256);
+    l.segb_off = align_up(l.sega_off + nseg * 64 * 16, 256);
+    l.rpart_off = align_up(l.segb_off + nseg * 4, 256);
     l.total = align_up(l.rpart_off + static_cast<size_t>(l.n_slabs) * RED_PARTS * 32 * 32, 256);
     return l;
 }
 
-Params make_params(const Args& a, const Layout& l, int64_t n_tt) {
+Params make_params(const Args& a, const Layout& l, int T, bool backward) {
+    const int64_t n_tt = l.n_tt;
+    const Segs sg = l.sg;
     Params p{};
     p.lambda = static_cast<const float4*>(a.lambda);
     p.in = static_cast<const float4*>(a.u);
@@ -669,37 +962,67 @@ Params make_params(const Args& a, const Layout& l, int64_t n_tt) {
     p.n_tt = n_tt;
     p.n_chains = l.n_chains;
     p.n_tiles = n_tt * l.n_chains;
+    p.n_seg = sg.G;
+    p.q_seg = sg.Q;
+    p.n_sc = l.n_chains * sg.G;
     unsigned char* ws = static_cast<unsigned char*>(a.workspace);
     p.hdr = reinterpret_cast<uint32_t*>(ws);
     p.node = reinterpret_cast<unsigned long long*>(ws + l.node_off);
     p.gpart = reinterpret_cast<float4*>(ws + l.gpart_off);
+    p.fix = sg.G > 1 ? reinterpret_cast<uint32_t*>(ws + l.fix_off) : nullptr;
+    p.pin = reinterpret_cast<float4*>(ws + l.pin_off);
+    p.segc = reinterpret_cast<float4*>(ws + l.segc_off);
+    p.sega = reinterpret_cast<float4*>(ws + l.sega_off);
+    p.segb = reinterpret_cast<uint32_t*>(ws + l.segb_off);
     const DebugKnobs k = debug_knobs();
     p.wait_ns = k.wait_ns;
     p.withhold = k.withhold_ticket;
     p.epoch = next_epoch();
+    p.full_nodes = a.lambda_per_step ? 1 : 0;
+    p.T = T;
+    // backward: the chain's first tile (processing order) is the ragged last
+    // time tile, and its step L-1 has multiplier 1 rather than conj(lambda)
+    p.rag = backward ? static_cast<int>(n_tt * T - a.L) + 1 : 0;
     return p;
 }
 
-// One CTA per tile; tiles are claimed in ticket order by the CTAs as they start.
+// One CTA per ticket; tickets are claimed in order by the CTAs as they
+// start.  With more than one segment per chain, two small kernels then add the
+// state entering each segment where it is missing.
 template <class C>
-memoroid_status_t launch(const Args& a, const Layout& l, cudaStream_t s) {
-    const int64_t n_tt = (a.L + C::T - 1) / C::T;
-    const int64_t n_tiles = n_tt * l.n_chains;
-    if (n_tiles >= 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;
+memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
+    const Layout l = layout(a.B, a.L, a.D, C::T);
+    const Segs sg = l.sg;
+    const int64_t n_tickets = sg.Q * l.n_chains * sg.G;
+    if (n_tickets >= 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;
     if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, s) != cudaSuccess) return MEMOROID_ERR_CUDA;
     auto kernel = diag_scan_kernel<C>;
     if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(C::SMEM)) != cudaSuccess)
         return MEMOROID_ERR_CUDA;
-    const Params p = make_params(a, l, n_tt);
-    kernel<<<static_cast<unsigned>(n_tiles), C::THREADS, C::SMEM, s>>>(p);
+    const Params p = make_params(a, l, C::T, C::REV);
+    kernel<<<static_cast<unsigned>(n_tickets), C::THREADS, C::SMEM, s>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    if (sg.G > 1) {
+        segment_carry_kernel<<<static_cast<unsigned>((l.n_chains + 7) / 8), 256, 0, s>>>(p, C::REV);
+        const int64_t n_tiles = l.n_chains * l.n_tt;
+        segment_fix_kernel<C><<<static_cast<unsigned>((n_tiles + 3) / 4), 128, 0, s>>>(p);
+        if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    }
+    if (out_layout) *out_layout = l;
     return MEMOROID_OK;
 }
 
 }  // namespace
 
-size_t workspace_bytes(int64_t B, int64_t L, int64_t D) { return layout(B, L, D).total; }
+size_t workspace_bytes(int64_t B, int64_t L, int64_t D) {
+    size_t m = 0;
+    for (int T : {FwdC::T, FwdS::T, BwdC::T, BwdS::T}) {
+        const size_t t = layout(B, L, D, T).total;
+        if (t > m) m = t;
+    }
+    return m;
+}
 
 #ifdef MEMOROID_TRACE
 extern "C" int memoroid_trace_set_buffer(void* dev_ptr) {
@@ -708,23 +1031,30 @@ extern "C" int memoroid_trace_set_buffer(void* dev_ptr) {
 }
 #endif
 
+int kernels_per_call(int64_t B, int64_t L, int64_t D, int per_step, int backward, int with_grad_lambda) {
+    if (B <= 0 || L <= 0 || D <= 0) return 0;
+    const int T = backward ? (per_step ? BwdS::T : BwdC::T) : (per_step ? FwdS::T : FwdC::T);
+    const Layout l = layout(B, L, D, T);
+    int n = l.sg.G > 1 ? 3 : 1;  // scan [+ segment carries + fix-up]
+    if (backward && !per_step && with_grad_lambda) n += 2;  // grad_lambda reduction
+    return n;
+}
+
 memoroid_status_t launch_fwd(const Args& a, cudaStream_t s) {
-    const Layout l = layout(a.B, a.L, a.D);
-    return a.lambda_per_step ? launch<FwdS>(a, l, s) : launch<FwdC>(a, l, s);
+    return a.lambda_per_step ? launch<FwdS>(a, s, nullptr) : launch<FwdC>(a, s, nullptr);
 }
 
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t s) {
-    const Layout l = layout(a.B, a.L, a.D);
     const bool ps = a.lambda_per_step != 0;
-    const memoroid_status_t st = ps ? launch<BwdS>(a, l, s) : launch<BwdC>(a, l, s);
+    Layout l{};
+    const memoroid_status_t st = ps ? launch<BwdS>(a, s, &l) : launch<BwdC>(a, s, &l);
     if (st != MEMOROID_OK) return st;
     if (!ps && a.grad_lambda != nullptr) {
-        const int64_t n_tt = (a.L + BwdC::T - 1) / BwdC::T;
         unsigned char* ws = static_cast<unsigned char*>(a.workspace);
         const float4* gpart = reinterpret_cast<const float4*>(ws + l.gpart_off);
         double* rpart = reinterpret_cast<double*>(ws + l.rpart_off);
         reduce_parts_kernel<<<dim3(static_cast<unsigned>(l.n_slabs), RED_PARTS), 256, 0, s>>>(
-            gpart, rpart, a.B, l.n_slabs, n_tt);
+            gpart, rpart, a.B, l.n_slabs, l.n_tt);
         reduce_final_kernel<<<static_cast<unsigned>(l.n_slabs), 32, 0, s>>>(
             rpart, static_cast<float4*>(a.grad_lambda), a.D / 2);
         if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;

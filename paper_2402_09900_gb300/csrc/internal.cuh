@@ -59,6 +59,7 @@ struct Args {
 };
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t D);
+int kernels_per_call(int64_t B, int64_t L, int64_t D, int per_step, int backward, int with_grad_lambda);
 memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream);
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream);
 

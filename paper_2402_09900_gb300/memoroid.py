@@ -41,6 +41,7 @@ SIGNATURES = {
     "memoroid_status_string": (ctypes.c_char_p, [_int]),
     "memoroid_version": (_int, []),
     "memoroid_scan_diag_workspace_bytes": (_sz, [_i64, _i64, _i64]),
+    "memoroid_scan_diag_kernels_per_call": (_int, [_i64, _i64, _i64, _int, _int, _int]),
     "memoroid_scan_diag_fwd": (_int, [_p, _int, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_scan_diag_bwd": (_int, [_p, _int, _p, _p, _p, _p, _p, _p, _p, _p, _i64, _i64, _i64,
                                       _p, _sz, _p]),
@@ -117,6 +118,11 @@ def _need_cuda(*ts):
 
 def memoroid_scan_diag_workspace_bytes(B, L, D) -> int:
     return int(load().memoroid_scan_diag_workspace_bytes(B, L, D))
+
+
+def memoroid_scan_diag_kernels_per_call(B, L, D, lambda_per_step, backward, with_grad_lambda) -> int:
+    return int(load().memoroid_scan_diag_kernels_per_call(B, L, D, int(lambda_per_step), int(backward),
+                                                          int(with_grad_lambda)))
 
 
 def memoroid_scan_diag_fwd(lam, lambda_per_step, u, start, h0, h, h_last, B, L, D, workspace,
