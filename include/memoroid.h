@@ -115,6 +115,34 @@ memoroid_status_t memoroid_scan_diag_bwd(const void *lambda, int lambda_per_step
                                          int64_t D, void *workspace, size_t workspace_bytes,
                                          void *stream);
 
+/* ------------------------------------------------------------------------ */
+/* Forward scan without a workspace argument (the paper has no counterpart:  */
+/* this is a deployment convenience).                                        */
+/* ------------------------------------------------------------------------ */
+
+/* Size of the library-owned scratch array used by memoroid_scan_diag_fwd_static. */
+#define MEMOROID_STATIC_WORKSPACE_BYTES (16u << 20)
+
+/*
+ * Same inputs, outputs and result as memoroid_scan_diag_fwd, for callers that
+ * cannot provide device scratch memory (code running where device allocation
+ * is unavailable or not allowed, e.g. inside an allocator callback or under a
+ * framework that owns the whole device memory budget).  The scratch space is a
+ * MEMOROID_STATIC_WORKSPACE_BYTES array in the library's own device memory,
+ * held on every device that loads the library until the process exits; this
+ * call allocates nothing.
+ *   - The first call on a device looks up the array's address with that
+ *     device current; make it outside any stream capture.
+ *   - All calls share the array: calls that overlap on the GPU (other streams,
+ *     or other host threads without ordering) race and give wrong results.
+ *   - Shapes needing more than MEMOROID_STATIC_WORKSPACE_BYTES of workspace
+ *     (memoroid_scan_diag_workspace_bytes) return MEMOROID_ERR_WORKSPACE.
+ */
+memoroid_status_t memoroid_scan_diag_fwd_static(const void *lambda, int lambda_per_step,
+                                                const void *u, const uint8_t *start, const void *h0,
+                                                void *h, void *h_last, int64_t B, int64_t L,
+                                                int64_t D, void *stream);
+
 /* ======================================================================== */
 /* Episode index list <-> begin flags (Algorithm 1 keeps I = where(b)).     */
 /* ======================================================================== */

@@ -45,6 +45,7 @@ SIGNATURES = {
     "memoroid_scan_diag_fwd": (_int, [_p, _int, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_scan_diag_bwd": (_int, [_p, _int, _p, _p, _p, _p, _p, _p, _p, _p, _i64, _i64, _i64,
                                       _p, _sz, _p]),
+    "memoroid_scan_diag_fwd_static": (_int, [_p, _int, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p]),
     "memoroid_starts_from_offsets": (_int, [_p, _i64, _i64, _p, _p]),
     "memoroid_offsets_workspace_bytes": (_sz, [_i64]),
     "memoroid_offsets_from_starts": (_int, [_p, _i64, _p, _p, _p, _sz, _p]),
@@ -142,6 +143,15 @@ def memoroid_scan_diag_bwd(lam, lambda_per_step, start, h0, h, grad_h, grad_h_la
                                        _ptr(grad_h0), B, L, D, _ptr(workspace),
                                        workspace.numel() if workspace is not None else 0, _stream(stream))
     _check(st, "memoroid_scan_diag_bwd")
+
+
+def memoroid_scan_diag_fwd_static(lam, lambda_per_step, u, start, h0, h, h_last, B, L, D, stream=None):
+    """Forward scan that takes no workspace: it uses a fixed-size scratch array
+    owned by the library (see include/memoroid.h for the rules of use)."""
+    _need_cuda(lam, u, start, h0, h, h_last)
+    st = load().memoroid_scan_diag_fwd_static(_ptr(lam), int(lambda_per_step), _ptr(u), _ptr(start), _ptr(h0),
+                                              _ptr(h), _ptr(h_last), B, L, D, _stream(stream))
+    _check(st, "memoroid_scan_diag_fwd_static")
 
 
 def memoroid_starts_from_offsets(offsets, E, L, start, stream=None):
