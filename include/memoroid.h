@@ -144,6 +144,50 @@ memoroid_status_t memoroid_scan_diag_fwd_static(const void *lambda, int lambda_p
                                                 int64_t D, void *stream);
 
 /* ======================================================================== */
+/* Decayed linear-attention memoroid: the Linear Transformer memoroid of    */
+/* the appendix on rewriting sequence models as memoroids, with a decay and  */
+/* reset by the begin flag through Theorem 3.2:                              */
+/*   S_t = [b_t = 0] gamma_t S_{t-1} + k_t v_t^T,   y_t = S_t^T q_t          */
+/* S_{-1} = S0 (NULL = 0).  No feature map and no normaliser: y is the raw   */
+/* read-out of the state.                                                    */
+/* ======================================================================== */
+
+/* Workspace bytes for memoroid_scan_linattn_fwd with this shape (0 for an
+ * unsupported shape).  dk == dv == D with D in {64, 128}; chunk in {64, 128}. */
+size_t memoroid_scan_linattn_workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t dk,
+                                             int64_t dv, int64_t chunk);
+
+/* Number of kernels one call launches for this shape (-1 if unsupported). */
+int memoroid_scan_linattn_kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t dk,
+                                           int64_t dv, int backward, int with_S_last);
+
+/*
+ * Forward pass.
+ *   q, k        bf16 [B, L, H, dk]   (in_dtype must be MEMOROID_BF16)
+ *   v           bf16 [B, L, H, dv]
+ *   gamma       fp32 [H] (gamma_per_step = 0) or [B, L, H]; the decay applied
+ *               to S_{t-1} at step t, ignored at start steps.  Values are
+ *               used through log2(gamma), clamped below at -126.
+ *   start       uint8 [B, L], nonzero = b_t (first step of an episode)
+ *   S0          fp32 [B, H, dk, dv] or NULL
+ *   y           fp32 [B, L, H, dv] output
+ *   S_last      fp32 [B, H, dk, dv] output (the state after step L-1) or NULL
+ * All arrays are row-major, contiguous device memory owned by the caller;
+ * q, k, v, S0, y and S_last must be 16-byte aligned, the workspace 256-byte
+ * aligned and at least memoroid_scan_linattn_workspace_bytes.  `chunk` is the
+ * block size of the chunked evaluation; 64 and 128 compute the same function
+ * (the kernels tile the tape by 128 steps, the tensor-core M, for both).
+ * Asynchronous on `stream`; argument errors return at once, device-side wait
+ * timeouts are read with memoroid_get_device_error(workspace).
+ */
+memoroid_status_t memoroid_scan_linattn_fwd(const void *q, const void *k, const void *v,
+                                            int in_dtype, const float *gamma, int gamma_per_step,
+                                            const uint8_t *start, const float *S0, float *y,
+                                            float *S_last, int64_t B, int64_t L, int64_t H,
+                                            int64_t dk, int64_t dv, int64_t chunk, void *workspace,
+                                            size_t workspace_bytes, void *stream);
+
+/* ======================================================================== */
 /* Episode index list <-> begin flags (Algorithm 1 keeps I = where(b)).     */
 /* ======================================================================== */
 

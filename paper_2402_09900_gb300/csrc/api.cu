@@ -210,4 +210,76 @@ memoroid_status_t memoroid_offsets_from_starts(const uint8_t* start, int64_t L, 
                                             as_stream(stream));
 }
 
+
+// ---------------------------------------------------------------------------
+// decayed linear attention
+// ---------------------------------------------------------------------------
+
+static bool la_shape_ok(int64_t B, int64_t L, int64_t H, int64_t dk, int64_t dv, int64_t chunk) {
+    if (B < 0 || L < 0 || H < 0) return false;
+    if (dk != dv || (dk != 64 && dk != 128)) return false;
+    return chunk == 64 || chunk == 128;
+}
+
+size_t memoroid_scan_linattn_workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t dk, int64_t dv,
+                                             int64_t chunk) {
+    if (!la_shape_ok(B, L, H, dk, dv, chunk)) return 0;
+    return la::workspace_bytes(B, L, H, dk);
+}
+
+int memoroid_scan_linattn_kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t dk, int64_t dv, int backward,
+                                           int with_S_last) {
+    if (!la_shape_ok(B, L, H, dk, dv, 64)) return -1;
+    return la::kernels_per_call(B, L, H, backward != 0, with_S_last != 0);
+}
+
+memoroid_status_t memoroid_scan_linattn_fwd(const void* q, const void* k, const void* v, int in_dtype,
+                                            const float* gamma, int gamma_per_step, const uint8_t* start,
+                                            const float* S0, float* y, float* S_last, int64_t B, int64_t L,
+                                            int64_t H, int64_t dk, int64_t dv, int64_t chunk, void* workspace,
+                                            size_t workspace_bytes, void* stream) {
+    if (B < 0 || L < 0 || H < 0 || dk < 0 || dv < 0) return MEMOROID_ERR_INVALID_ARG;
+    if (gamma_per_step != 0 && gamma_per_step != 1) return MEMOROID_ERR_INVALID_ARG;
+    if (in_dtype != MEMOROID_BF16 && in_dtype != MEMOROID_F32) return MEMOROID_ERR_INVALID_ARG;
+    if (!la_shape_ok(B, L, H, dk, dv, chunk) || in_dtype != MEMOROID_BF16) return MEMOROID_ERR_UNSUPPORTED;
+    const bool work = B > 0 && L > 0 && H > 0;
+    if (work) {
+        if (!q || !k || !v || !gamma || !start || !y) return MEMOROID_ERR_INVALID_ARG;
+        if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(y, 16) || !aligned(gamma, 4))
+            return MEMOROID_ERR_INVALID_ARG;
+    }
+    if ((S0 && !aligned(S0, 16)) || (S_last && !aligned(S_last, 16))) return MEMOROID_ERR_INVALID_ARG;
+    cudaStream_t s = as_stream(stream);
+    if (!work) {
+        // empty tape: S_last = S0 (or zero)
+        if (S_last && B > 0 && H > 0) {
+            const size_t bytes = static_cast<size_t>(B * H) * dk * dv * sizeof(float);
+            const cudaError_t e = S0 ? cudaMemcpyAsync(S_last, S0, bytes, cudaMemcpyDeviceToDevice, s)
+                                     : cudaMemsetAsync(S_last, 0, bytes, s);
+            if (e != cudaSuccess) return MEMOROID_ERR_CUDA;
+        }
+        return MEMOROID_OK;
+    }
+    if (workspace == nullptr || !aligned(workspace, 256) ||
+        workspace_bytes < la::workspace_bytes(B, L, H, dk))
+        return MEMOROID_ERR_WORKSPACE;
+    la::Args a{};
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.gamma = gamma;
+    a.gamma_per_step = gamma_per_step;
+    a.start = start;
+    a.S0 = S0;
+    a.y = y;
+    a.S_last = S_last;
+    a.B = B;
+    a.L = L;
+    a.H = H;
+    a.D = dk;
+    a.workspace = workspace;
+    a.workspace_bytes = workspace_bytes;
+    return la::launch_fwd(a, s);
+}
+
 }  // extern "C"

@@ -19,6 +19,7 @@ enum DeviceError : uint32_t {
     DEV_CARRY_TIMEOUT = 5,     // a compute warp's wait for its carry ran out
     DEV_ACC_TIMEOUT = 6,       // the wait for grad_lambda partials ran out
     DEV_DRAIN_TIMEOUT = 7,     // the final wait for in-flight copies ran out
+    DEV_MMA_TIMEOUT = 8,       // a wait for tensor-core completion ran out
 };
 
 // Workspace header (256 bytes): [0] error code, [1] tile ticket counter,
@@ -64,6 +65,29 @@ memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream);
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream);
 
 }  // namespace diag
+
+namespace la {
+
+struct Args {
+    const void* q;  // bf16 [B, L, H, D]
+    const void* k;
+    const void* v;
+    const float* gamma;  // [H] or [B, L, H]
+    int gamma_per_step;
+    const uint8_t* start;  // [B, L]
+    const float* S0;       // [B, H, D, D] or null
+    float* y;              // [B, L, H, D]
+    float* S_last;         // [B, H, D, D] or null
+    int64_t B, L, H, D;
+    void* workspace;
+    size_t workspace_bytes;
+};
+
+size_t workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D);
+int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_S_last);
+memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream);
+
+}  // namespace la
 
 namespace tape {
 size_t offsets_workspace_bytes(int64_t L);

@@ -46,6 +46,10 @@ SIGNATURES = {
     "memoroid_scan_diag_bwd": (_int, [_p, _int, _p, _p, _p, _p, _p, _p, _p, _p, _i64, _i64, _i64,
                                       _p, _sz, _p]),
     "memoroid_scan_diag_fwd_static": (_int, [_p, _int, _p, _p, _p, _p, _p, _i64, _i64, _i64, _p]),
+    "memoroid_scan_linattn_workspace_bytes": (_sz, [_i64, _i64, _i64, _i64, _i64, _i64]),
+    "memoroid_scan_linattn_kernels_per_call": (_int, [_i64, _i64, _i64, _i64, _i64, _int, _int]),
+    "memoroid_scan_linattn_fwd": (_int, [_p, _p, _p, _int, _p, _int, _p, _p, _p, _p, _i64, _i64, _i64,
+                                         _i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_starts_from_offsets": (_int, [_p, _i64, _i64, _p, _p]),
     "memoroid_offsets_workspace_bytes": (_sz, [_i64]),
     "memoroid_offsets_from_starts": (_int, [_p, _i64, _p, _p, _p, _sz, _p]),
@@ -154,6 +158,24 @@ def memoroid_scan_diag_fwd_static(lam, lambda_per_step, u, start, h0, h, h_last,
     _check(st, "memoroid_scan_diag_fwd_static")
 
 
+def memoroid_scan_linattn_workspace_bytes(B, L, H, dk, dv, chunk) -> int:
+    return int(load().memoroid_scan_linattn_workspace_bytes(B, L, H, dk, dv, chunk))
+
+
+def memoroid_scan_linattn_kernels_per_call(B, L, H, dk, dv, backward, with_S_last) -> int:
+    return int(load().memoroid_scan_linattn_kernels_per_call(B, L, H, dk, dv, int(backward), int(with_S_last)))
+
+
+def memoroid_scan_linattn_fwd(q, k, v, in_dtype, gamma, gamma_per_step, start, S0, y, S_last, B, L, H, dk, dv,
+                              chunk, workspace, stream=None):
+    _need_cuda(q, k, v, gamma, start, S0, y, S_last, workspace)
+    st = load().memoroid_scan_linattn_fwd(_ptr(q), _ptr(k), _ptr(v), int(in_dtype), _ptr(gamma),
+                                          int(gamma_per_step), _ptr(start), _ptr(S0), _ptr(y), _ptr(S_last),
+                                          B, L, H, dk, dv, chunk, _ptr(workspace),
+                                          workspace.numel() if workspace is not None else 0, _stream(stream))
+    _check(st, "memoroid_scan_linattn_fwd")
+
+
 def memoroid_starts_from_offsets(offsets, E, L, start, stream=None):
     _need_cuda(offsets, start)
     _check(load().memoroid_starts_from_offsets(_ptr(offsets), E, L, _ptr(start), _stream(stream)),
@@ -222,6 +244,25 @@ def diag_bwd(lam, start, h, grad_h, grad_h_last=None, h0=None, want_lambda=True,
     memoroid_scan_diag_bwd(lam, per_step, start, h0, h, grad_h, grad_h_last, grad_u, grad_lambda, grad_h0,
                            B, L, D, ws, stream)
     return grad_u, grad_lambda, grad_h0
+
+
+def linattn_workspace(B, L, H, d, device, chunk=64) -> torch.Tensor:
+    return workspace(memoroid_scan_linattn_workspace_bytes(B, L, H, d, d, chunk), device)
+
+
+def linattn_fwd(q, k, v, gamma, start, S0=None, want_last=True, chunk=64, ws=None, out=None, stream=None):
+    """y, S_last of the decayed linear-attention memoroid.  q, k, v: bf16
+    [B,L,H,d] (torch.bfloat16, or their bits as int16/uint16); gamma: fp32 [H]
+    or [B,L,H]; start: uint8 [B,L]; S0: fp32 [B,H,d,d] or None."""
+    B, L, H, d = q.shape
+    per_step = gamma.dim() == 3
+    if ws is None:
+        ws = linattn_workspace(B, L, H, d, q.device, chunk)
+    y = torch.empty((B, L, H, d), dtype=torch.float32, device=q.device) if out is None else out
+    S_last = torch.empty((B, H, d, d), dtype=torch.float32, device=q.device) if want_last else None
+    memoroid_scan_linattn_fwd(q, k, v, MEMOROID_BF16, gamma, per_step, start, S0, y, S_last, B, L, H, d, d, chunk,
+                              ws, stream)
+    return y, S_last
 
 
 def starts_from_offsets(offsets, L, stream=None):
