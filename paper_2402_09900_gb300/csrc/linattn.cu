@@ -13,12 +13,13 @@
 //   S_tile = [no start in tile] exp(Lam_end) S_prev + sum_{r >= last start} exp(Lam_end - Lam_r) k_r v_r^T.
 // Both are dense bf16 contractions with fp32 accumulators in tensor memory.
 //
-// Parallel structure: each CTA owns one (tape, head, segment) and walks the
-// segment's tiles in order, carrying the state in TMEM.  Segments start from
-// a zero state; a carry kernel then folds the segment end states in tape
-// order, and a fix-up kernel adds each segment's incoming state to the outputs
-// of its steps before its first start.  The reset makes the fold exact: a
-// start inside a segment cuts every dependence on earlier segments.
+// Parallel structure: the tape of each (tape, head) is cut into segments
+// whose boundaries are moved forward to the next begin flag, so every segment
+// (but the first, which may continue from S0) starts from the zero state: the
+// reset of Theorem 3.2 makes the segments independent, and no carry or fix-up
+// pass is needed.  Each CTA owns one (tape, head, segment) and walks its tiles
+// in order, carrying the state in TMEM.  A nominal segment without any begin
+// flag is absorbed by the segment before it.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -68,21 +69,57 @@ Plan make_plan(int64_t B, int64_t L, int64_t H) {
 }
 
 struct Layout {
-    size_t meta, seg_decay, seg_state, total;
+    size_t meta, seg_first, total;
 };
 
 Layout make_layout(int64_t B, int64_t L, int64_t H, int64_t D) {
+    (void)D;
     const Plan pl = make_plan(B, L, H);
     Layout ly;
     size_t off = kHeaderBytes;
     ly.meta = off;
     off = align_up(off + static_cast<size_t>(B * H * pl.n_tiles) * sizeof(TileMeta), 256);
-    ly.seg_decay = off;
-    off = align_up(off + static_cast<size_t>(B * H * pl.G) * sizeof(float), 256);
-    ly.seg_state = off;
-    off = align_up(off + static_cast<size_t>(B * H * pl.G) * D * D * sizeof(float), 256);
+    ly.seg_first = off;
+    off = align_up(off + static_cast<size_t>(B * pl.G) * sizeof(int64_t), 256);
     ly.total = off;
     return ly;
+}
+
+// ---------------------------------------------------------------------------
+// kernel 0: segment boundaries at begin flags
+// ---------------------------------------------------------------------------
+// first[b][g] = the first step t in the nominal range [g, g + 1) * seg_len with
+// start[b][t] = 1 (segment 0: step 0), or -1 if the range holds no begin flag.
+// One warp per (tape, segment); each lane tests 16 consecutive flags per pass.
+__global__ void __launch_bounds__(256) plan_kernel(const uint8_t* __restrict__ start, int64_t B, int64_t L,
+                                                   int64_t seg_len, int64_t G, int64_t* __restrict__ first) {
+    const int64_t wid = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (wid >= B * G) return;
+    const int64_t b = wid / G, g = wid % G;
+    if (g == 0) {
+        if (lane == 0) first[wid] = 0;
+        return;
+    }
+    const int64_t p0 = g * seg_len, p1 = min(L, p0 + seg_len);
+    const uint8_t* row = start + b * L;
+    int64_t found = -1;
+    for (int64_t base = p0; base < p1 && found < 0; base += 32 * 16) {
+        int hit = 16;
+        const int64_t t0 = base + lane * 16;
+#pragma unroll
+        for (int x = 15; x >= 0; --x) {
+            const int64_t t = t0 + x;
+            if (t < p1 && row[t] != 0) hit = x;
+        }
+        const unsigned m = __ballot_sync(0xffffffffu, hit < 16);
+        if (m != 0) {
+            const int src = __ffs(m) - 1;
+            const int h = __shfl_sync(0xffffffffu, hit, src);
+            found = base + src * 16 + h;
+        }
+    }
+    if (lane == 0) first[wid] = found;
 }
 
 // ---------------------------------------------------------------------------
@@ -245,6 +282,10 @@ struct FwdSmem {
     static constexpr int OFF_META = OFF_SB + D * D * 2;
     static constexpr int OFF_BAR = OFF_META + 4 * static_cast<int>(sizeof(TileMeta));
     static constexpr int BYTES = OFF_BAR + 32;
+    // fp32 output rows staged in the finished stage for bulk stores: one row
+    // per step, padded by 16 bytes so that 8 consecutive rows hit 8 bank groups
+    static constexpr int YROW = D * 4 + 16;
+    static_assert(T * YROW <= STAGE, "output staging fits in one stage");
     // TMEM columns: scores P, intra output, inter output, state S
     static constexpr uint32_t COL_P = 0, COL_YA = 128, COL_YI = 128 + D, COL_S = 128 + 2 * D;
     static constexpr uint32_t TMEM_COLS = 512;
@@ -258,21 +299,35 @@ struct FwdParams {
     const float* S0;
     float* y;
     const TileMeta* meta;
-    float* seg_state;
-    float* seg_decay;
+    const int64_t* seg_first;  // [B][G] from plan_kernel
+    float* S_last;
     uint32_t* hdr;
     int64_t B, L, H, n_tiles, tps;
     int G;
     uint64_t wait_ns;
 };
 
-// Thread -> (row, first column) of a D x D state accumulator in TMEM.  With
-// M = 128 the row is the TMEM lane; with M = 64 rows 16q..16q+15 sit in lanes
-// 32q..32q+15 and the upper 16 lanes of each quarter hold nothing.
+// Thread -> row of a D x D state accumulator in TMEM.  With M = 128 the row
+// is the TMEM lane; with M = 64 rows 16q..16q+15 sit in lanes 32q..32q+15 and
+// the upper 16 lanes of each quarter hold nothing (-1).
 template <int D>
 __device__ __forceinline__ int state_row(int quarter, int lane) {
     if (D == 128) return 32 * quarter + lane;
     return lane < 16 ? 16 * quarter + lane : -1;
+}
+
+__device__ __forceinline__ void store_bf16x16(unsigned char* base, uint32_t off0, uint32_t off1, const float* v) {
+    uint4 w0, w1;
+    w0.x = pack_bf16x2(v[0], v[1]);
+    w0.y = pack_bf16x2(v[2], v[3]);
+    w0.z = pack_bf16x2(v[4], v[5]);
+    w0.w = pack_bf16x2(v[6], v[7]);
+    w1.x = pack_bf16x2(v[8], v[9]);
+    w1.y = pack_bf16x2(v[10], v[11]);
+    w1.z = pack_bf16x2(v[12], v[13]);
+    w1.w = pack_bf16x2(v[14], v[15]);
+    *reinterpret_cast<uint4*>(base + off0) = w0;
+    *reinterpret_cast<uint4*>(base + off1) = w1;
 }
 
 template <int D>
@@ -284,8 +339,20 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
     const int64_t bh = blockIdx.x / p.G;
     const int g = static_cast<int>(blockIdx.x % p.G);
     const int64_t b = bh / p.H, h = bh % p.H;
-    const int64_t tile0 = static_cast<int64_t>(g) * p.tps;
-    const int nt = static_cast<int>(min(p.tps, p.n_tiles - tile0));
+    // this segment covers steps [seg_lo, seg_hi): from its first begin flag to
+    // the next segment's (or the tape end)
+    const int64_t* sf = p.seg_first + b * p.G;
+    const int64_t seg_lo = sf[g];
+    if (seg_lo < 0) return;  // no begin flag in the nominal range: covered by an earlier segment
+    int64_t seg_hi = p.L;
+    for (int g2 = g + 1; g2 < p.G; ++g2) {
+        if (sf[g2] >= 0) {
+            seg_hi = sf[g2];
+            break;
+        }
+    }
+    const int64_t tile0 = seg_lo / T;
+    const int nt = static_cast<int>((seg_hi + T - 1) / T - tile0);
     const int64_t row_stride = p.H * D;  // elements between consecutive steps of one head
 
     uint64_t* bar1 = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
@@ -327,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
     const uint32_t tm = *tslot;
 
     const int srow = state_row<D>(quarter, lane);
-    constexpr int SC = D / 2;  // state columns per thread
+    constexpr int SC = D / 2;  // state and output columns per thread
     const uint32_t lane_base = tm + (static_cast<uint32_t>(32 * quarter) << 16);
 
     // ---- incoming state: S0 for the first segment of a tape ----
@@ -338,7 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
         have_state = scale;
         const float a0 = metas[0].a;
         const float* s0 = p.S0 + bh * D * D;
-#pragma unroll
+#pragma unroll 1
         for (int cc = 0; cc < SC / 16; ++cc) {
             const int j0 = half * SC + cc * 16;
             float v[16];
@@ -351,17 +418,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
                     v[x + 2] = f.z;
                     v[x + 3] = f.w;
                 }
-                uint4 w0, w1;
-                w0.x = pack_bf16x2(v[0], v[1]);
-                w0.y = pack_bf16x2(v[2], v[3]);
-                w0.z = pack_bf16x2(v[4], v[5]);
-                w0.w = pack_bf16x2(v[6], v[7]);
-                w1.x = pack_bf16x2(v[8], v[9]);
-                w1.y = pack_bf16x2(v[10], v[11]);
-                w1.z = pack_bf16x2(v[12], v[13]);
-                w1.w = pack_bf16x2(v[14], v[15]);
-                *reinterpret_cast<uint4*>(smem + S::OFF_SB + core_off(srow, j0, D)) = w0;
-                *reinterpret_cast<uint4*>(smem + S::OFF_SB + core_off(srow, j0 + 8, D)) = w1;
+                store_bf16x16(smem + S::OFF_SB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
             } else {
 #pragma unroll
                 for (int x = 0; x < 16; ++x) v[x] = 0.f;
@@ -379,21 +436,24 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
     constexpr uint32_t ID_PV = tc::idesc_bf16(128, D, false, true);
     constexpr uint32_t ID_KV = tc::idesc_bf16(D, D, true, true);
 
-    float aprod = 1.f;
     bool failed = false;
+#pragma unroll 1
     for (int c = 0; c < nt; ++c) {
         const int s = c & 1;
         const TileMeta& mc = metas[c & 3];
+        // tile c's copies (issued one iteration ago) and the previous tile's
+        // output stores (which read stage s ^ 1) are complete
+        cp_async_wait<0>();
+        if (warp == 0) bulk_wait_read();
+        tc::fence_smem_to_async();
+        tc::fence_before();
+        __syncthreads();
+        tc::fence_after();
         if (c + 1 < nt) {
             issue_tile(c + 1, s ^ 1);
             if (c + 2 < nt) load_meta_async(smem_addr(&metas[(c + 2) & 3]), gmeta + c + 2, tid);
         }
         cp_async_commit();
-        cp_async_wait<1>();
-        tc::fence_smem_to_async();
-        tc::fence_before();
-        __syncthreads();
-        tc::fence_after();
 
         // ---- P = Q K^T and (with an incoming state) Y_inter = Q S_prev ----
         if (tid == 0) {
@@ -408,6 +468,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
                 tc::mma(tm + S::COL_P, desc_kmajor(sq, D, kk), desc_kmajor(sk, D, kk), ID_QK, kk > 0);
             tc::commit(bar1);
         }
+
         bool ok = wait_mbar(bar1, c & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
             failed = true;
@@ -421,28 +482,21 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
             const float lt = mc.lam2[t];
             const int st = mc.seg[t];
             unsigned char* pm = smem + (stage_pm(s) - sbase);
+            uint32_t raw[64];
+#pragma unroll
+            for (int cc = 0; cc < 4; ++cc) tc::ld16_nowait(lane_base + S::COL_P + half * 64 + cc * 16, raw + cc * 16);
+            tc::ld_wait();
 #pragma unroll
             for (int cc = 0; cc < 4; ++cc) {
                 const int r0 = half * 64 + cc * 16;
                 float v[16];
-                tc::ld16(lane_base + S::COL_P + r0, v);
 #pragma unroll
                 for (int x = 0; x < 16; ++x) {
                     const int r = r0 + x;
                     const bool in = r <= t && r >= st;
-                    v[x] = in ? v[x] * exp2f(lt - mc.lam2[r]) : 0.f;
+                    v[x] = in ? __uint_as_float(raw[cc * 16 + x]) * fast_exp2(lt - mc.lam2[r]) : 0.f;
                 }
-                uint4 w0, w1;
-                w0.x = pack_bf16x2(v[0], v[1]);
-                w0.y = pack_bf16x2(v[2], v[3]);
-                w0.z = pack_bf16x2(v[4], v[5]);
-                w0.w = pack_bf16x2(v[6], v[7]);
-                w1.x = pack_bf16x2(v[8], v[9]);
-                w1.y = pack_bf16x2(v[10], v[11]);
-                w1.z = pack_bf16x2(v[12], v[13]);
-                w1.w = pack_bf16x2(v[14], v[15]);
-                *reinterpret_cast<uint4*>(pm + core_off(t, r0, T)) = w0;
-                *reinterpret_cast<uint4*>(pm + core_off(t, r0 + 8, T)) = w1;
+                store_bf16x16(pm, core_off(t, r0, T), core_off(t, r0 + 8, T), v);
             }
         }
         // ---- K~[r] = exp2(lam2_end - lam2_r) K[r] for rows of the last episode ----
@@ -451,12 +505,12 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
             const float lend = mc.lam2[T - 1];
             const int ls = mc.last_start;
             constexpr int NCH = T * D / 8;
-#pragma unroll
+#pragma unroll 2
             for (int e = tid; e < NCH; e += kThreads) {
                 // e enumerates 16-byte chunks in memory order: a row group of 8
                 // rows holds D chunks, 8 per core matrix, one per row
                 const int r = (e / D) * 8 + (e & 7);
-                const float w = r >= ls ? exp2f(lend - mc.lam2[r]) : 0.f;
+                const float w = r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f;
                 if (w != 1.f) {
                     uint4 u = *reinterpret_cast<uint4*>(kt + e * 16);
                     float2 f;
@@ -488,7 +542,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
             for (int kk = 0; kk < T / 16; ++kk)
                 tc::mma(tm + S::COL_S, desc_mnmajor(sk, D, kk), desc_mnmajor(sv, D, kk), ID_KV, acc || kk > 0);
             tc::commit(bar2);
-            aprod *= mc.a;
         }
         ok = wait_mbar(bar2, c & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
@@ -497,28 +550,37 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
         }
         tc::fence_after();
 
-        // ---- y = Y_intra + w_in * Y_inter ----
+        // ---- y = Y_intra + w_in * Y_inter, staged as fp32 rows in stage s ----
+        const int64_t t0 = (tile0 + c) * T;
+        // rows of this tile that belong to the segment
+        const int r_lo = static_cast<int>(max(static_cast<int64_t>(0), seg_lo - t0));
+        const int r_hi = static_cast<int>(min(static_cast<int64_t>(T), seg_hi - t0));
         {
             const int t = 32 * quarter + lane;
-            const int64_t tg = (tile0 + c) * T + t;
-            const bool valid = tg < p.L;
-            const float w_in = (have_prev && mc.seg[t] < 0) ? exp2f(mc.lam2[t]) : 0.f;
-            float* yrow = p.y + ((b * p.L + tg) * p.H + h) * D;
+            const float w_in = (have_prev && mc.seg[t] < 0) ? fast_exp2(mc.lam2[t]) : 0.f;
+            unsigned char* yst = smem + s * S::STAGE + t * S::YROW;
 #pragma unroll
-            for (int cc = 0; cc < D / 2 / 16; ++cc) {
-                const int j0 = half * (D / 2) + cc * 16;
-                float ya[16];
-                tc::ld16(lane_base + S::COL_YA + j0, ya);
+            for (int cc = 0; cc < SC / 32; ++cc) {
+                const int j0 = half * SC + cc * 32;
+                uint32_t ya[32], yi[32];
+                tc::ld16_nowait(lane_base + S::COL_YA + j0, ya);
+                tc::ld16_nowait(lane_base + S::COL_YA + j0 + 16, ya + 16);
                 if (have_prev) {
-                    float yi[16];
-                    tc::ld16(lane_base + S::COL_YI + j0, yi);
-#pragma unroll
-                    for (int x = 0; x < 16; ++x) ya[x] = fmaf(w_in, yi[x], ya[x]);
+                    tc::ld16_nowait(lane_base + S::COL_YI + j0, yi);
+                    tc::ld16_nowait(lane_base + S::COL_YI + j0 + 16, yi + 16);
                 }
-                if (valid) {
+                tc::ld_wait();
 #pragma unroll
-                    for (int x = 0; x < 16; x += 4)
-                        *reinterpret_cast<float4*>(yrow + j0 + x) = make_float4(ya[x], ya[x + 1], ya[x + 2], ya[x + 3]);
+                for (int x = 0; x < 32; x += 4) {
+                    float4 o = make_float4(__uint_as_float(ya[x]), __uint_as_float(ya[x + 1]),
+                                           __uint_as_float(ya[x + 2]), __uint_as_float(ya[x + 3]));
+                    if (have_prev) {
+                        o.x = fmaf(w_in, __uint_as_float(yi[x]), o.x);
+                        o.y = fmaf(w_in, __uint_as_float(yi[x + 1]), o.y);
+                        o.z = fmaf(w_in, __uint_as_float(yi[x + 2]), o.z);
+                        o.w = fmaf(w_in, __uint_as_float(yi[x + 3]), o.w);
+                    }
+                    *reinterpret_cast<float4*>(yst + (j0 + x) * 4) = o;
                 }
             }
         }
@@ -528,31 +590,28 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
             const bool scale = mn.has_start == 0 && mn.a != 1.f;
             const float an = mn.a;
 #pragma unroll
-            for (int cc = 0; cc < SC / 16; ++cc) {
-                const int j0 = half * SC + cc * 16;
-                float v[16];
-                tc::ld16(lane_base + S::COL_S + j0, v);
+            for (int cc = 0; cc < SC / 32; ++cc) {
+                const int j0 = half * SC + cc * 32;
+                uint32_t raw[32];
+                tc::ld16_nowait(lane_base + S::COL_S + j0, raw);
+                tc::ld16_nowait(lane_base + S::COL_S + j0 + 16, raw + 16);
+                tc::ld_wait();
+                float v[32];
+#pragma unroll
+                for (int x = 0; x < 32; ++x) v[x] = __uint_as_float(raw[x]);
                 if (srow >= 0) {
-                    uint4 w0, w1;
-                    w0.x = pack_bf16x2(v[0], v[1]);
-                    w0.y = pack_bf16x2(v[2], v[3]);
-                    w0.z = pack_bf16x2(v[4], v[5]);
-                    w0.w = pack_bf16x2(v[6], v[7]);
-                    w1.x = pack_bf16x2(v[8], v[9]);
-                    w1.y = pack_bf16x2(v[10], v[11]);
-                    w1.z = pack_bf16x2(v[12], v[13]);
-                    w1.w = pack_bf16x2(v[14], v[15]);
-                    *reinterpret_cast<uint4*>(smem + S::OFF_SB + core_off(srow, j0, D)) = w0;
-                    *reinterpret_cast<uint4*>(smem + S::OFF_SB + core_off(srow, j0 + 8, D)) = w1;
+                    store_bf16x16(smem + S::OFF_SB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
+                    store_bf16x16(smem + S::OFF_SB, core_off(srow, j0 + 16, D), core_off(srow, j0 + 24, D), v + 16);
                 }
                 if (scale) {
 #pragma unroll
-                    for (int x = 0; x < 16; ++x) v[x] *= an;
+                    for (int x = 0; x < 32; ++x) v[x] *= an;
                     tc::st16(lane_base + S::COL_S + j0, v);
+                    tc::st16(lane_base + S::COL_S + j0 + 16, v + 16);
                 }
             }
-        } else {
-            float* dst = p.seg_state + (bh * p.G + g) * D * D;
+        } else if (seg_hi == p.L && p.S_last != nullptr) {
+            float* dst = p.S_last + bh * D * D;
 #pragma unroll
             for (int cc = 0; cc < SC / 16; ++cc) {
                 const int j0 = half * SC + cc * 16;
@@ -565,7 +624,16 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
                 }
             }
         }
+        // ---- bulk-store the staged output rows ----
+        tc::fence_smem_to_async();
         tc::fence_before();
+        __syncthreads();
+        if (warp == 0) {
+            float* ybase = p.y + ((b * p.L + t0) * p.H + h) * D;
+            for (int r = r_lo + lane; r < r_hi; r += 32)
+                bulk_s2g(ybase + static_cast<int64_t>(r) * row_stride, sbase + s * S::STAGE + r * S::YROW, D * 4);
+            bulk_commit();
+        }
         have_prev = true;
         have_state = true;
     }
@@ -573,89 +641,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
         if (tid == 0) record_error(p.hdr, DEV_MMA_TIMEOUT);
         cp_async_wait<0>();
     }
-    if (tid == 0) p.seg_decay[bh * p.G + g] = failed ? 0.f : aprod;
+    if (warp == 0) bulk_wait_all();
     tc::fence_before();
     __syncthreads();
     tc::fence_after();
     if (warp == 0) tc::dealloc(tm, S::TMEM_COLS);
-}
-
-// ---------------------------------------------------------------------------
-// kernel 3: fold the segment end states in tape order (elementwise over dk x dv)
-// ---------------------------------------------------------------------------
-// On exit slot g holds the true state at the end of segment g, i.e. the
-// incoming state of segment g + 1:  C_{g+1} = A_g C_g + S_loc_g, C_1 = S_loc_0.
-__global__ void __launch_bounds__(256) carry_fwd_kernel(float* __restrict__ seg_state,
-                                                        const float* __restrict__ seg_decay, float* __restrict__ S_last,
-                                                        int G, int64_t DD) {
-    const int64_t bh = blockIdx.y;
-    const int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-    if (e >= DD) return;
-    float* st = seg_state + bh * G * DD + e;
-    float prev = st[0];
-    for (int g = 1; g < G; ++g) {
-        prev = fmaf(seg_decay[bh * G + g], prev, st[static_cast<int64_t>(g) * DD]);
-        st[static_cast<int64_t>(g) * DD] = prev;
-    }
-    if (S_last != nullptr) S_last[bh * DD + e] = prev;
-}
-
-// ---------------------------------------------------------------------------
-// kernel 4: add each segment's incoming state to its steps before its first start
-// ---------------------------------------------------------------------------
-//   y_t += (prod_{j = segment begin}^{t} gamma_j) C_g^T q_t
-template <int D>
-__global__ void __launch_bounds__(kThreads, 1) fix_fwd_kernel(const uint16_t* __restrict__ q, float* __restrict__ y,
-                                                             const TileMeta* __restrict__ meta,
-                                                             const float* __restrict__ seg_state, int64_t L, int64_t H,
-                                                             int64_t n_tiles, int64_t tps, int G) {
-    extern __shared__ __align__(16) float qs[];  // [T][D] fp32
-    constexpr int NG = kThreads / D;
-    const int tid = threadIdx.x, grp = tid / D, j = tid % D;
-    const int64_t bh = blockIdx.x / (G - 1);
-    const int g = static_cast<int>(blockIdx.x % (G - 1)) + 1;
-    const int64_t b = bh / H, h = bh % H;
-    const float* C = seg_state + (bh * G + g - 1) * D * D;
-    float cj[D];
-#pragma unroll
-    for (int i = 0; i < D; ++i) cj[i] = C[i * D + j];
-    const int64_t tile0 = static_cast<int64_t>(g) * tps;
-    const int64_t tile_end = min(n_tiles, tile0 + tps);
-    float cum = 1.f;
-    for (int64_t tile = tile0; tile < tile_end; ++tile) {
-        const TileMeta* m = meta + bh * n_tiles + tile;
-        const int64_t t0 = tile * T;
-        const int nvalid = static_cast<int>(min(static_cast<int64_t>(T), L - t0));
-        const int hs = m->has_start;
-        const int nfix = hs ? min(m->first_start, nvalid) : nvalid;
-        __syncthreads();
-        for (int e = tid; e < nfix * (D / 8); e += kThreads) {
-            const int r = e / (D / 8), c8 = e % (D / 8);
-            const uint4 u = *reinterpret_cast<const uint4*>(q + ((b * L + t0 + r) * H + h) * D + c8 * 8);
-            float2 f0 = unpack_bf16x2(u.x), f1 = unpack_bf16x2(u.y), f2 = unpack_bf16x2(u.z), f3 = unpack_bf16x2(u.w);
-            float4* dst = reinterpret_cast<float4*>(qs + r * D + c8 * 8);
-            dst[0] = make_float4(f0.x, f0.y, f1.x, f1.y);
-            dst[1] = make_float4(f2.x, f2.y, f3.x, f3.y);
-        }
-        __syncthreads();
-        for (int r = grp; r < nfix; r += NG) {
-            const float w = cum * exp2f(m->lam2[r]);
-            float acc = 0.f;
-            const float4* qr = reinterpret_cast<const float4*>(qs + r * D);
-#pragma unroll
-            for (int i4 = 0; i4 < D / 4; ++i4) {
-                const float4 qq = qr[i4];
-                acc = fmaf(cj[4 * i4], qq.x, acc);
-                acc = fmaf(cj[4 * i4 + 1], qq.y, acc);
-                acc = fmaf(cj[4 * i4 + 2], qq.z, acc);
-                acc = fmaf(cj[4 * i4 + 3], qq.w, acc);
-            }
-            float* yp = y + ((b * L + t0 + r) * H + h) * D + j;
-            *yp = fmaf(w, acc, *yp);
-        }
-        if (hs) break;
-        cum *= m->a;
-    }
 }
 
 // ---------------------------------------------------------------------------
@@ -671,14 +661,16 @@ template <int D>
 memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, cudaStream_t stream) {
     unsigned char* ws = static_cast<unsigned char*>(a.workspace);
     TileMeta* meta = reinterpret_cast<TileMeta*>(ws + ly.meta);
-    float* seg_decay = reinterpret_cast<float*>(ws + ly.seg_decay);
-    float* seg_state = reinterpret_cast<float*>(ws + ly.seg_state);
+    int64_t* seg_first = reinterpret_cast<int64_t*>(ws + ly.seg_first);
     uint32_t* hdr = reinterpret_cast<uint32_t*>(ws);
 
-    const int64_t n_meta_warps = a.B * a.H * pl.n_tiles;
-    const int64_t meta_blocks = (n_meta_warps * 32 + 255) / 256;
+    const int64_t meta_blocks = (a.B * a.H * pl.n_tiles * 32 + 255) / 256;
     meta_kernel<<<static_cast<unsigned>(meta_blocks), 256, 0, stream>>>(a.gamma, a.gamma_per_step, a.start, a.B,
                                                                          a.L, a.H, pl.n_tiles, meta);
+    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    const int64_t plan_blocks = (a.B * pl.G * 32 + 255) / 256;
+    plan_kernel<<<static_cast<unsigned>(plan_blocks), 256, 0, stream>>>(a.start, a.B, a.L, pl.tps * T, pl.G,
+                                                                         seg_first);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
 
     FwdParams p;
@@ -688,8 +680,8 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     p.S0 = a.S0;
     p.y = a.y;
     p.meta = meta;
-    p.seg_state = seg_state;
-    p.seg_decay = seg_decay;
+    p.seg_first = seg_first;
+    p.S_last = a.S_last;
     p.hdr = hdr;
     p.B = a.B;
     p.L = a.L;
@@ -701,20 +693,6 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     if (set_smem(fwd_kernel<D>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
     fwd_kernel<D><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
-
-    const int64_t DD = static_cast<int64_t>(D) * D;
-    if (pl.G > 1 || a.S_last != nullptr) {
-        dim3 grid(static_cast<unsigned>((DD + 255) / 256), static_cast<unsigned>(a.B * a.H));
-        carry_fwd_kernel<<<grid, 256, 0, stream>>>(seg_state, seg_decay, a.S_last, static_cast<int>(pl.G), DD);
-        if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
-    }
-    if (pl.G > 1) {
-        const int fix_smem = T * D * static_cast<int>(sizeof(float));
-        if (set_smem(fix_fwd_kernel<D>, fix_smem) != cudaSuccess) return MEMOROID_ERR_CUDA;
-        fix_fwd_kernel<D><<<static_cast<unsigned>(a.B * a.H * (pl.G - 1)), kThreads, fix_smem, stream>>>(
-            p.q, a.y, meta, seg_state, a.L, a.H, pl.n_tiles, pl.tps, static_cast<int>(pl.G));
-        if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
-    }
     return MEMOROID_OK;
 }
 }  // namespace
@@ -723,12 +701,9 @@ size_t workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D) { return make
 
 int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_S_last) {
     (void)backward;
+    (void)with_S_last;
     if (B == 0 || L == 0 || H == 0) return 0;
-    const Plan pl = make_plan(B, L, H);
-    int n = 2;
-    if (pl.G > 1 || with_S_last) ++n;
-    if (pl.G > 1) ++n;
-    return n;
+    return 3;
 }
 
 memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream) {

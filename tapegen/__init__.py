@@ -230,3 +230,53 @@ def linattn_config(cfg: int):
     t["grad_S_last"] = None
     t["chunk"] = c["chunk"]
     return t
+
+
+def linattn_tape_device(B: int, L: int, H: int, d: int, seed: int, mean: float, gamma_mode: str = "step",
+                        gammas=(0.9, 0.99, 0.999, 1.0), device="cuda", with_grad: bool = True,
+                        rows_per_draw: int = 1 << 18):
+    """The linattn_tape recipe drawn on the device with torch's seeded CUDA
+    generator, for tapes too large to draw and copy from the host (the L = 2^22,
+    8-head, d = 128 workload holds 26 GB of q, k, v).  Start flags come from the
+    host generator (numpy, same recipe as linattn_tape).  q, k, v are returned
+    as int16 tensors holding bf16 bit patterns; gamma, grad_y as fp32.
+
+    Values differ from linattn_tape for the same seed (another generator);
+    parity tests compare the GPU path with the oracle on slices copied back.
+    """
+    import torch
+
+    rng = np.random.default_rng(seed)
+    start = np.zeros((B, L), dtype=np.uint8)
+    for b in range(B):
+        start[b] = geometric_tape_starts(rng, L, mean)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(seed))
+    scale = 1.0 / float(np.sqrt(d))
+
+    def draw(normalise: bool, s: float):
+        out = torch.empty((B, L, H, d), dtype=torch.bfloat16, device=device)
+        for b in range(B):
+            for r0 in range(0, L, rows_per_draw):
+                r1 = min(L, r0 + rows_per_draw)
+                x = torch.randn((r1 - r0, H, d), generator=gen, device=device, dtype=torch.float32)
+                if normalise:
+                    x = x / x.norm(dim=-1, keepdim=True).clamp_min(1e-12)
+                else:
+                    x = x * s
+                out[b, r0:r1] = x.to(torch.bfloat16)
+        return out.view(torch.int16)
+
+    q = draw(False, scale)
+    k = draw(True, 1.0)
+    v = draw(False, scale)
+    if gamma_mode == "head":
+        gamma = torch.tensor([gammas[h % len(gammas)] for h in range(H)], dtype=torch.float32, device=device)
+    else:
+        z = torch.randn((B, L, H), generator=gen, device=device, dtype=torch.float32) + 3.0
+        gamma = torch.sigmoid(z)
+    out = dict(B=B, L=L, H=H, dk=d, dv=d, q=q, k=k, v=v, gamma=gamma, gamma_per_step=(gamma_mode != "head"),
+               start=torch.from_numpy(start).to(device))
+    if with_grad:
+        out["grad_y"] = torch.randn((B, L, H, d), generator=gen, device=device, dtype=torch.float32)
+    return out
