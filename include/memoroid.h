@@ -152,14 +152,17 @@ memoroid_status_t memoroid_scan_diag_fwd_static(const void *lambda, int lambda_p
 /* read-out of the state.                                                    */
 /* ======================================================================== */
 
-/* Workspace bytes for memoroid_scan_linattn_fwd with this shape (0 for an
- * unsupported shape).  dk == dv == D with D in {64, 128}; chunk in {64, 128}. */
+/* Workspace bytes for memoroid_scan_linattn_fwd and _bwd with this shape (0
+ * for an unsupported shape).  dk == dv == D with D in {64, 128}; chunk in
+ * {64, 128}.  The forward alone needs a few bytes per tile; the backward adds
+ * a bf16 copy of grad_y and one bf16 D x D state per 128-step tile. */
 size_t memoroid_scan_linattn_workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t dk,
                                              int64_t dv, int64_t chunk);
 
-/* Number of kernels one call launches for this shape (-1 if unsupported). */
+/* Number of kernels one call launches for this shape (-1 if unsupported);
+ * with_dgamma_per_head: a backward call with a per-head gamma and dgamma. */
 int memoroid_scan_linattn_kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t dk,
-                                           int64_t dv, int backward, int with_S_last);
+                                           int64_t dv, int backward, int with_dgamma_per_head);
 
 /*
  * Forward pass.
@@ -185,6 +188,32 @@ memoroid_status_t memoroid_scan_linattn_fwd(const void *q, const void *k, const 
                                             const uint8_t *start, const float *S0, float *y,
                                             float *S_last, int64_t B, int64_t L, int64_t H,
                                             int64_t dk, int64_t dv, int64_t chunk, void *workspace,
+                                            size_t workspace_bytes, void *stream);
+
+/*
+ * Backward pass of memoroid_scan_linattn_fwd (same inputs).  With
+ * dS_t = dL/dS_t accumulated backwards,
+ *   dS_t = q_t dy_t^T + [b_{t+1} = 0] gamma_{t+1} dS_{t+1},  dS_{L-1} += grad_S_last
+ *   dq_t = S_t dy_t,  dk_t = dS_t v_t,  dv_t = dS_t^T k_t,
+ *   dgamma_t = [b_t = 0] <dS_t, S_{t-1}>_F,  dS0 = [b_0 = 0] gamma_0 dS_0.
+ *   grad_y       fp32 [B, L, H, dv]
+ *   grad_S_last  fp32 [B, H, dk, dv] or NULL (= 0)
+ *   dq, dk, dv   fp32 [B, L, H, dk|dv] outputs (all three required)
+ *   dgamma       fp32 [H] (per-head gamma: summed over B and L) or [B, L, H]
+ *                (per-step gamma; 0 at start steps), or NULL to skip
+ *   dS0          fp32 [B, H, dk, dv] output or NULL
+ * q, k, v are consumed as bf16 and grad_y is rounded to bf16 for the tensor
+ * cores; all accumulation is fp32.  Every reduction has a fixed order, so
+ * repeated calls are bit-identical.  Workspace: at least
+ * memoroid_scan_linattn_workspace_bytes.
+ */
+memoroid_status_t memoroid_scan_linattn_bwd(const void *q, const void *k, const void *v,
+                                            int in_dtype, const float *gamma, int gamma_per_step,
+                                            const uint8_t *start, const float *S0,
+                                            const float *grad_y, const float *grad_S_last,
+                                            float *dq, float *dk_out, float *dv_out, float *dgamma,
+                                            float *dS0, int64_t B, int64_t L, int64_t H, int64_t dk,
+                                            int64_t dv, int64_t chunk, void *workspace,
                                             size_t workspace_bytes, void *stream);
 
 /* ======================================================================== */

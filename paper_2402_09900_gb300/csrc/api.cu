@@ -228,9 +228,9 @@ size_t memoroid_scan_linattn_workspace_bytes(int64_t B, int64_t L, int64_t H, in
 }
 
 int memoroid_scan_linattn_kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t dk, int64_t dv, int backward,
-                                           int with_S_last) {
+                                           int with_dgamma_per_head) {
     if (!la_shape_ok(B, L, H, dk, dv, 64)) return -1;
-    return la::kernels_per_call(B, L, H, backward != 0, with_S_last != 0);
+    return la::kernels_per_call(B, L, H, backward != 0, with_dgamma_per_head != 0);
 }
 
 memoroid_status_t memoroid_scan_linattn_fwd(const void* q, const void* k, const void* v, int in_dtype,
@@ -261,7 +261,7 @@ memoroid_status_t memoroid_scan_linattn_fwd(const void* q, const void* k, const 
         return MEMOROID_OK;
     }
     if (workspace == nullptr || !aligned(workspace, 256) ||
-        workspace_bytes < la::workspace_bytes(B, L, H, dk))
+        workspace_bytes < la::fwd_workspace_bytes(B, L, H, dk))
         return MEMOROID_ERR_WORKSPACE;
     la::Args a{};
     a.q = q;
@@ -280,6 +280,67 @@ memoroid_status_t memoroid_scan_linattn_fwd(const void* q, const void* k, const 
     a.workspace = workspace;
     a.workspace_bytes = workspace_bytes;
     return la::launch_fwd(a, s);
+}
+
+memoroid_status_t memoroid_scan_linattn_bwd(const void* q, const void* k, const void* v, int in_dtype,
+                                            const float* gamma, int gamma_per_step, const uint8_t* start,
+                                            const float* S0, const float* grad_y, const float* grad_S_last,
+                                            float* dq, float* dk_out, float* dv_out, float* dgamma, float* dS0,
+                                            int64_t B, int64_t L, int64_t H, int64_t dk, int64_t dv, int64_t chunk,
+                                            void* workspace, size_t workspace_bytes, void* stream) {
+    if (B < 0 || L < 0 || H < 0 || dk < 0 || dv < 0) return MEMOROID_ERR_INVALID_ARG;
+    if (gamma_per_step != 0 && gamma_per_step != 1) return MEMOROID_ERR_INVALID_ARG;
+    if (in_dtype != MEMOROID_BF16 && in_dtype != MEMOROID_F32) return MEMOROID_ERR_INVALID_ARG;
+    if (!la_shape_ok(B, L, H, dk, dv, chunk) || in_dtype != MEMOROID_BF16) return MEMOROID_ERR_UNSUPPORTED;
+    const bool work = B > 0 && L > 0 && H > 0;
+    if (work) {
+        if (!q || !k || !v || !gamma || !start || !grad_y || !dq || !dk_out || !dv_out) return MEMOROID_ERR_INVALID_ARG;
+        if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(grad_y, 16) || !aligned(dq, 16) ||
+            !aligned(dk_out, 16) || !aligned(dv_out, 16) || !aligned(gamma, 4))
+            return MEMOROID_ERR_INVALID_ARG;
+        if (dgamma && !aligned(dgamma, 4)) return MEMOROID_ERR_INVALID_ARG;
+    }
+    if ((S0 && !aligned(S0, 16)) || (grad_S_last && !aligned(grad_S_last, 16)) || (dS0 && !aligned(dS0, 16)))
+        return MEMOROID_ERR_INVALID_ARG;
+    cudaStream_t s = as_stream(stream);
+    if (!work) {
+        // empty tape: dS0 = grad_S_last (or zero), dgamma = 0
+        if (dS0 && B > 0 && H > 0) {
+            const size_t bytes = static_cast<size_t>(B * H) * dk * dv * sizeof(float);
+            const cudaError_t e = grad_S_last ? cudaMemcpyAsync(dS0, grad_S_last, bytes, cudaMemcpyDeviceToDevice, s)
+                                              : cudaMemsetAsync(dS0, 0, bytes, s);
+            if (e != cudaSuccess) return MEMOROID_ERR_CUDA;
+        }
+        if (dgamma && !gamma_per_step && H > 0) {
+            if (cudaMemsetAsync(dgamma, 0, static_cast<size_t>(H) * sizeof(float), s) != cudaSuccess)
+                return MEMOROID_ERR_CUDA;
+        }
+        return MEMOROID_OK;
+    }
+    if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < la::workspace_bytes(B, L, H, dk))
+        return MEMOROID_ERR_WORKSPACE;
+    la::Args a{};
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.gamma = gamma;
+    a.gamma_per_step = gamma_per_step;
+    a.start = start;
+    a.S0 = S0;
+    a.grad_y = grad_y;
+    a.dS_last = grad_S_last;
+    a.dq = dq;
+    a.dk = dk_out;
+    a.dv = dv_out;
+    a.dgamma = dgamma;
+    a.dS0 = dS0;
+    a.B = B;
+    a.L = L;
+    a.H = H;
+    a.D = dk;
+    a.workspace = workspace;
+    a.workspace_bytes = workspace_bytes;
+    return la::launch_bwd(a, s);
 }
 
 }  // extern "C"

@@ -76,16 +76,25 @@ struct Args {
     int gamma_per_step;
     const uint8_t* start;  // [B, L]
     const float* S0;       // [B, H, D, D] or null
-    float* y;              // [B, L, H, D]
-    float* S_last;         // [B, H, D, D] or null
+    float* y;              // fwd: [B, L, H, D]
+    float* S_last;         // fwd: [B, H, D, D] or null
+    const float* grad_y;   // bwd: [B, L, H, D]
+    const float* dS_last;  // bwd: [B, H, D, D] or null
+    float* dq;             // bwd outputs: [B, L, H, D]
+    float* dk;
+    float* dv;
+    float* dgamma;  // [H] or [B, L, H], or null
+    float* dS0;     // [B, H, D, D] or null
     int64_t B, L, H, D;
     void* workspace;
     size_t workspace_bytes;
 };
 
-size_t workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D);
-int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_S_last);
+size_t workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D);      // forward and backward
+size_t fwd_workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D);  // forward only
+int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_dgamma_per_head);
 memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream);
+memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream);
 
 }  // namespace la
 

@@ -69,11 +69,11 @@ Plan make_plan(int64_t B, int64_t L, int64_t H) {
 }
 
 struct Layout {
-    size_t meta, seg_first, total;
+    size_t meta, seg_first, fwd_total;
+    size_t dy16, states, dlam_f, gpart, total;  // backward only
 };
 
 Layout make_layout(int64_t B, int64_t L, int64_t H, int64_t D) {
-    (void)D;
     const Plan pl = make_plan(B, L, H);
     Layout ly;
     size_t off = kHeaderBytes;
@@ -81,6 +81,15 @@ Layout make_layout(int64_t B, int64_t L, int64_t H, int64_t D) {
     off = align_up(off + static_cast<size_t>(B * H * pl.n_tiles) * sizeof(TileMeta), 256);
     ly.seg_first = off;
     off = align_up(off + static_cast<size_t>(B * pl.G) * sizeof(int64_t), 256);
+    ly.fwd_total = off;
+    ly.dy16 = off;
+    off = align_up(off + static_cast<size_t>(B * L * H * D) * sizeof(uint16_t), 256);
+    ly.states = off;
+    off = align_up(off + static_cast<size_t>(B * H * pl.n_tiles * D * D) * sizeof(uint16_t), 256);
+    ly.dlam_f = off;
+    off = align_up(off + static_cast<size_t>(B * L * H) * sizeof(float), 256);
+    ly.gpart = off;
+    off = align_up(off + static_cast<size_t>(B * H * pl.G) * sizeof(float), 256);
     ly.total = off;
     return ly;
 }
@@ -305,11 +314,33 @@ struct FwdParams {
     int64_t B, L, H, n_tiles, tps;
     int G;
     uint64_t wait_ns;
+    // backward pass F only (see fwd_kernel<D, true>)
+    const uint16_t* zq;  // q, bf16 [B, L, H, D]
+    float* dlam_f;       // [B, L, H]: the state-side terms of dL/dlog(gamma_t)
+    uint16_t* states;    // [B, H, n_tiles, D, D] bf16: S_{c-1}^T before tiles without a begin flag
 };
 
 // Thread -> row of a D x D state accumulator in TMEM.  With M = 128 the row
 // is the TMEM lane; with M = 64 rows 16q..16q+15 sit in lanes 32q..32q+15 and
 // the upper 16 lanes of each quarter hold nothing (-1).
+// 16 bf16 values of row `row` (columns j0..j0+15) of the stored state before tile `tile`.
+template <int D>
+__device__ __forceinline__ void store_state_row(uint16_t* states, int64_t bh, int64_t n_tiles, int64_t tile,
+                                                     int row, int j0, const float* v) {
+    uint16_t* dst = states + ((bh * n_tiles + tile) * D + row) * D + j0;
+    uint4 w0, w1;
+    w0.x = pack_bf16x2(v[0], v[1]);
+    w0.y = pack_bf16x2(v[2], v[3]);
+    w0.z = pack_bf16x2(v[4], v[5]);
+    w0.w = pack_bf16x2(v[6], v[7]);
+    w1.x = pack_bf16x2(v[8], v[9]);
+    w1.y = pack_bf16x2(v[10], v[11]);
+    w1.z = pack_bf16x2(v[12], v[13]);
+    w1.w = pack_bf16x2(v[14], v[15]);
+    reinterpret_cast<uint4*>(dst)[0] = w0;
+    reinterpret_cast<uint4*>(dst)[1] = w1;
+}
+
 template <int D>
 __device__ __forceinline__ int state_row(int quarter, int lane) {
     if (D == 128) return 32 * quarter + lane;
@@ -330,7 +361,15 @@ __device__ __forceinline__ void store_bf16x16(unsigned char* base, uint32_t off0
     *reinterpret_cast<uint4*>(base + off1) = w1;
 }
 
-template <int D>
+// BWD = false: the forward pass, y = S^T q.
+// BWD = true: pass F of the backward.  Called with (q, k, v) = (dy, v, k) and
+// S0^T, it carries S'_t = S_t^T and its output is dq_t = S_t dy_t.  It also
+// writes, per step s, the sum over t >= s in the tile of
+//   z_t = w_in_t q_t^T S_{c-1} dy_t
+// (the term of dL/dlog(gamma_s) that pairs the incoming state with the tile's
+// outputs), and stores S'_{c-1} as bf16 for every tile without a begin flag,
+// for pass R.
+template <int D, bool BWD>
 __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
     using S = FwdSmem<D>;
     extern __shared__ __align__(1024) unsigned char smem[];
@@ -410,15 +449,21 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
             const int j0 = half * SC + cc * 16;
             float v[16];
             if (srow >= 0) {
+                if (BWD) {
 #pragma unroll
-                for (int x = 0; x < 16; x += 4) {
-                    const float4 f = *reinterpret_cast<const float4*>(s0 + srow * D + j0 + x);
-                    v[x] = f.x;
-                    v[x + 1] = f.y;
-                    v[x + 2] = f.z;
-                    v[x + 3] = f.w;
+                    for (int x = 0; x < 16; ++x) v[x] = s0[(j0 + x) * D + srow];
+                } else {
+#pragma unroll
+                    for (int x = 0; x < 16; x += 4) {
+                        const float4 f = *reinterpret_cast<const float4*>(s0 + srow * D + j0 + x);
+                        v[x] = f.x;
+                        v[x + 1] = f.y;
+                        v[x + 2] = f.z;
+                        v[x + 3] = f.w;
+                    }
                 }
                 store_bf16x16(smem + S::OFF_SB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
+                if (BWD && metas[0].has_start == 0) store_state_row<D>(p.states, bh, p.n_tiles, 0, srow, j0, v);
             } else {
 #pragma unroll
                 for (int x = 0; x < 16; ++x) v[x] = 0.f;
@@ -429,6 +474,14 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
                 tc::st16(lane_base + S::COL_S + j0, v);
             }
         }
+    }
+
+    if (BWD && !have_prev && g == 0 && metas[0].has_start == 0 && srow >= 0) {
+        // the zero state before the tape's first tile
+        float zero[16];
+#pragma unroll
+        for (int x = 0; x < 16; ++x) zero[x] = 0.f;
+        for (int j0 = half * SC; j0 < half * SC + SC; j0 += 16) store_state_row<D>(p.states, bh, p.n_tiles, 0, srow, j0, zero);
     }
 
     constexpr uint32_t ID_QS = tc::idesc_bf16(128, D, false, true);
@@ -559,6 +612,10 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
             const int t = 32 * quarter + lane;
             const float w_in = (have_prev && mc.seg[t] < 0) ? fast_exp2(mc.lam2[t]) : 0.f;
             unsigned char* yst = smem + s * S::STAGE + t * S::YROW;
+            // BWD: z_t = w_in_t q_t . (S_{c-1} dy_t), the inter output dotted with q
+            const bool zrow = BWD && w_in != 0.f && t0 + t < p.L;
+            const uint16_t* qrow = BWD ? p.zq + ((b * p.L + t0 + t) * p.H + h) * D : nullptr;
+            float zacc = 0.f;
 #pragma unroll
             for (int cc = 0; cc < SC / 32; ++cc) {
                 const int j0 = half * SC + cc * 32;
@@ -582,7 +639,25 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
                     }
                     *reinterpret_cast<float4*>(yst + (j0 + x) * 4) = o;
                 }
+                if (zrow) {
+#pragma unroll
+                    for (int x = 0; x < 32; x += 8) {
+                        const uint4 u = *reinterpret_cast<const uint4*>(qrow + j0 + x);
+                        const float2 q0 = unpack_bf16x2(u.x), q1 = unpack_bf16x2(u.y), q2 = unpack_bf16x2(u.z),
+                                     q3 = unpack_bf16x2(u.w);
+                        zacc = fmaf(q0.x, __uint_as_float(yi[x]), zacc);
+                        zacc = fmaf(q0.y, __uint_as_float(yi[x + 1]), zacc);
+                        zacc = fmaf(q1.x, __uint_as_float(yi[x + 2]), zacc);
+                        zacc = fmaf(q1.y, __uint_as_float(yi[x + 3]), zacc);
+                        zacc = fmaf(q2.x, __uint_as_float(yi[x + 4]), zacc);
+                        zacc = fmaf(q2.y, __uint_as_float(yi[x + 5]), zacc);
+                        zacc = fmaf(q3.x, __uint_as_float(yi[x + 6]), zacc);
+                        zacc = fmaf(q3.y, __uint_as_float(yi[x + 7]), zacc);
+                    }
+                }
             }
+            // the row's 16 padding bytes hold the two column halves' partial z
+            if (BWD) *reinterpret_cast<float*>(yst + D * 4 + half * 4) = w_in * zacc;
         }
         // ---- state: bf16 copy for the next tile, decay by the next tile's a ----
         if (c + 1 < nt) {
@@ -602,6 +677,10 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
                 if (srow >= 0) {
                     store_bf16x16(smem + S::OFF_SB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
                     store_bf16x16(smem + S::OFF_SB, core_off(srow, j0 + 16, D), core_off(srow, j0 + 24, D), v + 16);
+                    if (BWD && mn.has_start == 0) {
+                        store_state_row<D>(p.states, bh, p.n_tiles, tile0 + c + 1, srow, j0, v);
+                        store_state_row<D>(p.states, bh, p.n_tiles, tile0 + c + 1, srow, j0 + 16, v + 16);
+                    }
                 }
                 if (scale) {
 #pragma unroll
@@ -634,6 +713,31 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
                 bulk_s2g(ybase + static_cast<int64_t>(r) * row_stride, sbase + s * S::STAGE + r * S::YROW, D * 4);
             bulk_commit();
         }
+        if (BWD && warp == 1) {
+            // suffix sums of z over the tile: dlam_f[t] = sum_{s >= t} z_s
+            const unsigned char* zst = smem + s * S::STAGE + D * 4;
+            float zv[4];
+#pragma unroll
+            for (int x = 0; x < 4; ++x) {
+                const float* zp = reinterpret_cast<const float*>(zst + (4 * lane + x) * S::YROW);
+                zv[x] = zp[0] + zp[1];
+            }
+#pragma unroll
+            for (int x = 2; x >= 0; --x) zv[x] += zv[x + 1];
+            float tot = zv[0];
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const float o = __shfl_down_sync(0xffffffffu, tot, off);
+                if (lane + off < 32) tot += o;
+            }
+            float after = __shfl_down_sync(0xffffffffu, tot, 1);
+            if (lane == 31) after = 0.f;
+#pragma unroll
+            for (int x = 0; x < 4; ++x) {
+                const int r = 4 * lane + x;
+                if (r >= r_lo && r < r_hi) p.dlam_f[(b * p.L + t0 + r) * p.H + h] = zv[x] + after;
+            }
+        }
         have_prev = true;
         have_state = true;
     }
@@ -649,6 +753,556 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
 }
 
 // ---------------------------------------------------------------------------
+// backward pass R: reverse sweep for dk, dv, the reverse state and dL/dgamma
+// ---------------------------------------------------------------------------
+// Per tile c, with G_c = dL/dS_c (the state at the tile's end) in TMEM:
+//   dk_r = sum_s M[s,r] (dy_s . v_r) q_s + w_out_r G_c v_r
+//   dv_r = sum_s M[s,r] (q_s . k_r) dy_s + w_out_r G_c^T k_r
+//   G_{c-1} = a_c G_c + sum_s w_in_s q_s dy_s^T
+// and dL/dlog(gamma_t) (t not a begin flag) = gamma_t <dS_t, S_{t-1}>, split
+// over the tile as
+//   sum_{s >= t > r} E[s,r]                     E = M o (Q K^T) o (dY V^T)
+//   + [no start in the tile up to t] sum_{s >= t} z_s      (pass F)
+//   + sum_{r < t} x_r,  x_r = w_out_r k_r^T G_c v_r
+//   + [no start in the tile] a_c <G_c, S_{c-1}>
+// The first term is sum_{u < t} (colsum_u(E) - rowsum_u(E)): both sums come
+// from the same fp32 E, so the telescoping cancels exactly up to fp32 rounding.
+template <int D>
+struct BwdSmem {
+    static constexpr int TILE = T * D * 2;
+    static constexpr int OFF_Q = 0, OFF_K = TILE, OFF_V = 2 * TILE, OFF_DY = 3 * TILE;
+    static constexpr int OFF_PM = 4 * TILE, OFF_DPM = 4 * TILE + T * T * 2;
+    static constexpr int OFF_GB = 4 * TILE + 2 * T * T * 2;
+    static constexpr int OFF_META = OFF_GB + D * D * 2;
+    static constexpr int OFF_BAR = OFF_META + static_cast<int>(sizeof(TileMeta));
+    static constexpr int BYTES = OFF_BAR + 64;
+    // statistics, in the V tile (free once the first contractions are done)
+    static constexpr int ST_COL = OFF_V;                // [4][T] column sums of E per lane quarter
+    static constexpr int ST_ROW = ST_COL + 4 * T * 4;   // [2][T] row sums of E per column half
+    static constexpr int ST_X = ST_ROW + 2 * T * 4;     // [2][T] x_r per column half
+    static constexpr int ST_IV = ST_X + 2 * T * 4;      // [8] per-warp partial <G, S>
+    static constexpr int ST_INTRA = ST_IV + 64;         // [T] intra-tile term
+    static_assert(ST_INTRA + T * 4 <= OFF_V + TILE, "statistics fit in the V tile");
+    // TMEM columns: P and dP, then dV and dK over them; V G^T; G
+    static constexpr uint32_t COL_P = 0, COL_DP = 128, COL_DV = 0, COL_DK = 128, COL_DKI = 256,
+                              COL_G = 256 + D, TMEM_COLS = 512;
+    static_assert(COL_G + D <= TMEM_COLS, "tensor memory budget");
+};
+
+struct BwdParams {
+    const uint16_t* q;
+    const uint16_t* k;
+    const uint16_t* v;
+    const uint16_t* dy;  // bf16 copy of grad_y
+    const float* gamma;
+    int gamma_per_step;
+    const float* dS_last;
+    float* dk;
+    float* dv;
+    float* dgamma;      // per step: [B, L, H] output; per head: null (partials go to gpart)
+    float* gpart;       // [B * H * G] per-segment sums of dL/dlog(gamma) (per-head mode)
+    float* dS0;
+    const TileMeta* meta;
+    const int64_t* seg_first;
+    const float* dlam_f;
+    const uint16_t* states;
+    uint32_t* hdr;
+    int64_t B, L, H, n_tiles;
+    int G;
+    uint64_t wait_ns;
+};
+
+// Reduces 32 values per lane over the warp's 32 lanes; lane l ends with the
+// total of value l (a butterfly that halves the vector at each step).
+__device__ __forceinline__ float warp_transpose_sum32(float (&v)[32], int lane) {
+#pragma unroll
+    for (int k = 16; k >= 1; k >>= 1) {
+        const bool upper = (lane & k) != 0;
+#pragma unroll
+        for (int i = 0; i < k; ++i) {
+            const float send = upper ? v[i] : v[i + k];
+            const float keep = upper ? v[i + k] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, k);
+        }
+    }
+    return v[0];
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
+    using S = BwdSmem<D>;
+    extern __shared__ __align__(1024) unsigned char smem[];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int quarter = warp & 3, half = warp >> 2;
+    const int64_t bh = blockIdx.x / p.G;
+    const int g = static_cast<int>(blockIdx.x % p.G);
+    const int64_t b = bh / p.H, h = bh % p.H;
+    const int64_t* sf = p.seg_first + b * p.G;
+    const int64_t seg_lo = sf[g];
+    if (seg_lo < 0) {
+        if (p.gpart != nullptr && tid == 0) p.gpart[bh * p.G + g] = 0.f;
+        return;
+    }
+    int64_t seg_hi = p.L;
+    for (int g2 = g + 1; g2 < p.G; ++g2) {
+        if (sf[g2] >= 0) {
+            seg_hi = sf[g2];
+            break;
+        }
+    }
+    const int64_t tile_lo = seg_lo / T, tile_hi = (seg_hi + T - 1) / T;  // tiles [tile_lo, tile_hi)
+    const int64_t row_stride = p.H * D;
+
+    uint64_t* bar1 = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
+    uint64_t* bar2 = bar1 + 1;
+    uint64_t* bar3 = bar1 + 2;
+    uint32_t* tslot = reinterpret_cast<uint32_t*>(bar1 + 3);
+    const TileMeta& mc = *reinterpret_cast<const TileMeta*>(smem + S::OFF_META);
+    const uint32_t sbase = smem_addr(smem);
+    const uint32_t sQ = sbase + S::OFF_Q, sK = sbase + S::OFF_K, sV = sbase + S::OFF_V, sDY = sbase + S::OFF_DY;
+    const uint32_t sPM = sbase + S::OFF_PM, sDPM = sbase + S::OFF_DPM, sGB = sbase + S::OFF_GB;
+    float* st_col = reinterpret_cast<float*>(smem + S::ST_COL);
+    float* st_row = reinterpret_cast<float*>(smem + S::ST_ROW);
+    float* st_x = reinterpret_cast<float*>(smem + S::ST_X);
+    float* st_iv = reinterpret_cast<float*>(smem + S::ST_IV);
+    float* st_intra = reinterpret_cast<float*>(smem + S::ST_INTRA);
+
+    auto issue_tile = [&](int64_t tile) {
+        const int64_t t0 = tile * T;
+        const int nvalid = static_cast<int>(min(static_cast<int64_t>(T), p.L - t0));
+        const int64_t off = ((b * p.L + t0) * p.H + h) * D;
+        load_tile_async<D>(sQ, p.q + off, row_stride, nvalid, tid);
+        load_tile_async<D>(sK, p.k + off, row_stride, nvalid, tid);
+        load_tile_async<D>(sV, p.v + off, row_stride, nvalid, tid);
+        load_tile_async<D>(sDY, p.dy + off, row_stride, nvalid, tid);
+        load_meta_async(sbase + S::OFF_META, p.meta + bh * p.n_tiles + tile, tid);
+        cp_async_commit();
+    };
+
+    if (tid == 0) {
+        mbar_init(bar1, 1);
+        mbar_init(bar2, 1);
+        mbar_init(bar3, 1);
+        fence_mbar_init();
+    }
+    if (warp == 0) tc::alloc(tslot, S::TMEM_COLS);
+    issue_tile(tile_hi - 1);
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    const uint32_t tm = *tslot;
+    const uint32_t lane_base = tm + (static_cast<uint32_t>(32 * quarter) << 16);
+    const int srow = state_row<D>(quarter, lane);
+    constexpr int SC = D / 2;
+
+    // ---- incoming reverse state: dS_last for the segment that ends the tape ----
+    bool have_g = false;
+    if (seg_hi == p.L && p.dS_last != nullptr) {
+        have_g = true;
+        const float* src = p.dS_last + bh * D * D;
+#pragma unroll 1
+        for (int cc = 0; cc < SC / 16; ++cc) {
+            const int j0 = half * SC + cc * 16;
+            float v[16];
+            if (srow >= 0) {
+#pragma unroll
+                for (int x = 0; x < 16; x += 4) {
+                    const float4 f = *reinterpret_cast<const float4*>(src + srow * D + j0 + x);
+                    v[x] = f.x;
+                    v[x + 1] = f.y;
+                    v[x + 2] = f.z;
+                    v[x + 3] = f.w;
+                }
+                store_bf16x16(smem + S::OFF_GB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
+            } else {
+#pragma unroll
+                for (int x = 0; x < 16; ++x) v[x] = 0.f;
+            }
+            tc::st16(lane_base + S::COL_G + j0, v);
+        }
+    }
+
+    constexpr uint32_t ID_SCORE = tc::idesc_bf16(128, T, false, false);  // P, dP
+    constexpr uint32_t ID_VG = tc::idesc_bf16(128, D, false, false);     // V G^T
+    constexpr uint32_t ID_PTDY = tc::idesc_bf16(128, D, true, true);     // Pm^T dY, dPm^T Q
+    constexpr uint32_t ID_KG = tc::idesc_bf16(128, D, false, true);      // K~ G
+    constexpr uint32_t ID_QDY = tc::idesc_bf16(D, D, true, true);        // Q~^T dY
+
+    float gsum = 0.f;  // per-head mode: sum of dL/dlog(gamma) over the segment's steps
+    bool failed = false;
+    int it = 0;
+#pragma unroll 1
+    for (int64_t tile = tile_hi - 1; tile >= tile_lo; --tile, ++it) {
+        const int64_t t0 = tile * T;
+        const int r_lo = static_cast<int>(max(static_cast<int64_t>(0), seg_lo - t0));
+        const int r_hi = static_cast<int>(min(static_cast<int64_t>(T), seg_hi - t0));
+        cp_async_wait<0>();
+        tc::fence_smem_to_async();
+        tc::fence_before();
+        __syncthreads();
+        tc::fence_after();
+        const bool tile_start = mc.has_start != 0;
+
+        // ---- B1: P = Q K^T, dP = dY V^T, dKi = V G^T ----
+        if (tid == 0) {
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk)
+                tc::mma(tm + S::COL_P, desc_kmajor(sQ, D, kk), desc_kmajor(sK, D, kk), ID_SCORE, kk > 0);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk)
+                tc::mma(tm + S::COL_DP, desc_kmajor(sDY, D, kk), desc_kmajor(sV, D, kk), ID_SCORE, kk > 0);
+            if (have_g) {
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk)
+                    tc::mma(tm + S::COL_DKI, desc_kmajor(sV, D, kk), desc_kmajor(sGB, D, kk), ID_VG, kk > 0);
+            }
+            tc::commit(bar1);
+        }
+        bool ok = wait_mbar(bar1, it & 1, p.wait_ns);
+        if (__syncthreads_or(!ok)) {
+            failed = true;
+            break;
+        }
+        tc::fence_after();
+
+        // ---- RP1: masks, E statistics, K~, <G_c, S_{c-1}>, G *= a ----
+        {
+            const int t = 32 * quarter + lane;  // the row s of P and dP this thread holds
+            const float lt = mc.lam2[t];
+            const int st = mc.seg[t];
+            float rsum = 0.f;
+#pragma unroll 1
+            for (int cc = 0; cc < 2; ++cc) {
+                const int r0 = half * 64 + cc * 32;
+                uint32_t rp[32], rd[32];
+                tc::ld16_nowait(lane_base + S::COL_P + r0, rp);
+                tc::ld16_nowait(lane_base + S::COL_P + r0 + 16, rp + 16);
+                tc::ld16_nowait(lane_base + S::COL_DP + r0, rd);
+                tc::ld16_nowait(lane_base + S::COL_DP + r0 + 16, rd + 16);
+                tc::ld_wait();
+                float pm[32], dpm[32], e[32];
+#pragma unroll
+                for (int x = 0; x < 32; ++x) {
+                    const int r = r0 + x;
+                    const float m = (r <= t && r >= st) ? fast_exp2(lt - mc.lam2[r]) : 0.f;
+                    const float pv = __uint_as_float(rp[x]), dv = __uint_as_float(rd[x]);
+                    pm[x] = m * pv;
+                    dpm[x] = m * dv;
+                    e[x] = pm[x] * dv;
+                    rsum += e[x];
+                }
+                unsigned char* pmb = smem + S::OFF_PM;
+                unsigned char* dpmb = smem + S::OFF_DPM;
+#pragma unroll
+                for (int x = 0; x < 32; x += 16) {
+                    store_bf16x16(pmb, core_off(t, r0 + x, T), core_off(t, r0 + x + 8, T), pm + x);
+                    store_bf16x16(dpmb, core_off(t, r0 + x, T), core_off(t, r0 + x + 8, T), dpm + x);
+                }
+                const float cs = warp_transpose_sum32(e, lane);
+                st_col[quarter * T + r0 + lane] = cs;
+            }
+            st_row[half * T + t] = rsum;
+        }
+        {
+            // K~ = w_out (.) K in place (K is not read unscaled after B1)
+            unsigned char* kt = smem + S::OFF_K;
+            const float lend = mc.lam2[T - 1];
+            const int ls = mc.last_start;
+            constexpr int NCH = T * D / 8;
+#pragma unroll 2
+            for (int e = tid; e < NCH; e += kThreads) {
+                const int r = (e / D) * 8 + (e & 7);
+                const float w = r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f;
+                if (w != 1.f) {
+                    uint4 u = *reinterpret_cast<uint4*>(kt + e * 16);
+                    float2 f;
+                    f = unpack_bf16x2(u.x);
+                    u.x = pack_bf16x2(f.x * w, f.y * w);
+                    f = unpack_bf16x2(u.y);
+                    u.y = pack_bf16x2(f.x * w, f.y * w);
+                    f = unpack_bf16x2(u.z);
+                    u.z = pack_bf16x2(f.x * w, f.y * w);
+                    f = unpack_bf16x2(u.w);
+                    u.w = pack_bf16x2(f.x * w, f.y * w);
+                    *reinterpret_cast<uint4*>(kt + e * 16) = u;
+                }
+            }
+        }
+        {
+            // <G_c, S_{c-1}> (tiles without a begin flag) and G <- a_c G
+            float ivp = 0.f;
+            const bool need_iv = have_g && !tile_start;
+            const bool scale = have_g && !tile_start && mc.a != 1.f;
+            if (need_iv || scale) {
+                const uint16_t* srows = p.states + (bh * p.n_tiles + tile) * D * D;  // S^T, row-major [j][i]
+#pragma unroll 1
+                for (int cc = 0; cc < SC / 16; ++cc) {
+                    const int j0 = half * SC + cc * 16;
+                    float v[16];
+                    tc::ld16(lane_base + S::COL_G + j0, v);
+                    if (need_iv && srow >= 0) {
+#pragma unroll
+                        for (int x = 0; x < 16; ++x) {
+                            const uint32_t bits = static_cast<uint32_t>(srows[(j0 + x) * D + srow]) << 16;
+                            ivp = fmaf(v[x], __uint_as_float(bits), ivp);
+                        }
+                    }
+                    if (scale) {
+#pragma unroll
+                        for (int x = 0; x < 16; ++x) v[x] *= mc.a;
+                        tc::st16(lane_base + S::COL_G + j0, v);
+                    }
+                }
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) ivp += __shfl_xor_sync(0xffffffffu, ivp, off);
+            if (lane == 0) st_iv[warp] = ivp;
+        }
+        tc::fence_smem_to_async();
+        tc::fence_before();
+        __syncthreads();
+        tc::fence_after();
+
+        // ---- B2: dV = Pm^T dY + K~ G, dK = dPm^T Q ----
+        if (tid == 0) {
+#pragma unroll
+            for (int kk = 0; kk < T / 16; ++kk)
+                tc::mma(tm + S::COL_DV, desc_mnmajor(sPM, T, kk), desc_mnmajor(sDY, D, kk), ID_PTDY, kk > 0);
+            if (have_g) {
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk)
+                    tc::mma(tm + S::COL_DV, desc_kmajor(sK, D, kk), desc_mnmajor(sGB, D, kk), ID_KG, true);
+            }
+#pragma unroll
+            for (int kk = 0; kk < T / 16; ++kk)
+                tc::mma(tm + S::COL_DK, desc_mnmajor(sDPM, T, kk), desc_mnmajor(sQ, D, kk), ID_PTDY, kk > 0);
+            tc::commit(bar2);
+        }
+        // intra-tile term while B2 runs: intra_t = sum_{u < t} (colsum_u - rowsum_u)
+        if (warp == 7) {
+            float d[4];
+#pragma unroll
+            for (int x = 0; x < 4; ++x) {
+                const int u = 4 * lane + x;
+                d[x] = (st_col[u] + st_col[T + u]) + (st_col[2 * T + u] + st_col[3 * T + u]) -
+                       (st_row[u] + st_row[T + u]);
+            }
+            float incl = d[0] + d[1] + d[2] + d[3];
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const float o = __shfl_up_sync(0xffffffffu, incl, off);
+                if (lane >= off) incl += o;
+            }
+            float run = incl - (d[0] + d[1] + d[2] + d[3]);
+#pragma unroll
+            for (int x = 0; x < 4; ++x) {
+                st_intra[4 * lane + x] = run;
+                run += d[x];
+            }
+        }
+        ok = wait_mbar(bar2, it & 1, p.wait_ns);
+        if (__syncthreads_or(!ok)) {
+            failed = true;
+            break;
+        }
+        tc::fence_after();
+
+        // ---- RP2: Q~ = w_in (.) Q in place, then B3: G += Q~^T dY ----
+        {
+            unsigned char* qt = smem + S::OFF_Q;
+            constexpr int NCH = T * D / 8;
+#pragma unroll 2
+            for (int e = tid; e < NCH; e += kThreads) {
+                const int r = (e / D) * 8 + (e & 7);
+                const float w = mc.seg[r] < 0 ? fast_exp2(mc.lam2[r]) : 0.f;
+                if (w != 1.f) {
+                    uint4 u = *reinterpret_cast<uint4*>(qt + e * 16);
+                    float2 f;
+                    f = unpack_bf16x2(u.x);
+                    u.x = pack_bf16x2(f.x * w, f.y * w);
+                    f = unpack_bf16x2(u.y);
+                    u.y = pack_bf16x2(f.x * w, f.y * w);
+                    f = unpack_bf16x2(u.z);
+                    u.z = pack_bf16x2(f.x * w, f.y * w);
+                    f = unpack_bf16x2(u.w);
+                    u.w = pack_bf16x2(f.x * w, f.y * w);
+                    *reinterpret_cast<uint4*>(qt + e * 16) = u;
+                }
+            }
+        }
+        tc::fence_smem_to_async();
+        tc::fence_before();
+        __syncthreads();
+        tc::fence_after();
+        if (tid == 0) {
+            const bool acc = have_g && !tile_start;
+#pragma unroll
+            for (int kk = 0; kk < T / 16; ++kk)
+                tc::mma(tm + S::COL_G, desc_mnmajor(sQ, D, kk), desc_mnmajor(sDY, D, kk), ID_QDY, acc || kk > 0);
+            tc::commit(bar3);
+        }
+
+        // ---- epilogue (while B3 runs): dk, dv, x_r ----
+        {
+            const int r = 32 * quarter + lane;
+            const bool store = r >= r_lo && r < r_hi;
+            const float w_out = r >= mc.last_start ? fast_exp2(mc.lam2[T - 1] - mc.lam2[r]) : 0.f;
+            float* dkrow = p.dk + ((b * p.L + t0 + r) * p.H + h) * D;
+            float* dvrow = p.dv + ((b * p.L + t0 + r) * p.H + h) * D;
+            float xacc = 0.f;
+#pragma unroll 1
+            for (int cc = 0; cc < SC / 16; ++cc) {
+                const int j0 = half * SC + cc * 16;
+                uint32_t rk[16], ri[16], rv[16];
+                tc::ld16_nowait(lane_base + S::COL_DK + j0, rk);
+                tc::ld16_nowait(lane_base + S::COL_DV + j0, rv);
+                if (have_g) tc::ld16_nowait(lane_base + S::COL_DKI + j0, ri);
+                tc::ld_wait();
+                float ok4[16];
+#pragma unroll
+                for (int x = 0; x < 16; ++x) {
+                    const float dki = have_g ? __uint_as_float(ri[x]) : 0.f;
+                    ok4[x] = fmaf(w_out, dki, __uint_as_float(rk[x]));
+                }
+                if (have_g) {
+                    // x_r = k~_r . dKi_r, with k~ = w_out k (the scaled K tile)
+                    const unsigned char* kt = smem + S::OFF_K;
+#pragma unroll
+                    for (int x = 0; x < 16; x += 8) {
+                        const uint4 u = *reinterpret_cast<const uint4*>(kt + core_off(r, j0 + x, D));
+                        const float2 k0 = unpack_bf16x2(u.x), k1 = unpack_bf16x2(u.y), k2 = unpack_bf16x2(u.z),
+                                     k3 = unpack_bf16x2(u.w);
+                        xacc = fmaf(k0.x, __uint_as_float(ri[x]), xacc);
+                        xacc = fmaf(k0.y, __uint_as_float(ri[x + 1]), xacc);
+                        xacc = fmaf(k1.x, __uint_as_float(ri[x + 2]), xacc);
+                        xacc = fmaf(k1.y, __uint_as_float(ri[x + 3]), xacc);
+                        xacc = fmaf(k2.x, __uint_as_float(ri[x + 4]), xacc);
+                        xacc = fmaf(k2.y, __uint_as_float(ri[x + 5]), xacc);
+                        xacc = fmaf(k3.x, __uint_as_float(ri[x + 6]), xacc);
+                        xacc = fmaf(k3.y, __uint_as_float(ri[x + 7]), xacc);
+                    }
+                }
+                if (store) {
+#pragma unroll
+                    for (int x = 0; x < 16; x += 4) {
+                        *reinterpret_cast<float4*>(dkrow + j0 + x) = make_float4(ok4[x], ok4[x + 1], ok4[x + 2], ok4[x + 3]);
+                        *reinterpret_cast<float4*>(dvrow + j0 + x) =
+                            make_float4(__uint_as_float(rv[x]), __uint_as_float(rv[x + 1]), __uint_as_float(rv[x + 2]),
+                                        __uint_as_float(rv[x + 3]));
+                    }
+                }
+            }
+            st_x[half * T + r] = xacc;
+        }
+        __syncthreads();
+        // ---- dL/dlog(gamma_t) for the tile's rows ----
+        if (warp < 4) {
+            const int t = 32 * warp + lane;
+            const float xt = st_x[t] + st_x[T + t];
+            // exclusive prefix of x over the tile: the lower warps' rows, then this warp's
+            float incl = xt;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const float o = __shfl_up_sync(0xffffffffu, incl, off);
+                if (lane >= off) incl += o;
+            }
+            float lower = 0.f;
+            for (int u = 0; u < 32 * warp; ++u) lower += st_x[u] + st_x[T + u];
+            const float xpre = lower + (incl - xt);
+            float iv = 0.f;
+            if (!tile_start) {
+                for (int w2 = 0; w2 < 8; ++w2) iv += st_iv[w2];
+                iv *= mc.a;
+            }
+            const bool in = t >= r_lo && t < r_hi;
+            const bool is_start = mc.seg[t] == t;
+            float dl = 0.f;
+            if (in && !is_start) {
+                const int64_t idx = (b * p.L + t0 + t) * p.H + h;
+                dl = st_intra[t] + xpre + iv + p.dlam_f[idx];
+                if (p.dgamma != nullptr) {
+                    const float gm = p.gamma_per_step ? p.gamma[idx] : p.gamma[h];
+                    p.dgamma[idx] = dl / gm;
+                }
+            } else if (in && p.dgamma != nullptr) {
+                p.dgamma[(b * p.L + t0 + t) * p.H + h] = 0.f;
+            }
+            // per-head mode: fixed-order tile total
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) dl += __shfl_xor_sync(0xffffffffu, dl, off);
+            if (lane == 0) st_iv[8 + warp] = dl;
+        }
+        ok = wait_mbar(bar3, it & 1, p.wait_ns);
+        if (__syncthreads_or(!ok)) {
+            failed = true;
+            break;
+        }
+        tc::fence_after();
+        if (tid == 0) gsum += (st_iv[8] + st_iv[9]) + (st_iv[10] + st_iv[11]);
+        have_g = true;
+
+        // ---- G_{c-1} -> bf16 operand for the next tile (and dS0 at the tape start) ----
+        {
+            const bool last = tile == tile_lo;
+            const bool write_ds0 = last && seg_lo == 0 && p.dS0 != nullptr;
+#pragma unroll 1
+            for (int cc = 0; cc < SC / 16; ++cc) {
+                const int j0 = half * SC + cc * 16;
+                float v[16];
+                tc::ld16(lane_base + S::COL_G + j0, v);
+                if (srow >= 0) {
+                    if (!last) store_bf16x16(smem + S::OFF_GB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
+                    if (write_ds0) {
+                        float* dst = p.dS0 + (bh * D + srow) * D + j0;
+#pragma unroll
+                        for (int x = 0; x < 16; x += 4)
+                            *reinterpret_cast<float4*>(dst + x) = make_float4(v[x], v[x + 1], v[x + 2], v[x + 3]);
+                    }
+                }
+            }
+        }
+        tc::fence_before();
+        __syncthreads();
+        if (tile > tile_lo) issue_tile(tile - 1);
+    }
+    if (failed) {
+        if (tid == 0) record_error(p.hdr, DEV_MMA_TIMEOUT);
+        cp_async_wait<0>();
+    }
+    if (tid == 0 && p.gpart != nullptr) p.gpart[bh * p.G + g] = gsum;
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    if (warp == 0) tc::dealloc(tm, S::TMEM_COLS);
+}
+
+// grad_y (fp32) -> bf16 operand copy (round to nearest even), 8 values per thread
+__global__ void __launch_bounds__(256) to_bf16_kernel(const float* __restrict__ x, uint16_t* __restrict__ y, int64_t n8) {
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n8;
+         i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const float4 a = reinterpret_cast<const float4*>(x)[2 * i];
+        const float4 c = reinterpret_cast<const float4*>(x)[2 * i + 1];
+        uint4 o;
+        o.x = pack_bf16x2(a.x, a.y);
+        o.y = pack_bf16x2(a.z, a.w);
+        o.z = pack_bf16x2(c.x, c.y);
+        o.w = pack_bf16x2(c.z, c.w);
+        reinterpret_cast<uint4*>(y)[i] = o;
+    }
+}
+
+// per-head dL/dgamma_h = (sum over tapes and segments of dL/dlog(gamma)) / gamma_h, fixed order
+__global__ void dgamma_head_kernel(const float* __restrict__ gpart, const float* __restrict__ gamma,
+                                   float* __restrict__ dgamma, int64_t B, int64_t H, int G) {
+    const int64_t h = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (h >= H) return;
+    double acc = 0.0;
+    for (int64_t b = 0; b < B; ++b)
+        for (int g = 0; g < G; ++g) acc += gpart[(b * H + h) * G + g];
+    dgamma[h] = static_cast<float>(acc / gamma[h]);
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 namespace {
@@ -657,13 +1311,9 @@ cudaError_t set_smem(K kernel, int bytes) {
     return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
-template <int D>
-memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, cudaStream_t stream) {
-    unsigned char* ws = static_cast<unsigned char*>(a.workspace);
-    TileMeta* meta = reinterpret_cast<TileMeta*>(ws + ly.meta);
-    int64_t* seg_first = reinterpret_cast<int64_t*>(ws + ly.seg_first);
-    uint32_t* hdr = reinterpret_cast<uint32_t*>(ws);
-
+// Tile metadata and segment boundaries (shared by the forward and backward passes).
+memoroid_status_t launch_prep(const Args& a, const Plan& pl, TileMeta* meta, int64_t* seg_first,
+                              cudaStream_t stream) {
     const int64_t meta_blocks = (a.B * a.H * pl.n_tiles * 32 + 255) / 256;
     meta_kernel<<<static_cast<unsigned>(meta_blocks), 256, 0, stream>>>(a.gamma, a.gamma_per_step, a.start, a.B,
                                                                          a.L, a.H, pl.n_tiles, meta);
@@ -672,6 +1322,17 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     plan_kernel<<<static_cast<unsigned>(plan_blocks), 256, 0, stream>>>(a.start, a.B, a.L, pl.tps * T, pl.G,
                                                                          seg_first);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    return MEMOROID_OK;
+}
+
+template <int D>
+memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, cudaStream_t stream) {
+    unsigned char* ws = static_cast<unsigned char*>(a.workspace);
+    TileMeta* meta = reinterpret_cast<TileMeta*>(ws + ly.meta);
+    int64_t* seg_first = reinterpret_cast<int64_t*>(ws + ly.seg_first);
+    uint32_t* hdr = reinterpret_cast<uint32_t*>(ws);
+    const memoroid_status_t st = launch_prep(a, pl, meta, seg_first, stream);
+    if (st != MEMOROID_OK) return st;
 
     FwdParams p;
     p.q = static_cast<const uint16_t*>(a.q);
@@ -690,20 +1351,110 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     p.tps = pl.tps;
     p.G = static_cast<int>(pl.G);
     p.wait_ns = debug_knobs().wait_ns;
-    if (set_smem(fwd_kernel<D>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    fwd_kernel<D><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(p);
+    p.zq = nullptr;
+    p.dlam_f = nullptr;
+    p.states = nullptr;
+    if (set_smem(fwd_kernel<D, false>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    fwd_kernel<D, false><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    return MEMOROID_OK;
+}
+template <int D>
+memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, cudaStream_t stream) {
+    unsigned char* ws = static_cast<unsigned char*>(a.workspace);
+    TileMeta* meta = reinterpret_cast<TileMeta*>(ws + ly.meta);
+    int64_t* seg_first = reinterpret_cast<int64_t*>(ws + ly.seg_first);
+    uint16_t* dy16 = reinterpret_cast<uint16_t*>(ws + ly.dy16);
+    uint16_t* states = reinterpret_cast<uint16_t*>(ws + ly.states);
+    float* dlam_f = reinterpret_cast<float*>(ws + ly.dlam_f);
+    float* gpart = reinterpret_cast<float*>(ws + ly.gpart);
+    uint32_t* hdr = reinterpret_cast<uint32_t*>(ws);
+    memoroid_status_t st = launch_prep(a, pl, meta, seg_first, stream);
+    if (st != MEMOROID_OK) return st;
+
+    const int64_t n8 = a.B * a.L * a.H * D / 8;
+    const int64_t cblocks = min((n8 + 255) / 256, static_cast<int64_t>(kTargetCtas) * 16);
+    to_bf16_kernel<<<static_cast<unsigned>(cblocks), 256, 0, stream>>>(a.grad_y, dy16, n8);
+    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+
+    // pass F: dq = S dy, with (q, k, v) -> (dy, v, k)
+    FwdParams f;
+    f.q = dy16;
+    f.k = static_cast<const uint16_t*>(a.v);
+    f.v = static_cast<const uint16_t*>(a.k);
+    f.S0 = a.S0;
+    f.y = a.dq;
+    f.meta = meta;
+    f.seg_first = seg_first;
+    f.S_last = nullptr;
+    f.hdr = hdr;
+    f.B = a.B;
+    f.L = a.L;
+    f.H = a.H;
+    f.n_tiles = pl.n_tiles;
+    f.tps = pl.tps;
+    f.G = static_cast<int>(pl.G);
+    f.wait_ns = debug_knobs().wait_ns;
+    f.zq = static_cast<const uint16_t*>(a.q);
+    f.dlam_f = dlam_f;
+    f.states = states;
+    if (set_smem(fwd_kernel<D, true>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    fwd_kernel<D, true><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
+    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+
+    // pass R: dk, dv, dgamma, dS0
+    BwdParams r;
+    r.q = static_cast<const uint16_t*>(a.q);
+    r.k = static_cast<const uint16_t*>(a.k);
+    r.v = static_cast<const uint16_t*>(a.v);
+    r.dy = dy16;
+    r.gamma = a.gamma;
+    r.gamma_per_step = a.gamma_per_step;
+    r.dS_last = a.dS_last;
+    r.dk = a.dk;
+    r.dv = a.dv;
+    r.dgamma = (a.dgamma != nullptr && a.gamma_per_step) ? a.dgamma : nullptr;
+    r.gpart = (a.dgamma != nullptr && !a.gamma_per_step) ? gpart : nullptr;
+    r.dS0 = a.dS0;
+    r.meta = meta;
+    r.seg_first = seg_first;
+    r.dlam_f = dlam_f;
+    r.states = states;
+    r.hdr = hdr;
+    r.B = a.B;
+    r.L = a.L;
+    r.H = a.H;
+    r.n_tiles = pl.n_tiles;
+    r.G = static_cast<int>(pl.G);
+    r.wait_ns = debug_knobs().wait_ns;
+    if (set_smem(bwd_kernel<D>, BwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    bwd_kernel<D><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, BwdSmem<D>::BYTES, stream>>>(r);
+    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    if (r.gpart != nullptr) {
+        dgamma_head_kernel<<<static_cast<unsigned>((a.H + 127) / 128), 128, 0, stream>>>(gpart, a.gamma, a.dgamma,
+                                                                                          a.B, a.H, static_cast<int>(pl.G));
+        if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    }
     return MEMOROID_OK;
 }
 }  // namespace
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D) { return make_layout(B, L, H, D).total; }
+size_t fwd_workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D) { return make_layout(B, L, H, D).fwd_total; }
 
-int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_S_last) {
-    (void)backward;
-    (void)with_S_last;
+int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_dgamma_per_head) {
     if (B == 0 || L == 0 || H == 0) return 0;
-    return 3;
+    if (!backward) return 3;
+    return 6 + (with_dgamma_per_head ? 1 : 0);
+}
+
+memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream) {
+    if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, stream) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    const Plan pl = make_plan(a.B, a.L, a.H);
+    const Layout ly = make_layout(a.B, a.L, a.H, a.D);
+    if (a.D == 64) return launch_bwd_d<64>(a, pl, ly, stream);
+    if (a.D == 128) return launch_bwd_d<128>(a, pl, ly, stream);
+    return MEMOROID_ERR_UNSUPPORTED;
 }
 
 memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream) {

@@ -50,6 +50,8 @@ SIGNATURES = {
     "memoroid_scan_linattn_kernels_per_call": (_int, [_i64, _i64, _i64, _i64, _i64, _int, _int]),
     "memoroid_scan_linattn_fwd": (_int, [_p, _p, _p, _int, _p, _int, _p, _p, _p, _p, _i64, _i64, _i64,
                                          _i64, _i64, _i64, _p, _sz, _p]),
+    "memoroid_scan_linattn_bwd": (_int, [_p, _p, _p, _int, _p, _int, _p, _p, _p, _p, _p, _p, _p, _p, _p, _i64,
+                                         _i64, _i64, _i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_starts_from_offsets": (_int, [_p, _i64, _i64, _p, _p]),
     "memoroid_offsets_workspace_bytes": (_sz, [_i64]),
     "memoroid_offsets_from_starts": (_int, [_p, _i64, _p, _p, _p, _sz, _p]),
@@ -162,8 +164,9 @@ def memoroid_scan_linattn_workspace_bytes(B, L, H, dk, dv, chunk) -> int:
     return int(load().memoroid_scan_linattn_workspace_bytes(B, L, H, dk, dv, chunk))
 
 
-def memoroid_scan_linattn_kernels_per_call(B, L, H, dk, dv, backward, with_S_last) -> int:
-    return int(load().memoroid_scan_linattn_kernels_per_call(B, L, H, dk, dv, int(backward), int(with_S_last)))
+def memoroid_scan_linattn_kernels_per_call(B, L, H, dk, dv, backward, with_dgamma_per_head) -> int:
+    return int(load().memoroid_scan_linattn_kernels_per_call(B, L, H, dk, dv, int(backward),
+                                                             int(with_dgamma_per_head)))
 
 
 def memoroid_scan_linattn_fwd(q, k, v, in_dtype, gamma, gamma_per_step, start, S0, y, S_last, B, L, H, dk, dv,
@@ -174,6 +177,17 @@ def memoroid_scan_linattn_fwd(q, k, v, in_dtype, gamma, gamma_per_step, start, S
                                           B, L, H, dk, dv, chunk, _ptr(workspace),
                                           workspace.numel() if workspace is not None else 0, _stream(stream))
     _check(st, "memoroid_scan_linattn_fwd")
+
+
+def memoroid_scan_linattn_bwd(q, k, v, in_dtype, gamma, gamma_per_step, start, S0, grad_y, grad_S_last, dq, dk_out,
+                              dv_out, dgamma, dS0, B, L, H, dk, dv, chunk, workspace, stream=None):
+    _need_cuda(q, k, v, gamma, start, S0, grad_y, grad_S_last, dq, dk_out, dv_out, dgamma, dS0, workspace)
+    st = load().memoroid_scan_linattn_bwd(_ptr(q), _ptr(k), _ptr(v), int(in_dtype), _ptr(gamma), int(gamma_per_step),
+                                          _ptr(start), _ptr(S0), _ptr(grad_y), _ptr(grad_S_last), _ptr(dq),
+                                          _ptr(dk_out), _ptr(dv_out), _ptr(dgamma), _ptr(dS0), B, L, H, dk, dv, chunk,
+                                          _ptr(workspace), workspace.numel() if workspace is not None else 0,
+                                          _stream(stream))
+    _check(st, "memoroid_scan_linattn_bwd")
 
 
 def memoroid_starts_from_offsets(offsets, E, L, start, stream=None):
@@ -263,6 +277,23 @@ def linattn_fwd(q, k, v, gamma, start, S0=None, want_last=True, chunk=64, ws=Non
     memoroid_scan_linattn_fwd(q, k, v, MEMOROID_BF16, gamma, per_step, start, S0, y, S_last, B, L, H, d, d, chunk,
                               ws, stream)
     return y, S_last
+
+
+def linattn_bwd(q, k, v, gamma, start, grad_y, grad_S_last=None, S0=None, want_gamma=True, want_S0=False, chunk=64,
+                ws=None, stream=None):
+    """dq, dk, dv, dgamma, dS0 of the decayed linear-attention memoroid."""
+    B, L, H, d = q.shape
+    per_step = gamma.dim() == 3
+    if ws is None:
+        ws = linattn_workspace(B, L, H, d, q.device, chunk)
+    dq = torch.empty((B, L, H, d), dtype=torch.float32, device=q.device)
+    dk = torch.empty_like(dq)
+    dv = torch.empty_like(dq)
+    dgamma = torch.empty_like(gamma) if want_gamma else None
+    dS0 = torch.empty((B, H, d, d), dtype=torch.float32, device=q.device) if want_S0 else None
+    memoroid_scan_linattn_bwd(q, k, v, MEMOROID_BF16, gamma, per_step, start, S0, grad_y, grad_S_last, dq, dk, dv,
+                              dgamma, dS0, B, L, H, d, d, chunk, ws, stream)
+    return dq, dk, dv, dgamma, dS0
 
 
 def starts_from_offsets(offsets, L, stream=None):

@@ -1,5 +1,5 @@
-"""GPU parity of the decayed linear-attention memoroid (forward) against the
-fp64 oracle, through the C ABI.
+"""GPU parity of the decayed linear-attention memoroid (forward and backward)
+against the fp64 oracle, through the C ABI.
 
 Bar: max |gpu - ref| / max |ref| <= 2e-2 for every output (bf16 q, k, v;
 the oracle takes the same bf16 values upcast, so only the arithmetic counts).
@@ -162,3 +162,77 @@ def test_fwd_config3_sampled_episodes():
         y_ref, _ = run_oracle_fwd(sub)
         worst = max(worst, rel_err(y[:, s:e], y_ref))
     assert worst <= TOL
+
+
+# ---------------------------------------------------------------------------
+# backward
+# ---------------------------------------------------------------------------
+
+def run_gpu_bwd(t, S0=None, dS_last=None, chunk=64):
+    m = _m()
+    q, k, v = bits_dev(t["q"]), bits_dev(t["k"]), bits_dev(t["v"])
+    gamma, start = dev(t["gamma"]), dev(t["start"])
+    B, L, H, d = t["q"].shape
+    ws = m.linattn_workspace(B, L, H, d, "cuda", chunk)
+    out = m.linattn_bwd(q, k, v, gamma, start, dev(t["grad_y"]), dev(dS_last), dev(S0), want_S0=True, chunk=chunk,
+                        ws=ws)
+    assert m.memoroid_get_device_error(ws) == m.MEMOROID_OK
+    torch.cuda.synchronize()
+    return [o.cpu().numpy() for o in out]
+
+
+def run_oracle_bwd(t, S0=None, dS_last=None):
+    f = oracle.bf16_bits_to_f64
+    return oracle.linattn_bwd(f(t["q"]), f(t["k"]), f(t["v"]), t["gamma"], t["start"], t["grad_y"], dS_last, S0)
+
+
+def check_bwd(t, S0=None, dS_last=None):
+    got = run_gpu_bwd(t, S0, dS_last)
+    ref = run_oracle_bwd(t, S0, dS_last)
+    errs = {name: rel_err(g, r) for name, g, r in zip(("dq", "dk", "dv", "dgamma", "dS0"), got, ref)}
+    assert all(e <= TOL for e in errs.values()), errs
+    return errs
+
+
+BWD_CASES = [
+    # B, L, H, d, gamma_mode, mean, with_S0, with_dS_last
+    (2, 1000, 3, 64, "head", 60.0, False, False),
+    (2, 1000, 3, 128, "step", 60.0, True, True),
+    (1, 3000, 2, 64, "step", 400.0, True, True),
+    (1, 3000, 1, 128, "head", 2000.0, False, True),
+    (3, 777, 2, 128, "head", 30.0, True, False),
+]
+
+
+@pytest.mark.parametrize("B,L,H,d,gm,mean,with_S0,with_dS", BWD_CASES)
+def test_bwd_matches_oracle(B, L, H, d, gm, mean, with_S0, with_dS):
+    t = tapegen.linattn_tape(B, L, H, d, d, seed=tapegen.seed_for(300 + L + d + H), mean=mean, gamma_mode=gm,
+                             gammas=(0.95, 0.99, 1.0), with_grad=True, with_S0=with_S0)
+    S0 = t.get("S0")
+    if S0 is not None:
+        t["start"][:, 0] = 0
+    check_bwd(t, S0, t["grad_S_last"] if with_dS else None)
+
+
+@pytest.mark.parametrize("mode", ["all", "none", "open"])
+@pytest.mark.parametrize("d", [64, 128])
+def test_bwd_degenerate_resets(mode, d):
+    t = tapegen.linattn_tape(2, 700, 2, d, d, seed=tapegen.seed_for(17 + d), gamma_mode="step", with_grad=True,
+                             with_S0=True, start_mode=mode)
+    check_bwd(t, t["S0"], t["grad_S_last"])
+
+
+@pytest.mark.parametrize("L", [1, 5, 127, 128, 129, 300])
+def test_bwd_short_tapes(L):
+    t = tapegen.linattn_tape(1, L, 2, 64, 64, seed=tapegen.seed_for(950 + L), mean=40.0, gamma_mode="step",
+                             with_grad=True, with_S0=True)
+    t["start"][:, 0] = 0
+    check_bwd(t, t["S0"], t["grad_S_last"])
+
+
+def test_bwd_deterministic():
+    t = tapegen.linattn_tape(1, 5000, 2, 128, 128, seed=tapegen.seed_for(59), mean=500.0, gamma_mode="head",
+                             with_grad=True)
+    a = run_gpu_bwd(t)
+    b = run_gpu_bwd(t)
+    assert all(np.array_equal(x, y) for x, y in zip(a, b))
