@@ -236,3 +236,45 @@ def test_bwd_deterministic():
     a = run_gpu_bwd(t)
     b = run_gpu_bwd(t)
     assert all(np.array_equal(x, y) for x, y in zip(a, b))
+
+
+def test_bwd_config3_full():
+    # the full L = 2^18, 4-head, d = 64 tape with per-head gamma, every output
+    t = tapegen.linattn_config(3)
+    t["grad_y"] = np.random.default_rng(tapegen.seed_for(3) + 1).standard_normal(t["q"].shape, dtype=np.float32)
+    errs = check_bwd(t)
+    assert errs["dgamma"] <= TOL
+
+
+def _episode_slices(start_row, rng, n):
+    starts = np.flatnonzero(start_row)
+    picks = rng.choice(len(starts) - 1, size=n, replace=False)
+    return [(int(starts[i]), int(starts[i + 1])) for i in sorted(picks)]
+
+
+def test_config5_sampled_episodes():
+    # L = 2^22, 8 heads, d = 128, per-step gamma, drawn on the device.  Whole
+    # episodes (not the tape's first or last) depend on nothing outside
+    # themselves, so the oracle checks them one at a time.
+    m = _m()
+    c = tapegen.LINATTN_CONFIGS[5]
+    B, L, H, d = c["B"], c["L"], c["H"], c["d"]
+    t = tapegen.linattn_tape_device(B, L, H, d, tapegen.seed_for(5), c["mean"], c["gamma"], with_grad=True)
+    ws = m.linattn_workspace(B, L, H, d, "cuda")
+    y, _ = m.linattn_fwd(t["q"], t["k"], t["v"], t["gamma"], t["start"], None, want_last=False, ws=ws)
+    dq, dk, dv, dg, _ = m.linattn_bwd(t["q"], t["k"], t["v"], t["gamma"], t["start"], t["grad_y"], ws=ws)
+    assert m.memoroid_get_device_error(ws) == m.MEMOROID_OK
+    torch.cuda.synchronize()
+    start = t["start"].cpu().numpy()
+    worst = {}
+    for s, e in _episode_slices(start[0], np.random.default_rng(5), 6):
+        sl = slice(s, e)
+        sub = dict(q=t["q"][:, sl].cpu().numpy().view(np.uint16), k=t["k"][:, sl].cpu().numpy().view(np.uint16),
+                   v=t["v"][:, sl].cpu().numpy().view(np.uint16), gamma=t["gamma"][:, sl].cpu().numpy(),
+                   start=start[:, sl], grad_y=t["grad_y"][:, sl].cpu().numpy())
+        y_ref, _ = run_oracle_fwd(sub)
+        rq, rk, rv, rg, _ = run_oracle_bwd(sub)
+        for name, got, ref in (("y", y[:, sl], y_ref), ("dq", dq[:, sl], rq), ("dk", dk[:, sl], rk),
+                               ("dv", dv[:, sl], rv), ("dgamma", dg[:, sl], rg)):
+            worst[name] = max(worst.get(name, 0.0), rel_err(got.cpu().numpy(), ref))
+    assert all(v <= TOL for v in worst.values()), worst
