@@ -4,7 +4,11 @@ Geometric(500) episodes clipped to [1, 10000] (the tape-based batch of
 Section 4.1 at GPU scale).
 
 One step = memoroid_scan_diag_fwd + memoroid_scan_diag_bwd (with grad_lambda)
-over the whole tape.  Prints one JSON line.
+over the whole tape.  Prints one JSON line.  Its "linattn" object times the
+decayed linear-attention memoroid on the largest linattn tape (L = 2^22,
+8 heads, d = 128, per-step gamma, Geometric(1000) episodes): one step =
+memoroid_scan_linattn_fwd + memoroid_scan_linattn_bwd, plus the tensor-core
+throughput of the intra-tile contraction alone (memoroid_bench_linattn_intra).
 
   python bench.py [--gpus N --steps K --warmup W] [--impl reference]
 
@@ -42,6 +46,9 @@ WORKLOAD = ("diag scan fwd+bwd (grad_u, grad_lambda): B=1 tape, L=2^20 steps, D=
 FWD_BYTES_PER_STEP_CH = 16
 BWD_BYTES_PER_STEP_CH = 24
 PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "diag_scan_traffic_L1M_D256.md")
+LA_CFG = 5
+LA_WORKLOAD = ("linattn fwd+bwd (dq, dk, dv, per-step dgamma): B=1 tape, L=2^22 steps, H=8 heads, d_k=d_v=128, "
+               "bf16 q/k/v, per-step gamma=sigmoid(N(3,1)), Geometric(1000) episodes")
 KERNEL_SRC = os.path.join(ROOT, "paper_2402_09900_gb300", "csrc", "diag_scan.cu")
 
 
@@ -60,6 +67,107 @@ def _peaks():
         return float(d["hbm_gbs"]), "measured"
     except Exception:
         return 6800.0, "fallback"
+
+
+def _tensor_peaks():
+    """(bf16 burst TFLOP/s, sustained TFLOP/s, kind)."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 1900.0, 1700.0, "fallback"
+
+
+def linattn_leg(args, m, dev, stream):
+    """Times the linear-attention memoroid (fwd + bwd) on the L = 2^22, 8-head,
+    d = 128 tape, and the intra-tile contraction alone."""
+    import torch
+
+    c = tapegen.LINATTN_CONFIGS[LA_CFG]
+    B, L, H, d = c["B"], c["L"], c["H"], c["d"]
+    t = tapegen.linattn_tape_device(B, L, H, d, tapegen.seed_for(LA_CFG), c["mean"], c["gamma"], device=dev)
+    per = 1 if t["gamma"].dim() == 3 else 0
+    ws = m.linattn_workspace(B, L, H, d, dev)
+    y = torch.empty((B, L, H, d), dtype=torch.float32, device=dev)
+    dq, dk, dv = torch.empty_like(y), torch.empty_like(y), torch.empty_like(y)
+    dg = torch.empty_like(t["gamma"])
+
+    def fwd():
+        m.memoroid_scan_linattn_fwd(t["q"], t["k"], t["v"], m.MEMOROID_BF16, t["gamma"], per, t["start"], None, y,
+                                    None, B, L, H, d, d, c["chunk"], ws, stream)
+
+    def bwd():
+        m.memoroid_scan_linattn_bwd(t["q"], t["k"], t["v"], m.MEMOROID_BF16, t["gamma"], per, t["start"], None,
+                                    t["grad_y"], None, dq, dk, dv, dg, None, B, L, H, d, d, c["chunk"], ws, stream)
+
+    for _ in range(3):
+        fwd()
+        bwd()
+    torch.cuda.synchronize()
+    if m.memoroid_get_device_error(ws) != m.MEMOROID_OK:
+        raise RuntimeError("device-side error in the linattn warm-up")
+    steps = args.la_steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for i in range(steps):
+        evs[i][0].record(stream)
+        fwd()
+        evs[i][1].record(stream)
+        bwd()
+        evs[i][2].record(stream)
+    torch.cuda.synchronize()
+    if m.memoroid_get_device_error(ws) != m.MEMOROID_OK:
+        raise RuntimeError("device-side error in the linattn timed region")
+    f_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / steps
+    b_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / steps
+    el = B * L * H * d
+    # algorithmic bytes: fwd reads q, k, v (bf16), gamma, start and writes y (fp32);
+    # bwd reads q, k, v, gamma, start, dy and writes dq, dk, dv, dgamma
+    fb = el * (3 * 2 + 4) + t["gamma"].numel() * 4 + B * L
+    bb = el * (3 * 2 + 4 + 3 * 4) + t["gamma"].numel() * 8 + B * L
+    peak, peak_kind = _peaks()
+    kpc = (m.memoroid_scan_linattn_kernels_per_call(B, L, H, d, d, 0, 0)
+           + m.memoroid_scan_linattn_kernels_per_call(B, L, H, d, d, 1, 0))
+
+    # the intra-tile contraction alone, operands resident in shared memory
+    scratch = m.workspace(m.memoroid_bench_linattn_intra_scratch_bytes(d), dev)
+    scratch.random_(0, 256)
+    reps, ctas = args.la_intra_reps, 152
+    m.memoroid_bench_linattn_intra(d, reps, ctas, scratch, stream)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    m.memoroid_bench_linattn_intra(d, reps, ctas, scratch, stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if m.memoroid_get_device_error(scratch) != m.MEMOROID_OK:
+        raise RuntimeError("device-side error in the intra-tile benchmark")
+    i_ms = e0.elapsed_time(e1)
+    i_tf = ctas * reps * 4 * 128 * 128 * d / (i_ms * 1e-3) / 1e12
+    burst, sustained, tkind = _tensor_peaks()
+    out = {
+        "workload": LA_WORKLOAD, "value": B * L / ((f_ms + b_ms) * 1e-3), "unit": UNIT, "steps": steps,
+        "ms_per_step": f_ms + b_ms, "fwd_ms": f_ms, "bwd_ms": b_ms,
+        "episodes": int(t["start"].sum().item()),
+        "roofline": {"bound": "hbm", "peak": peak, "unit": "GB/s", "peak_kind": f"{peak_kind} (copy bandwidth)",
+                     "fwd": {"algorithmic_bytes_per_call": fb, "achieved": fb / (f_ms * 1e-3) / 1e9,
+                             "frac": fb / (f_ms * 1e-3) / 1e9 / peak},
+                     "bwd": {"algorithmic_bytes_per_call": bb, "achieved": bb / (b_ms * 1e-3) / 1e9,
+                             "frac": bb / (b_ms * 1e-3) / 1e9 / peak},
+                     "step_frac": (fb + bb) / ((f_ms + b_ms) * 1e-3) / 1e9 / peak},
+        "intra_chunk_tensor": {"bound": "tensor", "achieved": i_tf, "unit": "TFLOP/s", "peak": burst,
+                               "frac": i_tf / burst, "frac_of_sustained": i_tf / sustained,
+                               "peak_kind": f"{tkind} bf16 dense (burst; sustained {sustained})",
+                               "ms": i_ms, "ctas": ctas, "reps": reps,
+                               "flops": ctas * reps * 4 * 128 * 128 * d,
+                               "what": "P = Q K^T (128x128x128) and Y = Pm V (128x128x128) per rep, tcgen05 "
+                                       "kind::f16 bf16->fp32, operands resident in shared memory"},
+        "gpu_launches": steps * kpc + 2,
+    }
+    del t, y, dq, dk, dv, ws
+    torch.cuda.empty_cache()
+    return out
 
 
 def _traffic_record():
@@ -353,6 +461,9 @@ def run_ours(args):
                 "fwd": {"achieved": fwd_gbs, "frac": fwd_gbs / peak, "avg_launch_ms": fwd_avg,
                         "algorithmic_bytes_per_launch": fwd_bytes},
                 "step_frac": (fwd_bytes + bwd_bytes) / (ms_per_step * 1e-3) / 1e9 / peak}
+    la = None
+    if ws == 1 and not args.skip_linattn:
+        la = linattn_leg(args, m, dev, stream)
     cpu = None
     if ws == 1 and not args.skip_cpu_baseline:
         cpu = cpu_baseline(t, args.cpu_seconds)
@@ -367,6 +478,7 @@ def run_ours(args):
         "gpu_launches": args.steps * (m.memoroid_scan_diag_kernels_per_call(B, L, D, 0, 0, 0)
                                       + m.memoroid_scan_diag_kernels_per_call(B, L, D, 0, 1, 1)),
         "clocks": clocks,
+        "linattn": la,
     }
     print(json.dumps(out), flush=True)
     if ws > 1:
@@ -385,6 +497,10 @@ def main():
     ap.add_argument("--ref-seconds", type=float, default=90.0,
                     help="approximate total oracle time of the --impl reference steps")
     ap.add_argument("--skip-cpu-baseline", action="store_true")
+    ap.add_argument("--skip-linattn", action="store_true", help="omit the linear-attention leg")
+    ap.add_argument("--la-steps", type=int, default=10, help="timed linattn fwd+bwd steps")
+    ap.add_argument("--la-intra-reps", type=int, default=2000,
+                    help="repetitions of the intra-tile contraction per CTA in the tensor benchmark")
     ap.add_argument("--tape-steps", type=int, default=0,
                     help="use only the first N steps of the tape (profiler captures); 0 = full workload")
     args = ap.parse_args()

@@ -216,6 +216,26 @@ memoroid_status_t memoroid_scan_linattn_bwd(const void *q, const void *k, const 
                                             int64_t dv, int64_t chunk, void *workspace,
                                             size_t workspace_bytes, void *stream);
 
+/* ------------------------------------------------------------------------ */
+/* Measurement only (the paper has no counterpart): throughput of the        */
+/* intra-tile tensor-core contraction of memoroid_scan_linattn_fwd alone.    */
+/* ------------------------------------------------------------------------ */
+
+/* Scratch bytes for memoroid_bench_linattn_intra (0 if d is unsupported). */
+size_t memoroid_bench_linattn_intra_scratch_bytes(int64_t d);
+
+/*
+ * Launches `ctas` CTAs; each stages one set of operand tiles taken from the
+ * scratch bytes (their values are irrelevant) in shared memory and then
+ * issues `reps` times the forward pass's two intra-tile contractions,
+ * P = Q K^T (128 x 128 x d) and Y = Pm V (128 x d x 128), with the same
+ * instruction shapes and operand layouts.  Executed flops: 4 * 128^2 * d per
+ * rep and CTA.  Time it with events on `stream`.  scratch: device memory,
+ * 256-byte aligned, at least memoroid_bench_linattn_intra_scratch_bytes(d).
+ */
+memoroid_status_t memoroid_bench_linattn_intra(int64_t d, int64_t reps, int64_t ctas, void *scratch,
+                                               size_t scratch_bytes, void *stream);
+
 /* ======================================================================== */
 /* Episode index list <-> begin flags (Algorithm 1 keeps I = where(b)).     */
 /* ======================================================================== */

@@ -343,4 +343,18 @@ memoroid_status_t memoroid_scan_linattn_bwd(const void* q, const void* k, const 
     return la::launch_bwd(a, s);
 }
 
+size_t memoroid_bench_linattn_intra_scratch_bytes(int64_t d) {
+    if (d != 64 && d != 128) return 0;
+    return la::intra_bench_scratch_bytes(d);
+}
+
+memoroid_status_t memoroid_bench_linattn_intra(int64_t d, int64_t reps, int64_t ctas, void* scratch,
+                                               size_t scratch_bytes, void* stream) {
+    if (d != 64 && d != 128) return MEMOROID_ERR_UNSUPPORTED;
+    if (reps < 1 || ctas < 1 || ctas > (1 << 20)) return MEMOROID_ERR_INVALID_ARG;
+    if (scratch == nullptr || !aligned(scratch, 256) || scratch_bytes < la::intra_bench_scratch_bytes(d))
+        return MEMOROID_ERR_WORKSPACE;
+    return la::launch_intra_bench(d, reps, ctas, scratch, as_stream(stream));
+}
+
 }  // extern "C"

@@ -95,6 +95,8 @@ size_t fwd_workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D);  // forw
 int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_dgamma_per_head);
 memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream);
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream);
+size_t intra_bench_scratch_bytes(int64_t D);
+memoroid_status_t launch_intra_bench(int64_t D, int64_t reps, int64_t ctas, void* scratch, cudaStream_t stream);
 
 }  // namespace la
 

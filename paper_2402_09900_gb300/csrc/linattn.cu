@@ -1303,6 +1303,101 @@ __global__ void dgamma_head_kernel(const float* __restrict__ gpart, const float*
 }
 
 // ---------------------------------------------------------------------------
+// measurement: the intra-tile contraction alone, operands resident in smem
+// ---------------------------------------------------------------------------
+// Each CTA stages one Q, K, V tile and one masked-score tile (any bits; the
+// values do not matter) and then issues `reps` times the two intra-tile
+// contractions of the forward pass, P = Q K^T and Y = Pm V, with the same
+// descriptors and instruction shapes as fwd_kernel, accumulating in TMEM.
+// Executed flops per rep: 4 * T * T * D.  No HBM traffic after the staging.
+template <int D>
+__global__ void __launch_bounds__(128, 1) intra_bench_kernel(const uint4* __restrict__ src, int reps,
+                                                            float* __restrict__ sink, uint32_t* hdr, uint64_t wait_ns) {
+    constexpr int TILE = T * D * 2, PM = T * T * 2;
+    extern __shared__ __align__(1024) unsigned char smem[];
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ uint32_t tslot;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int total16 = (3 * TILE + PM) / 16;
+    for (int i = tid; i < total16; i += blockDim.x) {
+        uint4 u = src[i];
+        // keep the values finite and moderate: clear the exponent's top bits
+        u.x &= 0x3fff3fffu;
+        u.y &= 0x3fff3fffu;
+        u.z &= 0x3fff3fffu;
+        u.w &= 0x3fff3fffu;
+        reinterpret_cast<uint4*>(smem)[i] = u;
+    }
+    if (tid == 0) {
+        mbar_init(&bar, 1);
+        fence_mbar_init();
+    }
+    if (warp == 0) tc::alloc(&tslot, 256);
+    tc::fence_smem_to_async();
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    const uint32_t tm = tslot;
+    const uint32_t sq = smem_addr(smem), sk = sq + TILE, sv = sq + 2 * TILE, spm = sq + 3 * TILE;
+    constexpr uint32_t ID_QK = tc::idesc_bf16(128, T, false, false);
+    constexpr uint32_t ID_PV = tc::idesc_bf16(128, D, false, true);
+    if (tid == 0) {
+        for (int r = 0; r < reps; ++r) {
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk)
+                tc::mma(tm, desc_kmajor(sq, D, kk), desc_kmajor(sk, D, kk), ID_QK, r > 0 || kk > 0);
+#pragma unroll
+            for (int kk = 0; kk < T / 16; ++kk)
+                tc::mma(tm + 128, desc_kmajor(spm, T, kk), desc_mnmajor(sv, D, kk), ID_PV, r > 0 || kk > 0);
+        }
+        tc::commit(&bar);
+    }
+    const bool ok = wait_mbar(&bar, 0, wait_ns);
+    tc::fence_after();
+    if (!ok && tid == 0) record_error(hdr, DEV_MMA_TIMEOUT);
+    if (ok) {
+        float v[16];
+        tc::ld16(tm + (static_cast<uint32_t>(32 * warp) << 16), v);
+        if (tid == 0) sink[blockIdx.x] = v[0];
+    }
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    if (warp == 0) tc::dealloc(tm, 256);
+}
+
+size_t intra_bench_scratch_bytes(int64_t D) {
+    return kHeaderBytes + static_cast<size_t>(3 * T * D * 2 + T * T * 2) + 4096 * sizeof(float);
+}
+
+memoroid_status_t launch_intra_bench(int64_t D, int64_t reps, int64_t ctas, void* scratch, cudaStream_t stream) {
+    unsigned char* ws = static_cast<unsigned char*>(scratch);
+    uint32_t* hdr = reinterpret_cast<uint32_t*>(ws);
+    const uint4* src = reinterpret_cast<const uint4*>(ws + kHeaderBytes);
+    float* sink = reinterpret_cast<float*>(ws + kHeaderBytes + 3 * T * D * 2 + T * T * 2);
+    const uint64_t wait_ns = debug_knobs().wait_ns;
+    if (cudaMemsetAsync(scratch, 0, kHeaderBytes, stream) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    if (D == 64) {
+        const int bytes = 3 * T * 64 * 2 + T * T * 2;
+        if (cudaFuncSetAttribute(intra_bench_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) !=
+            cudaSuccess)
+            return MEMOROID_ERR_CUDA;
+        intra_bench_kernel<64><<<static_cast<unsigned>(ctas), 128, bytes, stream>>>(src, static_cast<int>(reps), sink,
+                                                                                    hdr, wait_ns);
+    } else if (D == 128) {
+        const int bytes = 3 * T * 128 * 2 + T * T * 2;
+        if (cudaFuncSetAttribute(intra_bench_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) !=
+            cudaSuccess)
+            return MEMOROID_ERR_CUDA;
+        intra_bench_kernel<128><<<static_cast<unsigned>(ctas), 128, bytes, stream>>>(src, static_cast<int>(reps), sink,
+                                                                                     hdr, wait_ns);
+    } else {
+        return MEMOROID_ERR_UNSUPPORTED;
+    }
+    return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 namespace {

@@ -52,6 +52,8 @@ SIGNATURES = {
                                          _i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_scan_linattn_bwd": (_int, [_p, _p, _p, _int, _p, _int, _p, _p, _p, _p, _p, _p, _p, _p, _p, _i64,
                                          _i64, _i64, _i64, _i64, _i64, _p, _sz, _p]),
+    "memoroid_bench_linattn_intra_scratch_bytes": (_sz, [_i64]),
+    "memoroid_bench_linattn_intra": (_int, [_i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_starts_from_offsets": (_int, [_p, _i64, _i64, _p, _p]),
     "memoroid_offsets_workspace_bytes": (_sz, [_i64]),
     "memoroid_offsets_from_starts": (_int, [_p, _i64, _p, _p, _p, _sz, _p]),
@@ -188,6 +190,16 @@ def memoroid_scan_linattn_bwd(q, k, v, in_dtype, gamma, gamma_per_step, start, S
                                           _ptr(workspace), workspace.numel() if workspace is not None else 0,
                                           _stream(stream))
     _check(st, "memoroid_scan_linattn_bwd")
+
+
+def memoroid_bench_linattn_intra_scratch_bytes(d) -> int:
+    return int(load().memoroid_bench_linattn_intra_scratch_bytes(d))
+
+
+def memoroid_bench_linattn_intra(d, reps, ctas, scratch, stream=None):
+    _need_cuda(scratch)
+    _check(load().memoroid_bench_linattn_intra(d, reps, ctas, _ptr(scratch), scratch.numel(), _stream(stream)),
+           "memoroid_bench_linattn_intra")
 
 
 def memoroid_starts_from_offsets(offsets, E, L, start, stream=None):
