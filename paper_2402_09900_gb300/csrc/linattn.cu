@@ -20,8 +20,11 @@
 // pass is needed.  Each CTA owns one (tape, head, segment) and walks its tiles
 // in order, carrying the state in TMEM.  A nominal segment without any begin
 // flag is absorbed by the segment before it.
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
+
+#include <mutex>
 
 #include <cstdint>
 
@@ -239,29 +242,38 @@ __device__ __forceinline__ float2 unpack_bf16x2(uint32_t w) {
     return __bfloat1622float2(v);
 }
 
-// Copies rows [0, nvalid) of a [T x D] bf16 tile (row r at src + r * row_stride
-// elements) into the core-matrix layout with 16-byte cp.async; rows past
-// nvalid are zero-filled.  32 consecutive chunks of a warp cover 8 rows x 4
-// chunks: 64 contiguous global bytes per row, conflict-free shared stores.
-template <int D>
-__device__ __forceinline__ void load_tile_async(uint32_t dst, const uint16_t* __restrict__ src, int64_t row_stride,
-                                                int nvalid, int tid) {
-    constexpr int CPR = D / 8;
-    constexpr int NCH = T * CPR;
-#pragma unroll
-    for (int e = tid; e < NCH; e += kThreads) {
-        const int blk = e >> 5, ln = e & 31;
-        const int rg = blk / (CPR / 4), cq = blk % (CPR / 4);
-        const int r = rg * 8 + (ln & 7), c = cq * 4 + (ln >> 3);
-        const bool ok = r < nvalid;
-        const uint16_t* s = src + (ok ? static_cast<int64_t>(r) * row_stride + c * 8 : 0);
-        cp_async16(dst + rg * (D * 16) + c * 128 + (ln & 7) * 16, s, ok);
-    }
+// Operand tiles of T steps x D channels are loaded by TMA with 128-byte
+// swizzling: one box per 64 channels ("chunk", T rows of 128 bytes, chunk m at
+// m * T * 128), and within a chunk the 16-byte unit u of row r stored at unit
+// u ^ (r % 8):
+//   byte(row, col) = (col / 64) * T * 128 + row * 128 + (((col % 64) / 8) ^ (row % 8)) * 16 + (col % 8) * 2.
+// Read with rows as M/N and cols as K (K-major): SBO = 1024 (8-row groups),
+// the K step of 16 moves the start by 32 bytes inside a chunk.  Read with cols
+// as M/N and rows as K (MN-major): LBO = T * 128 (the next 64 columns), SBO =
+// 1024, K step of 16 rows = +2048 bytes.  Chunks are 1024-byte aligned.
+__device__ __forceinline__ uint32_t sw_off(int row, int col) {
+    return static_cast<uint32_t>((col >> 6) * (T * 128) + row * 128 + ((((col & 63) >> 3) ^ (row & 7)) << 4) +
+                                 (col & 7) * 2);
+}
+__device__ __forceinline__ uint64_t sw_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+    return tc::smem_desc(addr, lbo, sbo) | (static_cast<uint64_t>(2) << 61);  // layout: 128-byte swizzle
+}
+__device__ __forceinline__ uint64_t desc_sw_k(uint32_t base, int kk) {
+    return sw_desc(base + (kk >> 2) * (T * 128) + (kk & 3) * 32, 16, 1024);
+}
+__device__ __forceinline__ uint64_t desc_sw_mn(uint32_t base, int kk) {
+    return sw_desc(base + kk * 2048, T * 128, 1024);
 }
 
-__device__ __forceinline__ void load_meta_async(uint32_t dst, const TileMeta* src, int tid) {
-    constexpr int N = sizeof(TileMeta) / 16;
-    if (tid < N) cp_async16(dst + tid * 16, reinterpret_cast<const unsigned char*>(src) + tid * 16, true);
+// One [T x D] bf16 tile, steps t0..t0+T-1 of head h of tape b, from a 4-D
+// tensor map {D, H, L, B} with 128-byte swizzling: D/64 boxes of {64, 1, T, 1}.
+// Steps past L read as 0.
+template <int D>
+__device__ __forceinline__ void tma_tile(uint32_t dst, const CUtensorMap* map, int64_t h, int64_t t0, int64_t b,
+                                         uint64_t* bar) {
+#pragma unroll
+    for (int m = 0; m < D / 64; ++m)
+        tma_load_4d(dst + m * T * 128, map, 64 * m, static_cast<int>(h), static_cast<int>(t0), static_cast<int>(b), bar);
 }
 
 __device__ __forceinline__ bool wait_mbar(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
@@ -288,13 +300,15 @@ struct FwdSmem {
     static constexpr int STAGE = 3 * TILE;       // Q, K, V
     static constexpr int OFF_PM = PM_IN_Q ? 0 : 2 * STAGE;
     static constexpr int OFF_SB = 2 * STAGE + (PM_IN_Q ? 0 : PM);
+    static constexpr int NMETA = 3;  // metadata ring: tiles c, c+1 in use, c+2 loading
     static constexpr int OFF_META = OFF_SB + D * D * 2;
-    static constexpr int OFF_BAR = OFF_META + 4 * static_cast<int>(sizeof(TileMeta));
-    static constexpr int BYTES = OFF_BAR + 32;
-    // fp32 output rows staged in the finished stage for bulk stores: one row
-    // per step, padded by 16 bytes so that 8 consecutive rows hit 8 bank groups
-    static constexpr int YROW = D * 4 + 16;
-    static_assert(T * YROW <= STAGE, "output staging fits in one stage");
+    static constexpr int OFF_Z = OFF_META + NMETA * static_cast<int>(sizeof(TileMeta));  // [2][T] fp32 (pass F)
+    static constexpr int OFF_BAR = OFF_Z + 2 * T * 4;
+    static constexpr int BYTES = OFF_BAR + 64;
+    // the fp32 output tile is staged in the finished stage in the 128-byte
+    // swizzled layout of its TMA store (32 channels per 128-byte row, chunk
+    // of 32 channels at m * T * 128)
+    static_assert(T * D * 4 <= STAGE, "output staging fits in one stage");
     // TMEM columns: scores P, intra output, inter output, state S
     static constexpr uint32_t COL_P = 0, COL_YA = 128, COL_YI = 128 + D, COL_S = 128 + 2 * D;
     static constexpr uint32_t TMEM_COLS = 512;
@@ -302,6 +316,8 @@ struct FwdSmem {
 };
 
 struct FwdParams {
+    CUtensorMap map_q, map_k, map_v;  // the q, k, v operands (4-D {D, H, L, B}, box {64, 1, 128, 1})
+    CUtensorMap map_y;                // the fp32 output (4-D {D, H, L, B}, box {32, 1, 128, 1})
     const uint16_t* q;
     const uint16_t* k;
     const uint16_t* v;
@@ -318,7 +334,25 @@ struct FwdParams {
     const uint16_t* zq;  // q, bf16 [B, L, H, D]
     float* dlam_f;       // [B, L, H]: the state-side terms of dL/dlog(gamma_t)
     uint16_t* states;    // [B, H, n_tiles, D, D] bf16: S_{c-1}^T before tiles without a begin flag
+#ifdef MEMOROID_LA_TRACE
+    unsigned long long* trace;  // per-phase nanoseconds of CTA 0, thread 0
+#endif
 };
+
+#ifdef MEMOROID_LA_TRACE
+#define LA_MARK(i)                                  \
+    do {                                            \
+        if (trace_on) {                             \
+            const uint64_t now_ = globaltimer();    \
+            tr[i] += now_ - tr_last;                \
+            tr_last = now_;                         \
+        }                                           \
+    } while (0)
+#else
+#define LA_MARK(i) \
+    do {           \
+    } while (0)
+#endif
 
 // Thread -> row of a D x D state accumulator in TMEM.  With M = 128 the row
 // is the TMEM lane; with M = 64 rows 16q..16q+15 sit in lanes 32q..32q+15 and
@@ -370,7 +404,7 @@ __device__ __forceinline__ void store_bf16x16(unsigned char* base, uint32_t off0
 // outputs), and stores S'_{c-1} as bf16 for every tile without a begin flag,
 // for pass R.
 template <int D, bool BWD>
-__global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
+__global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant__ FwdParams p) {
     using S = FwdSmem<D>;
     extern __shared__ __align__(1024) unsigned char smem[];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -396,7 +430,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
 
     uint64_t* bar1 = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
     uint64_t* bar2 = bar1 + 1;
-    uint32_t* tslot = reinterpret_cast<uint32_t*>(bar1 + 2);
+    uint64_t* full = bar1 + 2;  // [2]: stage s loaded
+    uint32_t* tslot = reinterpret_cast<uint32_t*>(bar1 + 4);
     TileMeta* metas = reinterpret_cast<TileMeta*>(smem + S::OFF_META);
     const uint32_t sbase = smem_addr(smem);
     const uint32_t sSb = sbase + S::OFF_SB;
@@ -406,30 +441,36 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
     auto stage_k = [&](int s) { return sbase + s * S::STAGE + S::TILE; };
     auto stage_v = [&](int s) { return sbase + s * S::STAGE + 2 * S::TILE; };
     auto stage_pm = [&](int s) { return S::PM_IN_Q ? stage_q(s) : sbase + S::OFF_PM; };
-    auto issue_tile = [&](int c, int s) {
+    // thread 0: TMA loads of tile c into stage s and of metadata tiles m0 (and
+    // m1 >= 0) into their ring slots, all completing on full[s]
+    auto issue_tile = [&](int c, int s, int m0, int m1) {
+        const uint32_t meta_bytes = (m0 >= 0 ? sizeof(TileMeta) : 0) + (m1 >= 0 ? sizeof(TileMeta) : 0);
+        mbar_arrive_expect_tx(&full[s], 3 * S::TILE + meta_bytes);
         const int64_t t0 = (tile0 + c) * T;
-        const int nvalid = static_cast<int>(min(static_cast<int64_t>(T), p.L - t0));
-        const int64_t off = ((b * p.L + t0) * p.H + h) * D;
-        load_tile_async<D>(stage_q(s), p.q + off, row_stride, nvalid, tid);
-        load_tile_async<D>(stage_k(s), p.k + off, row_stride, nvalid, tid);
-        load_tile_async<D>(stage_v(s), p.v + off, row_stride, nvalid, tid);
+        tma_tile<D>(stage_q(s), &p.map_q, h, t0, b, &full[s]);
+        tma_tile<D>(stage_k(s), &p.map_k, h, t0, b, &full[s]);
+        tma_tile<D>(stage_v(s), &p.map_v, h, t0, b, &full[s]);
+        if (m0 >= 0) bulk_g2s(&metas[m0 % S::NMETA], gmeta + m0, sizeof(TileMeta), &full[s]);
+        if (m1 >= 0) bulk_g2s(&metas[m1 % S::NMETA], gmeta + m1, sizeof(TileMeta), &full[s]);
     };
 
     if (tid == 0) {
         mbar_init(bar1, 1);
         mbar_init(bar2, 1);
+        mbar_init(&full[0], 1);
+        mbar_init(&full[1], 1);
         fence_mbar_init();
+        prefetch_tensormap(&p.map_q);
+        prefetch_tensormap(&p.map_k);
+        prefetch_tensormap(&p.map_v);
+        prefetch_tensormap(&p.map_y);
     }
     if (warp == 0) tc::alloc(tslot, S::TMEM_COLS);
-
-    issue_tile(0, 0);
-    load_meta_async(smem_addr(&metas[0]), gmeta, tid);
-    if (nt > 1) load_meta_async(smem_addr(&metas[1]), gmeta + 1, tid);
-    cp_async_commit();
-    cp_async_wait<0>();
     tc::fence_before();
     __syncthreads();
     tc::fence_after();
+    if (tid == 0) issue_tile(0, 0, 0, nt > 1 ? 1 : -1);
+    const bool first_ok = wait_mbar(&full[0], 0, p.wait_ns);
     const uint32_t tm = *tslot;
 
     const int srow = state_row<D>(quarter, lane);
@@ -489,24 +530,34 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
     constexpr uint32_t ID_PV = tc::idesc_bf16(128, D, false, true);
     constexpr uint32_t ID_KV = tc::idesc_bf16(D, D, true, true);
 
-    bool failed = false;
+    bool failed = __syncthreads_or(!first_ok);
+    int pending = failed ? -1 : 0;  // the last issued tile whose load may still be in flight
+#ifdef MEMOROID_LA_TRACE
+    const bool trace_on = blockIdx.x == 0 && tid == 0 && p.trace != nullptr;
+    unsigned long long tr[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    uint64_t tr_last = globaltimer();
+#endif
 #pragma unroll 1
-    for (int c = 0; c < nt; ++c) {
+    for (int c = 0; c < nt && !failed; ++c) {
         const int s = c & 1;
-        const TileMeta& mc = metas[c & 3];
-        // tile c's copies (issued one iteration ago) and the previous tile's
+        const TileMeta& mc = metas[c % S::NMETA];
+        // tile c's loads (issued one iteration ago) and the previous tile's
         // output stores (which read stage s ^ 1) are complete
-        cp_async_wait<0>();
+        bool ok = wait_mbar(&full[s], (c >> 1) & 1, p.wait_ns);
         if (warp == 0) bulk_wait_read();
         tc::fence_smem_to_async();
         tc::fence_before();
-        __syncthreads();
-        tc::fence_after();
-        if (c + 1 < nt) {
-            issue_tile(c + 1, s ^ 1);
-            if (c + 2 < nt) load_meta_async(smem_addr(&metas[(c + 2) & 3]), gmeta + c + 2, tid);
+        if (__syncthreads_or(!ok)) {
+            failed = true;
+            break;
         }
-        cp_async_commit();
+        pending = -1;
+        tc::fence_after();
+        LA_MARK(0);
+        if (c + 1 < nt) {
+            if (tid == 0) issue_tile(c + 1, s ^ 1, c + 2 < nt ? c + 2 : -1, -1);
+            pending = c + 1;
+        }
 
         // ---- P = Q K^T and (with an incoming state) Y_inter = Q S_prev ----
         if (tid == 0) {
@@ -514,20 +565,21 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
             if (have_prev) {
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk)
-                    tc::mma(tm + S::COL_YI, desc_kmajor(sq, D, kk), desc_mnmajor(sSb, D, kk), ID_QS, kk > 0);
+                    tc::mma(tm + S::COL_YI, desc_sw_k(sq, kk), desc_mnmajor(sSb, D, kk), ID_QS, kk > 0);
             }
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk)
-                tc::mma(tm + S::COL_P, desc_kmajor(sq, D, kk), desc_kmajor(sk, D, kk), ID_QK, kk > 0);
+                tc::mma(tm + S::COL_P, desc_sw_k(sq, kk), desc_sw_k(sk, kk), ID_QK, kk > 0);
             tc::commit(bar1);
         }
-
-        bool ok = wait_mbar(bar1, c & 1, p.wait_ns);
+        LA_MARK(1);
+        ok = wait_mbar(bar1, c & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
             failed = true;
             break;
         }
         tc::fence_after();
+        LA_MARK(2);
 
         // ---- mask: Pm[t][r] = [seg_t <= r <= t] exp2(lam2_t - lam2_r) P[t][r] ----
         {
@@ -552,6 +604,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
                 store_bf16x16(pm, core_off(t, r0, T), core_off(t, r0 + 8, T), v);
             }
         }
+        LA_MARK(3);
         // ---- K~[r] = exp2(lam2_end - lam2_r) K[r] for rows of the last episode ----
         {
             unsigned char* kt = smem + (stage_k(s) - sbase);
@@ -560,9 +613,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
             constexpr int NCH = T * D / 8;
 #pragma unroll 2
             for (int e = tid; e < NCH; e += kThreads) {
-                // e enumerates 16-byte chunks in memory order: a row group of 8
-                // rows holds D chunks, 8 per core matrix, one per row
-                const int r = (e / D) * 8 + (e & 7);
+                // e enumerates 16-byte units in memory order: 8 per 128-byte row
+                const int r = (e >> 3) & (T - 1);
                 const float w = r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f;
                 if (w != 1.f) {
                     uint4 u = *reinterpret_cast<uint4*>(kt + e * 16);
@@ -589,19 +641,21 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
             const uint32_t spm = stage_pm(s), sk = stage_k(s), sv = stage_v(s);
 #pragma unroll
             for (int kk = 0; kk < T / 16; ++kk)
-                tc::mma(tm + S::COL_YA, desc_kmajor(spm, T, kk), desc_mnmajor(sv, D, kk), ID_PV, kk > 0);
+                tc::mma(tm + S::COL_YA, desc_kmajor(spm, T, kk), desc_sw_mn(sv, kk), ID_PV, kk > 0);
             const bool acc = have_state && mc.has_start == 0;
 #pragma unroll
             for (int kk = 0; kk < T / 16; ++kk)
-                tc::mma(tm + S::COL_S, desc_mnmajor(sk, D, kk), desc_mnmajor(sv, D, kk), ID_KV, acc || kk > 0);
+                tc::mma(tm + S::COL_S, desc_sw_mn(sk, kk), desc_sw_mn(sv, kk), ID_KV, acc || kk > 0);
             tc::commit(bar2);
         }
+        LA_MARK(4);
         ok = wait_mbar(bar2, c & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
             failed = true;
             break;
         }
         tc::fence_after();
+        LA_MARK(5);
 
         // ---- y = Y_intra + w_in * Y_inter, staged as fp32 rows in stage s ----
         const int64_t t0 = (tile0 + c) * T;
@@ -611,7 +665,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
         {
             const int t = 32 * quarter + lane;
             const float w_in = (have_prev && mc.seg[t] < 0) ? fast_exp2(mc.lam2[t]) : 0.f;
-            unsigned char* yst = smem + s * S::STAGE + t * S::YROW;
+            unsigned char* yst = smem + s * S::STAGE + t * 128;  // row t of chunk 0
             // BWD: z_t = w_in_t q_t . (S_{c-1} dy_t), the inter output dotted with q
             const bool zrow = BWD && w_in != 0.f && t0 + t < p.L;
             const uint16_t* qrow = BWD ? p.zq + ((b * p.L + t0 + t) * p.H + h) * D : nullptr;
@@ -637,7 +691,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
                         o.z = fmaf(w_in, __uint_as_float(yi[x + 2]), o.z);
                         o.w = fmaf(w_in, __uint_as_float(yi[x + 3]), o.w);
                     }
-                    *reinterpret_cast<float4*>(yst + (j0 + x) * 4) = o;
+                    const int j = j0 + x;  // 4 channels = one 16-byte unit
+                    *reinterpret_cast<float4*>(yst + (j >> 5) * (T * 128) + ((((j & 31) >> 2) ^ (t & 7)) << 4)) = o;
                 }
                 if (zrow) {
 #pragma unroll
@@ -656,12 +711,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
                     }
                 }
             }
-            // the row's 16 padding bytes hold the two column halves' partial z
-            if (BWD) *reinterpret_cast<float*>(yst + D * 4 + half * 4) = w_in * zacc;
+            if (BWD) reinterpret_cast<float*>(smem + S::OFF_Z)[half * T + t] = w_in * zacc;
         }
         // ---- state: bf16 copy for the next tile, decay by the next tile's a ----
         if (c + 1 < nt) {
-            const TileMeta& mn = metas[(c + 1) & 3];
+            const TileMeta& mn = metas[(c + 1) % S::NMETA];
             const bool scale = mn.has_start == 0 && mn.a != 1.f;
             const float an = mn.a;
 #pragma unroll
@@ -703,25 +757,41 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
                 }
             }
         }
+        LA_MARK(6);
         // ---- bulk-store the staged output rows ----
         tc::fence_smem_to_async();
         tc::fence_before();
         __syncthreads();
+        LA_MARK(7);
         if (warp == 0) {
-            float* ybase = p.y + ((b * p.L + t0) * p.H + h) * D;
-            for (int r = r_lo + lane; r < r_hi; r += 32)
-                bulk_s2g(ybase + static_cast<int64_t>(r) * row_stride, sbase + s * S::STAGE + r * S::YROW, D * 4);
+            const int full_rows = static_cast<int>(min(static_cast<int64_t>(T), p.L - t0));
+            if (r_lo == 0 && r_hi == full_rows) {
+                // whole tile: one TMA store per 32 channels (rows past L are clipped)
+                if (lane == 0) {
+#pragma unroll
+                    for (int m = 0; m < D / 32; ++m)
+                        tma_store_4d(&p.map_y, sbase + s * S::STAGE + m * T * 128, 32 * m, static_cast<int>(h),
+                                     static_cast<int>(t0), static_cast<int>(b));
+                }
+            } else {
+                // a tile shared with a neighbouring segment: only this segment's rows, 16 bytes at a time
+                float* ybase = p.y + ((b * p.L + t0) * p.H + h) * D;
+                const unsigned char* st = smem + s * S::STAGE;
+                for (int e = lane; e < (r_hi - r_lo) * (D / 4); e += 32) {
+                    const int r = r_lo + e / (D / 4), j = (e % (D / 4)) * 4;
+                    const float4 v = *reinterpret_cast<const float4*>(st + (j >> 5) * (T * 128) + r * 128 +
+                                                                      ((((j & 31) >> 2) ^ (r & 7)) << 4));
+                    *reinterpret_cast<float4*>(ybase + static_cast<int64_t>(r) * row_stride + j) = v;
+                }
+            }
             bulk_commit();
         }
         if (BWD && warp == 1) {
             // suffix sums of z over the tile: dlam_f[t] = sum_{s >= t} z_s
-            const unsigned char* zst = smem + s * S::STAGE + D * 4;
+            const float* zst = reinterpret_cast<const float*>(smem + S::OFF_Z);
             float zv[4];
 #pragma unroll
-            for (int x = 0; x < 4; ++x) {
-                const float* zp = reinterpret_cast<const float*>(zst + (4 * lane + x) * S::YROW);
-                zv[x] = zp[0] + zp[1];
-            }
+            for (int x = 0; x < 4; ++x) zv[x] = zst[4 * lane + x] + zst[T + 4 * lane + x];
 #pragma unroll
             for (int x = 2; x >= 0; --x) zv[x] += zv[x + 1];
             float tot = zv[0];
@@ -743,9 +813,16 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const FwdParams p) {
     }
     if (failed) {
         if (tid == 0) record_error(p.hdr, DEV_MMA_TIMEOUT);
-        cp_async_wait<0>();
+        // let a load still in flight land before the CTA's shared memory goes away
+        if (pending >= 0) wait_mbar(&full[pending & 1], (pending >> 1) & 1, p.wait_ns);
     }
     if (warp == 0) bulk_wait_all();
+#ifdef MEMOROID_LA_TRACE
+    if (trace_on) {
+        for (int i = 0; i < 8; ++i) p.trace[i] = tr[i];
+        p.trace[8] = static_cast<unsigned long long>(nt);
+    }
+#endif
     tc::fence_before();
     __syncthreads();
     tc::fence_after();
@@ -790,6 +867,7 @@ struct BwdSmem {
 };
 
 struct BwdParams {
+    CUtensorMap map_q, map_k, map_v, map_dy;
     const uint16_t* q;
     const uint16_t* k;
     const uint16_t* v;
@@ -829,7 +907,7 @@ __device__ __forceinline__ float warp_transpose_sum32(float (&v)[32], int lane) 
 }
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
+__global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant__ BwdParams p) {
     using S = BwdSmem<D>;
     extern __shared__ __align__(1024) unsigned char smem[];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -851,12 +929,12 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
         }
     }
     const int64_t tile_lo = seg_lo / T, tile_hi = (seg_hi + T - 1) / T;  // tiles [tile_lo, tile_hi)
-    const int64_t row_stride = p.H * D;
 
     uint64_t* bar1 = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
     uint64_t* bar2 = bar1 + 1;
     uint64_t* bar3 = bar1 + 2;
-    uint32_t* tslot = reinterpret_cast<uint32_t*>(bar1 + 3);
+    uint64_t* full = bar1 + 3;
+    uint32_t* tslot = reinterpret_cast<uint32_t*>(bar1 + 4);
     const TileMeta& mc = *reinterpret_cast<const TileMeta*>(smem + S::OFF_META);
     const uint32_t sbase = smem_addr(smem);
     const uint32_t sQ = sbase + S::OFF_Q, sK = sbase + S::OFF_K, sV = sbase + S::OFF_V, sDY = sbase + S::OFF_DY;
@@ -867,29 +945,33 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
     float* st_iv = reinterpret_cast<float*>(smem + S::ST_IV);
     float* st_intra = reinterpret_cast<float*>(smem + S::ST_INTRA);
 
+    // thread 0: TMA loads of a tile and its metadata, completing on `full`
     auto issue_tile = [&](int64_t tile) {
+        mbar_arrive_expect_tx(full, 4 * S::TILE + sizeof(TileMeta));
         const int64_t t0 = tile * T;
-        const int nvalid = static_cast<int>(min(static_cast<int64_t>(T), p.L - t0));
-        const int64_t off = ((b * p.L + t0) * p.H + h) * D;
-        load_tile_async<D>(sQ, p.q + off, row_stride, nvalid, tid);
-        load_tile_async<D>(sK, p.k + off, row_stride, nvalid, tid);
-        load_tile_async<D>(sV, p.v + off, row_stride, nvalid, tid);
-        load_tile_async<D>(sDY, p.dy + off, row_stride, nvalid, tid);
-        load_meta_async(sbase + S::OFF_META, p.meta + bh * p.n_tiles + tile, tid);
-        cp_async_commit();
+        tma_tile<D>(sQ, &p.map_q, h, t0, b, full);
+        tma_tile<D>(sK, &p.map_k, h, t0, b, full);
+        tma_tile<D>(sV, &p.map_v, h, t0, b, full);
+        tma_tile<D>(sDY, &p.map_dy, h, t0, b, full);
+        bulk_g2s(smem + S::OFF_META, p.meta + bh * p.n_tiles + tile, sizeof(TileMeta), full);
     };
 
     if (tid == 0) {
         mbar_init(bar1, 1);
         mbar_init(bar2, 1);
         mbar_init(bar3, 1);
+        mbar_init(full, 1);
         fence_mbar_init();
+        prefetch_tensormap(&p.map_q);
+        prefetch_tensormap(&p.map_k);
+        prefetch_tensormap(&p.map_v);
+        prefetch_tensormap(&p.map_dy);
     }
     if (warp == 0) tc::alloc(tslot, S::TMEM_COLS);
-    issue_tile(tile_hi - 1);
     tc::fence_before();
     __syncthreads();
     tc::fence_after();
+    if (tid == 0) issue_tile(tile_hi - 1);
     const uint32_t tm = *tslot;
     const uint32_t lane_base = tm + (static_cast<uint32_t>(32 * quarter) << 16);
     const int srow = state_row<D>(quarter, lane);
@@ -930,16 +1012,21 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
 
     float gsum = 0.f;  // per-head mode: sum of dL/dlog(gamma) over the segment's steps
     bool failed = false;
+    bool pending = true;  // a tile load may be in flight
     int it = 0;
 #pragma unroll 1
     for (int64_t tile = tile_hi - 1; tile >= tile_lo; --tile, ++it) {
         const int64_t t0 = tile * T;
         const int r_lo = static_cast<int>(max(static_cast<int64_t>(0), seg_lo - t0));
         const int r_hi = static_cast<int>(min(static_cast<int64_t>(T), seg_hi - t0));
-        cp_async_wait<0>();
+        bool ok = wait_mbar(full, it & 1, p.wait_ns);
         tc::fence_smem_to_async();
         tc::fence_before();
-        __syncthreads();
+        if (__syncthreads_or(!ok)) {
+            failed = true;
+            break;
+        }
+        pending = false;
         tc::fence_after();
         const bool tile_start = mc.has_start != 0;
 
@@ -947,18 +1034,18 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
         if (tid == 0) {
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk)
-                tc::mma(tm + S::COL_P, desc_kmajor(sQ, D, kk), desc_kmajor(sK, D, kk), ID_SCORE, kk > 0);
+                tc::mma(tm + S::COL_P, desc_sw_k(sQ, kk), desc_sw_k(sK, kk), ID_SCORE, kk > 0);
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk)
-                tc::mma(tm + S::COL_DP, desc_kmajor(sDY, D, kk), desc_kmajor(sV, D, kk), ID_SCORE, kk > 0);
+                tc::mma(tm + S::COL_DP, desc_sw_k(sDY, kk), desc_sw_k(sV, kk), ID_SCORE, kk > 0);
             if (have_g) {
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk)
-                    tc::mma(tm + S::COL_DKI, desc_kmajor(sV, D, kk), desc_kmajor(sGB, D, kk), ID_VG, kk > 0);
+                    tc::mma(tm + S::COL_DKI, desc_sw_k(sV, kk), desc_kmajor(sGB, D, kk), ID_VG, kk > 0);
             }
             tc::commit(bar1);
         }
-        bool ok = wait_mbar(bar1, it & 1, p.wait_ns);
+        ok = wait_mbar(bar1, it & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
             failed = true;
             break;
@@ -1011,7 +1098,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
             constexpr int NCH = T * D / 8;
 #pragma unroll 2
             for (int e = tid; e < NCH; e += kThreads) {
-                const int r = (e / D) * 8 + (e & 7);
+                const int r = (e >> 3) & (T - 1);
                 const float w = r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f;
                 if (w != 1.f) {
                     uint4 u = *reinterpret_cast<uint4*>(kt + e * 16);
@@ -1067,15 +1154,15 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
         if (tid == 0) {
 #pragma unroll
             for (int kk = 0; kk < T / 16; ++kk)
-                tc::mma(tm + S::COL_DV, desc_mnmajor(sPM, T, kk), desc_mnmajor(sDY, D, kk), ID_PTDY, kk > 0);
+                tc::mma(tm + S::COL_DV, desc_mnmajor(sPM, T, kk), desc_sw_mn(sDY, kk), ID_PTDY, kk > 0);
             if (have_g) {
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk)
-                    tc::mma(tm + S::COL_DV, desc_kmajor(sK, D, kk), desc_mnmajor(sGB, D, kk), ID_KG, true);
+                    tc::mma(tm + S::COL_DV, desc_sw_k(sK, kk), desc_mnmajor(sGB, D, kk), ID_KG, true);
             }
 #pragma unroll
             for (int kk = 0; kk < T / 16; ++kk)
-                tc::mma(tm + S::COL_DK, desc_mnmajor(sDPM, T, kk), desc_mnmajor(sQ, D, kk), ID_PTDY, kk > 0);
+                tc::mma(tm + S::COL_DK, desc_mnmajor(sDPM, T, kk), desc_sw_mn(sQ, kk), ID_PTDY, kk > 0);
             tc::commit(bar2);
         }
         // intra-tile term while B2 runs: intra_t = sum_{u < t} (colsum_u - rowsum_u)
@@ -1113,7 +1200,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
             constexpr int NCH = T * D / 8;
 #pragma unroll 2
             for (int e = tid; e < NCH; e += kThreads) {
-                const int r = (e / D) * 8 + (e & 7);
+                const int r = (e >> 3) & (T - 1);
                 const float w = mc.seg[r] < 0 ? fast_exp2(mc.lam2[r]) : 0.f;
                 if (w != 1.f) {
                     uint4 u = *reinterpret_cast<uint4*>(qt + e * 16);
@@ -1138,7 +1225,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
             const bool acc = have_g && !tile_start;
 #pragma unroll
             for (int kk = 0; kk < T / 16; ++kk)
-                tc::mma(tm + S::COL_G, desc_mnmajor(sQ, D, kk), desc_mnmajor(sDY, D, kk), ID_QDY, acc || kk > 0);
+                tc::mma(tm + S::COL_G, desc_sw_mn(sQ, kk), desc_sw_mn(sDY, kk), ID_QDY, acc || kk > 0);
             tc::commit(bar3);
         }
 
@@ -1169,7 +1256,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
                     const unsigned char* kt = smem + S::OFF_K;
 #pragma unroll
                     for (int x = 0; x < 16; x += 8) {
-                        const uint4 u = *reinterpret_cast<const uint4*>(kt + core_off(r, j0 + x, D));
+                        const uint4 u = *reinterpret_cast<const uint4*>(kt + sw_off(r, j0 + x));
                         const float2 k0 = unpack_bf16x2(u.x), k1 = unpack_bf16x2(u.y), k2 = unpack_bf16x2(u.z),
                                      k3 = unpack_bf16x2(u.w);
                         xacc = fmaf(k0.x, __uint_as_float(ri[x]), xacc);
@@ -1263,11 +1350,15 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const BwdParams p) {
         }
         tc::fence_before();
         __syncthreads();
-        if (tile > tile_lo) issue_tile(tile - 1);
+        if (tile > tile_lo) {
+            if (tid == 0) issue_tile(tile - 1);
+            pending = true;
+        }
     }
     if (failed) {
         if (tid == 0) record_error(p.hdr, DEV_MMA_TIMEOUT);
-        cp_async_wait<0>();
+        // let a load still in flight land before the CTA's shared memory goes away
+        if (pending) wait_mbar(full, it & 1, p.wait_ns);
     }
     if (tid == 0 && p.gpart != nullptr) p.gpart[bh * p.G + g] = gsum;
     tc::fence_before();
@@ -1345,10 +1436,10 @@ __global__ void __launch_bounds__(128, 1) intra_bench_kernel(const uint4* __rest
         for (int r = 0; r < reps; ++r) {
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk)
-                tc::mma(tm, desc_kmajor(sq, D, kk), desc_kmajor(sk, D, kk), ID_QK, r > 0 || kk > 0);
+                tc::mma(tm, desc_sw_k(sq, kk), desc_sw_k(sk, kk), ID_QK, r > 0 || kk > 0);
 #pragma unroll
             for (int kk = 0; kk < T / 16; ++kk)
-                tc::mma(tm + 128, desc_kmajor(spm, T, kk), desc_mnmajor(sv, D, kk), ID_PV, r > 0 || kk > 0);
+                tc::mma(tm + 128, desc_kmajor(spm, T, kk), desc_sw_mn(sv, kk), ID_PV, r > 0 || kk > 0);
         }
         tc::commit(&bar);
     }
@@ -1400,10 +1491,73 @@ memoroid_status_t launch_intra_bench(int64_t D, int64_t reps, int64_t ctas, void
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
+#ifdef MEMOROID_LA_TRACE
+__device__ unsigned long long g_la_trace[16];
+unsigned long long* la_trace_buffer() {
+    void* ptr = nullptr;
+    cudaGetSymbolAddress(&ptr, g_la_trace);
+    return static_cast<unsigned long long*>(ptr);
+}
+#endif
 namespace {
 template <typename K>
 cudaError_t set_smem(K kernel, int bytes) {
     return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+}
+
+// cuTensorMapEncodeTiled, taken from the driver at run time (the library does
+// not link libcuda).
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    });
+    return fn;
+}
+
+// A bf16 [B, L, H, D] tensor as a 4-D map {D, H, L, B} with 128-byte swizzled
+// boxes of 64 channels x T steps of one head ({64, 1, T, 1}); steps past L
+// read as zeros.
+bool tile_map_y(CUtensorMap* m, const void* base, int64_t B, int64_t L, int64_t H, int64_t D);
+
+bool tile_map(CUtensorMap* m, const void* base, int64_t B, int64_t L, int64_t H, int64_t D) {
+    const EncodeTiledFn fn = encode_tiled();
+    if (fn == nullptr) return false;
+    const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(H), static_cast<cuuint64_t>(L),
+                                static_cast<cuuint64_t>(B)};
+    const cuuint64_t strides[3] = {static_cast<cuuint64_t>(D * 2), static_cast<cuuint64_t>(H * D * 2),
+                                   static_cast<cuuint64_t>(L * H * D * 2)};
+    const cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(T), 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// An fp32 [B, L, H, D] output as a 4-D map {D, H, L, B} with 128-byte swizzled
+// boxes of 32 channels x T steps ({32, 1, T, 1}); stores past L are clipped.
+bool tile_map_y(CUtensorMap* m, const void* base, int64_t B, int64_t L, int64_t H, int64_t D) {
+    const EncodeTiledFn fn = encode_tiled();
+    if (fn == nullptr) return false;
+    const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(H), static_cast<cuuint64_t>(L),
+                                static_cast<cuuint64_t>(B)};
+    const cuuint64_t strides[3] = {static_cast<cuuint64_t>(D * 4), static_cast<cuuint64_t>(H * D * 4),
+                                   static_cast<cuuint64_t>(L * H * D * 4)};
+    const cuuint32_t box[4] = {32, 1, static_cast<cuuint32_t>(T), 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<void*>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // Tile metadata and segment boundaries (shared by the forward and backward passes).
@@ -1430,6 +1584,9 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     if (st != MEMOROID_OK) return st;
 
     FwdParams p;
+    if (!tile_map(&p.map_q, a.q, a.B, a.L, a.H, D) || !tile_map(&p.map_k, a.k, a.B, a.L, a.H, D) ||
+        !tile_map(&p.map_v, a.v, a.B, a.L, a.H, D) || !tile_map_y(&p.map_y, a.y, a.B, a.L, a.H, D))
+        return MEMOROID_ERR_CUDA;
     p.q = static_cast<const uint16_t*>(a.q);
     p.k = static_cast<const uint16_t*>(a.k);
     p.v = static_cast<const uint16_t*>(a.v);
@@ -1449,6 +1606,9 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     p.zq = nullptr;
     p.dlam_f = nullptr;
     p.states = nullptr;
+#ifdef MEMOROID_LA_TRACE
+    p.trace = la_trace_buffer();
+#endif
     if (set_smem(fwd_kernel<D, false>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
     fwd_kernel<D, false><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
@@ -1474,6 +1634,9 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
 
     // pass F: dq = S dy, with (q, k, v) -> (dy, v, k)
     FwdParams f;
+    if (!tile_map(&f.map_q, dy16, a.B, a.L, a.H, D) || !tile_map(&f.map_k, a.v, a.B, a.L, a.H, D) ||
+        !tile_map(&f.map_v, a.k, a.B, a.L, a.H, D) || !tile_map_y(&f.map_y, a.dq, a.B, a.L, a.H, D))
+        return MEMOROID_ERR_CUDA;
     f.q = dy16;
     f.k = static_cast<const uint16_t*>(a.v);
     f.v = static_cast<const uint16_t*>(a.k);
@@ -1493,12 +1656,18 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     f.zq = static_cast<const uint16_t*>(a.q);
     f.dlam_f = dlam_f;
     f.states = states;
+#ifdef MEMOROID_LA_TRACE
+    f.trace = nullptr;
+#endif
     if (set_smem(fwd_kernel<D, true>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
     fwd_kernel<D, true><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
 
     // pass R: dk, dv, dgamma, dS0
     BwdParams r;
+    if (!tile_map(&r.map_q, a.q, a.B, a.L, a.H, D) || !tile_map(&r.map_k, a.k, a.B, a.L, a.H, D) ||
+        !tile_map(&r.map_v, a.v, a.B, a.L, a.H, D) || !tile_map(&r.map_dy, dy16, a.B, a.L, a.H, D))
+        return MEMOROID_ERR_CUDA;
     r.q = static_cast<const uint16_t*>(a.q);
     r.k = static_cast<const uint16_t*>(a.k);
     r.v = static_cast<const uint16_t*>(a.v);
@@ -1563,3 +1732,10 @@ memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream) {
 
 }  // namespace la
 }  // namespace memoroid
+
+#ifdef MEMOROID_LA_TRACE
+// trace builds only: copies the forward kernel's per-phase times to the host
+extern "C" void memoroid_debug_la_trace(unsigned long long* host_out) {
+    cudaMemcpy(host_out, memoroid::la::la_trace_buffer(), 16 * sizeof(unsigned long long), cudaMemcpyDeviceToHost);
+}
+#endif

@@ -50,6 +50,30 @@ __device__ __forceinline__ void bulk_g2s(void* dst_smem, const void* src_gmem, u
         : "memory");
 }
 
+// ---- TMA tiled load (4-D tensor map, global -> shared), completes on an mbarrier ----
+// `map` is the address of a CUtensorMap in kernel-parameter (or constant/global)
+// memory.  Coordinates are element indices, innermost first; the innermost one
+// times the element size must be a multiple of 16 bytes.  Out-of-range
+// elements of the box are filled with zeros.
+__device__ __forceinline__ void tma_load_4d(uint32_t dst_smem, const void* map, int c0, int c1, int c2, int c3,
+                                            uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], "
+        "[%6];" ::"r"(dst_smem),
+        "l"(map), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_addr(bar))
+        : "memory");
+}
+// TMA tiled store (shared -> global) of one box; completes in the bulk group
+// (bulk_commit / bulk_wait_read / bulk_wait_all).  Out-of-range rows are clipped.
+__device__ __forceinline__ void tma_store_4d(const void* map, uint32_t src_smem, int c0, int c1, int c2, int c3) {
+    asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.tile.bulk_group [%0, {%2, %3, %4, %5}], [%1];" ::"l"(map),
+                 "r"(src_smem), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+                 : "memory");
+}
+__device__ __forceinline__ void prefetch_tensormap(const void* map) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
+}
+
 // ---- flags ---------------------------------------------------------------------
 __device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
     uint32_t v;
