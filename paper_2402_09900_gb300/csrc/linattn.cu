@@ -820,7 +820,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
 #ifdef MEMOROID_LA_TRACE
     if (trace_on) {
         for (int i = 0; i < 8; ++i) p.trace[i] = tr[i];
-        p.trace[8] = static_cast<unsigned long long>(nt);
     }
 #endif
     tc::fence_before();
@@ -859,7 +858,17 @@ struct BwdSmem {
     static constexpr int ST_X = ST_ROW + 2 * T * 4;     // [2][T] x_r per column half
     static constexpr int ST_IV = ST_X + 2 * T * 4;      // [8] per-warp partial <G, S>
     static constexpr int ST_INTRA = ST_IV + 64;         // [T] intra-tile term
-    static_assert(ST_INTRA + T * 4 <= OFF_V + TILE, "statistics fit in the V tile");
+    static constexpr int ST_WT = ST_INTRA + T * 4;      // [4] per-warp totals of x
+    static_assert(ST_WT + 64 <= OFF_V + TILE, "statistics fit in the V tile");
+    // fp32 dk / dv tiles staged for their TMA stores (128-byte swizzled, 32
+    // channels x T rows = 16 KB per chunk), in buffers free once B2 is done:
+    // dk in Pm | dPm; dv in dPm (d = 64) or K | G (d = 128)
+    static constexpr int CHUNK = T * 128;
+    __host__ __device__ static constexpr int dk_chunk(int m) { return OFF_PM + m * CHUNK; }
+    __host__ __device__ static constexpr int dv_chunk(int m) {
+        return D == 64 ? OFF_DPM + m * CHUNK : (m < 2 ? OFF_K + m * CHUNK : OFF_GB + (m - 2) * CHUNK);
+    }
+    static_assert(D == 64 ? 2 * CHUNK <= T * T * 2 : 4 * CHUNK <= 2 * T * T * 2, "dk staging fits");
     // TMEM columns: P and dP, then dV and dK over them; V G^T; G
     static constexpr uint32_t COL_P = 0, COL_DP = 128, COL_DV = 0, COL_DK = 128, COL_DKI = 256,
                               COL_G = 256 + D, TMEM_COLS = 512;
@@ -867,7 +876,8 @@ struct BwdSmem {
 };
 
 struct BwdParams {
-    CUtensorMap map_q, map_k, map_v, map_dy;
+    CUtensorMap map_q, map_k, map_v, map_dy;  // bf16 operands, box {64, 1, 128, 1}
+    CUtensorMap map_dk, map_dv;               // fp32 outputs, box {32, 1, 128, 1}
     const uint16_t* q;
     const uint16_t* k;
     const uint16_t* v;
@@ -888,6 +898,9 @@ struct BwdParams {
     int64_t B, L, H, n_tiles;
     int G;
     uint64_t wait_ns;
+#ifdef MEMOROID_LA_TRACE
+    unsigned long long* trace;
+#endif
 };
 
 // Reduces 32 values per lane over the warp's 32 lanes; lane l ends with the
@@ -904,6 +917,18 @@ __device__ __forceinline__ float warp_transpose_sum32(float (&v)[32], int lane) 
         }
     }
     return v[0];
+}
+
+// Stores one thread's 16 fp32 values (columns j0..j0+15 of row r) into a
+// 128-byte swizzled staging tile whose 32-channel chunks start at chunk(m).
+template <typename ChunkFn>
+__device__ __forceinline__ void stage_f32x16(unsigned char* smem, ChunkFn chunk, int r, int j0, const float* v) {
+#pragma unroll
+    for (int x = 0; x < 16; x += 4) {
+        const int j = j0 + x;
+        *reinterpret_cast<float4*>(smem + chunk(j >> 5) + r * 128 + ((((j & 31) >> 2) ^ (r & 7)) << 4)) =
+            make_float4(v[x], v[x + 1], v[x + 2], v[x + 3]);
+    }
 }
 
 template <int D>
@@ -929,6 +954,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         }
     }
     const int64_t tile_lo = seg_lo / T, tile_hi = (seg_hi + T - 1) / T;  // tiles [tile_lo, tile_hi)
+    const int64_t row_stride = p.H * D;
 
     uint64_t* bar1 = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
     uint64_t* bar2 = bar1 + 1;
@@ -944,6 +970,9 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
     float* st_x = reinterpret_cast<float*>(smem + S::ST_X);
     float* st_iv = reinterpret_cast<float*>(smem + S::ST_IV);
     float* st_intra = reinterpret_cast<float*>(smem + S::ST_INTRA);
+    float* st_wt = reinterpret_cast<float*>(smem + S::ST_WT);
+    auto dk_chunk = [](int m) { return S::dk_chunk(m); };
+    auto dv_chunk = [](int m) { return S::dv_chunk(m); };
 
     // thread 0: TMA loads of a tile and its metadata, completing on `full`
     auto issue_tile = [&](int64_t tile) {
@@ -966,6 +995,8 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         prefetch_tensormap(&p.map_k);
         prefetch_tensormap(&p.map_v);
         prefetch_tensormap(&p.map_dy);
+        prefetch_tensormap(&p.map_dk);
+        prefetch_tensormap(&p.map_dv);
     }
     if (warp == 0) tc::alloc(tslot, S::TMEM_COLS);
     tc::fence_before();
@@ -1014,6 +1045,11 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
     bool failed = false;
     bool pending = true;  // a tile load may be in flight
     int it = 0;
+#ifdef MEMOROID_LA_TRACE
+    const bool trace_on = blockIdx.x == 0 && tid == 0 && p.trace != nullptr;
+    unsigned long long tr[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    uint64_t tr_last = globaltimer();
+#endif
 #pragma unroll 1
     for (int64_t tile = tile_hi - 1; tile >= tile_lo; --tile, ++it) {
         const int64_t t0 = tile * T;
@@ -1028,6 +1064,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         }
         pending = false;
         tc::fence_after();
+        LA_MARK(0);
         const bool tile_start = mc.has_start != 0;
 
         // ---- B1: P = Q K^T, dP = dY V^T, dKi = V G^T ----
@@ -1045,14 +1082,36 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             }
             tc::commit(bar1);
         }
+        // while B1 runs: the stored state S_{c-1} (this thread's row of <G, S>),
+        // pass F's dgamma term and gamma for the rows of warps 0-3
+        const bool need_iv = have_g && !tile_start;
+        uint32_t sv[SC / 2];
+        if (need_iv && srow >= 0) {
+            const uint16_t* srows = p.states + (bh * p.n_tiles + tile) * D * D;  // S^T, row-major [j][i]
+#pragma unroll
+            for (int x = 0; x < SC; x += 2) {
+                const int j = half * SC + x;
+                sv[x / 2] = static_cast<uint32_t>(srows[j * D + srow]) | (static_cast<uint32_t>(srows[(j + 1) * D + srow]) << 16);
+            }
+        }
+        float dlf = 0.f, gmt = 1.f;
+        if (warp < 4) {
+            const int t = 32 * warp + lane;
+            if (t >= r_lo && t < r_hi) {
+                const int64_t idx = (b * p.L + t0 + t) * p.H + h;
+                dlf = p.dlam_f[idx];
+                if (p.dgamma != nullptr) gmt = p.gamma_per_step ? p.gamma[idx] : p.gamma[h];
+            }
+        }
         ok = wait_mbar(bar1, it & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
             failed = true;
             break;
         }
         tc::fence_after();
+        LA_MARK(1);
 
-        // ---- RP1: masks, E statistics, K~, <G_c, S_{c-1}>, G *= a ----
+        // ---- RP1: masks and E statistics; x_r; <G_c, S_{c-1}> and G *= a ----
         {
             const int t = 32 * quarter + lane;  // the row s of P and dP this thread holds
             const float lt = mc.lam2[t];
@@ -1089,9 +1148,67 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
                 st_col[quarter * T + r0 + lane] = cs;
             }
             st_row[half * T + t] = rsum;
+
+            // x_r = w_out_r k_r . (G_c v_r), from the unscaled K tile
+            float xacc = 0.f;
+            if (have_g) {
+                const unsigned char* kt = smem + S::OFF_K;
+#pragma unroll 1
+                for (int cc = 0; cc < SC / 16; ++cc) {
+                    const int j0 = half * SC + cc * 16;
+                    float gi[16];
+                    tc::ld16(lane_base + S::COL_DKI + j0, gi);
+#pragma unroll
+                    for (int x = 0; x < 16; x += 8) {
+                        const uint4 u = *reinterpret_cast<const uint4*>(kt + sw_off(t, j0 + x));
+                        const float2 k0 = unpack_bf16x2(u.x), k1 = unpack_bf16x2(u.y), k2 = unpack_bf16x2(u.z),
+                                     k3 = unpack_bf16x2(u.w);
+                        xacc = fmaf(k0.x, gi[x], xacc);
+                        xacc = fmaf(k0.y, gi[x + 1], xacc);
+                        xacc = fmaf(k1.x, gi[x + 2], xacc);
+                        xacc = fmaf(k1.y, gi[x + 3], xacc);
+                        xacc = fmaf(k2.x, gi[x + 4], xacc);
+                        xacc = fmaf(k2.y, gi[x + 5], xacc);
+                        xacc = fmaf(k3.x, gi[x + 6], xacc);
+                        xacc = fmaf(k3.y, gi[x + 7], xacc);
+                    }
+                }
+                const float w_out = t >= mc.last_start ? fast_exp2(mc.lam2[T - 1] - mc.lam2[t]) : 0.f;
+                xacc *= w_out;
+            }
+            st_x[half * T + t] = xacc;
         }
         {
-            // K~ = w_out (.) K in place (K is not read unscaled after B1)
+            float ivp = 0.f;
+            const bool scale = have_g && !tile_start && mc.a != 1.f;
+            if (need_iv || scale) {
+#pragma unroll
+                for (int cc = 0; cc < SC / 16; ++cc) {
+                    const int j0 = half * SC + cc * 16;
+                    float v[16];
+                    tc::ld16(lane_base + S::COL_G + j0, v);
+                    if (need_iv && srow >= 0) {
+#pragma unroll
+                        for (int x = 0; x < 16; x += 2) {
+                            const uint32_t w2 = sv[(cc * 16 + x) / 2];
+                            ivp = fmaf(v[x], __uint_as_float(w2 << 16), ivp);
+                            ivp = fmaf(v[x + 1], __uint_as_float(w2 & 0xffff0000u), ivp);
+                        }
+                    }
+                    if (scale) {
+#pragma unroll
+                        for (int x = 0; x < 16; ++x) v[x] *= mc.a;
+                        tc::st16(lane_base + S::COL_G + j0, v);
+                    }
+                }
+            }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) ivp += __shfl_xor_sync(0xffffffffu, ivp, off);
+            if (lane == 0) st_iv[warp] = ivp;
+        }
+        __syncthreads();  // every x_r has read the unscaled K
+        {
+            // K~ = w_out (.) K in place (K is not read unscaled after this)
             unsigned char* kt = smem + S::OFF_K;
             const float lend = mc.lam2[T - 1];
             const int ls = mc.last_start;
@@ -1115,40 +1232,11 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
                 }
             }
         }
-        {
-            // <G_c, S_{c-1}> (tiles without a begin flag) and G <- a_c G
-            float ivp = 0.f;
-            const bool need_iv = have_g && !tile_start;
-            const bool scale = have_g && !tile_start && mc.a != 1.f;
-            if (need_iv || scale) {
-                const uint16_t* srows = p.states + (bh * p.n_tiles + tile) * D * D;  // S^T, row-major [j][i]
-#pragma unroll 1
-                for (int cc = 0; cc < SC / 16; ++cc) {
-                    const int j0 = half * SC + cc * 16;
-                    float v[16];
-                    tc::ld16(lane_base + S::COL_G + j0, v);
-                    if (need_iv && srow >= 0) {
-#pragma unroll
-                        for (int x = 0; x < 16; ++x) {
-                            const uint32_t bits = static_cast<uint32_t>(srows[(j0 + x) * D + srow]) << 16;
-                            ivp = fmaf(v[x], __uint_as_float(bits), ivp);
-                        }
-                    }
-                    if (scale) {
-#pragma unroll
-                        for (int x = 0; x < 16; ++x) v[x] *= mc.a;
-                        tc::st16(lane_base + S::COL_G + j0, v);
-                    }
-                }
-            }
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) ivp += __shfl_xor_sync(0xffffffffu, ivp, off);
-            if (lane == 0) st_iv[warp] = ivp;
-        }
         tc::fence_smem_to_async();
         tc::fence_before();
         __syncthreads();
         tc::fence_after();
+        LA_MARK(2);
 
         // ---- B2: dV = Pm^T dY + K~ G, dK = dPm^T Q ----
         if (tid == 0) {
@@ -1187,12 +1275,27 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
                 run += d[x];
             }
         }
+        // x prefix within each of warps 0-3 (rows 32w..32w+31) while B2 runs
+        float xpre_in = 0.f;
+        if (warp < 4) {
+            const int t = 32 * warp + lane;
+            const float xt = st_x[t] + st_x[T + t];
+            float incl = xt;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const float o = __shfl_up_sync(0xffffffffu, incl, off);
+                if (lane >= off) incl += o;
+            }
+            xpre_in = incl - xt;
+            if (lane == 31) st_wt[warp] = incl;
+        }
         ok = wait_mbar(bar2, it & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
             failed = true;
             break;
         }
         tc::fence_after();
+        LA_MARK(3);
 
         // ---- RP2: Q~ = w_in (.) Q in place, then B3: G += Q~^T dY ----
         {
@@ -1228,15 +1331,12 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
                 tc::mma(tm + S::COL_G, desc_sw_mn(sQ, kk), desc_sw_mn(sDY, kk), ID_QDY, acc || kk > 0);
             tc::commit(bar3);
         }
+        LA_MARK(4);
 
-        // ---- epilogue (while B3 runs): dk, dv, x_r ----
+        // ---- epilogue (while B3 runs): dk = dK + w_out dKi and dv staged for TMA stores ----
         {
             const int r = 32 * quarter + lane;
-            const bool store = r >= r_lo && r < r_hi;
             const float w_out = r >= mc.last_start ? fast_exp2(mc.lam2[T - 1] - mc.lam2[r]) : 0.f;
-            float* dkrow = p.dk + ((b * p.L + t0 + r) * p.H + h) * D;
-            float* dvrow = p.dv + ((b * p.L + t0 + r) * p.H + h) * D;
-            float xacc = 0.f;
 #pragma unroll 1
             for (int cc = 0; cc < SC / 16; ++cc) {
                 const int j0 = half * SC + cc * 16;
@@ -1245,86 +1345,74 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
                 tc::ld16_nowait(lane_base + S::COL_DV + j0, rv);
                 if (have_g) tc::ld16_nowait(lane_base + S::COL_DKI + j0, ri);
                 tc::ld_wait();
-                float ok4[16];
+                float vk[16], vv[16];
 #pragma unroll
                 for (int x = 0; x < 16; ++x) {
-                    const float dki = have_g ? __uint_as_float(ri[x]) : 0.f;
-                    ok4[x] = fmaf(w_out, dki, __uint_as_float(rk[x]));
+                    vk[x] = have_g ? fmaf(w_out, __uint_as_float(ri[x]), __uint_as_float(rk[x])) : __uint_as_float(rk[x]);
+                    vv[x] = __uint_as_float(rv[x]);
                 }
-                if (have_g) {
-                    // x_r = k~_r . dKi_r, with k~ = w_out k (the scaled K tile)
-                    const unsigned char* kt = smem + S::OFF_K;
+                stage_f32x16(smem, dk_chunk, r, j0, vk);
+                stage_f32x16(smem, dv_chunk, r, j0, vv);
+            }
+        }
+        tc::fence_smem_to_async();
+        __syncthreads();
+        if (warp == 0) {
+            const int full_rows = static_cast<int>(min(static_cast<int64_t>(T), p.L - t0));
+            if (r_lo == 0 && r_hi == full_rows) {
+                if (lane == 0) {
 #pragma unroll
-                    for (int x = 0; x < 16; x += 8) {
-                        const uint4 u = *reinterpret_cast<const uint4*>(kt + sw_off(r, j0 + x));
-                        const float2 k0 = unpack_bf16x2(u.x), k1 = unpack_bf16x2(u.y), k2 = unpack_bf16x2(u.z),
-                                     k3 = unpack_bf16x2(u.w);
-                        xacc = fmaf(k0.x, __uint_as_float(ri[x]), xacc);
-                        xacc = fmaf(k0.y, __uint_as_float(ri[x + 1]), xacc);
-                        xacc = fmaf(k1.x, __uint_as_float(ri[x + 2]), xacc);
-                        xacc = fmaf(k1.y, __uint_as_float(ri[x + 3]), xacc);
-                        xacc = fmaf(k2.x, __uint_as_float(ri[x + 4]), xacc);
-                        xacc = fmaf(k2.y, __uint_as_float(ri[x + 5]), xacc);
-                        xacc = fmaf(k3.x, __uint_as_float(ri[x + 6]), xacc);
-                        xacc = fmaf(k3.y, __uint_as_float(ri[x + 7]), xacc);
+                    for (int m = 0; m < D / 32; ++m) {
+                        tma_store_4d(&p.map_dk, sbase + S::dk_chunk(m), 32 * m, static_cast<int>(h), static_cast<int>(t0),
+                                     static_cast<int>(b));
+                        tma_store_4d(&p.map_dv, sbase + S::dv_chunk(m), 32 * m, static_cast<int>(h), static_cast<int>(t0),
+                                     static_cast<int>(b));
                     }
+                    bulk_commit();
                 }
-                if (store) {
-#pragma unroll
-                    for (int x = 0; x < 16; x += 4) {
-                        *reinterpret_cast<float4*>(dkrow + j0 + x) = make_float4(ok4[x], ok4[x + 1], ok4[x + 2], ok4[x + 3]);
-                        *reinterpret_cast<float4*>(dvrow + j0 + x) =
-                            make_float4(__uint_as_float(rv[x]), __uint_as_float(rv[x + 1]), __uint_as_float(rv[x + 2]),
-                                        __uint_as_float(rv[x + 3]));
-                    }
+            } else {
+                float* dkb = p.dk + ((b * p.L + t0) * p.H + h) * D;
+                float* dvb = p.dv + ((b * p.L + t0) * p.H + h) * D;
+                for (int e = lane; e < (r_hi - r_lo) * (D / 4); e += 32) {
+                    const int r = r_lo + e / (D / 4), j = (e % (D / 4)) * 4;
+                    const int in = r * 128 + ((((j & 31) >> 2) ^ (r & 7)) << 4);
+                    *reinterpret_cast<float4*>(dkb + static_cast<int64_t>(r) * row_stride + j) =
+                        *reinterpret_cast<const float4*>(smem + S::dk_chunk(j >> 5) + in);
+                    *reinterpret_cast<float4*>(dvb + static_cast<int64_t>(r) * row_stride + j) =
+                        *reinterpret_cast<const float4*>(smem + S::dv_chunk(j >> 5) + in);
                 }
             }
-            st_x[half * T + r] = xacc;
         }
-        __syncthreads();
-        // ---- dL/dlog(gamma_t) for the tile's rows ----
+        // ---- dL/dlog(gamma_t) for the tile's rows (warps 0-3, one row per thread) ----
         if (warp < 4) {
             const int t = 32 * warp + lane;
-            const float xt = st_x[t] + st_x[T + t];
-            // exclusive prefix of x over the tile: the lower warps' rows, then this warp's
-            float incl = xt;
-#pragma unroll
-            for (int off = 1; off < 32; off <<= 1) {
-                const float o = __shfl_up_sync(0xffffffffu, incl, off);
-                if (lane >= off) incl += o;
-            }
             float lower = 0.f;
-            for (int u = 0; u < 32 * warp; ++u) lower += st_x[u] + st_x[T + u];
-            const float xpre = lower + (incl - xt);
+            for (int w2 = 0; w2 < warp; ++w2) lower += st_wt[w2];
             float iv = 0.f;
             if (!tile_start) {
+#pragma unroll
                 for (int w2 = 0; w2 < 8; ++w2) iv += st_iv[w2];
                 iv *= mc.a;
             }
             const bool in = t >= r_lo && t < r_hi;
             const bool is_start = mc.seg[t] == t;
             float dl = 0.f;
-            if (in && !is_start) {
-                const int64_t idx = (b * p.L + t0 + t) * p.H + h;
-                dl = st_intra[t] + xpre + iv + p.dlam_f[idx];
-                if (p.dgamma != nullptr) {
-                    const float gm = p.gamma_per_step ? p.gamma[idx] : p.gamma[h];
-                    p.dgamma[idx] = dl / gm;
-                }
-            } else if (in && p.dgamma != nullptr) {
-                p.dgamma[(b * p.L + t0 + t) * p.H + h] = 0.f;
-            }
+            if (in && !is_start) dl = st_intra[t] + (lower + xpre_in) + iv + dlf;
+            if (in && p.dgamma != nullptr) p.dgamma[(b * p.L + t0 + t) * p.H + h] = dl / gmt;
             // per-head mode: fixed-order tile total
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) dl += __shfl_xor_sync(0xffffffffu, dl, off);
             if (lane == 0) st_iv[8 + warp] = dl;
         }
+        LA_MARK(5);
         ok = wait_mbar(bar3, it & 1, p.wait_ns);
+        if (tid == 0) bulk_wait_read();  // dv staging in G / K and dk staging are read before reuse
         if (__syncthreads_or(!ok)) {
             failed = true;
             break;
         }
         tc::fence_after();
+        LA_MARK(6);
         if (tid == 0) gsum += (st_iv[8] + st_iv[9]) + (st_iv[10] + st_iv[11]);
         have_g = true;
 
@@ -1354,12 +1442,19 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             if (tid == 0) issue_tile(tile - 1);
             pending = true;
         }
+        LA_MARK(7);
     }
+#ifdef MEMOROID_LA_TRACE
+    if (trace_on) {
+        for (int i = 0; i < 8; ++i) p.trace[8 + i] = tr[i];
+    }
+#endif
     if (failed) {
         if (tid == 0) record_error(p.hdr, DEV_MMA_TIMEOUT);
         // let a load still in flight land before the CTA's shared memory goes away
         if (pending) wait_mbar(full, it & 1, p.wait_ns);
     }
+    if (tid == 0) bulk_wait_all();
     if (tid == 0 && p.gpart != nullptr) p.gpart[bh * p.G + g] = gsum;
     tc::fence_before();
     __syncthreads();
@@ -1666,7 +1761,8 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     // pass R: dk, dv, dgamma, dS0
     BwdParams r;
     if (!tile_map(&r.map_q, a.q, a.B, a.L, a.H, D) || !tile_map(&r.map_k, a.k, a.B, a.L, a.H, D) ||
-        !tile_map(&r.map_v, a.v, a.B, a.L, a.H, D) || !tile_map(&r.map_dy, dy16, a.B, a.L, a.H, D))
+        !tile_map(&r.map_v, a.v, a.B, a.L, a.H, D) || !tile_map(&r.map_dy, dy16, a.B, a.L, a.H, D) ||
+        !tile_map_y(&r.map_dk, a.dk, a.B, a.L, a.H, D) || !tile_map_y(&r.map_dv, a.dv, a.B, a.L, a.H, D))
         return MEMOROID_ERR_CUDA;
     r.q = static_cast<const uint16_t*>(a.q);
     r.k = static_cast<const uint16_t*>(a.k);
@@ -1691,6 +1787,9 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     r.n_tiles = pl.n_tiles;
     r.G = static_cast<int>(pl.G);
     r.wait_ns = debug_knobs().wait_ns;
+#ifdef MEMOROID_LA_TRACE
+    r.trace = la_trace_buffer();
+#endif
     if (set_smem(bwd_kernel<D>, BwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
     bwd_kernel<D><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, BwdSmem<D>::BYTES, stream>>>(r);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
