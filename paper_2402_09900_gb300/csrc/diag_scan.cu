@@ -87,7 +87,7 @@ constexpr int NB_READ = MEMOROID_NODE_BATCH;
 #ifndef MEMOROID_UNROLL_BWD
 #define MEMOROID_UNROLL_BWD 32
 #endif
-constexpr int RED_PARTS = 128;  // first-stage parts of the grad_lambda reduction
+constexpr int RED_PARTS = 512;  // first-stage parts of the grad_lambda reduction
 #ifndef MEMOROID_POLL_SLEEP_NS
 #define MEMOROID_POLL_SLEEP_NS 0  // longest back-off between flag polls
 #endif
@@ -854,24 +854,31 @@ __global__ void __launch_bounds__(256) reduce_parts_kernel(const float4* __restr
     }
 }
 
-__global__ void reduce_final_kernel(const double* __restrict__ rpart, float4* __restrict__ grad_lambda,
-                                    int64_t D2) {
-    const int slab = blockIdx.x, lane = threadIdx.x;
-    double r[4] = {0.0, 0.0, 0.0, 0.0};
-#pragma unroll 16
-    for (int part = 0; part < RED_PARTS; ++part) {
-        const double2* o = reinterpret_cast<const double2*>(
-            rpart + ((static_cast<int64_t>(slab) * RED_PARTS + part) * 32 + lane) * 4);
-        const double2 v0 = o[0], v1 = o[1];
-        r[0] += v0.x;
-        r[1] += v0.y;
-        r[2] += v1.x;
-        r[3] += v1.y;
+// One block of RED_PARTS threads per (slab, lane): thread p holds part p, then
+// a shared-memory tree with a fixed pairing sums the parts.
+__global__ void __launch_bounds__(RED_PARTS) reduce_final_kernel(const double* __restrict__ rpart,
+                                                                 float4* __restrict__ grad_lambda, int64_t D2) {
+    __shared__ double2 s[2][RED_PARTS];
+    const int slab = blockIdx.x >> 5, lane = blockIdx.x & 31, p = threadIdx.x;
+    const double2* o =
+        reinterpret_cast<const double2*>(rpart + ((static_cast<int64_t>(slab) * RED_PARTS + p) * 32 + lane) * 4);
+    s[0][p] = o[0];
+    s[1][p] = o[1];
+    __syncthreads();
+#pragma unroll
+    for (int w = RED_PARTS / 2; w > 0; w >>= 1) {
+        if (p < w) {
+            s[0][p].x += s[0][p + w].x;
+            s[0][p].y += s[0][p + w].y;
+            s[1][p].x += s[1][p + w].x;
+            s[1][p].y += s[1][p + w].y;
+        }
+        __syncthreads();
     }
     const int64_t col = static_cast<int64_t>(slab) * 32 + lane;
-    if (col < D2)
-        grad_lambda[col] = make_float4(static_cast<float>(r[0]), static_cast<float>(r[1]),
-                                       static_cast<float>(r[2]), static_cast<float>(r[3]));
+    if (p == 0 && col < D2)
+        grad_lambda[col] = make_float4(static_cast<float>(s[0][0].x), static_cast<float>(s[0][0].y),
+                                       static_cast<float>(s[1][0].x), static_cast<float>(s[1][0].y));
 }
 
 // ============================================================================
@@ -899,14 +906,18 @@ using BwdS = Cfg<4, 8, true, true>;
 #ifndef MEMOROID_TARGET_SC
 #define MEMOROID_TARGET_SC 512
 #endif
+#ifndef MEMOROID_TARGET_SC_BWD
+#define MEMOROID_TARGET_SC_BWD 256
+#endif
 constexpr int64_t MAX_SEG = 192;
 constexpr int64_t MIN_SEG_TILES = 8;
 
 struct Segs {
     int64_t G, Q;
 };
-Segs choose_segments(int64_t n_chains, int64_t n_tt) {
-    int64_t G = (MEMOROID_TARGET_SC + n_chains - 1) / n_chains;
+Segs choose_segments(int64_t n_chains, int64_t n_tt, bool rev) {
+    const int64_t target = rev ? MEMOROID_TARGET_SC_BWD : MEMOROID_TARGET_SC;
+    int64_t G = (target + n_chains - 1) / n_chains;
     G = lmin(G, lmin(MAX_SEG, n_tt / MIN_SEG_TILES));
     if (G < 1) G = 1;
     const int64_t Q = (n_tt + G - 1) / G;
@@ -919,13 +930,13 @@ struct Layout {
     size_t node_off, gpart_off, fix_off, pin_off, segc_off, sega_off, segb_off, rpart_off, total;
 };
 
-// Workspace layout for tiles of T steps.
-Layout layout(int64_t B, int64_t L, int64_t D, int T) {
+// Workspace layout for tiles of T steps (rev: the backward scan's segment target).
+Layout layout(int64_t B, int64_t L, int64_t D, int T, bool rev) {
     Layout l{};
     l.n_slabs = (D + SLAB - 1) / SLAB;
     l.n_chains = B * l.n_slabs;
     l.n_tt = (L + T - 1) / T;
-    l.sg = choose_segments(l.n_chains, l.n_tt);
+    l.sg = choose_segments(l.n_chains, l.n_tt, rev);
     const size_t tiles = static_cast<size_t>(l.n_chains) * static_cast<size_t>(l.n_tt);
     const size_t nodes = static_cast<size_t>(l.n_chains) * static_cast<size_t>(l.sg.G * l.sg.Q);
     l.node_off = kHeaderBytes;
@@ -991,7 +1002,7 @@ Params make_params(const Args& a, const Layout& l, int T, bool backward) {
 // state entering each segment where it is missing.
 template <class C>
 memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
-    const Layout l = layout(a.B, a.L, a.D, C::T);
+    const Layout l = layout(a.B, a.L, a.D, C::T, C::REV);
     const Segs sg = l.sg;
     const int64_t n_tickets = sg.Q * l.n_chains * sg.G;
     if (n_tickets >= 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;
@@ -1017,8 +1028,10 @@ memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t D) {
     size_t m = 0;
-    for (int T : {FwdC::T, FwdS::T, BwdC::T, BwdS::T}) {
-        const size_t t = layout(B, L, D, T).total;
+    const int Ts[4] = {FwdC::T, FwdS::T, BwdC::T, BwdS::T};
+    const bool revs[4] = {false, false, true, true};
+    for (int i = 0; i < 4; ++i) {
+        const size_t t = layout(B, L, D, Ts[i], revs[i]).total;
         if (t > m) m = t;
     }
     return m;
@@ -1034,7 +1047,7 @@ extern "C" int memoroid_trace_set_buffer(void* dev_ptr) {
 int kernels_per_call(int64_t B, int64_t L, int64_t D, int per_step, int backward, int with_grad_lambda) {
     if (B <= 0 || L <= 0 || D <= 0) return 0;
     const int T = backward ? (per_step ? BwdS::T : BwdC::T) : (per_step ? FwdS::T : FwdC::T);
-    const Layout l = layout(B, L, D, T);
+    const Layout l = layout(B, L, D, T, backward != 0);
     int n = l.sg.G > 1 ? 3 : 1;  // scan [+ segment carries + fix-up]
     if (backward && !per_step && with_grad_lambda) n += 2;  // grad_lambda reduction
     return n;
@@ -1055,7 +1068,7 @@ memoroid_status_t launch_bwd(const Args& a, cudaStream_t s) {
         double* rpart = reinterpret_cast<double*>(ws + l.rpart_off);
         reduce_parts_kernel<<<dim3(static_cast<unsigned>(l.n_slabs), RED_PARTS), 256, 0, s>>>(
             gpart, rpart, a.B, l.n_slabs, l.n_tt);
-        reduce_final_kernel<<<static_cast<unsigned>(l.n_slabs), 32, 0, s>>>(
+        reduce_final_kernel<<<static_cast<unsigned>(l.n_slabs * 32), RED_PARTS, 0, s>>>(
             rpart, static_cast<float4*>(a.grad_lambda), a.D / 2);
         if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     }
