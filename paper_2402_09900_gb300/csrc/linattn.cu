@@ -276,6 +276,37 @@ __device__ __forceinline__ void tma_tile(uint32_t dst, const CUtensorMap* map, i
         tma_load_4d(dst + m * T * 128, map, 64 * m, static_cast<int>(h), static_cast<int>(t0), static_cast<int>(b), bar);
 }
 
+// Scales row r of a 128-byte swizzled [T x D] bf16 tile by w[r] in place: one
+// thread per (row, 64-channel chunk) while there are enough threads, each
+// with one weight and eight 16-byte units (conflict-free: the swizzle spreads
+// the same unit of 8 consecutive rows over 8 bank groups).
+template <int D, typename WFn>
+__device__ __forceinline__ void scale_rows_sw(unsigned char* tile, int tid, WFn weight) {
+    constexpr int CHUNKS = D / 64;
+    constexpr int UNITS = 8 * CHUNKS * T / kThreads;  // units per thread: 8 (d = 128) or 4 (d = 64)
+    const int r = tid & (T - 1);
+    const float w = weight(r);
+    if (w == 1.f) return;
+    unsigned char* row = tile + r * 128;
+#pragma unroll
+    for (int i = 0; i < UNITS; ++i) {
+        // thread tid covers units (tid / T) * UNITS + i of its row (chunk = unit / 8)
+        const int unit = (tid / T) * UNITS + i;
+        unsigned char* a = row + (unit >> 3) * (T * 128) + (((unit & 7) ^ (r & 7)) << 4);
+        uint4 u = *reinterpret_cast<uint4*>(a);
+        float2 f;
+        f = unpack_bf16x2(u.x);
+        u.x = pack_bf16x2(f.x * w, f.y * w);
+        f = unpack_bf16x2(u.y);
+        u.y = pack_bf16x2(f.x * w, f.y * w);
+        f = unpack_bf16x2(u.z);
+        u.z = pack_bf16x2(f.x * w, f.y * w);
+        f = unpack_bf16x2(u.w);
+        u.w = pack_bf16x2(f.x * w, f.y * w);
+        *reinterpret_cast<uint4*>(a) = u;
+    }
+}
+
 __device__ __forceinline__ bool wait_mbar(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer();
@@ -555,7 +586,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         tc::fence_after();
         LA_MARK(0);
         if (c + 1 < nt) {
-            if (tid == 0) issue_tile(c + 1, s ^ 1, c + 2 < nt ? c + 2 : -1, -1);
+            if (tid == 32) issue_tile(c + 1, s ^ 1, c + 2 < nt ? c + 2 : -1, -1);
             pending = c + 1;
         }
 
@@ -607,29 +638,10 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         LA_MARK(3);
         // ---- K~[r] = exp2(lam2_end - lam2_r) K[r] for rows of the last episode ----
         {
-            unsigned char* kt = smem + (stage_k(s) - sbase);
             const float lend = mc.lam2[T - 1];
             const int ls = mc.last_start;
-            constexpr int NCH = T * D / 8;
-#pragma unroll 2
-            for (int e = tid; e < NCH; e += kThreads) {
-                // e enumerates 16-byte units in memory order: 8 per 128-byte row
-                const int r = (e >> 3) & (T - 1);
-                const float w = r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f;
-                if (w != 1.f) {
-                    uint4 u = *reinterpret_cast<uint4*>(kt + e * 16);
-                    float2 f;
-                    f = unpack_bf16x2(u.x);
-                    u.x = pack_bf16x2(f.x * w, f.y * w);
-                    f = unpack_bf16x2(u.y);
-                    u.y = pack_bf16x2(f.x * w, f.y * w);
-                    f = unpack_bf16x2(u.z);
-                    u.z = pack_bf16x2(f.x * w, f.y * w);
-                    f = unpack_bf16x2(u.w);
-                    u.w = pack_bf16x2(f.x * w, f.y * w);
-                    *reinterpret_cast<uint4*>(kt + e * 16) = u;
-                }
-            }
+            scale_rows_sw<D>(smem + (stage_k(s) - sbase), tid,
+                             [&](int r) { return r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f; });
         }
         tc::fence_smem_to_async();
         tc::fence_before();
@@ -1209,28 +1221,9 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         __syncthreads();  // every x_r has read the unscaled K
         {
             // K~ = w_out (.) K in place (K is not read unscaled after this)
-            unsigned char* kt = smem + S::OFF_K;
             const float lend = mc.lam2[T - 1];
             const int ls = mc.last_start;
-            constexpr int NCH = T * D / 8;
-#pragma unroll 2
-            for (int e = tid; e < NCH; e += kThreads) {
-                const int r = (e >> 3) & (T - 1);
-                const float w = r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f;
-                if (w != 1.f) {
-                    uint4 u = *reinterpret_cast<uint4*>(kt + e * 16);
-                    float2 f;
-                    f = unpack_bf16x2(u.x);
-                    u.x = pack_bf16x2(f.x * w, f.y * w);
-                    f = unpack_bf16x2(u.y);
-                    u.y = pack_bf16x2(f.x * w, f.y * w);
-                    f = unpack_bf16x2(u.z);
-                    u.z = pack_bf16x2(f.x * w, f.y * w);
-                    f = unpack_bf16x2(u.w);
-                    u.w = pack_bf16x2(f.x * w, f.y * w);
-                    *reinterpret_cast<uint4*>(kt + e * 16) = u;
-                }
-            }
+            scale_rows_sw<D>(smem + S::OFF_K, tid, [&](int r) { return r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f; });
         }
         tc::fence_smem_to_async();
         tc::fence_before();
@@ -1298,28 +1291,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         LA_MARK(3);
 
         // ---- RP2: Q~ = w_in (.) Q in place, then B3: G += Q~^T dY ----
-        {
-            unsigned char* qt = smem + S::OFF_Q;
-            constexpr int NCH = T * D / 8;
-#pragma unroll 2
-            for (int e = tid; e < NCH; e += kThreads) {
-                const int r = (e >> 3) & (T - 1);
-                const float w = mc.seg[r] < 0 ? fast_exp2(mc.lam2[r]) : 0.f;
-                if (w != 1.f) {
-                    uint4 u = *reinterpret_cast<uint4*>(qt + e * 16);
-                    float2 f;
-                    f = unpack_bf16x2(u.x);
-                    u.x = pack_bf16x2(f.x * w, f.y * w);
-                    f = unpack_bf16x2(u.y);
-                    u.y = pack_bf16x2(f.x * w, f.y * w);
-                    f = unpack_bf16x2(u.z);
-                    u.z = pack_bf16x2(f.x * w, f.y * w);
-                    f = unpack_bf16x2(u.w);
-                    u.w = pack_bf16x2(f.x * w, f.y * w);
-                    *reinterpret_cast<uint4*>(qt + e * 16) = u;
-                }
-            }
-        }
+        scale_rows_sw<D>(smem + S::OFF_Q, tid, [&](int r) { return mc.seg[r] < 0 ? fast_exp2(mc.lam2[r]) : 0.f; });
         tc::fence_smem_to_async();
         tc::fence_before();
         __syncthreads();
