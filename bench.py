@@ -87,6 +87,8 @@ def linattn_leg(args, m, dev, stream):
 
     c = tapegen.LINATTN_CONFIGS[LA_CFG]
     B, L, H, d = c["B"], c["L"], c["H"], c["d"]
+    if args.la_tape_steps:
+        L = args.la_tape_steps  # a shorter tape of the same workload (profiler captures)
     t = tapegen.linattn_tape_device(B, L, H, d, tapegen.seed_for(LA_CFG), c["mean"], c["gamma"], device=dev)
     per = 1 if t["gamma"].dim() == 3 else 0
     ws = m.linattn_workspace(B, L, H, d, dev)
@@ -102,7 +104,7 @@ def linattn_leg(args, m, dev, stream):
         m.memoroid_scan_linattn_bwd(t["q"], t["k"], t["v"], m.MEMOROID_BF16, t["gamma"], per, t["start"], None,
                                     t["grad_y"], None, dq, dk, dv, dg, None, B, L, H, d, d, c["chunk"], ws, stream)
 
-    for _ in range(3):
+    for _ in range(args.la_warmup):
         fwd()
         bwd()
     torch.cuda.synchronize()
@@ -147,7 +149,8 @@ def linattn_leg(args, m, dev, stream):
     i_tf = ctas * reps * 4 * 128 * 128 * d / (i_ms * 1e-3) / 1e12
     burst, sustained, tkind = _tensor_peaks()
     out = {
-        "workload": LA_WORKLOAD, "value": B * L / ((f_ms + b_ms) * 1e-3), "unit": UNIT, "steps": steps,
+        "workload": LA_WORKLOAD if not args.la_tape_steps else f"{LA_WORKLOAD} (first {L} steps only)",
+        "value": B * L / ((f_ms + b_ms) * 1e-3), "unit": UNIT, "steps": steps,
         "ms_per_step": f_ms + b_ms, "fwd_ms": f_ms, "bwd_ms": b_ms,
         "episodes": int(t["start"].sum().item()),
         "roofline": {"bound": "hbm", "peak": peak, "unit": "GB/s", "peak_kind": f"{peak_kind} (copy bandwidth)",
@@ -334,6 +337,10 @@ def run_ours(args):
     native_build.build()
     from paper_2402_09900_gb300 import memoroid as m
     m.load()
+    if args.only_linattn:
+        # profiling mode: the linattn leg alone (no diag step, no JSON contract line)
+        print(json.dumps({"linattn": linattn_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
+        return
 
     t = tapegen.diag_config(CFG)
     if args.tape_steps:
@@ -499,6 +506,11 @@ def main():
     ap.add_argument("--skip-cpu-baseline", action="store_true")
     ap.add_argument("--skip-linattn", action="store_true", help="omit the linear-attention leg")
     ap.add_argument("--la-steps", type=int, default=10, help="timed linattn fwd+bwd steps")
+    ap.add_argument("--la-warmup", type=int, default=3, help="untimed linattn fwd+bwd steps")
+    ap.add_argument("--la-tape-steps", type=int, default=0,
+                    help="linattn tape length (profiler captures); 0 = the full L = 2^22 workload")
+    ap.add_argument("--only-linattn", action="store_true",
+                    help="profiling mode: run and print only the linattn leg")
     ap.add_argument("--la-intra-reps", type=int, default=2000,
                     help="repetitions of the intra-tile contraction per CTA in the tensor benchmark")
     ap.add_argument("--tape-steps", type=int, default=0,
