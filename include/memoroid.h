@@ -266,9 +266,12 @@ memoroid_status_t memoroid_get_device_error(const void *workspace, void *stream)
  * (0 restores the default of 1 s).  Applies to later calls. */
 void memoroid_debug_set_wait_limit_ns(uint64_t ns);
 
-/* Fault injection for tests: the tile with this scheduling ticket skips
- * publishing its look-back status, so its successor's wait runs out
- * (-1 = off, the default).  Applies to later scan calls. */
+/* Fault injection for tests (-1 = off, the default; applies to later calls):
+ * in the diagonal scan the tile with this scheduling ticket skips publishing
+ * its look-back status, so its successor's wait runs out; in the linear-
+ * attention kernels the CTA with this index treats its first tensor-core wait
+ * as timed out (it drains its in-flight work, records MEMOROID_ERR_TIMEOUT in
+ * the workspace and stops). */
 void memoroid_debug_withhold_tile(int64_t ticket);
 
 #ifdef __cplusplus

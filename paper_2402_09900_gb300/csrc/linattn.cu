@@ -37,6 +37,9 @@ namespace la {
 using namespace ptx;
 
 constexpr int T = 128;         // steps per tile = the M of the tile contractions
+// After a wait has run out, in-flight TMA loads and tensor-core batches are
+// drained with this fixed limit before the CTA frees its TMEM and exits.
+constexpr uint64_t kDrainNs = 1000000000ull;
 constexpr int kThreads = 256;  // 8 warps: warp w reads TMEM lane quarter w % 4, column half w / 4
 constexpr int kTargetCtas = 152;
 
@@ -361,6 +364,7 @@ struct FwdParams {
     int64_t B, L, H, n_tiles, tps;
     int G;
     uint64_t wait_ns;
+    int64_t fail_cta;  // test knob: this CTA reports its first tensor-core wait as timed out (-1: none)
     // backward pass F only (see fwd_kernel<D, true>)
     const uint16_t* zq;  // q, bf16 [B, L, H, D]
     float* dlam_f;       // [B, L, H]: the state-side terms of dL/dlog(gamma_t)
@@ -562,7 +566,9 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     constexpr uint32_t ID_KV = tc::idesc_bf16(D, D, true, true);
 
     bool failed = __syncthreads_or(!first_ok);
-    int pending = failed ? -1 : 0;  // the last issued tile whose load may still be in flight
+    int pending = 0;       // the last issued tile whose load may still be in flight (-1: none)
+    int drain_bar = 0;     // 1 / 2: the batch on bar1 / bar2 was issued but not seen complete
+    uint32_t drain_par = 0;
 #ifdef MEMOROID_LA_TRACE
     const bool trace_on = blockIdx.x == 0 && tid == 0 && p.trace != nullptr;
     unsigned long long tr[8] = {0, 0, 0, 0, 0, 0, 0, 0};
@@ -604,9 +610,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             tc::commit(bar1);
         }
         LA_MARK(1);
-        ok = wait_mbar(bar1, c & 1, p.wait_ns);
+        ok = wait_mbar(bar1, c & 1, p.wait_ns) && !(c == 0 && static_cast<int64_t>(blockIdx.x) == p.fail_cta);
         if (__syncthreads_or(!ok)) {
             failed = true;
+            drain_bar = 1;
+            drain_par = c & 1;
             break;
         }
         tc::fence_after();
@@ -664,6 +672,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         ok = wait_mbar(bar2, c & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
             failed = true;
+            drain_bar = 2;
+            drain_par = c & 1;
             break;
         }
         tc::fence_after();
@@ -825,8 +835,10 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     }
     if (failed) {
         if (tid == 0) record_error(p.hdr, DEV_MMA_TIMEOUT);
-        // let a load still in flight land before the CTA's shared memory goes away
-        if (pending >= 0) wait_mbar(&full[pending & 1], (pending >> 1) & 1, p.wait_ns);
+        // let work still in flight finish before the CTA's TMEM and shared memory go away
+        if (drain_bar == 1) wait_mbar(bar1, drain_par, kDrainNs);
+        if (drain_bar == 2) wait_mbar(bar2, drain_par, kDrainNs);
+        if (pending >= 0) wait_mbar(&full[pending & 1], (pending >> 1) & 1, kDrainNs);
     }
     if (warp == 0) bulk_wait_all();
 #ifdef MEMOROID_LA_TRACE
@@ -910,6 +922,7 @@ struct BwdParams {
     int64_t B, L, H, n_tiles;
     int G;
     uint64_t wait_ns;
+    int64_t fail_cta;  // test knob (see FwdParams)
 #ifdef MEMOROID_LA_TRACE
     unsigned long long* trace;
 #endif
@@ -1056,6 +1069,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
     float gsum = 0.f;  // per-head mode: sum of dL/dlog(gamma) over the segment's steps
     bool failed = false;
     bool pending = true;  // a tile load may be in flight
+    uint64_t* drain = nullptr;  // a batch issued but not seen complete
     int it = 0;
 #ifdef MEMOROID_LA_TRACE
     const bool trace_on = blockIdx.x == 0 && tid == 0 && p.trace != nullptr;
@@ -1115,9 +1129,10 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
                 if (p.dgamma != nullptr) gmt = p.gamma_per_step ? p.gamma[idx] : p.gamma[h];
             }
         }
-        ok = wait_mbar(bar1, it & 1, p.wait_ns);
+        ok = wait_mbar(bar1, it & 1, p.wait_ns) && !(it == 0 && static_cast<int64_t>(blockIdx.x) == p.fail_cta);
         if (__syncthreads_or(!ok)) {
             failed = true;
+            drain = bar1;
             break;
         }
         tc::fence_after();
@@ -1285,6 +1300,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         ok = wait_mbar(bar2, it & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
             failed = true;
+            drain = bar2;
             break;
         }
         tc::fence_after();
@@ -1381,6 +1397,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         if (tid == 0) bulk_wait_read();  // dv staging in G / K and dk staging are read before reuse
         if (__syncthreads_or(!ok)) {
             failed = true;
+            drain = bar3;
             break;
         }
         tc::fence_after();
@@ -1423,8 +1440,9 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
 #endif
     if (failed) {
         if (tid == 0) record_error(p.hdr, DEV_MMA_TIMEOUT);
-        // let a load still in flight land before the CTA's shared memory goes away
-        if (pending) wait_mbar(full, it & 1, p.wait_ns);
+        // let work still in flight finish before the CTA's TMEM and shared memory go away
+        if (drain != nullptr) wait_mbar(drain, it & 1, kDrainNs);
+        if (pending) wait_mbar(full, it & 1, kDrainNs);
     }
     if (tid == 0) bulk_wait_all();
     if (tid == 0 && p.gpart != nullptr) p.gpart[bh * p.G + g] = gsum;
@@ -1511,6 +1529,7 @@ __global__ void __launch_bounds__(128, 1) intra_bench_kernel(const uint4* __rest
         tc::commit(&bar);
     }
     const bool ok = wait_mbar(&bar, 0, wait_ns);
+    if (!ok) wait_mbar(&bar, 0, kDrainNs);  // the contractions finish before TMEM is freed
     tc::fence_after();
     if (!ok && tid == 0) record_error(hdr, DEV_MMA_TIMEOUT);
     if (ok) {
@@ -1670,6 +1689,7 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     p.tps = pl.tps;
     p.G = static_cast<int>(pl.G);
     p.wait_ns = debug_knobs().wait_ns;
+    p.fail_cta = debug_knobs().withhold_ticket;
     p.zq = nullptr;
     p.dlam_f = nullptr;
     p.states = nullptr;
@@ -1720,6 +1740,7 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     f.tps = pl.tps;
     f.G = static_cast<int>(pl.G);
     f.wait_ns = debug_knobs().wait_ns;
+    f.fail_cta = debug_knobs().withhold_ticket;
     f.zq = static_cast<const uint16_t*>(a.q);
     f.dlam_f = dlam_f;
     f.states = states;
@@ -1759,6 +1780,7 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     r.n_tiles = pl.n_tiles;
     r.G = static_cast<int>(pl.G);
     r.wait_ns = debug_knobs().wait_ns;
+    r.fail_cta = debug_knobs().withhold_ticket;
 #ifdef MEMOROID_LA_TRACE
     r.trace = la_trace_buffer();
 #endif

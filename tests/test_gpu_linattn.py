@@ -278,3 +278,29 @@ def test_config5_sampled_episodes():
                                ("dv", dv[:, sl], rv), ("dgamma", dg[:, sl], rg)):
             worst[name] = max(worst.get(name, 0.0), rel_err(got.cpu().numpy(), ref))
     assert all(v <= TOL for v in worst.values()), worst
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_injected_wait_failure_reported_then_recovers(d):
+    # CTA 0 treats its first tensor-core wait as timed out: it drains its
+    # in-flight work, records the error and stops; no GPU fault, and the next
+    # calls on the same context are correct again
+    m = _m()
+    t = tapegen.linattn_tape(1, 3000, 2, d, d, seed=tapegen.seed_for(61 + d), mean=300.0, with_grad=True)
+    q, k, v = bits_dev(t["q"]), bits_dev(t["k"]), bits_dev(t["v"])
+    gamma, start = dev(t["gamma"]), dev(t["start"])
+    ws = m.linattn_workspace(1, 3000, 2, d, "cuda")
+    m.memoroid_debug_withhold_tile(0)
+    try:
+        m.linattn_fwd(q, k, v, gamma, start, ws=ws)
+        fwd_status = m.memoroid_get_device_error(ws)
+        m.linattn_bwd(q, k, v, gamma, start, dev(t["grad_y"]), ws=ws)
+        bwd_status = m.memoroid_get_device_error(ws)
+    finally:
+        m.memoroid_debug_withhold_tile(-1)
+    assert fwd_status == m.MEMOROID_ERR_TIMEOUT
+    assert bwd_status == m.MEMOROID_ERR_TIMEOUT
+    y, S_last = run_gpu_fwd(t, ws=ws)
+    y_ref, S_ref = run_oracle_fwd(t)
+    assert rel_err(y, y_ref) <= TOL and rel_err(S_last, S_ref) <= TOL
+    check_bwd(t)
