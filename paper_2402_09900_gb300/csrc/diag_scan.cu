@@ -76,7 +76,7 @@ constexpr int SLAB = 64;  // complex channels per slab
 // the summary's range) and is recomputed by the reader.
 constexpr int NODE_WORDS = 8;
 #ifndef MEMOROID_NODE_BATCH
-#define MEMOROID_NODE_BATCH 2  // summaries read per round trip in a look-back fold
+#define MEMOROID_NODE_BATCH 1  // summaries read per round trip in a look-back fold
 #endif
 constexpr int NB_READ = MEMOROID_NODE_BATCH;
 // Unroll factors of the per-step loops (measured: unrolling helps the
