@@ -73,6 +73,8 @@ def lib():
             L.oracle_linattn_fwd.argtypes = [_i64] * 5 + [_p] * 4 + [_c.c_int] + [_p] * 4
             L.oracle_linattn_bwd.argtypes = [_i64] * 5 + [_p] * 4 + [_c.c_int] + [_p] * 9
             L.oracle_starts_from_offsets.argtypes = [_p, _i64, _i64, _p]
+            L.oracle_discounted_return.argtypes = [_i64, _i64, _p, _p, _c.c_double, _p, _p]
+            L.oracle_gae.argtypes = [_i64, _i64, _p, _p, _p, _c.c_double, _c.c_double, _p, _p]
             L.oracle_offsets_from_starts.argtypes = [_p, _i64, _p]
             L.oracle_offsets_from_starts.restype = _i64
             L.oracle_set_threads.argtypes = [_c.c_int]
@@ -236,6 +238,29 @@ def linattn_bwd(q, k, v, gamma, start, dy, dS_last=None, S0=None, gamma_per_step
 # ---------------------------------------------------------------------------
 # episode index list <-> begin flags
 # ---------------------------------------------------------------------------
+
+def discounted_return(r, start, gamma, boot=None):
+    """G [B, L]: per-step discounted return within episodes (boot: [B] value
+    after the tape's last step, or None)."""
+    r = _f64(r)
+    B, L = r.shape
+    start = _u8(start)
+    boot = _f64(boot)
+    G = np.zeros((B, L), dtype=np.float64)
+    _check(lib().oracle_discounted_return(B, L, _ptr(r), _ptr(start), float(gamma), _ptr(boot), _ptr(G)))
+    return G
+
+
+def gae(r, v, start, gamma, lam, v_boot=None):
+    """A [B, L]: per-step generalised advantage estimate within episodes."""
+    r, v = _f64(r), _f64(v)
+    B, L = r.shape
+    start = _u8(start)
+    v_boot = _f64(v_boot)
+    A = np.zeros((B, L), dtype=np.float64)
+    _check(lib().oracle_gae(B, L, _ptr(r), _ptr(v), _ptr(start), float(gamma), float(lam), _ptr(v_boot), _ptr(A)))
+    return A
+
 
 def starts_from_offsets(offsets, L):
     offsets = np.ascontiguousarray(offsets, dtype=np.int64)

@@ -18,7 +18,11 @@
  *     "Linear Recurrent Unit");
  *   - the Linear Transformer sum monoid (X + X') (Appendix "Linear
  *     Transformer"), generalised with a per-step decay gamma_t that multiplies
- *     the carried state, read out as y_t = S_t^T q_t.
+ *     the carried state, read out as y_t = S_t^T q_t;
+ *   - the discounted-return and GAE memoroids (a, r) . (a', r') =
+ *     (a a', a r' + r), f = (gamma, r) resp. (gamma lambda, delta) (Appendix
+ *     "The Discounted Return as a Memoroid" and "The Generalized Advantage
+ *     Estimate as a Memoroid"), evaluated for every step of every episode.
  *
  * Conventions (readings of the paper, listed in the design notes):
  *   - b_t = 1 on the first step of an episode (Section 2.1).
@@ -416,4 +420,72 @@ int64_t oracle_offsets_from_starts(const uint8_t *start, int64_t L, int64_t *off
         if (start[t]) offsets[n++] = t;
     }
     return n;
+}
+
+
+/* ------------------------------------------------------------------------ */
+/* Discounted return and GAE per step, reset at episode boundaries           */
+/* ------------------------------------------------------------------------ */
+/*
+ * The return memoroid folds (1,0) . (gamma, r_t) . (gamma, r_{t+1}) . ... and
+ * its second element is sum_l gamma^l r_{t+l}; evaluated for every step t of
+ * an episode it is the suffix sum
+ *     G_t = sum_{l = 0}^{e - 1 - t} gamma^l r_{t+l}        (episode [s, e))
+ * i.e. G_t = r_t + gamma G_{t+1} inside the episode and G_{e-1} = r_{e-1}.
+ * The tape's last episode may be cut: if boot is given, G_{L-1} = r_{L-1} +
+ * gamma boot[b] (the value of the state after the tape).
+ * r, G: [B, L]; start: [B, L] (1 on the first step of an episode); boot: [B] or NULL.
+ */
+int oracle_discounted_return(int64_t B, int64_t L, const double *r, const uint8_t *start, double gamma,
+                             const double *boot, double *G)
+{
+    if (B < 0 || L < 0) return -1;
+    for (int64_t b = 0; b < B; ++b) {
+        /* episodes in reverse: e is one past the last step */
+        int64_t e = L;
+        while (e > 0) {
+            int64_t s = e - 1;
+            while (s > 0 && !start[b * L + s]) --s;
+            double next = (e == L && boot) ? boot[b] : 0.0;
+            for (int64_t t = e - 1; t >= s; --t) {
+                const double g = r[b * L + t] + gamma * next;
+                G[b * L + t] = g;
+                next = g;
+            }
+            e = s;
+        }
+    }
+    return 0;
+}
+
+/*
+ * GAE per step: A_t = sum_{l = 0}^{e - 1 - t} (gamma lambda)^l delta_{t+l} with
+ *     delta_t = r_t + gamma V_{t+1} - V_t,
+ * where V_{t+1} is the value of the next step of the same episode, 0 after an
+ * episode's last step (the episode ended), and v_boot[b] after the tape's last
+ * step when given (the cut episode continues).
+ * r, v, A: [B, L]; v_boot: [B] or NULL.
+ */
+int oracle_gae(int64_t B, int64_t L, const double *r, const double *v, const uint8_t *start, double gamma,
+               double lambda, const double *v_boot, double *A)
+{
+    if (B < 0 || L < 0) return -1;
+    for (int64_t b = 0; b < B; ++b) {
+        int64_t e = L;
+        while (e > 0) {
+            int64_t s = e - 1;
+            while (s > 0 && !start[b * L + s]) --s;
+            double next_v = (e == L && v_boot) ? v_boot[b] : 0.0;
+            double next_a = 0.0;
+            for (int64_t t = e - 1; t >= s; --t) {
+                const double delta = r[b * L + t] + gamma * next_v - v[b * L + t];
+                const double a = delta + gamma * lambda * next_a;
+                A[b * L + t] = a;
+                next_a = a;
+                next_v = v[b * L + t];
+            }
+            e = s;
+        }
+    }
+    return 0;
 }

@@ -517,3 +517,102 @@ def test_offsets_round_trip_random():
         offs = oracle.offsets_from_starts(start)
         np.testing.assert_array_equal(offs, np.flatnonzero(start))
         np.testing.assert_array_equal(oracle.starts_from_offsets(offs, L), start)
+
+
+# ---------------------------------------------------------------------------
+# discounted return and GAE memoroids (appendix "The Discounted Return as a
+# Memoroid" and "The Generalized Advantage Estimate as a Memoroid")
+# ---------------------------------------------------------------------------
+
+def _ret_combine(x, y):
+    # (a, r) . (a', r') = (a a', a r' + r), the left operand earlier in time
+    return (x[0] * y[0], x[0] * y[1] + x[1])
+
+
+def test_return_golden_worked_example():
+    rows = np.loadtxt(os.path.join(GOLDEN, "return_expansion.txt"))
+    r = rows[:, 1][None, :]
+    start = rows[:, 2].astype(np.uint8)[None, :]
+    G = oracle.discounted_return(r, start, 0.5)
+    assert np.array_equal(G[0], rows[:, 3])
+
+
+def test_return_equals_memoroid_fold_at_episode_heads():
+    rng = np.random.default_rng(41)
+    gamma = 0.9
+    r = rng.standard_normal((3, 200))
+    start = np.stack([tapegen.geometric_tape_starts(rng, 200, 15.0) for _ in range(3)])
+    G = oracle.discounted_return(r, start, gamma)
+    for b in range(3):
+        for s, e in tapegen.episode_bounds(start[b]):
+            acc = (1.0, 0.0)  # e_I
+            for t in range(s, e):
+                acc = _ret_combine(acc, (gamma, r[b, t]))
+            assert acc[0] == pytest.approx(gamma ** (e - s), rel=1e-12)
+            assert G[b, s] == pytest.approx(acc[1], rel=1e-12, abs=1e-12)
+
+
+def test_return_brute_force_suffix_sums_with_bootstrap():
+    rng = np.random.default_rng(42)
+    gamma = 0.8
+    r = rng.standard_normal((2, 60))
+    start = np.stack([tapegen.geometric_tape_starts(rng, 60, 8.0) for _ in range(2)])
+    boot = rng.standard_normal(2)
+    G = oracle.discounted_return(r, start, gamma, boot)
+    for b in range(2):
+        bounds = tapegen.episode_bounds(start[b])
+        for s, e in bounds:
+            for t in range(s, e):
+                want = sum(gamma ** (l - t) * r[b, l] for l in range(t, e))
+                if e == 60:
+                    want += gamma ** (e - t) * boot[b]
+                assert G[b, t] == pytest.approx(want, rel=1e-12, abs=1e-12)
+
+
+def test_return_matches_reverse_diagonal_scan():
+    # the return is the diagonal backward recurrence with a real multiplier:
+    # delta_t = g_t + [b_{t+1} = 0] gamma delta_{t+1}, g_last = gamma * boot
+    rng = np.random.default_rng(43)
+    gamma = 0.95
+    B, L = 2, 300
+    r = rng.standard_normal((B, L))
+    start = np.stack([tapegen.geometric_tape_starts(rng, L, 30.0) for _ in range(B)])
+    boot = rng.standard_normal(B)
+    G = oracle.discounted_return(r, start, gamma, boot)
+    lam = np.full(2, gamma, dtype=np.complex128)
+    g = np.zeros((B, L, 2), dtype=np.complex128)
+    g[:, :, 0] = r
+    h = np.zeros_like(g)
+    g_last = np.zeros((B, 2), dtype=np.complex128)
+    g_last[:, 0] = gamma * boot
+    gu, _, _ = oracle.diag_bwd(lam, start, h, g, g_last)
+    assert np.allclose(gu[:, :, 0].real, G, rtol=1e-12, atol=1e-12)
+
+
+def test_gae_special_cases_and_brute_force():
+    rng = np.random.default_rng(44)
+    gamma, lam = 0.9, 0.7
+    B, L = 2, 80
+    r = rng.standard_normal((B, L))
+    v = rng.standard_normal((B, L))
+    start = np.stack([tapegen.geometric_tape_starts(rng, L, 10.0) for _ in range(B)])
+    v_boot = rng.standard_normal(B)
+    # delta_t = r_t + gamma V_{t+1} - V_t (V after an episode's end: 0; after the tape: v_boot)
+    delta = np.zeros((B, L))
+    for b in range(B):
+        for s, e in tapegen.episode_bounds(start[b]):
+            for t in range(s, e):
+                nv = v[b, t + 1] if t + 1 < e else (v_boot[b] if e == L else 0.0)
+                delta[b, t] = r[b, t] + gamma * nv - v[b, t]
+    # lambda = 0: one-step TD error
+    assert np.allclose(oracle.gae(r, v, start, gamma, 0.0, v_boot), delta, rtol=1e-12, atol=1e-12)
+    # lambda = 1: the discounted return (bootstrapped by v_boot) minus the value
+    G = oracle.discounted_return(r, start, gamma, v_boot)
+    assert np.allclose(oracle.gae(r, v, start, gamma, 1.0, v_boot), G - v, rtol=1e-10, atol=1e-10)
+    # general lambda: sum_l (gamma lambda)^l delta_{t+l} within the episode
+    A = oracle.gae(r, v, start, gamma, lam, v_boot)
+    for b in range(B):
+        for s, e in tapegen.episode_bounds(start[b]):
+            for t in range(s, e):
+                want = sum((gamma * lam) ** (l - t) * delta[b, l] for l in range(t, e))
+                assert A[b, t] == pytest.approx(want, rel=1e-12, abs=1e-12)
