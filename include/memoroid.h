@@ -216,6 +216,42 @@ memoroid_status_t memoroid_scan_linattn_bwd(const void *q, const void *k, const 
                                             int64_t dv, int64_t chunk, void *workspace,
                                             size_t workspace_bytes, void *stream);
 
+/* ======================================================================== */
+/* Discounted return and GAE memoroids (appendices "The Discounted Return   */
+/* as a Memoroid" and "The Generalized Advantage Estimate as a Memoroid"):  */
+/* (a, r) . (a', r') = (a a', a r' + r), evaluated for every step of every  */
+/* episode of the tape, i.e. the reverse recurrences                        */
+/*   G_t = r_t + gamma [b_{t+1} = 0] G_{t+1}                                */
+/*   A_t = delta_t + gamma lambda [b_{t+1} = 0] A_{t+1},                    */
+/*   delta_t = r_t + gamma V_{t+1} - V_t,                                   */
+/* where V_{t+1} is 0 after an episode's last step and the tape's last step */
+/* continues into boot / v_boot when given (a cut episode).                 */
+/* ======================================================================== */
+
+/* Workspace bytes for memoroid_discounted_return and memoroid_gae. */
+size_t memoroid_returns_workspace_bytes(int64_t B, int64_t L);
+
+/*
+ *   r      fp32 [B, L] rewards
+ *   start  uint8 [B, L], nonzero = first step of an episode
+ *   boot   fp32 [B]: the return after each tape's last step, or NULL (= 0)
+ *   G      fp32 [B, L] output (may not alias r)
+ * Device memory owned by the caller; workspace 256-byte aligned, at least
+ * memoroid_returns_workspace_bytes.  Asynchronous on `stream`.
+ */
+memoroid_status_t memoroid_discounted_return(const float *r, const uint8_t *start, float gamma,
+                                             const float *boot, float *G, int64_t B, int64_t L,
+                                             void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ *   r, v   fp32 [B, L] rewards and values V(s_t)
+ *   v_boot fp32 [B]: V of the state after each tape's last step, or NULL (= 0)
+ *   A      fp32 [B, L] output (may not alias r or v)
+ */
+memoroid_status_t memoroid_gae(const float *r, const float *v, const uint8_t *start, float gamma,
+                               float lambda, const float *v_boot, float *A, int64_t B, int64_t L,
+                               void *workspace, size_t workspace_bytes, void *stream);
+
 /* ------------------------------------------------------------------------ */
 /* Measurement only (the paper has no counterpart): throughput of the        */
 /* intra-tile tensor-core contraction of memoroid_scan_linattn_fwd alone.    */

@@ -357,4 +357,39 @@ memoroid_status_t memoroid_bench_linattn_intra(int64_t d, int64_t reps, int64_t 
     return la::launch_intra_bench(d, reps, ctas, scratch, as_stream(stream));
 }
 
+// ---------------------------------------------------------------------------
+// discounted return and GAE
+// ---------------------------------------------------------------------------
+
+size_t memoroid_returns_workspace_bytes(int64_t B, int64_t L) {
+    if (B < 0 || L < 0) return 0;
+    return ret::workspace_bytes(B, L);
+}
+
+static memoroid_status_t returns_common(const float* r, const float* v, const uint8_t* start, float c, float gamma,
+                                        const float* boot, float* out, int64_t B, int64_t L, void* workspace,
+                                        size_t workspace_bytes, void* stream) {
+    if (B < 0 || L < 0) return MEMOROID_ERR_INVALID_ARG;
+    if (B == 0 || L == 0) return MEMOROID_OK;
+    if (!r || !start || !out) return MEMOROID_ERR_INVALID_ARG;
+    if (!aligned(r, 4) || !aligned(out, 4) || (v && !aligned(v, 4)) || (boot && !aligned(boot, 4)))
+        return MEMOROID_ERR_INVALID_ARG;
+    if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < ret::workspace_bytes(B, L))
+        return MEMOROID_ERR_WORKSPACE;
+    return ret::launch(r, v, start, c, gamma, boot, out, B, L, workspace, as_stream(stream));
+}
+
+memoroid_status_t memoroid_discounted_return(const float* r, const uint8_t* start, float gamma, const float* boot,
+                                             float* G, int64_t B, int64_t L, void* workspace,
+                                             size_t workspace_bytes, void* stream) {
+    return returns_common(r, nullptr, start, gamma, gamma, boot, G, B, L, workspace, workspace_bytes, stream);
+}
+
+memoroid_status_t memoroid_gae(const float* r, const float* v, const uint8_t* start, float gamma, float lambda,
+                               const float* v_boot, float* A, int64_t B, int64_t L, void* workspace,
+                               size_t workspace_bytes, void* stream) {
+    if (v == nullptr && B > 0 && L > 0) return MEMOROID_ERR_INVALID_ARG;
+    return returns_common(r, v, start, gamma * lambda, gamma, v_boot, A, B, L, workspace, workspace_bytes, stream);
+}
+
 }  // extern "C"

@@ -1646,6 +1646,17 @@ bool tile_map_y(CUtensorMap* m, const void* base, int64_t B, int64_t L, int64_t 
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+}  // namespace
+
+memoroid_status_t launch_segment_plan(const uint8_t* start, int64_t B, int64_t L, int64_t seg_len, int64_t G,
+                                      int64_t* first, cudaStream_t stream) {
+    if (B * G == 0) return MEMOROID_OK;
+    const int64_t blocks = (B * G * 32 + 255) / 256;
+    plan_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(start, B, L, seg_len, G, first);
+    return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
+}
+
+namespace {
 // Tile metadata and segment boundaries (shared by the forward and backward passes).
 memoroid_status_t launch_prep(const Args& a, const Plan& pl, TileMeta* meta, int64_t* seg_first,
                               cudaStream_t stream) {

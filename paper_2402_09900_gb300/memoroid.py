@@ -54,6 +54,9 @@ SIGNATURES = {
                                          _i64, _i64, _i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_bench_linattn_intra_scratch_bytes": (_sz, [_i64]),
     "memoroid_bench_linattn_intra": (_int, [_i64, _i64, _i64, _p, _sz, _p]),
+    "memoroid_returns_workspace_bytes": (_sz, [_i64, _i64]),
+    "memoroid_discounted_return": (_int, [_p, _p, ctypes.c_float, _p, _p, _i64, _i64, _p, _sz, _p]),
+    "memoroid_gae": (_int, [_p, _p, _p, ctypes.c_float, ctypes.c_float, _p, _p, _i64, _i64, _p, _sz, _p]),
     "memoroid_starts_from_offsets": (_int, [_p, _i64, _i64, _p, _p]),
     "memoroid_offsets_workspace_bytes": (_sz, [_i64]),
     "memoroid_offsets_from_starts": (_int, [_p, _i64, _p, _p, _p, _sz, _p]),
@@ -202,6 +205,24 @@ def memoroid_bench_linattn_intra(d, reps, ctas, scratch, stream=None):
            "memoroid_bench_linattn_intra")
 
 
+def memoroid_returns_workspace_bytes(B, L) -> int:
+    return int(load().memoroid_returns_workspace_bytes(B, L))
+
+
+def memoroid_discounted_return(r, start, gamma, boot, G, B, L, workspace, stream=None):
+    _need_cuda(r, start, boot, G, workspace)
+    _check(load().memoroid_discounted_return(_ptr(r), _ptr(start), float(gamma), _ptr(boot), _ptr(G), B, L,
+                                             _ptr(workspace), workspace.numel() if workspace is not None else 0,
+                                             _stream(stream)), "memoroid_discounted_return")
+
+
+def memoroid_gae(r, v, start, gamma, lam, v_boot, A, B, L, workspace, stream=None):
+    _need_cuda(r, v, start, v_boot, A, workspace)
+    _check(load().memoroid_gae(_ptr(r), _ptr(v), _ptr(start), float(gamma), float(lam), _ptr(v_boot), _ptr(A), B, L,
+                               _ptr(workspace), workspace.numel() if workspace is not None else 0, _stream(stream)),
+           "memoroid_gae")
+
+
 def memoroid_starts_from_offsets(offsets, E, L, start, stream=None):
     _need_cuda(offsets, start)
     _check(load().memoroid_starts_from_offsets(_ptr(offsets), E, L, _ptr(start), _stream(stream)),
@@ -306,6 +327,26 @@ def linattn_bwd(q, k, v, gamma, start, grad_y, grad_S_last=None, S0=None, want_g
     memoroid_scan_linattn_bwd(q, k, v, MEMOROID_BF16, gamma, per_step, start, S0, grad_y, grad_S_last, dq, dk, dv,
                               dgamma, dS0, B, L, H, d, d, chunk, ws, stream)
     return dq, dk, dv, dgamma, dS0
+
+
+def discounted_return(r, start, gamma, boot=None, ws=None, stream=None):
+    """G [B, L]: per-step discounted return within episodes."""
+    B, L = r.shape
+    if ws is None:
+        ws = workspace(memoroid_returns_workspace_bytes(B, L), r.device)
+    G = torch.empty_like(r)
+    memoroid_discounted_return(r, start, gamma, boot, G, B, L, ws, stream)
+    return G
+
+
+def gae(r, v, start, gamma, lam, v_boot=None, ws=None, stream=None):
+    """A [B, L]: per-step generalised advantage estimate within episodes."""
+    B, L = r.shape
+    if ws is None:
+        ws = workspace(memoroid_returns_workspace_bytes(B, L), r.device)
+    A = torch.empty_like(r)
+    memoroid_gae(r, v, start, gamma, lam, v_boot, A, B, L, ws, stream)
+    return A
 
 
 def starts_from_offsets(offsets, L, stream=None):
