@@ -9,6 +9,8 @@ decayed linear-attention memoroid on the largest linattn tape (L = 2^22,
 8 heads, d = 128, per-step gamma, Geometric(1000) episodes): one step =
 memoroid_scan_linattn_fwd + memoroid_scan_linattn_bwd, plus the tensor-core
 throughput of the intra-tile contraction alone (memoroid_bench_linattn_intra).
+Its "returns" object times the per-step discounted return and GAE with resets
+on 64 tapes of 2^20 steps.
 
   python bench.py [--gpus N --steps K --warmup W] [--impl reference]
 
@@ -78,6 +80,51 @@ def _tensor_peaks():
         return float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
     except Exception:
         return 1900.0, 1700.0, "fallback"
+
+
+RET_WORKLOAD = ("per-step discounted return and GAE with resets: B=64 tapes x L=2^20 steps (64 Mi steps), "
+                "fp32 rewards and values, Geometric(200) episodes, gamma=0.99, lambda=0.95")
+
+
+def returns_leg(args, m, dev, stream):
+    """Times memoroid_discounted_return and memoroid_gae on 64 tapes of 2^20 steps."""
+    import torch
+
+    B, L = 64, 1 << 20
+    rng = np.random.default_rng(tapegen.seed_for(6))
+    start = np.stack([tapegen.geometric_tape_starts(rng, L, 200.0) for _ in range(B)])
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(tapegen.seed_for(6))
+    r = torch.randn((B, L), generator=gen, device=dev, dtype=torch.float32)
+    v = torch.randn((B, L), generator=gen, device=dev, dtype=torch.float32)
+    st = torch.from_numpy(start).to(dev)
+    boot = torch.randn(B, generator=gen, device=dev, dtype=torch.float32)
+    ws = m.workspace(m.memoroid_returns_workspace_bytes(B, L), dev)
+    G = torch.empty_like(r)
+    A = torch.empty_like(r)
+    out = {"workload": RET_WORKLOAD}
+    peak, peak_kind = _peaks()
+    for name, fn, byts in (
+            ("return", lambda: m.memoroid_discounted_return(r, st, 0.99, boot, G, B, L, ws, stream), B * L * 9 + B * 4),
+            ("gae", lambda: m.memoroid_gae(r, v, st, 0.99, 0.95, boot, A, B, L, ws, stream), B * L * 13 + B * 4)):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.ret_steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / args.ret_steps
+        gbs = byts / (ms * 1e-3) / 1e9
+        out[name] = {"value": B * L / (ms * 1e-3), "unit": "steps/s", "ms": ms,
+                     "roofline": {"bound": "hbm", "algorithmic_bytes_per_call": byts, "achieved": gbs, "unit": "GB/s",
+                                  "peak": peak, "frac": gbs / peak, "peak_kind": f"{peak_kind} (copy bandwidth)"}}
+    out["gpu_launches"] = 2 * args.ret_steps  # one scan launch per call
+    del r, v, G, A, ws
+    torch.cuda.empty_cache()
+    return out
 
 
 def linattn_leg(args, m, dev, stream):
@@ -341,6 +388,10 @@ def run_ours(args):
         # profiling mode: the linattn leg alone (no diag step, no JSON contract line)
         print(json.dumps({"linattn": linattn_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
         return
+    if args.only_returns:
+        # profiling mode: the discounted-return / GAE leg alone
+        print(json.dumps({"returns": returns_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
+        return
 
     t = tapegen.diag_config(CFG)
     if args.tape_steps:
@@ -471,6 +522,9 @@ def run_ours(args):
     la = None
     if ws == 1 and not args.skip_linattn:
         la = linattn_leg(args, m, dev, stream)
+    rt = None
+    if ws == 1 and not args.skip_returns:
+        rt = returns_leg(args, m, dev, stream)
     cpu = None
     if ws == 1 and not args.skip_cpu_baseline:
         cpu = cpu_baseline(t, args.cpu_seconds)
@@ -486,6 +540,7 @@ def run_ours(args):
                                       + m.memoroid_scan_diag_kernels_per_call(B, L, D, 0, 1, 1)),
         "clocks": clocks,
         "linattn": la,
+        "returns": rt,
     }
     print(json.dumps(out), flush=True)
     if ws > 1:
@@ -511,6 +566,10 @@ def main():
                     help="linattn tape length (profiler captures); 0 = the full L = 2^22 workload")
     ap.add_argument("--only-linattn", action="store_true",
                     help="profiling mode: run and print only the linattn leg")
+    ap.add_argument("--skip-returns", action="store_true", help="omit the discounted-return / GAE leg")
+    ap.add_argument("--only-returns", action="store_true",
+                    help="profiling mode: run and print only the discounted-return / GAE leg")
+    ap.add_argument("--ret-steps", type=int, default=20, help="timed calls of each returns kernel")
     ap.add_argument("--la-intra-reps", type=int, default=2000,
                     help="repetitions of the intra-tile contraction per CTA in the tensor benchmark")
     ap.add_argument("--tape-steps", type=int, default=0,

@@ -228,7 +228,8 @@ memoroid_status_t memoroid_scan_linattn_bwd(const void *q, const void *k, const 
 /* continues into boot / v_boot when given (a cut episode).                 */
 /* ======================================================================== */
 
-/* Workspace bytes for memoroid_discounted_return and memoroid_gae. */
+/* Workspace bytes for memoroid_discounted_return and memoroid_gae (a small
+ * reserved block: each call is one kernel launch that keeps no state in it). */
 size_t memoroid_returns_workspace_bytes(int64_t B, int64_t L);
 
 /*

@@ -110,3 +110,41 @@ def test_deterministic():
     a = m.gae(dev(r), dev(v), dev(start), 0.99, 0.95, dev(boot)).cpu().numpy()
     b = m.gae(dev(r), dev(v), dev(start), 0.99, 0.95, dev(boot)).cpu().numpy()
     assert np.array_equal(a, b)
+
+
+def _offset(a, k):
+    # the same values at a base address k elements past an allocation's start
+    flat = torch.zeros(a.size + k, dtype=getattr(torch, str(a.dtype))).cuda()
+    out = flat[k:].view(a.shape)
+    out.copy_(torch.from_numpy(np.ascontiguousarray(a)))
+    return out
+
+
+@pytest.mark.parametrize("k", [1, 3])
+def test_unaligned_base_pointers(k):
+    # tapes whose length is a multiple of 8 but whose buffers start off a 16-byte boundary
+    m = _m()
+    r, v, start, boot = tape(3, 4096, 40.0, tapegen.seed_for(603 + k))
+    G = m.discounted_return(_offset(r, k), _offset(start, k), 0.98, dev(boot))
+    A = m.gae(_offset(r, k), _offset(v, k), _offset(start, k), 0.98, 0.9, dev(boot))
+    torch.cuda.synchronize()
+    assert rel_err(G.cpu().numpy(), oracle.discounted_return(r, start, 0.98, boot)) <= TOL
+    assert rel_err(A.cpu().numpy(), oracle.gae(r, v, start, 0.98, 0.9, boot)) <= TOL
+
+
+def test_full_size_tape_set():
+    # the measured workload: 64 tapes of 2^20 steps, episode lengths geometric with
+    # mean 200 (Bernoulli(1/200) begin flags); four tapes checked against the oracle
+    m = _m()
+    B, L, p = 64, 1 << 20, 1.0 / 200.0
+    rng = np.random.default_rng(tapegen.seed_for(604))
+    r = rng.standard_normal((B, L), dtype=np.float32)
+    v = rng.standard_normal((B, L), dtype=np.float32)
+    boot = rng.standard_normal(B).astype(np.float32)
+    start = (rng.random((B, L)) < p).astype(np.uint8)
+    start[:, 0] = 1
+    G = m.discounted_return(dev(r), dev(start), 0.99, dev(boot)).cpu().numpy()
+    A = m.gae(dev(r), dev(v), dev(start), 0.99, 0.95, dev(boot)).cpu().numpy()
+    rows = [0, 17, 40, 63]
+    assert rel_err(G[rows], oracle.discounted_return(r[rows], start[rows], 0.99, boot[rows])) <= TOL
+    assert rel_err(A[rows], oracle.gae(r[rows], v[rows], start[rows], 0.99, 0.95, boot[rows])) <= TOL
