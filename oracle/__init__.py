@@ -20,6 +20,16 @@ Parity status of each routine (what pins it, in tests/test_oracle_pins.py):
                      matmul, all-start tapes
   linattn_bwd        torch.autograd (fp64), finite differences
   starts/offsets     the tape example of Figure 2, numpy.flatnonzero
+  discounted_return  the appendix expansion worked by hand, the fold at each
+                     episode head, brute-force suffix sums, diag_bwd with a
+                     real multiplier
+  gae                brute-force sums of (gamma lambda)^l delta, lambda = 0
+                     (TD error) and lambda = 1 (return minus value)
+  ffm_fwd            the original FFM aggregator in closed form (Gamma(t)
+                     powers), diag_fwd with lambda_ij and broadcast input,
+                     all-start tapes
+  ffm_bwd            torch.autograd (fp64) through an independent loop,
+                     central finite differences in alpha and omega
 """
 from __future__ import annotations
 
@@ -76,6 +86,8 @@ def lib():
             L.oracle_discounted_return.argtypes = [_i64, _i64, _p, _p, _c.c_double, _p, _p]
             L.oracle_gae.argtypes = [_i64, _i64, _p, _p, _p, _c.c_double, _c.c_double, _p, _p]
             L.oracle_offsets_from_starts.argtypes = [_p, _i64, _p]
+            L.oracle_ffm_fwd.argtypes = [_i64] * 4 + [_p] * 7
+            L.oracle_ffm_bwd.argtypes = [_i64] * 4 + [_p] * 11
             L.oracle_offsets_from_starts.restype = _i64
             L.oracle_set_threads.argtypes = [_c.c_int]
             L.oracle_max_threads.restype = _c.c_int
@@ -260,6 +272,40 @@ def gae(r, v, start, gamma, lam, v_boot=None):
     A = np.zeros((B, L), dtype=np.float64)
     _check(lib().oracle_gae(B, L, _ptr(r), _ptr(v), _ptr(start), float(gamma), float(lam), _ptr(v_boot), _ptr(A)))
     return A
+
+
+def ffm_fwd(alpha, omega, xt, start, S0=None):
+    """Fast and Forgetful Memory memoroid.  alpha [m], omega [c], xt [B, L, m]
+    (the cell's gated input x~), start [B, L], S0 [B, m, c] complex or None.
+    Returns z [B, L, 2*m*c] (Re(X_t) || Im(X_t), each flattened i*c + j) and
+    S_last [B, m, c] complex."""
+    alpha, omega, xt = _f64(alpha), _f64(omega), _f64(xt)
+    B, L, m = xt.shape
+    c = omega.shape[0]
+    start = _u8(start)
+    S0 = _c128(S0)
+    z = np.zeros((B, L, 2 * m * c), dtype=np.float64)
+    S_last = np.zeros((B, m, c), dtype=np.complex128)
+    _check(lib().oracle_ffm_fwd(B, L, m, c, _ptr(alpha), _ptr(omega), _ptr(xt), _ptr(start), _ptr(S0),
+                                _ptr(z), _ptr(S_last)))
+    return z, S_last
+
+
+def ffm_bwd(alpha, omega, start, z, grad_z, grad_S_last=None, S0=None):
+    """Reverse-mode of ffm_fwd: returns grad_xt [B, L, m], grad_alpha [m],
+    grad_omega [c], grad_S0 [B, m, c] complex."""
+    alpha, omega, z, grad_z = _f64(alpha), _f64(omega), _f64(z), _f64(grad_z)
+    m, c = alpha.shape[0], omega.shape[0]
+    B, L = z.shape[0], z.shape[1]
+    start = _u8(start)
+    S0, grad_S_last = _c128(S0), _c128(grad_S_last)
+    gx = np.zeros((B, L, m), dtype=np.float64)
+    ga = np.zeros(m, dtype=np.float64)
+    go = np.zeros(c, dtype=np.float64)
+    gS0 = np.zeros((B, m, c), dtype=np.complex128)
+    _check(lib().oracle_ffm_bwd(B, L, m, c, _ptr(alpha), _ptr(omega), _ptr(start), _ptr(S0), _ptr(z),
+                                _ptr(grad_z), _ptr(grad_S_last), _ptr(gx), _ptr(ga), _ptr(go), _ptr(gS0)))
+    return gx, ga, go, gS0
 
 
 def starts_from_offsets(offsets, L):

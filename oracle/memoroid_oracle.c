@@ -38,6 +38,7 @@
  * i.e. C99 double complex.
  */
 #include <complex.h>
+#include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -487,5 +488,150 @@ int oracle_gae(int64_t B, int64_t L, const double *r, const double *v, const uin
             e = s;
         }
     }
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Fast and Forgetful Memory as a memoroid (Appendix "Fast and Forgetful     */
+/* Memory"):                                                                */
+/*   H = {(X, t)}, X complex m x c, t integer;  e_I = (0, 0);               */
+/*   (X, t) . (X', t') = (X (.) exp(t' (-|alpha| (+) i omega)) + X', t + t')  */
+/*   f(o, b) = (the m-vector x~ repeated over the c columns, 1).             */
+/* (+) is the outer sum: entry (i, j) of the exponent is t'(-|alpha_i| +    */
+/* i omega_j).  The cell's readout takes Re(X) || Im(X), each flattened     */
+/* row-major (i * c + j).  Made resettable by Theorem 3.2 (a begin flag     */
+/* replaces the left operand by e_I).                                        */
+/* ------------------------------------------------------------------------ */
+
+/* (X, t) . (X', t') for one entry (i, j) of the state */
+static void ffm_combine(cplx X, int64_t t, cplx Xp, int64_t tp, double alpha_i, double omega_j,
+                        cplx *out, int64_t *t_out)
+{
+    *out = X * cexp((double)tp * (-fabs(alpha_i) + I * omega_j)) + Xp;
+    *t_out = t + tp;
+}
+
+/*
+ * Forward: the state after every step, by folding the resettable combine
+ * from e_I over the lifted steps f(o_t, b_t) = (x~_t repeated, 1).
+ * xt: [B, L, m]; start: [B, L]; S0: [B, m*c] complex or NULL (the state
+ * before step 0 of a row that continues an episode); z: [B, L, 2*m*c] =
+ * Re(X_t) || Im(X_t); S_last: [B, m*c] complex or NULL.
+ */
+int oracle_ffm_fwd(int64_t B, int64_t L, int64_t m, int64_t c, const double *alpha, const double *omega,
+                   const double *xt, const uint8_t *start, const cplx *S0, double *z, cplx *S_last)
+{
+    if (B < 0 || L < 0 || m < 0 || c < 0) return -1;
+    const int64_t D = m * c;
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int64_t b = 0; b < B; ++b) {
+        for (int64_t ij = 0; ij < D; ++ij) {
+            const int64_t i = ij / c, j = ij % c;
+            cplx X = S0 ? S0[b * D + ij] : 0.0; /* e_I unless the row continues an episode */
+            int64_t tc = 0;
+            for (int64_t t = 0; t < L; ++t) {
+                const cplx Xp = xt[(b * L + t) * m + i];
+                if (start[b * L + t]) { /* Theorem 3.2: the left operand becomes e_I = (0, 0) */
+                    X = 0.0;
+                    tc = 0;
+                }
+                cplx nx;
+                int64_t nt;
+                ffm_combine(X, tc, Xp, 1, alpha[i], omega[j], &nx, &nt);
+                X = nx;
+                tc = nt;
+                z[(b * L + t) * 2 * D + ij] = creal(X);
+                z[(b * L + t) * 2 * D + D + ij] = cimag(X);
+            }
+            if (S_last) S_last[b * D + ij] = X;
+        }
+    }
+    return 0;
+}
+
+/*
+ * Backward (reverse-mode of the forward above).  With lambda_ij =
+ * exp(-|alpha_i| + i omega_j) and the upstream G_t = dL/dRe X_t + i dL/dIm X_t
+ * (read from grad_z's two halves), the adjoint of X_t is
+ *     delta_t = G_t + [b_{t+1} = 0] conj(lambda) delta_{t+1},
+ *     delta_{L-1} = G_{L-1} + grad_S_last,
+ * and
+ *     grad_xt[t, i]  = sum_j Re(delta_t[i, j])          (x~ enters every column)
+ *     grad_lambda_ij = sum_{t: b_t = 0} delta_t conj(X_{t-1})  (X_{-1} = S0 or 0)
+ *     grad_alpha_i   = sum_j Re(conj(grad_lambda_ij) * (-sign(alpha_i)) lambda_ij)
+ *     grad_omega_j   = sum_i Re(conj(grad_lambda_ij) * i lambda_ij)
+ *     grad_S0        = [b_0 = 0] conj(lambda) delta_0.
+ * z is the forward's output (X_t as Re || Im).  Outputs may be NULL.
+ */
+int oracle_ffm_bwd(int64_t B, int64_t L, int64_t m, int64_t c, const double *alpha, const double *omega,
+                   const uint8_t *start, const cplx *S0, const double *z, const double *grad_z,
+                   const cplx *grad_S_last, double *grad_xt, double *grad_alpha, double *grad_omega,
+                   cplx *grad_S0)
+{
+    if (B < 0 || L < 0 || m < 0 || c < 0) return -1;
+    const int64_t D = m * c;
+    cplx *glam = (cplx *)calloc((size_t)(D > 0 ? D : 1), sizeof(cplx));
+    if (!glam) return -2;
+    if (grad_xt) memset(grad_xt, 0, sizeof(double) * (size_t)(B * L * m));
+#pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < m; ++i) {
+        for (int64_t j = 0; j < c; ++j) {
+            const int64_t ij = i * c + j;
+            const cplx lam = cexp(-fabs(alpha[i]) + I * omega[j]);
+            cplx gl = 0.0;
+            for (int64_t b = 0; b < B; ++b) {
+                cplx dn = 0.0; /* delta_{t+1} */
+                for (int64_t t = L - 1; t >= 0; --t) {
+                    const double *gz = grad_z + (b * L + t) * 2 * D;
+                    cplx d = gz[ij] + I * gz[D + ij];
+                    if (t == L - 1) {
+                        if (grad_S_last) d += grad_S_last[b * D + ij];
+                    } else if (!start[b * L + t + 1]) {
+                        d += conj(lam) * dn;
+                    }
+                    /* each (t, i) row is written by this thread only (it owns i) */
+                    if (grad_xt) grad_xt[(b * L + t) * m + i] += creal(d);
+                    if (!start[b * L + t]) {
+                        cplx prev;
+                        if (t > 0) {
+                            const double *zp = z + (b * L + t - 1) * 2 * D;
+                            prev = zp[ij] + I * zp[D + ij];
+                        } else {
+                            prev = S0 ? S0[b * D + ij] : 0.0;
+                        }
+                        gl += d * conj(prev);
+                    }
+                    dn = d;
+                }
+                if (grad_S0) {
+                    grad_S0[b * D + ij] = (L > 0 && !start[b * L]) ? conj(lam) * dn
+                                                                   : (L == 0 && grad_S_last ? grad_S_last[b * D + ij] : 0.0);
+                }
+            }
+            glam[ij] = gl;
+        }
+    }
+    if (grad_alpha) {
+        for (int64_t i = 0; i < m; ++i) {
+            const double sg = alpha[i] > 0 ? 1.0 : (alpha[i] < 0 ? -1.0 : 0.0);
+            double acc = 0.0;
+            for (int64_t j = 0; j < c; ++j) {
+                const cplx lam = cexp(-fabs(alpha[i]) + I * omega[j]);
+                acc += creal(conj(glam[i * c + j]) * (-sg) * lam);
+            }
+            grad_alpha[i] = acc;
+        }
+    }
+    if (grad_omega) {
+        for (int64_t j = 0; j < c; ++j) {
+            double acc = 0.0;
+            for (int64_t i = 0; i < m; ++i) {
+                const cplx lam = cexp(-fabs(alpha[i]) + I * omega[j]);
+                acc += creal(conj(glam[i * c + j]) * I * lam);
+            }
+            grad_omega[j] = acc;
+        }
+    }
+    free(glam);
     return 0;
 }

@@ -616,3 +616,160 @@ def test_gae_special_cases_and_brute_force():
             for t in range(s, e):
                 want = sum((gamma * lam) ** (l - t) * delta[b, l] for l in range(t, e))
                 assert A[b, t] == pytest.approx(want, rel=1e-12, abs=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# Fast and Forgetful Memory (Appendix "Fast and Forgetful Memory")
+# ---------------------------------------------------------------------------
+
+def _ffm_inputs(rng, B, L, m, c, p=0.15, first=True):
+    alpha = rng.uniform(-0.3, 0.3, m)  # signed: the memoroid uses |alpha|
+    omega = rng.uniform(-np.pi, np.pi, c)
+    xt = rng.standard_normal((B, L, m))
+    start = _random_starts(rng, B, L, p, first=first)
+    S0 = _rand_c(rng, B, m, c)
+    return alpha, omega, xt, start, S0
+
+
+def _planar(X):
+    # Re(X) || Im(X), each flattened (i * c + j)
+    B, L, m, c = X.shape
+    return np.concatenate([X.real.reshape(B, L, m * c), X.imag.reshape(B, L, m * c)], axis=-1)
+
+
+def _ffm_aggregator(alpha, omega, xt, start, S0):
+    # The original FFM aggregator in closed form, episode by episode: for an
+    # episode that starts at step k, row i of the aggregator gives
+    #   S_{k+i} = Gamma(i + 1) * S_{k-1} + Gamma(i - t) * sum_{j<=i} Gamma(t - j) * (o_{k+j} 1^T)
+    # with Gamma(tau)[a, b] = exp(-tau (|alpha_a| + i w_b)) and t the episode's
+    # last row.  The aggregator's Gamma carries exp(-i tau w) while the
+    # memoroid's multiplier is exp(+i omega): w = -omega.  The positive powers
+    # Gamma(i - t) for i < t are what the memoroid form avoids; at these sizes
+    # they are exact enough in fp64.
+    B, L, m = xt.shape
+    c = omega.shape[0]
+    w = -omega
+    expo = np.abs(alpha)[:, None] + 1j * w[None, :]
+
+    def gamma(tau):
+        return np.exp(-tau * expo)
+
+    X = np.zeros((B, L, m, c), dtype=np.complex128)
+    for b in range(B):
+        for s, e in tapegen.episode_bounds(start[b]):
+            prev = S0[b] if (s == 0 and not start[b, 0]) else np.zeros((m, c), np.complex128)
+            t = e - 1 - s
+            for i in range(e - s):
+                acc = np.zeros((m, c), np.complex128)
+                for j in range(i + 1):
+                    acc += gamma(t - j) * np.repeat(xt[b, s + j][:, None], c, axis=1)
+                X[b, s + i] = gamma(i + 1) * prev + gamma(i - t) * acc
+    return X
+
+
+@pytest.mark.parametrize("first", [True, False])
+def test_ffm_fwd_matches_aggregator_closed_form(first):
+    rng = _rng(60)
+    B, L, m, c = 2, 40, 3, 4
+    alpha, omega, xt, start, S0 = _ffm_inputs(rng, B, L, m, c, 0.12, first=first)
+    z, S_last = oracle.ffm_fwd(alpha, omega, xt, start, S0)
+    X = _ffm_aggregator(alpha, omega, xt, start, S0)
+    np.testing.assert_allclose(z, _planar(X), rtol=1e-10, atol=1e-10)
+    np.testing.assert_allclose(S_last, X[:, -1], rtol=1e-10, atol=1e-10)
+
+
+def test_ffm_is_diag_scan_with_outer_sum_multiplier():
+    # lambda_ij = exp(-|alpha_i| + i omega_j) per channel, input x~_i in every column
+    rng = _rng(61)
+    B, L, m, c = 2, 50, 4, 3
+    alpha, omega, xt, start, S0 = _ffm_inputs(rng, B, L, m, c, 0.1, first=False)
+    lam = np.exp(-np.abs(alpha)[:, None] + 1j * omega[None, :]).reshape(m * c)
+    u = np.repeat(xt[..., None], c, axis=-1).reshape(B, L, m * c).astype(np.complex128)
+    h, hl = oracle.diag_fwd(lam, u, start, S0.reshape(B, m * c))
+    z, S_last = oracle.ffm_fwd(alpha, omega, xt, start, S0)
+    np.testing.assert_allclose(z, np.concatenate([h.real, h.imag], axis=-1), rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(S_last.reshape(B, m * c), hl, rtol=1e-12, atol=1e-12)
+
+
+def test_ffm_all_start_is_broadcast_input():
+    rng = _rng(62)
+    B, L, m, c = 1, 9, 2, 5
+    alpha, omega, xt, _, S0 = _ffm_inputs(rng, B, L, m, c)
+    start = np.ones((B, L), np.uint8)
+    z, _ = oracle.ffm_fwd(alpha, omega, xt, start, S0)
+    D = m * c
+    np.testing.assert_array_equal(z[..., :D], np.repeat(xt[..., None], c, axis=-1).reshape(B, L, D))
+    np.testing.assert_array_equal(z[..., D:], 0.0)
+
+
+def _torch_ffm_loss(torch, alpha, omega, xt, start, S0, gz, gSl):
+    # independent loop: X_t = lambda * X_{t-1} + x~_t (columns), X_t = x~_t at begin flags;
+    # loss = <gz, Re || Im> + Re(conj(gSl) X_last)
+    B, L, m = xt.shape
+    c = omega.shape[0]
+    lam = torch.exp(-torch.abs(alpha)[:, None] + 1j * omega[None, :])
+    loss = 0.0
+    for b in range(B):
+        X = S0[b]
+        for t in range(L):
+            inp = xt[b, t][:, None].expand(m, c).to(torch.complex128)
+            X = inp if start[b, t] else lam * X + inp
+            flat = torch.cat([X.real.reshape(-1), X.imag.reshape(-1)])
+            loss = loss + (gz[b, t] * flat).sum()
+        loss = loss + (torch.conj(gSl[b]) * X).real.sum()
+    return loss
+
+
+@pytest.mark.parametrize("first", [True, False])
+def test_ffm_bwd_vs_torch_autograd(first):
+    torch = pytest.importorskip("torch")
+    rng = _rng(63)
+    B, L, m, c = 2, 20, 3, 2
+    alpha, omega, xt, start, S0 = _ffm_inputs(rng, B, L, m, c, 0.2, first=first)
+    alpha[1] = -alpha[1] if alpha[1] > 0 else alpha[1]  # one negative alpha: sign(alpha) enters
+    gz = rng.standard_normal((B, L, 2 * m * c))
+    gSl = _rand_c(rng, B, m, c)
+    ta, to = torch.tensor(alpha, requires_grad=True), torch.tensor(omega, requires_grad=True)
+    tx, ts = torch.tensor(xt, requires_grad=True), torch.tensor(S0, requires_grad=True)
+    loss = _torch_ffm_loss(torch, ta, to, tx, start, ts, torch.tensor(gz), torch.tensor(gSl))
+    loss.backward()
+    z, _ = oracle.ffm_fwd(alpha, omega, xt, start, S0)
+    gx, ga, go, gS0 = oracle.ffm_bwd(alpha, omega, start, z, gz, gSl, S0)
+    np.testing.assert_allclose(gx, tx.grad.numpy(), rtol=1e-10, atol=1e-10)
+    np.testing.assert_allclose(ga, ta.grad.numpy(), rtol=1e-10, atol=1e-10)
+    np.testing.assert_allclose(go, to.grad.numpy(), rtol=1e-10, atol=1e-10)
+    ref_S0 = np.zeros_like(gS0) if ts.grad is None else ts.grad.numpy()
+    np.testing.assert_allclose(gS0, ref_S0, rtol=1e-10, atol=1e-10)
+
+
+def test_ffm_bwd_finite_differences():
+    rng = _rng(64)
+    B, L, m, c = 1, 14, 2, 3
+    alpha, omega, xt, start, S0 = _ffm_inputs(rng, B, L, m, c, 0.0, first=False)
+    start[0, [5, 10]] = 1
+    gz = rng.standard_normal((B, L, 2 * m * c))
+    gSl = _rand_c(rng, B, m, c)
+
+    def loss(a, o, x, s0):
+        z, Sl = oracle.ffm_fwd(a, o, x, start, s0)
+        return float(np.sum(gz * z) + np.sum((np.conj(gSl) * Sl).real))
+
+    z, _ = oracle.ffm_fwd(alpha, omega, xt, start, S0)
+    gx, ga, go, gS0 = oracle.ffm_bwd(alpha, omega, start, z, gz, gSl, S0)
+    eps = 1e-6
+
+    def fd(arr, idx, f, unit=1.0):
+        a1, a2 = arr.copy(), arr.copy()
+        a1[idx] += eps * unit
+        a2[idx] -= eps * unit
+        return (f(a1) - f(a2)) / (2 * eps)
+
+    for i in range(m):
+        assert abs(fd(alpha, (i,), lambda a: loss(a, omega, xt, S0)) - ga[i]) < 1e-6
+    for j in range(c):
+        assert abs(fd(omega, (j,), lambda o: loss(alpha, o, xt, S0)) - go[j]) < 1e-6
+    for idx in [(0, 0, 0), (0, 4, 1), (0, 5, 0), (0, 13, 1)]:
+        assert abs(fd(xt, idx, lambda x: loss(alpha, omega, x, S0)) - gx[idx]) < 1e-6
+    for idx in [(0, 0, 0), (0, 1, 2)]:
+        d = fd(S0, idx, lambda s: loss(alpha, omega, xt, s)) + 1j * fd(S0, idx, lambda s: loss(alpha, omega, xt, s), 1j)
+        assert abs(d - gS0[idx]) < 1e-6
