@@ -10,7 +10,8 @@ decayed linear-attention memoroid on the largest linattn tape (L = 2^22,
 memoroid_scan_linattn_fwd + memoroid_scan_linattn_bwd, plus the tensor-core
 throughput of the intra-tile contraction alone (memoroid_bench_linattn_intra).
 Its "returns" object times the per-step discounted return and GAE with resets
-on 64 tapes of 2^20 steps.
+on 64 tapes of 2^20 steps, and its "ffm" object the Fast and Forgetful Memory
+memoroid (fwd + bwd) on a 2^20-step tape with a 64 x 4 complex state.
 
   python bench.py [--gpus N --steps K --warmup W] [--impl reference]
 
@@ -123,6 +124,78 @@ def returns_leg(args, m, dev, stream):
                                   "peak": peak, "frac": gbs / peak, "peak_kind": f"{peak_kind} (copy bandwidth)"}}
     out["gpu_launches"] = 2 * args.ret_steps  # one scan launch per call
     del r, v, G, A, ws
+    torch.cuda.empty_cache()
+    return out
+
+
+FFM_WORKLOAD = ("Fast and Forgetful Memory memoroid fwd+bwd: B=1 tape x L=2^20 steps, m=64 trace x c=4 context "
+                "(D=256 complex state), fp32, Geometric(500) episodes clipped to [1, 10000]")
+
+
+def ffm_leg(args, m, dev, stream):
+    """Times memoroid_ffm_fwd + memoroid_ffm_bwd (with the alpha / omega
+    gradients) on one 2^20-step tape, m = 64, c = 4."""
+    import torch
+
+    B, L, mm, c = 1, (args.ffm_tape_steps or (1 << 20)), 64, 4
+    D = mm * c
+    small = tapegen.ffm_tape(B, 1, mm, c, tapegen.seed_for(7), with_grad=False)  # alpha, omega
+    rng = np.random.default_rng(tapegen.seed_for(7))
+    start = torch.from_numpy(np.stack([tapegen.geometric_tape_starts(rng, L, 500.0, 1, 10000)
+                                       for _ in range(B)])).to(dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(tapegen.seed_for(7))
+    x = torch.randn((B, L, mm), generator=gen, device=dev, dtype=torch.float32)
+    gz = torch.randn((B, L, 2 * D), generator=gen, device=dev, dtype=torch.float32)
+    alpha = torch.from_numpy(small["alpha"]).to(dev)
+    omega = torch.from_numpy(small["omega"]).to(dev)
+    ws = m.ffm_workspace(B, L, mm, c, dev)
+    z = torch.empty((B, L, 2 * D), dtype=torch.float32, device=dev)
+    gx = torch.empty_like(x)
+    ga, go = torch.empty_like(alpha), torch.empty_like(omega)
+
+    def fwd():
+        m.memoroid_ffm_fwd(x, alpha, omega, start, None, z, None, B, L, mm, c, ws, stream)
+
+    def bwd():
+        m.memoroid_ffm_bwd(alpha, omega, start, None, z, gz, None, gx, ga, go, None, B, L, mm, c, ws, stream)
+
+    for _ in range(3):
+        fwd()
+        bwd()
+    torch.cuda.synchronize()
+    steps = args.ffm_steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for i in range(steps):
+        evs[i][0].record(stream)
+        fwd()
+        evs[i][1].record(stream)
+        bwd()
+        evs[i][2].record(stream)
+    torch.cuda.synchronize()
+    if m.memoroid_get_device_error(ws) != m.MEMOROID_OK:
+        raise RuntimeError("device-side error in the FFM timed region")
+    f_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / steps
+    b_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / steps
+    # algorithmic bytes: fwd reads x~ (4 m) and the flag, writes z (8 D); bwd reads
+    # grad_z and z (8 D each) and the flag, writes grad_x~ (4 m)
+    fb = B * L * (4 * mm + 1 + 8 * D)
+    bb = B * L * (16 * D + 1 + 4 * mm)
+    peak, peak_kind = _peaks()
+    kpc = (m.memoroid_ffm_kernels_per_call(B, L, mm, c, 0, 0) + m.memoroid_ffm_kernels_per_call(B, L, mm, c, 1, 1))
+    out = {
+        "workload": FFM_WORKLOAD if not args.ffm_tape_steps else f"{FFM_WORKLOAD} (first {L} steps only)",
+        "value": B * L / ((f_ms + b_ms) * 1e-3), "unit": UNIT, "steps": steps,
+        "ms_per_step": f_ms + b_ms, "fwd_ms": f_ms, "bwd_ms": b_ms, "episodes": int(start.sum().item()),
+        "roofline": {"bound": "hbm", "peak": peak, "unit": "GB/s", "peak_kind": f"{peak_kind} (copy bandwidth)",
+                     "fwd": {"algorithmic_bytes_per_call": fb, "achieved": fb / (f_ms * 1e-3) / 1e9,
+                             "frac": fb / (f_ms * 1e-3) / 1e9 / peak},
+                     "bwd": {"algorithmic_bytes_per_call": bb, "achieved": bb / (b_ms * 1e-3) / 1e9,
+                             "frac": bb / (b_ms * 1e-3) / 1e9 / peak},
+                     "step_frac": (fb + bb) / ((f_ms + b_ms) * 1e-3) / 1e9 / peak},
+        "gpu_launches": steps * kpc,
+    }
+    del x, gz, z, gx, ws
     torch.cuda.empty_cache()
     return out
 
@@ -392,6 +465,10 @@ def run_ours(args):
         # profiling mode: the discounted-return / GAE leg alone
         print(json.dumps({"returns": returns_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
         return
+    if args.only_ffm:
+        # profiling mode: the Fast and Forgetful Memory leg alone
+        print(json.dumps({"ffm": ffm_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
+        return
 
     t = tapegen.diag_config(CFG)
     if args.tape_steps:
@@ -525,6 +602,9 @@ def run_ours(args):
     rt = None
     if ws == 1 and not args.skip_returns:
         rt = returns_leg(args, m, dev, stream)
+    ff = None
+    if ws == 1 and not args.skip_ffm:
+        ff = ffm_leg(args, m, dev, stream)
     cpu = None
     if ws == 1 and not args.skip_cpu_baseline:
         cpu = cpu_baseline(t, args.cpu_seconds)
@@ -541,6 +621,7 @@ def run_ours(args):
         "clocks": clocks,
         "linattn": la,
         "returns": rt,
+        "ffm": ff,
     }
     print(json.dumps(out), flush=True)
     if ws > 1:
@@ -570,6 +651,12 @@ def main():
     ap.add_argument("--only-returns", action="store_true",
                     help="profiling mode: run and print only the discounted-return / GAE leg")
     ap.add_argument("--ret-steps", type=int, default=20, help="timed calls of each returns kernel")
+    ap.add_argument("--skip-ffm", action="store_true", help="omit the Fast and Forgetful Memory leg")
+    ap.add_argument("--only-ffm", action="store_true",
+                    help="profiling mode: run and print only the Fast and Forgetful Memory leg")
+    ap.add_argument("--ffm-steps", type=int, default=20, help="timed FFM fwd+bwd steps")
+    ap.add_argument("--ffm-tape-steps", type=int, default=0,
+                    help="FFM tape length (profiler captures); 0 = the full L = 2^20 workload")
     ap.add_argument("--la-intra-reps", type=int, default=2000,
                     help="repetitions of the intra-tile contraction per CTA in the tensor benchmark")
     ap.add_argument("--tape-steps", type=int, default=0,

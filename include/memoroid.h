@@ -217,6 +217,62 @@ memoroid_status_t memoroid_scan_linattn_bwd(const void *q, const void *k, const 
                                             size_t workspace_bytes, void *stream);
 
 /* ======================================================================== */
+/* Fast and Forgetful Memory memoroid (appendix "Fast and Forgetful         */
+/* Memory"): (X, t) . (X', t') = (X (.) exp(t'(-|alpha| (+) i omega)) + X', */
+/* t + t') with f(o, b) = (x~ repeated over the c columns, 1), made         */
+/* resettable by Theorem 3.2.  With t' = 1 per step this is, per state      */
+/* entry (i, j),                                                            */
+/*   X_t[i,j] = [b_t = 0] lambda_ij X_{t-1}[i,j] + x~_t[i],                  */
+/*   lambda_ij = exp(-|alpha_i| + i omega_j),                               */
+/* the diagonal scan over D = m*c complex channels (channel i*c + j).  The  */
+/* output is the cell's readout input Re(X_t) || Im(X_t), each flattened.   */
+/* Shapes: m % 4 == 0, c in {1, 2, 4, 8, 16}.                               */
+/* ======================================================================== */
+
+/* Workspace bytes for memoroid_ffm_fwd and memoroid_ffm_bwd (0 for an
+ * unsupported shape). */
+size_t memoroid_ffm_workspace_bytes(int64_t B, int64_t L, int64_t m, int64_t c);
+
+/* Kernel launches of one call (-1 for an unsupported shape). */
+int memoroid_ffm_kernels_per_call(int64_t B, int64_t L, int64_t m, int64_t c, int backward,
+                                  int with_param_grads);
+
+/*
+ *   x      fp32 [B, L, m]: the cell's gated input x~_t (16-byte aligned)
+ *   alpha  fp32 [m] decay parameters (|alpha| is used), omega fp32 [c]
+ *   start  uint8 [B, L], nonzero = first step of an episode
+ *   S0     complex64 [B, m, c]: state before step 0 of rows with start[b][0]
+ *          = 0, or NULL (= 0)
+ *   z      fp32 [B, L, 2*m*c] output: Re(X_t) then Im(X_t), row-major (i, j)
+ *   S_last complex64 [B, m, c] output, or NULL
+ * Device memory owned by the caller; workspace 256-byte aligned, at least
+ * memoroid_ffm_workspace_bytes; asynchronous on `stream`.  Errors:
+ * INVALID_ARG (shape, NULL or misaligned pointer), WORKSPACE, CUDA; a
+ * look-back wait that runs out is reported by memoroid_get_device_error.
+ */
+memoroid_status_t memoroid_ffm_fwd(const float *x, const float *alpha, const float *omega,
+                                   const uint8_t *start, const void *S0, float *z, void *S_last,
+                                   int64_t B, int64_t L, int64_t m, int64_t c, void *workspace,
+                                   size_t workspace_bytes, void *stream);
+
+/*
+ * Backward of memoroid_ffm_fwd (PyTorch's complex-gradient convention for
+ * S0 / S_last: grad = dL/dRe + i dL/dIm).
+ *   z           the forward's output; grad_z fp32 [B, L, 2*m*c] = dL/dz
+ *   grad_S_last complex64 [B, m, c] or NULL
+ *   grad_x      fp32 [B, L, m] output: sum over j of Re(delta_t[i, j])
+ *   grad_alpha  fp32 [m], grad_omega fp32 [c]: sums over B and L (either may
+ *               be NULL); the order of every reduction is fixed
+ *   grad_S0     complex64 [B, m, c] or NULL
+ */
+memoroid_status_t memoroid_ffm_bwd(const float *alpha, const float *omega, const uint8_t *start,
+                                   const void *S0, const float *z, const float *grad_z,
+                                   const void *grad_S_last, float *grad_x, float *grad_alpha,
+                                   float *grad_omega, void *grad_S0, int64_t B, int64_t L,
+                                   int64_t m, int64_t c, void *workspace, size_t workspace_bytes,
+                                   void *stream);
+
+/* ======================================================================== */
 /* Discounted return and GAE memoroids (appendices "The Discounted Return   */
 /* as a Memoroid" and "The Generalized Advantage Estimate as a Memoroid"):  */
 /* (a, r) . (a', r') = (a a', a r' + r), evaluated for every step of every  */

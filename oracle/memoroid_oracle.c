@@ -523,30 +523,45 @@ int oracle_ffm_fwd(int64_t B, int64_t L, int64_t m, int64_t c, const double *alp
 {
     if (B < 0 || L < 0 || m < 0 || c < 0) return -1;
     const int64_t D = m * c;
-#pragma omp parallel for collapse(2) schedule(static)
+    int bad = 0;
+#pragma omp parallel for schedule(static) reduction(| : bad)
     for (int64_t b = 0; b < B; ++b) {
+        /* the state (X, t) of every entry, advanced step by step */
+        cplx *X = (cplx *)malloc(sizeof(cplx) * (size_t)(D > 0 ? D : 1));
+        int64_t *tc = (int64_t *)malloc(sizeof(int64_t) * (size_t)(D > 0 ? D : 1));
+        if (!X || !tc) {
+            free(X);
+            free(tc);
+            bad = 1;
+            continue;
+        }
         for (int64_t ij = 0; ij < D; ++ij) {
-            const int64_t i = ij / c, j = ij % c;
-            cplx X = S0 ? S0[b * D + ij] : 0.0; /* e_I unless the row continues an episode */
-            int64_t tc = 0;
-            for (int64_t t = 0; t < L; ++t) {
+            X[ij] = S0 ? S0[b * D + ij] : 0.0; /* e_I unless the row continues an episode */
+            tc[ij] = 0;
+        }
+        for (int64_t t = 0; t < L; ++t) {
+            for (int64_t ij = 0; ij < D; ++ij) {
+                const int64_t i = ij / c, j = ij % c;
                 const cplx Xp = xt[(b * L + t) * m + i];
                 if (start[b * L + t]) { /* Theorem 3.2: the left operand becomes e_I = (0, 0) */
-                    X = 0.0;
-                    tc = 0;
+                    X[ij] = 0.0;
+                    tc[ij] = 0;
                 }
                 cplx nx;
                 int64_t nt;
-                ffm_combine(X, tc, Xp, 1, alpha[i], omega[j], &nx, &nt);
-                X = nx;
-                tc = nt;
-                z[(b * L + t) * 2 * D + ij] = creal(X);
-                z[(b * L + t) * 2 * D + D + ij] = cimag(X);
+                ffm_combine(X[ij], tc[ij], Xp, 1, alpha[i], omega[j], &nx, &nt);
+                X[ij] = nx;
+                tc[ij] = nt;
+                z[(b * L + t) * 2 * D + ij] = creal(nx);
+                z[(b * L + t) * 2 * D + D + ij] = cimag(nx);
             }
-            if (S_last) S_last[b * D + ij] = X;
         }
+        if (S_last)
+            for (int64_t ij = 0; ij < D; ++ij) S_last[b * D + ij] = X[ij];
+        free(X);
+        free(tc);
     }
-    return 0;
+    return bad ? -2 : 0;
 }
 
 /*
@@ -570,27 +585,40 @@ int oracle_ffm_bwd(int64_t B, int64_t L, int64_t m, int64_t c, const double *alp
 {
     if (B < 0 || L < 0 || m < 0 || c < 0) return -1;
     const int64_t D = m * c;
-    cplx *glam = (cplx *)calloc((size_t)(D > 0 ? D : 1), sizeof(cplx));
-    if (!glam) return -2;
-    if (grad_xt) memset(grad_xt, 0, sizeof(double) * (size_t)(B * L * m));
-#pragma omp parallel for schedule(static)
-    for (int64_t i = 0; i < m; ++i) {
-        for (int64_t j = 0; j < c; ++j) {
-            const int64_t ij = i * c + j;
-            const cplx lam = cexp(-fabs(alpha[i]) + I * omega[j]);
-            cplx gl = 0.0;
-            for (int64_t b = 0; b < B; ++b) {
-                cplx dn = 0.0; /* delta_{t+1} */
-                for (int64_t t = L - 1; t >= 0; --t) {
-                    const double *gz = grad_z + (b * L + t) * 2 * D;
+    const size_t nD = (size_t)(D > 0 ? D : 1);
+    /* per tape: the running grad_lambda sum of every entry (summed over tapes in order below) */
+    cplx *glam_b = (cplx *)calloc(nD * (size_t)(B > 0 ? B : 1), sizeof(cplx));
+    cplx *glam = (cplx *)calloc(nD, sizeof(cplx));
+    cplx *lam = (cplx *)malloc(sizeof(cplx) * nD);
+    if (!glam_b || !glam || !lam) {
+        free(glam_b);
+        free(glam);
+        free(lam);
+        return -2;
+    }
+    for (int64_t ij = 0; ij < D; ++ij) lam[ij] = cexp(-fabs(alpha[ij / c]) + I * omega[ij % c]);
+    int bad = 0;
+#pragma omp parallel for schedule(static) reduction(| : bad)
+    for (int64_t b = 0; b < B; ++b) {
+        cplx *dn = (cplx *)malloc(sizeof(cplx) * nD); /* delta_{t+1} of every entry */
+        if (!dn) {
+            bad = 1;
+            continue;
+        }
+        cplx *gl = glam_b + b * D;
+        for (int64_t t = L - 1; t >= 0; --t) {
+            const double *gz = grad_z + (b * L + t) * 2 * D;
+            for (int64_t i = 0; i < m; ++i) {
+                double gx = 0.0;
+                for (int64_t j = 0; j < c; ++j) {
+                    const int64_t ij = i * c + j;
                     cplx d = gz[ij] + I * gz[D + ij];
                     if (t == L - 1) {
                         if (grad_S_last) d += grad_S_last[b * D + ij];
                     } else if (!start[b * L + t + 1]) {
-                        d += conj(lam) * dn;
+                        d += conj(lam[ij]) * dn[ij];
                     }
-                    /* each (t, i) row is written by this thread only (it owns i) */
-                    if (grad_xt) grad_xt[(b * L + t) * m + i] += creal(d);
+                    gx += creal(d);
                     if (!start[b * L + t]) {
                         cplx prev;
                         if (t > 0) {
@@ -599,39 +627,44 @@ int oracle_ffm_bwd(int64_t B, int64_t L, int64_t m, int64_t c, const double *alp
                         } else {
                             prev = S0 ? S0[b * D + ij] : 0.0;
                         }
-                        gl += d * conj(prev);
+                        gl[ij] += d * conj(prev);
                     }
-                    dn = d;
+                    dn[ij] = d;
                 }
-                if (grad_S0) {
-                    grad_S0[b * D + ij] = (L > 0 && !start[b * L]) ? conj(lam) * dn
-                                                                   : (L == 0 && grad_S_last ? grad_S_last[b * D + ij] : 0.0);
-                }
+                if (grad_xt) grad_xt[(b * L + t) * m + i] = gx;
             }
-            glam[ij] = gl;
         }
+        if (grad_S0) {
+            for (int64_t ij = 0; ij < D; ++ij)
+                grad_S0[b * D + ij] = (L > 0 && !start[b * L]) ? conj(lam[ij]) * dn[ij]
+                                                               : (L == 0 && grad_S_last ? grad_S_last[b * D + ij] : 0.0);
+        }
+        free(dn);
+    }
+    for (int64_t b = 0; b < B; ++b)
+        for (int64_t ij = 0; ij < D; ++ij) glam[ij] += glam_b[b * D + ij];
+    free(glam_b);
+    if (bad) {
+        free(glam);
+        free(lam);
+        return -2;
     }
     if (grad_alpha) {
         for (int64_t i = 0; i < m; ++i) {
             const double sg = alpha[i] > 0 ? 1.0 : (alpha[i] < 0 ? -1.0 : 0.0);
             double acc = 0.0;
-            for (int64_t j = 0; j < c; ++j) {
-                const cplx lam = cexp(-fabs(alpha[i]) + I * omega[j]);
-                acc += creal(conj(glam[i * c + j]) * (-sg) * lam);
-            }
+            for (int64_t j = 0; j < c; ++j) acc += creal(conj(glam[i * c + j]) * (-sg) * lam[i * c + j]);
             grad_alpha[i] = acc;
         }
     }
     if (grad_omega) {
         for (int64_t j = 0; j < c; ++j) {
             double acc = 0.0;
-            for (int64_t i = 0; i < m; ++i) {
-                const cplx lam = cexp(-fabs(alpha[i]) + I * omega[j]);
-                acc += creal(conj(glam[i * c + j]) * I * lam);
-            }
+            for (int64_t i = 0; i < m; ++i) acc += creal(conj(glam[i * c + j]) * I * lam[i * c + j]);
             grad_omega[j] = acc;
         }
     }
     free(glam);
+    free(lam);
     return 0;
 }

@@ -358,6 +358,125 @@ memoroid_status_t memoroid_bench_linattn_intra(int64_t d, int64_t reps, int64_t 
 }
 
 // ---------------------------------------------------------------------------
+// Fast and Forgetful Memory
+// ---------------------------------------------------------------------------
+
+static bool ffm_shape_ok(int64_t B, int64_t L, int64_t m, int64_t c) {
+    if (B < 0 || L < 0 || m <= 0 || (m % 4) != 0) return false;
+    return c == 1 || c == 2 || c == 4 || c == 8 || c == 16;
+}
+
+size_t memoroid_ffm_workspace_bytes(int64_t B, int64_t L, int64_t m, int64_t c) {
+    if (!ffm_shape_ok(B, L, m, c)) return 0;
+    return diag::ffm_workspace_bytes(B, L, m, c);
+}
+
+int memoroid_ffm_kernels_per_call(int64_t B, int64_t L, int64_t m, int64_t c, int backward,
+                                  int with_param_grads) {
+    if (!ffm_shape_ok(B, L, m, c)) return -1;
+    return diag::ffm_kernels_per_call(B, L, m, c, backward != 0, with_param_grads != 0);
+}
+
+static memoroid_status_t ffm_check_ws(int64_t B, int64_t L, int64_t m, int64_t c, const void* ws, size_t bytes) {
+    if (ws == nullptr || !aligned(ws, 256)) return MEMOROID_ERR_WORKSPACE;
+    if (bytes < diag::ffm_workspace_bytes(B, L, m, c)) return MEMOROID_ERR_WORKSPACE;
+    return MEMOROID_OK;
+}
+
+memoroid_status_t memoroid_ffm_fwd(const float* x, const float* alpha, const float* omega, const uint8_t* start,
+                                   const void* S0, float* z, void* S_last, int64_t B, int64_t L, int64_t m,
+                                   int64_t c, void* workspace, size_t workspace_bytes, void* stream) {
+    if (!ffm_shape_ok(B, L, m, c)) return MEMOROID_ERR_INVALID_ARG;
+    const bool work = B > 0 && L > 0;
+    if ((S0 && !aligned(S0, 16)) || (S_last && !aligned(S_last, 16))) return MEMOROID_ERR_INVALID_ARG;
+    cudaStream_t s = as_stream(stream);
+    if (!work) {
+        // empty tape: S_last = S0 (or e_I = 0)
+        if (S_last && B > 0) {
+            const size_t bytes = static_cast<size_t>(B) * m * c * 8;
+            const cudaError_t e = S0 ? cudaMemcpyAsync(S_last, S0, bytes, cudaMemcpyDeviceToDevice, s)
+                                     : cudaMemsetAsync(S_last, 0, bytes, s);
+            if (e != cudaSuccess) return MEMOROID_ERR_CUDA;
+        }
+        return MEMOROID_OK;
+    }
+    if (!x || !alpha || !omega || !start || !z) return MEMOROID_ERR_INVALID_ARG;
+    if (!aligned(x, 16) || !aligned(z, 16) || !aligned(alpha, 4) || !aligned(omega, 4))
+        return MEMOROID_ERR_INVALID_ARG;
+    const memoroid_status_t w = ffm_check_ws(B, L, m, c, workspace, workspace_bytes);
+    if (w != MEMOROID_OK) return w;
+    diag::FfmArgs f{};
+    f.backward = false;
+    f.x = x;
+    f.alpha = alpha;
+    f.omega = omega;
+    f.start = start;
+    f.S0 = S0;
+    f.z = z;
+    f.S_last = S_last;
+    f.B = B;
+    f.L = L;
+    f.m = m;
+    f.c = c;
+    f.workspace = workspace;
+    f.workspace_bytes = workspace_bytes;
+    return diag::launch_ffm(f, s);
+}
+
+memoroid_status_t memoroid_ffm_bwd(const float* alpha, const float* omega, const uint8_t* start, const void* S0,
+                                   const float* z, const float* grad_z, const void* grad_S_last, float* grad_x,
+                                   float* grad_alpha, float* grad_omega, void* grad_S0, int64_t B, int64_t L,
+                                   int64_t m, int64_t c, void* workspace, size_t workspace_bytes, void* stream) {
+    if (!ffm_shape_ok(B, L, m, c)) return MEMOROID_ERR_INVALID_ARG;
+    const bool work = B > 0 && L > 0;
+    if ((S0 && !aligned(S0, 16)) || (grad_S_last && !aligned(grad_S_last, 16)) || (grad_S0 && !aligned(grad_S0, 16)) ||
+        (grad_alpha && !aligned(grad_alpha, 4)) || (grad_omega && !aligned(grad_omega, 4)))
+        return MEMOROID_ERR_INVALID_ARG;
+    cudaStream_t s = as_stream(stream);
+    if (!work) {
+        if (grad_alpha && cudaMemsetAsync(grad_alpha, 0, static_cast<size_t>(m) * 4, s) != cudaSuccess)
+            return MEMOROID_ERR_CUDA;
+        if (grad_omega && cudaMemsetAsync(grad_omega, 0, static_cast<size_t>(c) * 4, s) != cudaSuccess)
+            return MEMOROID_ERR_CUDA;
+        if (grad_S0 && B > 0) {
+            const size_t bytes = static_cast<size_t>(B) * m * c * 8;
+            const cudaError_t e = grad_S_last
+                                      ? cudaMemcpyAsync(grad_S0, grad_S_last, bytes, cudaMemcpyDeviceToDevice, s)
+                                      : cudaMemsetAsync(grad_S0, 0, bytes, s);
+            if (e != cudaSuccess) return MEMOROID_ERR_CUDA;
+        }
+        return MEMOROID_OK;
+    }
+    if (!alpha || !omega || !start || !z || !grad_z || !grad_x) return MEMOROID_ERR_INVALID_ARG;
+    if (static_cast<const void*>(grad_x) == z || static_cast<const void*>(grad_x) == grad_z)
+        return MEMOROID_ERR_INVALID_ARG;
+    if (!aligned(z, 16) || !aligned(grad_z, 16) || !aligned(grad_x, 16) || !aligned(alpha, 4) || !aligned(omega, 4))
+        return MEMOROID_ERR_INVALID_ARG;
+    const memoroid_status_t w = ffm_check_ws(B, L, m, c, workspace, workspace_bytes);
+    if (w != MEMOROID_OK) return w;
+    diag::FfmArgs f{};
+    f.backward = true;
+    f.alpha = alpha;
+    f.omega = omega;
+    f.start = start;
+    f.S0 = S0;
+    f.z = const_cast<float*>(z);
+    f.grad_z = grad_z;
+    f.grad_S_last = grad_S_last;
+    f.grad_x = grad_x;
+    f.grad_alpha = grad_alpha;
+    f.grad_omega = grad_omega;
+    f.grad_S0 = grad_S0;
+    f.B = B;
+    f.L = L;
+    f.m = m;
+    f.c = c;
+    f.workspace = workspace;
+    f.workspace_bytes = workspace_bytes;
+    return diag::launch_ffm(f, s);
+}
+
+// ---------------------------------------------------------------------------
 // discounted return and GAE
 // ---------------------------------------------------------------------------
 

@@ -120,10 +120,80 @@ struct Params {
     int full_nodes;              // summaries store a (per-step lambda) or only x
     int T;                       // steps per tile
     int rag;                     // steps missing from the chain's first tile in processing order
+    // Fast and Forgetful Memory layout (FFM configurations only): the forward
+    // input is x~ [B, L, m], one real value per row i of the m x c state,
+    // repeated over its c columns (channel i * c + j); states and their
+    // gradients are stored as Re || Im halves [B, L, 2D] (same row size as
+    // the interleaved layout); the backward writes grad_x~ [B, L, m] = the
+    // sum over the c columns of Re(delta) instead of grad_u.
+    const float* ffm_x;
+    float* ffm_gx;
+    int64_t ffm_m;
+    int ffm_lc;  // log2 c
 };
 
 __host__ __device__ __forceinline__ int64_t lmin(int64_t a, int64_t b) { return a < b ? a : b; }
 __host__ __device__ __forceinline__ int64_t lmax(int64_t a, int64_t b) { return a > b ? a : b; }
+
+// ---- FFM layout: one lane's two channels (2 lane, 2 lane + 1 of the slab) ----
+// staged forward input row: x~ of the slab's rows i, repeated over the columns
+__device__ __forceinline__ float4 ffm_x_pair(const Params& p, const float4* row, int lane) {
+    const float* x = reinterpret_cast<const float*>(row);
+    return make_float4(x[(2 * lane) >> p.ffm_lc], 0.f, x[(2 * lane + 1) >> p.ffm_lc], 0.f);
+}
+// staged planar row: Re half in the first 256 bytes, Im half in the second
+__device__ __forceinline__ float4 ffm_planar_pair(const float4* row, int lane) {
+    const float2* r = reinterpret_cast<const float2*>(row);
+    const float2 re = r[lane], im = r[32 + lane];
+    return make_float4(re.x, im.x, re.y, im.y);
+}
+// global planar row (D2 float4 = 2D floats): float2 index col of Re, D2 + col of Im
+__device__ __forceinline__ float4 ffm_load_planar(const float4* rowbase, int64_t D2, int64_t col) {
+    const float2* r = reinterpret_cast<const float2*>(rowbase);
+    const float2 re = r[col], im = r[D2 + col];
+    return make_float4(re.x, im.x, re.y, im.y);
+}
+__device__ __forceinline__ void ffm_store_planar(float4* rowbase, int64_t D2, int64_t col, float4 v, bool stream) {
+    float2* r = reinterpret_cast<float2*>(rowbase);
+    if (stream) {
+        __stcs(r + col, make_float2(v.x, v.z));
+        __stcs(r + D2 + col, make_float2(v.y, v.w));
+    } else {
+        r[col] = make_float2(v.x, v.z);
+        r[D2 + col] = make_float2(v.y, v.w);
+    }
+}
+// grad_x~ of step row: Re of this lane's two channels summed over the c
+// columns of their row i (a fixed butterfly over groups of c/2 lanes; lanes of
+// a group are all active or all inactive, `mask` holds the active ones), then
+// stored (accumulate = add to the stored value) by the group's first lane.
+__device__ __forceinline__ void ffm_grad_x(const Params& p, int64_t row, int64_t col, float4 d, unsigned mask,
+                                           bool active, bool accumulate, bool stream) {
+    const int lane = threadIdx.x & 31;
+    float* gx = p.ffm_gx + row * p.ffm_m;
+    if (p.ffm_lc == 0) {  // c = 1: the two channels are two rows i
+        if (active) {
+            float2* g2 = reinterpret_cast<float2*>(gx + 2 * col);
+            float2 v = make_float2(d.x, d.z);
+            if (accumulate) {
+                const float2 o = *g2;
+                v = make_float2(o.x + v.x, o.y + v.y);
+            }
+            if (stream) __stcs(g2, v);
+            else *g2 = v;
+        }
+        return;
+    }
+    float v = d.x + d.z;
+    const int group = 1 << (p.ffm_lc - 1);  // lanes per row i
+    for (int o = 1; o < group; o <<= 1) v += __shfl_xor_sync(mask, v, o);
+    if (active && (lane & (group - 1)) == 0) {
+        float* g = gx + ((2 * col) >> p.ffm_lc);
+        if (accumulate) v += *g;
+        if (stream) __stcs(g, v);
+        else *g = v;
+    }
+}
 
 // ---- two complex numbers per float4: (re0, im0, re1, im1) -------------------
 __device__ __forceinline__ float4 one2() { return make_float4(1.f, 0.f, 1.f, 0.f); }
@@ -143,11 +213,13 @@ __device__ __forceinline__ float4 add2(float4 a, float4 b) {
 }
 
 // ---- tile shapes -------------------------------------------------------------
-// W warps x R steps per warp; REV = backward; PS = per-step lambda.
-template <int W_, int R_, bool REV_, bool PS_>
+// W warps x R steps per warp; REV = backward; PS = per-step lambda; FFM = the
+// Fast and Forgetful Memory layout (broadcast input, planar states).
+template <int W_, int R_, bool REV_, bool PS_, bool FFM_ = false>
 struct Cfg {
     static constexpr int W = W_, R = R_, T = W_ * R_;
-    static constexpr bool REV = REV_, PS = PS_;
+    static constexpr bool REV = REV_, PS = PS_, FFM = FFM_;
+    static_assert(!(PS_ && FFM_), "the FFM multiplier is per channel");
     static constexpr int UNROLL = REV_ ? MEMOROID_UNROLL_BWD : MEMOROID_UNROLL_FWD;
     // arrays staged per tile: input [, h (backward)] [, lambda (per step)]
     static constexpr int NB = 1 + (REV_ ? 1 : 0) + (PS_ ? 1 : 0);
@@ -437,15 +509,33 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
     if (warp == LB_PUBLISH) {
         // ----------------------------------------- stage the tile, publish its summary
         const uint32_t rb = static_cast<uint32_t>(t.width2) * 16u;
+        // FFM forward: a row stages the x~ of the slab's rows i (4 bytes per c channels)
+        const uint32_t rb_in =
+            (C::FFM && !C::REV) ? static_cast<uint32_t>((2 * t.width2) >> p.ffm_lc) * 4u : rb;
         const int h_rows = C::REV ? t.nrows - (t.t0 == 0 ? 1 : 0) : 0;  // rows t0-1 ..
         const int l_rows = !C::PS ? 0 : (C::REV ? static_cast<int>(lmin(t.nrows, p.L - 1 - t.t0)) : t.nrows);
-        if (lane == 0) ptx::mbar_arrive_expect_tx(bar, rb * (t.nrows + h_rows + l_rows));
+        if (lane == 0) ptx::mbar_arrive_expect_tx(bar, rb_in * t.nrows + rb * (h_rows + l_rows));
         __syncwarp();
         for (int r = lane; r < t.nrows; r += 32) {
-            const int64_t g = (t.b * p.L + t.t0 + r) * p.D2 + t.c2;
-            ptx::bulk_g2s(s_in + r * 32, p.in + g, rb, bar);
-            if (C::REV && t.t0 + r >= 1) ptx::bulk_g2s(s_h + r * 32, p.h + g - p.D2, rb, bar);
-            if (C::PS && r < l_rows) ptx::bulk_g2s(s_l + r * 32, p.lambda + g + (C::REV ? p.D2 : 0), rb, bar);
+            const int64_t row = t.b * p.L + t.t0 + r;
+            const int64_t g = row * p.D2 + t.c2;
+            if (C::FFM && !C::REV) {
+                ptx::bulk_g2s(s_in + r * 32, p.ffm_x + row * p.ffm_m + ((2 * t.c2) >> p.ffm_lc), rb_in, bar);
+            } else if (C::FFM) {
+                // planar rows: the Re and Im halves of the slab, each rb / 2 bytes
+                const float2* gi = reinterpret_cast<const float2*>(p.in + row * p.D2);
+                ptx::bulk_g2s(s_in + r * 32, gi + t.c2, rb / 2, bar);
+                ptx::bulk_g2s(s_in + r * 32 + 16, gi + p.D2 + t.c2, rb / 2, bar);
+                if (t.t0 + r >= 1) {
+                    const float2* hi = reinterpret_cast<const float2*>(p.h + (row - 1) * p.D2);
+                    ptx::bulk_g2s(s_h + r * 32, hi + t.c2, rb / 2, bar);
+                    ptx::bulk_g2s(s_h + r * 32 + 16, hi + p.D2 + t.c2, rb / 2, bar);
+                }
+            } else {
+                ptx::bulk_g2s(s_in + r * 32, p.in + g, rb, bar);
+                if (C::REV && t.t0 + r >= 1) ptx::bulk_g2s(s_h + r * 32, p.h + g - p.D2, rb, bar);
+                if (C::PS && r < l_rows) ptx::bulk_g2s(s_l + r * 32, p.lambda + g + (C::REV ? p.D2 : 0), rb, bar);
+            }
         }
         float4 Ca, Cx;
         bool Cb;
@@ -575,7 +665,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
 #pragma unroll C::UNROLL
             for (int k = 0; k < R; ++k) {
                 if (k < nv) {
-                    const float4 uu = sin[k * 32];
+                    const float4 uu = C::FFM ? ffm_x_pair(p, s_in + (warp * R + k) * 32, lane) : sin[k * 32];
                     const float4 ll = C::PS ? sl[k * 32] : lam;
                     if ((rmask >> k) & 1u) {
                         a = ll;
@@ -591,7 +681,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
             for (int kk = 0; kk < R; ++kk) {
                 const int k = R - 1 - kk;
                 if (k < nv) {
-                    const float4 gg = sin[k * 32];
+                    const float4 gg = C::FFM ? ffm_planar_pair(s_in + (warp * R + k) * 32, lane) : sin[k * 32];
                     const float4 m = (ts + k == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
                     if ((rmask >> k) & 1u) {
                         a = m;
@@ -628,10 +718,13 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
 #pragma unroll C::UNROLL
             for (int k = 0; k < R; ++k) {
                 if (k < nv) {
-                    const float4 uu = sin[k * 32];
+                    const float4 uu = C::FFM ? ffm_x_pair(p, s_in + (warp * R + k) * 32, lane) : sin[k * 32];
                     const float4 ll = C::PS ? sl[k * 32] : lam;
                     c = ((rmask >> k) & 1u) ? uu : cfma2(ll, c, uu);
-                    __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
+                    if (C::FFM)
+                        ffm_store_planar(p.out + (t.b * p.L + ts + k) * p.D2, p.D2, t.c2 + lane, c, true);
+                    else
+                        __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
                 }
             }
             if (p.out_last != nullptr && nv > 0 && ts + nv == p.L) p.out_last[t.b * p.D2 + t.c2 + lane] = c;
@@ -640,21 +733,26 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
     } else {
         const float4* sh = s_h + warp * R * 32 + lane;
         float4 acc = zero2();
-        if (lane_ok) {
+        // FFM: every lane runs the loop (grad_x~ is reduced across lanes); the
+        // lanes past the slab's width touch no global memory
+        if (C::FFM || lane_ok) {
             float4* dst = p.out + (t.b * p.L + ts) * p.D2 + t.c2 + lane;
 #pragma unroll C::UNROLL
             for (int kk = 0; kk < R; ++kk) {
                 const int k = R - 1 - kk;
                 if (k >= nv) continue;
                 const int64_t tt = ts + k;
-                const float4 gg = sin[k * 32];
+                const float4 gg = C::FFM ? ffm_planar_pair(s_in + (warp * R + k) * 32, lane) : sin[k * 32];
                 const float4 m = (tt == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
                 c = ((rmask >> k) & 1u) ? gg : cfma2(m, c, gg);
-                __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
+                if (C::FFM)
+                    ffm_grad_x(p, t.b * p.L + tt, t.c2 + lane, c, 0xffffffffu, lane_ok, false, true);
+                else
+                    __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
                 float4 gl = zero2();
-                if (!((bmask >> k) & 1u)) {
+                if (!((bmask >> k) & 1u) && lane_ok) {
                     float4 hp;
-                    if (tt > 0) hp = sh[k * 32];
+                    if (tt > 0) hp = C::FFM ? ffm_planar_pair(s_h + (warp * R + k) * 32, lane) : sh[k * 32];
                     else hp = (p.h0 != nullptr) ? p.h0[t.b * p.D2 + t.c2 + lane] : zero2();
                     gl = cmul2(c, conj2(hp));
                 }
@@ -663,7 +761,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
                 } else {
                     acc = add2(acc, gl);
                 }
-                if (tt == 0 && p.grad_h0 != nullptr) {
+                if (tt == 0 && p.grad_h0 != nullptr && lane_ok) {
                     const float4 l0 = C::PS ? p.lambda[(t.b * p.L) * p.D2 + t.c2 + lane] : lam;
                     p.grad_h0[t.b * p.D2 + t.c2 + lane] = (bmask & 1u) ? zero2() : cmul2(conj2(l0), c);
                 }
@@ -759,6 +857,9 @@ __global__ void __launch_bounds__(128) segment_fix_kernel(const Params p) {
             break;
         }
     }
+    // lanes of the slab (FFM: the butterfly over a row's lanes uses this mask;
+    // a row's lanes are all in the slab or all past it)
+    const unsigned act = __ballot_sync(0xffffffffu, lane < lmin(SLAB / 2, p.D2 - c2));
     if (lane >= lmin(SLAB / 2, p.D2 - c2)) return;
     const int64_t col = c2 + lane;
     float4 corr = cmul2(p.pin[tid * 32 + lane], p.segc[(chain * p.n_seg + g) * 32 + lane]);
@@ -770,10 +871,14 @@ __global__ void __launch_bounds__(128) segment_fix_kernel(const Params p) {
         for (int k = 0; k < BATCH; ++k) {
             if (k0 + k < nfix) {
                 const int64_t t = C::REV ? t0 + nrows - 1 - (k0 + k) : t0 + k0 + k;
-                v[k] = p.out[(b * p.L + t) * p.D2 + col];
+                if (!C::FFM) v[k] = p.out[(b * p.L + t) * p.D2 + col];
+                else if (!C::REV) v[k] = ffm_load_planar(p.out + (b * p.L + t) * p.D2, p.D2, col);
                 if (C::REV) {
-                    aux[k] = (t > 0) ? p.h[(b * p.L + t - 1) * p.D2 + col]
-                                     : ((p.h0 != nullptr) ? p.h0[b * p.D2 + col] : zero2());
+                    if (t > 0)
+                        aux[k] = C::FFM ? ffm_load_planar(p.h + (b * p.L + t - 1) * p.D2, p.D2, col)
+                                        : p.h[(b * p.L + t - 1) * p.D2 + col];
+                    else
+                        aux[k] = (p.h0 != nullptr) ? p.h0[b * p.D2 + col] : zero2();
                 }
             }
         }
@@ -789,7 +894,12 @@ __global__ void __launch_bounds__(128) segment_fix_kernel(const Params p) {
                                                 : conj2(C::PS ? p.lambda[(b * p.L + t + 1) * p.D2 + col] : lam);
                 corr = cmul2(m, corr);
             }
-            p.out[(b * p.L + t) * p.D2 + col] = add2(v[k], corr);
+            if (!C::FFM)
+                p.out[(b * p.L + t) * p.D2 + col] = add2(v[k], corr);
+            else if (!C::REV)
+                ffm_store_planar(p.out + (b * p.L + t) * p.D2, p.D2, col, add2(v[k], corr), false);
+            else
+                ffm_grad_x(p, b * p.L + t, col, corr, act, true, true, false);
             if (!C::REV) {
                 if (t == p.L - 1 && p.out_last != nullptr) {
                     float4* ol = p.out_last + b * p.D2 + col;
@@ -900,6 +1010,8 @@ using FwdC = Cfg<MEMOROID_FWD_W, MEMOROID_FWD_R, false, false>;
 using FwdS = Cfg<4, 8, false, true>;
 using BwdC = Cfg<MEMOROID_BWD_W, MEMOROID_BWD_R, true, false>;
 using BwdS = Cfg<4, 8, true, true>;
+using FwdF = Cfg<MEMOROID_FWD_W, MEMOROID_FWD_R, false, false, true>;
+using BwdF = Cfg<MEMOROID_BWD_W, MEMOROID_BWD_R, true, false, true>;
 
 // Segments per chain: enough segment chains that a tile's predecessor was
 // handed out long before it (target), at least MIN_SEG_TILES tiles each.
@@ -994,6 +1106,11 @@ Params make_params(const Args& a, const Layout& l, int T, bool backward) {
     // backward: the chain's first tile (processing order) is the ragged last
     // time tile, and its step L-1 has multiplier 1 rather than conj(lambda)
     p.rag = backward ? static_cast<int>(n_tt * T - a.L) + 1 : 0;
+    p.ffm_x = a.ffm_x;
+    p.ffm_gx = a.ffm_gx;
+    p.ffm_m = a.ffm_m;
+    p.ffm_lc = 0;
+    while ((int64_t{1} << p.ffm_lc) < a.ffm_c) ++p.ffm_lc;
     return p;
 }
 
@@ -1054,13 +1171,15 @@ int kernels_per_call(int64_t B, int64_t L, int64_t D, int per_step, int backward
 }
 
 memoroid_status_t launch_fwd(const Args& a, cudaStream_t s) {
+    if (a.ffm_c > 0) return launch<FwdF>(a, s, nullptr);
     return a.lambda_per_step ? launch<FwdS>(a, s, nullptr) : launch<FwdC>(a, s, nullptr);
 }
 
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t s) {
     const bool ps = a.lambda_per_step != 0;
     Layout l{};
-    const memoroid_status_t st = ps ? launch<BwdS>(a, s, &l) : launch<BwdC>(a, s, &l);
+    const memoroid_status_t st = a.ffm_c > 0 ? launch<BwdF>(a, s, &l)
+                                             : (ps ? launch<BwdS>(a, s, &l) : launch<BwdC>(a, s, &l));
     if (st != MEMOROID_OK) return st;
     if (!ps && a.grad_lambda != nullptr) {
         unsigned char* ws = static_cast<unsigned char*>(a.workspace);
@@ -1073,6 +1192,116 @@ memoroid_status_t launch_bwd(const Args& a, cudaStream_t s) {
         if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     }
     return MEMOROID_OK;
+}
+
+// ============================================================================
+// Fast and Forgetful Memory: lambda_ij = exp(-|alpha_i| + i omega_j) per
+// channel, then the diagonal scan in the FFM layout
+// ============================================================================
+namespace {
+
+// one thread per channel i * c + j; computed in fp64 and rounded once
+__global__ void __launch_bounds__(256) ffm_lambda_kernel(const float* __restrict__ alpha,
+                                                         const float* __restrict__ omega, int64_t m, int64_t c,
+                                                         float2* __restrict__ lam) {
+    const int64_t ij = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (ij >= m * c) return;
+    const int64_t i = ij / c, j = ij - i * c;
+    const double mag = exp(-fabs(static_cast<double>(alpha[i])));
+    double sn, cs;
+    sincos(static_cast<double>(omega[j]), &sn, &cs);
+    lam[ij] = make_float2(static_cast<float>(mag * cs), static_cast<float>(mag * sn));
+}
+
+// grad_alpha_i = sum_j Re(conj(g_ij) (-sign(alpha_i)) lambda_ij) and
+// grad_omega_j = sum_i Re(conj(g_ij) i lambda_ij), one thread per output,
+// fixed-order fp64 sums (lambda as the forward used it)
+__global__ void __launch_bounds__(256) ffm_param_grad_kernel(const float2* __restrict__ glam,
+                                                             const float2* __restrict__ lam,
+                                                             const float* __restrict__ alpha, int64_t m, int64_t c,
+                                                             float* __restrict__ grad_alpha,
+                                                             float* __restrict__ grad_omega) {
+    const int64_t k = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (k < m) {
+        if (grad_alpha == nullptr) return;
+        const double sg = alpha[k] > 0.f ? 1.0 : (alpha[k] < 0.f ? -1.0 : 0.0);
+        double acc = 0.0;
+        for (int64_t j = 0; j < c; ++j) {
+            const float2 g = glam[k * c + j], l = lam[k * c + j];
+            acc += -sg * (static_cast<double>(g.x) * l.x + static_cast<double>(g.y) * l.y);
+        }
+        grad_alpha[k] = static_cast<float>(acc);
+    } else if (k < m + c) {
+        if (grad_omega == nullptr) return;
+        const int64_t j = k - m;
+        double acc = 0.0;
+        for (int64_t i = 0; i < m; ++i) {
+            // Re(conj(g) * i * l) = g.x * (-l.y) + g.y * l.x
+            const float2 g = glam[i * c + j], l = lam[i * c + j];
+            acc += static_cast<double>(g.y) * l.x - static_cast<double>(g.x) * l.y;
+        }
+        grad_omega[j] = static_cast<float>(acc);
+    }
+}
+
+size_t ffm_lambda_off(int64_t B, int64_t L, int64_t D) { return align_up(workspace_bytes(B, L, D), 256); }
+size_t ffm_glam_off(int64_t B, int64_t L, int64_t D) {
+    return align_up(ffm_lambda_off(B, L, D) + static_cast<size_t>(D) * 8, 256);
+}
+
+}  // namespace
+
+size_t ffm_workspace_bytes(int64_t B, int64_t L, int64_t m, int64_t c) {
+    const int64_t D = m * c;
+    return align_up(ffm_glam_off(B, L, D) + static_cast<size_t>(D) * 8, 256);
+}
+
+int ffm_kernels_per_call(int64_t B, int64_t L, int64_t m, int64_t c, int backward, int with_param_grads) {
+    if (B <= 0 || L <= 0 || m <= 0 || c <= 0) return 0;
+    const int64_t D = m * c;
+    const Layout l = layout(B, L, D, backward ? BwdF::T : FwdF::T, backward != 0);
+    int n = 1 + (l.sg.G > 1 ? 3 : 1);  // lambda + scan [+ segment carries + fix-up]
+    if (backward && with_param_grads) n += 3;  // grad_lambda reduction + parameter gradients
+    return n;
+}
+
+memoroid_status_t launch_ffm(const FfmArgs& f, cudaStream_t s) {
+    const int64_t D = f.m * f.c;
+    unsigned char* ws = static_cast<unsigned char*>(f.workspace);
+    float2* lam = reinterpret_cast<float2*>(ws + ffm_lambda_off(f.B, f.L, D));
+    float2* glam = reinterpret_cast<float2*>(ws + ffm_glam_off(f.B, f.L, D));
+    ffm_lambda_kernel<<<static_cast<unsigned>((D + 255) / 256), 256, 0, s>>>(f.alpha, f.omega, f.m, f.c, lam);
+    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    const bool param = f.backward && (f.grad_alpha != nullptr || f.grad_omega != nullptr);
+    Args a{};
+    a.lambda = lam;
+    a.lambda_per_step = 0;
+    a.start = f.start;
+    a.h0 = f.S0;
+    a.B = f.B;
+    a.L = f.L;
+    a.D = D;
+    a.workspace = f.workspace;
+    a.workspace_bytes = f.workspace_bytes;
+    a.ffm_c = static_cast<int>(f.c);
+    a.ffm_m = f.m;
+    if (!f.backward) {
+        a.ffm_x = f.x;
+        a.out = f.z;
+        a.out_last = f.S_last;
+        return launch_fwd(a, s);
+    }
+    a.u = f.grad_z;
+    a.h = f.z;
+    a.g_last = f.grad_S_last;
+    a.ffm_gx = f.grad_x;
+    a.grad_lambda = param ? glam : nullptr;
+    a.grad_h0 = f.grad_S0;
+    const memoroid_status_t st = launch_bwd(a, s);
+    if (st != MEMOROID_OK || !param) return st;
+    ffm_param_grad_kernel<<<static_cast<unsigned>((f.m + f.c + 255) / 256), 256, 0, s>>>(
+        glam, lam, f.alpha, f.m, f.c, f.grad_alpha, f.grad_omega);
+    return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
 }
 
 }  // namespace diag

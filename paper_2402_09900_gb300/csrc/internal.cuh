@@ -57,7 +57,40 @@ struct Args {
     int64_t B, L, D;
     void* workspace;
     size_t workspace_bytes;
+    // Fast and Forgetful Memory layout (ffm_c > 0): forward input x~ [B, L, m]
+    // in place of u, planar Re || Im states and gradients, backward output
+    // grad_x~ [B, L, m] in place of grad_u
+    const float* ffm_x = nullptr;
+    float* ffm_gx = nullptr;
+    int64_t ffm_m = 0;
+    int ffm_c = 0;
 };
+
+// FFM call: lambda_ij = exp(-|alpha_i| + i omega_j) built in the workspace,
+// then the scan in the FFM layout (and, backward, the parameter gradients)
+struct FfmArgs {
+    bool backward;
+    const float* x;  // fwd: x~ [B, L, m]
+    const float* alpha;
+    const float* omega;
+    const uint8_t* start;
+    const void* S0;           // [B, m*c] complex or null
+    float* z;                 // fwd output / bwd input: [B, L, 2*m*c]
+    void* S_last;             // fwd: [B, m*c] complex or null
+    const float* grad_z;      // bwd
+    const void* grad_S_last;  // bwd, or null
+    float* grad_x;            // bwd: [B, L, m]
+    float* grad_alpha;        // bwd: [m] or null
+    float* grad_omega;        // bwd: [c] or null
+    void* grad_S0;            // bwd: [B, m*c] complex or null
+    int64_t B, L, m, c;
+    void* workspace;
+    size_t workspace_bytes;
+};
+
+size_t ffm_workspace_bytes(int64_t B, int64_t L, int64_t m, int64_t c);
+int ffm_kernels_per_call(int64_t B, int64_t L, int64_t m, int64_t c, int backward, int with_param_grads);
+memoroid_status_t launch_ffm(const FfmArgs& a, cudaStream_t stream);
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t D);
 int kernels_per_call(int64_t B, int64_t L, int64_t D, int per_step, int backward, int with_grad_lambda);

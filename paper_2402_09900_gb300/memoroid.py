@@ -55,6 +55,10 @@ SIGNATURES = {
     "memoroid_bench_linattn_intra_scratch_bytes": (_sz, [_i64]),
     "memoroid_bench_linattn_intra": (_int, [_i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_returns_workspace_bytes": (_sz, [_i64, _i64]),
+    "memoroid_ffm_workspace_bytes": (_sz, [_i64, _i64, _i64, _i64]),
+    "memoroid_ffm_kernels_per_call": (_int, [_i64, _i64, _i64, _i64, _int, _int]),
+    "memoroid_ffm_fwd": (_int, [_p, _p, _p, _p, _p, _p, _p, _i64, _i64, _i64, _i64, _p, _sz, _p]),
+    "memoroid_ffm_bwd": (_int, [_p] * 11 + [_i64, _i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_discounted_return": (_int, [_p, _p, ctypes.c_float, _p, _p, _i64, _i64, _p, _sz, _p]),
     "memoroid_gae": (_int, [_p, _p, _p, ctypes.c_float, ctypes.c_float, _p, _p, _i64, _i64, _p, _sz, _p]),
     "memoroid_starts_from_offsets": (_int, [_p, _i64, _i64, _p, _p]),
@@ -223,6 +227,31 @@ def memoroid_gae(r, v, start, gamma, lam, v_boot, A, B, L, workspace, stream=Non
            "memoroid_gae")
 
 
+def memoroid_ffm_workspace_bytes(B, L, m, c) -> int:
+    return int(load().memoroid_ffm_workspace_bytes(B, L, m, c))
+
+
+def memoroid_ffm_kernels_per_call(B, L, m, c, backward, with_param_grads) -> int:
+    return int(load().memoroid_ffm_kernels_per_call(B, L, m, c, int(backward), int(with_param_grads)))
+
+
+def memoroid_ffm_fwd(x, alpha, omega, start, S0, z, S_last, B, L, m, c, workspace, stream=None):
+    _need_cuda(x, alpha, omega, start, S0, z, S_last, workspace)
+    _check(load().memoroid_ffm_fwd(_ptr(x), _ptr(alpha), _ptr(omega), _ptr(start), _ptr(S0), _ptr(z), _ptr(S_last),
+                                   B, L, m, c, _ptr(workspace), workspace.numel() if workspace is not None else 0,
+                                   _stream(stream)), "memoroid_ffm_fwd")
+
+
+def memoroid_ffm_bwd(alpha, omega, start, S0, z, grad_z, grad_S_last, grad_x, grad_alpha, grad_omega, grad_S0,
+                     B, L, m, c, workspace, stream=None):
+    _need_cuda(alpha, omega, start, S0, z, grad_z, grad_S_last, grad_x, grad_alpha, grad_omega, grad_S0, workspace)
+    _check(load().memoroid_ffm_bwd(_ptr(alpha), _ptr(omega), _ptr(start), _ptr(S0), _ptr(z), _ptr(grad_z),
+                                   _ptr(grad_S_last), _ptr(grad_x), _ptr(grad_alpha), _ptr(grad_omega),
+                                   _ptr(grad_S0), B, L, m, c, _ptr(workspace),
+                                   workspace.numel() if workspace is not None else 0, _stream(stream)),
+           "memoroid_ffm_bwd")
+
+
 def memoroid_starts_from_offsets(offsets, E, L, start, stream=None):
     _need_cuda(offsets, start)
     _check(load().memoroid_starts_from_offsets(_ptr(offsets), E, L, _ptr(start), _stream(stream)),
@@ -347,6 +376,40 @@ def gae(r, v, start, gamma, lam, v_boot=None, ws=None, stream=None):
     A = torch.empty_like(r)
     memoroid_gae(r, v, start, gamma, lam, v_boot, A, B, L, ws, stream)
     return A
+
+
+def ffm_workspace(B, L, m, c, device) -> torch.Tensor:
+    return workspace(memoroid_ffm_workspace_bytes(B, L, m, c), device)
+
+
+def ffm_fwd(x, alpha, omega, start, S0=None, want_last=True, ws=None, stream=None):
+    """Fast and Forgetful Memory: x [B, L, m] fp32, alpha [m], omega [c];
+    returns z [B, L, 2*m*c] (Re || Im of the state) and S_last [B, m, c]
+    complex64 (or None)."""
+    B, L, m = x.shape
+    c = omega.shape[0]
+    if ws is None:
+        ws = ffm_workspace(B, L, m, c, x.device)
+    z = torch.empty((B, L, 2 * m * c), dtype=torch.float32, device=x.device)
+    S_last = torch.empty((B, m, c), dtype=torch.complex64, device=x.device) if want_last else None
+    memoroid_ffm_fwd(x, alpha, omega, start, S0, z, S_last, B, L, m, c, ws, stream)
+    return z, S_last
+
+
+def ffm_bwd(alpha, omega, start, z, grad_z, grad_S_last=None, S0=None, want_params=True, want_S0=False, ws=None,
+            stream=None):
+    """Backward of ffm_fwd: grad_x [B, L, m], grad_alpha [m], grad_omega [c]
+    (None unless want_params), grad_S0 [B, m, c] (None unless want_S0)."""
+    B, L = z.shape[0], z.shape[1]
+    m, c = alpha.shape[0], omega.shape[0]
+    if ws is None:
+        ws = ffm_workspace(B, L, m, c, z.device)
+    gx = torch.empty((B, L, m), dtype=torch.float32, device=z.device)
+    ga = torch.empty(m, dtype=torch.float32, device=z.device) if want_params else None
+    go = torch.empty(c, dtype=torch.float32, device=z.device) if want_params else None
+    gS0 = torch.empty((B, m, c), dtype=torch.complex64, device=z.device) if want_S0 else None
+    memoroid_ffm_bwd(alpha, omega, start, S0, z, grad_z, grad_S_last, gx, ga, go, gS0, B, L, m, c, ws, stream)
+    return gx, ga, go, gS0
 
 
 def starts_from_offsets(offsets, L, stream=None):

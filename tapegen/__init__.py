@@ -180,6 +180,37 @@ def diag_config(cfg: int):
     return t
 
 
+def ffm_tape(B: int, L: int, m: int, c: int, seed: int, mean: float = 500.0, hi: int | None = None,
+             with_grad: bool = True, with_S0: bool = False, start_mode: str = "geometric"):
+    """A Fast-and-Forgetful-Memory workload: alpha [m] with |alpha| ~
+    U(0.001, 0.105) and a random sign (so exp(-|alpha|) spans the decays of
+    the diagonal configs, 0.9 .. 0.999), omega [c] ~ U(-pi, pi), the gated
+    input x~ [B, L, m] ~ N(0, 1) (fp32), begin flags as in diag_tape,
+    optional S0 [B, m, c] ~ CN(0, 1) (complex64) and upstream gradients
+    grad_z [B, L, 2 m c] ~ N(0, 1), grad_S_last [B, m, c] with Re, Im ~ N(0, 1)."""
+    rng = np.random.default_rng(seed)
+    alpha = (rng.uniform(0.001, 0.105, m) * rng.choice([-1.0, 1.0], m)).astype(np.float32)
+    omega = rng.uniform(-np.pi, np.pi, c).astype(np.float32)
+    x = rng.standard_normal((B, L, m), dtype=np.float32)
+    start = np.zeros((B, L), dtype=np.uint8)
+    for b in range(B):
+        if start_mode == "all":
+            start[b, :] = 1
+        elif start_mode == "none":
+            start[b, 0] = 1 if L else 0
+        elif start_mode == "open":
+            pass
+        else:
+            start[b] = geometric_tape_starts(rng, L, mean, 1, hi)
+    out = dict(B=B, L=L, m=m, c=c, alpha=alpha, omega=omega, x=x, start=start)
+    if with_grad:
+        out["grad_z"] = rng.standard_normal((B, L, 2 * m * c), dtype=np.float32)
+        out["grad_S_last"] = complex_normal(rng, (B, m, c), scale=np.sqrt(2.0))
+    if with_S0:
+        out["S0"] = complex_normal(rng, (B, m, c))
+    return out
+
+
 def linattn_tape(B: int, L: int, H: int, dk: int, dv: int, seed: int, mean: float = 300.0,
                  gamma_mode: str = "head", gammas=(0.9, 0.99, 0.999, 1.0), scale: float | None = None,
                  with_grad: bool = True, with_S0: bool = False, start_mode: str = "geometric"):

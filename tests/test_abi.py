@@ -94,3 +94,42 @@ def test_tape_index_validation(lib):
     assert lib.memoroid_offsets_from_starts(FAKE, 8, FAKE, None, FAKE, 4096, None) == m.MEMOROID_ERR_INVALID_ARG
     assert lib.memoroid_offsets_from_starts(FAKE, 8, FAKE, FAKE, None, 4096, None) == m.MEMOROID_ERR_WORKSPACE
     assert lib.memoroid_offsets_from_starts(FAKE, 8, FAKE, FAKE, FAKE, 8, None) == m.MEMOROID_ERR_WORKSPACE
+
+
+def test_ffm_validation(lib):
+    assert lib.memoroid_ffm_workspace_bytes(1, 1 << 20, 64, 4) > lib.memoroid_scan_diag_workspace_bytes(1, 1 << 20, 256)
+    for m_, c_ in ((6, 4), (8, 3), (8, 32), (0, 4)):
+        assert lib.memoroid_ffm_workspace_bytes(1, 100, m_, c_) == 0
+        assert lib.memoroid_ffm_kernels_per_call(1, 100, m_, c_, 0, 0) == -1
+
+    def fwd(x=FAKE, z=FAKE + 0x1000, m_=8, c_=4, ws=FAKE, wsb=1 << 30, S0=None):
+        return lib.memoroid_ffm_fwd(x, FAKE, FAKE, FAKE, S0, z, None, 1, 8, m_, c_, ws, wsb, None)
+
+    assert fwd(m_=6) == m.MEMOROID_ERR_INVALID_ARG
+    assert fwd(c_=3) == m.MEMOROID_ERR_INVALID_ARG
+    assert fwd(x=None) == m.MEMOROID_ERR_INVALID_ARG
+    assert fwd(x=FAKE + 8) == m.MEMOROID_ERR_INVALID_ARG
+    assert fwd(S0=FAKE + 4) == m.MEMOROID_ERR_INVALID_ARG
+    assert fwd(ws=None) == m.MEMOROID_ERR_WORKSPACE
+    assert fwd(wsb=64) == m.MEMOROID_ERR_WORKSPACE
+
+    def bwd(gx=FAKE + 0x2000, z=FAKE, gz=FAKE + 0x1000, c_=4, wsb=1 << 30):
+        return lib.memoroid_ffm_bwd(FAKE, FAKE, FAKE, None, z, gz, None, gx, None, None, None, 1, 8, 8, c_,
+                                    FAKE, wsb, None)
+
+    assert bwd(c_=5) == m.MEMOROID_ERR_INVALID_ARG
+    assert bwd(gx=None) == m.MEMOROID_ERR_INVALID_ARG
+    assert bwd(gx=FAKE) == m.MEMOROID_ERR_INVALID_ARG  # aliases z
+    assert bwd(gx=FAKE + 0x1000) == m.MEMOROID_ERR_INVALID_ARG  # aliases grad_z
+    assert bwd(wsb=0) == m.MEMOROID_ERR_WORKSPACE
+
+
+def test_returns_validation(lib):
+    assert lib.memoroid_discounted_return(FAKE, FAKE, 0.9, None, FAKE, -1, 8, FAKE, 4096, None) == \
+        m.MEMOROID_ERR_INVALID_ARG
+    assert lib.memoroid_discounted_return(None, FAKE, 0.9, None, FAKE, 1, 8, FAKE, 4096, None) == \
+        m.MEMOROID_ERR_INVALID_ARG
+    assert lib.memoroid_discounted_return(FAKE, FAKE, 0.9, None, FAKE, 1, 8, None, 4096, None) == \
+        m.MEMOROID_ERR_WORKSPACE
+    assert lib.memoroid_gae(FAKE, None, FAKE, 0.9, 0.9, None, FAKE, 1, 8, FAKE, 4096, None) == \
+        m.MEMOROID_ERR_INVALID_ARG
