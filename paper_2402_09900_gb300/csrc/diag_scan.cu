@@ -23,8 +23,8 @@
 //     its steps serially from the identity, then rescans them from its carry
 //     and streams the outputs out with 16-byte stores.  HBM traffic is one
 //     read of the inputs and one write of the outputs.
-//   * Look-back warp 1 stages the tile into shared memory (one TMA bulk copy
-//     per row), folds the summaries it needs from earlier tiles while the
+//   * Look-back warp 1 stages the tile into shared memory (one TMA tensor
+//     load of T rows per staged array), folds the summaries it needs from earlier tiles while the
 //     copies are in flight, and publishes the tile's own summary as soon as
 //     the scan warps' partial aggregates are in; look-back warp 2 derives the
 //     carry into the tile from earlier tiles' summaries, also starting at
@@ -88,12 +88,17 @@ constexpr int NB_READ = MEMOROID_NODE_BATCH;
 #define MEMOROID_UNROLL_BWD 32
 #endif
 constexpr int RED_PARTS = 512;  // first-stage parts of the grad_lambda reduction
+
 #ifndef MEMOROID_POLL_SLEEP_NS
 #define MEMOROID_POLL_SLEEP_NS 0  // longest back-off between flag polls
 #endif
 
 
 struct Params {
+    // 3-D tensor maps {row floats, L, B} of the staged arrays, boxes of T rows:
+    // the input (u / grad_h, or FFM x~ / grad_z), the forward states (backward)
+    // and the per-step lambda
+    CUtensorMap map_in, map_h, map_l;
     const float4* lambda;  // [D/2] or [B, L, D/2]; one float4 = two complex channels
     const float4* in;      // fwd: u; bwd: grad_h
     const uint8_t* start;  // [B, L]
@@ -136,15 +141,18 @@ __host__ __device__ __forceinline__ int64_t lmin(int64_t a, int64_t b) { return 
 __host__ __device__ __forceinline__ int64_t lmax(int64_t a, int64_t b) { return a > b ? a : b; }
 
 // ---- FFM layout: one lane's two channels (2 lane, 2 lane + 1 of the slab) ----
-// staged forward input row: x~ of the slab's rows i, repeated over the columns
-__device__ __forceinline__ float4 ffm_x_pair(const Params& p, const float4* row, int lane) {
-    const float* x = reinterpret_cast<const float*>(row);
+// Staged forward input: x~ of the slab's rows i, repeated over the columns
+// (rows of 64 / c floats, packed).
+__device__ __forceinline__ float4 ffm_x_pair(const Params& p, const float4* buf, int r, int lane) {
+    const float* x = reinterpret_cast<const float*>(buf) + r * (64 >> p.ffm_lc);
     return make_float4(x[(2 * lane) >> p.ffm_lc], 0.f, x[(2 * lane + 1) >> p.ffm_lc], 0.f);
 }
-// staged planar row: Re half in the first 256 bytes, Im half in the second
-__device__ __forceinline__ float4 ffm_planar_pair(const float4* row, int lane) {
-    const float2* r = reinterpret_cast<const float2*>(row);
-    const float2 re = r[lane], im = r[32 + lane];
+// Staged planar rows of a T-step tile: the Re halves of all rows (64 floats
+// each), then the Im halves.
+template <int T>
+__device__ __forceinline__ float4 ffm_planar_pair(const float4* buf, int r, int lane) {
+    const float2* b = reinterpret_cast<const float2*>(buf);
+    const float2 re = b[r * 32 + lane], im = b[T * 32 + r * 32 + lane];
     return make_float4(re.x, im.x, re.y, im.y);
 }
 // global planar row (D2 float4 = 2D floats): float2 index col of Re, D2 + col of Im
@@ -469,7 +477,7 @@ __device__ bool fenwick_carry(const Params& p, int64_t fbase, int64_t j, float4 
 // the scan kernel (forward: REV = false; backward: REV = true), one tile per CTA
 // ============================================================================
 template <class C>
-__global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
+__global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_constant__ Params p) {
     constexpr int W = C::W, R = C::R;
     constexpr int LB_PUBLISH = W, LB_CARRY = W + 1;  // the two look-back warps
     // named barriers: 1 aggregates ready (scan warps -> publisher),
@@ -508,35 +516,30 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
 
     if (warp == LB_PUBLISH) {
         // ----------------------------------------- stage the tile, publish its summary
-        const uint32_t rb = static_cast<uint32_t>(t.width2) * 16u;
-        // FFM forward: a row stages the x~ of the slab's rows i (4 bytes per c channels)
-        const uint32_t rb_in =
-            (C::FFM && !C::REV) ? static_cast<uint32_t>((2 * t.width2) >> p.ffm_lc) * 4u : rb;
-        const int h_rows = C::REV ? t.nrows - (t.t0 == 0 ? 1 : 0) : 0;  // rows t0-1 ..
-        const int l_rows = !C::PS ? 0 : (C::REV ? static_cast<int>(lmin(t.nrows, p.L - 1 - t.t0)) : t.nrows);
-        if (lane == 0) ptx::mbar_arrive_expect_tx(bar, rb_in * t.nrows + rb * (h_rows + l_rows));
-        __syncwarp();
-        for (int r = lane; r < t.nrows; r += 32) {
-            const int64_t row = t.b * p.L + t.t0 + r;
-            const int64_t g = row * p.D2 + t.c2;
+        // one box of T rows per staged array; rows past the tape (and the row
+        // before step 0) read as zeros, and every box counts in full
+        if (lane == 0) {
+            const int x = static_cast<int>(4 * t.c2), y = static_cast<int>(t.t0), z = static_cast<int>(t.b);
+            constexpr uint32_t BOX = C::T * 512u;  // a full 512-byte row per step
             if (C::FFM && !C::REV) {
-                ptx::bulk_g2s(s_in + r * 32, p.ffm_x + row * p.ffm_m + ((2 * t.c2) >> p.ffm_lc), rb_in, bar);
+                ptx::mbar_arrive_expect_tx(bar, static_cast<uint32_t>(C::T) * static_cast<uint32_t>(256 >> p.ffm_lc));
+                ptx::tma_load_3d(ptx::smem_addr(s_in), &p.map_in, static_cast<int>((2 * t.c2) >> p.ffm_lc), y, z, bar);
             } else if (C::FFM) {
-                // planar rows: the Re and Im halves of the slab, each rb / 2 bytes
-                const float2* gi = reinterpret_cast<const float2*>(p.in + row * p.D2);
-                ptx::bulk_g2s(s_in + r * 32, gi + t.c2, rb / 2, bar);
-                ptx::bulk_g2s(s_in + r * 32 + 16, gi + p.D2 + t.c2, rb / 2, bar);
-                if (t.t0 + r >= 1) {
-                    const float2* hi = reinterpret_cast<const float2*>(p.h + (row - 1) * p.D2);
-                    ptx::bulk_g2s(s_h + r * 32, hi + t.c2, rb / 2, bar);
-                    ptx::bulk_g2s(s_h + r * 32 + 16, hi + p.D2 + t.c2, rb / 2, bar);
-                }
+                // Re halves at x = 2 c2, Im halves at x = D + 2 c2 (floats), T x 256 bytes each
+                const int re = static_cast<int>(2 * t.c2), im = static_cast<int>(2 * p.D2 + 2 * t.c2);
+                ptx::mbar_arrive_expect_tx(bar, 2 * BOX);
+                ptx::tma_load_3d(ptx::smem_addr(s_in), &p.map_in, re, y, z, bar);
+                ptx::tma_load_3d(ptx::smem_addr(s_in + C::T * 16), &p.map_in, im, y, z, bar);
+                ptx::tma_load_3d(ptx::smem_addr(s_h), &p.map_h, re, y - 1, z, bar);
+                ptx::tma_load_3d(ptx::smem_addr(s_h + C::T * 16), &p.map_h, im, y - 1, z, bar);
             } else {
-                ptx::bulk_g2s(s_in + r * 32, p.in + g, rb, bar);
-                if (C::REV && t.t0 + r >= 1) ptx::bulk_g2s(s_h + r * 32, p.h + g - p.D2, rb, bar);
-                if (C::PS && r < l_rows) ptx::bulk_g2s(s_l + r * 32, p.lambda + g + (C::REV ? p.D2 : 0), rb, bar);
+                ptx::mbar_arrive_expect_tx(bar, BOX * C::NB);
+                ptx::tma_load_3d(ptx::smem_addr(s_in), &p.map_in, x, y, z, bar);
+                if (C::REV) ptx::tma_load_3d(ptx::smem_addr(s_h), &p.map_h, x, y - 1, z, bar);
+                if (C::PS) ptx::tma_load_3d(ptx::smem_addr(s_l), &p.map_l, x, y + (C::REV ? 1 : 0), z, bar);
             }
         }
+        __syncwarp();
         float4 Ca, Cx;
         bool Cb;
         bool ok = fenwick_children(p, t.fbase, t.pos + 1, node_mul, node_rag, Ca, Cx, Cb, tk);
@@ -665,7 +668,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
 #pragma unroll C::UNROLL
             for (int k = 0; k < R; ++k) {
                 if (k < nv) {
-                    const float4 uu = C::FFM ? ffm_x_pair(p, s_in + (warp * R + k) * 32, lane) : sin[k * 32];
+                    const float4 uu = C::FFM ? ffm_x_pair(p, s_in, warp * R + k, lane) : sin[k * 32];
                     const float4 ll = C::PS ? sl[k * 32] : lam;
                     if ((rmask >> k) & 1u) {
                         a = ll;
@@ -681,7 +684,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
             for (int kk = 0; kk < R; ++kk) {
                 const int k = R - 1 - kk;
                 if (k < nv) {
-                    const float4 gg = C::FFM ? ffm_planar_pair(s_in + (warp * R + k) * 32, lane) : sin[k * 32];
+                    const float4 gg = C::FFM ? ffm_planar_pair<C::T>(s_in, warp * R + k, lane) : sin[k * 32];
                     const float4 m = (ts + k == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
                     if ((rmask >> k) & 1u) {
                         a = m;
@@ -718,7 +721,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
 #pragma unroll C::UNROLL
             for (int k = 0; k < R; ++k) {
                 if (k < nv) {
-                    const float4 uu = C::FFM ? ffm_x_pair(p, s_in + (warp * R + k) * 32, lane) : sin[k * 32];
+                    const float4 uu = C::FFM ? ffm_x_pair(p, s_in, warp * R + k, lane) : sin[k * 32];
                     const float4 ll = C::PS ? sl[k * 32] : lam;
                     c = ((rmask >> k) & 1u) ? uu : cfma2(ll, c, uu);
                     if (C::FFM)
@@ -742,7 +745,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
                 const int k = R - 1 - kk;
                 if (k >= nv) continue;
                 const int64_t tt = ts + k;
-                const float4 gg = C::FFM ? ffm_planar_pair(s_in + (warp * R + k) * 32, lane) : sin[k * 32];
+                const float4 gg = C::FFM ? ffm_planar_pair<C::T>(s_in, warp * R + k, lane) : sin[k * 32];
                 const float4 m = (tt == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
                 c = ((rmask >> k) & 1u) ? gg : cfma2(m, c, gg);
                 if (C::FFM)
@@ -752,7 +755,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const Params p) {
                 float4 gl = zero2();
                 if (!((bmask >> k) & 1u) && lane_ok) {
                     float4 hp;
-                    if (tt > 0) hp = C::FFM ? ffm_planar_pair(s_h + (warp * R + k) * 32, lane) : sh[k * 32];
+                    if (tt > 0) hp = C::FFM ? ffm_planar_pair<C::T>(s_h, warp * R + k, lane) : sh[k * 32];
                     else hp = (p.h0 != nullptr) ? p.h0[t.b * p.D2 + t.c2 + lane] : zero2();
                     gl = cmul2(c, conj2(hp));
                 }
@@ -1114,6 +1117,31 @@ Params make_params(const Args& a, const Layout& l, int T, bool backward) {
     return p;
 }
 
+// A [B, L, row] fp32 array as a 3-D map {row, L, B} with boxes of `box_x`
+// floats x T rows x 1 tape (no swizzle; out-of-range elements read as 0).
+bool map3(CUtensorMap* m, const void* base, int64_t B, int64_t L, int64_t row, int box_x, int T) {
+    const EncodeTiledFn fn = encode_tiled();
+    if (fn == nullptr || base == nullptr) return fn != nullptr;
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(row), static_cast<cuuint64_t>(L), static_cast<cuuint64_t>(B)};
+    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(row * 4), static_cast<cuuint64_t>(L * row * 4)};
+    const cuuint32_t box[3] = {static_cast<cuuint32_t>(box_x), static_cast<cuuint32_t>(T), 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void*>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// The staging maps of a launch (see Params::map_in).
+bool make_maps(Params& p, const Args& a, int T, bool backward) {
+    const int64_t row = 4 * p.D2;  // floats per step: D complex, or Re || Im
+    if (a.ffm_c > 0 && !backward) return map3(&p.map_in, a.ffm_x, a.B, a.L, a.ffm_m, 64 >> p.ffm_lc, T);
+    const int bx = a.ffm_c > 0 ? 64 : 128;
+    bool ok = map3(&p.map_in, a.u, a.B, a.L, row, bx, T);
+    if (backward) ok = ok && map3(&p.map_h, a.h, a.B, a.L, row, bx, T);
+    if (a.lambda_per_step) ok = ok && map3(&p.map_l, a.lambda, a.B, a.L, row, 128, T);
+    return ok;
+}
+
 // One CTA per ticket; tickets are claimed in order by the CTAs as they
 // start.  With more than one segment per chain, two small kernels then add the
 // state entering each segment where it is missing.
@@ -1128,7 +1156,8 @@ memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
     if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(C::SMEM)) != cudaSuccess)
         return MEMOROID_ERR_CUDA;
-    const Params p = make_params(a, l, C::T, C::REV);
+    Params p = make_params(a, l, C::T, C::REV);
+    if (!make_maps(p, a, C::T, C::REV)) return MEMOROID_ERR_CUDA;
     kernel<<<static_cast<unsigned>(n_tickets), C::THREADS, C::SMEM, s>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     if (sg.G > 1) {

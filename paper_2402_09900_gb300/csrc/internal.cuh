@@ -1,5 +1,6 @@
 // internal.cuh -- declarations shared by the C-ABI layer and the kernel files.
 #pragma once
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cstddef>
@@ -39,6 +40,13 @@ DebugKnobs debug_knobs();
 uint32_t next_epoch();
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// cuTensorMapEncodeTiled, taken from the driver at run time (the library does
+// not link libcuda); null if the driver does not provide it.
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_tiled();
 
 namespace diag {
 

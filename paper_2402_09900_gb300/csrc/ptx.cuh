@@ -63,6 +63,15 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst_smem, const void* map, 
         "l"(map), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_addr(bar))
         : "memory");
 }
+// ---- TMA tiled load (3-D tensor map, global -> shared), completes on an mbarrier ----
+__device__ __forceinline__ void tma_load_3d(uint32_t dst_smem, const void* map, int c0, int c1, int c2,
+                                            uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+        "[%5];" ::"r"(dst_smem),
+        "l"(map), "r"(c0), "r"(c1), "r"(c2), "r"(smem_addr(bar))
+        : "memory");
+}
 // TMA tiled store (shared -> global) of one box; completes in the bulk group
 // (bulk_commit / bulk_wait_read / bulk_wait_all).  Out-of-range rows are clipped.
 __device__ __forceinline__ void tma_store_4d(const void* map, uint32_t src_smem, int c0, int c1, int c2, int c3) {
