@@ -549,15 +549,42 @@ def run_ours(args):
         h2d = sum(x.numel() * x.element_size() for x in (hu, hg, hs, hl))
         d2h = sum(x.numel() * x.element_size() for x in (oh, ogu, ogl))
 
+        # Copies run on their own streams so that the two directions overlap each
+        # other and the kernels: inputs go up on s_in, results come down on s_out,
+        # the scans run on `stream`; every buffer is reused only after the last
+        # reader or writer of the previous step is done with it (events).
+        s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+        ev = {k: torch.cuda.Event() for k in ("u_in", "g_in", "fwd", "bwd", "h_out", "gu_out")}
+        for e in ev.values():
+            e.record(stream)
+
         def e2e_step():
-            u.copy_(hu, non_blocking=True)
-            grad_h.copy_(hg, non_blocking=True)
-            start.copy_(hs, non_blocking=True)
-            lam.copy_(hl, non_blocking=True)
-            step()
-            oh.copy_(h, non_blocking=True)
-            ogu.copy_(grad_u, non_blocking=True)
-            ogl.copy_(grad_lam, non_blocking=True)
+            with torch.cuda.stream(s_in):
+                s_in.wait_event(ev["fwd"])  # the previous forward has read u
+                u.copy_(hu, non_blocking=True)
+                s_in.wait_event(ev["bwd"])  # the previous backward has read start, lambda, grad_h
+                start.copy_(hs, non_blocking=True)
+                lam.copy_(hl, non_blocking=True)
+                ev["u_in"].record(s_in)
+                grad_h.copy_(hg, non_blocking=True)
+                ev["g_in"].record(s_in)
+            stream.wait_event(ev["u_in"])
+            stream.wait_event(ev["h_out"])  # h of the previous step is on the host
+            m.memoroid_scan_diag_fwd(lam, 0, u, start, None, h, None, B, L, D, work, stream)
+            ev["fwd"].record(stream)
+            stream.wait_event(ev["g_in"])
+            stream.wait_event(ev["gu_out"])  # grad_u / grad_lambda of the previous step are on the host
+            m.memoroid_scan_diag_bwd(lam, 0, start, None, h, grad_h, None, grad_u, grad_lam, None, B, L, D,
+                                     work, stream)
+            ev["bwd"].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev["fwd"])
+                oh.copy_(h, non_blocking=True)
+                ev["h_out"].record(s_out)
+                s_out.wait_event(ev["bwd"])
+                ogu.copy_(grad_u, non_blocking=True)
+                ogl.copy_(grad_lam, non_blocking=True)
+                ev["gu_out"].record(s_out)
 
         e2e_step()
         torch.cuda.synchronize()
