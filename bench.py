@@ -613,6 +613,9 @@ def run_ours(args):
     fwd_avg = sum(fwd_ms) / len(fwd_ms)
     bwd_avg = sum(bwd_ms) / len(bwd_ms)
     traffic, traffic_note = _traffic_record()
+    if args.tape_steps:
+        traffic, traffic_note = None, "the record is for the full tape; this run used a shorter one"
+
     bwd_gbs = bwd_bytes / (bwd_avg * 1e-3) / 1e9
     fwd_gbs = fwd_bytes / (fwd_avg * 1e-3) / 1e9
     roofline = {"bound": "hbm", "achieved": bwd_gbs, "peak": peak, "unit": "GB/s",
