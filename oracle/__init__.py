@@ -30,6 +30,9 @@ Parity status of each routine (what pins it, in tests/test_oracle_pins.py):
                      all-start tapes
   ffm_bwd            torch.autograd (fp64) through an independent loop,
                      central finite differences in alpha and omega
+  tbb_sample         the Figure 2 tape worked by hand, and on random inputs the
+                     properties that define the batch (whole episodes in draw
+                     order, cut at B, flags at piece starts, fewest draws)
 """
 from __future__ import annotations
 
@@ -86,6 +89,8 @@ def lib():
             L.oracle_discounted_return.argtypes = [_i64, _i64, _p, _p, _c.c_double, _p, _p]
             L.oracle_gae.argtypes = [_i64, _i64, _p, _p, _p, _c.c_double, _c.c_double, _p, _p]
             L.oracle_offsets_from_starts.argtypes = [_p, _i64, _p]
+            L.oracle_tbb_sample.argtypes = [_p, _i64, _i64, _p, _i64, _i64, _p, _p]
+            L.oracle_tbb_sample.restype = _i64
             L.oracle_ffm_fwd.argtypes = [_i64] * 4 + [_p] * 7
             L.oracle_ffm_bwd.argtypes = [_i64] * 4 + [_p] * 11
             L.oracle_offsets_from_starts.restype = _i64
@@ -306,6 +311,24 @@ def ffm_bwd(alpha, omega, start, z, grad_z, grad_S_last=None, S0=None):
     _check(lib().oracle_ffm_bwd(B, L, m, c, _ptr(alpha), _ptr(omega), _ptr(start), _ptr(S0), _ptr(z),
                                 _ptr(grad_z), _ptr(grad_S_last), _ptr(gx), _ptr(ga), _ptr(go), _ptr(gS0)))
     return gx, ga, go, gS0
+
+
+def tbb_sample(I, N, ep, B):
+    """Algorithm 2 with the draws given: I [E] episode begin indices into a
+    buffer of N transitions, ep [K] the drawn indices, B the batch size.
+    Returns (start [B] uint8, src [B] int64, draws used); raises ValueError
+    on an out-of-range index or too few draws."""
+    I = np.ascontiguousarray(I, dtype=np.int64)
+    ep = np.ascontiguousarray(ep, dtype=np.int64)
+    start = np.zeros(B, dtype=np.uint8)
+    src = np.zeros(B, dtype=np.int64)
+    n = lib().oracle_tbb_sample(_ptr(I), len(I), N, _ptr(ep), len(ep), B, _ptr(start), _ptr(src))
+    if n == -2:
+        raise ValueError("episode index out of range")
+    if n == -3:
+        raise ValueError("the draws do not fill the batch")
+    _check(0 if n >= 0 else n)
+    return start, src, int(n)
 
 
 def starts_from_offsets(offsets, L):

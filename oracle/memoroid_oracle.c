@@ -668,3 +668,39 @@ int oracle_ffm_bwd(int64_t B, int64_t L, int64_t m, int64_t c, const double *alp
     free(lam);
     return 0;
 }
+
+/* ------------------------------------------------------------------------ */
+/* Tape-based batching, sampling (Algorithm 2): starting from an empty       */
+/* batch, append the episode D[I[i] : I[i+1]] of a randomly drawn index i    */
+/* while the batch is shorter than B, then cut the batch to B transitions.  */
+/* The draws are an input here: ep[0..K) are the successive indices i, and  */
+/* begin[0..E) is the index list I.  The episode of the last index runs to  */
+/* the end of D (I[E] reads as N).                                          */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Outputs, for the B steps of the batch: src[t] = the index in D of the
+ * transition at step t; start[t] = 1 where an appended episode begins.
+ * Returns the number of draws used (>= 0), -1 on a bad argument, -2 if an
+ * index is out of range, -3 if the K draws do not fill B steps.
+ */
+int64_t oracle_tbb_sample(const int64_t *begin, int64_t E, int64_t N, const int64_t *ep, int64_t K, int64_t B,
+                          uint8_t *start, int64_t *src)
+{
+    if (E < 0 || N < 0 || K < 0 || B < 0) return -1;
+    int64_t len = 0; /* len(batch) */
+    int64_t k = 0;
+    while (len < B) {
+        if (k >= K) return -3;
+        const int64_t i = ep[k++];
+        if (i < 0 || i >= E) return -2;
+        const int64_t lo = begin[i], hi = (i + 1 < E) ? begin[i + 1] : N;
+        /* batch <- concat(batch, D[lo:hi]); the cut to B happens on the fly */
+        for (int64_t s = lo; s < hi && len < B; ++s) {
+            start[len] = (s == lo);
+            src[len] = s;
+            ++len;
+        }
+    }
+    return k;
+}

@@ -773,3 +773,70 @@ def test_ffm_bwd_finite_differences():
     for idx in [(0, 0, 0), (0, 1, 2)]:
         d = fd(S0, idx, lambda s: loss(alpha, omega, xt, s)) + 1j * fd(S0, idx, lambda s: loss(alpha, omega, xt, s), 1j)
         assert abs(d - gS0[idx]) < 1e-6
+
+
+# ---------------------------------------------------------------------------
+# tape-based batching, sampling (Algorithm 2)
+# ---------------------------------------------------------------------------
+
+FIG2_I = np.array([0, 4, 6, 7])
+FIG2_N = 9
+
+
+def test_tbb_sample_figure2_worked_by_hand():
+    with open(os.path.join(GOLDEN, "tbb_sample_figure2.txt")) as f:
+        rows = [l for l in f if l.strip() and not l.startswith("#")]
+    assert len(rows) == 2
+    for row in rows:
+        head, draws, used, src, start = [c.split() for c in row.split("|")]
+        B = int(head[1])
+        s, x, n = oracle.tbb_sample(FIG2_I, FIG2_N, np.array(draws, dtype=np.int64), B)
+        assert n == int(used[0])
+        assert np.array_equal(x, np.array(src, dtype=np.int64))
+        assert np.array_equal(s, np.array(start, dtype=np.uint8))
+
+
+def _episode_range(I, N, i):
+    return int(I[i]), int(I[i + 1]) if i + 1 < len(I) else N
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_tbb_sample_defining_properties(seed):
+    rng = np.random.default_rng(900 + seed)
+    N = int(rng.integers(50, 3000))
+    starts = tapegen.geometric_tape_starts(rng, N, float(rng.choice([1.5, 8.0, 60.0])))
+    I = np.flatnonzero(starts)
+    if seed == 5:
+        I = I[1:] if len(I) > 1 else I  # a buffer whose first transitions belong to a popped episode
+    B = int(rng.integers(1, 2 * N))
+    ep = rng.integers(0, len(I), size=4 * B + 8)
+    start, src, n = oracle.tbb_sample(I, N, ep, B)
+    heads = np.flatnonzero(start)
+    # one piece per draw used, starting at step 0, in draw order
+    assert len(heads) == n and heads[0] == 0
+    bounds = list(heads) + [B]
+    full = 0
+    for k in range(n):
+        lo, hi = _episode_range(I, N, int(ep[k]))
+        piece = src[bounds[k]:bounds[k + 1]]
+        # a piece is the drawn episode's transitions, consecutive, from its first one
+        assert piece[0] == lo
+        assert np.all(np.diff(piece) == 1)
+        if k < n - 1:
+            assert len(piece) == hi - lo  # whole episodes before the last
+            full += hi - lo
+        else:
+            assert 1 <= len(piece) <= hi - lo  # the last one is cut at B
+    # the fewest draws: the pieces before the last do not fill the batch
+    assert full < B
+
+
+def test_tbb_sample_exact_fit_and_errors():
+    # the episodes fill B exactly: nothing is cut
+    start, src, n = oracle.tbb_sample(FIG2_I, FIG2_N, np.array([1, 3, 2]), 5)
+    assert n == 3 and np.array_equal(src, [4, 5, 7, 8, 6]) and np.array_equal(start, [1, 0, 1, 0, 1])
+    assert oracle.tbb_sample(FIG2_I, FIG2_N, np.array([], dtype=np.int64), 0)[2] == 0
+    with pytest.raises(ValueError):
+        oracle.tbb_sample(FIG2_I, FIG2_N, np.array([2, 2]), 5)  # two 1-step episodes cannot fill 5 steps
+    with pytest.raises(ValueError):
+        oracle.tbb_sample(FIG2_I, FIG2_N, np.array([4]), 2)  # no episode 4
