@@ -10,8 +10,10 @@ decayed linear-attention memoroid on the largest linattn tape (L = 2^22,
 memoroid_scan_linattn_fwd + memoroid_scan_linattn_bwd, plus the tensor-core
 throughput of the intra-tile contraction alone (memoroid_bench_linattn_intra).
 Its "returns" object times the per-step discounted return and GAE with resets
-on 64 tapes of 2^20 steps, and its "ffm" object the Fast and Forgetful Memory
-memoroid (fwd + bwd) on a 2^20-step tape with a 64 x 4 complex state.
+on 64 tapes of 2^20 steps, its "ffm" object the Fast and Forgetful Memory
+memoroid (fwd + bwd) on a 2^20-step tape with a 64 x 4 complex state, and its
+"tbb" object the device-side sampling of a 2^20-step batch (Algorithm 2) and
+the gather of its 2 KB rows.
 
   python bench.py [--gpus N --steps K --warmup W] [--impl reference]
 
@@ -198,6 +200,63 @@ def ffm_leg(args, m, dev, stream):
     del x, gz, z, gx, ws
     torch.cuda.empty_cache()
     return out
+
+
+TBB_WORKLOAD = ("tape-based batching (Algorithm 2): a batch of B=2^20 steps sampled from a buffer of N=2^21 "
+                "transitions with Geometric(500) episodes, rows of 256 complex64 channels (2 KB) gathered into the tape")
+
+
+def tbb_leg(args, m, dev, stream):
+    """Times memoroid_tbb_sample (flags and source indices of the batch) and
+    memoroid_gather_rows (the batch's 2 KB rows) on the bench buffer."""
+    import torch
+
+    N, B, D = 1 << 21, 1 << 20, 256
+    rng = np.random.default_rng(tapegen.seed_for(8))
+    begin = torch.from_numpy(np.flatnonzero(tapegen.geometric_tape_starts(rng, N, 500.0))).to(dev)
+    E = begin.numel()
+    draws = torch.from_numpy(rng.integers(0, E, size=B // 100)).to(dev)  # ~2100 draws are used
+    K = draws.numel()
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(tapegen.seed_for(8))
+    rows = torch.randn((N, 2 * D), generator=gen, device=dev, dtype=torch.float32)
+    ws = m.workspace(m.memoroid_tbb_workspace_bytes(K), dev)
+    start = torch.empty(B, dtype=torch.uint8, device=dev)
+    src = torch.empty(B, dtype=torch.int64, device=dev)
+    n_used = torch.empty(1, dtype=torch.int64, device=dev)
+    out = torch.empty((B, 2 * D), dtype=torch.float32, device=dev)
+    row_bytes = 2 * D * 4
+
+    def sample():
+        m.memoroid_tbb_sample(begin, E, N, draws, K, B, start, src, n_used, ws, stream)
+
+    def gather():
+        m.memoroid_gather_rows(rows, N, row_bytes, src, B, out, ws, stream)
+
+    res = {"workload": TBB_WORKLOAD}
+    peak, peak_kind = _peaks()
+    for name, fn, byts in (("sample", sample, B * 9), ("gather", gather, B * (8 + 2 * row_bytes))):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.tbb_steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / args.tbb_steps
+        gbs = byts / (ms * 1e-3) / 1e9
+        res[name] = {"ms": ms, "value": B / (ms * 1e-3), "unit": "steps/s",
+                     "roofline": {"bound": "hbm", "algorithmic_bytes_per_call": byts, "achieved": gbs, "unit": "GB/s",
+                                  "peak": peak, "frac": gbs / peak, "peak_kind": f"{peak_kind} (copy bandwidth)"}}
+    if m.memoroid_get_device_error(ws) != m.MEMOROID_OK:
+        raise RuntimeError("device-side data check failed in the TBB leg")
+    res["draws_used"] = int(n_used.item())
+    res["gpu_launches"] = args.tbb_steps * 3  # offsets + fill, gather
+    del rows, out
+    torch.cuda.empty_cache()
+    return res
 
 
 def linattn_leg(args, m, dev, stream):
@@ -465,6 +524,10 @@ def run_ours(args):
         # profiling mode: the discounted-return / GAE leg alone
         print(json.dumps({"returns": returns_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
         return
+    if args.only_tbb:
+        # profiling mode: the tape-based batching leg alone
+        print(json.dumps({"tbb": tbb_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
+        return
     if args.only_ffm:
         # profiling mode: the Fast and Forgetful Memory leg alone
         print(json.dumps({"ffm": ffm_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
@@ -635,6 +698,9 @@ def run_ours(args):
     ff = None
     if ws == 1 and not args.skip_ffm:
         ff = ffm_leg(args, m, dev, stream)
+    tb = None
+    if ws == 1 and not args.skip_tbb:
+        tb = tbb_leg(args, m, dev, stream)
     cpu = None
     if ws == 1 and not args.skip_cpu_baseline:
         cpu = cpu_baseline(t, args.cpu_seconds)
@@ -652,6 +718,7 @@ def run_ours(args):
         "linattn": la,
         "returns": rt,
         "ffm": ff,
+        "tbb": tb,
     }
     print(json.dumps(out), flush=True)
     if ws > 1:
@@ -682,6 +749,10 @@ def main():
                     help="profiling mode: run and print only the discounted-return / GAE leg")
     ap.add_argument("--ret-steps", type=int, default=20, help="timed calls of each returns kernel")
     ap.add_argument("--skip-ffm", action="store_true", help="omit the Fast and Forgetful Memory leg")
+    ap.add_argument("--skip-tbb", action="store_true", help="omit the tape-based batching leg")
+    ap.add_argument("--only-tbb", action="store_true",
+                    help="profiling mode: run and print only the tape-based batching leg")
+    ap.add_argument("--tbb-steps", type=int, default=20, help="timed calls of the sampler and of the gather")
     ap.add_argument("--only-ffm", action="store_true",
                     help="profiling mode: run and print only the Fast and Forgetful Memory leg")
     ap.add_argument("--ffm-steps", type=int, default=20, help="timed FFM fwd+bwd steps")

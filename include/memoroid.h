@@ -42,7 +42,8 @@ typedef enum {
     MEMOROID_ERR_UNSUPPORTED = 2, /* a shape or mode this build does not implement */
     MEMOROID_ERR_WORKSPACE = 3,   /* workspace missing, misaligned or too small */
     MEMOROID_ERR_CUDA = 4,        /* a CUDA runtime call or launch failed */
-    MEMOROID_ERR_TIMEOUT = 5      /* a bounded device-side wait ran out */
+    MEMOROID_ERR_TIMEOUT = 5,     /* a bounded device-side wait ran out */
+    MEMOROID_ERR_BAD_DATA = 6     /* a device-side check of the data failed (see the call) */
 } memoroid_status_t;
 
 typedef enum { MEMOROID_F32 = 0, MEMOROID_BF16 = 1 } memoroid_dtype_t;
@@ -271,6 +272,49 @@ memoroid_status_t memoroid_ffm_bwd(const float *alpha, const float *omega, const
                                    float *grad_omega, void *grad_S0, int64_t B, int64_t L,
                                    int64_t m, int64_t c, void *workspace, size_t workspace_bytes,
                                    void *stream);
+
+/* ======================================================================== */
+/* Tape-based batching, sampling (Algorithm 2 "Sampling transitions using   */
+/* TBB"): starting from an empty batch, append the episode                 */
+/* D[I[i] : I[i+1]] of a drawn index i while the batch is shorter than B,   */
+/* then cut it to B transitions.  The draws are an input (the caller's      */
+/* generator), so the batch is a pure function of (I, N, draws, B).  The    */
+/* episode of the last index runs to the end of the buffer (I[E] = N).      */
+/* ======================================================================== */
+
+/* Workspace bytes for memoroid_tbb_sample with up to K draws (also enough
+ * for memoroid_gather_rows, which needs the 256-byte header only). */
+size_t memoroid_tbb_workspace_bytes(int64_t K);
+
+/*
+ *   begin   int64 [E]: the index list I, increasing, into a buffer of N
+ *           transitions (episode i is [begin[i], begin[i+1]), the last one
+ *           [begin[E-1], N))
+ *   draws   int64 [K]: the drawn episode indices, in draw order
+ *   start   uint8 [B] output: 1 where an appended episode begins in the batch
+ *   src     int64 [B] output: buffer index of the transition at each step
+ *   n_used  int64 [1] output (device), or NULL: the draws used (the fewest
+ *           that fill B steps)
+ * All device memory owned by the caller; asynchronous on `stream`.  Bad data
+ * (an index outside [0, E), an empty episode, draws that do not fill B
+ * steps; the uncovered steps get src = -1) is reported as
+ * MEMOROID_ERR_BAD_DATA by memoroid_get_device_error(workspace).
+ */
+memoroid_status_t memoroid_tbb_sample(const int64_t *begin, int64_t E, int64_t N, const int64_t *draws,
+                                      int64_t K, int64_t B, uint8_t *start, int64_t *src,
+                                      int64_t *n_used, void *workspace, size_t workspace_bytes,
+                                      void *stream);
+
+/*
+ * out[t] = rows[src[t]] for t in [0, B): rows is [N, row_bytes] (any row
+ * size; 16-byte copies when row_bytes % 16 == 0 and both arrays are 16-byte
+ * aligned), out is [B, row_bytes] and may not overlap rows.  A source index
+ * outside [0, N) gives a zero row and MEMOROID_ERR_BAD_DATA from
+ * memoroid_get_device_error(workspace).  Workspace: at least 256 bytes.
+ */
+memoroid_status_t memoroid_gather_rows(const void *rows, int64_t N, int64_t row_bytes,
+                                       const int64_t *src, int64_t B, void *out, void *workspace,
+                                       size_t workspace_bytes, void *stream);
 
 /* ======================================================================== */
 /* Discounted return and GAE memoroids (appendices "The Discounted Return   */

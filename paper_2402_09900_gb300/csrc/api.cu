@@ -60,6 +60,7 @@ const char* memoroid_status_string(memoroid_status_t s) {
         case MEMOROID_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
         case MEMOROID_ERR_CUDA: return "CUDA error";
         case MEMOROID_ERR_TIMEOUT: return "device-side wait timed out";
+        case MEMOROID_ERR_BAD_DATA: return "device-side data check failed";
     }
     return "unknown status";
 }
@@ -77,7 +78,8 @@ memoroid_status_t memoroid_get_device_error(const void* workspace, void* stream)
     if (cudaMemcpyAsync(&code, workspace, sizeof(code), cudaMemcpyDeviceToHost, s) != cudaSuccess)
         return MEMOROID_ERR_CUDA;
     if (cudaStreamSynchronize(s) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    return code == DEV_OK ? MEMOROID_OK : MEMOROID_ERR_TIMEOUT;
+    if (code == DEV_OK) return MEMOROID_OK;
+    return code == DEV_BAD_DATA ? MEMOROID_ERR_BAD_DATA : MEMOROID_ERR_TIMEOUT;
 }
 
 // ---------------------------------------------------------------------------
@@ -489,6 +491,45 @@ memoroid_status_t memoroid_ffm_bwd(const float* alpha, const float* omega, const
     f.workspace = workspace;
     f.workspace_bytes = workspace_bytes;
     return diag::launch_ffm(f, s);
+}
+
+// ---------------------------------------------------------------------------
+// tape-based batching: sampling and row gather
+// ---------------------------------------------------------------------------
+
+size_t memoroid_tbb_workspace_bytes(int64_t K) {
+    if (K < 0) return 0;
+    return tbb::workspace_bytes(K);
+}
+
+memoroid_status_t memoroid_tbb_sample(const int64_t* begin, int64_t E, int64_t N, const int64_t* draws, int64_t K,
+                                      int64_t B, uint8_t* start, int64_t* src, int64_t* n_used, void* workspace,
+                                      size_t workspace_bytes, void* stream) {
+    if (E < 0 || N < 0 || K < 0 || B < 0) return MEMOROID_ERR_INVALID_ARG;
+    if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < tbb::workspace_bytes(K))
+        return MEMOROID_ERR_WORKSPACE;
+    cudaStream_t s = as_stream(stream);
+    if (B == 0) {
+        if (cudaMemsetAsync(workspace, 0, kHeaderBytes, s) != cudaSuccess) return MEMOROID_ERR_CUDA;
+        if (n_used && cudaMemsetAsync(n_used, 0, sizeof(int64_t), s) != cudaSuccess) return MEMOROID_ERR_CUDA;
+        return MEMOROID_OK;
+    }
+    if (!start || !src || (K > 0 && (!begin || !draws))) return MEMOROID_ERR_INVALID_ARG;
+    if (!aligned(src, 8) || (begin && !aligned(begin, 8)) || (draws && !aligned(draws, 8)) ||
+        (n_used && !aligned(n_used, 8)))
+        return MEMOROID_ERR_INVALID_ARG;
+    return tbb::launch_sample(begin, E, N, draws, K, B, start, src, n_used, workspace, s);
+}
+
+memoroid_status_t memoroid_gather_rows(const void* rows, int64_t N, int64_t row_bytes, const int64_t* src, int64_t B,
+                                       void* out, void* workspace, size_t workspace_bytes, void* stream) {
+    if (N < 0 || row_bytes <= 0 || B < 0) return MEMOROID_ERR_INVALID_ARG;
+    if (workspace == nullptr || !aligned(workspace, 256) || workspace_bytes < kHeaderBytes)
+        return MEMOROID_ERR_WORKSPACE;
+    cudaStream_t s = as_stream(stream);
+    if (B == 0) return cudaMemsetAsync(workspace, 0, kHeaderBytes, s) == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
+    if (!src || !out || (N > 0 && !rows) || !aligned(src, 8)) return MEMOROID_ERR_INVALID_ARG;
+    return tbb::launch_gather(rows, N, row_bytes, src, B, out, workspace, s);
 }
 
 // ---------------------------------------------------------------------------

@@ -21,6 +21,7 @@ enum DeviceError : uint32_t {
     DEV_ACC_TIMEOUT = 6,       // the wait for grad_lambda partials ran out
     DEV_DRAIN_TIMEOUT = 7,     // the final wait for in-flight copies ran out
     DEV_MMA_TIMEOUT = 8,       // a wait for tensor-core completion ran out
+    DEV_BAD_DATA = 9,          // device-side data check failed (index out of range, too few draws)
 };
 
 // Workspace header (256 bytes): [0] error code, [1] tile ticket counter,
@@ -151,6 +152,14 @@ size_t workspace_bytes(int64_t B, int64_t L);
 memoroid_status_t launch(const float* r, const float* v, const uint8_t* start, float c, float gamma,
                          const float* boot, float* out, int64_t B, int64_t L, void* workspace, cudaStream_t s);
 }  // namespace ret
+
+namespace tbb {
+size_t workspace_bytes(int64_t K);
+memoroid_status_t launch_sample(const int64_t* begin, int64_t E, int64_t N, const int64_t* ep, int64_t K, int64_t B,
+                                uint8_t* start, int64_t* src, int64_t* n_used, void* workspace, cudaStream_t s);
+memoroid_status_t launch_gather(const void* rows, int64_t N, int64_t row_bytes, const int64_t* src, int64_t B,
+                                void* out, void* workspace, cudaStream_t s);
+}  // namespace tbb
 
 namespace tape {
 size_t offsets_workspace_bytes(int64_t L);

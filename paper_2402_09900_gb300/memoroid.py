@@ -25,6 +25,7 @@ MEMOROID_ERR_UNSUPPORTED = 2
 MEMOROID_ERR_WORKSPACE = 3
 MEMOROID_ERR_CUDA = 4
 MEMOROID_ERR_TIMEOUT = 5
+MEMOROID_ERR_BAD_DATA = 6
 MEMOROID_F32 = 0
 MEMOROID_BF16 = 1
 
@@ -55,6 +56,9 @@ SIGNATURES = {
     "memoroid_bench_linattn_intra_scratch_bytes": (_sz, [_i64]),
     "memoroid_bench_linattn_intra": (_int, [_i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_returns_workspace_bytes": (_sz, [_i64, _i64]),
+    "memoroid_tbb_workspace_bytes": (_sz, [_i64]),
+    "memoroid_tbb_sample": (_int, [_p, _i64, _i64, _p, _i64, _i64, _p, _p, _p, _p, _sz, _p]),
+    "memoroid_gather_rows": (_int, [_p, _i64, _i64, _p, _i64, _p, _p, _sz, _p]),
     "memoroid_ffm_workspace_bytes": (_sz, [_i64, _i64, _i64, _i64]),
     "memoroid_ffm_kernels_per_call": (_int, [_i64, _i64, _i64, _i64, _int, _int]),
     "memoroid_ffm_fwd": (_int, [_p, _p, _p, _p, _p, _p, _p, _i64, _i64, _i64, _i64, _p, _sz, _p]),
@@ -227,6 +231,24 @@ def memoroid_gae(r, v, start, gamma, lam, v_boot, A, B, L, workspace, stream=Non
            "memoroid_gae")
 
 
+def memoroid_tbb_workspace_bytes(K) -> int:
+    return int(load().memoroid_tbb_workspace_bytes(K))
+
+
+def memoroid_tbb_sample(begin, E, N, draws, K, B, start, src, n_used, workspace, stream=None):
+    _need_cuda(begin, draws, start, src, n_used, workspace)
+    _check(load().memoroid_tbb_sample(_ptr(begin), E, N, _ptr(draws), K, B, _ptr(start), _ptr(src), _ptr(n_used),
+                                      _ptr(workspace), workspace.numel() if workspace is not None else 0,
+                                      _stream(stream)), "memoroid_tbb_sample")
+
+
+def memoroid_gather_rows(rows, N, row_bytes, src, B, out, workspace, stream=None):
+    _need_cuda(rows, src, out, workspace)
+    _check(load().memoroid_gather_rows(_ptr(rows), N, row_bytes, _ptr(src), B, _ptr(out), _ptr(workspace),
+                                       workspace.numel() if workspace is not None else 0, _stream(stream)),
+           "memoroid_gather_rows")
+
+
 def memoroid_ffm_workspace_bytes(B, L, m, c) -> int:
     return int(load().memoroid_ffm_workspace_bytes(B, L, m, c))
 
@@ -376,6 +398,32 @@ def gae(r, v, start, gamma, lam, v_boot=None, ws=None, stream=None):
     A = torch.empty_like(r)
     memoroid_gae(r, v, start, gamma, lam, v_boot, A, B, L, ws, stream)
     return A
+
+
+def tbb_sample(begin, N, draws, B, ws=None, stream=None):
+    """Algorithm 2 with the draws given: returns start [B] uint8, src [B]
+    int64 and n_used [1] int64 (device tensors).  begin: int64 [E] episode
+    begin indices into a buffer of N transitions; draws: int64 [K]."""
+    E, K = begin.numel(), draws.numel()
+    if ws is None:
+        ws = workspace(memoroid_tbb_workspace_bytes(K), begin.device)
+    start = torch.empty(B, dtype=torch.uint8, device=begin.device)
+    src = torch.empty(B, dtype=torch.int64, device=begin.device)
+    n_used = torch.empty(1, dtype=torch.int64, device=begin.device)
+    memoroid_tbb_sample(begin, E, N, draws, K, B, start, src, n_used, ws, stream)
+    return start, src, n_used
+
+
+def gather_rows(rows, src, ws=None, stream=None):
+    """out[t] = rows[src[t]] for a [N, ...] tensor of rows (any dtype)."""
+    N = rows.shape[0]
+    B = src.numel()
+    row_bytes = rows[0].numel() * rows.element_size() if N > 0 else rows.element_size()
+    if ws is None:
+        ws = workspace(256, rows.device)
+    out = torch.empty((B,) + tuple(rows.shape[1:]), dtype=rows.dtype, device=rows.device)
+    memoroid_gather_rows(rows, N, row_bytes, src, B, out, ws, stream)
+    return out
 
 
 def ffm_workspace(B, L, m, c, device) -> torch.Tensor:
