@@ -30,6 +30,11 @@ Parity status of each routine (what pins it, in tests/test_oracle_pins.py):
                      all-start tapes
   ffm_bwd            torch.autograd (fp64) through an independent loop,
                      central finite differences in alpha and omega
+  linattn_norm_fwd   brute-force normalised weighted sums (gamma = 1: the
+                     paper's model), all-start tapes (y = v), shift equivariance
+                     in v, outputs inside each episode's range of v
+  linattn_norm_bwd   torch.autograd (fp64) through an independent loop,
+                     finite differences
   tbb_sample         the Figure 2 tape worked by hand, and on random inputs the
                      properties that define the batch (whole episodes in draw
                      order, cut at B, flags at piece starts, fewest draws)
@@ -89,6 +94,8 @@ def lib():
             L.oracle_discounted_return.argtypes = [_i64, _i64, _p, _p, _c.c_double, _p, _p]
             L.oracle_gae.argtypes = [_i64, _i64, _p, _p, _p, _c.c_double, _c.c_double, _p, _p]
             L.oracle_offsets_from_starts.argtypes = [_p, _i64, _p]
+            L.oracle_linattn_norm_fwd.argtypes = [_i64] * 5 + [_p] * 4 + [_c.c_int] + [_p] * 7
+            L.oracle_linattn_norm_bwd.argtypes = [_i64] * 5 + [_p] * 4 + [_c.c_int] + [_p] * 12
             L.oracle_tbb_sample.argtypes = [_p, _i64, _i64, _p, _i64, _i64, _p, _p]
             L.oracle_tbb_sample.restype = _i64
             L.oracle_ffm_fwd.argtypes = [_i64] * 4 + [_p] * 7
@@ -250,6 +257,46 @@ def linattn_bwd(q, k, v, gamma, start, dy, dS_last=None, S0=None, gamma_per_step
                                     _ptr(dS_last), _ptr(dq), _ptr(dkk), _ptr(dvv), _ptr(dgamma),
                                     _ptr(dS0)))
     return dq, dkk, dvv, dgamma, dS0
+
+
+def linattn_norm_fwd(q, k, v, gamma, start, S0=None, z0=None, gamma_per_step=None):
+    """The Linear Transformer memoroid with phi = 1 + ELU and its normalizer
+    (decayed by gamma; gamma = 1 is the paper's model): returns y [B,L,H,dv],
+    den [B,L,H], S_last [B,H,dk,dv], z_last [B,H,dk]."""
+    q, k, v, gamma = _f64(q), _f64(k), _f64(v), _f64(gamma)
+    B, L, H, dk = q.shape
+    dv = v.shape[-1]
+    if gamma_per_step is None:
+        gamma_per_step = gamma.ndim == 3
+    start = _u8(start)
+    S0, z0 = _f64(S0), _f64(z0)
+    y = np.zeros((B, L, H, dv))
+    den = np.zeros((B, L, H))
+    S_last = np.zeros((B, H, dk, dv))
+    z_last = np.zeros((B, H, dk))
+    _check(lib().oracle_linattn_norm_fwd(B, L, H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(gamma), int(gamma_per_step),
+                                         _ptr(start), _ptr(S0), _ptr(z0), _ptr(y), _ptr(den), _ptr(S_last),
+                                         _ptr(z_last)))
+    return y, den, S_last, z_last
+
+
+def linattn_norm_bwd(q, k, v, gamma, start, dy, dS_last=None, dz_last=None, S0=None, z0=None, gamma_per_step=None):
+    """Reverse mode of linattn_norm_fwd: dq, dk, dv, dgamma, dS0, dz0."""
+    q, k, v, gamma, dy = _f64(q), _f64(k), _f64(v), _f64(gamma), _f64(dy)
+    B, L, H, dk = q.shape
+    dv = v.shape[-1]
+    if gamma_per_step is None:
+        gamma_per_step = gamma.ndim == 3
+    start = _u8(start)
+    S0, z0, dS_last, dz_last = _f64(S0), _f64(z0), _f64(dS_last), _f64(dz_last)
+    dq, dkk, dvv = np.zeros_like(q), np.zeros_like(k), np.zeros_like(v)
+    dgamma = np.zeros_like(gamma)
+    dS0 = np.zeros((B, H, dk, dv))
+    dz0 = np.zeros((B, H, dk))
+    _check(lib().oracle_linattn_norm_bwd(B, L, H, dk, dv, _ptr(q), _ptr(k), _ptr(v), _ptr(gamma), int(gamma_per_step),
+                                         _ptr(start), _ptr(S0), _ptr(z0), _ptr(dy), _ptr(dS_last), _ptr(dz_last),
+                                         _ptr(dq), _ptr(dkk), _ptr(dvv), _ptr(dgamma), _ptr(dS0), _ptr(dz0)))
+    return dq, dkk, dvv, dgamma, dS0, dz0
 
 
 # ---------------------------------------------------------------------------

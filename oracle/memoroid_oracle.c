@@ -704,3 +704,203 @@ int64_t oracle_tbb_sample(const int64_t *begin, int64_t E, int64_t N, const int6
     }
     return k;
 }
+
+/* ------------------------------------------------------------------------ */
+/* The Linear Transformer memoroid with its feature map and normalizer      */
+/* (Appendix "Linear Transformer"):                                         */
+/*   (X, x) . (X', x') = (X + X', x + x'),                                   */
+/*   f(o, b) = (phi(k) v^T, phi(k)),  g = X^T phi(q) / (x^T phi(q)),         */
+/*   phi(z) = 1 + ELU(z) (= 1 + z for z > 0, exp(z) otherwise),              */
+/* with the same multiplicative decay gamma_t on the carried pair as the     */
+/* decayed memoroid above (gamma = 1 is the paper's model) and the reset of  */
+/* Theorem 3.2.  The readout X^T phi(q) follows the reading y = S^T q.      */
+/* ------------------------------------------------------------------------ */
+
+static inline double phi1(double z) { return z > 0.0 ? 1.0 + z : exp(z); }
+static inline double dphi1(double z) { return z > 0.0 ? 1.0 : exp(z); }
+
+/*
+ * q, k: [B,L,H,dk]; v: [B,L,H,dv]; gamma: [H] or [B,L,H]; start: [B,L];
+ * S0, S_last: [B,H,dk,dv] or NULL; z0, z_last: [B,H,dk] or NULL (the
+ * normalizer state x); y: [B,L,H,dv]; den: [B,L,H] or NULL (x^T phi(q)).
+ */
+int oracle_linattn_norm_fwd(int64_t B, int64_t L, int64_t H, int64_t dk, int64_t dv, const double *q,
+                            const double *k, const double *v, const double *gamma, int gamma_per_step,
+                            const uint8_t *start, const double *S0, const double *z0, double *y, double *den,
+                            double *S_last, double *z_last)
+{
+    if (B < 0 || L < 0 || H < 0 || dk <= 0 || dv <= 0) return -1;
+    int bad = 0;
+#pragma omp parallel for collapse(2) schedule(dynamic) reduction(| : bad)
+    for (int64_t b = 0; b < B; ++b) {
+        for (int64_t hh = 0; hh < H; ++hh) {
+            double *X = (double *)calloc((size_t)(dk * dv), sizeof(double));
+            double *x = (double *)calloc((size_t)dk, sizeof(double));
+            double *pk = (double *)malloc(sizeof(double) * (size_t)dk);
+            double *pq = (double *)malloc(sizeof(double) * (size_t)dk);
+            if (!X || !x || !pk || !pq) {
+                free(X); free(x); free(pk); free(pq);
+                bad = 1;
+                continue;
+            }
+            if (S0) memcpy(X, S0 + (b * H + hh) * dk * dv, sizeof(double) * dk * dv);
+            if (z0) memcpy(x, z0 + (b * H + hh) * dk, sizeof(double) * dk);
+            for (int64_t t = 0; t < L; ++t) {
+                const int64_t r = (b * L + t) * H + hh;
+                const int reset = start[b * L + t] != 0;
+                const double gt = reset ? 0.0 : gam_at(gamma, gamma_per_step, b, t, L, H, hh);
+                for (int64_t i = 0; i < dk; ++i) {
+                    pk[i] = phi1(k[r * dk + i]);
+                    pq[i] = phi1(q[r * dk + i]);
+                }
+                /* (X, x) <- gamma (X, x) . f(o_t), or f(o_t) at a begin flag */
+                for (int64_t i = 0; i < dk; ++i) {
+                    for (int64_t j = 0; j < dv; ++j)
+                        X[i * dv + j] = (reset ? 0.0 : gt * X[i * dv + j]) + pk[i] * v[r * dv + j];
+                    x[i] = (reset ? 0.0 : gt * x[i]) + pk[i];
+                }
+                double d = 0.0;
+                for (int64_t i = 0; i < dk; ++i) d += x[i] * pq[i];
+                for (int64_t j = 0; j < dv; ++j) {
+                    double n = 0.0;
+                    for (int64_t i = 0; i < dk; ++i) n += X[i * dv + j] * pq[i];
+                    y[r * dv + j] = n / d;
+                }
+                if (den) den[r] = d;
+            }
+            if (S_last) memcpy(S_last + (b * H + hh) * dk * dv, X, sizeof(double) * dk * dv);
+            if (z_last) memcpy(z_last + (b * H + hh) * dk, x, sizeof(double) * dk);
+            free(X); free(x); free(pk); free(pq);
+        }
+    }
+    return bad ? -2 : 0;
+}
+
+/*
+ * Backward of oracle_linattn_norm_fwd (reverse mode).  With n_t = X_t^T phi(q_t),
+ * d_t = x_t^T phi(q_t), y_t = n_t / d_t:
+ *   dn_t = dy_t / d_t,  dd_t = -(dy_t . y_t) / d_t,
+ *   dX_t = phi(q_t) dn_t^T + [b_{t+1} = 0] gamma_{t+1} dX_{t+1}   (+ dS_last at L-1)
+ *   dx_t = phi(q_t) dd_t   + [b_{t+1} = 0] gamma_{t+1} dx_{t+1}   (+ dz_last at L-1)
+ *   dq_t = (X_t dn_t + x_t dd_t) (.) phi'(q_t),  dk_t = (dX_t v_t + dx_t) (.) phi'(k_t),
+ *   dv_t = dX_t^T phi(k_t),  dgamma_t = [b_t = 0] (<dX_t, X_{t-1}> + dx_t . x_{t-1}),
+ *   dS0 = [b_0 = 0] gamma_0 dX_0,  dz0 = [b_0 = 0] gamma_0 dx_0.
+ * dgamma is [H] (summed over B, L) or [B,L,H].  Any output may be NULL.
+ */
+int oracle_linattn_norm_bwd(int64_t B, int64_t L, int64_t H, int64_t dk, int64_t dv, const double *q,
+                            const double *k, const double *v, const double *gamma, int gamma_per_step,
+                            const uint8_t *start, const double *S0, const double *z0, const double *dy,
+                            const double *dS_last, const double *dz_last, double *dq, double *dkk, double *dvv,
+                            double *dgamma, double *dS0, double *dz0)
+{
+    if (B < 0 || L < 0 || H < 0 || dk <= 0 || dv <= 0) return -1;
+    const int64_t M = dk * dv, W = M + dk; /* one state: X (M values) then x (dk values) */
+    double *gsum = (dgamma && !gamma_per_step) ? (double *)calloc((size_t)(B * H > 0 ? B * H : 1), sizeof(double)) : NULL;
+    int bad = 0;
+#pragma omp parallel for collapse(2) schedule(dynamic) reduction(| : bad)
+    for (int64_t b = 0; b < B; ++b) {
+        for (int64_t hh = 0; hh < H; ++hh) {
+            /* all states of the row: slot t + 1 holds (X_t, x_t), slot 0 the state before step 0 */
+            double *St = (double *)calloc((size_t)((L + 1) * W), sizeof(double));
+            double *G = (double *)calloc((size_t)W, sizeof(double)); /* (dX, dx) */
+            double *pq = (double *)malloc(sizeof(double) * (size_t)dk);
+            double *pk = (double *)malloc(sizeof(double) * (size_t)dk);
+            double *dn = (double *)malloc(sizeof(double) * (size_t)dv);
+            if (!St || !G || !pq || !pk || !dn) {
+                free(St); free(G); free(pq); free(pk); free(dn);
+                bad = 1;
+                continue;
+            }
+            if (S0) memcpy(St, S0 + (b * H + hh) * M, sizeof(double) * M);
+            if (z0) memcpy(St + M, z0 + (b * H + hh) * dk, sizeof(double) * dk);
+            for (int64_t t = 0; t < L; ++t) {
+                const int64_t r = (b * L + t) * H + hh;
+                const int reset = start[b * L + t] != 0;
+                const double gt = reset ? 0.0 : gam_at(gamma, gamma_per_step, b, t, L, H, hh);
+                const double *P = St + t * W;
+                double *C = St + (t + 1) * W;
+                for (int64_t i = 0; i < dk; ++i) {
+                    const double f = phi1(k[r * dk + i]);
+                    for (int64_t j = 0; j < dv; ++j) C[i * dv + j] = (reset ? 0.0 : gt * P[i * dv + j]) + f * v[r * dv + j];
+                    C[M + i] = (reset ? 0.0 : gt * P[M + i]) + f;
+                }
+            }
+            double gacc = 0.0;
+            for (int64_t t = L - 1; t >= 0; --t) {
+                const int64_t r = (b * L + t) * H + hh;
+                const double *C = St + (t + 1) * W, *P = St + t * W;
+                if (t == L - 1) {
+                    for (int64_t w = 0; w < W; ++w) G[w] = 0.0;
+                    if (dS_last) memcpy(G, dS_last + (b * H + hh) * M, sizeof(double) * M);
+                    if (dz_last) memcpy(G + M, dz_last + (b * H + hh) * dk, sizeof(double) * dk);
+                } else {
+                    const double gn = start[b * L + t + 1] ? 0.0 : gam_at(gamma, gamma_per_step, b, t + 1, L, H, hh);
+                    for (int64_t w = 0; w < W; ++w) G[w] *= gn;
+                }
+                for (int64_t i = 0; i < dk; ++i) {
+                    pq[i] = phi1(q[r * dk + i]);
+                    pk[i] = phi1(k[r * dk + i]);
+                }
+                double d = 0.0;
+                for (int64_t i = 0; i < dk; ++i) d += C[M + i] * pq[i];
+                double dyy = 0.0;
+                for (int64_t j = 0; j < dv; ++j) {
+                    double n = 0.0;
+                    for (int64_t i = 0; i < dk; ++i) n += C[i * dv + j] * pq[i];
+                    dyy += dy[r * dv + j] * (n / d);
+                    dn[j] = dy[r * dv + j] / d;
+                }
+                const double dd = -dyy / d;
+                for (int64_t i = 0; i < dk; ++i) {
+                    for (int64_t j = 0; j < dv; ++j) G[i * dv + j] += pq[i] * dn[j];
+                    G[M + i] += pq[i] * dd;
+                }
+                for (int64_t i = 0; i < dk; ++i) {
+                    double a = C[M + i] * dd, c = G[M + i];
+                    for (int64_t j = 0; j < dv; ++j) {
+                        a += C[i * dv + j] * dn[j];
+                        c += G[i * dv + j] * v[r * dv + j];
+                    }
+                    if (dq) dq[r * dk + i] = a * dphi1(q[r * dk + i]);
+                    if (dkk) dkk[r * dk + i] = c * dphi1(k[r * dk + i]);
+                }
+                if (dvv) {
+                    for (int64_t j = 0; j < dv; ++j) {
+                        double a = 0.0;
+                        for (int64_t i = 0; i < dk; ++i) a += G[i * dv + j] * pk[i];
+                        dvv[r * dv + j] = a;
+                    }
+                }
+                double dg = 0.0;
+                if (!start[b * L + t])
+                    for (int64_t w = 0; w < W; ++w) dg += G[w] * P[w];
+                if (dgamma) {
+                    if (gamma_per_step) dgamma[r] = dg;
+                    else gacc += dg;
+                }
+            }
+            if (dS0 || dz0) {
+                double g0 = (L > 0 && !start[b * L]) ? gam_at(gamma, gamma_per_step, b, 0, L, H, hh) : 0.0;
+                if (L == 0) { /* nothing between the states: the gradient passes through */
+                    for (int64_t w = 0; w < W; ++w) G[w] = 0.0;
+                    if (dS_last) memcpy(G, dS_last + (b * H + hh) * M, sizeof(double) * M);
+                    if (dz_last) memcpy(G + M, dz_last + (b * H + hh) * dk, sizeof(double) * dk);
+                    g0 = 1.0;
+                }
+                if (dS0) for (int64_t w = 0; w < M; ++w) dS0[(b * H + hh) * M + w] = g0 * G[w];
+                if (dz0) for (int64_t i = 0; i < dk; ++i) dz0[(b * H + hh) * dk + i] = g0 * G[M + i];
+            }
+            if (gsum) gsum[b * H + hh] = gacc;
+            free(St); free(G); free(pq); free(pk); free(dn);
+        }
+    }
+    if (gsum) {
+        for (int64_t hh = 0; hh < H; ++hh) {
+            double acc = 0.0;
+            for (int64_t b = 0; b < B; ++b) acc += gsum[b * H + hh];
+            dgamma[hh] = acc;
+        }
+        free(gsum);
+    }
+    return bad ? -2 : 0;
+}

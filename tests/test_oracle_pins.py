@@ -840,3 +840,145 @@ def test_tbb_sample_exact_fit_and_errors():
         oracle.tbb_sample(FIG2_I, FIG2_N, np.array([2, 2]), 5)  # two 1-step episodes cannot fill 5 steps
     with pytest.raises(ValueError):
         oracle.tbb_sample(FIG2_I, FIG2_N, np.array([4]), 2)  # no episode 4
+
+
+# ---------------------------------------------------------------------------
+# the Linear Transformer with phi = 1 + ELU and its normalizer (Appendix "Linear Transformer")
+# ---------------------------------------------------------------------------
+
+def _phi_np(z):
+    return np.where(z > 0, 1.0 + z, np.exp(np.minimum(z, 0.0)))
+
+
+def _norm_inputs(rng, B, L, H, d, per_step, p=0.1, first=True):
+    q = rng.standard_normal((B, L, H, d))
+    k = rng.standard_normal((B, L, H, d))
+    v = rng.standard_normal((B, L, H, d))
+    gamma = rng.uniform(0.7, 1.0, (B, L, H) if per_step else (H,))
+    start = _random_starts(rng, B, L, p, first=first)
+    S0 = rng.standard_normal((B, H, d, d))
+    z0 = rng.uniform(0.5, 2.0, (B, H, d))  # a normalizer state is a sum of positive features
+    return q, k, v, gamma, start, S0, z0
+
+
+@pytest.mark.parametrize("per_step", [False, True])
+@pytest.mark.parametrize("first", [True, False])
+def test_linattn_norm_brute_force_weighted_average(per_step, first):
+    # y_t = sum_r w_tr v_r / sum_r w_tr with w_tr = (prod of gamma over (r, t]) phi(q_t).phi(k_r)
+    # over the steps r <= t of t's episode (plus the incoming state for a continued row)
+    rng = _rng(70)
+    B, L, H, d = 2, 30, 2, 3
+    q, k, v, gamma, start, S0, z0 = _norm_inputs(rng, B, L, H, d, per_step, first=first)
+    y, den, S_last, z_last = oracle.linattn_norm_fwd(q, k, v, gamma, start, S0, z0)
+    for b in range(B):
+        for h in range(H):
+            for t in range(L):
+                s = t
+                while s > 0 and not start[b, s]:
+                    s -= 1
+                num = np.zeros(d)
+                dd = 0.0
+                for r in range(s, t + 1):
+                    w = 1.0
+                    for j in range(r + 1, t + 1):
+                        w *= gamma[b, j, h] if per_step else gamma[h]
+                    a = w * float(_phi_np(q[b, t, h]) @ _phi_np(k[b, r, h]))
+                    num += a * v[b, r, h]
+                    dd += a
+                if not start[b, s]:  # a continued row carries (S0, z0) decayed over [0, t]
+                    w = 1.0
+                    for j in range(0, t + 1):
+                        w *= gamma[b, j, h] if per_step else gamma[h]
+                    num += w * (S0[b, h].T @ _phi_np(q[b, t, h]))
+                    dd += w * float(z0[b, h] @ _phi_np(q[b, t, h]))
+                np.testing.assert_allclose(y[b, t, h], num / dd, rtol=1e-10, atol=1e-12)
+                assert den[b, t, h] == pytest.approx(dd, rel=1e-10)
+
+
+def test_linattn_norm_all_start_and_shift_equivariance():
+    rng = _rng(71)
+    B, L, H, d = 1, 40, 2, 4
+    q, k, v, gamma, _, _, _ = _norm_inputs(rng, B, L, H, d, False)
+    ones = np.ones((B, L), np.uint8)
+    y, _, _, _ = oracle.linattn_norm_fwd(q, k, v, gamma, ones)
+    np.testing.assert_allclose(y, v, rtol=1e-12, atol=1e-12)  # one term: the weight cancels
+    start = _random_starts(rng, B, L, 0.15)
+    y1, _, _, _ = oracle.linattn_norm_fwd(q, k, v, gamma, start)
+    y2, _, _, _ = oracle.linattn_norm_fwd(q, k, v + 3.5, gamma, start)
+    np.testing.assert_allclose(y2, y1 + 3.5, rtol=1e-12, atol=1e-11)  # normalised weights sum to 1
+    # each output lies within the range of v over its episode so far
+    for t in range(L):
+        s = t
+        while s > 0 and not start[0, s]:
+            s -= 1
+        lo = v[0, s:t + 1].min(axis=0)
+        hi = v[0, s:t + 1].max(axis=0)
+        assert np.all(y1[0, t] >= lo - 1e-12) and np.all(y1[0, t] <= hi + 1e-12)
+
+
+def _torch_norm_loss(torch, q, k, v, gamma, start, S0, z0, dy, dSl, dzl, per_step):
+    def phi(z):
+        return torch.where(z > 0, 1.0 + z, torch.exp(torch.clamp(z, max=0.0)))
+    B, L, H, d = q.shape
+    loss = 0.0
+    for b in range(B):
+        for h in range(H):
+            X, x = S0[b, h], z0[b, h]
+            for t in range(L):
+                g = gamma[b, t, h] if per_step else gamma[h]
+                pk, pq = phi(k[b, t, h]), phi(q[b, t, h])
+                if start[b, t]:
+                    X, x = torch.outer(pk, v[b, t, h]), pk
+                else:
+                    X, x = g * X + torch.outer(pk, v[b, t, h]), g * x + pk
+                y = (X.T @ pq) / (x @ pq)
+                loss = loss + (dy[b, t, h] * y).sum()
+            loss = loss + (dSl[b, h] * X).sum() + (dzl[b, h] * x).sum()
+    return loss
+
+
+@pytest.mark.parametrize("per_step", [False, True])
+@pytest.mark.parametrize("first", [True, False])
+def test_linattn_norm_bwd_vs_torch_autograd(per_step, first):
+    torch = pytest.importorskip("torch")
+    rng = _rng(72)
+    B, L, H, d = 2, 14, 2, 3
+    q, k, v, gamma, start, S0, z0 = _norm_inputs(rng, B, L, H, d, per_step, 0.2, first=first)
+    dy = rng.standard_normal((B, L, H, d))
+    dSl = rng.standard_normal((B, H, d, d))
+    dzl = rng.standard_normal((B, H, d))
+    T = [torch.tensor(a, requires_grad=True) for a in (q, k, v, gamma, S0, z0)]
+    loss = _torch_norm_loss(torch, *T[:4], start, T[4], T[5], torch.tensor(dy), torch.tensor(dSl),
+                            torch.tensor(dzl), per_step)
+    loss.backward()
+    got = oracle.linattn_norm_bwd(q, k, v, gamma, start, dy, dSl, dzl, S0, z0)
+    for g, t in zip(got, T):
+        ref = np.zeros_like(g) if t.grad is None else t.grad.numpy()
+        np.testing.assert_allclose(g, ref, rtol=1e-9, atol=1e-10)
+
+
+def test_linattn_norm_bwd_finite_differences():
+    rng = _rng(73)
+    B, L, H, d = 1, 10, 1, 2
+    q, k, v, gamma, start, S0, z0 = _norm_inputs(rng, B, L, H, d, False, 0.0, first=False)
+    start[0, 6] = 1
+    dy = rng.standard_normal((B, L, H, d))
+
+    def loss(q_, k_, v_, g_):
+        y, _, _, _ = oracle.linattn_norm_fwd(q_, k_, v_, g_, start, S0, z0)
+        return float(np.sum(dy * y))
+
+    dq, dk, dv, dg, _, _ = oracle.linattn_norm_bwd(q, k, v, gamma, start, dy, None, None, S0, z0)
+    eps = 1e-6
+
+    def fd(arr, idx, f):
+        a1, a2 = arr.copy(), arr.copy()
+        a1[idx] += eps
+        a2[idx] -= eps
+        return (f(a1) - f(a2)) / (2 * eps)
+
+    for idx in [(0, 0, 0, 0), (0, 5, 0, 1), (0, 6, 0, 0), (0, 9, 0, 1)]:
+        assert abs(fd(q, idx, lambda a: loss(a, k, v, gamma)) - dq[idx]) < 1e-6
+        assert abs(fd(k, idx, lambda a: loss(q, a, v, gamma)) - dk[idx]) < 1e-6
+        assert abs(fd(v, idx, lambda a: loss(q, k, a, gamma)) - dv[idx]) < 1e-6
+    assert abs(fd(gamma, (0,), lambda a: loss(q, k, v, a)) - dg[0]) < 1e-6
