@@ -11,9 +11,10 @@ memoroid_scan_linattn_fwd + memoroid_scan_linattn_bwd, plus the tensor-core
 throughput of the intra-tile contraction alone (memoroid_bench_linattn_intra).
 Its "returns" object times the per-step discounted return and GAE with resets
 on 64 tapes of 2^20 steps, its "ffm" object the Fast and Forgetful Memory
-memoroid (fwd + bwd) on a 2^20-step tape with a 64 x 4 complex state, and its
+memoroid (fwd + bwd) on a 2^20-step tape with a 64 x 4 complex state, its
 "tbb" object the device-side sampling of a 2^20-step batch (Algorithm 2) and
-the gather of its 2 KB rows.
+the gather of its 2 KB rows, and its "linattn_norm" object the paper's Linear
+Transformer (phi = 1 + ELU, normalizer) fwd + bwd on the config-3 shape.
 
   python bench.py [--gpus N --steps K --warmup W] [--impl reference]
 
@@ -198,6 +199,75 @@ def ffm_leg(args, m, dev, stream):
         "gpu_launches": steps * kpc,
     }
     del x, gz, z, gx, ws
+    torch.cuda.empty_cache()
+    return out
+
+
+LNORM_WORKLOAD = ("Linear Transformer with phi = 1 + ELU and its normalizer, fwd+bwd: B=1 tape x L=2^18 steps, "
+                  "4 heads, d=64, bf16 q/k/v ~ N(0,1), per-head gamma in {0.9, 0.99, 0.999, 1.0}, Geometric(300) episodes")
+
+
+def lnorm_leg(args, m, dev, stream):
+    """Times memoroid_linattn_norm_fwd + _bwd on the config-3 shape."""
+    import torch
+
+    B, L, H, d = 1, 1 << 18, 4, 64
+    t = tapegen.linattn_tape(B, L, H, d, d, tapegen.seed_for(9), mean=300.0, gamma_mode="head", scale=1.0,
+                             normalize_k=False)
+
+    def bits(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev)
+
+    q, k, v = bits(t["q"]), bits(t["k"]), bits(t["v"])
+    gamma, start = torch.from_numpy(t["gamma"]).to(dev), torch.from_numpy(t["start"]).to(dev)
+    dy = torch.from_numpy(t["grad_y"]).to(dev)
+    ws = m.workspace(m.memoroid_linattn_norm_workspace_bytes(B, L, H, d), dev)
+    y = torch.empty((B, L, H, d), dtype=torch.float32, device=dev)
+    den = torch.empty((B, L, H), dtype=torch.float32, device=dev)
+    dq, dk, dv = torch.empty_like(y), torch.empty_like(y), torch.empty_like(y)
+    dg = torch.empty_like(gamma)
+
+    def fwd():
+        m.memoroid_linattn_norm_fwd(q, k, v, gamma, 0, start, None, None, y, den, None, None, B, L, H, d, ws, stream)
+
+    def bwd():
+        m.memoroid_linattn_norm_bwd(q, k, v, gamma, 0, start, None, None, y, den, dy, None, None, dq, dk, dv, dg,
+                                    None, None, B, L, H, d, ws, stream)
+
+    for _ in range(3):
+        fwd()
+        bwd()
+    torch.cuda.synchronize()
+    steps = args.lnorm_steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for i in range(steps):
+        evs[i][0].record(stream)
+        fwd()
+        evs[i][1].record(stream)
+        bwd()
+        evs[i][2].record(stream)
+    torch.cuda.synchronize()
+    if m.memoroid_get_device_error(ws) != m.MEMOROID_OK:
+        raise RuntimeError("device-side error in the normalised linattn leg")
+    f_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / steps
+    b_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / steps
+    el = B * L * H * d
+    # algorithmic bytes: fwd reads q, k, v (bf16) and the flags, writes y and den; bwd reads
+    # q, k, v, y, den, dy and the flags, writes dq, dk, dv
+    fb = el * (3 * 2 + 4) + B * L * H * 4 + B * L
+    bb = el * (3 * 2 + 4 + 4 + 3 * 4) + B * L * H * 4 + B * L
+    peak, peak_kind = _peaks()
+    kpc = (m.memoroid_linattn_norm_kernels_per_call(B, L, H, d, 0, 0, 0)
+           + m.memoroid_linattn_norm_kernels_per_call(B, L, H, d, 1, 0, 0))
+    out = {"workload": LNORM_WORKLOAD, "value": B * L / ((f_ms + b_ms) * 1e-3), "unit": UNIT, "steps": steps,
+           "ms_per_step": f_ms + b_ms, "fwd_ms": f_ms, "bwd_ms": b_ms,
+           "roofline": {"bound": "hbm", "peak": peak, "unit": "GB/s", "peak_kind": f"{peak_kind} (copy bandwidth)",
+                        "fwd": {"algorithmic_bytes_per_call": fb, "achieved": fb / (f_ms * 1e-3) / 1e9,
+                                "frac": fb / (f_ms * 1e-3) / 1e9 / peak},
+                        "bwd": {"algorithmic_bytes_per_call": bb, "achieved": bb / (b_ms * 1e-3) / 1e9,
+                                "frac": bb / (b_ms * 1e-3) / 1e9 / peak}},
+           "gpu_launches": steps * kpc}
+    del q, k, v, y, dq, dk, dv, ws
     torch.cuda.empty_cache()
     return out
 
@@ -524,6 +594,10 @@ def run_ours(args):
         # profiling mode: the discounted-return / GAE leg alone
         print(json.dumps({"returns": returns_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
         return
+    if args.only_lnorm:
+        # profiling mode: the normalised Linear Transformer leg alone
+        print(json.dumps({"linattn_norm": lnorm_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
+        return
     if args.only_tbb:
         # profiling mode: the tape-based batching leg alone
         print(json.dumps({"tbb": tbb_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
@@ -698,6 +772,9 @@ def run_ours(args):
     ff = None
     if ws == 1 and not args.skip_ffm:
         ff = ffm_leg(args, m, dev, stream)
+    ln = None
+    if ws == 1 and not args.skip_lnorm:
+        ln = lnorm_leg(args, m, dev, stream)
     tb = None
     if ws == 1 and not args.skip_tbb:
         tb = tbb_leg(args, m, dev, stream)
@@ -719,6 +796,7 @@ def run_ours(args):
         "returns": rt,
         "ffm": ff,
         "tbb": tb,
+        "linattn_norm": ln,
     }
     print(json.dumps(out), flush=True)
     if ws > 1:
@@ -750,6 +828,10 @@ def main():
     ap.add_argument("--ret-steps", type=int, default=20, help="timed calls of each returns kernel")
     ap.add_argument("--skip-ffm", action="store_true", help="omit the Fast and Forgetful Memory leg")
     ap.add_argument("--skip-tbb", action="store_true", help="omit the tape-based batching leg")
+    ap.add_argument("--skip-lnorm", action="store_true", help="omit the normalised Linear Transformer leg")
+    ap.add_argument("--only-lnorm", action="store_true",
+                    help="profiling mode: run and print only the normalised Linear Transformer leg")
+    ap.add_argument("--lnorm-steps", type=int, default=10, help="timed normalised Linear Transformer steps")
     ap.add_argument("--only-tbb", action="store_true",
                     help="profiling mode: run and print only the tape-based batching leg")
     ap.add_argument("--tbb-steps", type=int, default=20, help="timed calls of the sampler and of the gather")

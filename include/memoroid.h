@@ -218,6 +218,56 @@ memoroid_status_t memoroid_scan_linattn_bwd(const void *q, const void *k, const 
                                             size_t workspace_bytes, void *stream);
 
 /* ======================================================================== */
+/* The Linear Transformer memoroid with its feature map and normalizer      */
+/* (appendix "Linear Transformer"): (X, x) . (X', x') = (X + X', x + x'),   */
+/* f(o) = (phi(k) v^T, phi(k)), y = X^T phi(q) / (x^T phi(q)),              */
+/* phi(z) = 1 + ELU(z); the pair is decayed by gamma_t like the decayed     */
+/* memoroid above (gamma = 1 is the paper's model) and reset at begin       */
+/* flags.  Heads of width d in {8, 16, ..., 120}; q, k, v bf16.            */
+/* ======================================================================== */
+
+/* Workspace bytes for memoroid_linattn_norm_fwd/_bwd (0 for a bad shape). */
+size_t memoroid_linattn_norm_workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t d);
+
+/* Kernel launches of one call (with_states: all optional state arguments given). */
+int memoroid_linattn_norm_kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t d, int backward,
+                                           int with_dgamma_per_head, int with_states);
+
+/*
+ *   q, k, v  bf16 [B, L, H, d] (16-byte aligned); gamma fp32 [H] or
+ *            [B, L, H] (gamma_per_step); start uint8 [B, L]
+ *   S0, z0   fp32 [B, H, d, d] and [B, H, d]: the pair (X, x) before step 0
+ *            of rows with start[b][0] = 0, or NULL (= 0)
+ *   y        fp32 [B, L, H, d] output; den fp32 [B, L, H] output x^T phi(q)
+ *            (needed by the backward), or NULL
+ *   S_last, z_last  the pair after the last step, or NULL
+ * B, L, H > 0 (an empty call returns MEMOROID_ERR_UNSUPPORTED).  Workspace
+ * 256-byte aligned, at least memoroid_linattn_norm_workspace_bytes; its
+ * header reports device-side waits through memoroid_get_device_error.
+ */
+memoroid_status_t memoroid_linattn_norm_fwd(const void *q, const void *k, const void *v,
+                                            const float *gamma, int gamma_per_step,
+                                            const uint8_t *start, const float *S0, const float *z0,
+                                            float *y, float *den, float *S_last, float *z_last,
+                                            int64_t B, int64_t L, int64_t H, int64_t d,
+                                            void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * Backward: y and den are the forward's outputs; grad_y fp32 [B, L, H, d];
+ * grad_S_last / grad_z_last or NULL; outputs dq, dk, dv fp32 [B, L, H, d],
+ * dgamma ([H] summed, or [B, L, H]; NULL to skip), dS0 / dz0 or NULL.
+ */
+memoroid_status_t memoroid_linattn_norm_bwd(const void *q, const void *k, const void *v,
+                                            const float *gamma, int gamma_per_step,
+                                            const uint8_t *start, const float *S0, const float *z0,
+                                            const float *y, const float *den, const float *grad_y,
+                                            const float *grad_S_last, const float *grad_z_last,
+                                            float *dq, float *dk, float *dv, float *dgamma,
+                                            float *dS0, float *dz0, int64_t B, int64_t L, int64_t H,
+                                            int64_t d, void *workspace, size_t workspace_bytes,
+                                            void *stream);
+
+/* ======================================================================== */
 /* Fast and Forgetful Memory memoroid (appendix "Fast and Forgetful         */
 /* Memory"): (X, t) . (X', t') = (X (.) exp(t'(-|alpha| (+) i omega)) + X', */
 /* t + t') with f(o, b) = (x~ repeated over the c columns, 1), made         */

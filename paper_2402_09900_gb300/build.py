@@ -19,7 +19,7 @@ INCLUDE = os.path.join(os.path.dirname(PKG), "include")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB_NAME = "libmemoroid.so"
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["api.cu", "diag_scan.cu", "linattn.cu", "returns.cu", "tbb.cu", "tape_index.cu", "no_alloc.cu"]
+SOURCES = ["api.cu", "diag_scan.cu", "linattn.cu", "linattn_norm.cu", "returns.cu", "tbb.cu", "tape_index.cu", "no_alloc.cu"]
 
 
 def nvcc() -> str:

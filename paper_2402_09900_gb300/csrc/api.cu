@@ -494,6 +494,100 @@ memoroid_status_t memoroid_ffm_bwd(const float* alpha, const float* omega, const
 }
 
 // ---------------------------------------------------------------------------
+// the Linear Transformer with phi = 1 + ELU and its normalizer
+// ---------------------------------------------------------------------------
+
+static bool lnorm_shape_ok(int64_t B, int64_t L, int64_t H, int64_t d) {
+    return B >= 0 && L >= 0 && H >= 0 && d >= 8 && d <= 120 && (d % 8) == 0;
+}
+
+size_t memoroid_linattn_norm_workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t d) {
+    if (!lnorm_shape_ok(B, L, H, d)) return 0;
+    return lnorm::workspace_bytes(B, L, H);
+}
+
+int memoroid_linattn_norm_kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t d, int backward,
+                                           int with_dgamma_per_head, int with_states) {
+    if (!lnorm_shape_ok(B, L, H, d)) return -1;
+    return lnorm::kernels_per_call(B, L, H, backward != 0, with_dgamma_per_head != 0, with_states != 0);
+}
+
+static memoroid_status_t lnorm_common(lnorm::Args& a, const float* gamma, int gamma_per_step, const uint8_t* start,
+                                      size_t workspace_bytes, void* stream) {
+    if (!lnorm_shape_ok(a.B, a.L, a.H, a.d)) return MEMOROID_ERR_INVALID_ARG;
+    if (gamma_per_step != 0 && gamma_per_step != 1) return MEMOROID_ERR_INVALID_ARG;
+    if (a.B == 0 || a.L == 0 || a.H == 0) return MEMOROID_ERR_UNSUPPORTED;  // nothing to scan: states pass through
+    if (!a.q || !a.k || !a.v || !gamma || !start || !a.y) return MEMOROID_ERR_INVALID_ARG;
+    if (!aligned(a.q, 16) || !aligned(a.k, 16) || !aligned(a.v, 16) || !aligned(a.y, 4) || !aligned(gamma, 4))
+        return MEMOROID_ERR_INVALID_ARG;
+    if (a.workspace == nullptr || !aligned(a.workspace, 256) ||
+        workspace_bytes < lnorm::workspace_bytes(a.B, a.L, a.H))
+        return MEMOROID_ERR_WORKSPACE;
+    a.gamma = gamma;
+    a.gamma_per_step = gamma_per_step;
+    a.start = start;
+    return lnorm::launch(a, as_stream(stream));
+}
+
+memoroid_status_t memoroid_linattn_norm_fwd(const void* q, const void* k, const void* v, const float* gamma,
+                                            int gamma_per_step, const uint8_t* start, const float* S0,
+                                            const float* z0, float* y, float* den, float* S_last, float* z_last,
+                                            int64_t B, int64_t L, int64_t H, int64_t d, void* workspace,
+                                            size_t workspace_bytes, void* stream) {
+    lnorm::Args a{};
+    a.backward = false;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.S0 = S0;
+    a.z0 = z0;
+    a.y = y;
+    a.den = den;
+    a.S_last = S_last;
+    a.z_last = z_last;
+    a.B = B;
+    a.L = L;
+    a.H = H;
+    a.d = d;
+    a.workspace = workspace;
+    return lnorm_common(a, gamma, gamma_per_step, start, workspace_bytes, stream);
+}
+
+memoroid_status_t memoroid_linattn_norm_bwd(const void* q, const void* k, const void* v, const float* gamma,
+                                            int gamma_per_step, const uint8_t* start, const float* S0,
+                                            const float* z0, const float* y, const float* den, const float* grad_y,
+                                            const float* grad_S_last, const float* grad_z_last, float* dq, float* dk,
+                                            float* dv, float* dgamma, float* dS0, float* dz0, int64_t B, int64_t L,
+                                            int64_t H, int64_t d, void* workspace, size_t workspace_bytes,
+                                            void* stream) {
+    if (B > 0 && L > 0 && H > 0 && (!den || !grad_y || !dq || !dk || !dv)) return MEMOROID_ERR_INVALID_ARG;
+    lnorm::Args a{};
+    a.backward = true;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.S0 = S0;
+    a.z0 = z0;
+    a.y = const_cast<float*>(y);
+    a.den = const_cast<float*>(den);
+    a.grad_y = grad_y;
+    a.dS_last = grad_S_last;
+    a.dz_last = grad_z_last;
+    a.dq = dq;
+    a.dk = dk;
+    a.dv = dv;
+    a.dgamma = dgamma;
+    a.dS0 = dS0;
+    a.dz0 = dz0;
+    a.B = B;
+    a.L = L;
+    a.H = H;
+    a.d = d;
+    a.workspace = workspace;
+    return lnorm_common(a, gamma, gamma_per_step, start, workspace_bytes, stream);
+}
+
+// ---------------------------------------------------------------------------
 // tape-based batching: sampling and row gather
 // ---------------------------------------------------------------------------
 

@@ -153,6 +153,30 @@ memoroid_status_t launch(const float* r, const float* v, const uint8_t* start, f
                          const float* boot, float* out, int64_t B, int64_t L, void* workspace, cudaStream_t s);
 }  // namespace ret
 
+namespace lnorm {
+// the Linear Transformer with phi and normalizer, by the padded-operand
+// construction over the d = 128 linear-attention kernels
+struct Args {
+    bool backward;
+    const void *q, *k, *v;  // bf16 [B, L, H, d]
+    const float* gamma;     // [H] or [B, L, H]
+    int gamma_per_step;
+    const uint8_t* start;
+    const float *S0, *z0;        // [B, H, d, d], [B, H, d] or null
+    float* y;                    // fwd output / bwd input: [B, L, H, d]
+    float* den;                  // fwd output (or null) / bwd input: [B, L, H]
+    float *S_last, *z_last;      // fwd outputs or null
+    const float* grad_y;         // bwd
+    const float *dS_last, *dz_last;
+    float *dq, *dk, *dv, *dgamma, *dS0, *dz0;
+    int64_t B, L, H, d;
+    void* workspace;
+};
+size_t workspace_bytes(int64_t B, int64_t L, int64_t H);
+int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_dgamma_per_head, int with_states);
+memoroid_status_t launch(const Args& a, cudaStream_t s);
+}  // namespace lnorm
+
 namespace tbb {
 size_t workspace_bytes(int64_t K);
 memoroid_status_t launch_sample(const int64_t* begin, int64_t E, int64_t N, const int64_t* ep, int64_t K, int64_t B,

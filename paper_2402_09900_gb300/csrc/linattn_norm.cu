@@ -1,0 +1,309 @@
+// linattn_norm.cu -- the paper's Linear Transformer memoroid with its feature
+// map and normalizer (Appendix "Linear Transformer"): the pair state
+//   (X, x) . (X', x') = (X + X', x + x'),  f(o) = (phi(k) v^T, phi(k)),
+//   y = X^T phi(q) / (x^T phi(q)),  phi(z) = 1 + ELU(z),
+// decayed by gamma_t and reset at begin flags like the decayed memoroid of
+// linattn.cu (gamma = 1 is the paper's model).
+//
+// Both halves of the state are one decayed outer-product state: with
+//   q' = [phi(q), 0],  k' = [phi(k), 0],  v' = [v, 1, 1, 0]   (width 128)
+// the state S' = sum decay k' v'^T holds X in its first d columns and x in
+// columns d and d + 1, and y' = S'^T q' holds the numerator X^T phi(q) and
+// the normalizer x^T phi(q).  So the tensor-core kernels of linattn.cu at
+// d = 128 compute both, and this file adds the element-wise steps around
+// them: building q', k', v' (and the padded states), the division, and in
+// the backward the upstream gradient of the pair,
+//   dy' = [g, hi, lo, 0],  g = bf16(dy / den),  hi + lo = -(g . y),
+// then the chain rule through phi, dq = dq'[:d] (.) phi'(q).  The gradient
+// with respect to q is a difference of two large terms, X g and x (g . y),
+// that cancel exactly at an episode's first step; so the normalizer term is
+// formed from the bf16 values the tensor cores will use and carried as a
+// pair of bf16 numbers (the second ones column of v'), which keeps the
+// difference exact for the rounded upstream g.  Heads of width d <= 120 (a
+// multiple of 8) are supported.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "internal.cuh"
+
+namespace memoroid {
+namespace lnorm {
+
+namespace {
+
+constexpr int kW = 128;  // width of the padded operands and states
+constexpr int kCtas = 152 * 8;
+
+__device__ __forceinline__ float phi(float z) { return z > 0.f ? 1.f + z : expf(z); }
+__device__ __forceinline__ float dphi(float z) { return z > 0.f ? 1.f : expf(z); }
+
+struct Buffers {
+    __nv_bfloat16 *q, *k, *v;  // [R, 128]
+    float* y;                   // fwd: y' [R, 128]; bwd: dy' [R, 128]
+    float *dq, *dk, *dv;        // bwd: [R, 128]
+    float *S0, *S1, *S2;        // [B*H, 128, 128]: incoming state, outgoing state (or its gradient), dS0
+    void* la;                   // the linear-attention workspace (at offset 0, so its header is ours)
+    size_t la_bytes;
+};
+
+size_t la_bytes(int64_t B, int64_t L, int64_t H) { return align_up(la::workspace_bytes(B, L, H, kW), 256); }
+
+Buffers carve(void* ws, int64_t B, int64_t L, int64_t H, bool backward) {
+    unsigned char* p = static_cast<unsigned char*>(ws);
+    const size_t R = static_cast<size_t>(B * L * H);
+    Buffers b{};
+    b.la = p;
+    b.la_bytes = la_bytes(B, L, H);
+    size_t o = b.la_bytes;
+    auto take = [&](size_t bytes) {
+        void* r = p + o;
+        o = align_up(o + bytes, 256);
+        return r;
+    };
+    b.q = static_cast<__nv_bfloat16*>(take(R * kW * 2));
+    b.k = static_cast<__nv_bfloat16*>(take(R * kW * 2));
+    b.v = static_cast<__nv_bfloat16*>(take(R * kW * 2));
+    b.y = static_cast<float*>(take(R * kW * 4));
+    if (backward) {
+        b.dq = static_cast<float*>(take(R * kW * 4));
+        b.dk = static_cast<float*>(take(R * kW * 4));
+        b.dv = static_cast<float*>(take(R * kW * 4));
+    }
+    b.S0 = static_cast<float*>(take(static_cast<size_t>(B * H) * kW * kW * 4));
+    b.S1 = static_cast<float*>(take(static_cast<size_t>(B * H) * kW * kW * 4));
+    if (backward) b.S2 = static_cast<float*>(take(static_cast<size_t>(B * H) * kW * kW * 4));
+    return b;
+}
+
+size_t total_bytes(int64_t B, int64_t L, int64_t H) {
+    const size_t R = static_cast<size_t>(B * L * H);
+    size_t o = la_bytes(B, L, H);
+    const size_t st = static_cast<size_t>(B * H) * kW * kW * 4;
+    for (size_t bytes : {R * kW * 2, R * kW * 2, R * kW * 2, R * kW * 4, R * kW * 4, R * kW * 4, R * kW * 4, st, st, st})
+        o = align_up(o + bytes, 256);
+    return o;
+}
+
+// q' = [phi(q), 0], k' = [phi(k), 0], v' = [v, 1, 0]: one thread per 16-byte
+// chunk (8 columns) of one padded row of one of the three operands.
+__global__ void __launch_bounds__(256) prep_kernel(const uint4* __restrict__ q, const uint4* __restrict__ k,
+                                                   const uint4* __restrict__ v, int64_t R, int d,
+                                                   uint4* __restrict__ qp, uint4* __restrict__ kp,
+                                                   uint4* __restrict__ vp) {
+    const int in_chunks = d / 8;
+    const int64_t n = R * 3 * (kW / 8);
+    for (int64_t g = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; g < n;
+         g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int c = static_cast<int>(g % (kW / 8));
+        const int which = static_cast<int>((g / (kW / 8)) % 3);
+        const int64_t r = g / (3 * (kW / 8));
+        uint4 out = make_uint4(0u, 0u, 0u, 0u);
+        if (c < in_chunks) {
+            const uint4* src = which == 0 ? q : (which == 1 ? k : v);
+            out = src[r * in_chunks + c];
+            if (which < 2) {
+                __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&out);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float2 f = __bfloat1622float2(h[e]);
+                    h[e] = __floats2bfloat162_rn(phi(f.x), phi(f.y));
+                }
+            }
+        } else if (which == 2 && c == in_chunks) {
+            __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&out);
+            h[0] = __floats2bfloat162_rn(1.f, 1.f);  // columns d and d + 1 of v' are 1
+        }
+        uint4* dst = which == 0 ? qp : (which == 1 ? kp : vp);
+        dst[r * (kW / 8) + c] = out;
+    }
+}
+
+// padded state from (S [d, d], z [d]) per (tape, head): S' = [[S, z, z2], [0]]
+// with z2 = z (a state) or 0 (the gradient of an outgoing state, read from
+// column d only); null inputs give zeros
+__global__ void __launch_bounds__(256) pad_state_kernel(const float* __restrict__ S, const float* __restrict__ z,
+                                                        int64_t BH, int d, int dup, float* __restrict__ Sp) {
+    const int64_t n = BH * kW * kW;
+    for (int64_t g = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; g < n;
+         g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int j = static_cast<int>(g % kW), i = static_cast<int>((g / kW) % kW);
+        const int64_t m = g / (kW * kW);
+        float val = 0.f;
+        if (i < d && j < d && S != nullptr) val = S[(m * d + i) * d + j];
+        else if (i < d && (j == d || (dup && j == d + 1)) && z != nullptr) val = z[m * d + i];
+        Sp[g] = val;
+    }
+}
+
+// (S, z) from a padded state: z = column d (a state), or columns d + d + 1
+// (the gradient of an incoming state, whose z feeds both columns)
+__global__ void __launch_bounds__(256) unpad_state_kernel(const float* __restrict__ Sp, int64_t BH, int d, int both,
+                                                          float* __restrict__ S, float* __restrict__ z) {
+    const int64_t n = BH * d * (d + 1);
+    for (int64_t g = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; g < n;
+         g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int j = static_cast<int>(g % (d + 1)), i = static_cast<int>((g / (d + 1)) % d);
+        const int64_t m = g / (static_cast<int64_t>(d) * (d + 1));
+        const float* row = Sp + (m * kW + i) * kW;
+        if (j < d) {
+            if (S != nullptr) S[(m * d + i) * d + j] = row[j];
+        } else if (z != nullptr) {
+            z[m * d + i] = both ? row[d] + row[d + 1] : row[d];
+        }
+    }
+}
+
+// y = y'[:d] / y'[d], den = y'[d]: one warp per row (lane l holds columns 4l..4l+3)
+__global__ void __launch_bounds__(256) divide_kernel(const float4* __restrict__ yp, int64_t R, int d,
+                                                     float* __restrict__ y, float* __restrict__ den) {
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+    for (int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; r < R; r += nw) {
+        const float4 a = yp[r * (kW / 4) + lane];
+        const float comp[4] = {a.x, a.y, a.z, a.w};
+        const float dn = __shfl_sync(0xffffffffu, comp[d & 3], d >> 2);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int j = 4 * lane + e;
+            if (j < d) y[r * d + j] = comp[e] / dn;
+        }
+        if (lane == 0 && den != nullptr) den[r] = dn;
+    }
+}
+
+__device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+
+// dy' = [g, hi, lo, 0] with g = bf16(dy / den) and hi + lo = -(g . y) (both
+// bf16): one warp per row, lane l holding columns 4l .. 4l + 3
+__global__ void __launch_bounds__(256) upstream_kernel(const float* __restrict__ dy, const float* __restrict__ y,
+                                                       const float* __restrict__ den, int64_t R, int d,
+                                                       float4* __restrict__ dyp) {
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+    for (int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; r < R; r += nw) {
+        float g[4], dot = 0.f;
+        const float inv = 1.f / den[r];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int j = 4 * lane + e;
+            g[e] = 0.f;
+            if (j < d) {
+                g[e] = bf16_round(dy[r * d + j] * inv);
+                dot = fmaf(g[e], y[r * d + j], dot);
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+        const float hi = bf16_round(-dot), lo = bf16_round(-dot - hi);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int j = 4 * lane + e;
+            if (j == d) g[e] = hi;
+            if (j == d + 1) g[e] = lo;
+        }
+        dyp[r * (kW / 4) + lane] = make_float4(g[0], g[1], g[2], g[3]);
+    }
+}
+
+// dq = dq'[:d] (.) phi'(q), dk = dk'[:d] (.) phi'(k), dv = dv'[:d]: one thread per column
+__global__ void __launch_bounds__(256) chain_kernel(const float* __restrict__ dqp, const float* __restrict__ dkp,
+                                                    const float* __restrict__ dvp, const __nv_bfloat16* __restrict__ q,
+                                                    const __nv_bfloat16* __restrict__ k, int64_t R, int d,
+                                                    float* __restrict__ dq, float* __restrict__ dk,
+                                                    float* __restrict__ dv) {
+    const int64_t n = R * d;
+    for (int64_t g = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; g < n;
+         g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t r = g / d;
+        const int j = static_cast<int>(g - r * d);
+        const int64_t p = r * kW + j;
+        dq[g] = dqp[p] * dphi(__bfloat162float(q[g]));
+        dk[g] = dkp[p] * dphi(__bfloat162float(k[g]));
+        dv[g] = dvp[p];
+    }
+}
+
+unsigned grid_for(int64_t n, int per_thread = 1) {
+    const int64_t want = (n / per_thread + 255) / 256;
+    return static_cast<unsigned>(want < 1 ? 1 : (want > kCtas ? kCtas : want));
+}
+
+}  // namespace
+
+size_t workspace_bytes(int64_t B, int64_t L, int64_t H) { return total_bytes(B, L, H); }
+
+int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_dgamma_per_head, int with_states) {
+    if (B == 0 || L == 0 || H == 0) return 0;
+    // prep, the linear-attention call, then the divide (forward) or the upstream
+    // gradient and the chain rule (backward); with states: their padding and unpadding
+    const int base = 2 + (backward ? 1 : 0) + la::kernels_per_call(B, L, H, backward, with_dgamma_per_head);
+    return base + (with_states ? (backward ? 3 : 2) : 0);
+}
+
+memoroid_status_t launch(const Args& a, cudaStream_t s) {
+    const int64_t R = a.B * a.L * a.H, BH = a.B * a.H;
+    const Buffers b = carve(a.workspace, a.B, a.L, a.H, a.backward);
+    prep_kernel<<<grid_for(R * 48), 256, 0, s>>>(static_cast<const uint4*>(a.q), static_cast<const uint4*>(a.k),
+                                                 static_cast<const uint4*>(a.v), R, static_cast<int>(a.d),
+                                                 reinterpret_cast<uint4*>(b.q), reinterpret_cast<uint4*>(b.k),
+                                                 reinterpret_cast<uint4*>(b.v));
+    // incoming state and (backward) outgoing-state gradient in the padded layout
+    const bool s_in = a.S0 != nullptr || a.z0 != nullptr;
+    const bool g_in = a.backward && (a.dS_last != nullptr || a.dz_last != nullptr);
+    if (s_in)
+        pad_state_kernel<<<grid_for(BH * kW * kW), 256, 0, s>>>(a.S0, a.z0, BH, static_cast<int>(a.d), 1, b.S0);
+    if (g_in)
+        pad_state_kernel<<<grid_for(BH * kW * kW), 256, 0, s>>>(a.dS_last, a.dz_last, BH, static_cast<int>(a.d), 0,
+                                                                b.S1);
+    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    la::Args l{};
+    l.q = b.q;
+    l.k = b.k;
+    l.v = b.v;
+    l.gamma = a.gamma;
+    l.gamma_per_step = a.gamma_per_step;
+    l.start = a.start;
+    l.S0 = s_in ? b.S0 : nullptr;
+    l.B = a.B;
+    l.L = a.L;
+    l.H = a.H;
+    l.D = kW;
+    l.workspace = b.la;
+    l.workspace_bytes = b.la_bytes;
+    if (!a.backward) {
+        l.y = b.y;
+        l.S_last = (a.S_last != nullptr || a.z_last != nullptr) ? b.S1 : nullptr;
+        const memoroid_status_t st = la::launch_fwd(l, s);
+        if (st != MEMOROID_OK) return st;
+        divide_kernel<<<grid_for(R * 32), 256, 0, s>>>(reinterpret_cast<const float4*>(b.y), R, static_cast<int>(a.d),
+                                                       a.y, a.den);
+        if (l.S_last != nullptr)
+            unpad_state_kernel<<<grid_for(BH * a.d * (a.d + 1)), 256, 0, s>>>(b.S1, BH, static_cast<int>(a.d), 0,
+                                                                               a.S_last, a.z_last);
+        return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
+    }
+    upstream_kernel<<<grid_for(R * 32), 256, 0, s>>>(a.grad_y, a.y, a.den, R, static_cast<int>(a.d),
+                                                     reinterpret_cast<float4*>(b.y));
+    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    l.grad_y = b.y;
+    l.dS_last = g_in ? b.S1 : nullptr;
+    l.dq = b.dq;
+    l.dk = b.dk;
+    l.dv = b.dv;
+    l.dgamma = a.dgamma;
+    l.dS0 = (a.dS0 != nullptr || a.dz0 != nullptr) ? b.S2 : nullptr;
+    const memoroid_status_t st = la::launch_bwd(l, s);
+    if (st != MEMOROID_OK) return st;
+    chain_kernel<<<grid_for(R * a.d), 256, 0, s>>>(b.dq, b.dk, b.dv, static_cast<const __nv_bfloat16*>(a.q),
+                                                   static_cast<const __nv_bfloat16*>(a.k), R, static_cast<int>(a.d),
+                                                   a.dq, a.dk, a.dv);
+    if (l.dS0 != nullptr)
+        unpad_state_kernel<<<grid_for(BH * a.d * (a.d + 1)), 256, 0, s>>>(b.S2, BH, static_cast<int>(a.d), 1, a.dS0,
+                                                                           a.dz0);
+    return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
+}
+
+}  // namespace lnorm
+}  // namespace memoroid

@@ -56,6 +56,12 @@ SIGNATURES = {
     "memoroid_bench_linattn_intra_scratch_bytes": (_sz, [_i64]),
     "memoroid_bench_linattn_intra": (_int, [_i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_returns_workspace_bytes": (_sz, [_i64, _i64]),
+    "memoroid_linattn_norm_workspace_bytes": (_sz, [_i64, _i64, _i64, _i64]),
+    "memoroid_linattn_norm_kernels_per_call": (_int, [_i64, _i64, _i64, _i64, _int, _int, _int]),
+    "memoroid_linattn_norm_fwd": (_int, [_p, _p, _p, _p, _int, _p, _p, _p, _p, _p, _p, _p,
+                                         _i64, _i64, _i64, _i64, _p, _sz, _p]),
+    "memoroid_linattn_norm_bwd": (_int, [_p, _p, _p, _p, _int, _p, _p, _p, _p, _p, _p, _p, _p,
+                                         _p, _p, _p, _p, _p, _p, _i64, _i64, _i64, _i64, _p, _sz, _p]),
     "memoroid_tbb_workspace_bytes": (_sz, [_i64]),
     "memoroid_tbb_sample": (_int, [_p, _i64, _i64, _p, _i64, _i64, _p, _p, _p, _p, _sz, _p]),
     "memoroid_gather_rows": (_int, [_p, _i64, _i64, _p, _i64, _p, _p, _sz, _p]),
@@ -231,6 +237,37 @@ def memoroid_gae(r, v, start, gamma, lam, v_boot, A, B, L, workspace, stream=Non
            "memoroid_gae")
 
 
+def memoroid_linattn_norm_workspace_bytes(B, L, H, d) -> int:
+    return int(load().memoroid_linattn_norm_workspace_bytes(B, L, H, d))
+
+
+def memoroid_linattn_norm_kernels_per_call(B, L, H, d, backward, with_dgamma_per_head, with_states) -> int:
+    return int(load().memoroid_linattn_norm_kernels_per_call(B, L, H, d, int(backward), int(with_dgamma_per_head),
+                                                             int(with_states)))
+
+
+def memoroid_linattn_norm_fwd(q, k, v, gamma, gamma_per_step, start, S0, z0, y, den, S_last, z_last, B, L, H, d,
+                              workspace, stream=None):
+    _need_cuda(q, k, v, gamma, start, S0, z0, y, den, S_last, z_last, workspace)
+    _check(load().memoroid_linattn_norm_fwd(_ptr(q), _ptr(k), _ptr(v), _ptr(gamma), int(gamma_per_step), _ptr(start),
+                                            _ptr(S0), _ptr(z0), _ptr(y), _ptr(den), _ptr(S_last), _ptr(z_last),
+                                            B, L, H, d, _ptr(workspace),
+                                            workspace.numel() if workspace is not None else 0, _stream(stream)),
+           "memoroid_linattn_norm_fwd")
+
+
+def memoroid_linattn_norm_bwd(q, k, v, gamma, gamma_per_step, start, S0, z0, y, den, grad_y, grad_S_last, grad_z_last,
+                              dq, dk, dv, dgamma, dS0, dz0, B, L, H, d, workspace, stream=None):
+    _need_cuda(q, k, v, gamma, start, S0, z0, y, den, grad_y, grad_S_last, grad_z_last, dq, dk, dv, dgamma, dS0, dz0,
+               workspace)
+    _check(load().memoroid_linattn_norm_bwd(_ptr(q), _ptr(k), _ptr(v), _ptr(gamma), int(gamma_per_step), _ptr(start),
+                                            _ptr(S0), _ptr(z0), _ptr(y), _ptr(den), _ptr(grad_y), _ptr(grad_S_last),
+                                            _ptr(grad_z_last), _ptr(dq), _ptr(dk), _ptr(dv), _ptr(dgamma), _ptr(dS0),
+                                            _ptr(dz0), B, L, H, d, _ptr(workspace),
+                                            workspace.numel() if workspace is not None else 0, _stream(stream)),
+           "memoroid_linattn_norm_bwd")
+
+
 def memoroid_tbb_workspace_bytes(K) -> int:
     return int(load().memoroid_tbb_workspace_bytes(K))
 
@@ -398,6 +435,38 @@ def gae(r, v, start, gamma, lam, v_boot=None, ws=None, stream=None):
     A = torch.empty_like(r)
     memoroid_gae(r, v, start, gamma, lam, v_boot, A, B, L, ws, stream)
     return A
+
+
+def linattn_norm_fwd(q, k, v, gamma, start, S0=None, z0=None, want_last=True, ws=None, stream=None):
+    """Linear Transformer with phi = 1 + ELU and its normalizer: q, k, v as
+    int16 views of bf16 [B, L, H, d]; returns y, den, S_last, z_last."""
+    B, L, H, d = q.shape
+    per = 1 if gamma.dim() == 3 else 0
+    if ws is None:
+        ws = workspace(memoroid_linattn_norm_workspace_bytes(B, L, H, d), q.device)
+    y = torch.empty((B, L, H, d), dtype=torch.float32, device=q.device)
+    den = torch.empty((B, L, H), dtype=torch.float32, device=q.device)
+    S_last = torch.empty((B, H, d, d), dtype=torch.float32, device=q.device) if want_last else None
+    z_last = torch.empty((B, H, d), dtype=torch.float32, device=q.device) if want_last else None
+    memoroid_linattn_norm_fwd(q, k, v, gamma, per, start, S0, z0, y, den, S_last, z_last, B, L, H, d, ws, stream)
+    return y, den, S_last, z_last
+
+
+def linattn_norm_bwd(q, k, v, gamma, start, y, den, grad_y, grad_S_last=None, grad_z_last=None, S0=None, z0=None,
+                     want_gamma=True, want_S0=False, ws=None, stream=None):
+    """Backward of linattn_norm_fwd: dq, dk, dv, dgamma, dS0, dz0."""
+    B, L, H, d = q.shape
+    per = 1 if gamma.dim() == 3 else 0
+    if ws is None:
+        ws = workspace(memoroid_linattn_norm_workspace_bytes(B, L, H, d), q.device)
+    dq = torch.empty((B, L, H, d), dtype=torch.float32, device=q.device)
+    dk, dv = torch.empty_like(dq), torch.empty_like(dq)
+    dgamma = torch.empty_like(gamma) if want_gamma else None
+    dS0 = torch.empty((B, H, d, d), dtype=torch.float32, device=q.device) if want_S0 else None
+    dz0 = torch.empty((B, H, d), dtype=torch.float32, device=q.device) if want_S0 else None
+    memoroid_linattn_norm_bwd(q, k, v, gamma, per, start, S0, z0, y, den, grad_y, grad_S_last, grad_z_last, dq, dk,
+                              dv, dgamma, dS0, dz0, B, L, H, d, ws, stream)
+    return dq, dk, dv, dgamma, dS0, dz0
 
 
 def tbb_sample(begin, N, draws, B, ws=None, stream=None):

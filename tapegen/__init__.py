@@ -213,12 +213,13 @@ def ffm_tape(B: int, L: int, m: int, c: int, seed: int, mean: float = 500.0, hi:
 
 def linattn_tape(B: int, L: int, H: int, dk: int, dv: int, seed: int, mean: float = 300.0,
                  gamma_mode: str = "head", gammas=(0.9, 0.99, 0.999, 1.0), scale: float | None = None,
-                 with_grad: bool = True, with_S0: bool = False, start_mode: str = "geometric"):
+                 with_grad: bool = True, with_S0: bool = False, start_mode: str = "geometric",
+                 normalize_k: bool = True):
     """A linear-attention workload: bf16 q, k, v (as uint16 bits), fp32 gamma,
     start flags and optional upstream gradients.
 
-    q, v ~ N(0, 1) * scale; k ~ N(0, 1) L2-normalised over d_k in fp32 before
-    the bf16 cast.  gamma_mode "head": one decay per head (cycled from
+    q, v ~ N(0, 1) * scale; k ~ N(0, 1), L2-normalised over d_k in fp32 before
+    the bf16 cast unless normalize_k is False.  gamma_mode "head": one decay per head (cycled from
     `gammas`); "step": gamma[b, t, h] = sigmoid(N(3, 1)).
     """
     rng = np.random.default_rng(seed)
@@ -226,7 +227,8 @@ def linattn_tape(B: int, L: int, H: int, dk: int, dv: int, seed: int, mean: floa
         scale = 1.0 / np.sqrt(dk)
     q = rng.standard_normal((B, L, H, dk), dtype=np.float32) * np.float32(scale)
     k = rng.standard_normal((B, L, H, dk), dtype=np.float32)
-    k /= np.maximum(np.linalg.norm(k, axis=-1, keepdims=True), np.float32(1e-12))
+    if normalize_k:
+        k /= np.maximum(np.linalg.norm(k, axis=-1, keepdims=True), np.float32(1e-12))
     v = rng.standard_normal((B, L, H, dv), dtype=np.float32) * np.float32(scale)
     if gamma_mode == "head":
         gamma = np.array([gammas[h % len(gammas)] for h in range(H)], dtype=np.float32)

@@ -1,0 +1,153 @@
+"""GPU parity of the Linear Transformer memoroid with phi = 1 + ELU and its
+normalizer (the padded-operand construction over the tensor-core linear
+attention kernels) against the fp64 oracle, through the C ABI.
+
+Bar: max |gpu - ref| / max |ref| <= 2e-2 per output (bf16 q, k, v; phi(q),
+phi(k) and the upstream gradient pass through bf16 on the tensor cores).
+"""
+import numpy as np
+import pytest
+
+import oracle
+import tapegen
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+TOL = 2e-2
+
+
+def _m():
+    from paper_2402_09900_gb300 import memoroid as m
+    m.load()
+    return m
+
+
+def rel_err(got, ref):
+    g = np.asarray(got, dtype=np.float64)
+    r = np.asarray(ref, dtype=np.float64)
+    return float(np.max(np.abs(g - r))) / max(float(np.max(np.abs(r))), 1e-30)
+
+
+def bits(a):
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda()
+
+
+def dev(a):
+    return None if a is None else torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def make(B, L, H, d, seed, mean, mode, with_states, start_mode="geometric", normalize_k=False):
+    # the paper's model feeds phi(W_k o): keys are not normalised (q, k, v ~ N(0, 1))
+    t = tapegen.linattn_tape(B, L, H, d, d, seed, mean=mean, gamma_mode=mode, scale=1.0, with_S0=with_states,
+                             start_mode=start_mode, normalize_k=normalize_k)
+    rng = np.random.default_rng(seed + 1)
+    if with_states:
+        t["z0"] = rng.uniform(0.5, 2.0, (B, H, d)).astype(np.float32)  # a sum of positive features
+        t["grad_z_last"] = rng.standard_normal((B, H, d)).astype(np.float32)
+        t["start"][:, 0] = 0  # rows continue from (S0, z0)
+    return t
+
+
+def run(t, with_states):
+    m = _m()
+    B, L, H, d = t["B"], t["L"], t["H"], t["dk"]
+    ws = m.workspace(m.memoroid_linattn_norm_workspace_bytes(B, L, H, d), "cuda")
+    q, k, v = bits(t["q"]), bits(t["k"]), bits(t["v"])
+    g, st = dev(t["gamma"]), dev(t["start"])
+    S0 = dev(t.get("S0")) if with_states else None
+    z0 = dev(t.get("z0")) if with_states else None
+    y, den, Sl, zl = m.linattn_norm_fwd(q, k, v, g, st, S0, z0, ws=ws)
+    assert m.memoroid_get_device_error(ws) == m.MEMOROID_OK
+    gS = dev(t["grad_S_last"]) if with_states else None
+    gz = dev(t["grad_z_last"]) if with_states else None
+    dq, dk, dv, dg, dS0, dz0 = m.linattn_norm_bwd(q, k, v, g, st, y, den, dev(t["grad_y"]), gS, gz, S0, z0,
+                                                  want_S0=with_states, ws=ws)
+    assert m.memoroid_get_device_error(ws) == m.MEMOROID_OK
+    torch.cuda.synchronize()
+    out = dict(y=y, den=den, S_last=Sl, z_last=zl, dq=dq, dk=dk, dv=dv, dgamma=dg, dS0=dS0, dz0=dz0)
+    return {kk: (None if vv is None else vv.cpu().numpy()) for kk, vv in out.items()}
+
+
+def ref(t, with_states):
+    f = oracle.bf16_bits_to_f64
+    q, k, v = f(t["q"]), f(t["k"]), f(t["v"])
+    S0 = t.get("S0") if with_states else None
+    z0 = t.get("z0") if with_states else None
+    y, den, Sl, zl = oracle.linattn_norm_fwd(q, k, v, t["gamma"], t["start"], S0, z0)
+    gS = t["grad_S_last"] if with_states else None
+    gz = t["grad_z_last"] if with_states else None
+    dq, dk, dv, dg, dS0, dz0 = oracle.linattn_norm_bwd(q, k, v, t["gamma"], t["start"], t["grad_y"], gS, gz, S0, z0)
+    out = dict(y=y, den=den, S_last=Sl, z_last=zl, dq=dq, dk=dk, dv=dv, dgamma=dg)
+    if with_states:
+        out.update(dS0=dS0, dz0=dz0)
+    return out
+
+
+def check(t, with_states):
+    got, want = run(t, with_states), ref(t, with_states)
+    errs = {kk: rel_err(got[kk], want[kk]) for kk in want}
+    bad = {kk: e for kk, e in errs.items() if not e <= TOL}
+    assert not bad, (bad, errs)
+
+
+@pytest.mark.parametrize("B,L,H,d,mean,mode,with_states", [
+    (1, 3000, 2, 64, 300.0, "head", False),
+    (2, 1500, 3, 32, 100.0, "step", True),
+    (1, 2000, 1, 16, 500.0, "step", False),
+    (1, 700, 2, 120, 80.0, "head", True),
+    (3, 900, 1, 8, 40.0, "head", False),
+])
+def test_parity(B, L, H, d, mean, mode, with_states):
+    check(make(B, L, H, d, tapegen.seed_for(800 + L + d), mean, mode, with_states), with_states)
+
+
+def test_paper_model_gamma_one():
+    # gamma = 1: the paper's undecayed Linear Transformer
+    t = make(1, 2500, 2, 64, tapegen.seed_for(810), 400.0, "head", False)
+    t["gamma"][:] = 1.0
+    check(t, False)
+
+
+def test_all_start_gives_v():
+    # one term per step: the weight cancels and y = v
+    t = make(1, 1000, 2, 32, tapegen.seed_for(811), 1.0, "step", False, start_mode="all")
+    got = run(t, False)
+    assert rel_err(got["y"], oracle.bf16_bits_to_f64(t["v"])) <= 1e-5
+
+
+def test_episode_isolation_bitwise():
+    m = _m()
+    t = make(1, 6000, 2, 64, tapegen.seed_for(812), 300.0, "step", False)
+    heads = np.flatnonzero(t["start"][0])
+    s, e = int(heads[6]), int(heads[7])
+    base = run(t, False)
+    t2 = dict(t)
+    v = oracle.bf16_bits_to_f64(t["v"]).astype(np.float32)
+    v[0, s:e] += 0.5
+    t2["v"] = tapegen.f32_to_bf16_bits(v)
+    pert = run(t2, False)
+    # tiles shared with the changed episode are recomputed, but rows outside it come out identical
+    outside = np.ones(t["L"], dtype=bool)
+    outside[s:e] = False
+    assert np.array_equal(base["y"][0, outside], pert["y"][0, outside])
+    assert not np.array_equal(base["y"][0, s:e], pert["y"][0, s:e])
+    del m
+
+
+def test_config3_shape_sampled_episodes():
+    # the config-3 shape (L = 2^18, 4 heads, d = 64): outputs and gradients on whole-episode
+    # windows (each starts at a begin flag and ends right before one)
+    t = make(1, 1 << 18, 4, 64, tapegen.seed_for(813), 300.0, "step", False)
+    got = run(t, False)
+    heads = np.flatnonzero(t["start"][0])
+    f = oracle.bf16_bits_to_f64
+    for pick in (3, len(heads) // 2, len(heads) - 12):
+        s, e = int(heads[pick]), int(heads[pick + 8])
+        sl = slice(s, e)
+        q, k, v = f(t["q"][:, sl]), f(t["k"][:, sl]), f(t["v"][:, sl])
+        y, den, _, _ = oracle.linattn_norm_fwd(q, k, v, t["gamma"][:, sl], t["start"][:, sl])
+        dq, dk, dv, dg, _, _ = oracle.linattn_norm_bwd(q, k, v, t["gamma"][:, sl], t["start"][:, sl],
+                                                       t["grad_y"][:, sl])
+        for name, r in (("y", y), ("den", den), ("dq", dq), ("dk", dk), ("dv", dv), ("dgamma", dg)):
+            assert rel_err(got[name][:, sl], r) <= TOL, name
