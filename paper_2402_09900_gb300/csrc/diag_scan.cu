@@ -231,7 +231,9 @@ struct Cfg {
     static constexpr int UNROLL = REV_ ? MEMOROID_UNROLL_BWD : MEMOROID_UNROLL_FWD;
     // arrays staged per tile: input [, h (backward)] [, lambda (per step)]
     static constexpr int NB = 1 + (REV_ ? 1 : 0) + (PS_ ? 1 : 0);
-    static constexpr int BUF_F4 = T * 32;  // float4 per staged array
+    // float4 per staged array: a 512-byte row per step, or for the FFM forward
+    // the row's x~ (at most 64 floats, c = 1)
+    static constexpr int BUF_F4 = (FFM_ && !REV_) ? T * 16 : T * 32;
     static constexpr int THREADS = (W_ + 2) * 32;  // W scan warps + 2 look-back warps
     static constexpr int NSYNC = (W_ + 1) * 32;    // scan warps + one look-back warp
     // shared memory layout (bytes)
