@@ -65,6 +65,25 @@ def _dist_env():
     return ws, rank, local
 
 
+def max_over_ranks(value, ws, device):
+    """The largest `value` over the ranks of the job (its time is its slowest
+    rank's); `value` itself for a single rank."""
+    if ws <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(ws, units_per_rank, ms_per_step):
+    """Whole-job throughput: the units every rank processed in one step,
+    divided by the step time (weak scaling: each rank has its own tape)."""
+    return ws * units_per_rank / (ms_per_step / 1e3)
+
+
 def _peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -663,15 +682,11 @@ def run_ours(args):
         dist.barrier()
     if m.memoroid_get_device_error(work) != m.MEMOROID_OK:
         raise RuntimeError("device-side error during the timed region")
-    elapsed_ms = t_begin.elapsed_time(t_end)
+    elapsed_ms = max_over_ranks(t_begin.elapsed_time(t_end), ws, dev)
     fwd_ms = [e[0].elapsed_time(e[1]) for e in evs]
     bwd_ms = [e[1].elapsed_time(e[2]) for e in evs]
-    if ws > 1:
-        tt = torch.tensor([elapsed_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(tt.item())
     ms_per_step = elapsed_ms / args.steps
-    value = ws * B * L / (ms_per_step / 1e3)
+    value = job_throughput(ws, B * L, ms_per_step)
 
     # ---- end to end through the C ABI with pinned host buffers ----
     e2e = None
@@ -731,12 +746,8 @@ def run_ours(args):
         for _ in range(args.e2e_steps):
             e2e_step()
         torch.cuda.synchronize()
-        e_ms = (time.perf_counter() - e0) * 1e3 / args.e2e_steps
-        if ws > 1:
-            tt = torch.tensor([e_ms], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e_ms = float(tt.item())
-        e2e = {"value": ws * B * L / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+        e_ms = max_over_ranks((time.perf_counter() - e0) * 1e3 / args.e2e_steps, ws, dev)
+        e2e = {"value": job_throughput(ws, B * L, e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "steps": args.e2e_steps, "ms_per_step": e_ms}
 
     if rank != 0:
