@@ -61,7 +61,8 @@
 //     timer; on expiry the kernel records an error in the workspace and
 //     returns.
 // grad_lambda (per-channel lambda) is accumulated per tile and reduced in a
-// fixed order by two small kernels, so it is deterministic as well.
+// fixed order by two small kernels (fp32 within a part of a few dozen tiles,
+// fp64 across parts), so it is deterministic as well.
 #include <cuda_runtime.h>
 
 #include "internal.cuh"
@@ -111,10 +112,11 @@ struct Params {
     float4* grad_h0;       // bwd: [B, D/2] or null
     int64_t B, L, D2, n_slabs, n_tt, n_chains, n_tiles;
     int64_t n_seg, q_seg, n_sc;  // segments per chain, tiles per segment, segment chains
-    uint32_t* hdr;               // workspace header: [0] error, [1] ticket counter
+    uint32_t* hdr;               // workspace header: [0] error, [1] ticket counter, [4] fix-up list length
     unsigned long long* node;    // [n_sc * q_seg * 32 * NODE_WORDS] tagged Fenwick nodes
     float4* gpart;               // [n_chains * n_tt * 32]      per-tile grad_lambda
-    uint32_t* fix;               // [n_chains * n_tt] tile needs its segment's carry added (n_seg > 1)
+    uint32_t* fix;               // [n_chains * n_tt] tiles that need their segment's carry added (n_seg > 1),
+                                 // a list of hdr[4] tile indices in completion order
     float4* pin;                 // [n_chains * n_tt * 32] product of multipliers from the segment start
     float4* segc;                // [n_chains * n_seg * 32] true state entering each segment
     float4* sega;                // [n_chains * n_seg * 32 * 2] each segment's aggregate (a, x)
@@ -592,8 +594,10 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
             // steps of this tile before its first begin flag miss the state entering the segment
             const int64_t tid = t.chain * p.n_tt + t.jt;
             const bool partial = (t.g > 0) && need_carry && !Rb;
-            if (partial) p.pin[tid * 32 + lane] = Ra;
-            if (lane == 0) p.fix[tid] = partial ? 1u : 0u;
+            if (partial) {
+                p.pin[tid * 32 + lane] = Ra;
+                if (lane == 0) p.fix[atomicAdd(p.hdr + 4, 1u)] = static_cast<uint32_t>(tid);
+            }
         }
         s_carry[lane] = carry;
         if (!ok && lane == 0) *s_abort = 1;
@@ -790,34 +794,77 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
 // ============================================================================
 // segment fix-up
 // ============================================================================
-// State entering each segment (one warp per chain): the segments' aggregates,
-// published by their last tiles, folded left to right from the chain's
-// initial state.
-__global__ void __launch_bounds__(256) segment_carry_kernel(const Params p, bool rev) {
-    const int lane = threadIdx.x & 31;
-    const int64_t chain = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
-    if (chain >= p.n_chains || ptx::ld_relaxed(p.hdr) != 0u) return;
+// State entering each segment, one CTA per chain: each warp folds a range of
+// the segments' aggregates (published by their last tiles) from the identity,
+// the warps' aggregates are folded in order from the chain's initial state,
+// and each warp then walks its range again from its own entering state.  A
+// begin flag inside a fold discards what is left of it, exactly.
+constexpr int CARRY_WARPS = 8;
+constexpr int CARRY_BATCH = 8;
+__global__ void __launch_bounds__(CARRY_WARPS * 32) segment_carry_kernel(const Params p, bool rev) {
+    __shared__ float4 s_a[CARRY_WARPS][32], s_x[CARRY_WARPS][32];
+    __shared__ uint32_t s_b[CARRY_WARPS];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t chain = blockIdx.x;
+    if (ptx::ld_relaxed(p.hdr) != 0u) return;  // uniform over the CTA
     const int64_t G = p.n_seg;
     const int64_t b = chain / p.n_slabs;
     const int64_t c2 = (chain - b * p.n_slabs) * (SLAB / 2);
     const bool lane_ok = lane < lmin(SLAB / 2, p.D2 - c2);
-    const float4* base_src = rev ? p.g_last : p.h0;
-    float4 c = (base_src != nullptr && lane_ok) ? base_src[b * p.D2 + c2 + lane] : zero2();
-    for (int64_t g0 = 0; g0 < G; g0 += 8) {
-        float4 a[8], x[8];
-        uint32_t bb[8];
+    const int64_t per = (G + CARRY_WARPS - 1) / CARRY_WARPS;
+    const int64_t g_lo = lmin(G, warp * per), g_hi = lmin(G, g_lo + per);
+    // this warp's range folded from the identity
+    float4 A = one2(), X = zero2();
+    bool Bf = false;
+    for (int64_t g0 = g_lo; g0 < g_hi; g0 += CARRY_BATCH) {
+        float4 a[CARRY_BATCH], x[CARRY_BATCH];
+        uint32_t bb[CARRY_BATCH];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
+        for (int k = 0; k < CARRY_BATCH; ++k) {
             const int64_t si = chain * G + g0 + k;
-            if (g0 + k < G) {
+            if (g0 + k < g_hi) {
                 a[k] = p.sega[si * 64 + lane];
                 x[k] = p.sega[si * 64 + 32 + lane];
                 bb[k] = p.segb[si];
             }
         }
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            if (g0 + k < G) {
+        for (int k = 0; k < CARRY_BATCH; ++k) {
+            if (g0 + k < g_hi) {
+                if (bb[k]) {
+                    A = a[k];
+                    X = x[k];
+                    Bf = true;
+                } else {
+                    X = cfma2(a[k], X, x[k]);
+                    A = cmul2(a[k], A);
+                }
+            }
+        }
+    }
+    s_a[warp][lane] = A;
+    s_x[warp][lane] = X;
+    if (lane == 0) s_b[warp] = Bf ? 1u : 0u;
+    __syncthreads();
+    // state entering this warp's range: the initial state through the warps before it
+    const float4* base_src = rev ? p.g_last : p.h0;
+    float4 c = (base_src != nullptr && lane_ok) ? base_src[b * p.D2 + c2 + lane] : zero2();
+    for (int w = 0; w < warp; ++w) c = s_b[w] ? s_x[w][lane] : cfma2(s_a[w][lane], c, s_x[w][lane]);
+    for (int64_t g0 = g_lo; g0 < g_hi; g0 += CARRY_BATCH) {
+        float4 a[CARRY_BATCH], x[CARRY_BATCH];
+        uint32_t bb[CARRY_BATCH];
+#pragma unroll
+        for (int k = 0; k < CARRY_BATCH; ++k) {
+            const int64_t si = chain * G + g0 + k;
+            if (g0 + k < g_hi) {
+                a[k] = p.sega[si * 64 + lane];
+                x[k] = p.sega[si * 64 + 32 + lane];
+                bb[k] = p.segb[si];
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < CARRY_BATCH; ++k) {
+            if (g0 + k < g_hi) {
                 p.segc[(chain * G + g0 + k) * 32 + lane] = c;
                 c = bb[k] ? x[k] : cfma2(a[k], c, x[k]);
             }
@@ -826,16 +873,14 @@ __global__ void __launch_bounds__(256) segment_carry_kernel(const Params p, bool
 }
 
 // Adds the state entering its segment to the outputs of a tile that the
-// scan computed from the identity, up to the tile's first begin flag (one warp
-// per tile; tiles that need nothing return at once).  The rows to fix are
+// scan computed from the identity, up to the tile's first begin flag: the
+// warps walk the list of such tiles the scan wrote (each tile touches only
+// its own rows, so the list's order does not matter).  The rows to fix are
 // counted first, so their loads can be issued in batches.
 template <class C>
-__global__ void __launch_bounds__(128) segment_fix_kernel(const Params p) {
+__device__ void segment_fix_tile(const Params& p, int64_t tid) {
     constexpr int BATCH = 8;
     const int lane = threadIdx.x & 31;
-    const int64_t tid = static_cast<int64_t>(blockIdx.x) * 4 + (threadIdx.x >> 5);
-    if (tid >= static_cast<int64_t>(p.n_chains) * p.n_tt) return;
-    if (p.fix[tid] == 0u || ptx::ld_relaxed(p.hdr) != 0u) return;
     const int64_t chain = tid / p.n_tt, jt = tid - chain * p.n_tt;
     const int64_t b = chain / p.n_slabs;
     const int64_t c2 = (chain - b * p.n_slabs) * (SLAB / 2);
@@ -931,8 +976,17 @@ __global__ void __launch_bounds__(128) segment_fix_kernel(const Params p) {
     if (C::REV && !C::PS) p.gpart[tid * 32 + lane] = add2(p.gpart[tid * 32 + lane], gl);
 }
 
+template <class C>
+__global__ void __launch_bounds__(128) segment_fix_kernel(const Params p) {
+    if (ptx::ld_relaxed(p.hdr) != 0u) return;
+    const int64_t n_fix = static_cast<int64_t>(ptx::ld_relaxed(p.hdr + 4));
+    const int64_t nw = static_cast<int64_t>(gridDim.x) * 4;
+    for (int64_t f = static_cast<int64_t>(blockIdx.x) * 4 + (threadIdx.x >> 5); f < n_fix; f += nw)
+        segment_fix_tile<C>(p, static_cast<int64_t>(p.fix[f]));
+}
+
 // ============================================================================
-// grad_lambda reduction (per-channel lambda): fixed-order fp64 sums
+// grad_lambda reduction (per-channel lambda): fixed-order sums (fp32 within a part, fp64 across parts)
 // ============================================================================
 __global__ void __launch_bounds__(256) reduce_parts_kernel(const float4* __restrict__ gpart,
                                                            double* __restrict__ rpart, int64_t B,
@@ -943,22 +997,31 @@ __global__ void __launch_bounds__(256) reduce_parts_kernel(const float4* __restr
     const int64_t total = B * n_tt;
     const int64_t per = (total + RED_PARTS - 1) / RED_PARTS;
     const int64_t k0 = part * per, k1 = lmin(total, k0 + per);
-    double acc[4] = {0.0, 0.0, 0.0, 0.0};
-    int64_t bb = (k0 + grp) / n_tt, jj = (k0 + grp) - bb * n_tt;
-#pragma unroll 8
-    for (int64_t k = k0 + grp; k < k1; k += 8) {
-        const float4 v = gpart[((bb * n_slabs + slab) * n_tt + jj) * 32 + lane];
-        jj += 8;
-        while (jj >= n_tt) {
-            jj -= n_tt;
-            ++bb;
+    // fp32 within a part (a few dozen tile partials), fp64 across parts and in the final tree
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    // this group's tiles k0 + grp, k0 + grp + 8, ...: loads issued in batches of 8, summed in that order
+    constexpr int RB = 8;
+    for (int64_t k = k0 + grp; k < k1; k += 8 * RB) {
+        float4 v[RB];
+#pragma unroll
+        for (int u = 0; u < RB; ++u) {
+            const int64_t kk = k + 8 * u;
+            if (kk < k1) {
+                const int64_t bb = kk / n_tt, jj = kk - bb * n_tt;
+                v[u] = gpart[((bb * n_slabs + slab) * n_tt + jj) * 32 + lane];
+            }
         }
-        acc[0] += v.x;
-        acc[1] += v.y;
-        acc[2] += v.z;
-        acc[3] += v.w;
+#pragma unroll
+        for (int u = 0; u < RB; ++u) {
+            if (k + 8 * u < k1) {
+                acc[0] += v[u].x;
+                acc[1] += v[u].y;
+                acc[2] += v[u].z;
+                acc[3] += v[u].w;
+            }
+        }
     }
-    for (int c = 0; c < 4; ++c) s[grp][lane][c] = acc[c];
+    for (int c = 0; c < 4; ++c) s[grp][lane][c] = static_cast<double>(acc[c]);
     __syncthreads();
     if (grp == 0) {
         double r[4] = {0.0, 0.0, 0.0, 0.0};
@@ -1163,9 +1226,10 @@ memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
     kernel<<<static_cast<unsigned>(n_tickets), C::THREADS, C::SMEM, s>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     if (sg.G > 1) {
-        segment_carry_kernel<<<static_cast<unsigned>((l.n_chains + 7) / 8), 256, 0, s>>>(p, C::REV);
+        segment_carry_kernel<<<static_cast<unsigned>(l.n_chains), CARRY_WARPS * 32, 0, s>>>(p, C::REV);
         const int64_t n_tiles = l.n_chains * l.n_tt;
-        segment_fix_kernel<C><<<static_cast<unsigned>((n_tiles + 3) / 4), 128, 0, s>>>(p);
+        const int64_t fix_ctas = lmin((n_tiles + 3) / 4, 152 * 8);  // the warps walk the list of tiles to fix
+        segment_fix_kernel<C><<<static_cast<unsigned>(fix_ctas), 128, 0, s>>>(p);
         if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     }
     if (out_layout) *out_layout = l;
