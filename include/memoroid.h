@@ -241,7 +241,8 @@ int memoroid_linattn_norm_kernels_per_call(int64_t B, int64_t L, int64_t H, int6
  *   y        fp32 [B, L, H, d] output; den fp32 [B, L, H] output x^T phi(q)
  *            (needed by the backward), or NULL
  *   S_last, z_last  the pair after the last step, or NULL
- * B, L, H > 0 (an empty call returns MEMOROID_ERR_UNSUPPORTED).  Workspace
+ * An empty call (B, L or H = 0) copies S0 / z0 to S_last / z_last (the
+ * backward: grad_S_last / grad_z_last to dS0 / dz0, dgamma = 0).  Workspace
  * 256-byte aligned, at least memoroid_linattn_norm_workspace_bytes; its
  * header reports device-side waits through memoroid_get_device_error.
  */

@@ -516,7 +516,28 @@ static memoroid_status_t lnorm_common(lnorm::Args& a, const float* gamma, int ga
                                       size_t workspace_bytes, void* stream) {
     if (!lnorm_shape_ok(a.B, a.L, a.H, a.d)) return MEMOROID_ERR_INVALID_ARG;
     if (gamma_per_step != 0 && gamma_per_step != 1) return MEMOROID_ERR_INVALID_ARG;
-    if (a.B == 0 || a.L == 0 || a.H == 0) return MEMOROID_ERR_UNSUPPORTED;  // nothing to scan: states pass through
+    if (a.B == 0 || a.L == 0 || a.H == 0) {
+        // nothing to scan: the outgoing state is the incoming one (and its gradient passes back)
+        cudaStream_t s = as_stream(stream);
+        const size_t nS = static_cast<size_t>(a.B * a.H * a.d * a.d) * 4, nz = static_cast<size_t>(a.B * a.H * a.d) * 4;
+        auto pass = [&](void* dst, const void* src, size_t bytes) {
+            if (dst == nullptr || bytes == 0) return cudaSuccess;
+            return src ? cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, s) : cudaMemsetAsync(dst, 0, bytes, s);
+        };
+        cudaError_t e = cudaSuccess;
+        if (!a.backward) {
+            if (e == cudaSuccess) e = pass(a.S_last, a.S0, nS);
+            if (e == cudaSuccess) e = pass(a.z_last, a.z0, nz);
+        } else {
+            if (e == cudaSuccess) e = pass(a.dS0, a.dS_last, nS);
+            if (e == cudaSuccess) e = pass(a.dz0, a.dz_last, nz);
+            if (e == cudaSuccess && a.dgamma != nullptr) {
+                const size_t ng = static_cast<size_t>(gamma_per_step ? a.B * a.L * a.H : a.H) * 4;
+                if (ng) e = cudaMemsetAsync(a.dgamma, 0, ng, s);
+            }
+        }
+        return e == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
+    }
     if (!a.q || !a.k || !a.v || !gamma || !start || !a.y) return MEMOROID_ERR_INVALID_ARG;
     if (!aligned(a.q, 16) || !aligned(a.k, 16) || !aligned(a.v, 16) || !aligned(a.y, 4) || !aligned(gamma, 4))
         return MEMOROID_ERR_INVALID_ARG;

@@ -133,3 +133,41 @@ def test_returns_validation(lib):
         m.MEMOROID_ERR_WORKSPACE
     assert lib.memoroid_gae(FAKE, None, FAKE, 0.9, 0.9, None, FAKE, 1, 8, FAKE, 4096, None) == \
         m.MEMOROID_ERR_INVALID_ARG
+
+
+def test_linattn_norm_validation(lib):
+    assert lib.memoroid_linattn_norm_workspace_bytes(1, 4096, 4, 64) > 0
+    for d in (0, 4, 12, 128):
+        assert lib.memoroid_linattn_norm_workspace_bytes(1, 100, 2, d) == 0
+        assert lib.memoroid_linattn_norm_kernels_per_call(1, 100, 2, d, 0, 0, 0) == -1
+
+    def fwd(q=FAKE, d=64, ws=FAKE, wsb=1 << 40, gps=0):
+        return lib.memoroid_linattn_norm_fwd(q, FAKE, FAKE, FAKE, gps, FAKE, None, None, FAKE + 0x1000, None, None,
+                                             None, 1, 256, 2, d, ws, wsb, None)
+
+    assert fwd(d=12) == m.MEMOROID_ERR_INVALID_ARG
+    assert fwd(gps=3) == m.MEMOROID_ERR_INVALID_ARG
+    assert fwd(q=None) == m.MEMOROID_ERR_INVALID_ARG
+    assert fwd(q=FAKE + 8) == m.MEMOROID_ERR_INVALID_ARG
+    assert fwd(ws=None) == m.MEMOROID_ERR_WORKSPACE
+    assert fwd(wsb=1024) == m.MEMOROID_ERR_WORKSPACE
+    # the backward needs den, grad_y and the three gradients
+    assert lib.memoroid_linattn_norm_bwd(FAKE, FAKE, FAKE, FAKE, 0, FAKE, None, None, FAKE, None, FAKE, None, None,
+                                         FAKE, FAKE, FAKE, None, None, None, 1, 256, 2, 64, FAKE, 1 << 40,
+                                         None) == m.MEMOROID_ERR_INVALID_ARG
+
+
+def test_tbb_validation(lib):
+    assert lib.memoroid_tbb_workspace_bytes(1000) >= 256 + 8 * 1002
+    assert lib.memoroid_tbb_workspace_bytes(-1) == 0
+    assert lib.memoroid_tbb_sample(FAKE, 4, 9, FAKE, 3, -1, FAKE, FAKE, None, FAKE, 1 << 20, None) == \
+        m.MEMOROID_ERR_INVALID_ARG
+    assert lib.memoroid_tbb_sample(FAKE, 4, 9, FAKE, 3, 5, None, FAKE, None, FAKE, 1 << 20, None) == \
+        m.MEMOROID_ERR_INVALID_ARG
+    assert lib.memoroid_tbb_sample(FAKE, 4, 9, FAKE, 3, 5, FAKE, FAKE + 4, None, FAKE, 1 << 20, None) == \
+        m.MEMOROID_ERR_INVALID_ARG
+    assert lib.memoroid_tbb_sample(FAKE, 4, 9, FAKE, 3, 5, FAKE, FAKE, None, FAKE, 16, None) == \
+        m.MEMOROID_ERR_WORKSPACE
+    assert lib.memoroid_gather_rows(FAKE, 10, 0, FAKE, 4, FAKE, FAKE, 256, None) == m.MEMOROID_ERR_INVALID_ARG
+    assert lib.memoroid_gather_rows(FAKE, 10, 16, None, 4, FAKE, FAKE, 256, None) == m.MEMOROID_ERR_INVALID_ARG
+    assert lib.memoroid_gather_rows(FAKE, 10, 16, FAKE, 4, FAKE, None, 256, None) == m.MEMOROID_ERR_WORKSPACE

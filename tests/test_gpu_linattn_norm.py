@@ -151,3 +151,18 @@ def test_config3_shape_sampled_episodes():
                                                        t["grad_y"][:, sl])
         for name, r in (("y", y), ("den", den), ("dq", dq), ("dk", dk), ("dv", dv), ("dgamma", dg)):
             assert rel_err(got[name][:, sl], r) <= TOL, name
+
+
+def test_empty_tape_passes_the_state_through():
+    m = _m()
+    rng = np.random.default_rng(5)
+    B, H, d = 2, 3, 16
+    S0 = rng.standard_normal((B, H, d, d)).astype(np.float32)
+    z0 = rng.uniform(0.5, 2.0, (B, H, d)).astype(np.float32)
+    q = torch.zeros((B, 0, H, d), dtype=torch.int16, device="cuda")
+    g = torch.ones(H, device="cuda")
+    st = torch.zeros((B, 0), dtype=torch.uint8, device="cuda")
+    ws = m.workspace(256, "cuda")
+    y, den, Sl, zl = m.linattn_norm_fwd(q, q, q, g, st, dev(S0), dev(z0), ws=ws)
+    torch.cuda.synchronize()
+    assert np.array_equal(Sl.cpu().numpy(), S0) and np.array_equal(zl.cpu().numpy(), z0)
