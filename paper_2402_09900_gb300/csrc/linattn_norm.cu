@@ -86,37 +86,39 @@ size_t total_bytes(int64_t B, int64_t L, int64_t H) {
     return o;
 }
 
-// q' = [phi(q), 0], k' = [phi(k), 0], v' = [v, 1, 0]: one thread per 16-byte
-// chunk (8 columns) of one padded row of one of the three operands.
+// q' = [phi(q), 0], k' = [phi(k), 0], v' = [v, 1, 1, 0]: one thread per
+// 16-byte chunk (8 columns) of a padded row, for all three operands
 __global__ void __launch_bounds__(256) prep_kernel(const uint4* __restrict__ q, const uint4* __restrict__ k,
                                                    const uint4* __restrict__ v, int64_t R, int d,
                                                    uint4* __restrict__ qp, uint4* __restrict__ kp,
                                                    uint4* __restrict__ vp) {
+    constexpr int CH = kW / 8;  // chunks per padded row
     const int in_chunks = d / 8;
-    const int64_t n = R * 3 * (kW / 8);
+    const int64_t n = R * CH;
     for (int64_t g = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; g < n;
          g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int c = static_cast<int>(g % (kW / 8));
-        const int which = static_cast<int>((g / (kW / 8)) % 3);
-        const int64_t r = g / (3 * (kW / 8));
-        uint4 out = make_uint4(0u, 0u, 0u, 0u);
+        const int c = static_cast<int>(g & (CH - 1));
+        const int64_t r = g >> 4;
+        uint4 oq = make_uint4(0u, 0u, 0u, 0u), ok = oq, ov = oq;
         if (c < in_chunks) {
-            const uint4* src = which == 0 ? q : (which == 1 ? k : v);
-            out = src[r * in_chunks + c];
-            if (which < 2) {
-                __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&out);
+            const int64_t src = r * in_chunks + c;
+            oq = q[src];
+            ok = k[src];
+            ov = v[src];
+            __nv_bfloat162* hq = reinterpret_cast<__nv_bfloat162*>(&oq);
+            __nv_bfloat162* hk = reinterpret_cast<__nv_bfloat162*>(&ok);
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float2 f = __bfloat1622float2(h[e]);
-                    h[e] = __floats2bfloat162_rn(phi(f.x), phi(f.y));
-                }
+            for (int e = 0; e < 4; ++e) {
+                const float2 fq = __bfloat1622float2(hq[e]), fk = __bfloat1622float2(hk[e]);
+                hq[e] = __floats2bfloat162_rn(phi(fq.x), phi(fq.y));
+                hk[e] = __floats2bfloat162_rn(phi(fk.x), phi(fk.y));
             }
-        } else if (which == 2 && c == in_chunks) {
-            __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&out);
-            h[0] = __floats2bfloat162_rn(1.f, 1.f);  // columns d and d + 1 of v' are 1
+        } else if (c == in_chunks) {
+            reinterpret_cast<__nv_bfloat162*>(&ov)[0] = __floats2bfloat162_rn(1.f, 1.f);  // columns d, d + 1 of v'
         }
-        uint4* dst = which == 0 ? qp : (which == 1 ? kp : vp);
-        dst[r * (kW / 8) + c] = out;
+        qp[g] = oq;
+        kp[g] = ok;
+        vp[g] = ov;
     }
 }
 
@@ -162,12 +164,14 @@ __global__ void __launch_bounds__(256) divide_kernel(const float4* __restrict__ 
     const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
     for (int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; r < R; r += nw) {
         const float4 a = yp[r * (kW / 4) + lane];
+        // d is a multiple of 8: column d is component 0 of lane d / 4
+        const float dn = __shfl_sync(0xffffffffu, a.x, d >> 2);
+        const float inv = 1.f / dn;
         const float comp[4] = {a.x, a.y, a.z, a.w};
-        const float dn = __shfl_sync(0xffffffffu, comp[d & 3], d >> 2);
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             const int j = 4 * lane + e;
-            if (j < d) y[r * d + j] = comp[e] / dn;
+            if (j < d) y[r * d + j] = comp[e] * inv;
         }
         if (lane == 0 && den != nullptr) den[r] = dn;
     }
@@ -207,21 +211,21 @@ __global__ void __launch_bounds__(256) upstream_kernel(const float* __restrict__
     }
 }
 
-// dq = dq'[:d] (.) phi'(q), dk = dk'[:d] (.) phi'(k), dv = dv'[:d]: one thread per column
+// dq = dq'[:d] (.) phi'(q), dk = dk'[:d] (.) phi'(k), dv = dv'[:d]: one warp per row
 __global__ void __launch_bounds__(256) chain_kernel(const float* __restrict__ dqp, const float* __restrict__ dkp,
                                                     const float* __restrict__ dvp, const __nv_bfloat16* __restrict__ q,
                                                     const __nv_bfloat16* __restrict__ k, int64_t R, int d,
                                                     float* __restrict__ dq, float* __restrict__ dk,
                                                     float* __restrict__ dv) {
-    const int64_t n = R * d;
-    for (int64_t g = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; g < n;
-         g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t r = g / d;
-        const int j = static_cast<int>(g - r * d);
-        const int64_t p = r * kW + j;
-        dq[g] = dqp[p] * dphi(__bfloat162float(q[g]));
-        dk[g] = dkp[p] * dphi(__bfloat162float(k[g]));
-        dv[g] = dvp[p];
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+    for (int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; r < R; r += nw) {
+        for (int j = lane; j < d; j += 32) {
+            const int64_t o = r * d + j, pp = r * kW + j;
+            dq[o] = dqp[pp] * dphi(__bfloat162float(q[o]));
+            dk[o] = dkp[pp] * dphi(__bfloat162float(k[o]));
+            dv[o] = dvp[pp];
+        }
     }
 }
 
@@ -245,7 +249,7 @@ int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_dga
 memoroid_status_t launch(const Args& a, cudaStream_t s) {
     const int64_t R = a.B * a.L * a.H, BH = a.B * a.H;
     const Buffers b = carve(a.workspace, a.B, a.L, a.H, a.backward);
-    prep_kernel<<<grid_for(R * 48), 256, 0, s>>>(static_cast<const uint4*>(a.q), static_cast<const uint4*>(a.k),
+    prep_kernel<<<grid_for(R * 16), 256, 0, s>>>(static_cast<const uint4*>(a.q), static_cast<const uint4*>(a.k),
                                                  static_cast<const uint4*>(a.v), R, static_cast<int>(a.d),
                                                  reinterpret_cast<uint4*>(b.q), reinterpret_cast<uint4*>(b.k),
                                                  reinterpret_cast<uint4*>(b.v));
@@ -296,7 +300,7 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
     l.dS0 = (a.dS0 != nullptr || a.dz0 != nullptr) ? b.S2 : nullptr;
     const memoroid_status_t st = la::launch_bwd(l, s);
     if (st != MEMOROID_OK) return st;
-    chain_kernel<<<grid_for(R * a.d), 256, 0, s>>>(b.dq, b.dk, b.dv, static_cast<const __nv_bfloat16*>(a.q),
+    chain_kernel<<<grid_for(R * 32), 256, 0, s>>>(b.dq, b.dk, b.dv, static_cast<const __nv_bfloat16*>(a.q),
                                                    static_cast<const __nv_bfloat16*>(a.k), R, static_cast<int>(a.d),
                                                    a.dq, a.dk, a.dv);
     if (l.dS0 != nullptr)
