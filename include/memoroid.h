@@ -255,7 +255,8 @@ memoroid_status_t memoroid_linattn_norm_fwd(const void *q, const void *k, const 
 
 /*
  * Backward: y and den are the forward's outputs; grad_y fp32 [B, L, H, d];
- * grad_S_last / grad_z_last or NULL; outputs dq, dk, dv fp32 [B, L, H, d],
+ * grad_S_last / grad_z_last or NULL; outputs dq, dk, dv fp32 [B, L, H, d]
+ * (16-byte aligned; B * L * H * d < 2^32),
  * dgamma ([H] summed, or [B, L, H]; NULL to skip), dS0 / dz0 or NULL.
  */
 memoroid_status_t memoroid_linattn_norm_bwd(const void *q, const void *k, const void *v,

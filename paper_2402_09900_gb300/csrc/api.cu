@@ -541,6 +541,9 @@ static memoroid_status_t lnorm_common(lnorm::Args& a, const float* gamma, int ga
     if (!a.q || !a.k || !a.v || !gamma || !start || !a.y) return MEMOROID_ERR_INVALID_ARG;
     if (!aligned(a.q, 16) || !aligned(a.k, 16) || !aligned(a.v, 16) || !aligned(a.y, 4) || !aligned(gamma, 4))
         return MEMOROID_ERR_INVALID_ARG;
+    if (a.backward && (!aligned(a.dq, 16) || !aligned(a.dk, 16) || !aligned(a.dv, 16)))
+        return MEMOROID_ERR_INVALID_ARG;
+    if (a.B * a.L * a.H * a.d >= (int64_t{1} << 32)) return MEMOROID_ERR_UNSUPPORTED;  // 32-bit element indices
     if (a.workspace == nullptr || !aligned(a.workspace, 256) ||
         workspace_bytes < lnorm::workspace_bytes(a.B, a.L, a.H))
         return MEMOROID_ERR_WORKSPACE;

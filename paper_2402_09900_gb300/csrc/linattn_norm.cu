@@ -211,21 +211,26 @@ __global__ void __launch_bounds__(256) upstream_kernel(const float* __restrict__
     }
 }
 
-// dq = dq'[:d] (.) phi'(q), dk = dk'[:d] (.) phi'(k), dv = dv'[:d]: one warp per row
-__global__ void __launch_bounds__(256) chain_kernel(const float* __restrict__ dqp, const float* __restrict__ dkp,
-                                                    const float* __restrict__ dvp, const __nv_bfloat16* __restrict__ q,
-                                                    const __nv_bfloat16* __restrict__ k, int64_t R, int d,
-                                                    float* __restrict__ dq, float* __restrict__ dk,
-                                                    float* __restrict__ dv) {
-    const int lane = threadIdx.x & 31;
-    const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
-    for (int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; r < R; r += nw) {
-        for (int j = lane; j < d; j += 32) {
-            const int64_t o = r * d + j, pp = r * kW + j;
-            dq[o] = dqp[pp] * dphi(__bfloat162float(q[o]));
-            dk[o] = dkp[pp] * dphi(__bfloat162float(k[o]));
-            dv[o] = dvp[pp];
-        }
+// dq = dq'[:d] (.) phi'(q), dk = dk'[:d] (.) phi'(k), dv = dv'[:d]: one
+// thread per 4 columns (16-byte loads and stores; 32-bit index arithmetic)
+__global__ void __launch_bounds__(256) chain_kernel(const float4* __restrict__ dqp, const float4* __restrict__ dkp,
+                                                    const float4* __restrict__ dvp, const uint2* __restrict__ q,
+                                                    const uint2* __restrict__ k, uint32_t R, uint32_t d4,
+                                                    float4* __restrict__ dq, float4* __restrict__ dk,
+                                                    float4* __restrict__ dv) {
+    const uint32_t n = R * d4;
+    for (uint32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < n; g += gridDim.x * blockDim.x) {
+        const uint32_t r = g / d4, c = g - r * d4;
+        const uint32_t pp = r * (kW / 4) + c;
+        const uint2 qb = q[g], kb = k[g];
+        const float2 q0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qb.x));
+        const float2 q1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qb.y));
+        const float2 k0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kb.x));
+        const float2 k1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kb.y));
+        const float4 a = dqp[pp], bb = dkp[pp];
+        dq[g] = make_float4(a.x * dphi(q0.x), a.y * dphi(q0.y), a.z * dphi(q1.x), a.w * dphi(q1.y));
+        dk[g] = make_float4(bb.x * dphi(k0.x), bb.y * dphi(k0.y), bb.z * dphi(k1.x), bb.w * dphi(k1.y));
+        dv[g] = dvp[pp];
     }
 }
 
@@ -300,9 +305,11 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
     l.dS0 = (a.dS0 != nullptr || a.dz0 != nullptr) ? b.S2 : nullptr;
     const memoroid_status_t st = la::launch_bwd(l, s);
     if (st != MEMOROID_OK) return st;
-    chain_kernel<<<grid_for(R * 32), 256, 0, s>>>(b.dq, b.dk, b.dv, static_cast<const __nv_bfloat16*>(a.q),
-                                                   static_cast<const __nv_bfloat16*>(a.k), R, static_cast<int>(a.d),
-                                                   a.dq, a.dk, a.dv);
+    chain_kernel<<<grid_for(R * a.d / 4), 256, 0, s>>>(
+        reinterpret_cast<const float4*>(b.dq), reinterpret_cast<const float4*>(b.dk),
+        reinterpret_cast<const float4*>(b.dv), static_cast<const uint2*>(a.q), static_cast<const uint2*>(a.k),
+        static_cast<uint32_t>(R), static_cast<uint32_t>(a.d / 4), reinterpret_cast<float4*>(a.dq),
+        reinterpret_cast<float4*>(a.dk), reinterpret_cast<float4*>(a.dv));
     if (l.dS0 != nullptr)
         unpad_state_kernel<<<grid_for(BH * a.d * (a.d + 1)), 256, 0, s>>>(b.S2, BH, static_cast<int>(a.d), 1, a.dS0,
                                                                            a.dz0);
