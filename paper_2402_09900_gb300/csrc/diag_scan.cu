@@ -1071,7 +1071,7 @@ namespace {
 #define MEMOROID_FWD_R 24
 #endif
 #ifndef MEMOROID_BWD_W
-#define MEMOROID_BWD_W 4
+#define MEMOROID_BWD_W 8
 #define MEMOROID_BWD_R 12
 #endif
 using FwdC = Cfg<MEMOROID_FWD_W, MEMOROID_FWD_R, false, false>;
