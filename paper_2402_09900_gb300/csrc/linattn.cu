@@ -1393,6 +1393,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             if (lane == 0) st_iv[8 + warp] = dl;
         }
         LA_MARK(5);
+        tc::fence_smem_to_async();  // the statistics in the V tile are overwritten by the next tile's load
         ok = wait_mbar(bar3, it & 1, p.wait_ns);
         if (tid == 0) bulk_wait_read();  // dv staging in G / K and dk staging are read before reuse
         if (__syncthreads_or(!ok)) {
@@ -1404,6 +1405,12 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         LA_MARK(6);
         if (tid == 0) gsum += (st_iv[8] + st_iv[9]) + (st_iv[10] + st_iv[11]);
         have_g = true;
+        // Q, K, V and dY are free (B3 is done, the staged stores are read): the next tile's
+        // loads go out now, while G becomes the next tile's bf16 operand
+        if (tile > tile_lo) {
+            if (tid == 0) issue_tile(tile - 1);
+            pending = true;
+        }
 
         // ---- G_{c-1} -> bf16 operand for the next tile (and dS0 at the tape start) ----
         {
@@ -1427,10 +1434,6 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         }
         tc::fence_before();
         __syncthreads();
-        if (tile > tile_lo) {
-            if (tid == 0) issue_tile(tile - 1);
-            pending = true;
-        }
         LA_MARK(7);
     }
 #ifdef MEMOROID_LA_TRACE
