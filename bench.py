@@ -56,6 +56,7 @@ LA_CFG = 5
 LA_WORKLOAD = ("linattn fwd+bwd (dq, dk, dv, per-step dgamma): B=1 tape, L=2^22 steps, H=8 heads, d_k=d_v=128, "
                "bf16 q/k/v, per-step gamma=sigmoid(N(3,1)), Geometric(1000) episodes")
 KERNEL_SRC = os.path.join(ROOT, "paper_2402_09900_gb300", "csrc", "diag_scan.cu")
+DATASHEET_HBM_GBS = 7900.0  # nominal HBM3e bandwidth, printed beside the fraction of the measured peak
 
 
 def _dist_env():
@@ -552,9 +553,44 @@ def cpu_baseline(t, target_s):
     s = oracle_sample(t, steps)
     dt = time_oracle_step(s)
     B = s["u"].shape[0]
-    return {"value": B * steps / dt, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+    # the same oracle on one thread, on a tenth of the sample
+    cores = oracle.max_threads()
+    steps1 = max(1024, steps // 10)
+    oracle.set_threads(1)
+    try:
+        dt1 = time_oracle_step(oracle_sample(t, steps1))
+    finally:
+        oracle.set_threads(cores)
+    return {"value": B * steps / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "single_thread_value": B * steps1 / dt1,
             "sample": f"first {steps} steps of the tape (x {s['u'].shape[2]} channels), fwd+bwd incl. "
-                      f"grad_lambda, fp64 C oracle with OpenMP over channels; {dt:.2f} s"}
+                      f"grad_lambda, fp64 C oracle with OpenMP over channels; {dt:.2f} s "
+                      f"(one thread: first {steps1} steps, {dt1:.2f} s)"}
+
+
+def linattn_cpu_baseline(target_steps):
+    """The linear-attention oracle (fwd+bwd with per-step dgamma) on the first
+    whole episodes of the linattn tape reaching `target_steps` steps, on the host
+    cores: transitions (steps) per second."""
+    import oracle
+    oracle.build()
+    c = tapegen.LINATTN_CONFIGS[LA_CFG]
+    rng = np.random.default_rng(tapegen.seed_for(LA_CFG))
+    starts = tapegen.geometric_tape_starts(rng, 4 * target_steps, c["mean"])
+    heads = np.flatnonzero(starts)
+    n = int(heads[np.searchsorted(heads, target_steps)]) if heads[-1] >= target_steps else len(starts)
+    t = tapegen.linattn_tape(1, n, c["H"], c["d"], c["d"], tapegen.seed_for(LA_CFG), mean=c["mean"],
+                             gamma_mode="step")
+    f = oracle.bf16_bits_to_f64
+    q, k, v = f(t["q"]), f(t["k"]), f(t["v"])
+    t0 = time.perf_counter()
+    oracle.linattn_fwd(q, k, v, t["gamma"], t["start"])
+    oracle.linattn_bwd(q, k, v, t["gamma"], t["start"], t["grad_y"])
+    dt = time.perf_counter() - t0
+    return {"value": n / dt, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+            "sample": f"{n} steps of whole episodes (the workload's recipe: {c['H']} heads, d={c['d']}, "
+                      f"per-step gamma, Geometric({c['mean']:.0f})), fwd+bwd incl. per-step dgamma, "
+                      f"fp64 C oracle with OpenMP over heads; {dt:.2f} s"}
 
 
 def run_reference(args):
@@ -773,10 +809,14 @@ def run_ours(args):
                 "peak_kind": f"{peak_kind} (copy bandwidth)", "traffic_note": traffic_note,
                 "fwd": {"achieved": fwd_gbs, "frac": fwd_gbs / peak, "avg_launch_ms": fwd_avg,
                         "algorithmic_bytes_per_launch": fwd_bytes},
-                "step_frac": (fwd_bytes + bwd_bytes) / (ms_per_step * 1e-3) / 1e9 / peak}
+                "step_frac": (fwd_bytes + bwd_bytes) / (ms_per_step * 1e-3) / 1e9 / peak,
+                "frac_of_datasheet": bwd_gbs / DATASHEET_HBM_GBS,
+                "step_frac_of_datasheet": (fwd_bytes + bwd_bytes) / (ms_per_step * 1e-3) / 1e9 / DATASHEET_HBM_GBS}
     la = None
     if ws == 1 and not args.skip_linattn:
         la = linattn_leg(args, m, dev, stream)
+        if not args.skip_cpu_baseline:
+            la["cpu_baseline"] = linattn_cpu_baseline(args.la_cpu_steps)
     rt = None
     if ws == 1 and not args.skip_returns:
         rt = returns_leg(args, m, dev, stream)
@@ -851,6 +891,8 @@ def main():
     ap.add_argument("--ffm-steps", type=int, default=20, help="timed FFM fwd+bwd steps")
     ap.add_argument("--ffm-tape-steps", type=int, default=0,
                     help="FFM tape length (profiler captures); 0 = the full L = 2^20 workload")
+    ap.add_argument("--la-cpu-steps", type=int, default=1 << 14,
+                    help="steps (whole episodes) of the linattn oracle baseline")
     ap.add_argument("--la-intra-reps", type=int, default=2000,
                     help="repetitions of the intra-tile contraction per CTA in the tensor benchmark")
     ap.add_argument("--tape-steps", type=int, default=0,
