@@ -1078,8 +1078,18 @@ using FwdC = Cfg<MEMOROID_FWD_W, MEMOROID_FWD_R, false, false>;
 using FwdS = Cfg<4, 8, false, true>;
 using BwdC = Cfg<MEMOROID_BWD_W, MEMOROID_BWD_R, true, false>;
 using BwdS = Cfg<4, 8, true, true>;
-using FwdF = Cfg<MEMOROID_FWD_W, MEMOROID_FWD_R, false, false, true>;
-using BwdF = Cfg<MEMOROID_BWD_W, MEMOROID_BWD_R, true, false, true>;
+// The FFM forward stages only x~ (a few bytes per step), so larger tiles pay:
+// 6 x 31 (186-step tiles) was the measured best on GB300.
+#ifndef MEMOROID_FFM_FWD_W
+#define MEMOROID_FFM_FWD_W 6
+#define MEMOROID_FFM_FWD_R 31
+#endif
+#ifndef MEMOROID_FFM_BWD_W
+#define MEMOROID_FFM_BWD_W MEMOROID_BWD_W
+#define MEMOROID_FFM_BWD_R MEMOROID_BWD_R
+#endif
+using FwdF = Cfg<MEMOROID_FFM_FWD_W, MEMOROID_FFM_FWD_R, false, false, true>;
+using BwdF = Cfg<MEMOROID_FFM_BWD_W, MEMOROID_FFM_BWD_R, true, false, true>;
 
 // Segments per chain: enough segment chains that a tile's predecessor was
 // handed out long before it (target), at least MIN_SEG_TILES tiles each.

@@ -95,8 +95,9 @@ def test_ffm_degenerate_flags(mode):
     check(t, with_S0=True)
 
 
-@pytest.mark.parametrize("L", [1, 2, 95, 96, 97])
+@pytest.mark.parametrize("L", [1, 2, 95, 96, 97, 185, 186, 187, 373])
 def test_ffm_tiny_tapes(L):
+    # around the forward's 186-step and the backward's 96-step tile edges
     t = tapegen.ffm_tape(2, L, 8, 2, tapegen.seed_for(720 + L), mean=3.0, with_S0=True)
     t["start"][1, 0] = 0
     check(t, with_S0=True)
