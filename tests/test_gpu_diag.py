@@ -103,12 +103,14 @@ def test_long_single_episode():
 def test_resets_on_tile_edges():
     L = 1024
     t = tapegen.diag_tape(1, L, 64, seed=9, start_mode="none")
-    for s in (1, 15, 16, 17, 63, 64, 65, 127, 128, 129, 255, 256, 512, 1023):
+    # around 16-, 32-, 64- and 128-step edges and the 96-step tiles of the scans
+    for s in (1, 11, 12, 13, 15, 16, 17, 23, 24, 25, 63, 64, 65, 95, 96, 97, 127, 128, 129, 191, 192, 193, 255,
+              256, 287, 288, 512, 1023):
         t["start"][0, s] = 1
     check(t, g_last=t["grad_h_last"])
 
 
-@pytest.mark.parametrize("L", [1, 2, 31, 33])
+@pytest.mark.parametrize("L", [1, 2, 31, 33, 95, 96, 97, 191, 193])
 def test_tiny_tapes(L):
     t = tapegen.diag_tape(2, L, 4, seed=10 + L, mean=3.0, with_h0=True)
     t["start"][1, 0] = 0
