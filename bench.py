@@ -227,6 +227,70 @@ LNORM_WORKLOAD = ("Linear Transformer with phi = 1 + ELU and its normalizer, fwd
                   "4 heads, d=64, bf16 q/k/v ~ N(0,1), per-head gamma in {0.9, 0.99, 0.999, 1.0}, Geometric(300) episodes")
 
 
+PS_WORKLOAD = ("diag scan fwd+bwd with a per-step lambda (input-dependent decay): B=1 tape, L=2^20 steps, "
+               "D=256 complex64 channels, |lambda_t| ~ U(0.9, 0.999), Geometric(500) episodes clipped to [1,10000]")
+
+
+def per_step_leg(args, m, dev, stream):
+    """Times the diagonal scan with a per-step lambda ([B, L, D], grad_lambda per
+    step) on the bench tape's shape."""
+    import torch
+
+    B, L, D = 1, 1 << 20, 256
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(tapegen.seed_for(10))
+    mag = 0.9 + 0.099 * torch.rand((B, L, D), generator=gen, device=dev)
+    ph = 2 * np.pi * torch.rand((B, L, D), generator=gen, device=dev)
+    lam = torch.polar(mag, ph).to(torch.complex64)
+    u = torch.randn((B, L, D), generator=gen, device=dev, dtype=torch.complex64)
+    g = torch.randn((B, L, D), generator=gen, device=dev, dtype=torch.complex64)
+    rng = np.random.default_rng(tapegen.seed_for(10))
+    st = torch.from_numpy(tapegen.geometric_tape_starts(rng, L, 500.0, 1, 10000)[None]).to(dev)
+    h, gu, gl = torch.empty_like(u), torch.empty_like(u), torch.empty_like(lam)
+    ws = m.diag_workspace(B, L, D, dev)
+
+    def fwd():
+        m.memoroid_scan_diag_fwd(lam, 1, u, st, None, h, None, B, L, D, ws, stream)
+
+    def bwd():
+        m.memoroid_scan_diag_bwd(lam, 1, st, None, h, g, None, gu, gl, None, B, L, D, ws, stream)
+
+    for _ in range(3):
+        fwd()
+        bwd()
+    torch.cuda.synchronize()
+    steps = args.ps_steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for i in range(steps):
+        evs[i][0].record(stream)
+        fwd()
+        evs[i][1].record(stream)
+        bwd()
+        evs[i][2].record(stream)
+    torch.cuda.synchronize()
+    if m.memoroid_get_device_error(ws) != m.MEMOROID_OK:
+        raise RuntimeError("device-side error in the per-step lambda leg")
+    f_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / steps
+    b_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / steps
+    # fwd reads u and lambda, writes h; bwd reads grad_h, h and lambda, writes grad_u and grad_lambda
+    fb = B * L * D * 24 + B * L
+    bb = B * L * D * 40 + B * L
+    peak, peak_kind = _peaks()
+    kpc = (m.memoroid_scan_diag_kernels_per_call(B, L, D, 1, 0, 0) + m.memoroid_scan_diag_kernels_per_call(B, L, D, 1, 1, 1))
+    out = {"workload": PS_WORKLOAD, "value": B * L / ((f_ms + b_ms) * 1e-3), "unit": UNIT, "steps": steps,
+           "ms_per_step": f_ms + b_ms, "fwd_ms": f_ms, "bwd_ms": b_ms,
+           "roofline": {"bound": "hbm", "peak": peak, "unit": "GB/s", "peak_kind": f"{peak_kind} (copy bandwidth)",
+                        "fwd": {"algorithmic_bytes_per_call": fb, "achieved": fb / (f_ms * 1e-3) / 1e9,
+                                "frac": fb / (f_ms * 1e-3) / 1e9 / peak},
+                        "bwd": {"algorithmic_bytes_per_call": bb, "achieved": bb / (b_ms * 1e-3) / 1e9,
+                                "frac": bb / (b_ms * 1e-3) / 1e9 / peak},
+                        "step_frac": (fb + bb) / ((f_ms + b_ms) * 1e-3) / 1e9 / peak},
+           "gpu_launches": steps * kpc}
+    del lam, u, g, h, gu, gl, ws
+    torch.cuda.empty_cache()
+    return out
+
+
 def lnorm_leg(args, m, dev, stream):
     """Times memoroid_linattn_norm_fwd + _bwd on the config-3 shape."""
     import torch
@@ -653,6 +717,11 @@ def run_ours(args):
         # profiling mode: the normalised Linear Transformer leg alone
         print(json.dumps({"linattn_norm": lnorm_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
         return
+    if args.only_per_step:
+        # profiling mode: the per-step lambda diag leg alone
+        print(json.dumps({"diag_per_step_lambda": per_step_leg(args, m, dev, torch.cuda.current_stream())}),
+              flush=True)
+        return
     if args.only_tbb:
         # profiling mode: the tape-based batching leg alone
         print(json.dumps({"tbb": tbb_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
@@ -823,6 +892,9 @@ def run_ours(args):
     ff = None
     if ws == 1 and not args.skip_ffm:
         ff = ffm_leg(args, m, dev, stream)
+    ps = None
+    if ws == 1 and not args.skip_per_step:
+        ps = per_step_leg(args, m, dev, stream)
     ln = None
     if ws == 1 and not args.skip_lnorm:
         ln = lnorm_leg(args, m, dev, stream)
@@ -848,6 +920,7 @@ def run_ours(args):
         "ffm": ff,
         "tbb": tb,
         "linattn_norm": ln,
+        "diag_per_step_lambda": ps,
     }
     print(json.dumps(out), flush=True)
     if ws > 1:
@@ -880,6 +953,10 @@ def main():
     ap.add_argument("--skip-ffm", action="store_true", help="omit the Fast and Forgetful Memory leg")
     ap.add_argument("--skip-tbb", action="store_true", help="omit the tape-based batching leg")
     ap.add_argument("--skip-lnorm", action="store_true", help="omit the normalised Linear Transformer leg")
+    ap.add_argument("--skip-per-step", action="store_true", help="omit the per-step lambda diag leg")
+    ap.add_argument("--ps-steps", type=int, default=20, help="timed per-step lambda fwd+bwd steps")
+    ap.add_argument("--only-per-step", action="store_true",
+                    help="profiling mode: run and print only the per-step lambda diag leg")
     ap.add_argument("--only-lnorm", action="store_true",
                     help="profiling mode: run and print only the normalised Linear Transformer leg")
     ap.add_argument("--lnorm-steps", type=int, default=10, help="timed normalised Linear Transformer steps")

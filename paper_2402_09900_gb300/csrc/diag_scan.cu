@@ -1075,9 +1075,18 @@ namespace {
 #define MEMOROID_BWD_R 12
 #endif
 using FwdC = Cfg<MEMOROID_FWD_W, MEMOROID_FWD_R, false, false>;
-using FwdS = Cfg<4, 8, false, true>;
+// per-step lambda (two staged arrays forward, three backward): measured best shapes
+#ifndef MEMOROID_FWDS_W
+#define MEMOROID_FWDS_W 4
+#define MEMOROID_FWDS_R 12
+#endif
+#ifndef MEMOROID_BWDS_W
+#define MEMOROID_BWDS_W 8
+#define MEMOROID_BWDS_R 8
+#endif
+using FwdS = Cfg<MEMOROID_FWDS_W, MEMOROID_FWDS_R, false, true>;
 using BwdC = Cfg<MEMOROID_BWD_W, MEMOROID_BWD_R, true, false>;
-using BwdS = Cfg<4, 8, true, true>;
+using BwdS = Cfg<MEMOROID_BWDS_W, MEMOROID_BWDS_R, true, true>;
 // The FFM forward stages only x~ (a few bytes per step), so larger tiles pay:
 // 6 x 31 (186-step tiles) was the measured best on GB300.
 #ifndef MEMOROID_FFM_FWD_W
