@@ -50,13 +50,15 @@ __device__ __forceinline__ int64_t episode(const int64_t* begin, int64_t E, int6
 __global__ void __launch_bounds__(kScanThreads) offsets_kernel(const int64_t* __restrict__ begin, int64_t E, int64_t N,
                                                                const int64_t* __restrict__ ep, int64_t K, int64_t B,
                                                                int64_t* __restrict__ off, int64_t* __restrict__ meta,
-                                                               uint32_t* __restrict__ hdr) {
+                                                               uint32_t* __restrict__ hdr,
+                                                               int64_t* __restrict__ n_used) {
     __shared__ int64_t warp_sum[kScanThreads / 32];
     __shared__ int64_t s_carry;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (tid == 0) {
         s_carry = 0;
         meta[0] = 0;  // draws used
+        *hdr = 0u;    // this call's error word (this kernel runs first)
     }
     __syncthreads();
     for (int64_t c0 = 0; c0 < K; c0 += kChunk) {
@@ -111,12 +113,14 @@ __global__ void __launch_bounds__(kScanThreads) offsets_kernel(const int64_t* __
         __syncthreads();
         if (total >= B) break;
     }
+    __syncthreads();  // meta[0] is written by the thread that holds the last piece
     if (tid == 0) {
         if (s_carry < B) {  // the draws do not fill the batch
             bad_data(hdr);
             meta[0] = K;
         }
         meta[1] = s_carry < B ? s_carry : B;  // steps covered by pieces
+        if (n_used != nullptr) *n_used = meta[0];
     }
 }
 
@@ -201,14 +205,9 @@ memoroid_status_t launch_sample(const int64_t* begin, int64_t E, int64_t N, cons
     uint32_t* hdr = reinterpret_cast<uint32_t*>(ws);
     int64_t* meta = reinterpret_cast<int64_t*>(ws + kHeaderBytes);
     int64_t* off = meta + 2;
-    if (cudaMemsetAsync(workspace, 0, kHeaderBytes, s) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    offsets_kernel<<<1, kScanThreads, 0, s>>>(begin, E, N, ep, K, B, off, meta, hdr);
+    offsets_kernel<<<1, kScanThreads, 0, s>>>(begin, E, N, ep, K, B, off, meta, hdr, n_used);
     fill_kernel<<<kFillCtas, 256, 0, s>>>(begin, E, N, ep, B, off, meta, start, src);
-    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
-    if (n_used != nullptr &&
-        cudaMemcpyAsync(n_used, meta, sizeof(int64_t), cudaMemcpyDeviceToDevice, s) != cudaSuccess)
-        return MEMOROID_ERR_CUDA;
-    return MEMOROID_OK;
+    return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
 }
 
 memoroid_status_t launch_gather(const void* rows, int64_t N, int64_t row_bytes, const int64_t* src, int64_t B,
