@@ -342,7 +342,8 @@ struct FwdSmem {
     // the fp32 output tile is staged in the finished stage in the 128-byte
     // swizzled layout of its TMA store (32 channels per 128-byte row, chunk
     // of 32 channels at m * T * 128)
-    static_assert(T * D * 4 <= STAGE, "output staging fits in one stage");
+    static_assert(T * D * 4 <= 2 * TILE, "output staging fits in the Q and K slots of one stage");
+    static_assert(D * D * 2 <= TILE, "pass F's stored state is staged in the V slot of the same stage");
     // TMEM columns: scores P, intra output, inter output, state S
     static constexpr uint32_t COL_P = 0, COL_YA = 128, COL_YI = 128 + D, COL_S = 128 + 2 * D;
     static constexpr uint32_t TMEM_COLS = 512;
@@ -392,11 +393,20 @@ struct FwdParams {
 // Thread -> row of a D x D state accumulator in TMEM.  With M = 128 the row
 // is the TMEM lane; with M = 64 rows 16q..16q+15 sit in lanes 32q..32q+15 and
 // the upper 16 lanes of each quarter hold nothing (-1).
-// 16 bf16 values of row `row` (columns j0..j0+15) of the stored state before tile `tile`.
+// Byte offset of element (row, col) in the stored image of a D x D bf16
+// state: rows of 2D bytes whose 16-byte unit u sits at u ^ (row % (D / 8)),
+// so that eight consecutive rows written 16 bytes at a time (pass F), and one
+// row read 2 bytes at a time by 32 consecutive columns (pass R), touch
+// distinct bank groups of shared memory.
 template <int D>
-__device__ __forceinline__ void store_state_row(uint16_t* states, int64_t bh, int64_t n_tiles, int64_t tile,
-                                                     int row, int j0, const float* v) {
-    uint16_t* dst = states + ((bh * n_tiles + tile) * D + row) * D + j0;
+__device__ __forceinline__ uint32_t state_off(int row, int col) {
+    return static_cast<uint32_t>(row * (2 * D) + ((((col >> 3) ^ (row & (D / 8 - 1)))) << 4) + (col & 7) * 2);
+}
+
+// 16 bf16 values of row `row` (columns j0..j0+15, j0 a multiple of 16) of a
+// stored state image at `base` (global or shared memory).
+template <int D>
+__device__ __forceinline__ void store_state_row(unsigned char* base, int row, int j0, const float* v) {
     uint4 w0, w1;
     w0.x = pack_bf16x2(v[0], v[1]);
     w0.y = pack_bf16x2(v[2], v[3]);
@@ -406,8 +416,12 @@ __device__ __forceinline__ void store_state_row(uint16_t* states, int64_t bh, in
     w1.y = pack_bf16x2(v[10], v[11]);
     w1.z = pack_bf16x2(v[12], v[13]);
     w1.w = pack_bf16x2(v[14], v[15]);
-    reinterpret_cast<uint4*>(dst)[0] = w0;
-    reinterpret_cast<uint4*>(dst)[1] = w1;
+    *reinterpret_cast<uint4*>(base + state_off<D>(row, j0)) = w0;
+    *reinterpret_cast<uint4*>(base + state_off<D>(row, j0 + 8)) = w1;
+}
+template <int D>
+__device__ __forceinline__ unsigned char* state_image(uint16_t* states, int64_t bh, int64_t n_tiles, int64_t tile) {
+    return reinterpret_cast<unsigned char*>(states + (bh * n_tiles + tile) * D * D);
 }
 
 template <int D>
@@ -539,7 +553,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                     }
                 }
                 store_bf16x16(smem + S::OFF_SB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
-                if (BWD && metas[0].has_start == 0) store_state_row<D>(p.states, bh, p.n_tiles, 0, srow, j0, v);
+                if (BWD && metas[0].has_start == 0)
+                    store_state_row<D>(state_image<D>(p.states, bh, p.n_tiles, 0), srow, j0, v);
             } else {
 #pragma unroll
                 for (int x = 0; x < 16; ++x) v[x] = 0.f;
@@ -557,7 +572,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         float zero[16];
 #pragma unroll
         for (int x = 0; x < 16; ++x) zero[x] = 0.f;
-        for (int j0 = half * SC; j0 < half * SC + SC; j0 += 16) store_state_row<D>(p.states, bh, p.n_tiles, 0, srow, j0, zero);
+        for (int j0 = half * SC; j0 < half * SC + SC; j0 += 16)
+            store_state_row<D>(state_image<D>(p.states, bh, p.n_tiles, 0), srow, j0, zero);
     }
 
     constexpr uint32_t ID_QS = tc::idesc_bf16(128, D, false, true);
@@ -578,6 +594,12 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     for (int c = 0; c < nt && !failed; ++c) {
         const int s = c & 1;
         const TileMeta& mc = metas[c % S::NMETA];
+        if (BWD && have_prev) {
+            // pass F reads q_t for the z term in the epilogue: bring this thread's part of the row into L2
+            const int t = 32 * quarter + lane;
+            const int64_t tt = (tile0 + c) * T + t;
+            if (mc.seg[t] < 0 && tt < p.L) prefetch_l2(p.zq + ((b * p.L + tt) * p.H + h) * D + half * SC);
+        }
         // tile c's loads (issued one iteration ago) and the previous tile's
         // output stores (which read stage s ^ 1) are complete
         bool ok = wait_mbar(&full[s], (c >> 1) & 1, p.wait_ns);
@@ -695,6 +717,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
 #pragma unroll
             for (int cc = 0; cc < SC / 32; ++cc) {
                 const int j0 = half * SC + cc * 32;
+                uint4 qv[4];  // pass F: q_t, columns j0..j0+31, in flight while the outputs are read
+                if (zrow) {
+#pragma unroll
+                    for (int x = 0; x < 4; ++x) qv[x] = *reinterpret_cast<const uint4*>(qrow + j0 + 8 * x);
+                }
                 uint32_t ya[32], yi[32];
                 tc::ld16_nowait(lane_base + S::COL_YA + j0, ya);
                 tc::ld16_nowait(lane_base + S::COL_YA + j0 + 16, ya + 16);
@@ -719,7 +746,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 if (zrow) {
 #pragma unroll
                     for (int x = 0; x < 32; x += 8) {
-                        const uint4 u = *reinterpret_cast<const uint4*>(qrow + j0 + x);
+                        const uint4 u = qv[x / 8];
                         const float2 q0 = unpack_bf16x2(u.x), q1 = unpack_bf16x2(u.y), q2 = unpack_bf16x2(u.z),
                                      q3 = unpack_bf16x2(u.w);
                         zacc = fmaf(q0.x, __uint_as_float(yi[x]), zacc);
@@ -754,8 +781,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                     store_bf16x16(smem + S::OFF_SB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
                     store_bf16x16(smem + S::OFF_SB, core_off(srow, j0 + 16, D), core_off(srow, j0 + 24, D), v + 16);
                     if (BWD && mn.has_start == 0) {
-                        store_state_row<D>(p.states, bh, p.n_tiles, tile0 + c + 1, srow, j0, v);
-                        store_state_row<D>(p.states, bh, p.n_tiles, tile0 + c + 1, srow, j0 + 16, v + 16);
+                        // staged in this stage's V slot (free once the tile's contractions are
+                        // done) and bulk-stored with the output rows
+                        unsigned char* img = smem + (stage_v(s) - sbase);
+                        store_state_row<D>(img, srow, j0, v);
+                        store_state_row<D>(img, srow, j0 + 16, v + 16);
                     }
                 }
                 if (scale) {
@@ -806,6 +836,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                     *reinterpret_cast<float4*>(ybase + static_cast<int64_t>(r) * row_stride + j) = v;
                 }
             }
+            if (BWD && lane == 0 && c + 1 < nt && metas[(c + 1) % S::NMETA].has_start == 0)
+                bulk_s2g(state_image<D>(p.states, bh, p.n_tiles, tile0 + c + 1), stage_v(s), D * D * 2);
             bulk_commit();
         }
         if (BWD && warp == 1) {
@@ -873,6 +905,10 @@ struct BwdSmem {
     static constexpr int OFF_Q = 0, OFF_K = TILE, OFF_V = 2 * TILE, OFF_DY = 3 * TILE;
     static constexpr int OFF_PM = 4 * TILE, OFF_DPM = 4 * TILE + T * T * 2;
     static constexpr int OFF_GB = 4 * TILE + 2 * T * T * 2;
+    // the stored state S_{c-1} (bf16, [j][i]) arrives with the tile in the dPm
+    // buffer, which RP1 overwrites only after B1 is done
+    static constexpr int OFF_SS = OFF_DPM;
+    static_assert(D * D * 2 <= T * T * 2, "stored state fits in the dPm buffer");
     static constexpr int OFF_META = OFF_GB + D * D * 2;
     static constexpr int OFF_BAR = OFF_META + static_cast<int>(sizeof(TileMeta));
     static constexpr int BYTES = OFF_BAR + 64;
@@ -999,16 +1035,22 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
     auto dk_chunk = [](int m) { return S::dk_chunk(m); };
     auto dv_chunk = [](int m) { return S::dv_chunk(m); };
 
-    // thread 0: TMA loads of a tile and its metadata, completing on `full`
-    auto issue_tile = [&](int64_t tile) {
-        mbar_arrive_expect_tx(full, 4 * S::TILE + sizeof(TileMeta));
+    // thread 0: TMA loads of a tile, its metadata and (once a reverse state
+    // exists) the stored forward state before it, completing on `full`.  The
+    // state slot of a tile with a begin flag was never written: it is loaded
+    // all the same and not read.
+    auto issue_tile = [&](int64_t tile, bool with_state) {
+        constexpr uint32_t kStateBytes = D * D * 2;
+        mbar_arrive_expect_tx(full, 4 * S::TILE + sizeof(TileMeta) + (with_state ? kStateBytes : 0u));
         const int64_t t0 = tile * T;
         tma_tile<D>(sQ, &p.map_q, h, t0, b, full);
         tma_tile<D>(sK, &p.map_k, h, t0, b, full);
         tma_tile<D>(sV, &p.map_v, h, t0, b, full);
         tma_tile<D>(sDY, &p.map_dy, h, t0, b, full);
         bulk_g2s(smem + S::OFF_META, p.meta + bh * p.n_tiles + tile, sizeof(TileMeta), full);
+        if (with_state) bulk_g2s(smem + S::OFF_SS, p.states + (bh * p.n_tiles + tile) * D * D, kStateBytes, full);
     };
+    bool have_g = seg_hi == p.L && p.dS_last != nullptr;  // a reverse state enters the current tile
 
     if (tid == 0) {
         mbar_init(bar1, 1);
@@ -1027,16 +1069,14 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
     tc::fence_before();
     __syncthreads();
     tc::fence_after();
-    if (tid == 0) issue_tile(tile_hi - 1);
+    if (tid == 0) issue_tile(tile_hi - 1, have_g);
     const uint32_t tm = *tslot;
     const uint32_t lane_base = tm + (static_cast<uint32_t>(32 * quarter) << 16);
     const int srow = state_row<D>(quarter, lane);
     constexpr int SC = D / 2;
 
     // ---- incoming reverse state: dS_last for the segment that ends the tape ----
-    bool have_g = false;
-    if (seg_hi == p.L && p.dS_last != nullptr) {
-        have_g = true;
+    if (have_g) {
         const float* src = p.dS_last + bh * D * D;
 #pragma unroll 1
         for (int cc = 0; cc < SC / 16; ++cc) {
@@ -1108,17 +1148,35 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             }
             tc::commit(bar1);
         }
-        // while B1 runs: the stored state S_{c-1} (this thread's row of <G, S>),
-        // pass F's dgamma term and gamma for the rows of warps 0-3
+        // while B1 runs (it reads G only through its bf16 copy): this thread's row
+        // of <G_c, S_{c-1}> and G *= a_c in tensor memory; pass F's dgamma term
+        // and gamma for the rows of warps 0-3
         const bool need_iv = have_g && !tile_start;
-        uint32_t sv[SC / 2];
-        if (need_iv && srow >= 0) {
-            const uint16_t* srows = p.states + (bh * p.n_tiles + tile) * D * D;  // S^T, row-major [j][i]
+        float ivp = 0.f;
+        {
+            const bool scale = have_g && !tile_start && mc.a != 1.f;
+            if (need_iv || scale) {
+                const unsigned char* ss = smem + S::OFF_SS;  // S_{c-1}: element [j][i] at state_off(j, i)
 #pragma unroll
-            for (int x = 0; x < SC; x += 2) {
-                const int j = half * SC + x;
-                sv[x / 2] = static_cast<uint32_t>(srows[j * D + srow]) | (static_cast<uint32_t>(srows[(j + 1) * D + srow]) << 16);
+                for (int cc = 0; cc < SC / 16; ++cc) {
+                    const int j0 = half * SC + cc * 16;
+                    float v[16];
+                    tc::ld16(lane_base + S::COL_G + j0, v);
+                    if (need_iv && srow >= 0) {
+#pragma unroll
+                        for (int x = 0; x < 16; ++x)
+                            ivp = fmaf(v[x], __uint_as_float(static_cast<uint32_t>(*reinterpret_cast<const uint16_t*>(
+                                                                 ss + state_off<D>(j0 + x, srow))) << 16), ivp);
+                    }
+                    if (scale) {
+#pragma unroll
+                        for (int x = 0; x < 16; ++x) v[x] *= mc.a;
+                        tc::st16(lane_base + S::COL_G + j0, v);
+                    }
+                }
             }
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) ivp += __shfl_xor_sync(0xffffffffu, ivp, off);
         }
         float dlf = 0.f, gmt = 1.f;
         if (warp < 4) {
@@ -1205,34 +1263,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             }
             st_x[half * T + t] = xacc;
         }
-        {
-            float ivp = 0.f;
-            const bool scale = have_g && !tile_start && mc.a != 1.f;
-            if (need_iv || scale) {
-#pragma unroll
-                for (int cc = 0; cc < SC / 16; ++cc) {
-                    const int j0 = half * SC + cc * 16;
-                    float v[16];
-                    tc::ld16(lane_base + S::COL_G + j0, v);
-                    if (need_iv && srow >= 0) {
-#pragma unroll
-                        for (int x = 0; x < 16; x += 2) {
-                            const uint32_t w2 = sv[(cc * 16 + x) / 2];
-                            ivp = fmaf(v[x], __uint_as_float(w2 << 16), ivp);
-                            ivp = fmaf(v[x + 1], __uint_as_float(w2 & 0xffff0000u), ivp);
-                        }
-                    }
-                    if (scale) {
-#pragma unroll
-                        for (int x = 0; x < 16; ++x) v[x] *= mc.a;
-                        tc::st16(lane_base + S::COL_G + j0, v);
-                    }
-                }
-            }
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) ivp += __shfl_xor_sync(0xffffffffu, ivp, off);
-            if (lane == 0) st_iv[warp] = ivp;
-        }
+        if (lane == 0) st_iv[warp] = ivp;
         __syncthreads();  // every x_r has read the unscaled K
         {
             // K~ = w_out (.) K in place (K is not read unscaled after this)
@@ -1408,7 +1439,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         // Q, K, V and dY are free (B3 is done, the staged stores are read): the next tile's
         // loads go out now, while G becomes the next tile's bf16 operand
         if (tile > tile_lo) {
-            if (tid == 0) issue_tile(tile - 1);
+            if (tid == 0) issue_tile(tile - 1, true);
             pending = true;
         }
 
@@ -1739,7 +1770,7 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     f.dlam_f = dlam_f;
     f.states = states;
 #ifdef MEMOROID_LA_TRACE
-    f.trace = nullptr;
+    f.trace = la_trace_buffer();  // pass F's phases replace the forward's in slots 0-7
 #endif
     if (set_smem(fwd_kernel<D, true>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
     fwd_kernel<D, true><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);

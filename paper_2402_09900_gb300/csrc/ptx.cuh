@@ -79,6 +79,8 @@ __device__ __forceinline__ void tma_store_4d(const void* map, uint32_t src_smem,
                  "r"(src_smem), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
                  : "memory");
 }
+// Brings the 128-byte line holding `ptr` into L2 (no register is written).
+__device__ __forceinline__ void prefetch_l2(const void* ptr) { asm volatile("prefetch.global.L2 [%0];" ::"l"(ptr)); }
 __device__ __forceinline__ void prefetch_tensormap(const void* map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
 }

@@ -561,3 +561,87 @@ class DiagScan(torch.autograd.Function):
         gu, gl, gh0 = diag_bwd(lam, start, h, grad_h.contiguous(), None, h0,
                                want_lambda=ctx.needs_input_grad[0], want_h0=ctx.has_h0)
         return gl, gu, None, gh0
+
+
+def _bf16_bits(t):
+    """The int16 view the C ABI takes for a bf16 tensor (bf16 tensors in, int16 views pass through)."""
+    if t.dtype == torch.bfloat16:
+        return t.contiguous().view(torch.int16)
+    if t.dtype == torch.int16:
+        return t.contiguous()
+    raise ValueError("q, k, v must be bfloat16 tensors (or their int16 bit views)")
+
+
+class LinAttnScan(torch.autograd.Function):
+    """Autograd wrapper of the decayed linear-attention memoroid:
+    y = LinAttnScan.apply(q, k, v, gamma, start, S0) with q, k, v bfloat16
+    [B, L, H, d], gamma fp32 [H] or [B, L, H], S0 fp32 [B, H, d, d] or None.
+    Gradients come back in the inputs' dtypes (dq, dk, dv rounded to bf16)."""
+
+    @staticmethod
+    def forward(ctx, q, k, v, gamma, start, S0=None):
+        qb, kb, vb = _bf16_bits(q), _bf16_bits(k), _bf16_bits(v)
+        y, _ = linattn_fwd(qb, kb, vb, gamma.contiguous(), start, S0, want_last=False)
+        ctx.save_for_backward(qb, kb, vb, gamma, start, S0 if S0 is not None else torch.empty(0))
+        ctx.has_S0 = S0 is not None
+        ctx.dtypes = (q.dtype, k.dtype, v.dtype)
+        return y
+
+    @staticmethod
+    def backward(ctx, grad_y):
+        qb, kb, vb, gamma, start, S0 = ctx.saved_tensors
+        S0 = S0 if ctx.has_S0 else None
+        dq, dk, dv, dg, dS0 = linattn_bwd(qb, kb, vb, gamma.contiguous(), start, grad_y.contiguous(), None, S0,
+                                          want_gamma=ctx.needs_input_grad[3], want_S0=ctx.has_S0)
+
+        def cast(g, dt):
+            return g.to(torch.bfloat16) if dt == torch.bfloat16 else None  # int16 views take no gradient
+
+        return cast(dq, ctx.dtypes[0]), cast(dk, ctx.dtypes[1]), cast(dv, ctx.dtypes[2]), dg, None, dS0
+
+
+class FFMScan(torch.autograd.Function):
+    """Autograd wrapper of the Fast and Forgetful Memory memoroid:
+    z = FFMScan.apply(x, alpha, omega, start, S0) with x fp32 [B, L, m],
+    alpha [m], omega [c], S0 complex64 [B, m, c] or None; z = Re(X) || Im(X)."""
+
+    @staticmethod
+    def forward(ctx, x, alpha, omega, start, S0=None):
+        z, _ = ffm_fwd(x.contiguous(), alpha.contiguous(), omega.contiguous(), start, S0, want_last=False)
+        ctx.save_for_backward(alpha, omega, start, S0 if S0 is not None else torch.empty(0), z)
+        ctx.has_S0 = S0 is not None
+        return z
+
+    @staticmethod
+    def backward(ctx, grad_z):
+        alpha, omega, start, S0, z = ctx.saved_tensors
+        S0 = S0 if ctx.has_S0 else None
+        gx, ga, go, gS0 = ffm_bwd(alpha.contiguous(), omega.contiguous(), start, z, grad_z.contiguous(), None, S0,
+                                  want_params=ctx.needs_input_grad[1] or ctx.needs_input_grad[2],
+                                  want_S0=ctx.has_S0)
+        return gx, ga, go, None, gS0
+
+
+class LinAttnNormScan(torch.autograd.Function):
+    """Autograd wrapper of the Linear Transformer with phi = 1 + ELU and its
+    normalizer: y = LinAttnNormScan.apply(q, k, v, gamma, start) with q, k, v
+    bfloat16 [B, L, H, d] (d a multiple of 8, at most 120)."""
+
+    @staticmethod
+    def forward(ctx, q, k, v, gamma, start):
+        qb, kb, vb = _bf16_bits(q), _bf16_bits(k), _bf16_bits(v)
+        y, den, _, _ = linattn_norm_fwd(qb, kb, vb, gamma.contiguous(), start, want_last=False)
+        ctx.save_for_backward(qb, kb, vb, gamma, start, y, den)
+        ctx.dtypes = (q.dtype, k.dtype, v.dtype)
+        return y
+
+    @staticmethod
+    def backward(ctx, grad_y):
+        qb, kb, vb, gamma, start, y, den = ctx.saved_tensors
+        dq, dk, dv, dg, _, _ = linattn_norm_bwd(qb, kb, vb, gamma.contiguous(), start, y, den, grad_y.contiguous(),
+                                                want_gamma=ctx.needs_input_grad[3])
+
+        def cast(g, dt):
+            return g.to(torch.bfloat16) if dt == torch.bfloat16 else None
+
+        return cast(dq, ctx.dtypes[0]), cast(dk, ctx.dtypes[1]), cast(dv, ctx.dtypes[2]), dg, None

@@ -246,6 +246,58 @@ def test_bwd_config3_full():
     assert errs["dgamma"] <= TOL
 
 
+
+def test_bwd_episode_isolation_bitwise():
+    # changing grad_y inside one episode leaves dq, dk, dv of every other episode unchanged, bit for bit
+    t = tapegen.linattn_tape(1, 2000, 2, 64, 64, seed=tapegen.seed_for(60), mean=200.0, gamma_mode="step",
+                             with_grad=True)
+    a = run_gpu_bwd(t)
+    starts = np.flatnonzero(t["start"][0])
+    s, e = int(starts[3]), int(starts[4])
+    t2 = dict(t)
+    t2["grad_y"] = t["grad_y"].copy()
+    t2["grad_y"][0, s:e] += 0.75
+    b = run_gpu_bwd(t2)
+    outside = np.ones(2000, dtype=bool)
+    outside[s:e] = False
+    for name, x, y in zip(("dq", "dk", "dv"), a[:3], b[:3]):
+        assert np.array_equal(x[0, outside], y[0, outside]), name
+        assert not np.array_equal(x[0, s:e], y[0, s:e]), name
+
+
+@pytest.mark.parametrize("cut,tol,tol_b", [(1280, 1e-5, 2.0 ** -8), (1300, TOL, TOL)])
+def test_split_resume_fwd_and_bwd(cut, tol, tol_b):
+    # a tape scanned in two calls (S_last of the first is S0 of the second) gives the
+    # one-call outputs; the second call's dS0 fed as the first call's dS_last gives
+    # the one-call gradients.  A cut on a 128-step tile edge leaves every tile's
+    # operands as in one call, so the forward agrees to fp32 rounding; the backward
+    # recomputes the state at the cut with transposed operands, whose fp32 sum can
+    # round to the neighbouring bf16 value (one bf16 ulp, 2^-8 relative, of the
+    # carried state).  A ragged cut re-tiles the rest of the tape, so its bf16
+    # roundings of the masked scores and states differ and the bar is the kernels' own.
+    L = 3000
+    t = tapegen.linattn_tape(2, L, 2, 64, 64, seed=tapegen.seed_for(62), mean=400.0, gamma_mode="step",
+                             with_grad=True, with_S0=True)
+    t["start"][:, 0] = 0
+    t["start"][:, cut] = 0  # an episode runs across the cut
+
+    def part(sl):
+        return dict(q=t["q"][:, sl], k=t["k"][:, sl], v=t["v"][:, sl], gamma=t["gamma"][:, sl],
+                    start=t["start"][:, sl], grad_y=t["grad_y"][:, sl])
+
+    y, S_last = run_gpu_fwd(t, S0=t["S0"])
+    p1, p2 = part(slice(0, cut)), part(slice(cut, L))
+    y1, S1 = run_gpu_fwd(p1, S0=t["S0"])
+    y2, S2 = run_gpu_fwd(p2, S0=S1)
+    assert rel_err(np.concatenate([y1, y2], axis=1), y) <= tol
+    assert rel_err(S2, S_last) <= tol
+    full = run_gpu_bwd(t, t["S0"], t["grad_S_last"])
+    g2 = run_gpu_bwd(p2, S1, t["grad_S_last"])
+    g1 = run_gpu_bwd(p1, t["S0"], g2[4])
+    for i, name in enumerate(("dq", "dk", "dv", "dgamma")):
+        assert rel_err(np.concatenate([g1[i], g2[i]], axis=1), full[i]) <= tol_b, name
+    assert rel_err(g1[4], full[4]) <= tol_b
+
 def _episode_slices(start_row, rng, n):
     starts = np.flatnonzero(start_row)
     picks = rng.choice(len(starts) - 1, size=n, replace=False)
