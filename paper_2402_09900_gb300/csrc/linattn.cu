@@ -600,10 +600,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             const int64_t tt = (tile0 + c) * T + t;
             if (mc.seg[t] < 0 && tt < p.L) prefetch_l2(p.zq + ((b * p.L + tt) * p.H + h) * D + half * SC);
         }
-        // tile c's loads (issued one iteration ago) and the previous tile's
-        // output stores (which read stage s ^ 1) are complete
+        // tile c's loads (issued during the previous tile) are complete
         bool ok = wait_mbar(&full[s], (c >> 1) & 1, p.wait_ns);
-        if (warp == 0) bulk_wait_read();
         tc::fence_smem_to_async();
         tc::fence_before();
         if (__syncthreads_or(!ok)) {
@@ -613,10 +611,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         pending = -1;
         tc::fence_after();
         LA_MARK(0);
-        if (c + 1 < nt) {
-            if (tid == 32) issue_tile(c + 1, s ^ 1, c + 2 < nt ? c + 2 : -1, -1);
-            pending = c + 1;
-        }
 
         // ---- P = Q K^T and (with an incoming state) Y_inter = Q S_prev ----
         if (tid == 0) {
@@ -673,10 +667,18 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             scale_rows_sw<D>(smem + (stage_k(s) - sbase), tid,
                              [&](int r) { return r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f; });
         }
+        // the previous tile's output stores, which read stage s ^ 1, have drained
+        // behind this tile's first contractions and mask pass
+        if (warp == 0) bulk_wait_read();
         tc::fence_smem_to_async();
         tc::fence_before();
         __syncthreads();
         tc::fence_after();
+        // the next tile's loads into stage s ^ 1
+        if (c + 1 < nt) {
+            if (tid == 32) issue_tile(c + 1, s ^ 1, c + 2 < nt ? c + 2 : -1, -1);
+            pending = c + 1;
+        }
 
         // ---- Y_intra = Pm V and S = a S + K~^T V ----
         if (tid == 0) {
@@ -691,6 +693,15 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             tc::commit(bar2);
         }
         LA_MARK(4);
+        const int64_t t0 = (tile0 + c) * T;
+        // pass F: this thread's part of q_t for the z term, in flight while the contractions run
+        uint4 qv[BWD ? SC / 8 : 1];
+        const bool zrow = BWD && have_prev && mc.seg[32 * quarter + lane] < 0 && t0 + 32 * quarter + lane < p.L;
+        if (zrow) {
+            const uint16_t* qrow = p.zq + ((b * p.L + t0 + 32 * quarter + lane) * p.H + h) * D + half * SC;
+#pragma unroll
+            for (int x = 0; x < SC / 8; ++x) qv[x] = *reinterpret_cast<const uint4*>(qrow + 8 * x);
+        }
         ok = wait_mbar(bar2, c & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
             failed = true;
@@ -702,7 +713,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         LA_MARK(5);
 
         // ---- y = Y_intra + w_in * Y_inter, staged as fp32 rows in stage s ----
-        const int64_t t0 = (tile0 + c) * T;
         // rows of this tile that belong to the segment
         const int r_lo = static_cast<int>(max(static_cast<int64_t>(0), seg_lo - t0));
         const int r_hi = static_cast<int>(min(static_cast<int64_t>(T), seg_hi - t0));
@@ -711,17 +721,10 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             const float w_in = (have_prev && mc.seg[t] < 0) ? fast_exp2(mc.lam2[t]) : 0.f;
             unsigned char* yst = smem + s * S::STAGE + t * 128;  // row t of chunk 0
             // BWD: z_t = w_in_t q_t . (S_{c-1} dy_t), the inter output dotted with q
-            const bool zrow = BWD && w_in != 0.f && t0 + t < p.L;
-            const uint16_t* qrow = BWD ? p.zq + ((b * p.L + t0 + t) * p.H + h) * D : nullptr;
             float zacc = 0.f;
 #pragma unroll
             for (int cc = 0; cc < SC / 32; ++cc) {
                 const int j0 = half * SC + cc * 32;
-                uint4 qv[4];  // pass F: q_t, columns j0..j0+31, in flight while the outputs are read
-                if (zrow) {
-#pragma unroll
-                    for (int x = 0; x < 4; ++x) qv[x] = *reinterpret_cast<const uint4*>(qrow + j0 + 8 * x);
-                }
                 uint32_t ya[32], yi[32];
                 tc::ld16_nowait(lane_base + S::COL_YA + j0, ya);
                 tc::ld16_nowait(lane_base + S::COL_YA + j0 + 16, ya + 16);
@@ -746,7 +749,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 if (zrow) {
 #pragma unroll
                     for (int x = 0; x < 32; x += 8) {
-                        const uint4 u = qv[x / 8];
+                        const uint4 u = qv[cc * 4 + x / 8];
                         const float2 q0 = unpack_bf16x2(u.x), q1 = unpack_bf16x2(u.y), q2 = unpack_bf16x2(u.z),
                                      q3 = unpack_bf16x2(u.w);
                         zacc = fmaf(q0.x, __uint_as_float(yi[x]), zacc);
@@ -1157,21 +1160,24 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             const bool scale = have_g && !tile_start && mc.a != 1.f;
             if (need_iv || scale) {
                 const unsigned char* ss = smem + S::OFF_SS;  // S_{c-1}: element [j][i] at state_off(j, i)
+                uint32_t gv[SC];
 #pragma unroll
-                for (int cc = 0; cc < SC / 16; ++cc) {
-                    const int j0 = half * SC + cc * 16;
-                    float v[16];
-                    tc::ld16(lane_base + S::COL_G + j0, v);
-                    if (need_iv && srow >= 0) {
+                for (int cc = 0; cc < SC / 16; ++cc) tc::ld16_nowait(lane_base + S::COL_G + half * SC + cc * 16, gv + cc * 16);
+                tc::ld_wait();
+                if (need_iv && srow >= 0) {
 #pragma unroll
-                        for (int x = 0; x < 16; ++x)
-                            ivp = fmaf(v[x], __uint_as_float(static_cast<uint32_t>(*reinterpret_cast<const uint16_t*>(
-                                                                 ss + state_off<D>(j0 + x, srow))) << 16), ivp);
-                    }
-                    if (scale) {
+                    for (int x = 0; x < SC; ++x)
+                        ivp = fmaf(__uint_as_float(gv[x]),
+                                   __uint_as_float(static_cast<uint32_t>(*reinterpret_cast<const uint16_t*>(
+                                                       ss + state_off<D>(half * SC + x, srow))) << 16), ivp);
+                }
+                if (scale) {
 #pragma unroll
-                        for (int x = 0; x < 16; ++x) v[x] *= mc.a;
-                        tc::st16(lane_base + S::COL_G + j0, v);
+                    for (int cc = 0; cc < SC / 16; ++cc) {
+                        float v[16];
+#pragma unroll
+                        for (int x = 0; x < 16; ++x) v[x] = __uint_as_float(gv[cc * 16 + x]) * mc.a;
+                        tc::st16(lane_base + S::COL_G + half * SC + cc * 16, v);
                     }
                 }
             }
@@ -1238,25 +1244,23 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             float xacc = 0.f;
             if (have_g) {
                 const unsigned char* kt = smem + S::OFF_K;
-#pragma unroll 1
-                for (int cc = 0; cc < SC / 16; ++cc) {
-                    const int j0 = half * SC + cc * 16;
-                    float gi[16];
-                    tc::ld16(lane_base + S::COL_DKI + j0, gi);
+                uint32_t gi[SC];  // this thread's half row of V G^T, all loads in flight at once
 #pragma unroll
-                    for (int x = 0; x < 16; x += 8) {
-                        const uint4 u = *reinterpret_cast<const uint4*>(kt + sw_off(t, j0 + x));
-                        const float2 k0 = unpack_bf16x2(u.x), k1 = unpack_bf16x2(u.y), k2 = unpack_bf16x2(u.z),
-                                     k3 = unpack_bf16x2(u.w);
-                        xacc = fmaf(k0.x, gi[x], xacc);
-                        xacc = fmaf(k0.y, gi[x + 1], xacc);
-                        xacc = fmaf(k1.x, gi[x + 2], xacc);
-                        xacc = fmaf(k1.y, gi[x + 3], xacc);
-                        xacc = fmaf(k2.x, gi[x + 4], xacc);
-                        xacc = fmaf(k2.y, gi[x + 5], xacc);
-                        xacc = fmaf(k3.x, gi[x + 6], xacc);
-                        xacc = fmaf(k3.y, gi[x + 7], xacc);
-                    }
+                for (int cc = 0; cc < SC / 16; ++cc) tc::ld16_nowait(lane_base + S::COL_DKI + half * SC + cc * 16, gi + cc * 16);
+                tc::ld_wait();
+#pragma unroll
+                for (int x = 0; x < SC; x += 8) {
+                    const uint4 u = *reinterpret_cast<const uint4*>(kt + sw_off(t, half * SC + x));
+                    const float2 k0 = unpack_bf16x2(u.x), k1 = unpack_bf16x2(u.y), k2 = unpack_bf16x2(u.z),
+                                 k3 = unpack_bf16x2(u.w);
+                    xacc = fmaf(k0.x, __uint_as_float(gi[x]), xacc);
+                    xacc = fmaf(k0.y, __uint_as_float(gi[x + 1]), xacc);
+                    xacc = fmaf(k1.x, __uint_as_float(gi[x + 2]), xacc);
+                    xacc = fmaf(k1.y, __uint_as_float(gi[x + 3]), xacc);
+                    xacc = fmaf(k2.x, __uint_as_float(gi[x + 4]), xacc);
+                    xacc = fmaf(k2.y, __uint_as_float(gi[x + 5]), xacc);
+                    xacc = fmaf(k3.x, __uint_as_float(gi[x + 6]), xacc);
+                    xacc = fmaf(k3.y, __uint_as_float(gi[x + 7]), xacc);
                 }
                 const float w_out = t >= mc.last_start ? fast_exp2(mc.lam2[T - 1] - mc.lam2[t]) : 0.f;
                 xacc *= w_out;
@@ -1357,21 +1361,30 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             const int r = 32 * quarter + lane;
             const float w_out = r >= mc.last_start ? fast_exp2(mc.lam2[T - 1] - mc.lam2[r]) : 0.f;
 #pragma unroll 1
-            for (int cc = 0; cc < SC / 16; ++cc) {
-                const int j0 = half * SC + cc * 16;
-                uint32_t rk[16], ri[16], rv[16];
+            for (int cc = 0; cc < SC / 32; ++cc) {
+                const int j0 = half * SC + cc * 32;
+                uint32_t rk[32], ri[32], rv[32];
                 tc::ld16_nowait(lane_base + S::COL_DK + j0, rk);
+                tc::ld16_nowait(lane_base + S::COL_DK + j0 + 16, rk + 16);
                 tc::ld16_nowait(lane_base + S::COL_DV + j0, rv);
-                if (have_g) tc::ld16_nowait(lane_base + S::COL_DKI + j0, ri);
-                tc::ld_wait();
-                float vk[16], vv[16];
-#pragma unroll
-                for (int x = 0; x < 16; ++x) {
-                    vk[x] = have_g ? fmaf(w_out, __uint_as_float(ri[x]), __uint_as_float(rk[x])) : __uint_as_float(rk[x]);
-                    vv[x] = __uint_as_float(rv[x]);
+                tc::ld16_nowait(lane_base + S::COL_DV + j0 + 16, rv + 16);
+                if (have_g) {
+                    tc::ld16_nowait(lane_base + S::COL_DKI + j0, ri);
+                    tc::ld16_nowait(lane_base + S::COL_DKI + j0 + 16, ri + 16);
                 }
-                stage_f32x16(smem, dk_chunk, r, j0, vk);
-                stage_f32x16(smem, dv_chunk, r, j0, vv);
+                tc::ld_wait();
+#pragma unroll
+                for (int hh = 0; hh < 32; hh += 16) {
+                    float vk[16], vv[16];
+#pragma unroll
+                    for (int x = 0; x < 16; ++x) {
+                        vk[x] = have_g ? fmaf(w_out, __uint_as_float(ri[hh + x]), __uint_as_float(rk[hh + x]))
+                                       : __uint_as_float(rk[hh + x]);
+                        vv[x] = __uint_as_float(rv[hh + x]);
+                    }
+                    stage_f32x16(smem, dk_chunk, r, j0 + hh, vk);
+                    stage_f32x16(smem, dv_chunk, r, j0 + hh, vv);
+                }
             }
         }
         tc::fence_smem_to_async();
@@ -1447,11 +1460,16 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         {
             const bool last = tile == tile_lo;
             const bool write_ds0 = last && seg_lo == 0 && p.dS0 != nullptr;
-#pragma unroll 1
+            uint32_t gv[SC];
+#pragma unroll
+            for (int cc = 0; cc < SC / 16; ++cc) tc::ld16_nowait(lane_base + S::COL_G + half * SC + cc * 16, gv + cc * 16);
+            tc::ld_wait();
+#pragma unroll
             for (int cc = 0; cc < SC / 16; ++cc) {
                 const int j0 = half * SC + cc * 16;
                 float v[16];
-                tc::ld16(lane_base + S::COL_G + j0, v);
+#pragma unroll
+                for (int x = 0; x < 16; ++x) v[x] = __uint_as_float(gv[cc * 16 + x]);
                 if (srow >= 0) {
                     if (!last) store_bf16x16(smem + S::OFF_GB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
                     if (write_ds0) {
