@@ -40,7 +40,8 @@ constexpr int T = 128;         // steps per tile = the M of the tile contraction
 // After a wait has run out, in-flight TMA loads and tensor-core batches are
 // drained with this fixed limit before the CTA frees its TMEM and exits.
 constexpr uint64_t kDrainNs = 1000000000ull;
-constexpr int kThreads = 256;  // 8 warps: warp w reads TMEM lane quarter w % 4, column half w / 4
+constexpr int kThreads = 256;   // forward / pass F: 8 warps, warp w reads TMEM lane quarter w % 4, column half w / 4
+constexpr int kRThreads = 512;  // pass R: 16 warps, warp w reads lane quarter w % 4, column quarter w / 4
 constexpr int kTargetCtas = 152;
 
 // Per-tile decay and reset summary, computed once per (tape, head, tile).
@@ -283,10 +284,11 @@ __device__ __forceinline__ void tma_tile(uint32_t dst, const CUtensorMap* map, i
 // thread per (row, 64-channel chunk) while there are enough threads, each
 // with one weight and eight 16-byte units (conflict-free: the swizzle spreads
 // the same unit of 8 consecutive rows over 8 bank groups).
-template <int D, typename WFn>
+template <int D, int NT = kThreads, typename WFn>
 __device__ __forceinline__ void scale_rows_sw(unsigned char* tile, int tid, WFn weight) {
     constexpr int CHUNKS = D / 64;
-    constexpr int UNITS = 8 * CHUNKS * T / kThreads;  // units per thread: 8 (d = 128) or 4 (d = 64)
+    constexpr int UNITS = 8 * CHUNKS * T / NT;  // units per thread (NT threads)
+    static_assert(UNITS >= 1, "at most one thread per 16-byte unit");
     const int r = tid & (T - 1);
     const float w = weight(r);
     if (w == 1.f) return;
@@ -917,10 +919,10 @@ struct BwdSmem {
     static constexpr int BYTES = OFF_BAR + 64;
     // statistics, in the V tile (free once the first contractions are done)
     static constexpr int ST_COL = OFF_V;                // [4][T] column sums of E per lane quarter
-    static constexpr int ST_ROW = ST_COL + 4 * T * 4;   // [2][T] row sums of E per column half
-    static constexpr int ST_X = ST_ROW + 2 * T * 4;     // [2][T] x_r per column half
-    static constexpr int ST_IV = ST_X + 2 * T * 4;      // [8] per-warp partial <G, S>
-    static constexpr int ST_INTRA = ST_IV + 64;         // [T] intra-tile term
+    static constexpr int ST_ROW = ST_COL + 4 * T * 4;   // [4][T] row sums of E per column quarter
+    static constexpr int ST_X = ST_ROW + 4 * T * 4;     // [4][T] x_r per column quarter
+    static constexpr int ST_IV = ST_X + 4 * T * 4;      // [16] per-warp partial <G, S>, then [4] tile totals
+    static constexpr int ST_INTRA = ST_IV + 128;        // [T] intra-tile term
     static constexpr int ST_WT = ST_INTRA + T * 4;      // [4] per-warp totals of x
     static_assert(ST_WT + 64 <= OFF_V + TILE, "statistics fit in the V tile");
     // fp32 dk / dv tiles staged for their TMA stores (128-byte swizzled, 32
@@ -996,11 +998,11 @@ __device__ __forceinline__ void stage_f32x16(unsigned char* smem, ChunkFn chunk,
 }
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant__ BwdParams p) {
+__global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant__ BwdParams p) {
     using S = BwdSmem<D>;
     extern __shared__ __align__(1024) unsigned char smem[];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int quarter = warp & 3, half = warp >> 2;
+    const int quarter = warp & 3, cq = warp >> 2;  // TMEM lane quarter, column quarter
     const int64_t bh = blockIdx.x / p.G;
     const int g = static_cast<int>(blockIdx.x % p.G);
     const int64_t b = bh / p.H, h = bh % p.H;
@@ -1076,14 +1078,15 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
     const uint32_t tm = *tslot;
     const uint32_t lane_base = tm + (static_cast<uint32_t>(32 * quarter) << 16);
     const int srow = state_row<D>(quarter, lane);
-    constexpr int SC = D / 2;
+    constexpr int SC = D / 4;  // state and output columns per thread
+    constexpr int PC = T / 4;  // score columns per thread
 
     // ---- incoming reverse state: dS_last for the segment that ends the tape ----
     if (have_g) {
         const float* src = p.dS_last + bh * D * D;
 #pragma unroll 1
         for (int cc = 0; cc < SC / 16; ++cc) {
-            const int j0 = half * SC + cc * 16;
+            const int j0 = cq * SC + cc * 16;
             float v[16];
             if (srow >= 0) {
 #pragma unroll
@@ -1162,14 +1165,14 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
                 const unsigned char* ss = smem + S::OFF_SS;  // S_{c-1}: element [j][i] at state_off(j, i)
                 uint32_t gv[SC];
 #pragma unroll
-                for (int cc = 0; cc < SC / 16; ++cc) tc::ld16_nowait(lane_base + S::COL_G + half * SC + cc * 16, gv + cc * 16);
+                for (int cc = 0; cc < SC / 16; ++cc) tc::ld16_nowait(lane_base + S::COL_G + cq * SC + cc * 16, gv + cc * 16);
                 tc::ld_wait();
                 if (need_iv && srow >= 0) {
 #pragma unroll
                     for (int x = 0; x < SC; ++x)
                         ivp = fmaf(__uint_as_float(gv[x]),
                                    __uint_as_float(static_cast<uint32_t>(*reinterpret_cast<const uint16_t*>(
-                                                       ss + state_off<D>(half * SC + x, srow))) << 16), ivp);
+                                                       ss + state_off<D>(cq * SC + x, srow))) << 16), ivp);
                 }
                 if (scale) {
 #pragma unroll
@@ -1177,7 +1180,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
                         float v[16];
 #pragma unroll
                         for (int x = 0; x < 16; ++x) v[x] = __uint_as_float(gv[cc * 16 + x]) * mc.a;
-                        tc::st16(lane_base + S::COL_G + half * SC + cc * 16, v);
+                        tc::st16(lane_base + S::COL_G + cq * SC + cc * 16, v);
                     }
                 }
             }
@@ -1208,49 +1211,46 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             const float lt = mc.lam2[t];
             const int st = mc.seg[t];
             float rsum = 0.f;
-#pragma unroll 1
-            for (int cc = 0; cc < 2; ++cc) {
-                const int r0 = half * 64 + cc * 32;
-                uint32_t rp[32], rd[32];
-                tc::ld16_nowait(lane_base + S::COL_P + r0, rp);
-                tc::ld16_nowait(lane_base + S::COL_P + r0 + 16, rp + 16);
-                tc::ld16_nowait(lane_base + S::COL_DP + r0, rd);
-                tc::ld16_nowait(lane_base + S::COL_DP + r0 + 16, rd + 16);
-                tc::ld_wait();
-                float pm[32], dpm[32], e[32];
+            const int r0 = cq * PC;  // this warp's 32 score columns, in two batches of 16
+            float e[PC];
+            unsigned char* pmb = smem + S::OFF_PM;
+            unsigned char* dpmb = smem + S::OFF_DPM;
 #pragma unroll
-                for (int x = 0; x < 32; ++x) {
-                    const int r = r0 + x;
+            for (int cc = 0; cc < PC; cc += 16) {
+                uint32_t rp[16], rd[16];
+                tc::ld16_nowait(lane_base + S::COL_P + r0 + cc, rp);
+                tc::ld16_nowait(lane_base + S::COL_DP + r0 + cc, rd);
+                tc::ld_wait();
+                float pm[16], dpm[16];
+#pragma unroll
+                for (int x = 0; x < 16; ++x) {
+                    const int r = r0 + cc + x;
                     const float m = (r <= t && r >= st) ? fast_exp2(lt - mc.lam2[r]) : 0.f;
                     const float pv = __uint_as_float(rp[x]), dv = __uint_as_float(rd[x]);
                     pm[x] = m * pv;
                     dpm[x] = m * dv;
-                    e[x] = pm[x] * dv;
-                    rsum += e[x];
+                    e[cc + x] = pm[x] * dv;
+                    rsum += e[cc + x];
                 }
-                unsigned char* pmb = smem + S::OFF_PM;
-                unsigned char* dpmb = smem + S::OFF_DPM;
-#pragma unroll
-                for (int x = 0; x < 32; x += 16) {
-                    store_bf16x16(pmb, core_off(t, r0 + x, T), core_off(t, r0 + x + 8, T), pm + x);
-                    store_bf16x16(dpmb, core_off(t, r0 + x, T), core_off(t, r0 + x + 8, T), dpm + x);
-                }
-                const float cs = warp_transpose_sum32(e, lane);
-                st_col[quarter * T + r0 + lane] = cs;
+                store_bf16x16(pmb, core_off(t, r0 + cc, T), core_off(t, r0 + cc + 8, T), pm);
+                store_bf16x16(dpmb, core_off(t, r0 + cc, T), core_off(t, r0 + cc + 8, T), dpm);
             }
-            st_row[half * T + t] = rsum;
+            static_assert(PC == 32, "one transposed warp sum per thread's score columns");
+            const float cs = warp_transpose_sum32(e, lane);
+            st_col[quarter * T + r0 + lane] = cs;
+            st_row[cq * T + t] = rsum;
 
             // x_r = w_out_r k_r . (G_c v_r), from the unscaled K tile
             float xacc = 0.f;
             if (have_g) {
                 const unsigned char* kt = smem + S::OFF_K;
-                uint32_t gi[SC];  // this thread's half row of V G^T, all loads in flight at once
+                uint32_t gi[SC];  // this thread's quarter row of V G^T, all loads in flight at once
 #pragma unroll
-                for (int cc = 0; cc < SC / 16; ++cc) tc::ld16_nowait(lane_base + S::COL_DKI + half * SC + cc * 16, gi + cc * 16);
+                for (int cc = 0; cc < SC / 16; ++cc) tc::ld16_nowait(lane_base + S::COL_DKI + cq * SC + cc * 16, gi + cc * 16);
                 tc::ld_wait();
 #pragma unroll
                 for (int x = 0; x < SC; x += 8) {
-                    const uint4 u = *reinterpret_cast<const uint4*>(kt + sw_off(t, half * SC + x));
+                    const uint4 u = *reinterpret_cast<const uint4*>(kt + sw_off(t, cq * SC + x));
                     const float2 k0 = unpack_bf16x2(u.x), k1 = unpack_bf16x2(u.y), k2 = unpack_bf16x2(u.z),
                                  k3 = unpack_bf16x2(u.w);
                     xacc = fmaf(k0.x, __uint_as_float(gi[x]), xacc);
@@ -1265,7 +1265,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
                 const float w_out = t >= mc.last_start ? fast_exp2(mc.lam2[T - 1] - mc.lam2[t]) : 0.f;
                 xacc *= w_out;
             }
-            st_x[half * T + t] = xacc;
+            st_x[cq * T + t] = xacc;
         }
         if (lane == 0) st_iv[warp] = ivp;
         __syncthreads();  // every x_r has read the unscaled K
@@ -1273,7 +1273,8 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             // K~ = w_out (.) K in place (K is not read unscaled after this)
             const float lend = mc.lam2[T - 1];
             const int ls = mc.last_start;
-            scale_rows_sw<D>(smem + S::OFF_K, tid, [&](int r) { return r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f; });
+            scale_rows_sw<D, kRThreads>(smem + S::OFF_K, tid,
+                                        [&](int r) { return r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f; });
         }
         tc::fence_smem_to_async();
         tc::fence_before();
@@ -1303,7 +1304,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             for (int x = 0; x < 4; ++x) {
                 const int u = 4 * lane + x;
                 d[x] = (st_col[u] + st_col[T + u]) + (st_col[2 * T + u] + st_col[3 * T + u]) -
-                       (st_row[u] + st_row[T + u]);
+                       ((st_row[u] + st_row[T + u]) + (st_row[2 * T + u] + st_row[3 * T + u]));
             }
             float incl = d[0] + d[1] + d[2] + d[3];
 #pragma unroll
@@ -1322,7 +1323,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         float xpre_in = 0.f;
         if (warp < 4) {
             const int t = 32 * warp + lane;
-            const float xt = st_x[t] + st_x[T + t];
+            const float xt = (st_x[t] + st_x[T + t]) + (st_x[2 * T + t] + st_x[3 * T + t]);
             float incl = xt;
 #pragma unroll
             for (int off = 1; off < 32; off <<= 1) {
@@ -1342,7 +1343,8 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         LA_MARK(3);
 
         // ---- RP2: Q~ = w_in (.) Q in place, then B3: G += Q~^T dY ----
-        scale_rows_sw<D>(smem + S::OFF_Q, tid, [&](int r) { return mc.seg[r] < 0 ? fast_exp2(mc.lam2[r]) : 0.f; });
+        scale_rows_sw<D, kRThreads>(smem + S::OFF_Q, tid,
+                                    [&](int r) { return mc.seg[r] < 0 ? fast_exp2(mc.lam2[r]) : 0.f; });
         tc::fence_smem_to_async();
         tc::fence_before();
         __syncthreads();
@@ -1360,31 +1362,22 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         {
             const int r = 32 * quarter + lane;
             const float w_out = r >= mc.last_start ? fast_exp2(mc.lam2[T - 1] - mc.lam2[r]) : 0.f;
-#pragma unroll 1
-            for (int cc = 0; cc < SC / 32; ++cc) {
-                const int j0 = half * SC + cc * 32;
-                uint32_t rk[32], ri[32], rv[32];
+#pragma unroll
+            for (int cc = 0; cc < SC / 16; ++cc) {
+                const int j0 = cq * SC + cc * 16;
+                uint32_t rk[16], ri[16], rv[16];
                 tc::ld16_nowait(lane_base + S::COL_DK + j0, rk);
-                tc::ld16_nowait(lane_base + S::COL_DK + j0 + 16, rk + 16);
                 tc::ld16_nowait(lane_base + S::COL_DV + j0, rv);
-                tc::ld16_nowait(lane_base + S::COL_DV + j0 + 16, rv + 16);
-                if (have_g) {
-                    tc::ld16_nowait(lane_base + S::COL_DKI + j0, ri);
-                    tc::ld16_nowait(lane_base + S::COL_DKI + j0 + 16, ri + 16);
-                }
+                if (have_g) tc::ld16_nowait(lane_base + S::COL_DKI + j0, ri);
                 tc::ld_wait();
+                float vk[16], vv[16];
 #pragma unroll
-                for (int hh = 0; hh < 32; hh += 16) {
-                    float vk[16], vv[16];
-#pragma unroll
-                    for (int x = 0; x < 16; ++x) {
-                        vk[x] = have_g ? fmaf(w_out, __uint_as_float(ri[hh + x]), __uint_as_float(rk[hh + x]))
-                                       : __uint_as_float(rk[hh + x]);
-                        vv[x] = __uint_as_float(rv[hh + x]);
-                    }
-                    stage_f32x16(smem, dk_chunk, r, j0 + hh, vk);
-                    stage_f32x16(smem, dv_chunk, r, j0 + hh, vv);
+                for (int x = 0; x < 16; ++x) {
+                    vk[x] = have_g ? fmaf(w_out, __uint_as_float(ri[x]), __uint_as_float(rk[x])) : __uint_as_float(rk[x]);
+                    vv[x] = __uint_as_float(rv[x]);
                 }
+                stage_f32x16(smem, dk_chunk, r, j0, vk);
+                stage_f32x16(smem, dv_chunk, r, j0, vv);
             }
         }
         tc::fence_smem_to_async();
@@ -1423,7 +1416,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             float iv = 0.f;
             if (!tile_start) {
 #pragma unroll
-                for (int w2 = 0; w2 < 8; ++w2) iv += st_iv[w2];
+                for (int w2 = 0; w2 < kRThreads / 32; ++w2) iv += st_iv[w2];
                 iv *= mc.a;
             }
             const bool in = t >= r_lo && t < r_hi;
@@ -1434,7 +1427,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             // per-head mode: fixed-order tile total
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1) dl += __shfl_xor_sync(0xffffffffu, dl, off);
-            if (lane == 0) st_iv[8 + warp] = dl;
+            if (lane == 0) st_iv[16 + warp] = dl;
         }
         LA_MARK(5);
         tc::fence_smem_to_async();  // the statistics in the V tile are overwritten by the next tile's load
@@ -1447,7 +1440,7 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
         }
         tc::fence_after();
         LA_MARK(6);
-        if (tid == 0) gsum += (st_iv[8] + st_iv[9]) + (st_iv[10] + st_iv[11]);
+        if (tid == 0) gsum += (st_iv[16] + st_iv[17]) + (st_iv[18] + st_iv[19]);
         have_g = true;
         // Q, K, V and dY are free (B3 is done, the staged stores are read): the next tile's
         // loads go out now, while G becomes the next tile's bf16 operand
@@ -1462,11 +1455,11 @@ __global__ void __launch_bounds__(kThreads, 1) bwd_kernel(const __grid_constant_
             const bool write_ds0 = last && seg_lo == 0 && p.dS0 != nullptr;
             uint32_t gv[SC];
 #pragma unroll
-            for (int cc = 0; cc < SC / 16; ++cc) tc::ld16_nowait(lane_base + S::COL_G + half * SC + cc * 16, gv + cc * 16);
+            for (int cc = 0; cc < SC / 16; ++cc) tc::ld16_nowait(lane_base + S::COL_G + cq * SC + cc * 16, gv + cc * 16);
             tc::ld_wait();
 #pragma unroll
             for (int cc = 0; cc < SC / 16; ++cc) {
-                const int j0 = half * SC + cc * 16;
+                const int j0 = cq * SC + cc * 16;
                 float v[16];
 #pragma unroll
                 for (int x = 0; x < 16; ++x) v[x] = __uint_as_float(gv[cc * 16 + x]);
@@ -1828,7 +1821,7 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     r.trace = la_trace_buffer();
 #endif
     if (set_smem(bwd_kernel<D>, BwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    bwd_kernel<D><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, BwdSmem<D>::BYTES, stream>>>(r);
+    bwd_kernel<D><<<static_cast<unsigned>(a.B * a.H * pl.G), kRThreads, BwdSmem<D>::BYTES, stream>>>(r);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     if (r.gpart != nullptr) {
         dgamma_head_kernel<<<static_cast<unsigned>((a.H + 127) / 128), 128, 0, stream>>>(gpart, a.gamma, a.dgamma,
