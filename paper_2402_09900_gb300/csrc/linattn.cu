@@ -1027,6 +1027,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     uint64_t* bar3 = bar1 + 2;
     uint64_t* full = bar1 + 3;
     uint32_t* tslot = reinterpret_cast<uint32_t*>(bar1 + 4);
+    uint64_t* bar4 = bar1 + 5;  // V G^T of B1, committed apart from P and dP
     const TileMeta& mc = *reinterpret_cast<const TileMeta*>(smem + S::OFF_META);
     const uint32_t sbase = smem_addr(smem);
     const uint32_t sQ = sbase + S::OFF_Q, sK = sbase + S::OFF_K, sV = sbase + S::OFF_V, sDY = sbase + S::OFF_DY;
@@ -1055,6 +1056,21 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         bulk_g2s(smem + S::OFF_META, p.meta + bh * p.n_tiles + tile, sizeof(TileMeta), full);
         if (with_state) bulk_g2s(smem + S::OFF_SS, p.states + (bh * p.n_tiles + tile) * D * D, kStateBytes, full);
     };
+    // the same loads in two groups for every later tile: Q, V, dY and the metadata
+    // as soon as B3 is done, K and the state once the staged output stores (in
+    // K, G, Pm and dPm) have been read
+    auto issue_tile_a = [&](int64_t tile) {
+        mbar_arrive_expect_tx(full, 4 * S::TILE + sizeof(TileMeta) + D * D * 2);
+        const int64_t t0 = tile * T;
+        tma_tile<D>(sQ, &p.map_q, h, t0, b, full);
+        tma_tile<D>(sV, &p.map_v, h, t0, b, full);
+        tma_tile<D>(sDY, &p.map_dy, h, t0, b, full);
+        bulk_g2s(smem + S::OFF_META, p.meta + bh * p.n_tiles + tile, sizeof(TileMeta), full);
+    };
+    auto issue_tile_b = [&](int64_t tile) {
+        tma_tile<D>(sK, &p.map_k, h, tile * T, b, full);
+        bulk_g2s(smem + S::OFF_SS, p.states + (bh * p.n_tiles + tile) * D * D, D * D * 2, full);
+    };
     bool have_g = seg_hi == p.L && p.dS_last != nullptr;  // a reverse state enters the current tile
 
     if (tid == 0) {
@@ -1062,6 +1078,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         mbar_init(bar2, 1);
         mbar_init(bar3, 1);
         mbar_init(full, 1);
+        mbar_init(bar4, 1);
         fence_mbar_init();
         prefetch_tensormap(&p.map_q);
         prefetch_tensormap(&p.map_k);
@@ -1116,6 +1133,8 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     bool failed = false;
     bool pending = true;  // a tile load may be in flight
     uint64_t* drain = nullptr;  // a batch issued but not seen complete
+    uint32_t drain_par = 0;
+    uint32_t ph4 = 0;           // phase of bar4 (committed only on tiles with a reverse state)
     int it = 0;
 #ifdef MEMOROID_LA_TRACE
     const bool trace_on = blockIdx.x == 0 && tid == 0 && p.trace != nullptr;
@@ -1147,12 +1166,13 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk)
                 tc::mma(tm + S::COL_DP, desc_sw_k(sDY, kk), desc_sw_k(sV, kk), ID_SCORE, kk > 0);
+            tc::commit(bar1);
             if (have_g) {
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk)
                     tc::mma(tm + S::COL_DKI, desc_sw_k(sV, kk), desc_kmajor(sGB, D, kk), ID_VG, kk > 0);
+                tc::commit(bar4);
             }
-            tc::commit(bar1);
         }
         // while B1 runs (it reads G only through its bf16 copy): this thread's row
         // of <G_c, S_{c-1}> and G *= a_c in tensor memory; pass F's dgamma term
@@ -1199,7 +1219,8 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         ok = wait_mbar(bar1, it & 1, p.wait_ns) && !(it == 0 && static_cast<int64_t>(blockIdx.x) == p.fail_cta);
         if (__syncthreads_or(!ok)) {
             failed = true;
-            drain = bar1;
+            drain = have_g ? bar4 : bar1;  // bar4 completes after every batch before it
+            drain_par = have_g ? ph4 : (it & 1);
             break;
         }
         tc::fence_after();
@@ -1240,9 +1261,11 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
             st_col[quarter * T + r0 + lane] = cs;
             st_row[cq * T + t] = rsum;
 
-            // x_r = w_out_r k_r . (G_c v_r), from the unscaled K tile
+            // x_r = w_out_r k_r . (G_c v_r), from the unscaled K tile, once V G^T is done
             float xacc = 0.f;
             if (have_g) {
+                ok = wait_mbar(bar4, ph4, p.wait_ns);
+                tc::fence_after();
                 const unsigned char* kt = smem + S::OFF_K;
                 uint32_t gi[SC];  // this thread's quarter row of V G^T, all loads in flight at once
 #pragma unroll
@@ -1268,7 +1291,13 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
             st_x[cq * T + t] = xacc;
         }
         if (lane == 0) st_iv[warp] = ivp;
-        __syncthreads();  // every x_r has read the unscaled K
+        if (__syncthreads_or(!ok)) {  // every x_r has read the unscaled K
+            failed = true;
+            drain = bar4;
+            drain_par = ph4;
+            break;
+        }
+        if (have_g) ph4 ^= 1;
         {
             // K~ = w_out (.) K in place (K is not read unscaled after this)
             const float lend = mc.lam2[T - 1];
@@ -1337,6 +1366,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         if (__syncthreads_or(!ok)) {
             failed = true;
             drain = bar2;
+            drain_par = it & 1;
             break;
         }
         tc::fence_after();
@@ -1432,22 +1462,29 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         LA_MARK(5);
         tc::fence_smem_to_async();  // the statistics in the V tile are overwritten by the next tile's load
         ok = wait_mbar(bar3, it & 1, p.wait_ns);
-        if (tid == 0) bulk_wait_read();  // dv staging in G / K and dk staging are read before reuse
         if (__syncthreads_or(!ok)) {
             failed = true;
             drain = bar3;
+            drain_par = it & 1;
             break;
         }
         tc::fence_after();
         LA_MARK(6);
-        if (tid == 0) gsum += (st_iv[16] + st_iv[17]) + (st_iv[18] + st_iv[19]);
-        have_g = true;
-        // Q, K, V and dY are free (B3 is done, the staged stores are read): the next tile's
-        // loads go out now, while G becomes the next tile's bf16 operand
-        if (tile > tile_lo) {
-            if (tid == 0) issue_tile(tile - 1, true);
-            pending = true;
+        const bool next = tile > tile_lo;
+        if (tid == 0) {
+            gsum += (st_iv[16] + st_iv[17]) + (st_iv[18] + st_iv[19]);
+            // Q, V, dY and the metadata are free (B3 is done, the statistics are read):
+            // their loads go out while the staged dk / dv stores drain
+            if (next) {
+                tc::fence_smem_to_async();
+                issue_tile_a(tile - 1);
+            }
+            bulk_wait_read();  // dv staging in G / K and dk staging in Pm / dPm are read
         }
+        if (next) pending = true;
+        have_g = true;
+        __syncthreads();
+        if (next && tid == 0) issue_tile_b(tile - 1);
 
         // ---- G_{c-1} -> bf16 operand for the next tile (and dS0 at the tape start) ----
         {
@@ -1486,7 +1523,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     if (failed) {
         if (tid == 0) record_error(p.hdr, DEV_MMA_TIMEOUT);
         // let work still in flight finish before the CTA's TMEM and shared memory go away
-        if (drain != nullptr) wait_mbar(drain, it & 1, kDrainNs);
+        if (drain != nullptr) wait_mbar(drain, drain_par, kDrainNs);
         if (pending) wait_mbar(full, it & 1, kDrainNs);
     }
     if (tid == 0) bulk_wait_all();
