@@ -332,20 +332,24 @@ template <int D>
 struct FwdSmem {
     static constexpr int TILE = T * D * 2;
     static constexpr int PM = T * T * 2;
-    static constexpr bool PM_IN_Q = TILE >= PM;  // d = 128: the masked scores overwrite Q
     static constexpr int STAGE = 3 * TILE;       // Q, K, V
-    static constexpr int OFF_PM = PM_IN_Q ? 0 : 2 * STAGE;
-    static constexpr int OFF_SB = 2 * STAGE + (PM_IN_Q ? 0 : PM);
+    static constexpr int OFF_SB = 2 * STAGE;     // bf16 state operand of the inter-tile term
+    // d = 128: the masked scores live in the state operand's buffer, free from the
+    // end of the first contractions to the epilogue, which writes the next state
+    static constexpr bool PM_IN_SB = D * D * 2 >= PM;
+    static constexpr int OFF_PM = PM_IN_SB ? OFF_SB : OFF_SB + D * D * 2;
     static constexpr int NMETA = 3;  // metadata ring: tiles c, c+1 in use, c+2 loading
-    static constexpr int OFF_META = OFF_SB + D * D * 2;
+    static constexpr int OFF_META = PM_IN_SB ? OFF_SB + D * D * 2 : OFF_PM + PM;
     static constexpr int OFF_Z = OFF_META + NMETA * static_cast<int>(sizeof(TileMeta));  // [2][T] fp32 (pass F)
     static constexpr int OFF_BAR = OFF_Z + 2 * T * 4;
     static constexpr int BYTES = OFF_BAR + 64;
-    // the fp32 output tile is staged in the finished stage in the 128-byte
-    // swizzled layout of its TMA store (32 channels per 128-byte row, chunk
-    // of 32 channels at m * T * 128)
-    static_assert(T * D * 4 <= 2 * TILE, "output staging fits in the Q and K slots of one stage");
-    static_assert(D * D * 2 <= TILE, "pass F's stored state is staged in the V slot of the same stage");
+    // the fp32 output tile is staged in the K and V slots of the finished stage
+    // in the 128-byte swizzled layout of its TMA store (32 channels per 128-byte
+    // row, chunk of 32 channels at m * T * 128); pass F loads the q tile into the
+    // Q slot once the first contractions are done and then stages its stored state there
+    static constexpr int OFF_Y = TILE;
+    static_assert(T * D * 4 <= 2 * TILE, "output staging fits in the K and V slots of one stage");
+    static_assert(D * D * 2 <= TILE, "pass F's stored state is staged in the Q slot of the same stage");
     // TMEM columns: scores P, intra output, inter output, state S
     static constexpr uint32_t COL_P = 0, COL_YA = 128, COL_YI = 128 + D, COL_S = 128 + 2 * D;
     static constexpr uint32_t TMEM_COLS = 512;
@@ -355,6 +359,7 @@ struct FwdSmem {
 struct FwdParams {
     CUtensorMap map_q, map_k, map_v;  // the q, k, v operands (4-D {D, H, L, B}, box {64, 1, 128, 1})
     CUtensorMap map_y;                // the fp32 output (4-D {D, H, L, B}, box {32, 1, 128, 1})
+    CUtensorMap map_zq;               // pass F: q for the z term (as map_q)
     const uint16_t* q;
     const uint16_t* k;
     const uint16_t* v;
@@ -369,7 +374,6 @@ struct FwdParams {
     uint64_t wait_ns;
     int64_t fail_cta;  // test knob: this CTA reports its first tensor-core wait as timed out (-1: none)
     // backward pass F only (see fwd_kernel<D, true>)
-    const uint16_t* zq;  // q, bf16 [B, L, H, D]
     float* dlam_f;       // [B, L, H]: the state-side terms of dL/dlog(gamma_t)
     uint16_t* states;    // [B, H, n_tiles, D, D] bf16: S_{c-1}^T before tiles without a begin flag
 #ifdef MEMOROID_LA_TRACE
@@ -483,6 +487,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     uint64_t* bar2 = bar1 + 1;
     uint64_t* full = bar1 + 2;  // [2]: stage s loaded
     uint32_t* tslot = reinterpret_cast<uint32_t*>(bar1 + 4);
+    uint64_t* qbar = bar1 + 5;  // pass F: the q tile of the z term
     TileMeta* metas = reinterpret_cast<TileMeta*>(smem + S::OFF_META);
     const uint32_t sbase = smem_addr(smem);
     const uint32_t sSb = sbase + S::OFF_SB;
@@ -491,7 +496,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     auto stage_q = [&](int s) { return sbase + s * S::STAGE; };
     auto stage_k = [&](int s) { return sbase + s * S::STAGE + S::TILE; };
     auto stage_v = [&](int s) { return sbase + s * S::STAGE + 2 * S::TILE; };
-    auto stage_pm = [&](int s) { return S::PM_IN_Q ? stage_q(s) : sbase + S::OFF_PM; };
+    const uint32_t sPm = sbase + S::OFF_PM;
     // thread 0: TMA loads of tile c into stage s and of metadata tiles m0 (and
     // m1 >= 0) into their ring slots, all completing on full[s]
     auto issue_tile = [&](int c, int s, int m0, int m1) {
@@ -510,11 +515,13 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         mbar_init(bar2, 1);
         mbar_init(&full[0], 1);
         mbar_init(&full[1], 1);
+        mbar_init(qbar, 1);
         fence_mbar_init();
         prefetch_tensormap(&p.map_q);
         prefetch_tensormap(&p.map_k);
         prefetch_tensormap(&p.map_v);
         prefetch_tensormap(&p.map_y);
+        if (BWD) prefetch_tensormap(&p.map_zq);
     }
     if (warp == 0) tc::alloc(tslot, S::TMEM_COLS);
     tc::fence_before();
@@ -587,6 +594,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     int pending = 0;       // the last issued tile whose load may still be in flight (-1: none)
     int drain_bar = 0;     // 1 / 2: the batch on bar1 / bar2 was issued but not seen complete
     uint32_t drain_par = 0;
+    bool q_pending = false;  // pass F: a q tile load not seen complete
+    uint32_t q_par = 0;
 #ifdef MEMOROID_LA_TRACE
     const bool trace_on = blockIdx.x == 0 && tid == 0 && p.trace != nullptr;
     unsigned long long tr[8] = {0, 0, 0, 0, 0, 0, 0, 0};
@@ -596,12 +605,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     for (int c = 0; c < nt && !failed; ++c) {
         const int s = c & 1;
         const TileMeta& mc = metas[c % S::NMETA];
-        if (BWD && have_prev) {
-            // pass F reads q_t for the z term in the epilogue: bring this thread's part of the row into L2
-            const int t = 32 * quarter + lane;
-            const int64_t tt = (tile0 + c) * T + t;
-            if (mc.seg[t] < 0 && tt < p.L) prefetch_l2(p.zq + ((b * p.L + tt) * p.H + h) * D + half * SC);
-        }
         // tile c's loads (issued during the previous tile) are complete
         bool ok = wait_mbar(&full[s], (c >> 1) & 1, p.wait_ns);
         tc::fence_smem_to_async();
@@ -636,6 +639,16 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             break;
         }
         tc::fence_after();
+        // pass F: the Q slot (dy) is free once the first contractions are done; the
+        // q tile of the z term goes there
+        const bool zload = BWD && have_prev;
+        if (zload) {
+            if (tid == 0) {
+                mbar_arrive_expect_tx(qbar, S::TILE);
+                tma_tile<D>(stage_q(s), &p.map_zq, h, (tile0 + c) * T, b, qbar);
+            }
+            q_pending = true;
+        }
         LA_MARK(2);
 
         // ---- mask: Pm[t][r] = [seg_t <= r <= t] exp2(lam2_t - lam2_r) P[t][r] ----
@@ -643,7 +656,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             const int t = 32 * quarter + lane;
             const float lt = mc.lam2[t];
             const int st = mc.seg[t];
-            unsigned char* pm = smem + (stage_pm(s) - sbase);
+            unsigned char* pm = smem + S::OFF_PM;
             uint32_t raw[64];
 #pragma unroll
             for (int cc = 0; cc < 4; ++cc) tc::ld16_nowait(lane_base + S::COL_P + half * 64 + cc * 16, raw + cc * 16);
@@ -684,7 +697,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
 
         // ---- Y_intra = Pm V and S = a S + K~^T V ----
         if (tid == 0) {
-            const uint32_t spm = stage_pm(s), sk = stage_k(s), sv = stage_v(s);
+            const uint32_t spm = sPm, sk = stage_k(s), sv = stage_v(s);
 #pragma unroll
             for (int kk = 0; kk < T / 16; ++kk)
                 tc::mma(tm + S::COL_YA, desc_kmajor(spm, T, kk), desc_sw_mn(sv, kk), ID_PV, kk > 0);
@@ -696,14 +709,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         }
         LA_MARK(4);
         const int64_t t0 = (tile0 + c) * T;
-        // pass F: this thread's part of q_t for the z term, in flight while the contractions run
-        uint4 qv[BWD ? SC / 8 : 1];
-        const bool zrow = BWD && have_prev && mc.seg[32 * quarter + lane] < 0 && t0 + 32 * quarter + lane < p.L;
-        if (zrow) {
-            const uint16_t* qrow = p.zq + ((b * p.L + t0 + 32 * quarter + lane) * p.H + h) * D + half * SC;
-#pragma unroll
-            for (int x = 0; x < SC / 8; ++x) qv[x] = *reinterpret_cast<const uint4*>(qrow + 8 * x);
-        }
         ok = wait_mbar(bar2, c & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
             failed = true;
@@ -712,6 +717,15 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             break;
         }
         tc::fence_after();
+        if (zload) {
+            ok = wait_mbar(qbar, q_par, p.wait_ns);
+            if (__syncthreads_or(!ok)) {
+                failed = true;
+                break;
+            }
+            q_pending = false;
+            q_par ^= 1;
+        }
         LA_MARK(5);
 
         // ---- y = Y_intra + w_in * Y_inter, staged as fp32 rows in stage s ----
@@ -721,7 +735,9 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         {
             const int t = 32 * quarter + lane;
             const float w_in = (have_prev && mc.seg[t] < 0) ? fast_exp2(mc.lam2[t]) : 0.f;
-            unsigned char* yst = smem + s * S::STAGE + t * 128;  // row t of chunk 0
+            unsigned char* yst = smem + s * S::STAGE + S::OFF_Y + t * 128;  // row t of chunk 0
+            const unsigned char* qs = smem + (stage_q(s) - sbase);  // pass F: the q tile
+            const bool zrow = zload && w_in != 0.f;
             // BWD: z_t = w_in_t q_t . (S_{c-1} dy_t), the inter output dotted with q
             float zacc = 0.f;
 #pragma unroll
@@ -751,7 +767,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 if (zrow) {
 #pragma unroll
                     for (int x = 0; x < 32; x += 8) {
-                        const uint4 u = qv[cc * 4 + x / 8];
+                        const uint4 u = *reinterpret_cast<const uint4*>(qs + sw_off(t, j0 + x));
                         const float2 q0 = unpack_bf16x2(u.x), q1 = unpack_bf16x2(u.y), q2 = unpack_bf16x2(u.z),
                                      q3 = unpack_bf16x2(u.w);
                         zacc = fmaf(q0.x, __uint_as_float(yi[x]), zacc);
@@ -767,6 +783,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             }
             if (BWD) reinterpret_cast<float*>(smem + S::OFF_Z)[half * T + t] = w_in * zacc;
         }
+        if (BWD) __syncthreads();  // every z term has read the q tile, where the state is staged next
         // ---- state: bf16 copy for the next tile, decay by the next tile's a ----
         if (c + 1 < nt) {
             const TileMeta& mn = metas[(c + 1) % S::NMETA];
@@ -786,9 +803,9 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                     store_bf16x16(smem + S::OFF_SB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
                     store_bf16x16(smem + S::OFF_SB, core_off(srow, j0 + 16, D), core_off(srow, j0 + 24, D), v + 16);
                     if (BWD && mn.has_start == 0) {
-                        // staged in this stage's V slot (free once the tile's contractions are
-                        // done) and bulk-stored with the output rows
-                        unsigned char* img = smem + (stage_v(s) - sbase);
+                        // staged in this stage's Q slot (the z term has read q) and
+                        // bulk-stored with the output rows
+                        unsigned char* img = smem + (stage_q(s) - sbase);
                         store_state_row<D>(img, srow, j0, v);
                         store_state_row<D>(img, srow, j0 + 16, v + 16);
                     }
@@ -827,13 +844,13 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 if (lane == 0) {
 #pragma unroll
                     for (int m = 0; m < D / 32; ++m)
-                        tma_store_4d(&p.map_y, sbase + s * S::STAGE + m * T * 128, 32 * m, static_cast<int>(h),
+                        tma_store_4d(&p.map_y, sbase + s * S::STAGE + S::OFF_Y + m * T * 128, 32 * m, static_cast<int>(h),
                                      static_cast<int>(t0), static_cast<int>(b));
                 }
             } else {
                 // a tile shared with a neighbouring segment: only this segment's rows, 16 bytes at a time
                 float* ybase = p.y + ((b * p.L + t0) * p.H + h) * D;
-                const unsigned char* st = smem + s * S::STAGE;
+                const unsigned char* st = smem + s * S::STAGE + S::OFF_Y;
                 for (int e = lane; e < (r_hi - r_lo) * (D / 4); e += 32) {
                     const int r = r_lo + e / (D / 4), j = (e % (D / 4)) * 4;
                     const float4 v = *reinterpret_cast<const float4*>(st + (j >> 5) * (T * 128) + r * 128 +
@@ -842,7 +859,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 }
             }
             if (BWD && lane == 0 && c + 1 < nt && metas[(c + 1) % S::NMETA].has_start == 0)
-                bulk_s2g(state_image<D>(p.states, bh, p.n_tiles, tile0 + c + 1), stage_v(s), D * D * 2);
+                bulk_s2g(state_image<D>(p.states, bh, p.n_tiles, tile0 + c + 1), stage_q(s), D * D * 2);
             bulk_commit();
         }
         if (BWD && warp == 1) {
@@ -876,6 +893,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         if (drain_bar == 1) wait_mbar(bar1, drain_par, kDrainNs);
         if (drain_bar == 2) wait_mbar(bar2, drain_par, kDrainNs);
         if (pending >= 0) wait_mbar(&full[pending & 1], (pending >> 1) & 1, kDrainNs);
+        if (q_pending) wait_mbar(qbar, q_par, kDrainNs);
     }
     if (warp == 0) bulk_wait_all();
 #ifdef MEMOROID_LA_TRACE
@@ -1763,7 +1781,7 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     p.G = static_cast<int>(pl.G);
     p.wait_ns = debug_knobs().wait_ns;
     p.fail_cta = debug_knobs().withhold_ticket;
-    p.zq = nullptr;
+    p.map_zq = p.map_q;  // not read by the forward
     p.dlam_f = nullptr;
     p.states = nullptr;
 #ifdef MEMOROID_LA_TRACE
@@ -1795,7 +1813,8 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     // pass F: dq = S dy, with (q, k, v) -> (dy, v, k)
     FwdParams f;
     if (!tile_map(&f.map_q, dy16, a.B, a.L, a.H, D) || !tile_map(&f.map_k, a.v, a.B, a.L, a.H, D) ||
-        !tile_map(&f.map_v, a.k, a.B, a.L, a.H, D) || !tile_map_y(&f.map_y, a.dq, a.B, a.L, a.H, D))
+        !tile_map(&f.map_v, a.k, a.B, a.L, a.H, D) || !tile_map_y(&f.map_y, a.dq, a.B, a.L, a.H, D) ||
+        !tile_map(&f.map_zq, a.q, a.B, a.L, a.H, D))
         return MEMOROID_ERR_CUDA;
     f.q = dy16;
     f.k = static_cast<const uint16_t*>(a.v);
@@ -1814,7 +1833,6 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     f.G = static_cast<int>(pl.G);
     f.wait_ns = debug_knobs().wait_ns;
     f.fail_cta = debug_knobs().withhold_ticket;
-    f.zq = static_cast<const uint16_t*>(a.q);
     f.dlam_f = dlam_f;
     f.states = states;
 #ifdef MEMOROID_LA_TRACE
