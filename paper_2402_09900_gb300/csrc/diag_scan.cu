@@ -874,11 +874,16 @@ __global__ void __launch_bounds__(CARRY_WARPS * 32) segment_carry_kernel(const P
 
 // Adds the state entering its segment to the outputs of a tile that the
 // scan computed from the identity, up to the tile's first begin flag: the
-// warps walk the list of such tiles the scan wrote (each tile touches only
+// CTAs walk the list of such tiles the scan wrote (each tile touches only
 // its own rows, so the list's order does not matter).  The rows to fix are
-// counted first, so their loads can be issued in batches.
+// counted first, so their loads can be issued in batches.  With a
+// per-channel lambda the rows are split over `nparts` warps: part w starts
+// from the carry times m^k (m = lambda, or conj(lambda) in reverse; k = the
+// rows before the part, by repeated squaring) and leaves its grad_lambda
+// partial in gl_out[w] for a fixed-order sum; with a per-step lambda one
+// warp takes the whole tile (nparts = 1).
 template <class C>
-__device__ void segment_fix_tile(const Params& p, int64_t tid) {
+__device__ void segment_fix_tile(const Params& p, int64_t tid, int part, int nparts, float4* gl_out) {
     constexpr int BATCH = 8;
     const int lane = threadIdx.x & 31;
     const int64_t chain = tid / p.n_tt, jt = tid - chain * p.n_tt;
@@ -909,17 +914,26 @@ __device__ void segment_fix_tile(const Params& p, int64_t tid) {
     }
     // lanes of the slab (FFM: the butterfly over a row's lanes uses this mask;
     // a row's lanes are all in the slab or all past it)
-    const unsigned act = __ballot_sync(0xffffffffu, lane < lmin(SLAB / 2, p.D2 - c2));
-    if (lane >= lmin(SLAB / 2, p.D2 - c2)) return;
+    const bool active = lane < lmin(SLAB / 2, p.D2 - c2);
+    const unsigned act = __ballot_sync(0xffffffffu, active);
+    float4 gl = zero2();
+    if (!active) return;
     const int64_t col = c2 + lane;
     float4 corr = cmul2(p.pin[tid * 32 + lane], p.segc[(chain * p.n_seg + g) * 32 + lane]);
     const float4 lam = C::PS ? one2() : p.lambda[col];
-    float4 gl = zero2();
-    for (int k0 = 0; k0 < nfix; k0 += BATCH) {
+    const int per = (nfix + nparts - 1) / nparts;
+    const int k_lo = min(nfix, part * per), k_hi = min(nfix, k_lo + per);
+    if (k_lo > 0) {
+        // the rows before this part: every one multiplies the carry by m, except
+        // that in reverse the tape's last step (processed first) multiplies by 1
+        const int skip = (C::REV && t0 + nrows == p.L) ? 1 : 0;
+        corr = cmul2(cpow2(C::REV ? conj2(lam) : lam, k_lo - skip), corr);
+    }
+    for (int k0 = k_lo; k0 < k_hi; k0 += BATCH) {
         float4 v[BATCH], aux[BATCH];
 #pragma unroll
         for (int k = 0; k < BATCH; ++k) {
-            if (k0 + k < nfix) {
+            if (k0 + k < k_hi) {
                 const int64_t t = C::REV ? t0 + nrows - 1 - (k0 + k) : t0 + k0 + k;
                 if (!C::FFM) v[k] = p.out[(b * p.L + t) * p.D2 + col];
                 else if (!C::REV) v[k] = ffm_load_planar(p.out + (b * p.L + t) * p.D2, p.D2, col);
@@ -934,7 +948,7 @@ __device__ void segment_fix_tile(const Params& p, int64_t tid) {
         }
 #pragma unroll
         for (int k = 0; k < BATCH; ++k) {
-            if (k0 + k >= nfix) break;
+            if (k0 + k >= k_hi) break;
             const int64_t t = C::REV ? t0 + nrows - 1 - (k0 + k) : t0 + k0 + k;
             if (!C::REV) {
                 const float4 l = C::PS ? p.lambda[(b * p.L + t) * p.D2 + col] : lam;
@@ -973,16 +987,37 @@ __device__ void segment_fix_tile(const Params& p, int64_t tid) {
             }
         }
     }
-    if (C::REV && !C::PS) p.gpart[tid * 32 + lane] = add2(p.gpart[tid * 32 + lane], gl);
+    if (gl_out != nullptr) gl_out[part * 32 + lane] = gl;
+    else if (C::REV && !C::PS) p.gpart[tid * 32 + lane] = add2(p.gpart[tid * 32 + lane], gl);
 }
 
 template <class C>
 __global__ void __launch_bounds__(128) segment_fix_kernel(const Params p) {
     if (ptx::ld_relaxed(p.hdr) != 0u) return;
     const int64_t n_fix = static_cast<int64_t>(ptx::ld_relaxed(p.hdr + 4));
-    const int64_t nw = static_cast<int64_t>(gridDim.x) * 4;
-    for (int64_t f = static_cast<int64_t>(blockIdx.x) * 4 + (threadIdx.x >> 5); f < n_fix; f += nw)
-        segment_fix_tile<C>(p, static_cast<int64_t>(p.fix[f]));
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (C::PS) {
+        // per-step lambda: one warp per tile
+        const int64_t nw = static_cast<int64_t>(gridDim.x) * 4;
+        for (int64_t f = static_cast<int64_t>(blockIdx.x) * 4 + warp; f < n_fix; f += nw)
+            segment_fix_tile<C>(p, static_cast<int64_t>(p.fix[f]), 0, 1, nullptr);
+        return;
+    }
+    // per-channel lambda: the four warps of a CTA split a tile's rows
+    __shared__ float4 gl[4 * 32];
+    for (int64_t f = blockIdx.x; f < n_fix; f += gridDim.x) {
+        const int64_t tid = static_cast<int64_t>(p.fix[f]);
+        segment_fix_tile<C>(p, tid, warp, 4, C::REV ? gl : nullptr);
+        if (C::REV) {
+            __syncthreads();
+            const int64_t c2 = (tid / p.n_tt % p.n_slabs) * (SLAB / 2);
+            if (warp == 0 && lane < lmin(SLAB / 2, p.D2 - c2)) {
+                const float4 sum = add2(add2(gl[lane], gl[32 + lane]), add2(gl[64 + lane], gl[96 + lane]));
+                p.gpart[tid * 32 + lane] = add2(p.gpart[tid * 32 + lane], sum);
+            }
+            __syncthreads();
+        }
+    }
 }
 
 // ============================================================================
@@ -1247,7 +1282,8 @@ memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
     if (sg.G > 1) {
         segment_carry_kernel<<<static_cast<unsigned>(l.n_chains), CARRY_WARPS * 32, 0, s>>>(p, C::REV);
         const int64_t n_tiles = l.n_chains * l.n_tt;
-        const int64_t fix_ctas = lmin((n_tiles + 3) / 4, 152 * 8);  // the warps walk the list of tiles to fix
+        // the CTAs (per-channel lambda) or warps (per-step lambda) walk the list of tiles to fix
+        const int64_t fix_ctas = lmin(C::PS ? (n_tiles + 3) / 4 : n_tiles, 152 * 8);
         segment_fix_kernel<C><<<static_cast<unsigned>(fix_ctas), 128, 0, s>>>(p);
         if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     }
