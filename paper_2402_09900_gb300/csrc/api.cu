@@ -509,7 +509,7 @@ size_t memoroid_linattn_norm_workspace_bytes(int64_t B, int64_t L, int64_t H, in
 int memoroid_linattn_norm_kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t d, int backward,
                                            int with_dgamma_per_head, int with_states) {
     if (!lnorm_shape_ok(B, L, H, d)) return -1;
-    return lnorm::kernels_per_call(B, L, H, backward != 0, with_dgamma_per_head != 0, with_states != 0);
+    return lnorm::kernels_per_call(B, L, H, d, backward != 0, with_dgamma_per_head != 0, with_states != 0);
 }
 
 static memoroid_status_t lnorm_common(lnorm::Args& a, const float* gamma, int gamma_per_step, const uint8_t* start,

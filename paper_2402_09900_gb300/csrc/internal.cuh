@@ -130,6 +130,11 @@ struct Args {
     int64_t B, L, H, D;
     void* workspace;
     size_t workspace_bytes;
+    // forward only, norm = 1: the Linear Transformer with phi and its normalizer
+    // for 64-channel heads at D = 128 (q, k, v and y [B, L, H, 64]; S0 and
+    // S_last in the padded [B, H, 128, 128] layout; den [B, L, H] or null)
+    int norm = 0;
+    float* den = nullptr;
 };
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D);      // forward and backward
@@ -173,7 +178,8 @@ struct Args {
     void* workspace;
 };
 size_t workspace_bytes(int64_t B, int64_t L, int64_t H);
-int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_dgamma_per_head, int with_states);
+int kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t d, int backward, int with_dgamma_per_head,
+                     int with_states);
 memoroid_status_t launch(const Args& a, cudaStream_t s);
 }  // namespace lnorm
 

@@ -360,6 +360,7 @@ struct FwdParams {
     CUtensorMap map_q, map_k, map_v;  // the q, k, v operands (4-D {D, H, L, B}, box {64, 1, 128, 1})
     CUtensorMap map_y;                // the fp32 output (4-D {D, H, L, B}, box {32, 1, 128, 1})
     CUtensorMap map_zq;               // pass F: q for the z term (as map_q)
+    float* den;                       // normalised forward: the normalizer [B, L, H] (or null)
     const uint16_t* q;
     const uint16_t* k;
     const uint16_t* v;
@@ -458,9 +459,21 @@ __device__ __forceinline__ void store_bf16x16(unsigned char* base, uint32_t off0
 // (the term of dL/dlog(gamma_s) that pairs the incoming state with the tile's
 // outputs), and stores S'_{c-1} as bf16 for every tile without a begin flag,
 // for pass R.
-template <int D, bool BWD>
+template <int D, bool BWD, bool NORM = false>
 __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant__ FwdParams p) {
+    static_assert(!NORM || (D == 128 && !BWD), "the normalised forward runs the d = 128 forward");
     using S = FwdSmem<D>;
+    // NORM: the Linear Transformer with phi and its normalizer for heads of 64
+    // channels.  q, k, v are the unpadded [B, L, H, 64] tensors; each operand
+    // slot holds them in its first 64 channels (one TMA box), phi is applied to
+    // q and k in shared memory, the contractions over the q/k channels stop at
+    // 64, the second half of the K slot holds zeros and that of the V slot the
+    // columns [1, 1, 0, ...], so the 128-wide state is [[X, x, x], [0]] and
+    // column 64 of the output is the normalizer; the epilogue writes
+    // y = y'[:64] / y'[64] and the normalizer.
+    constexpr int KQ = NORM ? 64 : D;     // channels of the q/k contractions
+    constexpr int DOUT = NORM ? 64 : D;   // output channels
+    constexpr int Y_OFF = NORM ? 0 : S::OFF_Y;  // output staging: the Q slot (NORM) or the K and V slots
     extern __shared__ __align__(1024) unsigned char smem[];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int quarter = warp & 3, half = warp >> 2;
@@ -481,7 +494,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     }
     const int64_t tile0 = seg_lo / T;
     const int nt = static_cast<int>((seg_hi + T - 1) / T - tile0);
-    const int64_t row_stride = p.H * D;  // elements between consecutive steps of one head
+    const int64_t row_stride = p.H * DOUT;  // output elements between consecutive steps of one head
 
     uint64_t* bar1 = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
     uint64_t* bar2 = bar1 + 1;
@@ -501,11 +514,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     // m1 >= 0) into their ring slots, all completing on full[s]
     auto issue_tile = [&](int c, int s, int m0, int m1) {
         const uint32_t meta_bytes = (m0 >= 0 ? sizeof(TileMeta) : 0) + (m1 >= 0 ? sizeof(TileMeta) : 0);
-        mbar_arrive_expect_tx(&full[s], 3 * S::TILE + meta_bytes);
+        mbar_arrive_expect_tx(&full[s], 3 * (T * KQ * 2) + meta_bytes);
         const int64_t t0 = (tile0 + c) * T;
-        tma_tile<D>(stage_q(s), &p.map_q, h, t0, b, &full[s]);
-        tma_tile<D>(stage_k(s), &p.map_k, h, t0, b, &full[s]);
-        tma_tile<D>(stage_v(s), &p.map_v, h, t0, b, &full[s]);
+        tma_tile<KQ>(stage_q(s), &p.map_q, h, t0, b, &full[s]);
+        tma_tile<KQ>(stage_k(s), &p.map_k, h, t0, b, &full[s]);
+        tma_tile<KQ>(stage_v(s), &p.map_v, h, t0, b, &full[s]);
         if (m0 >= 0) bulk_g2s(&metas[m0 % S::NMETA], gmeta + m0, sizeof(TileMeta), &full[s]);
         if (m1 >= 0) bulk_g2s(&metas[m1 % S::NMETA], gmeta + m1, sizeof(TileMeta), &full[s]);
     };
@@ -524,6 +537,19 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         if (BWD) prefetch_tensormap(&p.map_zq);
     }
     if (warp == 0) tc::alloc(tslot, S::TMEM_COLS);
+    if (NORM) {
+        // the constant second halves of the K slots (zeros) and V slots ([1, 1, 0, ...]
+        // per row) of both stages; the loads only ever write the first halves
+        for (int i = tid; i < 2 * T * 8; i += kThreads) {
+            const int st = i / (T * 8), r = (i / 8) % T, u = i % 8;
+            unsigned char* kc = smem + st * S::STAGE + S::TILE + T * 128 + r * 128 + u * 16;
+            unsigned char* vc = smem + st * S::STAGE + 2 * S::TILE + T * 128 + r * 128 + u * 16;
+            *reinterpret_cast<uint4*>(kc) = make_uint4(0u, 0u, 0u, 0u);
+            // unit u of row r holds channels 8 (u ^ (r % 8)) .. + 7 of the half
+            const uint32_t ones = pack_bf16x2(1.f, 1.f);
+            *reinterpret_cast<uint4*>(vc) = make_uint4((u ^ (r & 7)) == 0 ? ones : 0u, 0u, 0u, 0u);
+        }
+    }
     tc::fence_before();
     __syncthreads();
     tc::fence_after();
@@ -616,17 +642,42 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         pending = -1;
         tc::fence_after();
         LA_MARK(0);
+        if (NORM) {
+            // phi(z) = 1 + ELU(z) on the loaded q and k, in place (bf16, round to
+            // nearest); rows past the tape end stay 0, as the padded operands would
+            const int64_t tb = (tile0 + c) * T;
+#pragma unroll
+            for (int i = 0; i < 2 * T * 8 / kThreads; ++i) {
+                const int unit = i * kThreads + tid;  // 16-byte units of the Q then the K half-tile
+                const int row = (unit % (T * 8)) / 8;
+                unsigned char* a = smem + s * S::STAGE + (unit >= T * 8 ? S::TILE : 0) + (unit % (T * 8)) * 16;
+                uint4 u = *reinterpret_cast<uint4*>(a);
+                uint32_t* w = reinterpret_cast<uint32_t*>(&u);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float2 f = unpack_bf16x2(w[e]);
+                    w[e] = tb + row < p.L
+                               ? pack_bf16x2(f.x > 0.f ? 1.f + f.x : __expf(f.x), f.y > 0.f ? 1.f + f.y : __expf(f.y))
+                               : 0u;
+                }
+                *reinterpret_cast<uint4*>(a) = u;
+            }
+            tc::fence_smem_to_async();
+            tc::fence_before();
+            __syncthreads();
+            tc::fence_after();
+        }
 
         // ---- P = Q K^T and (with an incoming state) Y_inter = Q S_prev ----
         if (tid == 0) {
             const uint32_t sq = stage_q(s), sk = stage_k(s);
             if (have_prev) {
 #pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk)
+                for (int kk = 0; kk < KQ / 16; ++kk)
                     tc::mma(tm + S::COL_YI, desc_sw_k(sq, kk), desc_mnmajor(sSb, D, kk), ID_QS, kk > 0);
             }
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk)
+            for (int kk = 0; kk < KQ / 16; ++kk)
                 tc::mma(tm + S::COL_P, desc_sw_k(sq, kk), desc_sw_k(sk, kk), ID_QK, kk > 0);
             tc::commit(bar1);
         }
@@ -732,10 +783,43 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         // rows of this tile that belong to the segment
         const int r_lo = static_cast<int>(max(static_cast<int64_t>(0), seg_lo - t0));
         const int r_hi = static_cast<int>(min(static_cast<int64_t>(T), seg_hi - t0));
-        {
+        if (NORM) {
+            // y = y'[:64] / y'[64]: every thread reads the normalizer (column 64) of
+            // its row and divides its 32 of the 64 output columns
             const int t = 32 * quarter + lane;
             const float w_in = (have_prev && mc.seg[t] < 0) ? fast_exp2(mc.lam2[t]) : 0.f;
-            unsigned char* yst = smem + s * S::STAGE + S::OFF_Y + t * 128;  // row t of chunk 0
+            const int j0 = half * 32;
+            uint32_t ya[32], yi[32], na[16], ni[16];
+            tc::ld16_nowait(lane_base + S::COL_YA + 64, na);
+            tc::ld16_nowait(lane_base + S::COL_YA + j0, ya);
+            tc::ld16_nowait(lane_base + S::COL_YA + j0 + 16, ya + 16);
+            if (have_prev) {
+                tc::ld16_nowait(lane_base + S::COL_YI + 64, ni);
+                tc::ld16_nowait(lane_base + S::COL_YI + j0, yi);
+                tc::ld16_nowait(lane_base + S::COL_YI + j0 + 16, yi + 16);
+            }
+            tc::ld_wait();
+            const float dn = have_prev ? fmaf(w_in, __uint_as_float(ni[0]), __uint_as_float(na[0])) : __uint_as_float(na[0]);
+            if (half == 0 && p.den != nullptr && t >= r_lo && t < r_hi) p.den[(b * p.L + t0 + t) * p.H + h] = dn;
+            const float inv = 1.f / dn;
+            unsigned char* yst = smem + s * S::STAGE + Y_OFF + t * 128;  // row t of chunk 0
+#pragma unroll
+            for (int x = 0; x < 32; x += 4) {
+                float o[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    o[e] = __uint_as_float(ya[x + e]);
+                    if (have_prev) o[e] = fmaf(w_in, __uint_as_float(yi[x + e]), o[e]);
+                    o[e] *= inv;
+                }
+                const int j = j0 + x;
+                *reinterpret_cast<float4*>(yst + (j >> 5) * (T * 128) + ((((j & 31) >> 2) ^ (t & 7)) << 4)) =
+                    make_float4(o[0], o[1], o[2], o[3]);
+            }
+        } else {
+            const int t = 32 * quarter + lane;
+            const float w_in = (have_prev && mc.seg[t] < 0) ? fast_exp2(mc.lam2[t]) : 0.f;
+            unsigned char* yst = smem + s * S::STAGE + Y_OFF + t * 128;  // row t of chunk 0
             const unsigned char* qs = smem + (stage_q(s) - sbase);  // pass F: the q tile
             const bool zrow = zload && w_in != 0.f;
             // BWD: z_t = w_in_t q_t . (S_{c-1} dy_t), the inter output dotted with q
@@ -843,16 +927,16 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 // whole tile: one TMA store per 32 channels (rows past L are clipped)
                 if (lane == 0) {
 #pragma unroll
-                    for (int m = 0; m < D / 32; ++m)
-                        tma_store_4d(&p.map_y, sbase + s * S::STAGE + S::OFF_Y + m * T * 128, 32 * m, static_cast<int>(h),
+                    for (int m = 0; m < DOUT / 32; ++m)
+                        tma_store_4d(&p.map_y, sbase + s * S::STAGE + Y_OFF + m * T * 128, 32 * m, static_cast<int>(h),
                                      static_cast<int>(t0), static_cast<int>(b));
                 }
             } else {
                 // a tile shared with a neighbouring segment: only this segment's rows, 16 bytes at a time
-                float* ybase = p.y + ((b * p.L + t0) * p.H + h) * D;
-                const unsigned char* st = smem + s * S::STAGE + S::OFF_Y;
-                for (int e = lane; e < (r_hi - r_lo) * (D / 4); e += 32) {
-                    const int r = r_lo + e / (D / 4), j = (e % (D / 4)) * 4;
+                float* ybase = p.y + ((b * p.L + t0) * p.H + h) * DOUT;
+                const unsigned char* st = smem + s * S::STAGE + Y_OFF;
+                for (int e = lane; e < (r_hi - r_lo) * (DOUT / 4); e += 32) {
+                    const int r = r_lo + e / (DOUT / 4), j = (e % (DOUT / 4)) * 4;
                     const float4 v = *reinterpret_cast<const float4*>(st + (j >> 5) * (T * 128) + r * 128 +
                                                                       ((((j & 31) >> 2) ^ (r & 7)) << 4));
                     *reinterpret_cast<float4*>(ybase + static_cast<int64_t>(r) * row_stride + j) = v;
@@ -1751,7 +1835,7 @@ memoroid_status_t launch_prep(const Args& a, const Plan& pl, TileMeta* meta, int
     return MEMOROID_OK;
 }
 
-template <int D>
+template <int D, bool NORM = false>
 memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, cudaStream_t stream) {
     unsigned char* ws = static_cast<unsigned char*>(a.workspace);
     TileMeta* meta = reinterpret_cast<TileMeta*>(ws + ly.meta);
@@ -1761,9 +1845,11 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     if (st != MEMOROID_OK) return st;
 
     FwdParams p;
-    if (!tile_map(&p.map_q, a.q, a.B, a.L, a.H, D) || !tile_map(&p.map_k, a.k, a.B, a.L, a.H, D) ||
-        !tile_map(&p.map_v, a.v, a.B, a.L, a.H, D) || !tile_map_y(&p.map_y, a.y, a.B, a.L, a.H, D))
+    constexpr int KQ = NORM ? 64 : D;  // channels of q, k, v (and of y) in memory
+    if (!tile_map(&p.map_q, a.q, a.B, a.L, a.H, KQ) || !tile_map(&p.map_k, a.k, a.B, a.L, a.H, KQ) ||
+        !tile_map(&p.map_v, a.v, a.B, a.L, a.H, KQ) || !tile_map_y(&p.map_y, a.y, a.B, a.L, a.H, KQ))
         return MEMOROID_ERR_CUDA;
+    p.den = NORM ? a.den : nullptr;
     p.q = static_cast<const uint16_t*>(a.q);
     p.k = static_cast<const uint16_t*>(a.k);
     p.v = static_cast<const uint16_t*>(a.v);
@@ -1787,8 +1873,8 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
 #ifdef MEMOROID_LA_TRACE
     p.trace = la_trace_buffer();
 #endif
-    if (set_smem(fwd_kernel<D, false>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    fwd_kernel<D, false><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(p);
+    if (set_smem(fwd_kernel<D, false, NORM>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    fwd_kernel<D, false, NORM><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     return MEMOROID_OK;
 }
@@ -1816,6 +1902,7 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
         !tile_map(&f.map_v, a.k, a.B, a.L, a.H, D) || !tile_map_y(&f.map_y, a.dq, a.B, a.L, a.H, D) ||
         !tile_map(&f.map_zq, a.q, a.B, a.L, a.H, D))
         return MEMOROID_ERR_CUDA;
+    f.den = nullptr;
     f.q = dy16;
     f.k = static_cast<const uint16_t*>(a.v);
     f.v = static_cast<const uint16_t*>(a.k);
@@ -1906,9 +1993,11 @@ memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream) {
 }
 
 memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream) {
+    if (a.norm && a.D != 128) return MEMOROID_ERR_UNSUPPORTED;
     if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, stream) != cudaSuccess) return MEMOROID_ERR_CUDA;
     const Plan pl = make_plan(a.B, a.L, a.H);
     const Layout ly = make_layout(a.B, a.L, a.H, a.D);
+    if (a.norm) return launch_fwd_d<128, true>(a, pl, ly, stream);
     if (a.D == 64) return launch_fwd_d<64>(a, pl, ly, stream);
     if (a.D == 128) return launch_fwd_d<128>(a, pl, ly, stream);
     return MEMOROID_ERR_UNSUPPORTED;

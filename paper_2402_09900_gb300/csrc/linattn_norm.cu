@@ -36,7 +36,10 @@ namespace {
 constexpr int kW = 128;  // width of the padded operands and states
 constexpr int kCtas = 152 * 8;
 
-__device__ __forceinline__ float phi(float z) { return z > 0.f ? 1.f + z : expf(z); }
+// phi(z) = 1 + ELU(z), rounded to bf16 right after, so the SFU exponential
+// (__expf, a few ulp of fp32) is exact enough; the fused forward of linattn.cu
+// computes the same expression
+__device__ __forceinline__ float phi(float z) { return z > 0.f ? 1.f + z : __expf(z); }
 __device__ __forceinline__ float dphi(float z) { return z > 0.f ? 1.f : expf(z); }
 
 struct Buffers {
@@ -243,21 +246,29 @@ unsigned grid_for(int64_t n, int per_thread = 1) {
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t H) { return total_bytes(B, L, H); }
 
-int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_dgamma_per_head, int with_states) {
+int kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t d, int backward, int with_dgamma_per_head,
+                     int with_states) {
     if (B == 0 || L == 0 || H == 0) return 0;
     // prep, the linear-attention call, then the divide (forward) or the upstream
-    // gradient and the chain rule (backward); with states: their padding and unpadding
-    const int base = 2 + (backward ? 1 : 0) + la::kernels_per_call(B, L, H, backward, with_dgamma_per_head);
+    // gradient and the chain rule (backward); with states: their padding and
+    // unpadding.  The forward of 64-channel heads (y 16-byte aligned) is the fused call alone.
+    const bool fused = !backward && d == 64;
+    const int base = (fused ? 0 : 2 + (backward ? 1 : 0)) + la::kernels_per_call(B, L, H, backward, with_dgamma_per_head);
     return base + (with_states ? (backward ? 3 : 2) : 0);
 }
 
 memoroid_status_t launch(const Args& a, cudaStream_t s) {
     const int64_t R = a.B * a.L * a.H, BH = a.B * a.H;
     const Buffers b = carve(a.workspace, a.B, a.L, a.H, a.backward);
-    prep_kernel<<<grid_for(R * 16), 256, 0, s>>>(static_cast<const uint4*>(a.q), static_cast<const uint4*>(a.k),
-                                                 static_cast<const uint4*>(a.v), R, static_cast<int>(a.d),
-                                                 reinterpret_cast<uint4*>(b.q), reinterpret_cast<uint4*>(b.k),
-                                                 reinterpret_cast<uint4*>(b.v));
+    // the forward of 64-channel heads applies phi, the padding and the division
+    // inside the tensor-core kernel (la::Args::norm); everything else goes
+    // through the padded operands
+    const bool fused = !a.backward && a.d == 64 && (reinterpret_cast<uintptr_t>(a.y) & 15u) == 0;  // y: TMA stores
+    if (!fused)
+        prep_kernel<<<grid_for(R * 16), 256, 0, s>>>(static_cast<const uint4*>(a.q), static_cast<const uint4*>(a.k),
+                                                     static_cast<const uint4*>(a.v), R, static_cast<int>(a.d),
+                                                     reinterpret_cast<uint4*>(b.q), reinterpret_cast<uint4*>(b.k),
+                                                     reinterpret_cast<uint4*>(b.v));
     // incoming state and (backward) outgoing-state gradient in the padded layout
     const bool s_in = a.S0 != nullptr || a.z0 != nullptr;
     const bool g_in = a.backward && (a.dS_last != nullptr || a.dz_last != nullptr);
@@ -282,12 +293,22 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
     l.workspace = b.la;
     l.workspace_bytes = b.la_bytes;
     if (!a.backward) {
-        l.y = b.y;
         l.S_last = (a.S_last != nullptr || a.z_last != nullptr) ? b.S1 : nullptr;
+        if (fused) {
+            l.q = a.q;
+            l.k = a.k;
+            l.v = a.v;
+            l.y = a.y;
+            l.den = a.den;
+            l.norm = 1;
+        } else {
+            l.y = b.y;
+        }
         const memoroid_status_t st = la::launch_fwd(l, s);
         if (st != MEMOROID_OK) return st;
-        divide_kernel<<<grid_for(R * 32), 256, 0, s>>>(reinterpret_cast<const float4*>(b.y), R, static_cast<int>(a.d),
-                                                       a.y, a.den);
+        if (!fused)
+            divide_kernel<<<grid_for(R * 32), 256, 0, s>>>(reinterpret_cast<const float4*>(b.y), R,
+                                                           static_cast<int>(a.d), a.y, a.den);
         if (l.S_last != nullptr)
             unpad_state_kernel<<<grid_for(BH * a.d * (a.d + 1)), 256, 0, s>>>(b.S1, BH, static_cast<int>(a.d), 0,
                                                                                a.S_last, a.z_last);

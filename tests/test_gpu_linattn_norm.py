@@ -166,3 +166,37 @@ def test_empty_tape_passes_the_state_through():
     y, den, Sl, zl = m.linattn_norm_fwd(q, q, q, g, st, dev(S0), dev(z0), ws=ws)
     torch.cuda.synchronize()
     assert np.array_equal(Sl.cpu().numpy(), S0) and np.array_equal(zl.cpu().numpy(), z0)
+
+
+@pytest.mark.parametrize("mode,with_states", [("step", True), ("head", False)])
+def test_fused_forward_matches_padded_path_bitwise(mode, with_states):
+    # 64-channel heads run the fused forward (phi, the padding and the division inside
+    # the tensor-core kernel) when y is 16-byte aligned; an output buffer one float off
+    # that alignment takes the padded-operand path.  Both compute the same bits: the
+    # fused contractions only leave out terms that are exactly zero.
+    m = _m()
+    B, L, H, d = 2, 1700, 2, 64
+    t = make(B, L, H, d, tapegen.seed_for(815), 200.0, mode, with_states)
+    ws = m.workspace(m.memoroid_linattn_norm_workspace_bytes(B, L, H, d), "cuda")
+    q, k, v = bits(t["q"]), bits(t["k"]), bits(t["v"])
+    g, st = dev(t["gamma"]), dev(t["start"])
+    S0 = dev(t.get("S0")) if with_states else None
+    z0 = dev(t.get("z0")) if with_states else None
+    per = 1 if mode == "step" else 0
+    outs = []
+    for off in (0, 1):
+        buf = torch.empty(B * L * H * d + 4, dtype=torch.float32, device="cuda")
+        y = buf[off:off + B * L * H * d]
+        den = torch.empty((B, L, H), dtype=torch.float32, device="cuda")
+        Sl = torch.empty((B, H, d, d), dtype=torch.float32, device="cuda")
+        zl = torch.empty((B, H, d), dtype=torch.float32, device="cuda")
+        m.memoroid_linattn_norm_fwd(q, k, v, g, per, st, S0, z0, y, den, Sl, zl, B, L, H, d, ws)
+        torch.cuda.synchronize()
+        assert m.memoroid_get_device_error(ws) == m.MEMOROID_OK
+        outs.append([x.cpu().numpy() for x in (y, den, Sl, zl)])
+    for a, b_ in zip(*outs):
+        assert np.array_equal(a, b_)
+    ref_y, ref_den, _, _ = oracle.linattn_norm_fwd(*(oracle.bf16_bits_to_f64(t[x]) for x in ("q", "k", "v")), t["gamma"],
+                                                   t["start"], t.get("S0") if with_states else None,
+                                                   t.get("z0") if with_states else None)
+    assert rel_err(outs[0][0].reshape(B, L, H, d), ref_y) <= TOL
