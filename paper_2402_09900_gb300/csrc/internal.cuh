@@ -135,6 +135,9 @@ struct Args {
     // S_last in the padded [B, H, 128, 128] layout; den [B, L, H] or null)
     int norm = 0;
     float* den = nullptr;
+    // backward only: grad_y already in bf16 [B, L, H, D] (exact values), used as
+    // the operand directly instead of the workspace copy
+    const uint16_t* grad_y16 = nullptr;
 };
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D);      // forward and backward

@@ -1883,7 +1883,8 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     unsigned char* ws = static_cast<unsigned char*>(a.workspace);
     TileMeta* meta = reinterpret_cast<TileMeta*>(ws + ly.meta);
     int64_t* seg_first = reinterpret_cast<int64_t*>(ws + ly.seg_first);
-    uint16_t* dy16 = reinterpret_cast<uint16_t*>(ws + ly.dy16);
+    // the bf16 operand copy of grad_y, unless the caller passes grad_y in bf16 already
+    const uint16_t* dy16 = a.grad_y16 != nullptr ? a.grad_y16 : reinterpret_cast<uint16_t*>(ws + ly.dy16);
     uint16_t* states = reinterpret_cast<uint16_t*>(ws + ly.states);
     float* dlam_f = reinterpret_cast<float*>(ws + ly.dlam_f);
     float* gpart = reinterpret_cast<float*>(ws + ly.gpart);
@@ -1891,10 +1892,13 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     memoroid_status_t st = launch_prep(a, pl, meta, seg_first, stream);
     if (st != MEMOROID_OK) return st;
 
-    const int64_t n8 = a.B * a.L * a.H * D / 8;
-    const int64_t cblocks = min((n8 + 255) / 256, static_cast<int64_t>(kTargetCtas) * 16);
-    to_bf16_kernel<<<static_cast<unsigned>(cblocks), 256, 0, stream>>>(a.grad_y, dy16, n8);
-    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    if (a.grad_y16 == nullptr) {
+        const int64_t n8 = a.B * a.L * a.H * D / 8;
+        const int64_t cblocks = min((n8 + 255) / 256, static_cast<int64_t>(kTargetCtas) * 16);
+        to_bf16_kernel<<<static_cast<unsigned>(cblocks), 256, 0, stream>>>(a.grad_y, reinterpret_cast<uint16_t*>(ws + ly.dy16),
+                                                                            n8);
+        if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    }
 
     // pass F: dq = S dy, with (q, k, v) -> (dy, v, k)
     FwdParams f;

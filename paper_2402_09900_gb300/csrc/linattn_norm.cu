@@ -183,10 +183,11 @@ __global__ void __launch_bounds__(256) divide_kernel(const float4* __restrict__ 
 __device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
 
 // dy' = [g, hi, lo, 0] with g = bf16(dy / den) and hi + lo = -(g . y) (both
-// bf16): one warp per row, lane l holding columns 4l .. 4l + 3
+// bf16), written in bf16 (every value is one already) as the backward's
+// tensor-core operand: one warp per row, lane l holding columns 4l .. 4l + 3
 __global__ void __launch_bounds__(256) upstream_kernel(const float* __restrict__ dy, const float* __restrict__ y,
                                                        const float* __restrict__ den, int64_t R, int d,
-                                                       float4* __restrict__ dyp) {
+                                                       uint2* __restrict__ dyp) {
     const int lane = threadIdx.x & 31;
     const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
     for (int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5; r < R; r += nw) {
@@ -210,7 +211,8 @@ __global__ void __launch_bounds__(256) upstream_kernel(const float* __restrict__
             if (j == d) g[e] = hi;
             if (j == d + 1) g[e] = lo;
         }
-        dyp[r * (kW / 4) + lane] = make_float4(g[0], g[1], g[2], g[3]);
+        __nv_bfloat162 w0 = __floats2bfloat162_rn(g[0], g[1]), w1 = __floats2bfloat162_rn(g[2], g[3]);
+        dyp[r * (kW / 4) + lane] = make_uint2(*reinterpret_cast<uint32_t*>(&w0), *reinterpret_cast<uint32_t*>(&w1));
     }
 }
 
@@ -253,7 +255,10 @@ int kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t d, int backward, i
     // gradient and the chain rule (backward); with states: their padding and
     // unpadding.  The forward of 64-channel heads (y 16-byte aligned) is the fused call alone.
     const bool fused = !backward && d == 64;
-    const int base = (fused ? 0 : 2 + (backward ? 1 : 0)) + la::kernels_per_call(B, L, H, backward, with_dgamma_per_head);
+    // the backward hands its bf16 upstream gradient to the linear-attention call,
+    // which then skips its own bf16 copy
+    const int base = (fused ? 0 : 2 + (backward ? 1 : 0)) + la::kernels_per_call(B, L, H, backward, with_dgamma_per_head) -
+                     (backward ? 1 : 0);
     return base + (with_states ? (backward ? 3 : 2) : 0);
 }
 
@@ -315,9 +320,9 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
         return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
     }
     upstream_kernel<<<grid_for(R * 32), 256, 0, s>>>(a.grad_y, a.y, a.den, R, static_cast<int>(a.d),
-                                                     reinterpret_cast<float4*>(b.y));
+                                                     reinterpret_cast<uint2*>(b.y));
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
-    l.grad_y = b.y;
+    l.grad_y16 = reinterpret_cast<const uint16_t*>(b.y);  // bf16 [R, 128] in the fp32 buffer's first half
     l.dS_last = g_in ? b.S1 : nullptr;
     l.dq = b.dq;
     l.dk = b.dk;
