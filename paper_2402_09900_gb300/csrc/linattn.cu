@@ -1029,13 +1029,18 @@ struct BwdSmem {
     static_assert(ST_WT + 64 <= OFF_V + TILE, "statistics fit in the V tile");
     // fp32 dk / dv tiles staged for their TMA stores (128-byte swizzled, 32
     // channels x T rows = 16 KB per chunk), in buffers free once B2 is done:
-    // dk in Pm | dPm; dv in dPm (d = 64) or K | G (d = 128)
+    // d = 64: dk in Pm, dv in dPm; d = 128: dk in K | dPm (the buffers the next
+    // tile's K and stored state go to, so that those loads wait only for the dk
+    // stores), dv in Pm | G
     static constexpr int CHUNK = T * 128;
-    __host__ __device__ static constexpr int dk_chunk(int m) { return OFF_PM + m * CHUNK; }
-    __host__ __device__ static constexpr int dv_chunk(int m) {
-        return D == 64 ? OFF_DPM + m * CHUNK : (m < 2 ? OFF_K + m * CHUNK : OFF_GB + (m - 2) * CHUNK);
+    __host__ __device__ static constexpr int dk_chunk(int m) {
+        return D == 64 ? OFF_PM + m * CHUNK : (m < 2 ? OFF_K + m * CHUNK : OFF_DPM + (m - 2) * CHUNK);
     }
-    static_assert(D == 64 ? 2 * CHUNK <= T * T * 2 : 4 * CHUNK <= 2 * T * T * 2, "dk staging fits");
+    __host__ __device__ static constexpr int dv_chunk(int m) {
+        return D == 64 ? OFF_DPM + m * CHUNK : (m < 2 ? OFF_PM + m * CHUNK : OFF_GB + (m - 2) * CHUNK);
+    }
+    static_assert(D == 64 ? 2 * CHUNK <= T * T * 2 : 2 * CHUNK <= TILE && 2 * CHUNK <= T * T * 2 && 2 * CHUNK <= D * D * 2,
+                  "output staging fits");
     // TMEM columns: P and dP, then dV and dK over them; V G^T; G
     static constexpr uint32_t COL_P = 0, COL_DP = 128, COL_DV = 0, COL_DK = 128, COL_DKI = 256,
                               COL_G = 256 + D, TMEM_COLS = 512;
@@ -1490,56 +1495,65 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         }
         LA_MARK(4);
 
-        // ---- epilogue (while B3 runs): dk = dK + w_out dKi and dv staged for TMA stores ----
+        // ---- epilogue (while B3 runs): dk = dK + w_out dKi, then dv, each staged and
+        // stored on its own, so that the dk stores drain while dv is staged ----
+        const int full_rows = static_cast<int>(min(static_cast<int64_t>(T), p.L - t0));
+        // warp 0: the staged tile's rows of this segment (one TMA store per 32 channels
+        // for a whole tile, else row by row)
+        auto store_tile = [&](bool is_dv) {
+            const CUtensorMap* map = is_dv ? &p.map_dv : &p.map_dk;
+            if (r_lo == 0 && r_hi == full_rows) {
+                if (lane == 0) {
+#pragma unroll
+                    for (int m = 0; m < D / 32; ++m)
+                        tma_store_4d(map, sbase + (is_dv ? S::dv_chunk(m) : S::dk_chunk(m)), 32 * m,
+                                     static_cast<int>(h), static_cast<int>(t0), static_cast<int>(b));
+                    bulk_commit();
+                }
+            } else {
+                float* ob = (is_dv ? p.dv : p.dk) + ((b * p.L + t0) * p.H + h) * D;
+                for (int e = lane; e < (r_hi - r_lo) * (D / 4); e += 32) {
+                    const int r = r_lo + e / (D / 4), j = (e % (D / 4)) * 4;
+                    const int in = r * 128 + ((((j & 31) >> 2) ^ (r & 7)) << 4);
+                    const int ch = is_dv ? S::dv_chunk(j >> 5) : S::dk_chunk(j >> 5);
+                    *reinterpret_cast<float4*>(ob + static_cast<int64_t>(r) * row_stride + j) =
+                        *reinterpret_cast<const float4*>(smem + ch + in);
+                }
+            }
+        };
         {
             const int r = 32 * quarter + lane;
             const float w_out = r >= mc.last_start ? fast_exp2(mc.lam2[T - 1] - mc.lam2[r]) : 0.f;
 #pragma unroll
             for (int cc = 0; cc < SC / 16; ++cc) {
                 const int j0 = cq * SC + cc * 16;
-                uint32_t rk[16], ri[16], rv[16];
+                uint32_t rk[16], ri[16];
                 tc::ld16_nowait(lane_base + S::COL_DK + j0, rk);
-                tc::ld16_nowait(lane_base + S::COL_DV + j0, rv);
                 if (have_g) tc::ld16_nowait(lane_base + S::COL_DKI + j0, ri);
                 tc::ld_wait();
-                float vk[16], vv[16];
+                float vk[16];
 #pragma unroll
-                for (int x = 0; x < 16; ++x) {
+                for (int x = 0; x < 16; ++x)
                     vk[x] = have_g ? fmaf(w_out, __uint_as_float(ri[x]), __uint_as_float(rk[x])) : __uint_as_float(rk[x]);
-                    vv[x] = __uint_as_float(rv[x]);
-                }
                 stage_f32x16(smem, dk_chunk, r, j0, vk);
+            }
+        }
+        tc::fence_smem_to_async();
+        __syncthreads();
+        if (warp == 0) store_tile(false);
+        {
+            const int r = 32 * quarter + lane;
+#pragma unroll
+            for (int cc = 0; cc < SC / 16; ++cc) {
+                const int j0 = cq * SC + cc * 16;
+                float vv[16];
+                tc::ld16(lane_base + S::COL_DV + j0, vv);
                 stage_f32x16(smem, dv_chunk, r, j0, vv);
             }
         }
         tc::fence_smem_to_async();
         __syncthreads();
-        if (warp == 0) {
-            const int full_rows = static_cast<int>(min(static_cast<int64_t>(T), p.L - t0));
-            if (r_lo == 0 && r_hi == full_rows) {
-                if (lane == 0) {
-#pragma unroll
-                    for (int m = 0; m < D / 32; ++m) {
-                        tma_store_4d(&p.map_dk, sbase + S::dk_chunk(m), 32 * m, static_cast<int>(h), static_cast<int>(t0),
-                                     static_cast<int>(b));
-                        tma_store_4d(&p.map_dv, sbase + S::dv_chunk(m), 32 * m, static_cast<int>(h), static_cast<int>(t0),
-                                     static_cast<int>(b));
-                    }
-                    bulk_commit();
-                }
-            } else {
-                float* dkb = p.dk + ((b * p.L + t0) * p.H + h) * D;
-                float* dvb = p.dv + ((b * p.L + t0) * p.H + h) * D;
-                for (int e = lane; e < (r_hi - r_lo) * (D / 4); e += 32) {
-                    const int r = r_lo + e / (D / 4), j = (e % (D / 4)) * 4;
-                    const int in = r * 128 + ((((j & 31) >> 2) ^ (r & 7)) << 4);
-                    *reinterpret_cast<float4*>(dkb + static_cast<int64_t>(r) * row_stride + j) =
-                        *reinterpret_cast<const float4*>(smem + S::dk_chunk(j >> 5) + in);
-                    *reinterpret_cast<float4*>(dvb + static_cast<int64_t>(r) * row_stride + j) =
-                        *reinterpret_cast<const float4*>(smem + S::dv_chunk(j >> 5) + in);
-                }
-            }
-        }
+        if (warp == 0) store_tile(true);
         // ---- dL/dlog(gamma_t) for the tile's rows (warps 0-3, one row per thread) ----
         if (warp < 4) {
             const int t = 32 * warp + lane;
@@ -1581,12 +1595,18 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
                 tc::fence_smem_to_async();
                 issue_tile_a(tile - 1);
             }
-            bulk_wait_read();  // dv staging in G / K and dk staging in Pm / dPm are read
+            if (D == 128) {
+                // K and dPm held the dk staging: once the dk stores (the older group)
+                // have read it, the next tile's K and stored state go there
+                bulk_wait_read_1();
+                if (next) issue_tile_b(tile - 1);
+            }
+            bulk_wait_read();  // every staged store has been read (G is written next)
         }
         if (next) pending = true;
         have_g = true;
         __syncthreads();
-        if (next && tid == 0) issue_tile_b(tile - 1);
+        if (D == 64 && next && tid == 0) issue_tile_b(tile - 1);
 
         // ---- G_{c-1} -> bf16 operand for the next tile (and dS0 at the tape start) ----
         {
