@@ -60,9 +60,10 @@ def test_linattn_autograd_matches_oracle():
         assert rel_err(np32(got), ref) <= 2e-2, name
 
 
-def test_linattn_norm_autograd_matches_oracle():
+@pytest.mark.parametrize("d", [32, 64])  # 64: the fused forward
+def test_linattn_norm_autograd_matches_oracle(d):
     m = _m()
-    t = tapegen.linattn_tape(1, 800, 2, 32, 32, seed=tapegen.seed_for(1201), mean=90.0, gamma_mode="head",
+    t = tapegen.linattn_tape(1, 800, 2, d, d, seed=tapegen.seed_for(1201 + d), mean=90.0, gamma_mode="head",
                              scale=1.0, normalize_k=False, with_grad=True)
     q, k, v = bf16_leaf(t["q"]), bf16_leaf(t["k"]), bf16_leaf(t["v"])
     gamma = dev(t["gamma"]).requires_grad_(True)

@@ -84,6 +84,32 @@ def test_linattn_norm_outputs():
         assert x.intact()
 
 
+def test_linattn_norm_fused_forward_outputs():
+    # 64-channel heads with a 16-byte aligned y take the fused forward (TMA stores of y,
+    # the normalizer written per row); the tape ends inside a tile
+    m = _m()
+    B, L, H, d = 2, 1111, 3, 64
+    t = tapegen.linattn_tape(B, L, H, d, d, tapegen.seed_for(903), mean=70.0, gamma_mode="step", scale=1.0,
+                             normalize_k=False, with_S0=True)
+    q, k, v = bits(t["q"]), bits(t["k"]), bits(t["v"])
+    g, st = dev(t["gamma"]), dev(t["start"])
+    rng = np.random.default_rng(9)
+    S0 = dev(t["S0"])
+    z0 = dev(rng.uniform(0.5, 2.0, (B, H, d)).astype(np.float32))
+    y = Guarded((B, L, H, d), torch.float32, 6.5)
+    den = Guarded((B, L, H), torch.float32, 6.5)
+    Sl = Guarded((B, H, d, d), torch.float32, 6.5)
+    zl = Guarded((B, H, d), torch.float32, 6.5)
+    assert y.t.data_ptr() % 16 == 0
+    ws = m.workspace(m.memoroid_linattn_norm_workspace_bytes(B, L, H, d), "cuda")
+    m.memoroid_linattn_norm_fwd(q, k, v, g, 1, st, S0, z0, y.t, den.t, Sl.t, zl.t, B, L, H, d, ws)
+    torch.cuda.synchronize()
+    assert m.memoroid_get_device_error(ws) == m.MEMOROID_OK
+    for x in (y, den, Sl, zl):
+        assert x.intact()
+    assert bool(torch.isfinite(y.t).all()) and bool((den.t > 0).all())
+
+
 def test_returns_outputs():
     m = _m()
     rng = np.random.default_rng(3)
