@@ -138,6 +138,9 @@ struct Args {
     // backward only: grad_y already in bf16 [B, L, H, D] (exact values), used as
     // the operand directly instead of the workspace copy
     const uint16_t* grad_y16 = nullptr;
+    // backward only: 64 (with D = 128) writes only the first 64 columns of dq,
+    // dk, dv, as [B, L, H, 64] arrays; 0 writes all D
+    int64_t out_cols = 0;
 };
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D);      // forward and backward

@@ -459,9 +459,12 @@ __device__ __forceinline__ void store_bf16x16(unsigned char* base, uint32_t off0
 // (the term of dL/dlog(gamma_s) that pairs the incoming state with the tile's
 // outputs), and stores S'_{c-1} as bf16 for every tile without a begin flag,
 // for pass R.
-template <int D, bool BWD, bool NORM = false>
+template <int D, bool BWD, bool NORM = false, bool HALF_OUT = false>
 __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant__ FwdParams p) {
     static_assert(!NORM || (D == 128 && !BWD), "the normalised forward runs the d = 128 forward");
+    // HALF_OUT (pass F at d = 128): only the first 64 output columns are written,
+    // to a [B, L, H, 64] output (the normalised path needs no more of dq')
+    static_assert(!HALF_OUT || (D == 128 && BWD), "half-width output for pass F at d = 128");
     using S = FwdSmem<D>;
     // NORM: the Linear Transformer with phi and its normalizer for heads of 64
     // channels.  q, k, v are the unpadded [B, L, H, 64] tensors; each operand
@@ -472,7 +475,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     // column 64 of the output is the normalizer; the epilogue writes
     // y = y'[:64] / y'[64] and the normalizer.
     constexpr int KQ = NORM ? 64 : D;     // channels of the q/k contractions
-    constexpr int DOUT = NORM ? 64 : D;   // output channels
+    constexpr int DOUT = (NORM || HALF_OUT) ? 64 : D;  // output channels written
     constexpr int Y_OFF = NORM ? 0 : S::OFF_Y;  // output staging: the Q slot (NORM) or the K and V slots
     extern __shared__ __align__(1024) unsigned char smem[];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -1104,8 +1107,12 @@ __device__ __forceinline__ void stage_f32x16(unsigned char* smem, ChunkFn chunk,
     }
 }
 
-template <int D>
+template <int D, bool HALF_OUT = false>
 __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant__ BwdParams p) {
+    static_assert(!HALF_OUT || D == 128, "half-width output at d = 128");
+    // HALF_OUT: only the first 64 columns of dk and dv are written, to [B, L, H, 64]
+    // outputs (the normalised path needs no more of dk' and dv')
+    constexpr int DOUT = HALF_OUT ? 64 : D;
     using S = BwdSmem<D>;
     extern __shared__ __align__(1024) unsigned char smem[];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -1127,7 +1134,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         }
     }
     const int64_t tile_lo = seg_lo / T, tile_hi = (seg_hi + T - 1) / T;  // tiles [tile_lo, tile_hi)
-    const int64_t row_stride = p.H * D;
+    const int64_t row_stride = p.H * DOUT;
 
     uint64_t* bar1 = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
     uint64_t* bar2 = bar1 + 1;
@@ -1505,15 +1512,15 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
             if (r_lo == 0 && r_hi == full_rows) {
                 if (lane == 0) {
 #pragma unroll
-                    for (int m = 0; m < D / 32; ++m)
+                    for (int m = 0; m < DOUT / 32; ++m)
                         tma_store_4d(map, sbase + (is_dv ? S::dv_chunk(m) : S::dk_chunk(m)), 32 * m,
                                      static_cast<int>(h), static_cast<int>(t0), static_cast<int>(b));
                     bulk_commit();
                 }
             } else {
-                float* ob = (is_dv ? p.dv : p.dk) + ((b * p.L + t0) * p.H + h) * D;
-                for (int e = lane; e < (r_hi - r_lo) * (D / 4); e += 32) {
-                    const int r = r_lo + e / (D / 4), j = (e % (D / 4)) * 4;
+                float* ob = (is_dv ? p.dv : p.dk) + ((b * p.L + t0) * p.H + h) * DOUT;
+                for (int e = lane; e < (r_hi - r_lo) * (DOUT / 4); e += 32) {
+                    const int r = r_lo + e / (DOUT / 4), j = (e % (DOUT / 4)) * 4;
                     const int in = r * 128 + ((((j & 31) >> 2) ^ (r & 7)) << 4);
                     const int ch = is_dv ? S::dv_chunk(j >> 5) : S::dk_chunk(j >> 5);
                     *reinterpret_cast<float4*>(ob + static_cast<int64_t>(r) * row_stride + j) =
@@ -1898,7 +1905,7 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     return MEMOROID_OK;
 }
-template <int D>
+template <int D, bool HALF_OUT = false>
 memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, cudaStream_t stream) {
     unsigned char* ws = static_cast<unsigned char*>(a.workspace);
     TileMeta* meta = reinterpret_cast<TileMeta*>(ws + ly.meta);
@@ -1923,8 +1930,8 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     // pass F: dq = S dy, with (q, k, v) -> (dy, v, k)
     FwdParams f;
     if (!tile_map(&f.map_q, dy16, a.B, a.L, a.H, D) || !tile_map(&f.map_k, a.v, a.B, a.L, a.H, D) ||
-        !tile_map(&f.map_v, a.k, a.B, a.L, a.H, D) || !tile_map_y(&f.map_y, a.dq, a.B, a.L, a.H, D) ||
-        !tile_map(&f.map_zq, a.q, a.B, a.L, a.H, D))
+        !tile_map(&f.map_v, a.k, a.B, a.L, a.H, D) ||
+        !tile_map_y(&f.map_y, a.dq, a.B, a.L, a.H, HALF_OUT ? 64 : D) || !tile_map(&f.map_zq, a.q, a.B, a.L, a.H, D))
         return MEMOROID_ERR_CUDA;
     f.den = nullptr;
     f.q = dy16;
@@ -1949,15 +1956,16 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
 #ifdef MEMOROID_LA_TRACE
     f.trace = la_trace_buffer();  // pass F's phases replace the forward's in slots 0-7
 #endif
-    if (set_smem(fwd_kernel<D, true>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    fwd_kernel<D, true><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
+    if (set_smem(fwd_kernel<D, true, false, HALF_OUT>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    fwd_kernel<D, true, false, HALF_OUT><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
 
     // pass R: dk, dv, dgamma, dS0
     BwdParams r;
     if (!tile_map(&r.map_q, a.q, a.B, a.L, a.H, D) || !tile_map(&r.map_k, a.k, a.B, a.L, a.H, D) ||
         !tile_map(&r.map_v, a.v, a.B, a.L, a.H, D) || !tile_map(&r.map_dy, dy16, a.B, a.L, a.H, D) ||
-        !tile_map_y(&r.map_dk, a.dk, a.B, a.L, a.H, D) || !tile_map_y(&r.map_dv, a.dv, a.B, a.L, a.H, D))
+        !tile_map_y(&r.map_dk, a.dk, a.B, a.L, a.H, HALF_OUT ? 64 : D) ||
+        !tile_map_y(&r.map_dv, a.dv, a.B, a.L, a.H, HALF_OUT ? 64 : D))
         return MEMOROID_ERR_CUDA;
     r.q = static_cast<const uint16_t*>(a.q);
     r.k = static_cast<const uint16_t*>(a.k);
@@ -1986,8 +1994,8 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
 #ifdef MEMOROID_LA_TRACE
     r.trace = la_trace_buffer();
 #endif
-    if (set_smem(bwd_kernel<D>, BwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    bwd_kernel<D><<<static_cast<unsigned>(a.B * a.H * pl.G), kRThreads, BwdSmem<D>::BYTES, stream>>>(r);
+    if (set_smem(bwd_kernel<D, HALF_OUT>, BwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    bwd_kernel<D, HALF_OUT><<<static_cast<unsigned>(a.B * a.H * pl.G), kRThreads, BwdSmem<D>::BYTES, stream>>>(r);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     if (r.gpart != nullptr) {
         dgamma_head_kernel<<<static_cast<unsigned>((a.H + 127) / 128), 128, 0, stream>>>(gpart, a.gamma, a.dgamma,
@@ -2011,6 +2019,8 @@ memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream) {
     if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, stream) != cudaSuccess) return MEMOROID_ERR_CUDA;
     const Plan pl = make_plan(a.B, a.L, a.H);
     const Layout ly = make_layout(a.B, a.L, a.H, a.D);
+    if (a.out_cols != 0 && !(a.out_cols == 64 && a.D == 128)) return MEMOROID_ERR_UNSUPPORTED;
+    if (a.out_cols == 64) return launch_bwd_d<128, true>(a, pl, ly, stream);
     if (a.D == 64) return launch_bwd_d<64>(a, pl, ly, stream);
     if (a.D == 128) return launch_bwd_d<128>(a, pl, ly, stream);
     return MEMOROID_ERR_UNSUPPORTED;

@@ -216,17 +216,18 @@ __global__ void __launch_bounds__(256) upstream_kernel(const float* __restrict__
     }
 }
 
-// dq = dq'[:d] (.) phi'(q), dk = dk'[:d] (.) phi'(k), dv = dv'[:d]: one
-// thread per 4 columns (16-byte loads and stores; 32-bit index arithmetic)
+// dq = dq'[:d] (.) phi'(q), dk = dk'[:d] (.) phi'(k), dv = dv'[:d] from
+// padded gradients with rows of w4 float4s: one thread per 4 columns (16-byte
+// loads and stores; 32-bit index arithmetic)
 __global__ void __launch_bounds__(256) chain_kernel(const float4* __restrict__ dqp, const float4* __restrict__ dkp,
                                                     const float4* __restrict__ dvp, const uint2* __restrict__ q,
-                                                    const uint2* __restrict__ k, uint32_t R, uint32_t d4,
+                                                    const uint2* __restrict__ k, uint32_t R, uint32_t d4, uint32_t w4,
                                                     float4* __restrict__ dq, float4* __restrict__ dk,
                                                     float4* __restrict__ dv) {
     const uint32_t n = R * d4;
     for (uint32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < n; g += gridDim.x * blockDim.x) {
         const uint32_t r = g / d4, c = g - r * d4;
-        const uint32_t pp = r * (kW / 4) + c;
+        const uint32_t pp = r * w4 + c;
         const uint2 qb = q[g], kb = k[g];
         const float2 q0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qb.x));
         const float2 q1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&qb.y));
@@ -324,6 +325,9 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     l.grad_y16 = reinterpret_cast<const uint16_t*>(b.y);  // bf16 [R, 128] in the fp32 buffer's first half
     l.dS_last = g_in ? b.S1 : nullptr;
+    // heads of up to 64 channels need only the first 64 columns of dq', dk', dv'
+    const int64_t wout = a.d <= 64 ? 64 : kW;
+    l.out_cols = a.d <= 64 ? 64 : 0;
     l.dq = b.dq;
     l.dk = b.dk;
     l.dv = b.dv;
@@ -334,7 +338,8 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
     chain_kernel<<<grid_for(R * a.d / 4), 256, 0, s>>>(
         reinterpret_cast<const float4*>(b.dq), reinterpret_cast<const float4*>(b.dk),
         reinterpret_cast<const float4*>(b.dv), static_cast<const uint2*>(a.q), static_cast<const uint2*>(a.k),
-        static_cast<uint32_t>(R), static_cast<uint32_t>(a.d / 4), reinterpret_cast<float4*>(a.dq),
+        static_cast<uint32_t>(R), static_cast<uint32_t>(a.d / 4), static_cast<uint32_t>(wout / 4),
+        reinterpret_cast<float4*>(a.dq),
         reinterpret_cast<float4*>(a.dk), reinterpret_cast<float4*>(a.dv));
     if (l.dS0 != nullptr)
         unpad_state_kernel<<<grid_for(BH * a.d * (a.d + 1)), 256, 0, s>>>(b.S2, BH, static_cast<int>(a.d), 1, a.dS0,
