@@ -463,6 +463,12 @@ void memoroid_debug_set_wait_limit_ns(uint64_t ns);
  * the workspace and stops). */
 void memoroid_debug_withhold_tile(int64_t ticket);
 
+/* Test knob (0 = off, the default; applies to later calls): the Linear
+ * Transformer calls (memoroid_linattn_norm_*) always build padded operands in
+ * separate kernels, instead of the in-kernel construction they use for
+ * 64-channel heads; both compute the same bits. */
+void memoroid_debug_lnorm_padded(int on);
+
 #ifdef __cplusplus
 }
 #endif

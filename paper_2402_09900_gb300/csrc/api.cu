@@ -15,6 +15,7 @@ namespace {
 constexpr uint64_t kDefaultWaitNs = 1000000000ull;  // 1 s
 std::atomic<uint64_t> g_wait_ns{kDefaultWaitNs};
 std::atomic<int64_t> g_withhold{-1};
+std::atomic<int> g_lnorm_padded{0};
 // seeded from the clock so that two processes sharing a workspace are
 // unlikely to reuse each other's tags
 std::atomic<uint32_t> g_epoch{static_cast<uint32_t>(
@@ -24,7 +25,7 @@ inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintp
 inline cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
 }  // namespace
 
-DebugKnobs debug_knobs() { return DebugKnobs{g_wait_ns.load(), g_withhold.load()}; }
+DebugKnobs debug_knobs() { return DebugKnobs{g_wait_ns.load(), g_withhold.load(), g_lnorm_padded.load()}; }
 
 EncodeTiledFn encode_tiled() {
     static EncodeTiledFn fn = nullptr;
@@ -70,6 +71,8 @@ int memoroid_version(void) { return 100; }
 void memoroid_debug_set_wait_limit_ns(uint64_t ns) { g_wait_ns.store(ns == 0 ? kDefaultWaitNs : ns); }
 
 void memoroid_debug_withhold_tile(int64_t ticket) { g_withhold.store(ticket); }
+
+void memoroid_debug_lnorm_padded(int on) { g_lnorm_padded.store(on != 0 ? 1 : 0); }
 
 memoroid_status_t memoroid_get_device_error(const void* workspace, void* stream) {
     if (workspace == nullptr) return MEMOROID_ERR_INVALID_ARG;

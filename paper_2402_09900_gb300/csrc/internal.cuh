@@ -32,6 +32,7 @@ constexpr size_t kHeaderBytes = 256;
 struct DebugKnobs {
     uint64_t wait_ns;
     int64_t withhold_ticket;
+    int lnorm_padded;  // the normalised calls always take the padded-operand path
 };
 DebugKnobs debug_knobs();
 
@@ -130,9 +131,12 @@ struct Args {
     int64_t B, L, H, D;
     void* workspace;
     size_t workspace_bytes;
-    // forward only, norm = 1: the Linear Transformer with phi and its normalizer
-    // for 64-channel heads at D = 128 (q, k, v and y [B, L, H, 64]; S0 and
-    // S_last in the padded [B, H, 128, 128] layout; den [B, L, H] or null)
+    // norm = 1: the Linear Transformer with phi and its normalizer for
+    // 64-channel heads at D = 128, with q, k, v the unpadded [B, L, H, 64]
+    // tensors.  Forward: y [B, L, H, 64] and den [B, L, H] (or null); S0 and
+    // S_last in the padded [B, H, 128, 128] layout.  Backward: the padded bf16
+    // upstream gradient in grad_y16 and out_cols = 64 (the padded gradients'
+    // first 64 columns; the chain rule through phi is the caller's).
     int norm = 0;
     float* den = nullptr;
     // backward only: grad_y already in bf16 [B, L, H, D] (exact values), used as

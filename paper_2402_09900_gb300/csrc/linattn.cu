@@ -312,6 +312,40 @@ __device__ __forceinline__ void scale_rows_sw(unsigned char* tile, int tid, WFn 
     }
 }
 
+// phi(z) = 1 + ELU(z) in place on the first 64-channel box of a [T x 128]
+// operand slot (bf16, round to nearest, the SFU exponential); rows at or past
+// `valid` become 0, as rows past the tape end of padded operands are.  NT
+// threads, one 16-byte unit (8 channels) of one row per step.
+template <int NT>
+__device__ __forceinline__ void phi_box(unsigned char* slot, int tid, int64_t valid) {
+#pragma unroll
+    for (int i = 0; i < T * 8 / NT; ++i) {
+        const int unit = i * NT + tid, row = unit / 8;
+        uint4* a = reinterpret_cast<uint4*>(slot + unit * 16);
+        uint4 u = *a;
+        uint32_t* w = reinterpret_cast<uint32_t*>(&u);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = unpack_bf16x2(w[e]);
+            w[e] = row < valid ? pack_bf16x2(f.x > 0.f ? 1.f + f.x : __expf(f.x), f.y > 0.f ? 1.f + f.y : __expf(f.y))
+                               : 0u;
+        }
+        *a = u;
+    }
+}
+
+// The second 64-channel box of a [T x 128] operand slot as a constant: zeros,
+// or (ones) channels 64 and 65 of every row 1 and the rest 0.  Unit u of row r
+// holds channels 8 (u ^ (r % 8)) .. + 7 of the box.
+template <int NT>
+__device__ __forceinline__ void const_box(unsigned char* slot, int tid, bool ones) {
+    const uint32_t one2 = pack_bf16x2(1.f, 1.f);
+    for (int i = tid; i < T * 8; i += NT) {
+        const int r = i / 8, u = i % 8;
+        *reinterpret_cast<uint4*>(slot + T * 128 + i * 16) = make_uint4(ones && (u ^ (r & 7)) == 0 ? one2 : 0u, 0u, 0u, 0u);
+    }
+}
+
 __device__ __forceinline__ bool wait_mbar(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer();
@@ -461,7 +495,7 @@ __device__ __forceinline__ void store_bf16x16(unsigned char* base, uint32_t off0
 // for pass R.
 template <int D, bool BWD, bool NORM = false, bool HALF_OUT = false>
 __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant__ FwdParams p) {
-    static_assert(!NORM || (D == 128 && !BWD), "the normalised forward runs the d = 128 forward");
+    static_assert(!NORM || (D == 128 && (!BWD || HALF_OUT)), "the normalised operands run the d = 128 kernels");
     // HALF_OUT (pass F at d = 128): only the first 64 output columns are written,
     // to a [B, L, H, 64] output (the normalised path needs no more of dq')
     static_assert(!HALF_OUT || (D == 128 && BWD), "half-width output for pass F at d = 128");
@@ -474,9 +508,17 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     // columns [1, 1, 0, ...], so the 128-wide state is [[X, x, x], [0]] and
     // column 64 of the output is the normalizer; the epilogue writes
     // y = y'[:64] / y'[64] and the normalizer.
-    constexpr int KQ = NORM ? 64 : D;     // channels of the q/k contractions
+    // NORM with BWD: pass F of the normalised backward for 64-channel heads, on
+    // (dy', v', k') with dy' padded by the caller, v' = [v, 1, 1, 0] and
+    // k' = [phi(k), 0] built in the K and V slots the same way, and q' = [phi(q), 0]
+    // for the z term (phi applied as the tile is read).  The output rows are
+    // staged in the K slot, whose constant half is written again once they drain.
+    constexpr bool NF = NORM && !BWD, NB = NORM && BWD;
+    constexpr int KQ = NF ? 64 : D;          // channels of the first contractions
+    constexpr int BQ = NF ? 64 : D;          // channels loaded into the Q slot
+    constexpr int BKV = NORM ? 64 : D;       // channels loaded into the K and V slots
     constexpr int DOUT = (NORM || HALF_OUT) ? 64 : D;  // output channels written
-    constexpr int Y_OFF = NORM ? 0 : S::OFF_Y;  // output staging: the Q slot (NORM) or the K and V slots
+    constexpr int Y_OFF = NF ? 0 : S::OFF_Y;  // output staging: the Q slot (NF) or the K and V slots
     extern __shared__ __align__(1024) unsigned char smem[];
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int quarter = warp & 3, half = warp >> 2;
@@ -517,11 +559,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     // m1 >= 0) into their ring slots, all completing on full[s]
     auto issue_tile = [&](int c, int s, int m0, int m1) {
         const uint32_t meta_bytes = (m0 >= 0 ? sizeof(TileMeta) : 0) + (m1 >= 0 ? sizeof(TileMeta) : 0);
-        mbar_arrive_expect_tx(&full[s], 3 * (T * KQ * 2) + meta_bytes);
+        mbar_arrive_expect_tx(&full[s], T * BQ * 2 + 2 * (T * BKV * 2) + meta_bytes);
         const int64_t t0 = (tile0 + c) * T;
-        tma_tile<KQ>(stage_q(s), &p.map_q, h, t0, b, &full[s]);
-        tma_tile<KQ>(stage_k(s), &p.map_k, h, t0, b, &full[s]);
-        tma_tile<KQ>(stage_v(s), &p.map_v, h, t0, b, &full[s]);
+        tma_tile<BQ>(stage_q(s), &p.map_q, h, t0, b, &full[s]);
+        tma_tile<BKV>(stage_k(s), &p.map_k, h, t0, b, &full[s]);
+        tma_tile<BKV>(stage_v(s), &p.map_v, h, t0, b, &full[s]);
         if (m0 >= 0) bulk_g2s(&metas[m0 % S::NMETA], gmeta + m0, sizeof(TileMeta), &full[s]);
         if (m1 >= 0) bulk_g2s(&metas[m1 % S::NMETA], gmeta + m1, sizeof(TileMeta), &full[s]);
     };
@@ -541,16 +583,12 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     }
     if (warp == 0) tc::alloc(tslot, S::TMEM_COLS);
     if (NORM) {
-        // the constant second halves of the K slots (zeros) and V slots ([1, 1, 0, ...]
-        // per row) of both stages; the loads only ever write the first halves
-        for (int i = tid; i < 2 * T * 8; i += kThreads) {
-            const int st = i / (T * 8), r = (i / 8) % T, u = i % 8;
-            unsigned char* kc = smem + st * S::STAGE + S::TILE + T * 128 + r * 128 + u * 16;
-            unsigned char* vc = smem + st * S::STAGE + 2 * S::TILE + T * 128 + r * 128 + u * 16;
-            *reinterpret_cast<uint4*>(kc) = make_uint4(0u, 0u, 0u, 0u);
-            // unit u of row r holds channels 8 (u ^ (r % 8)) .. + 7 of the half
-            const uint32_t ones = pack_bf16x2(1.f, 1.f);
-            *reinterpret_cast<uint4*>(vc) = make_uint4((u ^ (r & 7)) == 0 ? ones : 0u, 0u, 0u, 0u);
+        // the constant second halves of the K and V slots of both stages (the forward:
+        // zeros for k, [1, 1, 0, ...] for v; pass F: the v' constants in the K slot,
+        // zeros for k in the V slot); the loads only ever write the first halves
+        for (int st = 0; st < 2; ++st) {
+            const_box<kThreads>(smem + st * S::STAGE + S::TILE, tid, NB);
+            const_box<kThreads>(smem + st * S::STAGE + 2 * S::TILE, tid, NF);
         }
     }
     tc::fence_before();
@@ -646,24 +684,13 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         tc::fence_after();
         LA_MARK(0);
         if (NORM) {
-            // phi(z) = 1 + ELU(z) on the loaded q and k, in place (bf16, round to
-            // nearest); rows past the tape end stay 0, as the padded operands would
-            const int64_t tb = (tile0 + c) * T;
-#pragma unroll
-            for (int i = 0; i < 2 * T * 8 / kThreads; ++i) {
-                const int unit = i * kThreads + tid;  // 16-byte units of the Q then the K half-tile
-                const int row = (unit % (T * 8)) / 8;
-                unsigned char* a = smem + s * S::STAGE + (unit >= T * 8 ? S::TILE : 0) + (unit % (T * 8)) * 16;
-                uint4 u = *reinterpret_cast<uint4*>(a);
-                uint32_t* w = reinterpret_cast<uint32_t*>(&u);
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float2 f = unpack_bf16x2(w[e]);
-                    w[e] = tb + row < p.L
-                               ? pack_bf16x2(f.x > 0.f ? 1.f + f.x : __expf(f.x), f.y > 0.f ? 1.f + f.y : __expf(f.y))
-                               : 0u;
-                }
-                *reinterpret_cast<uint4*>(a) = u;
+            // phi on the loaded q and k (the forward) or k (pass F), in place
+            const int64_t valid = p.L - (tile0 + c) * T;
+            if (NF) {
+                phi_box<kThreads>(smem + s * S::STAGE, tid, valid);
+                phi_box<kThreads>(smem + s * S::STAGE + S::TILE, tid, valid);
+            } else {
+                phi_box<kThreads>(smem + s * S::STAGE + 2 * S::TILE, tid, valid);
             }
             tc::fence_smem_to_async();
             tc::fence_before();
@@ -698,8 +725,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         const bool zload = BWD && have_prev;
         if (zload) {
             if (tid == 0) {
-                mbar_arrive_expect_tx(qbar, S::TILE);
-                tma_tile<D>(stage_q(s), &p.map_zq, h, (tile0 + c) * T, b, qbar);
+                mbar_arrive_expect_tx(qbar, T * BKV * 2);
+                tma_tile<BKV>(stage_q(s), &p.map_zq, h, (tile0 + c) * T, b, qbar);
             }
             q_pending = true;
         }
@@ -743,6 +770,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         tc::fence_before();
         __syncthreads();
         tc::fence_after();
+        // pass F (normalised): the output rows were staged over the v' constants of stage s ^ 1
+        if (NB) const_box<kThreads>(smem + (s ^ 1) * S::STAGE + S::TILE, tid, true);
         // the next tile's loads into stage s ^ 1
         if (c + 1 < nt) {
             if (tid == 32) issue_tile(c + 1, s ^ 1, c + 2 < nt ? c + 2 : -1, -1);
@@ -786,7 +815,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         // rows of this tile that belong to the segment
         const int r_lo = static_cast<int>(max(static_cast<int64_t>(0), seg_lo - t0));
         const int r_hi = static_cast<int>(min(static_cast<int64_t>(T), seg_hi - t0));
-        if (NORM) {
+        if (NF) {
             // y = y'[:64] / y'[64]: every thread reads the normalizer (column 64) of
             // its row and divides its 32 of the 64 output columns
             const int t = 32 * quarter + lane;
@@ -819,12 +848,21 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 *reinterpret_cast<float4*>(yst + (j >> 5) * (T * 128) + ((((j & 31) >> 2) ^ (t & 7)) << 4)) =
                     make_float4(o[0], o[1], o[2], o[3]);
             }
+        } else if (HALF_OUT && half == 1) {
+            // output channels 64..127 are not written, and q' is zero there (d <= 64)
+            reinterpret_cast<float*>(smem + S::OFF_Z)[T + 32 * quarter + lane] = 0.f;
         } else {
             const int t = 32 * quarter + lane;
             const float w_in = (have_prev && mc.seg[t] < 0) ? fast_exp2(mc.lam2[t]) : 0.f;
             unsigned char* yst = smem + s * S::STAGE + Y_OFF + t * 128;  // row t of chunk 0
             const unsigned char* qs = smem + (stage_q(s) - sbase);  // pass F: the q tile
             const bool zrow = zload && w_in != 0.f;
+            // q' of the z term: the loaded values, or (normalised) phi of them rounded to bf16
+            auto qpair = [](uint32_t w) {
+                float2 f = unpack_bf16x2(w);
+                if (NB) f = unpack_bf16x2(pack_bf16x2(f.x > 0.f ? 1.f + f.x : __expf(f.x), f.y > 0.f ? 1.f + f.y : __expf(f.y)));
+                return f;
+            };
             // BWD: z_t = w_in_t q_t . (S_{c-1} dy_t), the inter output dotted with q
             float zacc = 0.f;
 #pragma unroll
@@ -855,8 +893,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
 #pragma unroll
                     for (int x = 0; x < 32; x += 8) {
                         const uint4 u = *reinterpret_cast<const uint4*>(qs + sw_off(t, j0 + x));
-                        const float2 q0 = unpack_bf16x2(u.x), q1 = unpack_bf16x2(u.y), q2 = unpack_bf16x2(u.z),
-                                     q3 = unpack_bf16x2(u.w);
+                        const float2 q0 = qpair(u.x), q1 = qpair(u.y), q2 = qpair(u.z), q3 = qpair(u.w);
                         zacc = fmaf(q0.x, __uint_as_float(yi[x]), zacc);
                         zacc = fmaf(q0.y, __uint_as_float(yi[x + 1]), zacc);
                         zacc = fmaf(q1.x, __uint_as_float(yi[x + 2]), zacc);
@@ -1107,9 +1144,16 @@ __device__ __forceinline__ void stage_f32x16(unsigned char* smem, ChunkFn chunk,
     }
 }
 
-template <int D, bool HALF_OUT = false>
+template <int D, bool HALF_OUT = false, bool NORM = false>
 __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant__ BwdParams p) {
     static_assert(!HALF_OUT || D == 128, "half-width output at d = 128");
+    static_assert(!NORM || HALF_OUT, "the normalised operands come with half-width outputs");
+    // NORM: the normalised backward for 64-channel heads: q, k, v are the unpadded
+    // [B, L, H, 64] tensors loaded into the first halves of their slots, phi is
+    // applied to q and k in shared memory, and the second halves hold zeros (q, k)
+    // or the columns [1, 1, 0, ...] (v); dY is the caller's padded dy'.  K's zero
+    // half, where dk rows are staged, is written again once they drain.
+    constexpr int BKV = NORM ? 64 : D;  // channels loaded into the Q, K and V slots
     // HALF_OUT: only the first 64 columns of dk and dv are written, to [B, L, H, 64]
     // outputs (the normalised path needs no more of dk' and dv')
     constexpr int DOUT = HALF_OUT ? 64 : D;
@@ -1159,13 +1203,14 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     // exists) the stored forward state before it, completing on `full`.  The
     // state slot of a tile with a begin flag was never written: it is loaded
     // all the same and not read.
+    constexpr uint32_t kTileBytes = 3 * (T * BKV * 2) + S::TILE;  // Q, K, V and dY
     auto issue_tile = [&](int64_t tile, bool with_state) {
         constexpr uint32_t kStateBytes = D * D * 2;
-        mbar_arrive_expect_tx(full, 4 * S::TILE + sizeof(TileMeta) + (with_state ? kStateBytes : 0u));
+        mbar_arrive_expect_tx(full, kTileBytes + sizeof(TileMeta) + (with_state ? kStateBytes : 0u));
         const int64_t t0 = tile * T;
-        tma_tile<D>(sQ, &p.map_q, h, t0, b, full);
-        tma_tile<D>(sK, &p.map_k, h, t0, b, full);
-        tma_tile<D>(sV, &p.map_v, h, t0, b, full);
+        tma_tile<BKV>(sQ, &p.map_q, h, t0, b, full);
+        tma_tile<BKV>(sK, &p.map_k, h, t0, b, full);
+        tma_tile<BKV>(sV, &p.map_v, h, t0, b, full);
         tma_tile<D>(sDY, &p.map_dy, h, t0, b, full);
         bulk_g2s(smem + S::OFF_META, p.meta + bh * p.n_tiles + tile, sizeof(TileMeta), full);
         if (with_state) bulk_g2s(smem + S::OFF_SS, p.states + (bh * p.n_tiles + tile) * D * D, kStateBytes, full);
@@ -1174,15 +1219,15 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     // as soon as B3 is done, K and the state once the staged output stores (in
     // K, G, Pm and dPm) have been read
     auto issue_tile_a = [&](int64_t tile) {
-        mbar_arrive_expect_tx(full, 4 * S::TILE + sizeof(TileMeta) + D * D * 2);
+        mbar_arrive_expect_tx(full, kTileBytes + sizeof(TileMeta) + D * D * 2);
         const int64_t t0 = tile * T;
-        tma_tile<D>(sQ, &p.map_q, h, t0, b, full);
-        tma_tile<D>(sV, &p.map_v, h, t0, b, full);
+        tma_tile<BKV>(sQ, &p.map_q, h, t0, b, full);
+        tma_tile<BKV>(sV, &p.map_v, h, t0, b, full);
         tma_tile<D>(sDY, &p.map_dy, h, t0, b, full);
         bulk_g2s(smem + S::OFF_META, p.meta + bh * p.n_tiles + tile, sizeof(TileMeta), full);
     };
     auto issue_tile_b = [&](int64_t tile) {
-        tma_tile<D>(sK, &p.map_k, h, tile * T, b, full);
+        tma_tile<BKV>(sK, &p.map_k, h, tile * T, b, full);
         bulk_g2s(smem + S::OFF_SS, p.states + (bh * p.n_tiles + tile) * D * D, D * D * 2, full);
     };
     bool have_g = seg_hi == p.L && p.dS_last != nullptr;  // a reverse state enters the current tile
@@ -1202,6 +1247,11 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         prefetch_tensormap(&p.map_dv);
     }
     if (warp == 0) tc::alloc(tslot, S::TMEM_COLS);
+    if (NORM) {
+        const_box<kRThreads>(smem + S::OFF_Q, tid, false);
+        const_box<kRThreads>(smem + S::OFF_K, tid, false);
+        const_box<kRThreads>(smem + S::OFF_V, tid, true);
+    }
     tc::fence_before();
     __syncthreads();
     tc::fence_after();
@@ -1269,6 +1319,13 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         }
         pending = false;
         tc::fence_after();
+        if (NORM) {
+            const int64_t valid = p.L - t0;
+            phi_box<kRThreads>(smem + S::OFF_Q, tid, valid);
+            phi_box<kRThreads>(smem + S::OFF_K, tid, valid);
+            tc::fence_smem_to_async();
+            __syncthreads();
+        }
         LA_MARK(0);
         const bool tile_start = mc.has_start != 0;
 
@@ -1614,6 +1671,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         have_g = true;
         __syncthreads();
         if (D == 64 && next && tid == 0) issue_tile_b(tile - 1);
+        if (NORM) const_box<kRThreads>(smem + S::OFF_K, tid, false);  // K's zero half held dk rows
 
         // ---- G_{c-1} -> bf16 operand for the next tile (and dS0 at the tape start) ----
         {
@@ -1905,7 +1963,7 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     return MEMOROID_OK;
 }
-template <int D, bool HALF_OUT = false>
+template <int D, bool HALF_OUT = false, bool NORM = false>
 memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, cudaStream_t stream) {
     unsigned char* ws = static_cast<unsigned char*>(a.workspace);
     TileMeta* meta = reinterpret_cast<TileMeta*>(ws + ly.meta);
@@ -1929,9 +1987,10 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
 
     // pass F: dq = S dy, with (q, k, v) -> (dy, v, k)
     FwdParams f;
-    if (!tile_map(&f.map_q, dy16, a.B, a.L, a.H, D) || !tile_map(&f.map_k, a.v, a.B, a.L, a.H, D) ||
-        !tile_map(&f.map_v, a.k, a.B, a.L, a.H, D) ||
-        !tile_map_y(&f.map_y, a.dq, a.B, a.L, a.H, HALF_OUT ? 64 : D) || !tile_map(&f.map_zq, a.q, a.B, a.L, a.H, D))
+    constexpr int BKV = NORM ? 64 : D;  // channels of q, k, v in memory (the normalised path: unpadded)
+    if (!tile_map(&f.map_q, dy16, a.B, a.L, a.H, D) || !tile_map(&f.map_k, a.v, a.B, a.L, a.H, BKV) ||
+        !tile_map(&f.map_v, a.k, a.B, a.L, a.H, BKV) ||
+        !tile_map_y(&f.map_y, a.dq, a.B, a.L, a.H, HALF_OUT ? 64 : D) || !tile_map(&f.map_zq, a.q, a.B, a.L, a.H, BKV))
         return MEMOROID_ERR_CUDA;
     f.den = nullptr;
     f.q = dy16;
@@ -1956,14 +2015,14 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
 #ifdef MEMOROID_LA_TRACE
     f.trace = la_trace_buffer();  // pass F's phases replace the forward's in slots 0-7
 #endif
-    if (set_smem(fwd_kernel<D, true, false, HALF_OUT>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    fwd_kernel<D, true, false, HALF_OUT><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
+    if (set_smem(fwd_kernel<D, true, NORM, HALF_OUT>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    fwd_kernel<D, true, NORM, HALF_OUT><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
 
     // pass R: dk, dv, dgamma, dS0
     BwdParams r;
-    if (!tile_map(&r.map_q, a.q, a.B, a.L, a.H, D) || !tile_map(&r.map_k, a.k, a.B, a.L, a.H, D) ||
-        !tile_map(&r.map_v, a.v, a.B, a.L, a.H, D) || !tile_map(&r.map_dy, dy16, a.B, a.L, a.H, D) ||
+    if (!tile_map(&r.map_q, a.q, a.B, a.L, a.H, BKV) || !tile_map(&r.map_k, a.k, a.B, a.L, a.H, BKV) ||
+        !tile_map(&r.map_v, a.v, a.B, a.L, a.H, BKV) || !tile_map(&r.map_dy, dy16, a.B, a.L, a.H, D) ||
         !tile_map_y(&r.map_dk, a.dk, a.B, a.L, a.H, HALF_OUT ? 64 : D) ||
         !tile_map_y(&r.map_dv, a.dv, a.B, a.L, a.H, HALF_OUT ? 64 : D))
         return MEMOROID_ERR_CUDA;
@@ -1994,8 +2053,8 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
 #ifdef MEMOROID_LA_TRACE
     r.trace = la_trace_buffer();
 #endif
-    if (set_smem(bwd_kernel<D, HALF_OUT>, BwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    bwd_kernel<D, HALF_OUT><<<static_cast<unsigned>(a.B * a.H * pl.G), kRThreads, BwdSmem<D>::BYTES, stream>>>(r);
+    if (set_smem(bwd_kernel<D, HALF_OUT, NORM>, BwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    bwd_kernel<D, HALF_OUT, NORM><<<static_cast<unsigned>(a.B * a.H * pl.G), kRThreads, BwdSmem<D>::BYTES, stream>>>(r);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     if (r.gpart != nullptr) {
         dgamma_head_kernel<<<static_cast<unsigned>((a.H + 127) / 128), 128, 0, stream>>>(gpart, a.gamma, a.dgamma,
@@ -2020,6 +2079,10 @@ memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream) {
     const Plan pl = make_plan(a.B, a.L, a.H);
     const Layout ly = make_layout(a.B, a.L, a.H, a.D);
     if (a.out_cols != 0 && !(a.out_cols == 64 && a.D == 128)) return MEMOROID_ERR_UNSUPPORTED;
+    if (a.norm) {
+        if (a.out_cols != 64 || a.grad_y16 == nullptr) return MEMOROID_ERR_UNSUPPORTED;
+        return launch_bwd_d<128, true, true>(a, pl, ly, stream);
+    }
     if (a.out_cols == 64) return launch_bwd_d<128, true>(a, pl, ly, stream);
     if (a.D == 64) return launch_bwd_d<64>(a, pl, ly, stream);
     if (a.D == 128) return launch_bwd_d<128>(a, pl, ly, stream);

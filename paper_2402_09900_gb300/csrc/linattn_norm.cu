@@ -254,12 +254,14 @@ int kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t d, int backward, i
     if (B == 0 || L == 0 || H == 0) return 0;
     // prep, the linear-attention call, then the divide (forward) or the upstream
     // gradient and the chain rule (backward); with states: their padding and
-    // unpadding.  The forward of 64-channel heads (y 16-byte aligned) is the fused call alone.
-    const bool fused = !backward && d == 64;
+    // unpadding.  The forward of 64-channel heads (y 16-byte aligned) is the fused
+    // call alone; their backward builds its operands in the kernels (no prep).
+    const bool pad = debug_knobs().lnorm_padded != 0;
+    const bool fused_fwd = !backward && d == 64 && !pad, no_prep = d == 64 && !pad;
     // the backward hands its bf16 upstream gradient to the linear-attention call,
     // which then skips its own bf16 copy
-    const int base = (fused ? 0 : 2 + (backward ? 1 : 0)) + la::kernels_per_call(B, L, H, backward, with_dgamma_per_head) -
-                     (backward ? 1 : 0);
+    const int base = (no_prep ? 0 : 1) + (backward ? 2 : (fused_fwd ? 0 : 1)) +
+                     la::kernels_per_call(B, L, H, backward, with_dgamma_per_head) - (backward ? 1 : 0);
     return base + (with_states ? (backward ? 3 : 2) : 0);
 }
 
@@ -269,7 +271,9 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
     // the forward of 64-channel heads applies phi, the padding and the division
     // inside the tensor-core kernel (la::Args::norm); everything else goes
     // through the padded operands
-    const bool fused = !a.backward && a.d == 64 && (reinterpret_cast<uintptr_t>(a.y) & 15u) == 0;  // y: TMA stores
+    // (the backward of 64-channel heads also builds its operands in the kernels)
+    const bool fused = debug_knobs().lnorm_padded == 0 &&
+                       (a.backward ? a.d == 64 : a.d == 64 && (reinterpret_cast<uintptr_t>(a.y) & 15u) == 0);  // y: TMA stores
     if (!fused)
         prep_kernel<<<grid_for(R * 16), 256, 0, s>>>(static_cast<const uint4*>(a.q), static_cast<const uint4*>(a.k),
                                                      static_cast<const uint4*>(a.v), R, static_cast<int>(a.d),
@@ -328,6 +332,12 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
     // heads of up to 64 channels need only the first 64 columns of dq', dk', dv'
     const int64_t wout = a.d <= 64 ? 64 : kW;
     l.out_cols = a.d <= 64 ? 64 : 0;
+    if (fused) {
+        l.q = a.q;
+        l.k = a.k;
+        l.v = a.v;
+        l.norm = 1;
+    }
     l.dq = b.dq;
     l.dk = b.dk;
     l.dv = b.dv;

@@ -77,6 +77,7 @@ SIGNATURES = {
     "memoroid_get_device_error": (_int, [_p, _p]),
     "memoroid_debug_set_wait_limit_ns": (None, [ctypes.c_uint64]),
     "memoroid_debug_withhold_tile": (None, [_i64]),
+    "memoroid_debug_lnorm_padded": (None, [_int]),
 }
 
 
@@ -339,6 +340,10 @@ def memoroid_debug_set_wait_limit_ns(ns: int) -> None:
 
 def memoroid_debug_withhold_tile(ticket: int) -> None:
     load().memoroid_debug_withhold_tile(int(ticket))
+
+
+def memoroid_debug_lnorm_padded(on: bool) -> None:
+    load().memoroid_debug_lnorm_padded(1 if on else 0)
 
 
 # ---------------------------------------------------------------------------
