@@ -667,7 +667,9 @@ def run_reference(args):
     oracle.build()
     t = tapegen.diag_config(CFG)
     per = _calibrate(t)
-    steps = int(min(t["L"], max(1024, args.ref_seconds / max(args.steps, 1) / per)))
+    # at most 2^18 steps per step: the oracle's rate is flat well below that, and
+    # its fp64 copies of a sample stay near 1 GB whatever --steps is
+    steps = int(min(t["L"], 1 << 18, max(1024, args.ref_seconds / max(args.steps, 1) / per)))
     s = oracle_sample(t, steps)
     for _ in range(args.warmup):
         time_oracle_step(oracle_sample(t, min(steps, 1024)))
