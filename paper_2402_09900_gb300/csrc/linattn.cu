@@ -500,8 +500,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     // to a [B, L, H, 64] output (the normalised path needs no more of dq')
     static_assert(!HALF_OUT || (D == 128 && BWD), "half-width output for pass F at d = 128");
     using S = FwdSmem<D>;
-    // NORM: the Linear Transformer with phi and its normalizer for heads of 64
-    // channels.  q, k, v are the unpadded [B, L, H, 64] tensors; each operand
+    // NORM without BWD: the forward of the Linear Transformer with phi and its
+    // normalizer for heads of 64 channels.  q, k, v are the unpadded [B, L, H, 64] tensors; each operand
     // slot holds them in its first 64 channels (one TMA box), phi is applied to
     // q and k in shared memory, the contractions over the q/k channels stop at
     // 64, the second half of the K slot holds zeros and that of the V slot the
