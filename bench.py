@@ -988,7 +988,7 @@ def main():
     ap.add_argument("--ffm-steps", type=int, default=20, help="timed FFM fwd+bwd steps")
     ap.add_argument("--ffm-tape-steps", type=int, default=0,
                     help="FFM tape length (profiler captures); 0 = the full L = 2^20 workload")
-    ap.add_argument("--la-cpu-steps", type=int, default=1 << 14,
+    ap.add_argument("--la-cpu-steps", type=int, default=1 << 16,
                     help="steps (whole episodes) of the linattn oracle baseline")
     ap.add_argument("--la-intra-reps", type=int, default=2000,
                     help="repetitions of the intra-tile contraction per CTA in the tensor benchmark")
