@@ -669,7 +669,35 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
 
     // phase 1: aggregate of this warp's steps, from the identity, in processing order
     float4 a = one2(), x = zero2();
-    if (landed) {
+    if (landed && C::FFM) {
+        // FFM (a constant lambda per channel): the aggregate's multiplier is lambda^n
+        // over the n steps after the last reset in processing order (lambda -> 1 at the
+        // tape's last step in reverse), taken once by repeated squaring
+        const uint32_t rv = rmask & ((nv >= 32) ? 0xffffffffu : ((1u << nv) - 1u));
+        if (!C::REV) {
+#pragma unroll C::UNROLL
+            for (int k = 0; k < R; ++k) {
+                if (k < nv) {
+                    const float4 uu = ffm_x_pair(p, s_in, warp * R + k, lane);
+                    x = ((rmask >> k) & 1u) ? uu : cfma2(lam, x, uu);
+                }
+            }
+            a = cpow2(lam, rv ? nv - (31 - __clz(rv)) : nv);
+        } else {
+#pragma unroll C::UNROLL
+            for (int kk = 0; kk < R; ++kk) {
+                const int k = R - 1 - kk;
+                if (k < nv) {
+                    const float4 gg = ffm_planar_pair<C::T>(s_in, warp * R + k, lane);
+                    const float4 m = (ts + k == p.L - 1) ? one2() : mlam;
+                    x = ((rmask >> k) & 1u) ? gg : cfma2(m, x, gg);
+                }
+            }
+            const int cnt = rv ? __ffs(rv) : nv;  // steps k < cnt multiply the carry
+            const int64_t kl = p.L - 1 - ts;      // the tape's last step, if in this warp
+            a = cpow2(mlam, cnt - ((kl >= 0 && kl < cnt) ? 1 : 0));
+        }
+    } else if (landed) {
         if (!C::REV) {
 #pragma unroll C::UNROLL
             for (int k = 0; k < R; ++k) {
@@ -996,26 +1024,26 @@ __global__ void __launch_bounds__(128) segment_fix_kernel(const Params p) {
     if (ptx::ld_relaxed(p.hdr) != 0u) return;
     const int64_t n_fix = static_cast<int64_t>(ptx::ld_relaxed(p.hdr + 4));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (C::PS) {
+    if constexpr (C::PS) {
         // per-step lambda: one warp per tile
         const int64_t nw = static_cast<int64_t>(gridDim.x) * 4;
         for (int64_t f = static_cast<int64_t>(blockIdx.x) * 4 + warp; f < n_fix; f += nw)
             segment_fix_tile<C>(p, static_cast<int64_t>(p.fix[f]), 0, 1, nullptr);
-        return;
-    }
-    // per-channel lambda: the four warps of a CTA split a tile's rows
-    __shared__ float4 gl[4 * 32];
-    for (int64_t f = blockIdx.x; f < n_fix; f += gridDim.x) {
-        const int64_t tid = static_cast<int64_t>(p.fix[f]);
-        segment_fix_tile<C>(p, tid, warp, 4, C::REV ? gl : nullptr);
-        if (C::REV) {
-            __syncthreads();
-            const int64_t c2 = (tid / p.n_tt % p.n_slabs) * (SLAB / 2);
-            if (warp == 0 && lane < lmin(SLAB / 2, p.D2 - c2)) {
-                const float4 sum = add2(add2(gl[lane], gl[32 + lane]), add2(gl[64 + lane], gl[96 + lane]));
-                p.gpart[tid * 32 + lane] = add2(p.gpart[tid * 32 + lane], sum);
+    } else {
+        // per-channel lambda: the four warps of a CTA split a tile's rows
+        __shared__ float4 gl[4 * 32];
+        for (int64_t f = blockIdx.x; f < n_fix; f += gridDim.x) {
+            const int64_t tid = static_cast<int64_t>(p.fix[f]);
+            segment_fix_tile<C>(p, tid, warp, 4, C::REV ? gl : nullptr);
+            if (C::REV) {
+                __syncthreads();
+                const int64_t c2 = (tid / p.n_tt % p.n_slabs) * (SLAB / 2);
+                if (warp == 0 && lane < lmin(SLAB / 2, p.D2 - c2)) {
+                    const float4 sum = add2(add2(gl[lane], gl[32 + lane]), add2(gl[64 + lane], gl[96 + lane]));
+                    p.gpart[tid * 32 + lane] = add2(p.gpart[tid * 32 + lane], sum);
+                }
+                __syncthreads();
             }
-            __syncthreads();
         }
     }
 }
