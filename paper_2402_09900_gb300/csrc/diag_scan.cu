@@ -669,16 +669,16 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
 
     // phase 1: aggregate of this warp's steps, from the identity, in processing order
     float4 a = one2(), x = zero2();
-    if (landed && C::FFM) {
-        // FFM (a constant lambda per channel): the aggregate's multiplier is lambda^n
-        // over the n steps after the last reset in processing order (lambda -> 1 at the
-        // tape's last step in reverse), taken once by repeated squaring
+    if (landed && !C::PS) {
+        // a constant lambda per channel: the aggregate's multiplier is lambda^n over the
+        // n steps after the last reset in processing order (lambda -> 1 at the tape's
+        // last step in reverse), taken once by repeated squaring
         const uint32_t rv = rmask & ((nv >= 32) ? 0xffffffffu : ((1u << nv) - 1u));
         if (!C::REV) {
 #pragma unroll C::UNROLL
             for (int k = 0; k < R; ++k) {
                 if (k < nv) {
-                    const float4 uu = ffm_x_pair(p, s_in, warp * R + k, lane);
+                    const float4 uu = C::FFM ? ffm_x_pair(p, s_in, warp * R + k, lane) : sin[k * 32];
                     x = ((rmask >> k) & 1u) ? uu : cfma2(lam, x, uu);
                 }
             }
@@ -688,7 +688,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
             for (int kk = 0; kk < R; ++kk) {
                 const int k = R - 1 - kk;
                 if (k < nv) {
-                    const float4 gg = ffm_planar_pair<C::T>(s_in, warp * R + k, lane);
+                    const float4 gg = C::FFM ? ffm_planar_pair<C::T>(s_in, warp * R + k, lane) : sin[k * 32];
                     const float4 m = (ts + k == p.L - 1) ? one2() : mlam;
                     x = ((rmask >> k) & 1u) ? gg : cfma2(m, x, gg);
                 }
@@ -698,12 +698,13 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
             a = cpow2(mlam, cnt - ((kl >= 0 && kl < cnt) ? 1 : 0));
         }
     } else if (landed) {
+        // a lambda per step: the multiplier is the running product
         if (!C::REV) {
 #pragma unroll C::UNROLL
             for (int k = 0; k < R; ++k) {
                 if (k < nv) {
-                    const float4 uu = C::FFM ? ffm_x_pair(p, s_in, warp * R + k, lane) : sin[k * 32];
-                    const float4 ll = C::PS ? sl[k * 32] : lam;
+                    const float4 uu = sin[k * 32];
+                    const float4 ll = sl[k * 32];
                     if ((rmask >> k) & 1u) {
                         a = ll;
                         x = uu;
@@ -718,8 +719,8 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
             for (int kk = 0; kk < R; ++kk) {
                 const int k = R - 1 - kk;
                 if (k < nv) {
-                    const float4 gg = C::FFM ? ffm_planar_pair<C::T>(s_in, warp * R + k, lane) : sin[k * 32];
-                    const float4 m = (ts + k == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
+                    const float4 gg = sin[k * 32];
+                    const float4 m = (ts + k == p.L - 1) ? one2() : conj2(sl[k * 32]);
                     if ((rmask >> k) & 1u) {
                         a = m;
                         x = gg;
