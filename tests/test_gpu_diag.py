@@ -110,6 +110,22 @@ def test_resets_on_tile_edges():
     check(t, g_last=t["grad_h_last"])
 
 
+@pytest.mark.parametrize("per_step", [False, True])
+@pytest.mark.parametrize("period", [5, 13, 37, 50])
+@pytest.mark.parametrize("L", [997, 1152])
+def test_periodic_resets_every_row_offset(per_step, period, L):
+    # begin flags every `period` steps, at two phases: across the scan warps' row
+    # blocks (24 steps forward, 12 backward) a flag falls on every position of a
+    # block, some blocks hold none, and the tape ends inside a block (997) or on a
+    # tile edge (1152 = 12 x 96); tape 1 continues an episode from h0
+    t = tapegen.diag_tape(2, L, 64, seed=12 + period + L, start_mode="none", lambda_per_step=per_step,
+                          with_h0=True)
+    t["start"][0, ::period] = 1
+    t["start"][1, :] = 0
+    t["start"][1, period // 2::period] = 1
+    check(t, h0=t["h0"], g_last=t["grad_h_last"])
+
+
 @pytest.mark.parametrize("L", [1, 2, 31, 33, 95, 96, 97, 191, 193])
 def test_tiny_tapes(L):
     t = tapegen.diag_tape(2, L, 4, seed=10 + L, mean=3.0, with_h0=True)

@@ -95,6 +95,19 @@ def test_ffm_degenerate_flags(mode):
     check(t, with_S0=True)
 
 
+@pytest.mark.parametrize("period", [7, 31, 32, 45])
+def test_ffm_periodic_resets_every_row_offset(period):
+    # begin flags every `period` steps at two phases: a flag falls on every position
+    # of the scan warps' row blocks (31 steps forward, 12 backward), some blocks hold
+    # none, and the tape ends inside a block; row 1 continues an episode from S0
+    t = tapegen.ffm_tape(2, 1001, 16, 4, tapegen.seed_for(740 + period), start_mode="none", with_S0=True)
+    t["start"][0, :] = 0
+    t["start"][0, ::period] = 1
+    t["start"][1, :] = 0
+    t["start"][1, period // 2::period] = 1
+    check(t, with_S0=True)
+
+
 @pytest.mark.parametrize("L", [1, 2, 95, 96, 97, 185, 186, 187, 373])
 def test_ffm_tiny_tapes(L):
     # around the forward's 186-step and the backward's 96-step tile edges
