@@ -1,5 +1,6 @@
 // ptx.cuh -- thin inline-PTX wrappers used by the sm_103a kernels:
-// mbarriers, TMA bulk copies, acquire/release flag words, the global timer.
+// mbarriers, TMA bulk and tensor copies, tcgen05 (TMEM allocation, MMA, loads),
+// relaxed flag and summary words, named barriers, the global timer.
 #pragma once
 #include <cstdint>
 
@@ -23,9 +24,6 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
                  "r"(bytes)
                  : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     uint32_t ok;
@@ -79,29 +77,16 @@ __device__ __forceinline__ void tma_store_4d(const void* map, uint32_t src_smem,
                  "r"(src_smem), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
                  : "memory");
 }
-// Brings the 128-byte line holding `ptr` into L2 (no register is written).
-__device__ __forceinline__ void prefetch_l2(const void* ptr) { asm volatile("prefetch.global.L2 [%0];" ::"l"(ptr)); }
 __device__ __forceinline__ void prefetch_tensormap(const void* map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
 }
 
 // ---- flags ---------------------------------------------------------------------
-__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
-    uint32_t v;
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v) {
-    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
 __device__ __forceinline__ uint32_t ld_relaxed(const uint32_t* p) {
     uint32_t v;
     asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
-
-// Acquire / release fences at GPU scope.
-__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
 
 // ---- named barriers over a subset of the CTA's warps ---------------------------
 __device__ __forceinline__ void named_sync(int id, int nthreads) {
@@ -120,19 +105,6 @@ __device__ __forceinline__ void ld_relaxed_v2u64(const unsigned long long* p, un
 __device__ __forceinline__ void st_relaxed_v2u64(unsigned long long* p, unsigned long long a,
                                                  unsigned long long b) {
     asm volatile("st.relaxed.gpu.global.v2.u64 [%0], {%1, %2};" ::"l"(p), "l"(a), "l"(b) : "memory");
-}
-
-// ---- cp.async (16-byte global -> shared copies, per thread) ---------------------
-// src_bytes 0 fills the 16 destination bytes with zeros and reads nothing.
-__device__ __forceinline__ void cp_async16(uint32_t dst_smem, const void* src, bool valid) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst_smem), "l"(src),
-                 "r"(valid ? 16 : 0)
-                 : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
 // ---- bulk shared -> global stores (TMA, untiled) ---------------------------------
