@@ -2075,8 +2075,9 @@ int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_dga
 }
 
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream) {
-    if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, stream) != cudaSuccess) return MEMOROID_ERR_CUDA;
     const Plan pl = make_plan(a.B, a.L, a.H);
+    if (a.B * a.H * pl.G >= 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;  // one CTA per segment chain
+    if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, stream) != cudaSuccess) return MEMOROID_ERR_CUDA;
     const Layout ly = make_layout(a.B, a.L, a.H, a.D);
     if (a.out_cols != 0 && !(a.out_cols == 64 && a.D == 128)) return MEMOROID_ERR_UNSUPPORTED;
     if (a.norm) {
@@ -2091,8 +2092,9 @@ memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream) {
 
 memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream) {
     if (a.norm && a.D != 128) return MEMOROID_ERR_UNSUPPORTED;
-    if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, stream) != cudaSuccess) return MEMOROID_ERR_CUDA;
     const Plan pl = make_plan(a.B, a.L, a.H);
+    if (a.B * a.H * pl.G >= 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;  // one CTA per segment chain
+    if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, stream) != cudaSuccess) return MEMOROID_ERR_CUDA;
     const Layout ly = make_layout(a.B, a.L, a.H, a.D);
     if (a.norm) return launch_fwd_d<128, true>(a, pl, ly, stream);
     if (a.D == 64) return launch_fwd_d<64>(a, pl, ly, stream);
