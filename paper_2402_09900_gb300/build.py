@@ -29,12 +29,9 @@ def nvcc() -> str:
     return cand
 
 
-def _flags(debug: bool):
-    f = ["-std=c++17", "-O3", "-lineinfo", "-Xcompiler", "-fPIC,-O2", "--expt-relaxed-constexpr",
-         "-I", INCLUDE, "-I", CSRC] + ARCH
-    if debug:
-        f += ["-DMEMOROID_DEBUG=1"]
-    return f
+def _flags():
+    return ["-std=c++17", "-O3", "-lineinfo", "-Xcompiler", "-fPIC,-O2", "--expt-relaxed-constexpr",
+            "-I", INCLUDE, "-I", CSRC] + ARCH
 
 
 def _newest_input_mtime():
@@ -48,13 +45,13 @@ def lib_path() -> str:
     return os.path.join(OUT_DIR, LIB_NAME)
 
 
-def build(force: bool = False, verbose: bool = False, debug: bool = False, ptxas_info: bool = False) -> str:
+def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) -> str:
     out = lib_path()
     if not force and os.path.exists(out) and os.path.getmtime(out) >= _newest_input_mtime():
         return out
     os.makedirs(OUT_DIR, exist_ok=True)
     cc = nvcc()
-    flags = _flags(debug)
+    flags = _flags()
     if ptxas_info:
         flags = flags + ["-Xptxas", "-v"]
 

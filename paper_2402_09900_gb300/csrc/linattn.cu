@@ -411,25 +411,8 @@ struct FwdParams {
     // backward pass F only (see fwd_kernel<D, true>)
     float* dlam_f;       // [B, L, H]: the state-side terms of dL/dlog(gamma_t)
     uint16_t* states;    // [B, H, n_tiles, D, D] bf16: S_{c-1}^T before tiles without a begin flag
-#ifdef MEMOROID_LA_TRACE
-    unsigned long long* trace;  // per-phase nanoseconds of CTA 0, thread 0
-#endif
 };
 
-#ifdef MEMOROID_LA_TRACE
-#define LA_MARK(i)                                  \
-    do {                                            \
-        if (trace_on) {                             \
-            const uint64_t now_ = globaltimer();    \
-            tr[i] += now_ - tr_last;                \
-            tr_last = now_;                         \
-        }                                           \
-    } while (0)
-#else
-#define LA_MARK(i) \
-    do {           \
-    } while (0)
-#endif
 
 // Thread -> row of a D x D state accumulator in TMEM.  With M = 128 the row
 // is the TMEM lane; with M = 64 rows 16q..16q+15 sit in lanes 32q..32q+15 and
@@ -663,11 +646,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     uint32_t drain_par = 0;
     bool q_pending = false;  // pass F: a q tile load not seen complete
     uint32_t q_par = 0;
-#ifdef MEMOROID_LA_TRACE
-    const bool trace_on = blockIdx.x == 0 && tid == 0 && p.trace != nullptr;
-    unsigned long long tr[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-    uint64_t tr_last = globaltimer();
-#endif
 #pragma unroll 1
     for (int c = 0; c < nt && !failed; ++c) {
         const int s = c & 1;
@@ -682,7 +660,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         }
         pending = -1;
         tc::fence_after();
-        LA_MARK(0);
         if (NORM) {
             // phi on the loaded q and k (the forward) or k (pass F), in place
             const int64_t valid = p.L - (tile0 + c) * T;
@@ -711,7 +688,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 tc::mma(tm + S::COL_P, desc_sw_k(sq, kk), desc_sw_k(sk, kk), ID_QK, kk > 0);
             tc::commit(bar1);
         }
-        LA_MARK(1);
         ok = wait_mbar(bar1, c & 1, p.wait_ns) && !(c == 0 && static_cast<int64_t>(blockIdx.x) == p.fail_cta);
         if (__syncthreads_or(!ok)) {
             failed = true;
@@ -730,7 +706,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             }
             q_pending = true;
         }
-        LA_MARK(2);
 
         // ---- mask: Pm[t][r] = [seg_t <= r <= t] exp2(lam2_t - lam2_r) P[t][r] ----
         {
@@ -755,7 +730,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 store_bf16x16(pm, core_off(t, r0, T), core_off(t, r0 + 8, T), v);
             }
         }
-        LA_MARK(3);
         // ---- K~[r] = exp2(lam2_end - lam2_r) K[r] for rows of the last episode ----
         {
             const float lend = mc.lam2[T - 1];
@@ -790,7 +764,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 tc::mma(tm + S::COL_S, desc_sw_mn(sk, kk), desc_sw_mn(sv, kk), ID_KV, acc || kk > 0);
             tc::commit(bar2);
         }
-        LA_MARK(4);
         const int64_t t0 = (tile0 + c) * T;
         ok = wait_mbar(bar2, c & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
@@ -809,7 +782,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             q_pending = false;
             q_par ^= 1;
         }
-        LA_MARK(5);
 
         // ---- y = Y_intra + w_in * Y_inter, staged as fp32 rows in stage s ----
         // rows of this tile that belong to the segment
@@ -955,12 +927,10 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 }
             }
         }
-        LA_MARK(6);
         // ---- bulk-store the staged output rows ----
         tc::fence_smem_to_async();
         tc::fence_before();
         __syncthreads();
-        LA_MARK(7);
         if (warp == 0) {
             const int full_rows = static_cast<int>(min(static_cast<int64_t>(T), p.L - t0));
             if (r_lo == 0 && r_hi == full_rows) {
@@ -1020,11 +990,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         if (q_pending) wait_mbar(qbar, q_par, kDrainNs);
     }
     if (warp == 0) bulk_wait_all();
-#ifdef MEMOROID_LA_TRACE
-    if (trace_on) {
-        for (int i = 0; i < 8; ++i) p.trace[i] = tr[i];
-    }
-#endif
     tc::fence_before();
     __syncthreads();
     tc::fence_after();
@@ -1111,9 +1076,6 @@ struct BwdParams {
     int G;
     uint64_t wait_ns;
     int64_t fail_cta;  // test knob (see FwdParams)
-#ifdef MEMOROID_LA_TRACE
-    unsigned long long* trace;
-#endif
 };
 
 // Reduces 32 values per lane over the warp's 32 lanes; lane l ends with the
@@ -1300,11 +1262,6 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     uint32_t drain_par = 0;
     uint32_t ph4 = 0;           // phase of bar4 (committed only on tiles with a reverse state)
     int it = 0;
-#ifdef MEMOROID_LA_TRACE
-    const bool trace_on = blockIdx.x == 0 && tid == 0 && p.trace != nullptr;
-    unsigned long long tr[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-    uint64_t tr_last = globaltimer();
-#endif
 #pragma unroll 1
     for (int64_t tile = tile_hi - 1; tile >= tile_lo; --tile, ++it) {
         const int64_t t0 = tile * T;
@@ -1326,7 +1283,6 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
             tc::fence_smem_to_async();
             __syncthreads();
         }
-        LA_MARK(0);
         const bool tile_start = mc.has_start != 0;
 
         // ---- B1: P = Q K^T, dP = dY V^T, dKi = V G^T ----
@@ -1395,7 +1351,6 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
             break;
         }
         tc::fence_after();
-        LA_MARK(1);
 
         // ---- RP1: masks and E statistics; x_r; <G_c, S_{c-1}> and G *= a ----
         {
@@ -1480,7 +1435,6 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         tc::fence_before();
         __syncthreads();
         tc::fence_after();
-        LA_MARK(2);
 
         // ---- B2: dV = Pm^T dY + K~ G, dK = dPm^T Q ----
         if (tid == 0) {
@@ -1541,7 +1495,6 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
             break;
         }
         tc::fence_after();
-        LA_MARK(3);
 
         // ---- RP2: Q~ = w_in (.) Q in place, then B3: G += Q~^T dY ----
         scale_rows_sw<D, kRThreads>(smem + S::OFF_Q, tid,
@@ -1557,7 +1510,6 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
                 tc::mma(tm + S::COL_G, desc_sw_mn(sQ, kk), desc_sw_mn(sDY, kk), ID_QDY, acc || kk > 0);
             tc::commit(bar3);
         }
-        LA_MARK(4);
 
         // ---- epilogue (while B3 runs): dk = dK + w_out dKi, then dv, each staged and
         // stored on its own, so that the dk stores drain while dv is staged ----
@@ -1639,7 +1591,6 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
             for (int off = 16; off > 0; off >>= 1) dl += __shfl_xor_sync(0xffffffffu, dl, off);
             if (lane == 0) st_iv[16 + warp] = dl;
         }
-        LA_MARK(5);
         tc::fence_smem_to_async();  // the statistics in the V tile are overwritten by the next tile's load
         ok = wait_mbar(bar3, it & 1, p.wait_ns);
         if (__syncthreads_or(!ok)) {
@@ -1649,7 +1600,6 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
             break;
         }
         tc::fence_after();
-        LA_MARK(6);
         const bool next = tile > tile_lo;
         if (tid == 0) {
             gsum += (st_iv[16] + st_iv[17]) + (st_iv[18] + st_iv[19]);
@@ -1700,13 +1650,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         }
         tc::fence_before();
         __syncthreads();
-        LA_MARK(7);
     }
-#ifdef MEMOROID_LA_TRACE
-    if (trace_on) {
-        for (int i = 0; i < 8; ++i) p.trace[8 + i] = tr[i];
-    }
-#endif
     if (failed) {
         if (tid == 0) record_error(p.hdr, DEV_MMA_TIMEOUT);
         // let work still in flight finish before the CTA's TMEM and shared memory go away
@@ -1846,14 +1790,6 @@ memoroid_status_t launch_intra_bench(int64_t D, int64_t reps, int64_t ctas, void
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
-#ifdef MEMOROID_LA_TRACE
-__device__ unsigned long long g_la_trace[16];
-unsigned long long* la_trace_buffer() {
-    void* ptr = nullptr;
-    cudaGetSymbolAddress(&ptr, g_la_trace);
-    return static_cast<unsigned long long*>(ptr);
-}
-#endif
 namespace {
 template <typename K>
 cudaError_t set_smem(K kernel, int bytes) {
@@ -1955,9 +1891,6 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     p.map_zq = p.map_q;  // not read by the forward
     p.dlam_f = nullptr;
     p.states = nullptr;
-#ifdef MEMOROID_LA_TRACE
-    p.trace = la_trace_buffer();
-#endif
     if (set_smem(fwd_kernel<D, false, NORM>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
     fwd_kernel<D, false, NORM><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
@@ -2012,9 +1945,6 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     f.fail_cta = debug_knobs().withhold_ticket;
     f.dlam_f = dlam_f;
     f.states = states;
-#ifdef MEMOROID_LA_TRACE
-    f.trace = la_trace_buffer();  // pass F's phases replace the forward's in slots 0-7
-#endif
     if (set_smem(fwd_kernel<D, true, NORM, HALF_OUT>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
     fwd_kernel<D, true, NORM, HALF_OUT><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
@@ -2050,9 +1980,6 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     r.G = static_cast<int>(pl.G);
     r.wait_ns = debug_knobs().wait_ns;
     r.fail_cta = debug_knobs().withhold_ticket;
-#ifdef MEMOROID_LA_TRACE
-    r.trace = la_trace_buffer();
-#endif
     if (set_smem(bwd_kernel<D, HALF_OUT, NORM>, BwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
     bwd_kernel<D, HALF_OUT, NORM><<<static_cast<unsigned>(a.B * a.H * pl.G), kRThreads, BwdSmem<D>::BYTES, stream>>>(r);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
@@ -2077,13 +2004,12 @@ int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_dga
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream) {
     const Plan pl = make_plan(a.B, a.L, a.H);
     if (a.B * a.H * pl.G >= 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;  // one CTA per segment chain
+    if (a.out_cols != 0 && !(a.out_cols == 64 && a.D == 128)) return MEMOROID_ERR_UNSUPPORTED;
+    if (a.norm && (a.out_cols != 64 || a.grad_y16 == nullptr)) return MEMOROID_ERR_UNSUPPORTED;
+    if (a.D != 64 && a.D != 128) return MEMOROID_ERR_UNSUPPORTED;
     if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, stream) != cudaSuccess) return MEMOROID_ERR_CUDA;
     const Layout ly = make_layout(a.B, a.L, a.H, a.D);
-    if (a.out_cols != 0 && !(a.out_cols == 64 && a.D == 128)) return MEMOROID_ERR_UNSUPPORTED;
-    if (a.norm) {
-        if (a.out_cols != 64 || a.grad_y16 == nullptr) return MEMOROID_ERR_UNSUPPORTED;
-        return launch_bwd_d<128, true, true>(a, pl, ly, stream);
-    }
+    if (a.norm) return launch_bwd_d<128, true, true>(a, pl, ly, stream);
     if (a.out_cols == 64) return launch_bwd_d<128, true>(a, pl, ly, stream);
     if (a.D == 64) return launch_bwd_d<64>(a, pl, ly, stream);
     if (a.D == 128) return launch_bwd_d<128>(a, pl, ly, stream);
@@ -2094,6 +2020,7 @@ memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream) {
     if (a.norm && a.D != 128) return MEMOROID_ERR_UNSUPPORTED;
     const Plan pl = make_plan(a.B, a.L, a.H);
     if (a.B * a.H * pl.G >= 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;  // one CTA per segment chain
+    if (a.D != 64 && a.D != 128) return MEMOROID_ERR_UNSUPPORTED;
     if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, stream) != cudaSuccess) return MEMOROID_ERR_CUDA;
     const Layout ly = make_layout(a.B, a.L, a.H, a.D);
     if (a.norm) return launch_fwd_d<128, true>(a, pl, ly, stream);
@@ -2105,9 +2032,3 @@ memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream) {
 }  // namespace la
 }  // namespace memoroid
 
-#ifdef MEMOROID_LA_TRACE
-// trace builds only: copies the forward kernel's per-phase times to the host
-extern "C" void memoroid_debug_la_trace(unsigned long long* host_out) {
-    cudaMemcpy(host_out, memoroid::la::la_trace_buffer(), 16 * sizeof(unsigned long long), cudaMemcpyDeviceToHost);
-}
-#endif
