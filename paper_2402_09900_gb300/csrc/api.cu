@@ -3,9 +3,10 @@
 #include <cuda_runtime.h>
 
 #include <atomic>
-#include <chrono>
 #include <cstdint>
+#include <map>
 #include <mutex>
+#include <utility>
 
 #include "internal.cuh"
 
@@ -16,10 +17,18 @@ constexpr uint64_t kDefaultWaitNs = 1000000000ull;  // 1 s
 std::atomic<uint64_t> g_wait_ns{kDefaultWaitNs};
 std::atomic<int64_t> g_withhold{-1};
 std::atomic<int> g_lnorm_padded{0};
-// seeded from the clock so that two processes sharing a workspace are
-// unlikely to reuse each other's tags
-std::atomic<uint32_t> g_epoch{static_cast<uint32_t>(
-    std::chrono::steady_clock::now().time_since_epoch().count() * 2654435761ull)};
+// Launch counter: bits 0..30 are the launch's tag, the bits above count the
+// times the tag has wrapped ("generation").
+std::atomic<uint64_t> g_epoch{1};
+// Per (device, workspace address): the generation in which this process last
+// cleared the workspace's tagged region, and how far that clear reached.
+struct Cleared {
+    uint64_t generation;
+    size_t end;
+};
+std::mutex g_cleared_mutex;
+std::map<std::pair<int, uintptr_t>, Cleared> g_cleared;
+constexpr size_t kMaxClearedEntries = 4096;
 
 inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 inline cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
@@ -41,10 +50,21 @@ EncodeTiledFn encode_tiled() {
     return fn;
 }
 
-uint32_t next_epoch() {
-    uint32_t e = 0;
-    while (e == 0) e = g_epoch.fetch_add(1u) & 0x7fffffffu;
-    return e;
+uint32_t tagged_epoch(const void* workspace, size_t region_end, bool* clear) {
+    uint64_t c = 0;
+    while ((c & 0x7fffffffull) == 0) c = g_epoch.fetch_add(1u);
+    const uint64_t generation = c >> 31;
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) dev = -1;
+    const std::pair<int, uintptr_t> key{dev, reinterpret_cast<uintptr_t>(workspace)};
+    std::lock_guard<std::mutex> lock(g_cleared_mutex);
+    auto it = g_cleared.find(key);
+    *clear = it == g_cleared.end() || it->second.generation != generation || it->second.end < region_end;
+    if (*clear) {
+        if (it == g_cleared.end() && g_cleared.size() >= kMaxClearedEntries) g_cleared.clear();  // forget, clear again later
+        g_cleared[key] = Cleared{generation, region_end};
+    }
+    return static_cast<uint32_t>(c & 0x7fffffffull);
 }
 
 }  // namespace memoroid

@@ -76,23 +76,12 @@ constexpr int SLAB = 64;  // complex channels per slab
 // x alone (4 floats) with a per-channel lambda, whose a is lambda^(steps in
 // the summary's range) and is recomputed by the reader.
 constexpr int NODE_WORDS = 8;
-#ifndef MEMOROID_NODE_BATCH
-#define MEMOROID_NODE_BATCH 1  // summaries read per round trip in a look-back fold
-#endif
-constexpr int NB_READ = MEMOROID_NODE_BATCH;
+constexpr int NB_READ = 1;  // summaries read per round trip in a look-back fold
 // Unroll factors of the per-step loops (measured: unrolling helps the
 // backward scan and slows the forward one).
-#ifndef MEMOROID_UNROLL_FWD
-#define MEMOROID_UNROLL_FWD 1
-#endif
-#ifndef MEMOROID_UNROLL_BWD
-#define MEMOROID_UNROLL_BWD 32
-#endif
+constexpr int UNROLL_FWD = 1;
+constexpr int UNROLL_BWD = 32;
 constexpr int RED_PARTS = 512;  // first-stage parts of the grad_lambda reduction
-
-#ifndef MEMOROID_POLL_SLEEP_NS
-#define MEMOROID_POLL_SLEEP_NS 0  // longest back-off between flag polls
-#endif
 
 
 struct Params {
@@ -230,7 +219,7 @@ struct Cfg {
     static constexpr int W = W_, R = R_, T = W_ * R_;
     static constexpr bool REV = REV_, PS = PS_, FFM = FFM_;
     static_assert(!(PS_ && FFM_), "the FFM multiplier is per channel");
-    static constexpr int UNROLL = REV_ ? MEMOROID_UNROLL_BWD : MEMOROID_UNROLL_FWD;
+    static constexpr int UNROLL = REV_ ? UNROLL_BWD : UNROLL_FWD;
     // arrays staged per tile: input [, h (backward)] [, lambda (per step)]
     static constexpr int NB = 1 + (REV_ ? 1 : 0) + (PS_ ? 1 : 0);
     // float4 per staged array: a 512-byte row per step, or for the FFM forward
@@ -272,13 +261,8 @@ __device__ __forceinline__ Tile decode(const Params& p, int64_t tk) {
     t.tk = tk;
     const int64_t q = tk / p.n_sc;
     const int64_t sc = tk - q * p.n_sc;
-#ifndef MEMOROID_CHAIN_MAJOR
     t.g = sc / p.n_chains;
     t.chain = sc - t.g * p.n_chains;
-#else
-    t.chain = sc / p.n_seg;
-    t.g = sc - t.chain * p.n_seg;
-#endif
     t.pos = q;
     const int64_t jg = t.g * p.q_seg + q;  // position in the whole chain
     t.valid = (q < p.q_seg) && (jg < p.n_tt);
@@ -291,29 +275,6 @@ __device__ __forceinline__ Tile decode(const Params& p, int64_t tk) {
     t.fbase = sc * p.q_seg;
     return t;
 }
-
-// ---- optional per-tile timeline (tuning builds only) ---------------------------
-#ifdef MEMOROID_TRACE
-__device__ unsigned long long* g_trace;  // [ticket][16] global-timer stamps
-#define TRACE_TK(ticket, slot)                                                                   \
-    do {                                                                                         \
-        if (g_trace != nullptr && (threadIdx.x & 31) == 0 && (slot) >= 0)                        \
-            g_trace[(ticket) * 16 + (slot)] = static_cast<unsigned long long>(ptx::globaltimer()); \
-    } while (0)
-#else
-#define TRACE_TK(ticket, slot) (void)0
-#endif
-#define TRACE(slot) TRACE_TK(tk, slot)
-
-// ---- optional wait profiling (tuning builds only) -----------------------------
-#ifdef MEMOROID_PROFILE_WAITS
-#define PROF_T0() const uint64_t _pt0 = ptx::globaltimer()
-#define PROF_ADD(slot) atomicAdd(reinterpret_cast<unsigned long long*>(p.hdr + 32) + (slot), \
-                                 static_cast<unsigned long long>(ptx::globaltimer() - _pt0))
-#else
-#define PROF_T0() (void)0
-#define PROF_ADD(slot) (void)0
-#endif
 
 // ---- errors and bounded waits -------------------------------------------------
 __device__ __forceinline__ void record_error(const Params& p, uint32_t code, int64_t ticket) {
@@ -386,10 +347,10 @@ __device__ __forceinline__ bool load_node(const Params& p, int64_t fbase, int64_
 // node o R = (R.a * node.a, R.a * node.x + R.x, node.b) while R holds no begin
 // flag.  The fold stops after the first node whose range holds one (every
 // node further left would be discarded by the select of Theorem 3.2, so
-// stopping changes no bit).  Nodes are read four at a time and re-read until
-// every lane sees them complete.  Warp-wide; false on timeout / error.
+// stopping changes no bit).  Nodes are read NB_READ at a time and re-read
+// until every lane sees them complete.  Warp-wide; false on timeout / error.
 __device__ bool fold_nodes(const Params& p, int64_t fbase, int64_t mypos, int n, float4 mul, int rag,
-                           float4& Ra, float4& Rx, bool& Rb, int64_t ticket, int trace_slot = -1) {
+                           float4& Ra, float4& Rx, bool& Rb, int64_t ticket) {
     for (int m0 = 0; m0 < n && !Rb; m0 += NB_READ) {
         int64_t pk[NB_READ];
 #pragma unroll
@@ -416,7 +377,6 @@ __device__ bool fold_nodes(const Params& p, int64_t fbase, int64_t mypos, int n,
                     return false;
                 }
             }
-            if (MEMOROID_POLL_SLEEP_NS > 0) __nanosleep(MEMOROID_POLL_SLEEP_NS);
         }
 #pragma unroll
         for (int k = 0; k < NB_READ; ++k) {
@@ -427,7 +387,6 @@ __device__ bool fold_nodes(const Params& p, int64_t fbase, int64_t mypos, int n,
             }
         }
     }
-    TRACE_TK(ticket, trace_slot);
     return true;
 }
 
@@ -446,7 +405,7 @@ __device__ bool fenwick_children(const Params& p, int64_t fbase, int64_t pos, fl
     Cb = false;
     if (nc == 0) return true;
     const int64_t child = pos - (int64_t(1) << (lane < nc ? lane : 0));
-    return fold_nodes(p, fbase, child, nc, mul, rag, Ca, Cx, Cb, ticket, 9);
+    return fold_nodes(p, fbase, child, nc, mul, rag, Ca, Cx, Cb, ticket);
 }
 
 // Publishes node j+1 = C o T (T: the tile's own aggregate) unless !ok or the
@@ -472,7 +431,7 @@ __device__ bool fenwick_carry(const Params& p, int64_t fbase, int64_t j, float4 
     Rx = zero2();
     Ra = one2();
     Rb = false;
-    if (!fold_nodes(p, fbase, q, nq, mul, rag, Ra, Rx, Rb, ticket, 8)) return false;
+    if (!fold_nodes(p, fbase, q, nq, mul, rag, Ra, Rx, Rb, ticket)) return false;
     carry = Rb ? Rx : cfma2(Ra, base, Rx);
     return true;
 }
@@ -516,7 +475,6 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
     float4 node_mul = one2();
     if (!C::PS && lane_ok) node_mul = C::REV ? conj2(p.lambda[t.c2 + lane]) : p.lambda[t.c2 + lane];
     const int node_rag = (t.g == 0) ? p.rag : 0;
-    if (warp == 0) TRACE(0);
 
     if (warp == LB_PUBLISH) {
         // ----------------------------------------- stage the tile, publish its summary
@@ -547,9 +505,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
         float4 Ca, Cx;
         bool Cb;
         bool ok = fenwick_children(p, t.fbase, t.pos + 1, node_mul, node_rag, Ca, Cx, Cb, tk);
-        TRACE(1);
         ptx::named_sync(BAR_AGG, C::NSYNC);
-        TRACE(2);
         // the tile's aggregate: the scan warps' aggregates folded in processing order
         float4 Ta = one2(), Tx = zero2();
         bool Tb = false;
@@ -567,7 +523,6 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
         }
         ok = ok && (*s_abort == 0);
         fenwick_publish(p, t.fbase, t.pos, Ca, Cx, Cb, Ta, Tx, Tb, ok, tk == p.withhold);
-        TRACE(3);
         return;
     }
 
@@ -589,7 +544,6 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
         bool Rb = false, ok = true;
         if (need_carry && t.pos > 0)
             ok = fenwick_carry(p, t.fbase, t.pos, node_mul, node_rag, base, carry, Ra, Rx, Rb, tk);
-        TRACE(4);
         if (p.fix != nullptr) {
             // steps of this tile before its first begin flag miss the state entering the segment
             const int64_t tid = t.chain * p.n_tt + t.jt;
@@ -665,7 +619,6 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
         }
     }
     if (!landed && lane == 0) *s_abort = 1;
-    if (warp == 0) TRACE(5);
 
     // phase 1: aggregate of this warp's steps, from the identity, in processing order
     float4 a = one2(), x = zero2();
@@ -767,7 +720,6 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
             }
             if (p.out_last != nullptr && nv > 0 && ts + nv == p.L) p.out_last[t.b * p.D2 + t.c2 + lane] = c;
         }
-        if (warp == 0) TRACE(6);
     } else {
         const float4* sh = s_h + warp * R * 32 + lane;
         float4 acc = zero2();
@@ -809,15 +761,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
             s_acc[warp * 32 + lane] = acc;
             ptx::named_arrive(BAR_ACC, C::NSYNC);
         }
-        if (warp == 0) TRACE(6);
     }
-#ifdef MEMOROID_TRACE
-    if (warp == 0 && lane == 0 && g_trace != nullptr) {
-        unsigned smid;
-        asm volatile("mov.u32 %0, %%smid;" : "=r"(smid));
-        g_trace[tk * 16 + 7] = smid;
-    }
-#endif
 }
 
 // ============================================================================
@@ -1128,50 +1072,21 @@ __global__ void __launch_bounds__(RED_PARTS) reduce_final_kernel(const double* _
 // ============================================================================
 namespace {
 
-// Tile shapes (warps, steps per warp).  The defaults are the measured best on
-// GB300; the macros exist for tuning sweeps.
-#ifndef MEMOROID_FWD_W
-#define MEMOROID_FWD_W 4
-#define MEMOROID_FWD_R 24
-#endif
-#ifndef MEMOROID_BWD_W
-#define MEMOROID_BWD_W 8
-#define MEMOROID_BWD_R 12
-#endif
-using FwdC = Cfg<MEMOROID_FWD_W, MEMOROID_FWD_R, false, false>;
-// per-step lambda (two staged arrays forward, three backward): measured best shapes
-#ifndef MEMOROID_FWDS_W
-#define MEMOROID_FWDS_W 4
-#define MEMOROID_FWDS_R 12
-#endif
-#ifndef MEMOROID_BWDS_W
-#define MEMOROID_BWDS_W 8
-#define MEMOROID_BWDS_R 8
-#endif
-using FwdS = Cfg<MEMOROID_FWDS_W, MEMOROID_FWDS_R, false, true>;
-using BwdC = Cfg<MEMOROID_BWD_W, MEMOROID_BWD_R, true, false>;
-using BwdS = Cfg<MEMOROID_BWDS_W, MEMOROID_BWDS_R, true, true>;
+// Tile shapes (scan warps, steps per warp): the measured best on GB300.
+using FwdC = Cfg<4, 24, false, false>;
+// per-step lambda (two staged arrays forward, three backward)
+using FwdS = Cfg<4, 12, false, true>;
+using BwdC = Cfg<8, 12, true, false>;
+using BwdS = Cfg<8, 8, true, true>;
 // The FFM forward stages only x~ (a few bytes per step), so larger tiles pay:
 // 6 x 31 (186-step tiles) was the measured best on GB300.
-#ifndef MEMOROID_FFM_FWD_W
-#define MEMOROID_FFM_FWD_W 6
-#define MEMOROID_FFM_FWD_R 31
-#endif
-#ifndef MEMOROID_FFM_BWD_W
-#define MEMOROID_FFM_BWD_W MEMOROID_BWD_W
-#define MEMOROID_FFM_BWD_R MEMOROID_BWD_R
-#endif
-using FwdF = Cfg<MEMOROID_FFM_FWD_W, MEMOROID_FFM_FWD_R, false, false, true>;
-using BwdF = Cfg<MEMOROID_FFM_BWD_W, MEMOROID_FFM_BWD_R, true, false, true>;
+using FwdF = Cfg<6, 31, false, false, true>;
+using BwdF = Cfg<8, 12, true, false, true>;
 
 // Segments per chain: enough segment chains that a tile's predecessor was
 // handed out long before it (target), at least MIN_SEG_TILES tiles each.
-#ifndef MEMOROID_TARGET_SC
-#define MEMOROID_TARGET_SC 512
-#endif
-#ifndef MEMOROID_TARGET_SC_BWD
-#define MEMOROID_TARGET_SC_BWD 256
-#endif
+constexpr int64_t TARGET_SC = 512;
+constexpr int64_t TARGET_SC_BWD = 256;
 constexpr int64_t MAX_SEG = 192;
 constexpr int64_t MIN_SEG_TILES = 8;
 
@@ -1179,7 +1094,7 @@ struct Segs {
     int64_t G, Q;
 };
 Segs choose_segments(int64_t n_chains, int64_t n_tt, bool rev) {
-    const int64_t target = rev ? MEMOROID_TARGET_SC_BWD : MEMOROID_TARGET_SC;
+    const int64_t target = rev ? TARGET_SC_BWD : TARGET_SC;
     int64_t G = (target + n_chains - 1) / n_chains;
     G = lmin(G, lmin(MAX_SEG, n_tt / MIN_SEG_TILES));
     if (G < 1) G = 1;
@@ -1251,7 +1166,7 @@ Params make_params(const Args& a, const Layout& l, int T, bool backward) {
     const DebugKnobs k = debug_knobs();
     p.wait_ns = k.wait_ns;
     p.withhold = k.withhold_ticket;
-    p.epoch = next_epoch();
+    p.epoch = 0;  // set at launch (tagged_epoch)
     p.full_nodes = a.lambda_per_step ? 1 : 0;
     p.T = T;
     // backward: the chain's first tile (processing order) is the ragged last
@@ -1306,6 +1221,12 @@ memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
         return MEMOROID_ERR_CUDA;
     Params p = make_params(a, l, C::T, C::REV);
     if (!make_maps(p, a, C::T, C::REV)) return MEMOROID_ERR_CUDA;
+    // the summaries' tag; their region is zeroed where an old word could carry it
+    bool clear = false;
+    p.epoch = tagged_epoch(a.workspace, l.gpart_off, &clear);
+    if (clear && cudaMemsetAsync(static_cast<unsigned char*>(a.workspace) + l.node_off, 0, l.gpart_off - l.node_off, s) !=
+                     cudaSuccess)
+        return MEMOROID_ERR_CUDA;
     kernel<<<static_cast<unsigned>(n_tickets), C::THREADS, C::SMEM, s>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     if (sg.G > 1) {
@@ -1333,12 +1254,6 @@ size_t workspace_bytes(int64_t B, int64_t L, int64_t D) {
     return m;
 }
 
-#ifdef MEMOROID_TRACE
-extern "C" int memoroid_trace_set_buffer(void* dev_ptr) {
-    unsigned long long* ptr = static_cast<unsigned long long*>(dev_ptr);
-    return static_cast<int>(cudaMemcpyToSymbol(g_trace, &ptr, sizeof(ptr)));
-}
-#endif
 
 int kernels_per_call(int64_t B, int64_t L, int64_t D, int per_step, int backward, int with_grad_lambda) {
     if (B <= 0 || L <= 0 || D <= 0) return 0;

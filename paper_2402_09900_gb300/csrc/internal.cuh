@@ -36,10 +36,16 @@ struct DebugKnobs {
 };
 DebugKnobs debug_knobs();
 
-// A fresh 31-bit, non-zero tag per launch.  Look-back summaries carry it, so
-// that words left in a workspace by an earlier launch are never mistaken for
-// this launch's.
-uint32_t next_epoch();
+// A fresh 31-bit, non-zero tag for a launch whose look-back summaries, in
+// the bytes [kHeaderBytes, region_end) of `workspace`, carry it.  Tags are
+// handed out in sequence and repeat only after 2^31 launches (a new
+// "generation").  *clear is set when the caller must zero that region before
+// the launch: the first time this process uses the workspace address on the
+// current device, the first time in each generation, or when the region
+// reaches further than the last clear.  So a summary word with this launch's
+// tag was written by this launch: every earlier write of the same tag is in a
+// past generation, and the region was cleared since.
+uint32_t tagged_epoch(const void* workspace, size_t region_end, bool* clear);
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
