@@ -138,11 +138,21 @@ memoroid_status_t memoroid_scan_diag_bwd(const void *lambda, int lambda_per_step
  *     or other host threads without ordering) race and give wrong results.
  *   - Shapes needing more than MEMOROID_STATIC_WORKSPACE_BYTES of workspace
  *     (memoroid_scan_diag_workspace_bytes) return MEMOROID_ERR_WORKSPACE.
+ *   - A device-side wait that runs out is reported by
+ *     memoroid_get_static_device_error (the array is not the caller's to read).
+ *   - The array's address is cached per device; after cudaDeviceReset do not
+ *     call this entry point on that device again in the same process.
  */
 memoroid_status_t memoroid_scan_diag_fwd_static(const void *lambda, int lambda_per_step,
                                                 const void *u, const uint8_t *start, const void *h0,
                                                 void *h, void *h_last, int64_t B, int64_t L,
                                                 int64_t D, void *stream);
+
+/* Synchronises `stream`, then reads the error word that the last
+ * memoroid_scan_diag_fwd_static call on the current device left in the
+ * library-owned scratch array: MEMOROID_OK or MEMOROID_ERR_TIMEOUT (the same
+ * reading as memoroid_get_device_error gives for a caller's workspace). */
+memoroid_status_t memoroid_get_static_device_error(void *stream);
 
 /* ======================================================================== */
 /* Decayed linear-attention memoroid: the Linear Transformer memoroid of    */

@@ -20,6 +20,11 @@
 //     without ordering) race on the array and give wrong results.
 //   * Shapes whose workspace would exceed the array are rejected with
 //     MEMOROID_ERR_WORKSPACE; nothing is allocated, on any path.
+//   * A bounded device-side wait that runs out records MEMOROID_ERR_TIMEOUT in
+//     the array's header like in any workspace; callers never see the array's
+//     address, so memoroid_get_static_device_error reads it for them.
+//   * The address is cached per device: after cudaDeviceReset the process
+//     must not call these entry points on that device again.
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -68,4 +73,10 @@ extern "C" memoroid_status_t memoroid_scan_diag_fwd_static(const void* lambda, i
     if (memoroid::static_workspace(&ws) != cudaSuccess) return MEMOROID_ERR_CUDA;
     return memoroid_scan_diag_fwd(lambda, lambda_per_step, u, start, h0, h, h_last, B, L, D, ws,
                                   static_cast<size_t>(MEMOROID_STATIC_WORKSPACE_BYTES), stream);
+}
+
+extern "C" memoroid_status_t memoroid_get_static_device_error(void* stream) {
+    void* ws = nullptr;
+    if (memoroid::static_workspace(&ws) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    return memoroid_get_device_error(ws, stream);
 }

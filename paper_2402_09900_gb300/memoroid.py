@@ -75,6 +75,7 @@ SIGNATURES = {
     "memoroid_offsets_workspace_bytes": (_sz, [_i64]),
     "memoroid_offsets_from_starts": (_int, [_p, _i64, _p, _p, _p, _sz, _p]),
     "memoroid_get_device_error": (_int, [_p, _p]),
+    "memoroid_get_static_device_error": (_int, [_p]),
     "memoroid_debug_set_wait_limit_ns": (None, [ctypes.c_uint64]),
     "memoroid_debug_withhold_tile": (None, [_i64]),
     "memoroid_debug_lnorm_padded": (None, [_int]),
@@ -332,6 +333,10 @@ def memoroid_offsets_from_starts(start, L, offsets, count, workspace, stream=Non
 
 def memoroid_get_device_error(workspace, stream=None) -> int:
     return int(load().memoroid_get_device_error(_ptr(workspace), _stream(stream)))
+
+
+def memoroid_get_static_device_error(stream=None) -> int:
+    return int(load().memoroid_get_static_device_error(_stream(stream)))
 
 
 def memoroid_debug_set_wait_limit_ns(ns: int) -> None:

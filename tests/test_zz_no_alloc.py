@@ -72,3 +72,32 @@ def test_static_workspace_rejects_oversized_shapes():
     with pytest.raises(m.MemoroidError) as e:
         m.memoroid_scan_diag_fwd_static(small, 0, small, flags, None, small, None, B, L, D)
     assert e.value.status == m.MEMOROID_ERR_WORKSPACE
+
+
+def test_static_workspace_reports_a_timed_out_wait_then_recovers():
+    # a look-back wait that runs out is recorded in the library-owned array's
+    # header; memoroid_get_static_device_error reads it (the caller never sees
+    # the array), and the next call on the same array is correct again
+    m = _m()
+    B, L, D = 1, 4096, 64
+    t = tapegen.diag_tape(B, L, D, seed=73, start_mode="none")
+    dev = torch.device("cuda")
+    lam = torch.from_numpy(t["lam"]).to(dev)
+    u = torch.from_numpy(t["u"]).to(dev)
+    start = torch.from_numpy(t["start"]).to(dev)
+    h = torch.empty_like(u)
+    try:
+        m.memoroid_debug_set_wait_limit_ns(20_000_000)  # 20 ms
+        m.memoroid_debug_withhold_tile(3)
+        m.memoroid_scan_diag_fwd_static(lam, 0, u, start, None, h, None, B, L, D)
+        assert m.memoroid_get_static_device_error() == m.MEMOROID_ERR_TIMEOUT
+    finally:
+        m.memoroid_debug_withhold_tile(-1)
+        m.memoroid_debug_set_wait_limit_ns(0)
+    m.memoroid_scan_diag_fwd_static(lam, 0, u, start, None, h, None, B, L, D)
+    assert m.memoroid_get_static_device_error() == m.MEMOROID_OK
+    ws = m.diag_workspace(B, L, D, dev)
+    h_ref = torch.empty_like(u)
+    m.memoroid_scan_diag_fwd(lam, 0, u, start, None, h_ref, None, B, L, D, ws)
+    torch.cuda.synchronize()
+    assert _rel(h, h_ref) <= TOL
