@@ -97,9 +97,12 @@ def test_ffm_autograd_matches_oracle():
 
 
 def test_two_layer_graph_backpropagates():
-    # FFM output -> a linear map -> linear attention; the gradient reaching x
-    # equals the one torch computes when the scans' own backward calls are
-    # replaced by their oracle gradients chained by hand
+    # FFM output -> a linear map -> linear attention.  Each link of the chain
+    # is checked on its own: the attention's gradients (returned in bf16, the
+    # dtype of its inputs) against the oracle on the same bf16 operands at the
+    # attention's 2e-2 bar; the gradient reaching z against those returned
+    # gradients pushed through W by hand (fp64); and the gradient reaching x
+    # against the FFM oracle's backward of that z gradient.
     m = _m()
     B, L, mm, c, H, d = 1, 600, 8, 2, 2, 64  # the tensor-core path takes d = 64 or 128
     tf = tapegen.ffm_tape(B, L, mm, c, tapegen.seed_for(1203), mean=80.0)
@@ -112,18 +115,20 @@ def test_two_layer_graph_backpropagates():
     z.retain_grad()
     qkv = (z @ dev(W)).to(torch.bfloat16).view(B, L, 3, H, d)
     q, k, v = qkv[:, :, 0].contiguous(), qkv[:, :, 1].contiguous(), qkv[:, :, 2].contiguous()
+    for a in (q, k, v):
+        a.retain_grad()
     y = m.LinAttnScan.apply(q, k, v, dev(gamma), dev(tf["start"]), None)
     (y * dev(gy)).sum().backward()
-    # by hand: oracle backward of the attention on the same bf16 operands, then through W, then FFM
     f = oracle.bf16_bits_to_f64
 
     def bits(t_):
         return t_.detach().cpu().view(torch.int16).numpy().view(np.uint16)
 
     rq, rk, rv, _, _ = oracle.linattn_bwd(f(bits(q)), f(bits(k)), f(bits(v)), gamma, tf["start"], gy)
-    dqkv = np.stack([rq, rk, rv], axis=2).reshape(B, L, 3 * H * d)
-    dz = dqkv @ W.astype(np.float64).T
-    assert rel_err(z.grad.cpu().numpy(), dz) <= 3e-2
+    for name, got, ref in (("dq", q.grad, rq), ("dk", k.grad, rk), ("dv", v.grad, rv)):
+        assert rel_err(np32(got), ref) <= 2e-2, name
+    got_qkv = np.stack([np32(q.grad), np32(k.grad), np32(v.grad)], axis=2).astype(np.float64).reshape(B, L, 3 * H * d)
+    assert rel_err(z.grad.cpu().numpy(), got_qkv @ W.astype(np.float64).T) <= 1e-5
     rz, _ = oracle.ffm_fwd(tf["alpha"], tf["omega"], tf["x"], tf["start"])
     rgx, _, _, _ = oracle.ffm_bwd(tf["alpha"], tf["omega"], tf["start"], rz, z.grad.cpu().numpy().astype(np.float64))
     assert rel_err(x.grad.cpu().numpy(), rgx) <= 1e-4

@@ -147,21 +147,14 @@ def test_fwd_deterministic():
     assert np.array_equal(a, b) and np.array_equal(sa, sb)
 
 
-def test_fwd_config3_sampled_episodes():
-    # the full L = 2^18, 4-head, d = 64 tape; checked on whole episodes, each
-    # of which the oracle evaluates alone (a start cuts all earlier context)
+def test_fwd_config3_full():
+    # the full L = 2^18, 4-head, d = 64 tape with per-head gamma: every output
+    # against the oracle run over the whole tape
     t = tapegen.linattn_config(3)
-    y, _ = run_gpu_fwd(t, chunk=t["chunk"])
-    starts = np.flatnonzero(t["start"][0])
-    rng = np.random.default_rng(3)
-    picks = rng.choice(len(starts) - 1, size=12, replace=False)
-    worst = 0.0
-    for i in picks:
-        s, e = int(starts[i]), int(starts[i + 1])
-        sub = dict(q=t["q"][:, s:e], k=t["k"][:, s:e], v=t["v"][:, s:e], gamma=t["gamma"], start=t["start"][:, s:e])
-        y_ref, _ = run_oracle_fwd(sub)
-        worst = max(worst, rel_err(y[:, s:e], y_ref))
-    assert worst <= TOL
+    y, S_last = run_gpu_fwd(t, chunk=t["chunk"])
+    y_ref, S_ref = run_oracle_fwd(t)
+    assert rel_err(y, y_ref) <= TOL
+    assert rel_err(S_last, S_ref) <= TOL
 
 
 # ---------------------------------------------------------------------------
@@ -298,37 +291,58 @@ def test_split_resume_fwd_and_bwd(cut, tol, tol_b):
         assert rel_err(np.concatenate([g1[i], g2[i]], axis=1), full[i]) <= tol_b, name
     assert rel_err(g1[4], full[4]) <= tol_b
 
-def _episode_slices(start_row, rng, n):
-    starts = np.flatnonzero(start_row)
-    picks = rng.choice(len(starts) - 1, size=n, replace=False)
-    return [(int(starts[i]), int(starts[i + 1])) for i in sorted(picks)]
-
-
 def test_config5_sampled_episodes():
-    # L = 2^22, 8 heads, d = 128, per-step gamma, drawn on the device.  Whole
-    # episodes (not the tape's first or last) depend on nothing outside
-    # themselves, so the oracle checks them one at a time.
+    # L = 2^22, 8 heads, d = 128, per-step gamma, drawn on the device.  The
+    # first episode continues from S0 and the last one is cut by the tape's
+    # end (it gives S_last and takes grad_S_last); every episode depends on
+    # nothing outside itself (the reset of Theorem 3.2), so the oracle checks
+    # them one at a time: the first, the last, the longest and 64 others
+    # drawn at random, every output (y, S_last, dq, dk, dv, dgamma, dS0).
     m = _m()
     c = tapegen.LINATTN_CONFIGS[5]
     B, L, H, d = c["B"], c["L"], c["H"], c["d"]
     t = tapegen.linattn_tape_device(B, L, H, d, tapegen.seed_for(5), c["mean"], c["gamma"], with_grad=True)
+    t["start"][:, 0] = 0
+    rng = np.random.default_rng(tapegen.seed_for(5) + 1)
+    S0 = (rng.standard_normal((B, H, d, d)) * 0.3).astype(np.float32)
+    dS_last = rng.standard_normal((B, H, d, d)).astype(np.float32)
     ws = m.linattn_workspace(B, L, H, d, "cuda")
-    y, _ = m.linattn_fwd(t["q"], t["k"], t["v"], t["gamma"], t["start"], None, want_last=False, ws=ws)
-    dq, dk, dv, dg, _ = m.linattn_bwd(t["q"], t["k"], t["v"], t["gamma"], t["start"], t["grad_y"], ws=ws)
+    y, S_last = m.linattn_fwd(t["q"], t["k"], t["v"], t["gamma"], t["start"], dev(S0), want_last=True, ws=ws)
+    dq, dk, dv, dg, dS0 = m.linattn_bwd(t["q"], t["k"], t["v"], t["gamma"], t["start"], t["grad_y"], dev(dS_last),
+                                        dev(S0), want_S0=True, ws=ws)
     assert m.memoroid_get_device_error(ws) == m.MEMOROID_OK
     torch.cuda.synchronize()
     start = t["start"].cpu().numpy()
+    heads = np.flatnonzero(start[0])
+    bounds = np.concatenate([[0], heads, [L]])
+    episodes = list(zip(bounds[:-1].tolist(), bounds[1:].tolist()))
+    first, last = episodes[0], episodes[-1]
+    inner = episodes[1:-1]
+    longest = max(inner, key=lambda se: se[1] - se[0])
+    others = [se for se in inner if se != longest]
+    picks = [others[i] for i in sorted(rng.choice(len(others), size=64, replace=False))]
     worst = {}
-    for s, e in _episode_slices(start[0], np.random.default_rng(5), 6):
+
+    def note(name, got, ref):
+        worst[name] = max(worst.get(name, 0.0), rel_err(got, ref))
+
+    for s, e in [first, longest, *picks, last]:
         sl = slice(s, e)
         sub = dict(q=t["q"][:, sl].cpu().numpy().view(np.uint16), k=t["k"][:, sl].cpu().numpy().view(np.uint16),
                    v=t["v"][:, sl].cpu().numpy().view(np.uint16), gamma=t["gamma"][:, sl].cpu().numpy(),
                    start=start[:, sl], grad_y=t["grad_y"][:, sl].cpu().numpy())
-        y_ref, _ = run_oracle_fwd(sub)
-        rq, rk, rv, rg, _ = run_oracle_bwd(sub)
+        s0 = S0 if s == 0 else None
+        ds = dS_last if e == L else None
+        y_ref, S_ref = run_oracle_fwd(sub, s0)
+        rq, rk, rv, rg, rS0 = run_oracle_bwd(sub, s0, ds)
         for name, got, ref in (("y", y[:, sl], y_ref), ("dq", dq[:, sl], rq), ("dk", dk[:, sl], rk),
                                ("dv", dv[:, sl], rv), ("dgamma", dg[:, sl], rg)):
-            worst[name] = max(worst.get(name, 0.0), rel_err(got.cpu().numpy(), ref))
+            note(name, got.cpu().numpy(), ref)
+        if s == 0:
+            note("dS0", dS0.cpu().numpy(), rS0)
+        if e == L:
+            note("S_last", S_last.cpu().numpy(), S_ref)
+    assert set(worst) == {"y", "dq", "dk", "dv", "dgamma", "dS0", "S_last"}
     assert all(v <= TOL for v in worst.values()), worst
 
 
