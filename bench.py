@@ -292,6 +292,134 @@ def per_step_leg(args, m, dev, stream):
     return out
 
 
+CFG3_WORKLOAD = ("linattn fwd+bwd (dq, dk, dv, per-head dgamma): B=1 tape, L=2^18 steps, H=4 heads, d_k=d_v=64, "
+                 "bf16 q/k/v (k L2-normalised), gamma per head in {0.9, 0.99, 0.999, 1.0}, Geometric(300) "
+                 "episodes, chunk 64")
+CFG4_WORKLOAD = ("diag scan fwd+bwd (grad_u, grad_lambda): B=64 tapes x L=16384 steps, D=128 complex64 channels, "
+                 "tapes 0-31 Geometric(20) episodes, tapes 32-63 one episode each")
+
+
+def _timed_pair(fwd, bwd, steps, stream):
+    """Mean milliseconds of fwd and bwd over `steps` back-to-back pairs (CUDA
+    events on `stream`, after 3 untimed pairs)."""
+    import torch
+
+    for _ in range(3):
+        fwd()
+        bwd()
+    torch.cuda.synchronize()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for i in range(steps):
+        evs[i][0].record(stream)
+        fwd()
+        evs[i][1].record(stream)
+        bwd()
+        evs[i][2].record(stream)
+    torch.cuda.synchronize()
+    f_ms = sum(e[0].elapsed_time(e[1]) for e in evs) / steps
+    b_ms = sum(e[1].elapsed_time(e[2]) for e in evs) / steps
+    return f_ms, b_ms
+
+
+def _hbm_roofline(fb, bb, f_ms, b_ms):
+    peak, peak_kind = _peaks()
+    return {"bound": "hbm", "peak": peak, "unit": "GB/s", "peak_kind": f"{peak_kind} (copy bandwidth)",
+            "fwd": {"algorithmic_bytes_per_call": fb, "achieved": fb / (f_ms * 1e-3) / 1e9,
+                    "frac": fb / (f_ms * 1e-3) / 1e9 / peak},
+            "bwd": {"algorithmic_bytes_per_call": bb, "achieved": bb / (b_ms * 1e-3) / 1e9,
+                    "frac": bb / (b_ms * 1e-3) / 1e9 / peak},
+            "step_frac": (fb + bb) / ((f_ms + b_ms) * 1e-3) / 1e9 / peak}
+
+
+def linattn_cfg3_leg(args, m, dev, stream):
+    """Times the linear-attention memoroid (fwd, bwd with per-head dgamma) on the
+    L = 2^18, 4-head, d = 64 tape with per-head decays."""
+    import torch
+
+    c = tapegen.LINATTN_CONFIGS[3]
+    B, L, H, d = c["B"], c["L"], c["H"], c["d"]
+    t = tapegen.linattn_tape_device(B, L, H, d, tapegen.seed_for(3), c["mean"], c["gamma"], device=dev)
+    ws = m.linattn_workspace(B, L, H, d, dev)
+    y = torch.empty((B, L, H, d), dtype=torch.float32, device=dev)
+    dq, dk, dv = torch.empty_like(y), torch.empty_like(y), torch.empty_like(y)
+    dg = torch.empty_like(t["gamma"])
+
+    def fwd():
+        m.memoroid_scan_linattn_fwd(t["q"], t["k"], t["v"], m.MEMOROID_BF16, t["gamma"], 0, t["start"], None, y,
+                                    None, B, L, H, d, d, c["chunk"], ws, stream)
+
+    def bwd():
+        m.memoroid_scan_linattn_bwd(t["q"], t["k"], t["v"], m.MEMOROID_BF16, t["gamma"], 0, t["start"], None,
+                                    t["grad_y"], None, dq, dk, dv, dg, None, B, L, H, d, d, c["chunk"], ws, stream)
+
+    f_ms, b_ms = _timed_pair(fwd, bwd, args.cfg3_steps, stream)
+    if m.memoroid_get_device_error(ws) != m.MEMOROID_OK:
+        raise RuntimeError("device-side error in the config-3 linattn leg")
+    el = B * L * H * d
+    fb = el * (3 * 2 + 4) + H * 4 + B * L
+    bb = el * (3 * 2 + 4 + 3 * 4) + H * 8 + B * L
+    kpc = (m.memoroid_scan_linattn_kernels_per_call(B, L, H, d, d, 0, 0)
+           + m.memoroid_scan_linattn_kernels_per_call(B, L, H, d, d, 1, 1))
+    out = {"workload": CFG3_WORKLOAD, "value": B * L / ((f_ms + b_ms) * 1e-3), "unit": UNIT,
+           "steps": args.cfg3_steps, "ms_per_step": f_ms + b_ms, "fwd_ms": f_ms, "bwd_ms": b_ms,
+           "episodes": int(t["start"].sum().item()), "roofline": _hbm_roofline(fb, bb, f_ms, b_ms),
+           "l2": "q, k, v 32 MiB each, y and gradients 64 MiB each: the working set of a call (0.67 / 1.48 GB) "
+                 "exceeds the 129 MB L2",
+           "gpu_launches": args.cfg3_steps * kpc}
+    del t, y, dq, dk, dv, ws
+    torch.cuda.empty_cache()
+    return out
+
+
+def diag_cfg4_leg(args, m, dev, stream):
+    """Times the diagonal scan (fwd, bwd with grad_lambda) on 64 tapes of 16384
+    steps at D = 128: half the tapes with short Geometric(20) episodes, half
+    one episode each (the extremes of reset density)."""
+    import torch
+
+    B, L, D = 64, 16384, 128
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(tapegen.seed_for(4))
+    mag = 0.9 + 0.099 * torch.rand((D,), generator=gen, device=dev)
+    ph = 2 * np.pi * torch.rand((D,), generator=gen, device=dev)
+    lam = torch.polar(mag, ph).to(torch.complex64)
+    u = torch.randn((B, L, D), generator=gen, device=dev, dtype=torch.complex64)
+    g = torch.randn((B, L, D), generator=gen, device=dev, dtype=torch.complex64) * np.sqrt(2.0)
+    rng = np.random.default_rng(tapegen.seed_for(4))
+    st_np = np.zeros((B, L), dtype=np.uint8)
+    for b in range(B):
+        if b < B // 2:
+            st_np[b] = tapegen.geometric_tape_starts(rng, L, 20.0)
+        else:
+            st_np[b, 0] = 1
+    st = torch.from_numpy(st_np).to(dev)
+    h, gu, gl = torch.empty_like(u), torch.empty_like(u), torch.empty_like(lam)
+    ws = m.diag_workspace(B, L, D, dev)
+
+    def fwd():
+        m.memoroid_scan_diag_fwd(lam, 0, u, st, None, h, None, B, L, D, ws, stream)
+
+    def bwd():
+        m.memoroid_scan_diag_bwd(lam, 0, st, None, h, g, None, gu, gl, None, B, L, D, ws, stream)
+
+    f_ms, b_ms = _timed_pair(fwd, bwd, args.cfg4_steps, stream)
+    if m.memoroid_get_device_error(ws) != m.MEMOROID_OK:
+        raise RuntimeError("device-side error in the config-4 diag leg")
+    fb = B * L * D * FWD_BYTES_PER_STEP_CH + B * L
+    bb = B * L * D * BWD_BYTES_PER_STEP_CH + B * L
+    kpc = (m.memoroid_scan_diag_kernels_per_call(B, L, D, 0, 0, 0)
+           + m.memoroid_scan_diag_kernels_per_call(B, L, D, 0, 1, 1))
+    out = {"workload": CFG4_WORKLOAD, "value": B * L / ((f_ms + b_ms) * 1e-3), "unit": UNIT,
+           "steps": args.cfg4_steps, "ms_per_step": f_ms + b_ms, "fwd_ms": f_ms, "bwd_ms": b_ms,
+           "fwd_value": B * L / (f_ms * 1e-3), "episodes": int(st_np.sum()),
+           "roofline": _hbm_roofline(fb, bb, f_ms, b_ms),
+           "l2": "inputs 1 GiB per tensor vs 129 MB L2; no flush needed",
+           "gpu_launches": args.cfg4_steps * kpc}
+    del lam, u, g, h, gu, gl, ws
+    torch.cuda.empty_cache()
+    return out
+
+
 def lnorm_leg(args, m, dev, stream):
     """Times memoroid_linattn_norm_fwd + _bwd on the config-3 shape."""
     import torch
@@ -934,6 +1062,23 @@ def run_ours(args):
     tb = None
     if ws == 1 and not args.skip_tbb:
         tb = tbb_leg(args, m, dev, stream)
+    c3 = None
+    if ws == 1 and not args.skip_cfg3:
+        c3 = linattn_cfg3_leg(args, m, dev, stream)
+    c4 = None
+    if ws == 1 and not args.skip_cfg4:
+        c4 = diag_cfg4_leg(args, m, dev, stream)
+    # the other legs' roofline fractions, also inside the headline roofline object
+    legs = {}
+    for name, leg in (("linattn_cfg5", la), ("linattn_cfg3", c3), ("diag_cfg4", c4), ("diag_per_step_lambda", ps),
+                      ("linattn_norm", ln), ("ffm", ff)):
+        if leg is not None:
+            r = leg["roofline"]
+            legs[name] = {"fwd_frac": r["fwd"]["frac"], "bwd_frac": r["bwd"]["frac"], "step_frac": r.get("step_frac"),
+                          "fwd_ms": leg["fwd_ms"], "bwd_ms": leg["bwd_ms"], "value": leg["value"]}
+    if rt is not None:
+        legs["returns"] = {k: rt[k]["roofline"]["frac"] for k in ("return", "gae") if k in rt}
+    roofline["legs"] = legs
     cpu = None
     if ws == 1 and not args.skip_cpu_baseline:
         cpu = cpu_baseline(t, args.cpu_seconds)
@@ -954,6 +1099,8 @@ def run_ours(args):
         "tbb": tb,
         "linattn_norm": ln,
         "diag_per_step_lambda": ps,
+        "linattn_cfg3": c3,
+        "diag_cfg4": c4,
     }
     print(json.dumps(out), flush=True)
     if ws > 1:
@@ -987,6 +1134,10 @@ def main():
     ap.add_argument("--skip-tbb", action="store_true", help="omit the tape-based batching leg")
     ap.add_argument("--skip-lnorm", action="store_true", help="omit the normalised Linear Transformer leg")
     ap.add_argument("--skip-per-step", action="store_true", help="omit the per-step lambda diag leg")
+    ap.add_argument("--skip-cfg3", action="store_true", help="omit the L=2^18, 4-head, d=64 linattn leg")
+    ap.add_argument("--cfg3-steps", type=int, default=20, help="timed config-3 linattn fwd+bwd steps")
+    ap.add_argument("--skip-cfg4", action="store_true", help="omit the 64-tape, D=128 diag leg")
+    ap.add_argument("--cfg4-steps", type=int, default=20, help="timed config-4 diag fwd+bwd steps")
     ap.add_argument("--ps-steps", type=int, default=20, help="timed per-step lambda fwd+bwd steps")
     ap.add_argument("--only-per-step", action="store_true",
                     help="profiling mode: run and print only the per-step lambda diag leg")
