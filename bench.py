@@ -558,12 +558,12 @@ def linattn_leg(args, m, dev, stream):
     dq, dk, dv = torch.empty_like(y), torch.empty_like(y), torch.empty_like(y)
     dg = torch.empty_like(t["gamma"])
 
-    def fwd():
-        m.memoroid_scan_linattn_fwd(t["q"], t["k"], t["v"], m.MEMOROID_BF16, t["gamma"], per, t["start"], None, y,
+    def fwd(start=t["start"], gamma=t["gamma"]):
+        m.memoroid_scan_linattn_fwd(t["q"], t["k"], t["v"], m.MEMOROID_BF16, gamma, per, start, None, y,
                                     None, B, L, H, d, d, c["chunk"], ws, stream)
 
-    def bwd():
-        m.memoroid_scan_linattn_bwd(t["q"], t["k"], t["v"], m.MEMOROID_BF16, t["gamma"], per, t["start"], None,
+    def bwd(start=t["start"], gamma=t["gamma"]):
+        m.memoroid_scan_linattn_bwd(t["q"], t["k"], t["v"], m.MEMOROID_BF16, gamma, per, start, None,
                                     t["grad_y"], None, dq, dk, dv, dg, None, B, L, H, d, d, c["chunk"], ws, stream)
 
     for _ in range(args.la_warmup):
@@ -610,11 +610,26 @@ def linattn_leg(args, m, dev, stream):
     i_ms = e0.elapsed_time(e1)
     i_tf = ctas * reps * 4 * 128 * 128 * d / (i_ms * 1e-3) / 1e12
     burst, sustained, tkind = _tensor_peaks()
+
+    # the same tape with a single begin flag (t = 0): one episode, the extreme of
+    # reset density; with the workload's decays and with gamma = 1 (no decay, so
+    # every state reaches across the whole tape)
+    one = torch.zeros_like(t["start"])
+    one[:, 0] = 1
+    sparse = {}
+    for name, gam in (("workload_gamma", t["gamma"]), ("gamma_1", torch.ones_like(t["gamma"]))):
+        sf, sb = _timed_pair(lambda: fwd(one, gam), lambda: bwd(one, gam), steps, stream)
+        if m.memoroid_get_device_error(ws) != m.MEMOROID_OK:
+            raise RuntimeError("device-side error in the single-episode linattn steps")
+        sparse[name] = {"fwd_ms": sf, "bwd_ms": sb, "ms_per_step": sf + sb,
+                        "vs_workload_step": (sf + sb) / (f_ms + b_ms),
+                        "value": B * L / ((sf + sb) * 1e-3)}
     out = {
         "workload": LA_WORKLOAD if not args.la_tape_steps else f"{LA_WORKLOAD} (first {L} steps only)",
         "value": B * L / ((f_ms + b_ms) * 1e-3), "unit": UNIT, "steps": steps,
         "ms_per_step": f_ms + b_ms, "fwd_ms": f_ms, "bwd_ms": b_ms,
         "episodes": int(t["start"].sum().item()),
+        "single_episode": sparse,
         "roofline": {"bound": "hbm", "peak": peak, "unit": "GB/s", "peak_kind": f"{peak_kind} (copy bandwidth)",
                      "fwd": {"algorithmic_bytes_per_call": fb, "achieved": fb / (f_ms * 1e-3) / 1e9,
                              "frac": fb / (f_ms * 1e-3) / 1e9 / peak},
@@ -628,7 +643,7 @@ def linattn_leg(args, m, dev, stream):
                                "flops": ctas * reps * 4 * 128 * 128 * d,
                                "what": "P = Q K^T (128x128x128) and Y = Pm V (128x128x128) per rep, tcgen05 "
                                        "kind::f16 bf16->fp32, operands resident in shared memory"},
-        "gpu_launches": steps * kpc + 2,
+        "gpu_launches": 3 * steps * kpc + 2,  # timed: the workload and the two single-episode cases, the microbenchmark
     }
     del t, y, dq, dk, dv, ws
     torch.cuda.empty_cache()

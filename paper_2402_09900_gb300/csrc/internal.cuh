@@ -160,9 +160,6 @@ memoroid_status_t launch_fwd(const Args& a, cudaStream_t stream);
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream);
 size_t intra_bench_scratch_bytes(int64_t D);
 memoroid_status_t launch_intra_bench(int64_t D, int64_t reps, int64_t ctas, void* scratch, cudaStream_t stream);
-// first[b][g] = first begin flag of tape b in [g, g + 1) * seg_len (segment 0: step 0), or -1
-memoroid_status_t launch_segment_plan(const uint8_t* start, int64_t B, int64_t L, int64_t seg_len, int64_t G,
-                                      int64_t* first, cudaStream_t stream);
 
 }  // namespace la
 

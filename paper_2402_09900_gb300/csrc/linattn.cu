@@ -13,13 +13,17 @@
 //   S_tile = [no start in tile] exp(Lam_end) S_prev + sum_{r >= last start} exp(Lam_end - Lam_r) k_r v_r^T.
 // Both are dense bf16 contractions with fp32 accumulators in tensor memory.
 //
-// Parallel structure: the tape of each (tape, head) is cut into segments
-// whose boundaries are moved forward to the next begin flag, so every segment
-// (but the first, which may continue from S0) starts from the zero state: the
-// reset of Theorem 3.2 makes the segments independent, and no carry or fix-up
-// pass is needed.  Each CTA owns one (tape, head, segment) and walks its tiles
-// in order, carrying the state in TMEM.  A nominal segment without any begin
-// flag is absorbed by the segment before it.
+// Parallel structure: the tape of each (tape, head) is cut into G segments of
+// tps whole tiles, one CTA each, which walks its tiles in order carrying the
+// state in TMEM from the state entering the segment.  Those entry states come
+// from a resettable scan over the segments (Theorem 3.2 applied to segment
+// aggregates): a summary kernel computes, per segment, the state its rows
+// after the last begin flag leave behind from a zero start (rows whose decay
+// weight underflows are skipped), and a carry kernel folds the summaries in
+// order, S_exit(g) = [no flag in g] a_g S_exit(g-1) + X_g.  The backward
+// runs the same scan in reverse for the reverse state.  The amount of work
+// therefore does not depend on where the begin flags fall: a tape with one
+// episode runs on as many CTAs as one with many.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -58,6 +62,7 @@ static_assert(sizeof(TileMeta) == 656, "TileMeta is copied as 41 16-byte chunks"
 // ---------------------------------------------------------------------------
 // segment plan and workspace layout
 // ---------------------------------------------------------------------------
+// Segment g of a (tape, head) holds tiles [g * tps, min((g + 1) * tps, n_tiles)).
 struct Plan {
     int64_t n_tiles, tps, G;  // tiles per tape, tiles per segment, segments per (tape, head)
 };
@@ -76,18 +81,21 @@ Plan make_plan(int64_t B, int64_t L, int64_t H) {
 }
 
 struct Layout {
-    size_t meta, seg_first, fwd_total;
-    size_t dy16, states, dlam_f, gpart, total;  // backward only
+    size_t meta, info, carry_f, fwd_total;
+    size_t dy16, states, dlam_f, gpart, carry_r, total;  // backward only
 };
 
 Layout make_layout(int64_t B, int64_t L, int64_t H, int64_t D) {
     const Plan pl = make_plan(B, L, H);
+    const size_t nseg = static_cast<size_t>(B * H * pl.G);
     Layout ly;
     size_t off = kHeaderBytes;
     ly.meta = off;
     off = align_up(off + static_cast<size_t>(B * H * pl.n_tiles) * sizeof(TileMeta), 256);
-    ly.seg_first = off;
-    off = align_up(off + static_cast<size_t>(B * pl.G) * sizeof(int64_t), 256);
+    ly.info = off;  // per segment: (begin flag in the segment, log2 of its decay)
+    off = align_up(off + nseg * sizeof(float2), 256);
+    ly.carry_f = off;  // per segment: its summary, then (carry) the state leaving it
+    off = align_up(off + nseg * static_cast<size_t>(D * D) * sizeof(float), 256);
     ly.fwd_total = off;
     ly.dy16 = off;
     off = align_up(off + static_cast<size_t>(B * L * H * D) * sizeof(uint16_t), 256);
@@ -97,45 +105,10 @@ Layout make_layout(int64_t B, int64_t L, int64_t H, int64_t D) {
     off = align_up(off + static_cast<size_t>(B * L * H) * sizeof(float), 256);
     ly.gpart = off;
     off = align_up(off + static_cast<size_t>(B * H * pl.G) * sizeof(float), 256);
+    ly.carry_r = off;  // per segment: its reverse summary, then the reverse state leaving it
+    off = align_up(off + nseg * static_cast<size_t>(D * D) * sizeof(float), 256);
     ly.total = off;
     return ly;
-}
-
-// ---------------------------------------------------------------------------
-// kernel 0: segment boundaries at begin flags
-// ---------------------------------------------------------------------------
-// first[b][g] = the first step t in the nominal range [g, g + 1) * seg_len with
-// start[b][t] = 1 (segment 0: step 0), or -1 if the range holds no begin flag.
-// One warp per (tape, segment); each lane tests 16 consecutive flags per pass.
-__global__ void __launch_bounds__(256) plan_kernel(const uint8_t* __restrict__ start, int64_t B, int64_t L,
-                                                   int64_t seg_len, int64_t G, int64_t* __restrict__ first) {
-    const int64_t wid = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    if (wid >= B * G) return;
-    const int64_t b = wid / G, g = wid % G;
-    if (g == 0) {
-        if (lane == 0) first[wid] = 0;
-        return;
-    }
-    const int64_t p0 = g * seg_len, p1 = min(L, p0 + seg_len);
-    const uint8_t* row = start + b * L;
-    int64_t found = -1;
-    for (int64_t base = p0; base < p1 && found < 0; base += 32 * 16) {
-        int hit = 16;
-        const int64_t t0 = base + lane * 16;
-#pragma unroll
-        for (int x = 15; x >= 0; --x) {
-            const int64_t t = t0 + x;
-            if (t < p1 && row[t] != 0) hit = x;
-        }
-        const unsigned m = __ballot_sync(0xffffffffu, hit < 16);
-        if (m != 0) {
-            const int src = __ffs(m) - 1;
-            const int h = __shfl_sync(0xffffffffu, hit, src);
-            found = base + src * 16 + h;
-        }
-    }
-    if (lane == 0) first[wid] = found;
 }
 
 // ---------------------------------------------------------------------------
@@ -164,8 +137,9 @@ __global__ void __launch_bounds__(256) meta_kernel(const float* __restrict__ gam
         float l = 0.f;
         if (valid && !st) {
             const float g = per_step ? gamma[(b * L + t) * H + h] : gamma[h];
-            // gamma = 0 gives a weight of at most 2^-126 instead of 0
-            l = fmaxf(log2f(g), -126.f);
+            // gamma is a decay: clamped to [2^-126, 1] (gamma = 0 gives a weight of at
+            // most 2^-126 instead of 0)
+            l = fminf(fmaxf(log2f(g), -126.f), 0.f);
         }
         lg[k] = l;
         sg[k] = st ? r : -1;
@@ -401,7 +375,7 @@ struct FwdParams {
     const float* S0;
     float* y;
     const TileMeta* meta;
-    const int64_t* seg_first;  // [B][G] from plan_kernel
+    const float* carry;  // [B * H * G][D][D]: the state leaving each segment (g < G - 1)
     float* S_last;
     uint32_t* hdr;
     int64_t B, L, H, n_tiles, tps;
@@ -508,21 +482,13 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     const int64_t bh = blockIdx.x / p.G;
     const int g = static_cast<int>(blockIdx.x % p.G);
     const int64_t b = bh / p.H, h = bh % p.H;
-    // this segment covers steps [seg_lo, seg_hi): from its first begin flag to
-    // the next segment's (or the tape end)
-    const int64_t* sf = p.seg_first + b * p.G;
-    const int64_t seg_lo = sf[g];
-    if (seg_lo < 0) return;  // no begin flag in the nominal range: covered by an earlier segment
-    int64_t seg_hi = p.L;
-    for (int g2 = g + 1; g2 < p.G; ++g2) {
-        if (sf[g2] >= 0) {
-            seg_hi = sf[g2];
-            break;
-        }
-    }
-    const int64_t tile0 = seg_lo / T;
-    const int nt = static_cast<int>((seg_hi + T - 1) / T - tile0);
-    const int64_t row_stride = p.H * DOUT;  // output elements between consecutive steps of one head
+    // this segment: tiles [tile0, tile0 + nt), steps up to seg_hi (the tape end for the last)
+    const int64_t tile0 = static_cast<int64_t>(g) * p.tps;
+    const int nt = static_cast<int>(min(p.tps, p.n_tiles - tile0));
+    const int64_t seg_hi = min(p.L, (tile0 + nt) * T);
+    // the state entering the segment: S0 for the first, else the carry
+    const float* s_in = g == 0 ? (p.S0 != nullptr ? p.S0 + bh * D * D : nullptr)
+                               : p.carry + (bh * p.G + g - 1) * D * D;
 
     uint64_t* bar1 = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
     uint64_t* bar2 = bar1 + 1;
@@ -585,14 +551,14 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     constexpr int SC = D / 2;  // state and output columns per thread
     const uint32_t lane_base = tm + (static_cast<uint32_t>(32 * quarter) << 16);
 
-    // ---- incoming state: S0 for the first segment of a tape ----
+    // ---- incoming state (unless the segment's first step begins an episode) ----
     bool have_prev = false, have_state = false;
-    if (g == 0 && p.S0 != nullptr && metas[0].first_start != 0) {
+    if (s_in != nullptr && metas[0].first_start != 0) {
         have_prev = true;
         const bool scale = metas[0].has_start == 0;
         have_state = scale;
         const float a0 = metas[0].a;
-        const float* s0 = p.S0 + bh * D * D;
+        const float* s0 = s_in;
 #pragma unroll 1
         for (int cc = 0; cc < SC / 16; ++cc) {
             const int j0 = half * SC + cc * 16;
@@ -613,7 +579,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 }
                 store_bf16x16(smem + S::OFF_SB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
                 if (BWD && metas[0].has_start == 0)
-                    store_state_row<D>(state_image<D>(p.states, bh, p.n_tiles, 0), srow, j0, v);
+                    store_state_row<D>(state_image<D>(p.states, bh, p.n_tiles, tile0), srow, j0, v);
             } else {
 #pragma unroll
                 for (int x = 0; x < 16; ++x) v[x] = 0.f;
@@ -626,13 +592,13 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         }
     }
 
-    if (BWD && !have_prev && g == 0 && metas[0].has_start == 0 && srow >= 0) {
-        // the zero state before the tape's first tile
+    if (BWD && !have_prev && metas[0].has_start == 0 && srow >= 0) {
+        // the zero state before the tape's first tile (no S0)
         float zero[16];
 #pragma unroll
         for (int x = 0; x < 16; ++x) zero[x] = 0.f;
         for (int j0 = half * SC; j0 < half * SC + SC; j0 += 16)
-            store_state_row<D>(state_image<D>(p.states, bh, p.n_tiles, 0), srow, j0, zero);
+            store_state_row<D>(state_image<D>(p.states, bh, p.n_tiles, tile0), srow, j0, zero);
     }
 
     constexpr uint32_t ID_QS = tc::idesc_bf16(128, D, false, true);
@@ -784,8 +750,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         }
 
         // ---- y = Y_intra + w_in * Y_inter, staged as fp32 rows in stage s ----
-        // rows of this tile that belong to the segment
-        const int r_lo = static_cast<int>(max(static_cast<int64_t>(0), seg_lo - t0));
+        // rows of this tile inside the tape
         const int r_hi = static_cast<int>(min(static_cast<int64_t>(T), seg_hi - t0));
         if (NF) {
             // y = y'[:64] / y'[64]: every thread reads the normalizer (column 64) of
@@ -804,7 +769,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             }
             tc::ld_wait();
             const float dn = have_prev ? fmaf(w_in, __uint_as_float(ni[0]), __uint_as_float(na[0])) : __uint_as_float(na[0]);
-            if (half == 0 && p.den != nullptr && t >= r_lo && t < r_hi) p.den[(b * p.L + t0 + t) * p.H + h] = dn;
+            if (half == 0 && p.den != nullptr && t < r_hi) p.den[(b * p.L + t0 + t) * p.H + h] = dn;
             const float inv = 1.f / dn;
             unsigned char* yst = smem + s * S::STAGE + Y_OFF + t * 128;  // row t of chunk 0
 #pragma unroll
@@ -932,25 +897,12 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         tc::fence_before();
         __syncthreads();
         if (warp == 0) {
-            const int full_rows = static_cast<int>(min(static_cast<int64_t>(T), p.L - t0));
-            if (r_lo == 0 && r_hi == full_rows) {
-                // whole tile: one TMA store per 32 channels (rows past L are clipped)
-                if (lane == 0) {
+            // one TMA store per 32 channels (rows past L are clipped)
+            if (lane == 0) {
 #pragma unroll
-                    for (int m = 0; m < DOUT / 32; ++m)
-                        tma_store_4d(&p.map_y, sbase + s * S::STAGE + Y_OFF + m * T * 128, 32 * m, static_cast<int>(h),
-                                     static_cast<int>(t0), static_cast<int>(b));
-                }
-            } else {
-                // a tile shared with a neighbouring segment: only this segment's rows, 16 bytes at a time
-                float* ybase = p.y + ((b * p.L + t0) * p.H + h) * DOUT;
-                const unsigned char* st = smem + s * S::STAGE + Y_OFF;
-                for (int e = lane; e < (r_hi - r_lo) * (DOUT / 4); e += 32) {
-                    const int r = r_lo + e / (DOUT / 4), j = (e % (DOUT / 4)) * 4;
-                    const float4 v = *reinterpret_cast<const float4*>(st + (j >> 5) * (T * 128) + r * 128 +
-                                                                      ((((j & 31) >> 2) ^ (r & 7)) << 4));
-                    *reinterpret_cast<float4*>(ybase + static_cast<int64_t>(r) * row_stride + j) = v;
-                }
+                for (int m = 0; m < DOUT / 32; ++m)
+                    tma_store_4d(&p.map_y, sbase + s * S::STAGE + Y_OFF + m * T * 128, 32 * m, static_cast<int>(h),
+                                 static_cast<int>(t0), static_cast<int>(b));
             }
             if (BWD && lane == 0 && c + 1 < nt && metas[(c + 1) % S::NMETA].has_start == 0)
                 bulk_s2g(state_image<D>(p.states, bh, p.n_tiles, tile0 + c + 1), stage_q(s), D * D * 2);
@@ -975,7 +927,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
 #pragma unroll
             for (int x = 0; x < 4; ++x) {
                 const int r = 4 * lane + x;
-                if (r >= r_lo && r < r_hi) p.dlam_f[(b * p.L + t0 + r) * p.H + h] = zv[x] + after;
+                if (r < r_hi) p.dlam_f[(b * p.L + t0 + r) * p.H + h] = zv[x] + after;
             }
         }
         have_prev = true;
@@ -994,6 +946,319 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     __syncthreads();
     tc::fence_after();
     if (warp == 0) tc::dealloc(tm, S::TMEM_COLS);
+}
+
+// ---------------------------------------------------------------------------
+// segment summaries and the carry between segments
+// ---------------------------------------------------------------------------
+// REV = false (the forward's "tail" summary, for segments g < G - 1): the state
+// that the segment's rows after its last begin flag (all its rows if it has
+// none) leave at its end from a zero start,
+//   X_g = sum_r exp2(Lam_end - Lam_r) k_r v_r^T,
+// REV = true (the backward's "head" summary, for segments g >= 1): the reverse
+// state that the rows before its first begin flag pass to the segment before,
+//   X_g = sum_s exp2(Lam_s - Lam_begin) q_s dy_s^T,
+// with Lam the running sum of log2(gamma) over the segment.  Also per segment:
+// info[g] = (1 if it holds a begin flag, log2 of its total decay).  Both are
+// dense bf16 contractions K~^T V (or Q~^T dY) over the segment's tiles with
+// fp32 accumulation in TMEM.  gamma <= 1, so the weights only shrink away from
+// the segment's end (start); tiles whose weights all underflow to 0 are not
+// read.
+template <int D>
+struct SegSmem {
+    static constexpr int TILE = T * D * 2;
+    static constexpr int NST = 3;  // stages: tile i computes while i + 1 and i + 2 load
+    static constexpr int STAGE = 2 * TILE;  // X (k or q), Y (v or dy)
+    static constexpr int OFF_META = NST * STAGE;
+    static constexpr int OFF_RED = OFF_META + NST * static_cast<int>(sizeof(TileMeta));  // [256] floats + [256] ints
+    static constexpr int OFF_BAR = OFF_RED + 256 * 8 + 64;
+    static constexpr int BYTES = OFF_BAR + 64;
+};
+
+struct SegParams {
+    CUtensorMap map_x, map_y;  // forward: k, v; reverse: q, dy
+    const TileMeta* meta;
+    float2* info;  // [B * H * G]
+    float* out;    // [B * H * G][D][D]
+    uint32_t* hdr;
+    int64_t L, H, n_tiles, tps;
+    int G;
+    uint64_t wait_ns;
+};
+
+// log2 weights below this underflow to 0 in fast_exp2 (flush-to-zero), so
+// every row of a tile past this offset contributes exactly nothing
+constexpr float kUnderflowLog2 = -152.f;
+
+template <int D, bool REV, bool NORM = false>
+__global__ void __launch_bounds__(kThreads, 1) seg_state_kernel(const __grid_constant__ SegParams p) {
+    // NORM: the Linear Transformer with phi for 64-channel heads: the X tile
+    // holds phi(k) (phi(q)) in its first 64 channels and zeros after; the
+    // forward's Y tile holds v and the columns [1, 1, 0, ...]; the reverse Y
+    // is the padded dy' (128 channels, loaded whole)
+    static_assert(!NORM || D == 128, "the normalised operands run at d = 128");
+    using S = SegSmem<D>;
+    constexpr int BX = NORM ? 64 : D;
+    constexpr int BY = (NORM && !REV) ? 64 : D;
+    extern __shared__ __align__(1024) unsigned char smem[];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int quarter = warp & 3, half = warp >> 2;
+    const int per_bh = p.G - 1;
+    const int64_t bh = blockIdx.x / per_bh;
+    const int g = static_cast<int>(blockIdx.x % per_bh) + (REV ? 1 : 0);
+    const int64_t b = bh / p.H, h = bh % p.H;
+    const int64_t c0 = static_cast<int64_t>(g) * p.tps, c1 = min(p.n_tiles, c0 + p.tps);
+    const TileMeta* gm = p.meta + bh * p.n_tiles;
+
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);  // [NST]
+    uint64_t* mbar = full + S::NST;                                   // [NST]: the contraction reading stage s is done
+    uint32_t* tslot = reinterpret_cast<uint32_t*>(mbar + S::NST);
+    float* red_f = reinterpret_cast<float*>(smem + S::OFF_RED);
+    int* red_i = reinterpret_cast<int*>(smem + S::OFF_RED + 256 * 4);
+    int* bcast = reinterpret_cast<int*>(smem + S::OFF_RED + 256 * 8);
+    TileMeta* metas = reinterpret_cast<TileMeta*>(smem + S::OFF_META);
+    const uint32_t sbase = smem_addr(smem);
+
+    if (tid == 0) {
+        for (int i = 0; i < S::NST; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&mbar[i], 1);
+        }
+        fence_mbar_init();
+        prefetch_tensormap(&p.map_x);
+        prefetch_tensormap(&p.map_y);
+    }
+    if (warp == 0) tc::alloc(tslot, 128);
+    if (NORM) {
+        for (int st = 0; st < S::NST; ++st) {
+            const_box<kThreads>(smem + st * S::STAGE, tid, false);
+            if (!REV) const_box<kThreads>(smem + st * S::STAGE + S::TILE, tid, true);
+        }
+    }
+
+    // ---- which tiles: a pass over the segment's metadata ----
+    // Each thread takes a run of consecutive tiles: the sum of their log2
+    // decays (in order) and the latest (forward) / earliest (reverse) tile
+    // holding a begin flag.
+    const int64_t n = c1 - c0;
+    const int64_t per = (n + kThreads - 1) / kThreads;
+    const int64_t a0 = c0 + tid * per, a1 = min(c1, a0 + per);
+    float run = 0.f;
+    int flag_tile = REV ? 0x7fffffff : -1;
+    for (int64_t c = a0; c < a1; ++c) {
+        run += gm[c].lam2[T - 1];
+        if (gm[c].has_start != 0) flag_tile = REV ? min(flag_tile, static_cast<int>(c - c0)) : static_cast<int>(c - c0);
+    }
+    red_f[tid] = run;
+    red_i[tid] = flag_tile;
+    __syncthreads();
+    if (warp == 0) {
+        // exclusive prefix of the runs' sums in thread order (fixed order), and the flag tile
+        float v[8];
+        float sum8 = 0.f;
+        int ft = REV ? 0x7fffffff : -1;
+#pragma unroll
+        for (int x = 0; x < 8; ++x) {
+            v[x] = red_f[lane * 8 + x];
+            sum8 += v[x];
+            const int f = red_i[lane * 8 + x];
+            ft = REV ? min(ft, f) : max(ft, f);
+        }
+        float incl = sum8;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const float o = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += o;
+            const int of = __shfl_xor_sync(0xffffffffu, ft, off);
+            ft = REV ? min(ft, of) : max(ft, of);
+        }
+        float pre = incl - sum8;
+#pragma unroll
+        for (int x = 0; x < 8; ++x) {
+            red_f[lane * 8 + x] = pre;  // sum of the runs before thread lane * 8 + x
+            pre += v[x];
+        }
+        const float total = __shfl_sync(0xffffffffu, incl, 31);
+        if (lane == 0) {
+            bcast[0] = ft;
+            bcast[1] = __float_as_int(total);
+            const bool has_flag = REV ? ft != 0x7fffffff : ft >= 0;
+            p.info[bh * p.G + g] = make_float2(has_flag ? 1.f : 0.f, total);
+        }
+    }
+    __syncthreads();
+    const int ft = bcast[0];
+    const float total = __int_as_float(bcast[1]);
+    // the farthest tile (from the end forward, from the start reverse) whose
+    // offset is still above the underflow bound: offsets only decrease
+    {
+        const float before = red_f[tid];  // the sum over tiles c0 .. a0 - 1
+        int far = REV ? -1 : 0x7fffffff;
+        if (REV) {
+            float off = before;  // sum over tiles c0 .. c - 1
+            for (int64_t c = a0; c < a1; ++c) {
+                if (off >= kUnderflowLog2) far = static_cast<int>(c - c0);
+                off += gm[c].lam2[T - 1];
+            }
+        } else {
+            float off = total - before;  // sum over tiles a0 .. c1 - 1, then c + 1 .. c1 - 1
+            for (int64_t c = a0; c < a1; ++c) {
+                off -= gm[c].lam2[T - 1];
+                if (off >= kUnderflowLog2 && far == 0x7fffffff) far = static_cast<int>(c - c0);
+            }
+        }
+        red_i[tid] = far;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        int far = REV ? -1 : 0x7fffffff;
+#pragma unroll
+        for (int x = 0; x < 8; ++x) far = REV ? max(far, red_i[lane * 8 + x]) : min(far, red_i[lane * 8 + x]);
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+            const int o = __shfl_xor_sync(0xffffffffu, far, off);
+            far = REV ? max(far, o) : min(far, o);
+        }
+        if (lane == 0) bcast[2] = far;
+    }
+    __syncthreads();
+    const int far = bcast[2];
+    // tiles processed, in order: forward c1 - 1 down to c0 + lo, reverse c0 up to c0 + hi
+    int n_proc;
+    if (REV) {
+        const int hi = min(ft == 0x7fffffff ? static_cast<int>(n) - 1 : ft, far);
+        n_proc = hi + 1;
+    } else {
+        const int lo = max(ft < 0 ? 0 : ft, far);
+        n_proc = static_cast<int>(n) - lo;
+    }
+    auto tile_of = [&](int i) -> int64_t { return REV ? c0 + i : c1 - 1 - i; };
+
+    // thread 0: TMA loads of processed tile i into stage i % NST
+    auto issue = [&](int i) {
+        const int st = i % S::NST;
+        mbar_arrive_expect_tx(&full[st], T * BX * 2 + T * BY * 2 + sizeof(TileMeta));
+        const int64_t c = tile_of(i);
+        tma_tile<BX>(sbase + st * S::STAGE, &p.map_x, h, c * T, b, &full[st]);
+        tma_tile<BY>(sbase + st * S::STAGE + S::TILE, &p.map_y, h, c * T, b, &full[st]);
+        bulk_g2s(&metas[st], gm + c, sizeof(TileMeta), &full[st]);
+    };
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    const uint32_t tm = *tslot;
+    int issued = 0;  // thread 0: tiles whose loads were issued
+    if (tid == 0) {
+        for (; issued < S::NST - 1 && issued < n_proc; ++issued) issue(issued);
+    }
+    constexpr uint32_t ID_XY = tc::idesc_bf16(D, D, true, true);
+    bool failed = false;
+    float off = 0.f;  // log2 decay between the segment's end (start) and this tile
+    int i = 0;
+#pragma unroll 1
+    for (; i < n_proc; ++i) {
+        const int st = i % S::NST;
+        bool issue_ok = true;
+        if (tid == 0 && issued < n_proc) {
+            // the stage of tile i + NST - 1 held tile i - 1: free once its contraction is done
+            if (i >= 1) issue_ok = wait_mbar(&mbar[(i - 1) % S::NST], ((i - 1) / S::NST) & 1, p.wait_ns);
+            if (issue_ok) issue(issued++);
+        }
+        const bool ok = wait_mbar(&full[st], (i / S::NST) & 1, p.wait_ns);
+        if (__syncthreads_or(!ok || !issue_ok)) {
+            failed = true;
+            break;
+        }
+        const TileMeta& mc = metas[st];
+        const int64_t t0 = tile_of(i) * T;
+        if (NORM) {
+            phi_box<kThreads>(smem + st * S::STAGE, tid, p.L - t0);
+            __syncthreads();
+        }
+        // X~ = w (.) X in place
+        if (REV) {
+            scale_rows_sw<D>(smem + st * S::STAGE, tid,
+                             [&](int r) { return mc.seg[r] < 0 ? fast_exp2(off + mc.lam2[r]) : 0.f; });
+        } else {
+            const float lend = mc.lam2[T - 1];
+            const int ls = mc.last_start;
+            scale_rows_sw<D>(smem + st * S::STAGE, tid,
+                             [&](int r) { return r >= ls ? fast_exp2(off + lend - mc.lam2[r]) : 0.f; });
+        }
+        off += mc.lam2[T - 1];
+        tc::fence_smem_to_async();
+        tc::fence_before();
+        __syncthreads();
+        tc::fence_after();
+        if (tid == 0) {
+            const uint32_t sx = sbase + st * S::STAGE, sy = sx + S::TILE;
+#pragma unroll
+            for (int kk = 0; kk < T / 16; ++kk)
+                tc::mma(tm, desc_sw_mn(sx, kk), desc_sw_mn(sy, kk), ID_XY, i > 0 || kk > 0);
+            tc::commit(&mbar[st]);
+        }
+    }
+    // the last contraction (and with it every earlier one) is done
+    const bool ok = !failed && wait_mbar(&mbar[(n_proc - 1) % S::NST], ((n_proc - 1) / S::NST) & 1, p.wait_ns);
+    if (!ok && tid == 0) {
+        record_error(p.hdr, DEV_MMA_TIMEOUT);
+        // drain every issued load and contraction before TMEM and shared memory go away
+        for (int j = i; j < issued; ++j) wait_mbar(&full[j % S::NST], (j / S::NST) & 1, kDrainNs);
+        if (i >= 1) wait_mbar(&mbar[(i - 1) % S::NST], ((i - 1) / S::NST) & 1, kDrainNs);
+    }
+    __syncthreads();
+    tc::fence_after();
+    if (ok) {
+        const int srow = state_row<D>(quarter, lane);
+        const uint32_t lane_base = tm + (static_cast<uint32_t>(32 * quarter) << 16);
+        float* dst = p.out + (bh * p.G + g) * D * D;
+        constexpr int SC = D / 2;
+#pragma unroll 1
+        for (int cc = 0; cc < SC / 16; ++cc) {
+            const int j0 = half * SC + cc * 16;
+            float v[16];
+            tc::ld16(lane_base + j0, v);
+            if (srow >= 0) {
+#pragma unroll
+                for (int x = 0; x < 16; x += 4)
+                    *reinterpret_cast<float4*>(dst + srow * D + j0 + x) = make_float4(v[x], v[x + 1], v[x + 2], v[x + 3]);
+            }
+        }
+    }
+    tc::fence_before();
+    __syncthreads();
+    tc::fence_after();
+    if (warp == 0) tc::dealloc(tm, 128);
+}
+
+// The resettable scan over the segments, in place (one thread per 4 state
+// entries, segments in order):
+//   forward: E_0 = S0 (or 0);  buf[g] <- [no flag in g] a_g E_g + X_g = E_{g+1}
+//   reverse: R_{G-1} = dS_last (or 0);  buf[g] <- [no flag in g] a_g R_g + X_g = R_{g-1}
+// with a_g = exp2(info[g].y) the segment's total decay; the flag selects, as
+// in Theorem 3.2, so nothing from before a begin flag (NaN included) crosses it.
+template <bool REV>
+__global__ void __launch_bounds__(256) seg_carry_kernel(float* __restrict__ buf, const float2* __restrict__ info,
+                                                       const float* __restrict__ init, int G, int DD) {
+    const int64_t bh = blockIdx.y;
+    const int e = (blockIdx.x * 256 + threadIdx.x) * 4;
+    if (e >= DD) return;
+    float* base = buf + bh * G * DD + e;
+    const float2* inf = info + bh * G;
+    float4 c = init != nullptr ? *reinterpret_cast<const float4*>(init + bh * DD + e) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+    for (int k = 0; k < G - 1; ++k) {
+        const int g = REV ? G - 1 - k : k;
+        const float2 f = inf[g];
+        const float4 x = *reinterpret_cast<const float4*>(base + static_cast<int64_t>(g) * DD);
+        if (f.x != 0.f) {
+            c = x;
+        } else {
+            const float a = exp2f(f.y);
+            c = make_float4(fmaf(a, c.x, x.x), fmaf(a, c.y, x.y), fmaf(a, c.z, x.z), fmaf(a, c.w, x.w));
+        }
+        *reinterpret_cast<float4*>(base + static_cast<int64_t>(g) * DD) = c;
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -1068,11 +1333,11 @@ struct BwdParams {
     float* gpart;       // [B * H * G] per-segment sums of dL/dlog(gamma) (per-head mode)
     float* dS0;
     const TileMeta* meta;
-    const int64_t* seg_first;
+    const float* carry;  // [B * H * G][D][D]: the reverse state leaving each segment (g >= 1)
     const float* dlam_f;
     const uint16_t* states;
     uint32_t* hdr;
-    int64_t B, L, H, n_tiles;
+    int64_t B, L, H, n_tiles, tps;
     int G;
     uint64_t wait_ns;
     int64_t fail_cta;  // test knob (see FwdParams)
@@ -1126,21 +1391,13 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     const int64_t bh = blockIdx.x / p.G;
     const int g = static_cast<int>(blockIdx.x % p.G);
     const int64_t b = bh / p.H, h = bh % p.H;
-    const int64_t* sf = p.seg_first + b * p.G;
-    const int64_t seg_lo = sf[g];
-    if (seg_lo < 0) {
-        if (p.gpart != nullptr && tid == 0) p.gpart[bh * p.G + g] = 0.f;
-        return;
-    }
-    int64_t seg_hi = p.L;
-    for (int g2 = g + 1; g2 < p.G; ++g2) {
-        if (sf[g2] >= 0) {
-            seg_hi = sf[g2];
-            break;
-        }
-    }
-    const int64_t tile_lo = seg_lo / T, tile_hi = (seg_hi + T - 1) / T;  // tiles [tile_lo, tile_hi)
-    const int64_t row_stride = p.H * DOUT;
+    // this segment: tiles [tile_lo, tile_hi), steps up to seg_hi (the tape end for the last)
+    const int64_t tile_lo = static_cast<int64_t>(g) * p.tps, tile_hi = min(p.n_tiles, tile_lo + p.tps);
+    const int64_t seg_hi = min(p.L, tile_hi * T);
+    // the reverse state entering the segment's last step: dS_last for the last
+    // segment, else the carry
+    const float* g_in = g == p.G - 1 ? (p.dS_last != nullptr ? p.dS_last + bh * D * D : nullptr)
+                                     : p.carry + (bh * p.G + g + 1) * D * D;
 
     uint64_t* bar1 = reinterpret_cast<uint64_t*>(smem + S::OFF_BAR);
     uint64_t* bar2 = bar1 + 1;
@@ -1192,7 +1449,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         tma_tile<BKV>(sK, &p.map_k, h, tile * T, b, full);
         bulk_g2s(smem + S::OFF_SS, p.states + (bh * p.n_tiles + tile) * D * D, D * D * 2, full);
     };
-    bool have_g = seg_hi == p.L && p.dS_last != nullptr;  // a reverse state enters the current tile
+    bool have_g = g_in != nullptr;  // a reverse state enters the current tile
 
     if (tid == 0) {
         mbar_init(bar1, 1);
@@ -1224,9 +1481,9 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     constexpr int SC = D / 4;  // state and output columns per thread
     constexpr int PC = T / 4;  // score columns per thread
 
-    // ---- incoming reverse state: dS_last for the segment that ends the tape ----
+    // ---- incoming reverse state ----
     if (have_g) {
-        const float* src = p.dS_last + bh * D * D;
+        const float* src = g_in;
 #pragma unroll 1
         for (int cc = 0; cc < SC / 16; ++cc) {
             const int j0 = cq * SC + cc * 16;
@@ -1265,8 +1522,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
 #pragma unroll 1
     for (int64_t tile = tile_hi - 1; tile >= tile_lo; --tile, ++it) {
         const int64_t t0 = tile * T;
-        const int r_lo = static_cast<int>(max(static_cast<int64_t>(0), seg_lo - t0));
-        const int r_hi = static_cast<int>(min(static_cast<int64_t>(T), seg_hi - t0));
+        const int r_hi = static_cast<int>(min(static_cast<int64_t>(T), seg_hi - t0));  // rows inside the tape
         bool ok = wait_mbar(full, it & 1, p.wait_ns);
         tc::fence_smem_to_async();
         tc::fence_before();
@@ -1337,7 +1593,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         float dlf = 0.f, gmt = 1.f;
         if (warp < 4) {
             const int t = 32 * warp + lane;
-            if (t >= r_lo && t < r_hi) {
+            if (t < r_hi) {
                 const int64_t idx = (b * p.L + t0 + t) * p.H + h;
                 dlf = p.dlam_f[idx];
                 if (p.dgamma != nullptr) gmt = p.gamma_per_step ? p.gamma[idx] : p.gamma[h];
@@ -1513,28 +1769,15 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
 
         // ---- epilogue (while B3 runs): dk = dK + w_out dKi, then dv, each staged and
         // stored on its own, so that the dk stores drain while dv is staged ----
-        const int full_rows = static_cast<int>(min(static_cast<int64_t>(T), p.L - t0));
-        // warp 0: the staged tile's rows of this segment (one TMA store per 32 channels
-        // for a whole tile, else row by row)
+        // warp 0: one TMA store of the staged tile per 32 channels (rows past L are clipped)
         auto store_tile = [&](bool is_dv) {
             const CUtensorMap* map = is_dv ? &p.map_dv : &p.map_dk;
-            if (r_lo == 0 && r_hi == full_rows) {
-                if (lane == 0) {
+            if (lane == 0) {
 #pragma unroll
-                    for (int m = 0; m < DOUT / 32; ++m)
-                        tma_store_4d(map, sbase + (is_dv ? S::dv_chunk(m) : S::dk_chunk(m)), 32 * m,
-                                     static_cast<int>(h), static_cast<int>(t0), static_cast<int>(b));
-                    bulk_commit();
-                }
-            } else {
-                float* ob = (is_dv ? p.dv : p.dk) + ((b * p.L + t0) * p.H + h) * DOUT;
-                for (int e = lane; e < (r_hi - r_lo) * (DOUT / 4); e += 32) {
-                    const int r = r_lo + e / (DOUT / 4), j = (e % (DOUT / 4)) * 4;
-                    const int in = r * 128 + ((((j & 31) >> 2) ^ (r & 7)) << 4);
-                    const int ch = is_dv ? S::dv_chunk(j >> 5) : S::dk_chunk(j >> 5);
-                    *reinterpret_cast<float4*>(ob + static_cast<int64_t>(r) * row_stride + j) =
-                        *reinterpret_cast<const float4*>(smem + ch + in);
-                }
+                for (int m = 0; m < DOUT / 32; ++m)
+                    tma_store_4d(map, sbase + (is_dv ? S::dv_chunk(m) : S::dk_chunk(m)), 32 * m, static_cast<int>(h),
+                                 static_cast<int>(t0), static_cast<int>(b));
+                bulk_commit();
             }
         };
         {
@@ -1581,7 +1824,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
                 for (int w2 = 0; w2 < kRThreads / 32; ++w2) iv += st_iv[w2];
                 iv *= mc.a;
             }
-            const bool in = t >= r_lo && t < r_hi;
+            const bool in = t < r_hi;
             const bool is_start = mc.seg[t] == t;
             float dl = 0.f;
             if (in && !is_start) dl = st_intra[t] + (lower + xpre_in) + iv + dlf;
@@ -1626,7 +1869,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         // ---- G_{c-1} -> bf16 operand for the next tile (and dS0 at the tape start) ----
         {
             const bool last = tile == tile_lo;
-            const bool write_ds0 = last && seg_lo == 0 && p.dS0 != nullptr;
+            const bool write_ds0 = last && g == 0 && p.dS0 != nullptr;
             uint32_t gv[SC];
 #pragma unroll
             for (int cc = 0; cc < SC / 16; ++cc) tc::ld16_nowait(lane_base + S::COL_G + cq * SC + cc * 16, gv + cc * 16);
@@ -1833,36 +2076,54 @@ bool tile_map_y(CUtensorMap* m, const void* base, int64_t B, int64_t L, int64_t 
 
 }  // namespace
 
-memoroid_status_t launch_segment_plan(const uint8_t* start, int64_t B, int64_t L, int64_t seg_len, int64_t G,
-                                      int64_t* first, cudaStream_t stream) {
-    if (B * G == 0) return MEMOROID_OK;
-    const int64_t blocks = (B * G * 32 + 255) / 256;
-    plan_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(start, B, L, seg_len, G, first);
-    return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
-}
-
 namespace {
-// Tile metadata and segment boundaries (shared by the forward and backward passes).
-memoroid_status_t launch_prep(const Args& a, const Plan& pl, TileMeta* meta, int64_t* seg_first,
-                              cudaStream_t stream) {
+// Tile metadata (shared by the forward and backward passes).
+memoroid_status_t launch_prep(const Args& a, const Plan& pl, TileMeta* meta, cudaStream_t stream) {
     const int64_t meta_blocks = (a.B * a.H * pl.n_tiles * 32 + 255) / 256;
     meta_kernel<<<static_cast<unsigned>(meta_blocks), 256, 0, stream>>>(a.gamma, a.gamma_per_step, a.start, a.B,
                                                                          a.L, a.H, pl.n_tiles, meta);
+    return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
+}
+
+// The states entering the segments (REV = false, from the X = k, Y = v
+// summaries and S0) or the reverse states entering them from the right
+// (REV = true, from X = q, Y = dy and dS_last): the summary kernel, then the
+// carry over the segments, in place in `buf`.  Nothing to do for one segment.
+template <int D, bool REV, bool NORM>
+memoroid_status_t launch_seg_carry(const Args& a, const Plan& pl, const TileMeta* meta, float2* info, float* buf,
+                                   const CUtensorMap& map_x, const CUtensorMap& map_y, const float* init,
+                                   uint32_t* hdr, cudaStream_t stream) {
+    if (pl.G <= 1) return MEMOROID_OK;
+    SegParams p;
+    p.map_x = map_x;
+    p.map_y = map_y;
+    p.meta = meta;
+    p.info = info;
+    p.out = buf;
+    p.hdr = hdr;
+    p.L = a.L;
+    p.H = a.H;
+    p.n_tiles = pl.n_tiles;
+    p.tps = pl.tps;
+    p.G = static_cast<int>(pl.G);
+    p.wait_ns = debug_knobs().wait_ns;
+    if (set_smem(seg_state_kernel<D, REV, NORM>, SegSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    seg_state_kernel<D, REV, NORM><<<static_cast<unsigned>(a.B * a.H * (pl.G - 1)), kThreads, SegSmem<D>::BYTES,
+                                     stream>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
-    const int64_t plan_blocks = (a.B * pl.G * 32 + 255) / 256;
-    plan_kernel<<<static_cast<unsigned>(plan_blocks), 256, 0, stream>>>(a.start, a.B, a.L, pl.tps * T, pl.G,
-                                                                         seg_first);
-    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
-    return MEMOROID_OK;
+    const dim3 grid(static_cast<unsigned>((D * D / 4 + 255) / 256), static_cast<unsigned>(a.B * a.H));
+    seg_carry_kernel<REV><<<grid, 256, 0, stream>>>(buf, info, init, static_cast<int>(pl.G), D * D);
+    return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
 }
 
 template <int D, bool NORM = false>
 memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, cudaStream_t stream) {
     unsigned char* ws = static_cast<unsigned char*>(a.workspace);
     TileMeta* meta = reinterpret_cast<TileMeta*>(ws + ly.meta);
-    int64_t* seg_first = reinterpret_cast<int64_t*>(ws + ly.seg_first);
+    float2* info = reinterpret_cast<float2*>(ws + ly.info);
+    float* carry = reinterpret_cast<float*>(ws + ly.carry_f);
     uint32_t* hdr = reinterpret_cast<uint32_t*>(ws);
-    const memoroid_status_t st = launch_prep(a, pl, meta, seg_first, stream);
+    memoroid_status_t st = launch_prep(a, pl, meta, stream);
     if (st != MEMOROID_OK) return st;
 
     FwdParams p;
@@ -1870,6 +2131,8 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     if (!tile_map(&p.map_q, a.q, a.B, a.L, a.H, KQ) || !tile_map(&p.map_k, a.k, a.B, a.L, a.H, KQ) ||
         !tile_map(&p.map_v, a.v, a.B, a.L, a.H, KQ) || !tile_map_y(&p.map_y, a.y, a.B, a.L, a.H, KQ))
         return MEMOROID_ERR_CUDA;
+    st = launch_seg_carry<D, false, NORM>(a, pl, meta, info, carry, p.map_k, p.map_v, a.S0, hdr, stream);
+    if (st != MEMOROID_OK) return st;
     p.den = NORM ? a.den : nullptr;
     p.q = static_cast<const uint16_t*>(a.q);
     p.k = static_cast<const uint16_t*>(a.k);
@@ -1877,7 +2140,7 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     p.S0 = a.S0;
     p.y = a.y;
     p.meta = meta;
-    p.seg_first = seg_first;
+    p.carry = carry;
     p.S_last = a.S_last;
     p.hdr = hdr;
     p.B = a.B;
@@ -1900,14 +2163,16 @@ template <int D, bool HALF_OUT = false, bool NORM = false>
 memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, cudaStream_t stream) {
     unsigned char* ws = static_cast<unsigned char*>(a.workspace);
     TileMeta* meta = reinterpret_cast<TileMeta*>(ws + ly.meta);
-    int64_t* seg_first = reinterpret_cast<int64_t*>(ws + ly.seg_first);
+    float2* info = reinterpret_cast<float2*>(ws + ly.info);
+    float* carry_f = reinterpret_cast<float*>(ws + ly.carry_f);
+    float* carry_r = reinterpret_cast<float*>(ws + ly.carry_r);
     // the bf16 operand copy of grad_y, unless the caller passes grad_y in bf16 already
     const uint16_t* dy16 = a.grad_y16 != nullptr ? a.grad_y16 : reinterpret_cast<uint16_t*>(ws + ly.dy16);
     uint16_t* states = reinterpret_cast<uint16_t*>(ws + ly.states);
     float* dlam_f = reinterpret_cast<float*>(ws + ly.dlam_f);
     float* gpart = reinterpret_cast<float*>(ws + ly.gpart);
     uint32_t* hdr = reinterpret_cast<uint32_t*>(ws);
-    memoroid_status_t st = launch_prep(a, pl, meta, seg_first, stream);
+    memoroid_status_t st = launch_prep(a, pl, meta, stream);
     if (st != MEMOROID_OK) return st;
 
     if (a.grad_y16 == nullptr) {
@@ -1918,9 +2183,23 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
         if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     }
 
+    // the operand maps of pass R, also read by the segment summaries
+    BwdParams r;
+    constexpr int BKV = NORM ? 64 : D;  // channels of q, k, v in memory (the normalised path: unpadded)
+    if (!tile_map(&r.map_q, a.q, a.B, a.L, a.H, BKV) || !tile_map(&r.map_k, a.k, a.B, a.L, a.H, BKV) ||
+        !tile_map(&r.map_v, a.v, a.B, a.L, a.H, BKV) || !tile_map(&r.map_dy, dy16, a.B, a.L, a.H, D) ||
+        !tile_map_y(&r.map_dk, a.dk, a.B, a.L, a.H, HALF_OUT ? 64 : D) ||
+        !tile_map_y(&r.map_dv, a.dv, a.B, a.L, a.H, HALF_OUT ? 64 : D))
+        return MEMOROID_ERR_CUDA;
+    // the forward states entering the segments (for pass F) and the reverse
+    // states entering them from the right (for pass R)
+    st = launch_seg_carry<D, false, NORM>(a, pl, meta, info, carry_f, r.map_k, r.map_v, a.S0, hdr, stream);
+    if (st != MEMOROID_OK) return st;
+    st = launch_seg_carry<D, true, NORM>(a, pl, meta, info, carry_r, r.map_q, r.map_dy, a.dS_last, hdr, stream);
+    if (st != MEMOROID_OK) return st;
+
     // pass F: dq = S dy, with (q, k, v) -> (dy, v, k)
     FwdParams f;
-    constexpr int BKV = NORM ? 64 : D;  // channels of q, k, v in memory (the normalised path: unpadded)
     if (!tile_map(&f.map_q, dy16, a.B, a.L, a.H, D) || !tile_map(&f.map_k, a.v, a.B, a.L, a.H, BKV) ||
         !tile_map(&f.map_v, a.k, a.B, a.L, a.H, BKV) ||
         !tile_map_y(&f.map_y, a.dq, a.B, a.L, a.H, HALF_OUT ? 64 : D) || !tile_map(&f.map_zq, a.q, a.B, a.L, a.H, BKV))
@@ -1932,7 +2211,7 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     f.S0 = a.S0;
     f.y = a.dq;
     f.meta = meta;
-    f.seg_first = seg_first;
+    f.carry = carry_f;
     f.S_last = nullptr;
     f.hdr = hdr;
     f.B = a.B;
@@ -1950,12 +2229,6 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
 
     // pass R: dk, dv, dgamma, dS0
-    BwdParams r;
-    if (!tile_map(&r.map_q, a.q, a.B, a.L, a.H, BKV) || !tile_map(&r.map_k, a.k, a.B, a.L, a.H, BKV) ||
-        !tile_map(&r.map_v, a.v, a.B, a.L, a.H, BKV) || !tile_map(&r.map_dy, dy16, a.B, a.L, a.H, D) ||
-        !tile_map_y(&r.map_dk, a.dk, a.B, a.L, a.H, HALF_OUT ? 64 : D) ||
-        !tile_map_y(&r.map_dv, a.dv, a.B, a.L, a.H, HALF_OUT ? 64 : D))
-        return MEMOROID_ERR_CUDA;
     r.q = static_cast<const uint16_t*>(a.q);
     r.k = static_cast<const uint16_t*>(a.k);
     r.v = static_cast<const uint16_t*>(a.v);
@@ -1969,7 +2242,7 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     r.gpart = (a.dgamma != nullptr && !a.gamma_per_step) ? gpart : nullptr;
     r.dS0 = a.dS0;
     r.meta = meta;
-    r.seg_first = seg_first;
+    r.carry = carry_r;
     r.dlam_f = dlam_f;
     r.states = states;
     r.hdr = hdr;
@@ -1977,6 +2250,7 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     r.L = a.L;
     r.H = a.H;
     r.n_tiles = pl.n_tiles;
+    r.tps = pl.tps;
     r.G = static_cast<int>(pl.G);
     r.wait_ns = debug_knobs().wait_ns;
     r.fail_cta = debug_knobs().withhold_ticket;
@@ -1997,8 +2271,10 @@ size_t fwd_workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D) { return 
 
 int kernels_per_call(int64_t B, int64_t L, int64_t H, int backward, int with_dgamma_per_head) {
     if (B == 0 || L == 0 || H == 0) return 0;
-    if (!backward) return 3;
-    return 6 + (with_dgamma_per_head ? 1 : 0);
+    // the segment summary and carry kernels run once per direction when there are several segments
+    const int carry = make_plan(B, L, H).G > 1 ? 2 : 0;
+    if (!backward) return 2 + carry;  // meta, forward
+    return 4 + 2 * carry + (with_dgamma_per_head ? 1 : 0);  // meta, bf16 copy, pass F, pass R
 }
 
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t stream) {

@@ -121,6 +121,38 @@ def test_fwd_one_segment_per_tape():
     assert rel_err(S_last, S_ref) <= TOL
 
 
+def _long_episode_tape(d, gamma_lo, gamma_hi, seed, starts=()):
+    # B = 1, L = 2^16, 2 heads: 512 tiles cut into many segments, begin flags
+    # only at the given steps (none: one episode continuing from S0), a
+    # per-step gamma drawn from [gamma_lo, gamma_hi]
+    L = 1 << 16
+    t = tapegen.linattn_tape(1, L, 2, d, d, seed=seed, gamma_mode="step", with_grad=True, with_S0=True,
+                             start_mode="open")
+    rng = np.random.default_rng(seed + 1)
+    t["gamma"] = rng.uniform(gamma_lo, gamma_hi, size=(1, L, 2)).astype(np.float32)
+    for s_ in starts:
+        t["start"][0, s_] = 1
+    return t
+
+
+@pytest.mark.parametrize("d,gamma_lo,gamma_hi,starts", [
+    (64, 0.9995, 1.0, ()),              # one episode: the state crosses every segment boundary
+    (128, 0.9999, 1.0, (40000,)),       # two episodes, the second from the middle of a segment
+    (64, 0.5, 0.6, ()),                 # strong decay: the segment summaries skip underflowing tiles
+    (128, 1.0, 1.0, (777, 30001)),      # gamma = 1, flags in two segments only
+])
+def test_reset_sparse_long_tape(d, gamma_lo, gamma_hi, starts):
+    # the inter-segment carry: a tape with few or no begin flags runs on as
+    # many segments (CTAs) as any other, each starting from the state that
+    # the carry brings in; forward and backward against the oracle
+    t = _long_episode_tape(d, gamma_lo, gamma_hi, tapegen.seed_for(70 + d + len(starts)), starts)
+    y, S_last = run_gpu_fwd(t, S0=t["S0"])
+    y_ref, S_ref = run_oracle_fwd(t, t["S0"])
+    assert rel_err(y, y_ref) <= TOL
+    assert rel_err(S_last, S_ref) <= TOL
+    check_bwd(t, t["S0"], t["grad_S_last"])
+
+
 def test_fwd_episode_isolation_bitwise():
     # changing q/k/v inside one episode leaves every other episode's outputs unchanged, bit for bit
     t = tapegen.linattn_tape(1, 2000, 2, 64, 64, seed=tapegen.seed_for(57), mean=200.0, with_grad=False)

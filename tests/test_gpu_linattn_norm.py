@@ -109,6 +109,18 @@ def test_paper_model_gamma_one():
     check(t, False)
 
 
+@pytest.mark.parametrize("d,with_states", [(64, True), (32, False)])
+def test_one_long_episode(d, with_states):
+    # one episode over 2^15 steps with gamma = 1 (the paper's model): the
+    # normalised pair crosses every segment boundary through the carry between
+    # segments (d = 64: operands built inside the kernels; d = 32: padded)
+    t = make(1, 1 << 15, 2, d, tapegen.seed_for(817 + d), 1.0, "step", with_states, start_mode="none")
+    t["gamma"][:] = 1.0
+    if with_states:
+        t["start"][:, 0] = 0
+    check(t, with_states)
+
+
 def test_all_start_gives_v():
     # one term per step: the weight cancels and y = v
     t = make(1, 1000, 2, 32, tapegen.seed_for(811), 1.0, "step", False, start_mode="all")
