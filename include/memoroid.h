@@ -181,7 +181,8 @@ int memoroid_scan_linattn_kernels_per_call(int64_t B, int64_t L, int64_t H, int6
  *   v           bf16 [B, L, H, dv]
  *   gamma       fp32 [H] (gamma_per_step = 0) or [B, L, H]; the decay applied
  *               to S_{t-1} at step t, ignored at start steps.  Values are
- *               used through log2(gamma), clamped below at -126.
+ *               used through log2(gamma), clamped to [-126, 0]: a decay
+ *               above 1 acts as 1, one below 2^-126 (0 included) as 2^-126.
  *   start       uint8 [B, L], nonzero = b_t (first step of an episode)
  *   S0          fp32 [B, H, dk, dv] or NULL
  *   y           fp32 [B, L, H, dv] output

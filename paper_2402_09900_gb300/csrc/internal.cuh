@@ -151,6 +151,9 @@ struct Args {
     // backward only: 64 (with D = 128) writes only the first 64 columns of dq,
     // dk, dv, as [B, L, H, 64] arrays; 0 writes all D
     int64_t out_cols = 0;
+    // backward only: >= 0 adds column fold_col of dq to every column of dq (the
+    // normalised backward's sum channel); -1 = off
+    int64_t fold_col = -1;
 };
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t H, int64_t D);      // forward and backward

@@ -308,6 +308,73 @@ __device__ __forceinline__ void phi_box(unsigned char* slot, int tid, int64_t va
     }
 }
 
+// psi(z) = ELU(z) = phi(z) - 1 in place on the first 64-channel box (the
+// normalised backward's key operand; rows at or past `valid` become 0).
+template <int NT>
+__device__ __forceinline__ void psi_box(unsigned char* slot, int tid, int64_t valid) {
+#pragma unroll
+    for (int i = 0; i < T * 8 / NT; ++i) {
+        const int unit = i * NT + tid, row = unit / 8;
+        uint4* a = reinterpret_cast<uint4*>(slot + unit * 16);
+        uint4 u = *a;
+        uint32_t* w = reinterpret_cast<uint32_t*>(&u);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = unpack_bf16x2(w[e]);
+            w[e] = row < valid ? pack_bf16x2(f.x > 0.f ? f.x : __expf(f.x) - 1.f, f.y > 0.f ? f.y : __expf(f.y) - 1.f)
+                               : 0u;
+        }
+        *a = u;
+    }
+}
+
+// Sum of the 8 values of a 16-byte unit of bf16, in channel order.
+__device__ __forceinline__ float unit_sum(const uint4& u) {
+    const uint32_t* w = reinterpret_cast<const uint32_t*>(&u);
+    float acc = 0.f;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const float2 f = unpack_bf16x2(w[e]);
+        acc += f.x;
+        acc += f.y;
+    }
+    return acc;
+}
+
+// The normalised backward's query operand in place: phi on the first box (as
+// phi_box) and, in channels 64 and 65 of the second box, sigma = sum of the
+// row's 64 phi values as a bf16 pair (hi, lo = bf16(sigma - hi)); the rest of
+// that 16-byte unit is 0 (the other units of the box are zeros already).  The
+// 8 units of a row are 8 consecutive threads: unit sums in channel order,
+// then a fixed butterfly over the units (the same association as the padded
+// operands' builder, whatever the swizzle).
+template <int NT>
+__device__ __forceinline__ void phiq_box(unsigned char* slot, int tid, int64_t valid) {
+#pragma unroll
+    for (int i = 0; i < T * 8 / NT; ++i) {
+        const int unit = i * NT + tid, row = unit / 8;
+        uint4* a = reinterpret_cast<uint4*>(slot + unit * 16);
+        uint4 u = *a;
+        uint32_t* w = reinterpret_cast<uint32_t*>(&u);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = unpack_bf16x2(w[e]);
+            w[e] = row < valid ? pack_bf16x2(f.x > 0.f ? 1.f + f.x : __expf(f.x), f.y > 0.f ? 1.f + f.y : __expf(f.y))
+                               : 0u;
+        }
+        *a = u;
+        float sg = unit_sum(u);
+        sg += __shfl_xor_sync(0xffffffffu, sg, 1);
+        sg += __shfl_xor_sync(0xffffffffu, sg, 2);
+        sg += __shfl_xor_sync(0xffffffffu, sg, 4);
+        if ((unit & 7) == 0) {
+            const float hi = __bfloat162float(__float2bfloat16_rn(sg));
+            *reinterpret_cast<uint4*>(slot + T * 128 + row * 128 + ((row & 7) << 4)) =
+                make_uint4(pack_bf16x2(hi, sg - hi), 0u, 0u, 0u);
+        }
+    }
+}
+
 // The second 64-channel box of a [T x 128] operand slot as a constant: zeros,
 // or (ones) channels 64 and 65 of every row 1 and the rest 0.  Unit u of row r
 // holds channels 8 (u ^ (r % 8)) .. + 7 of the box.
@@ -385,6 +452,7 @@ struct FwdParams {
     // backward pass F only (see fwd_kernel<D, true>)
     float* dlam_f;       // [B, L, H]: the state-side terms of dL/dlog(gamma_t)
     uint16_t* states;    // [B, H, n_tiles, D, D] bf16: S_{c-1}^T before tiles without a begin flag
+    int fold_col;        // >= 0: output column added to every output column (pass F, normalised), else -1
 };
 
 
@@ -466,10 +534,13 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     // column 64 of the output is the normalizer; the epilogue writes
     // y = y'[:64] / y'[64] and the normalizer.
     // NORM with BWD: pass F of the normalised backward for 64-channel heads, on
-    // (dy', v', k') with dy' padded by the caller, v' = [v, 1, 1, 0] and
-    // k' = [phi(k), 0] built in the K and V slots the same way, and q' = [phi(q), 0]
-    // for the z term (phi applied as the tile is read).  The output rows are
-    // staged in the K slot, whose constant half is written again once they drain.
+    // (dy', v', k'') with dy' padded by the caller and v' = [v, 1, 1, 0],
+    // k'' = [psi(k), 1, 1, 0] (psi = phi - 1) built in the K and V slots the same
+    // way, and q'' = [phi(q), sigma_hi, sigma_lo, 0] for the z term (phi applied
+    // as the tile is read, sigma = sum of phi(q) formed by the upper half of the
+    // threads).  The output rows are staged in the K slot, whose constant half is
+    // written again once they drain.  Column 64 of the output (the gradient of
+    // the sum channel) is added to the other columns (fold_col).
     constexpr bool NF = NORM && !BWD, NB = NORM && BWD;
     constexpr int KQ = NF ? 64 : D;          // channels of the first contractions
     constexpr int BQ = NF ? 64 : D;          // channels loaded into the Q slot
@@ -537,7 +608,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         // zeros for k in the V slot); the loads only ever write the first halves
         for (int st = 0; st < 2; ++st) {
             const_box<kThreads>(smem + st * S::STAGE + S::TILE, tid, NB);
-            const_box<kThreads>(smem + st * S::STAGE + 2 * S::TILE, tid, NF);
+            const_box<kThreads>(smem + st * S::STAGE + 2 * S::TILE, tid, true);
         }
     }
     tc::fence_before();
@@ -633,7 +704,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 phi_box<kThreads>(smem + s * S::STAGE, tid, valid);
                 phi_box<kThreads>(smem + s * S::STAGE + S::TILE, tid, valid);
             } else {
-                phi_box<kThreads>(smem + s * S::STAGE + 2 * S::TILE, tid, valid);
+                psi_box<kThreads>(smem + s * S::STAGE + 2 * S::TILE, tid, valid);
             }
             tc::fence_smem_to_async();
             tc::fence_before();
@@ -785,48 +856,100 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 *reinterpret_cast<float4*>(yst + (j >> 5) * (T * 128) + ((((j & 31) >> 2) ^ (t & 7)) << 4)) =
                     make_float4(o[0], o[1], o[2], o[3]);
             }
-        } else if (HALF_OUT && half == 1) {
-            // output channels 64..127 are not written, and q' is zero there (d <= 64)
-            reinterpret_cast<float*>(smem + S::OFF_Z)[T + 32 * quarter + lane] = 0.f;
         } else {
             const int t = 32 * quarter + lane;
             const float w_in = (have_prev && mc.seg[t] < 0) ? fast_exp2(mc.lam2[t]) : 0.f;
             unsigned char* yst = smem + s * S::STAGE + Y_OFF + t * 128;  // row t of chunk 0
             const unsigned char* qs = smem + (stage_q(s) - sbase);  // pass F: the q tile
             const bool zrow = zload && w_in != 0.f;
+            // HALF_OUT: the upper half of the threads writes no output, only its part of z
+            const bool out_half = !(HALF_OUT && half == 1);
             // q' of the z term: the loaded values, or (normalised) phi of them rounded to bf16
             auto qpair = [](uint32_t w) {
                 float2 f = unpack_bf16x2(w);
                 if (NB) f = unpack_bf16x2(pack_bf16x2(f.x > 0.f ? 1.f + f.x : __expf(f.x), f.y > 0.f ? 1.f + f.y : __expf(f.y)));
                 return f;
             };
+            // the normalised backward: the output column of the sum channel, added to every column
+            float ofold = 0.f;
+            if (BWD && p.fold_col >= 0 && out_half) {
+                const int fb = p.fold_col & ~15, fx = p.fold_col & 15;
+                uint32_t fa[16], fi[16];
+                tc::ld16_nowait(lane_base + S::COL_YA + fb, fa);
+                if (have_prev) tc::ld16_nowait(lane_base + S::COL_YI + fb, fi);
+                tc::ld_wait();
+                float va = 0.f, vi = 0.f;
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    if (e == fx) {
+                        va = __uint_as_float(fa[e]);
+                        vi = __uint_as_float(fi[e]);
+                    }
+                }
+                ofold = have_prev ? fmaf(w_in, vi, va) : va;
+            }
             // BWD: z_t = w_in_t q_t . (S_{c-1} dy_t), the inter output dotted with q
             float zacc = 0.f;
 #pragma unroll
             for (int cc = 0; cc < SC / 32; ++cc) {
                 const int j0 = half * SC + cc * 32;
                 uint32_t ya[32], yi[32];
-                tc::ld16_nowait(lane_base + S::COL_YA + j0, ya);
-                tc::ld16_nowait(lane_base + S::COL_YA + j0 + 16, ya + 16);
+                if (out_half) {
+                    tc::ld16_nowait(lane_base + S::COL_YA + j0, ya);
+                    tc::ld16_nowait(lane_base + S::COL_YA + j0 + 16, ya + 16);
+                }
                 if (have_prev) {
                     tc::ld16_nowait(lane_base + S::COL_YI + j0, yi);
                     tc::ld16_nowait(lane_base + S::COL_YI + j0 + 16, yi + 16);
                 }
                 tc::ld_wait();
+                if (out_half) {
 #pragma unroll
-                for (int x = 0; x < 32; x += 4) {
-                    float4 o = make_float4(__uint_as_float(ya[x]), __uint_as_float(ya[x + 1]),
-                                           __uint_as_float(ya[x + 2]), __uint_as_float(ya[x + 3]));
-                    if (have_prev) {
-                        o.x = fmaf(w_in, __uint_as_float(yi[x]), o.x);
-                        o.y = fmaf(w_in, __uint_as_float(yi[x + 1]), o.y);
-                        o.z = fmaf(w_in, __uint_as_float(yi[x + 2]), o.z);
-                        o.w = fmaf(w_in, __uint_as_float(yi[x + 3]), o.w);
+                    for (int x = 0; x < 32; x += 4) {
+                        float4 o = make_float4(__uint_as_float(ya[x]), __uint_as_float(ya[x + 1]),
+                                               __uint_as_float(ya[x + 2]), __uint_as_float(ya[x + 3]));
+                        if (have_prev) {
+                            o.x = fmaf(w_in, __uint_as_float(yi[x]), o.x);
+                            o.y = fmaf(w_in, __uint_as_float(yi[x + 1]), o.y);
+                            o.z = fmaf(w_in, __uint_as_float(yi[x + 2]), o.z);
+                            o.w = fmaf(w_in, __uint_as_float(yi[x + 3]), o.w);
+                        }
+                        if (BWD && p.fold_col >= 0) {
+                            o.x += ofold;
+                            o.y += ofold;
+                            o.z += ofold;
+                            o.w += ofold;
+                        }
+                        const int j = j0 + x;  // 4 channels = one 16-byte unit
+                        *reinterpret_cast<float4*>(yst + (j >> 5) * (T * 128) + ((((j & 31) >> 2) ^ (t & 7)) << 4)) = o;
                     }
-                    const int j = j0 + x;  // 4 channels = one 16-byte unit
-                    *reinterpret_cast<float4*>(yst + (j >> 5) * (T * 128) + ((((j & 31) >> 2) ^ (t & 7)) << 4)) = o;
                 }
-                if (zrow) {
+                if (zrow && NB && half == 1) {
+                    // q'' channels 64 and 65: sigma as a bf16 pair (the rest of the upper half is 0)
+                    if (cc == 0) {
+                        float su[8];
+#pragma unroll
+                        for (int u = 0; u < 8; ++u) {
+                            const uint4 w = *reinterpret_cast<const uint4*>(qs + sw_off(t, 8 * u));
+                            const float2 a = qpair(w.x), b2 = qpair(w.y), c2 = qpair(w.z), d2 = qpair(w.w);
+                            float acc = 0.f;
+                            acc += a.x;
+                            acc += a.y;
+                            acc += b2.x;
+                            acc += b2.y;
+                            acc += c2.x;
+                            acc += c2.y;
+                            acc += d2.x;
+                            acc += d2.y;
+                            su[u] = acc;
+                        }
+                        const float sg = ((su[0] + su[1]) + (su[2] + su[3])) + ((su[4] + su[5]) + (su[6] + su[7]));
+                        const float hi = __bfloat162float(__float2bfloat16_rn(sg));
+                        const float lo = __bfloat162float(__float2bfloat16_rn(sg - hi));
+                        zacc = fmaf(hi, __uint_as_float(yi[0]), zacc);
+                        zacc = fmaf(lo, __uint_as_float(yi[1]), zacc);
+                    }
+                } else if (zrow) {
 #pragma unroll
                     for (int x = 0; x < 32; x += 8) {
                         const uint4 u = *reinterpret_cast<const uint4*>(qs + sw_off(t, j0 + x));
@@ -990,13 +1113,15 @@ struct SegParams {
 // every row of a tile past this offset contributes exactly nothing
 constexpr float kUnderflowLog2 = -152.f;
 
-template <int D, bool REV, bool NORM = false>
+template <int D, bool REV, bool NORM = false, bool PSI = false>
 __global__ void __launch_bounds__(kThreads, 1) seg_state_kernel(const __grid_constant__ SegParams p) {
-    // NORM: the Linear Transformer with phi for 64-channel heads: the X tile
-    // holds phi(k) (phi(q)) in its first 64 channels and zeros after; the
-    // forward's Y tile holds v and the columns [1, 1, 0, ...]; the reverse Y
-    // is the padded dy' (128 channels, loaded whole)
+    // NORM: the Linear Transformer with phi for 64-channel heads, operands built
+    // in shared memory as the tensor-core kernels build them: forward X = k' =
+    // [phi(k), 0] (the forward's basis) or, PSI (the backward's), k'' = [psi(k),
+    // 1, 1, 0]; reverse X = q'' = [phi(q), sigma_hi, sigma_lo, 0]; the forward's
+    // Y holds v and the columns [1, 1, 0, ...]; the reverse Y is the padded dy'
     static_assert(!NORM || D == 128, "the normalised operands run at d = 128");
+    static_assert(!REV || !NORM || PSI, "the reverse summary runs in the backward's basis");
     using S = SegSmem<D>;
     constexpr int BX = NORM ? 64 : D;
     constexpr int BY = (NORM && !REV) ? 64 : D;
@@ -1031,7 +1156,7 @@ __global__ void __launch_bounds__(kThreads, 1) seg_state_kernel(const __grid_con
     if (warp == 0) tc::alloc(tslot, 128);
     if (NORM) {
         for (int st = 0; st < S::NST; ++st) {
-            const_box<kThreads>(smem + st * S::STAGE, tid, false);
+            const_box<kThreads>(smem + st * S::STAGE, tid, PSI && !REV);
             if (!REV) const_box<kThreads>(smem + st * S::STAGE + S::TILE, tid, true);
         }
     }
@@ -1172,7 +1297,9 @@ __global__ void __launch_bounds__(kThreads, 1) seg_state_kernel(const __grid_con
         const TileMeta& mc = metas[st];
         const int64_t t0 = tile_of(i) * T;
         if (NORM) {
-            phi_box<kThreads>(smem + st * S::STAGE, tid, p.L - t0);
+            if (REV) phiq_box<kThreads>(smem + st * S::STAGE, tid, p.L - t0);
+            else if (PSI) psi_box<kThreads>(smem + st * S::STAGE, tid, p.L - t0);
+            else phi_box<kThreads>(smem + st * S::STAGE, tid, p.L - t0);
             __syncthreads();
         }
         // X~ = w (.) X in place
@@ -1376,10 +1503,10 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     static_assert(!HALF_OUT || D == 128, "half-width output at d = 128");
     static_assert(!NORM || HALF_OUT, "the normalised operands come with half-width outputs");
     // NORM: the normalised backward for 64-channel heads: q, k, v are the unpadded
-    // [B, L, H, 64] tensors loaded into the first halves of their slots, phi is
-    // applied to q and k in shared memory, and the second halves hold zeros (q, k)
-    // or the columns [1, 1, 0, ...] (v); dY is the caller's padded dy'.  K's zero
-    // half, where dk rows are staged, is written again once they drain.
+    // [B, L, H, 64] tensors loaded into the first halves of their slots and built
+    // in shared memory into q'' = [phi(q), sigma_hi, sigma_lo, 0], k'' = [psi(k),
+    // 1, 1, 0] and v' = [v, 1, 1, 0]; dY is the caller's padded dy'.  K's
+    // constant half, where dk rows are staged, is written again once they drain.
     constexpr int BKV = NORM ? 64 : D;  // channels loaded into the Q, K and V slots
     // HALF_OUT: only the first 64 columns of dk and dv are written, to [B, L, H, 64]
     // outputs (the normalised path needs no more of dk' and dv')
@@ -1468,7 +1595,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     if (warp == 0) tc::alloc(tslot, S::TMEM_COLS);
     if (NORM) {
         const_box<kRThreads>(smem + S::OFF_Q, tid, false);
-        const_box<kRThreads>(smem + S::OFF_K, tid, false);
+        const_box<kRThreads>(smem + S::OFF_K, tid, true);
         const_box<kRThreads>(smem + S::OFF_V, tid, true);
     }
     tc::fence_before();
@@ -1534,8 +1661,8 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         tc::fence_after();
         if (NORM) {
             const int64_t valid = p.L - t0;
-            phi_box<kRThreads>(smem + S::OFF_Q, tid, valid);
-            phi_box<kRThreads>(smem + S::OFF_K, tid, valid);
+            phiq_box<kRThreads>(smem + S::OFF_Q, tid, valid);
+            psi_box<kRThreads>(smem + S::OFF_K, tid, valid);
             tc::fence_smem_to_async();
             __syncthreads();
         }
@@ -1864,7 +1991,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         have_g = true;
         __syncthreads();
         if (D == 64 && next && tid == 0) issue_tile_b(tile - 1);
-        if (NORM) const_box<kRThreads>(smem + S::OFF_K, tid, false);  // K's zero half held dk rows
+        if (NORM) const_box<kRThreads>(smem + S::OFF_K, tid, true);  // K's constant half held dk rows
 
         // ---- G_{c-1} -> bf16 operand for the next tile (and dS0 at the tape start) ----
         {
@@ -2089,7 +2216,7 @@ memoroid_status_t launch_prep(const Args& a, const Plan& pl, TileMeta* meta, cud
 // summaries and S0) or the reverse states entering them from the right
 // (REV = true, from X = q, Y = dy and dS_last): the summary kernel, then the
 // carry over the segments, in place in `buf`.  Nothing to do for one segment.
-template <int D, bool REV, bool NORM>
+template <int D, bool REV, bool NORM, bool PSI>
 memoroid_status_t launch_seg_carry(const Args& a, const Plan& pl, const TileMeta* meta, float2* info, float* buf,
                                    const CUtensorMap& map_x, const CUtensorMap& map_y, const float* init,
                                    uint32_t* hdr, cudaStream_t stream) {
@@ -2107,8 +2234,8 @@ memoroid_status_t launch_seg_carry(const Args& a, const Plan& pl, const TileMeta
     p.tps = pl.tps;
     p.G = static_cast<int>(pl.G);
     p.wait_ns = debug_knobs().wait_ns;
-    if (set_smem(seg_state_kernel<D, REV, NORM>, SegSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    seg_state_kernel<D, REV, NORM><<<static_cast<unsigned>(a.B * a.H * (pl.G - 1)), kThreads, SegSmem<D>::BYTES,
+    if (set_smem(seg_state_kernel<D, REV, NORM, PSI>, SegSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+    seg_state_kernel<D, REV, NORM, PSI><<<static_cast<unsigned>(a.B * a.H * (pl.G - 1)), kThreads, SegSmem<D>::BYTES,
                                      stream>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     const dim3 grid(static_cast<unsigned>((D * D / 4 + 255) / 256), static_cast<unsigned>(a.B * a.H));
@@ -2131,7 +2258,7 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     if (!tile_map(&p.map_q, a.q, a.B, a.L, a.H, KQ) || !tile_map(&p.map_k, a.k, a.B, a.L, a.H, KQ) ||
         !tile_map(&p.map_v, a.v, a.B, a.L, a.H, KQ) || !tile_map_y(&p.map_y, a.y, a.B, a.L, a.H, KQ))
         return MEMOROID_ERR_CUDA;
-    st = launch_seg_carry<D, false, NORM>(a, pl, meta, info, carry, p.map_k, p.map_v, a.S0, hdr, stream);
+    st = launch_seg_carry<D, false, NORM, false>(a, pl, meta, info, carry, p.map_k, p.map_v, a.S0, hdr, stream);
     if (st != MEMOROID_OK) return st;
     p.den = NORM ? a.den : nullptr;
     p.q = static_cast<const uint16_t*>(a.q);
@@ -2154,6 +2281,7 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     p.map_zq = p.map_q;  // not read by the forward
     p.dlam_f = nullptr;
     p.states = nullptr;
+    p.fold_col = -1;
     if (set_smem(fwd_kernel<D, false, NORM>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
     fwd_kernel<D, false, NORM><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
@@ -2193,9 +2321,9 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
         return MEMOROID_ERR_CUDA;
     // the forward states entering the segments (for pass F) and the reverse
     // states entering them from the right (for pass R)
-    st = launch_seg_carry<D, false, NORM>(a, pl, meta, info, carry_f, r.map_k, r.map_v, a.S0, hdr, stream);
+    st = launch_seg_carry<D, false, NORM, NORM>(a, pl, meta, info, carry_f, r.map_k, r.map_v, a.S0, hdr, stream);
     if (st != MEMOROID_OK) return st;
-    st = launch_seg_carry<D, true, NORM>(a, pl, meta, info, carry_r, r.map_q, r.map_dy, a.dS_last, hdr, stream);
+    st = launch_seg_carry<D, true, NORM, NORM>(a, pl, meta, info, carry_r, r.map_q, r.map_dy, a.dS_last, hdr, stream);
     if (st != MEMOROID_OK) return st;
 
     // pass F: dq = S dy, with (q, k, v) -> (dy, v, k)
@@ -2224,6 +2352,7 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     f.fail_cta = debug_knobs().withhold_ticket;
     f.dlam_f = dlam_f;
     f.states = states;
+    f.fold_col = static_cast<int>(a.fold_col);
     if (set_smem(fwd_kernel<D, true, NORM, HALF_OUT>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
     fwd_kernel<D, true, NORM, HALF_OUT><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;

@@ -14,13 +14,23 @@
 // them: building q', k', v' (and the padded states), the division, and in
 // the backward the upstream gradient of the pair,
 //   dy' = [g, hi, lo, 0],  g = bf16(dy / den),  hi + lo = -(g . y),
-// then the chain rule through phi, dq = dq'[:d] (.) phi'(q).  The gradient
-// with respect to q is a difference of two large terms, X g and x (g . y),
-// that cancel exactly at an episode's first step; so the normalizer term is
-// formed from the bf16 values the tensor cores will use and carried as a
-// pair of bf16 numbers (the second ones column of v'), which keeps the
-// difference exact for the rounded upstream g.  Heads of width d <= 120 (a
-// multiple of 8) are supported.
+// then the chain rule through phi.  The gradient with respect to q is a
+// difference of two large terms, X g and x (g . y), that cancel exactly at an
+// episode's first step; so the normalizer term is formed from the bf16 values
+// the tensor cores will use and carried as a pair of bf16 numbers (the second
+// ones column of v'), which keeps the difference exact for the rounded
+// upstream g.  The backward also works in another basis of the same bilinear
+// form: phi(q) . phi(k) = phi(q) . psi(k) + sigma(q) with psi = phi - 1 = ELU
+// and sigma(q) = sum_i phi(q)_i, i.e.
+//   q'' = [phi(q), sigma_hi, sigma_lo, 0],  k'' = [psi(k), 1, 1, 0]
+// (sigma as a bf16 pair).  bf16 holds psi(k) with a relative error where
+// phi(k) = 1 + psi(k) loses the low bits of psi(k) next to the 1, and dq sums
+// phi(k) against the cancelling terms above, so the rounding of phi(k) was
+// the largest error in dq for nearly constant features (unit-norm keys).  In
+// this basis the state S'' = sum decay k'' v'^T has the incoming (X, x) in its
+// first d rows and sum decay v'^T in rows d and d + 1; dphi(q)_i = dq''_i +
+// dq''_d (folded in the kernel), dq = dphi(q) (.) phi'(q), dk = dk''[:d] (.)
+// phi'(k).  Heads of width d <= 120 (a multiple of 8) are supported.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -89,21 +99,34 @@ size_t total_bytes(int64_t B, int64_t L, int64_t H) {
     return o;
 }
 
-// q' = [phi(q), 0], k' = [phi(k), 0], v' = [v, 1, 1, 0]: one thread per
-// 16-byte chunk (8 columns) of a padded row, for all three operands
+// psi(z) = ELU(z) = phi(z) - 1, rounded to bf16 right after (as phi)
+__device__ __forceinline__ float psi(float z) { return z > 0.f ? z : __expf(z) - 1.f; }
+
+// Forward: q' = [phi(q), 0], k' = [phi(k), 0], v' = [v, 1, 1, 0].  Backward
+// (the basis above): q'' = [phi(q), sigma_hi, sigma_lo, 0], k'' = [psi(k), 1,
+// 1, 0], v'.  One thread per 16-byte chunk (8 columns) of a padded row, the
+// 16 chunks of a row in 16 consecutive lanes; sigma = unit sums of the bf16
+// phi values in column order, then a fixed butterfly over the row's first 8
+// chunks (the association the in-kernel construction of 64-channel heads
+// uses, so both give the same bits), plus the sum of chunks 8.. (d > 64).
 __global__ void __launch_bounds__(256) prep_kernel(const uint4* __restrict__ q, const uint4* __restrict__ k,
-                                                   const uint4* __restrict__ v, int64_t R, int d,
+                                                   const uint4* __restrict__ v, int64_t R, int d, int backward,
                                                    uint4* __restrict__ qp, uint4* __restrict__ kp,
                                                    uint4* __restrict__ vp) {
     constexpr int CH = kW / 8;  // chunks per padded row
     const int in_chunks = d / 8;
     const int64_t n = R * CH;
-    for (int64_t g = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; g < n;
-         g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int lane = threadIdx.x & 31;
+    const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    // warp-uniform loop: every lane takes part in the shuffles
+    for (int64_t base = static_cast<int64_t>(blockIdx.x) * blockDim.x + (threadIdx.x & ~31); base < n; base += stride) {
+        const int64_t g = base + lane;
+        const bool live = g < n;
         const int c = static_cast<int>(g & (CH - 1));
         const int64_t r = g >> 4;
         uint4 oq = make_uint4(0u, 0u, 0u, 0u), ok = oq, ov = oq;
-        if (c < in_chunks) {
+        float su = 0.f;
+        if (live && c < in_chunks) {
             const int64_t src = r * in_chunks + c;
             oq = q[src];
             ok = k[src];
@@ -114,20 +137,38 @@ __global__ void __launch_bounds__(256) prep_kernel(const uint4* __restrict__ q, 
             for (int e = 0; e < 4; ++e) {
                 const float2 fq = __bfloat1622float2(hq[e]), fk = __bfloat1622float2(hk[e]);
                 hq[e] = __floats2bfloat162_rn(phi(fq.x), phi(fq.y));
-                hk[e] = __floats2bfloat162_rn(phi(fk.x), phi(fk.y));
+                hk[e] = backward ? __floats2bfloat162_rn(psi(fk.x), psi(fk.y))
+                                 : __floats2bfloat162_rn(phi(fk.x), phi(fk.y));
+                const float2 pq = __bfloat1622float2(hq[e]);
+                su += pq.x;
+                su += pq.y;
             }
-        } else if (c == in_chunks) {
+        } else if (live && c == in_chunks) {
             reinterpret_cast<__nv_bfloat162*>(&ov)[0] = __floats2bfloat162_rn(1.f, 1.f);  // columns d, d + 1 of v'
+            if (backward) reinterpret_cast<__nv_bfloat162*>(&ok)[0] = __floats2bfloat162_rn(1.f, 1.f);
         }
-        qp[g] = oq;
-        kp[g] = ok;
-        vp[g] = ov;
+        su += __shfl_xor_sync(0xffffffffu, su, 1);
+        su += __shfl_xor_sync(0xffffffffu, su, 2);
+        su += __shfl_xor_sync(0xffffffffu, su, 4);
+        // chunks 8.. (d > 64); for d <= 64 their sum is +0, which leaves the bits as they are
+        const float sg = su + __shfl_xor_sync(0xffffffffu, su, 8);
+        if (backward && live && c == in_chunks) {
+            const float hi = __bfloat162float(__float2bfloat16_rn(sg));
+            reinterpret_cast<__nv_bfloat162*>(&oq)[0] = __floats2bfloat162_rn(hi, sg - hi);
+        }
+        if (live) {
+            qp[g] = oq;
+            kp[g] = ok;
+            vp[g] = ov;
+        }
     }
 }
 
 // padded state from (S [d, d], z [d]) per (tape, head): S' = [[S, z, z2], [0]]
 // with z2 = z (a state) or 0 (the gradient of an outgoing state, read from
-// column d only); null inputs give zeros
+// column d only); null inputs give zeros.  A gradient (dup = 0) is the one of
+// the backward's basis, where the outgoing state is S''[:d] + S''[d]: its row d
+// holds the column sums of rows 0..d-1 (summed in row order).
 __global__ void __launch_bounds__(256) pad_state_kernel(const float* __restrict__ S, const float* __restrict__ z,
                                                         int64_t BH, int d, int dup, float* __restrict__ Sp) {
     const int64_t n = BH * kW * kW;
@@ -138,6 +179,11 @@ __global__ void __launch_bounds__(256) pad_state_kernel(const float* __restrict_
         float val = 0.f;
         if (i < d && j < d && S != nullptr) val = S[(m * d + i) * d + j];
         else if (i < d && (j == d || (dup && j == d + 1)) && z != nullptr) val = z[m * d + i];
+        else if (!dup && i == d && j < d && S != nullptr) {
+            for (int i2 = 0; i2 < d; ++i2) val += S[(m * d + i2) * d + j];
+        } else if (!dup && i == d && j == d && z != nullptr) {
+            for (int i2 = 0; i2 < d; ++i2) val += z[m * d + i2];
+        }
         Sp[g] = val;
     }
 }
@@ -216,7 +262,8 @@ __global__ void __launch_bounds__(256) upstream_kernel(const float* __restrict__
     }
 }
 
-// dq = dq'[:d] (.) phi'(q), dk = dk'[:d] (.) phi'(k), dv = dv'[:d] from
+// dq = dq''[:d] (.) phi'(q) (dq'' with its sum channel already folded in),
+// dk = dk''[:d] (.) phi'(k) (psi' = phi'), dv = dv'[:d] from
 // padded gradients with rows of w4 float4s: one thread per 4 columns (16-byte
 // loads and stores; 32-bit index arithmetic)
 __global__ void __launch_bounds__(256) chain_kernel(const float4* __restrict__ dqp, const float4* __restrict__ dkp,
@@ -277,8 +324,8 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
     if (!fused)
         prep_kernel<<<grid_for(R * 16), 256, 0, s>>>(static_cast<const uint4*>(a.q), static_cast<const uint4*>(a.k),
                                                      static_cast<const uint4*>(a.v), R, static_cast<int>(a.d),
-                                                     reinterpret_cast<uint4*>(b.q), reinterpret_cast<uint4*>(b.k),
-                                                     reinterpret_cast<uint4*>(b.v));
+                                                     a.backward ? 1 : 0, reinterpret_cast<uint4*>(b.q),
+                                                     reinterpret_cast<uint4*>(b.k), reinterpret_cast<uint4*>(b.v));
     // incoming state and (backward) outgoing-state gradient in the padded layout
     const bool s_in = a.S0 != nullptr || a.z0 != nullptr;
     const bool g_in = a.backward && (a.dS_last != nullptr || a.dz_last != nullptr);
@@ -332,6 +379,7 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
     // heads of up to 64 channels need only the first 64 columns of dq', dk', dv'
     const int64_t wout = a.d <= 64 ? 64 : kW;
     l.out_cols = a.d <= 64 ? 64 : 0;
+    l.fold_col = a.d;  // dphi(q)_i = dq''_i + dq''_d
     if (fused) {
         l.q = a.q;
         l.k = a.k;

@@ -98,8 +98,13 @@ def check(t, with_states):
     (1, 700, 2, 120, 80.0, "head", True),
     (3, 900, 1, 8, 40.0, "head", False),
 ])
-def test_parity(B, L, H, d, mean, mode, with_states):
-    check(make(B, L, H, d, tapegen.seed_for(800 + L + d), mean, mode, with_states), with_states)
+@pytest.mark.parametrize("normalize_k", [False, True])
+def test_parity(B, L, H, d, mean, mode, with_states, normalize_k):
+    # keys as the paper feeds them (phi(W_k o), not normalised) and L2-normalised
+    # keys (the other linear-attention workloads), where phi(k) is nearly constant
+    # and dq is a strongly cancelling sum
+    check(make(B, L, H, d, tapegen.seed_for(800 + L + d), mean, mode, with_states, normalize_k=normalize_k),
+          with_states)
 
 
 def test_paper_model_gamma_one():
@@ -147,10 +152,12 @@ def test_episode_isolation_bitwise():
     del m
 
 
-def test_config3_shape_sampled_episodes():
+@pytest.mark.parametrize("normalize_k", [False, True])
+def test_config3_shape_sampled_episodes(normalize_k):
     # the config-3 shape (L = 2^18, 4 heads, d = 64): outputs and gradients on whole-episode
-    # windows (each starts at a begin flag and ends right before one)
-    t = make(1, 1 << 18, 4, 64, tapegen.seed_for(813), 300.0, "step", False)
+    # windows (each starts at a begin flag and ends right before one); keys as
+    # the paper feeds them, and L2-normalised as in the config-3 workload
+    t = make(1, 1 << 18, 4, 64, tapegen.seed_for(813), 300.0, "step", False, normalize_k=normalize_k)
     got = run(t, False)
     heads = np.flatnonzero(t["start"][0])
     f = oracle.bf16_bits_to_f64
