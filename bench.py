@@ -108,7 +108,8 @@ def _tensor_peaks():
 
 
 RET_WORKLOAD = ("per-step discounted return and GAE with resets: B=64 tapes x L=2^20 steps (64 Mi steps), "
-                "fp32 rewards and values, Geometric(200) episodes, gamma=0.99, lambda=0.95")
+                "fp32 rewards and values, Geometric(200) episodes (and, *_single_episode, one episode per tape), "
+                "gamma=0.99, lambda=0.95")
 
 
 def returns_leg(args, m, dev, stream):
@@ -129,9 +130,15 @@ def returns_leg(args, m, dev, stream):
     A = torch.empty_like(r)
     out = {"workload": RET_WORKLOAD}
     peak, peak_kind = _peaks()
+    one = torch.zeros_like(st)  # one episode per tape: the reset-density extreme
+    one[:, 0] = 1
     for name, fn, byts in (
             ("return", lambda: m.memoroid_discounted_return(r, st, 0.99, boot, G, B, L, ws, stream), B * L * 9 + B * 4),
-            ("gae", lambda: m.memoroid_gae(r, v, st, 0.99, 0.95, boot, A, B, L, ws, stream), B * L * 13 + B * 4)):
+            ("gae", lambda: m.memoroid_gae(r, v, st, 0.99, 0.95, boot, A, B, L, ws, stream), B * L * 13 + B * 4),
+            ("return_single_episode", lambda: m.memoroid_discounted_return(r, one, 0.99, boot, G, B, L, ws, stream),
+             B * L * 9 + B * 4),
+            ("gae_single_episode", lambda: m.memoroid_gae(r, v, one, 0.99, 0.95, boot, A, B, L, ws, stream),
+             B * L * 13 + B * 4)):
         for _ in range(3):
             fn()
         torch.cuda.synchronize()
@@ -146,7 +153,8 @@ def returns_leg(args, m, dev, stream):
         out[name] = {"value": B * L / (ms * 1e-3), "unit": "steps/s", "ms": ms,
                      "roofline": {"bound": "hbm", "algorithmic_bytes_per_call": byts, "achieved": gbs, "unit": "GB/s",
                                   "peak": peak, "frac": gbs / peak, "peak_kind": f"{peak_kind} (copy bandwidth)"}}
-    out["gpu_launches"] = 2 * args.ret_steps  # one scan launch per call
+    # one map launch and one scan launch per call (64 tapes: several ranges per tape)
+    out["gpu_launches"] = 4 * 2 * args.ret_steps
     del r, v, G, A, ws
     torch.cuda.empty_cache()
     return out

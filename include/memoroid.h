@@ -392,7 +392,8 @@ memoroid_status_t memoroid_gather_rows(const void *rows, int64_t N, int64_t row_
 /* ======================================================================== */
 
 /* Workspace bytes for memoroid_discounted_return and memoroid_gae (a small
- * reserved block: each call is one kernel launch that keeps no state in it). */
+ * block: a header and one affine map per range of a tape, about 78 KB; a
+ * call launches one or two kernels and keeps nothing in it afterwards). */
 size_t memoroid_returns_workspace_bytes(int64_t B, int64_t L);
 
 /*

@@ -8,13 +8,21 @@
 // with x_t = r_t (return) or delta_t = r_t + gamma V_{t+1} - V_t (GAE, V after
 // an episode's last step 0, after the tape's last step v_boot).
 //
-// A step whose successor starts an episode has m_t = 0, so a stretch of the
-// tape that ends right before a begin flag does not depend on later steps.
-// Each tape is cut into G nominal ranges of seg_len steps, one warp each; a
-// warp's segment runs from the first begin flag in its range (step 0 for the
-// first range) to the first begin flag after its range (or the tape's end),
-// found by the warp itself, so no planning pass, carry or fix-up is needed.
-// The warp walks its segment backwards in chunks of 32 * kElems steps on
+// Each tape is cut into G ranges of seg_len steps, one warp each, which
+// scans its range from the value entering it from the right.  Those values
+// come from a resettable scan over the ranges.  Every range publishes its
+// affine map G_start = X + A G_after, where only the steps up to its first
+// cut matter (a step whose successor starts an episode has m_t = 0, so X
+// stops there and A = 0), and composes, in a fixed order, the maps of the
+// ranges after it up to the first cut (or the tape's end and its bootstrap).
+// Warps take tickets in order and ranges are handed out from each tape's end,
+// so a warp only ever waits for maps of warps that started before it.  With a
+// cut, the steps before it are final from a zero value (they are written
+// while the map is formed) and the rest are scanned once the carry is known:
+// one pass over the tape.  Without one, the range is read twice (for its map,
+// then for its outputs).  So a tape without begin flags runs on as many warps
+// as any other.
+// A warp walks its range backwards in chunks of 32 * kElems steps on
 // absolute chunk boundaries (16-byte loads and stores when the tape length is
 // a multiple of 8 and the buffers are aligned), loading the chunk before
 // while it scans the current one: each lane folds its kElems steps into an
@@ -27,6 +35,7 @@
 #include <cstdint>
 
 #include "internal.cuh"
+#include "ptx.cuh"
 
 namespace memoroid {
 namespace ret {
@@ -38,7 +47,11 @@ constexpr int kChunk = 32 * kElems;
 // upper bound on the warps of one launch
 constexpr int64_t kMaxWarps = 152 * 64;
 
-size_t workspace_bytes(int64_t, int64_t) { return kHeaderBytes; }
+// header (error word, ticket counter), then the ranges' maps (A, X) as two
+// tagged 64-bit words each: at most kMaxWarps of them (with more than one
+// range per tape, B * G <= the warps of one launch)
+constexpr size_t kMapBytes = static_cast<size_t>(kMaxWarps) * 16;
+size_t workspace_bytes(int64_t, int64_t) { return kHeaderBytes + kMapBytes; }
 
 struct Params {
     const float* r;
@@ -46,10 +59,14 @@ struct Params {
     const uint8_t* start;
     const float* boot;  // return: value after the tape's last step; GAE: v_boot
     float* out;
+    unsigned long long* maps;  // [B * G][2]: (A, X) of each range, each value next to the launch's tag
+    uint32_t* hdr;             // [0] error word, [1] ticket counter
     int64_t B, L, G, seg_len;
     int vec;      // 16-byte loads and stores: L % 8 == 0 and aligned base pointers
     float c;      // per-step multiplier: gamma or gamma * lambda
     float gamma;  // GAE: the discount inside delta
+    uint32_t epoch;
+    uint64_t wait_ns;
 };
 
 // (A, X) maps G_in -> X + A G_in; compose(earlier, later) applies `later` first.
@@ -117,35 +134,18 @@ __device__ __forceinline__ void load_blk(Blk& d, const Params& p, const float* r
 
 __device__ __forceinline__ bool flag_of(const Blk& d, int e) { return ((d.s[e >> 2] >> (8 * (e & 3))) & 0xffu) != 0; }
 
-template <bool GAE>
-__global__ void __launch_bounds__(kThreads) scan_kernel(const Params p) {
-    const int lane = threadIdx.x & 31;
-    const int64_t wid = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
-    if (wid >= p.B * p.G) return;
-    const int64_t b = wid / p.G, g = wid % p.G;
-    const int64_t a = g * p.seg_len;
-    if (a >= p.L) return;
-    const int64_t e_nom = min(a + p.seg_len, p.L);
-    const uint8_t* st = p.start + b * p.L;
-    // segment [lo, hi): lo the first begin flag of the range (step 0 for the
-    // first range), hi the first begin flag after the range, else the tape's end
-    const int64_t lo = g == 0 ? 0 : find_flag(st, a, e_nom, lane);
-    if (lo < 0) return;  // no episode starts here: the segment before covers the range
-    int64_t hi = e_nom < p.L ? find_flag(st, e_nom, p.L, lane) : -1;
-    if (hi < 0) hi = p.L;
-
+// Walks steps [lo, hi) of tape b backwards from the value `carry` entering step
+// hi - 1 from after it; next_flag / next_v: the begin flag and V of step hi
+// (true / 0 past the tape).  OUT: writes every step's value.  Returns the
+// value at step lo.  Warp-wide.
+template <bool GAE, bool OUT>
+__device__ float walk(const Params& p, int64_t b, int64_t lo, int64_t hi, float carry, bool next_flag, float next_v,
+                      int lane) {
     const float* r = p.r + b * p.L;
     const float* v = GAE ? p.v + b * p.L : nullptr;
+    const uint8_t* st = p.start + b * p.L;
     float* o = p.out + b * p.L;
     const float boot = p.boot != nullptr ? p.boot[b] : 0.f;
-    // value entering the segment's last step from after it: the bootstrap at the
-    // tape's end (return only; the advantage after the tape is 0)
-    float carry = (!GAE && hi == p.L) ? boot : 0.f;
-    // begin flag and value of the step after the current chunk (lane 31's successor):
-    // for the segment's last chunk that step is hi, a begin flag or past the tape
-    bool next_flag = true;
-    float next_v = 0.f;
-
     const int64_t k_last = (hi - 1) / kChunk, k_first = lo / kChunk;
     Blk cur;
     load_blk<GAE>(cur, p, r, v, st, k_last * kChunk + lane * kElems);
@@ -156,6 +156,8 @@ __global__ void __launch_bounds__(kThreads) scan_kernel(const Params p) {
         // successor of this lane's last step: the next lane's first step
         const bool f_up = __shfl_down_sync(0xffffffffu, flag_of(cur, 0) ? 1 : 0, 1) != 0;
         const float v_up = GAE ? __shfl_down_sync(0xffffffffu, cur.v[0], 1) : 0.f;
+        // the step after this chunk's last one: hi (the caller's) for the range's
+        // last chunk, else the first step of the chunk after it
         const bool succ_flag = lane == 31 ? next_flag : f_up;
         const float succ_v = lane == 31 ? next_v : v_up;
         next_flag = __shfl_sync(0xffffffffu, flag_of(cur, 0) ? 1 : 0, 0) != 0;
@@ -167,6 +169,8 @@ __global__ void __launch_bounds__(kThreads) scan_kernel(const Params p) {
             const int64_t t = t0 + e;
             if (t >= lo && t < hi) {
                 const bool last = t + 1 >= p.L;
+                // the successor: inside the lane's block (loaded from memory even past hi),
+                // or for the block's last step the next lane's first (hi for lane 31)
                 const bool sflag = e + 1 < kElems ? flag_of(cur, e + 1) : succ_flag;
                 const bool cont = !last && !sflag;  // the next step is in the same episode
                 m[e] = (last || cont) ? p.c : 0.f;
@@ -178,7 +182,7 @@ __global__ void __launch_bounds__(kThreads) scan_kernel(const Params p) {
                     x[e] = cur.r[e];
                 }
             } else {
-                m[e] = 1.f;  // identity outside the segment
+                m[e] = 1.f;  // identity outside the range
                 x[e] = 0.f;
             }
         }
@@ -203,28 +207,117 @@ __global__ void __launch_bounds__(kThreads) scan_kernel(const Params p) {
         const float wa = __shfl_sync(0xffffffffu, suf.a, 0);
         const float wx = __shfl_sync(0xffffffffu, suf.x, 0);
         carry = fmaf(wa, carry, wx);
-        float out[kElems];
+        if (OUT) {
+            float out[kElems];
 #pragma unroll
-        for (int e = kElems - 1; e >= 0; --e) {
-            gin = fmaf(m[e], gin, x[e]);
-            out[e] = gin;
-        }
-        if (p.vec && t0 >= lo && t0 + kElems <= hi) {
-            __stcs(reinterpret_cast<float4*>(o + t0), make_float4(out[0], out[1], out[2], out[3]));
-            __stcs(reinterpret_cast<float4*>(o + t0 + 4), make_float4(out[4], out[5], out[6], out[7]));
-        } else {
+            for (int e = kElems - 1; e >= 0; --e) {
+                gin = fmaf(m[e], gin, x[e]);
+                out[e] = gin;
+            }
+            if (p.vec && t0 >= lo && t0 + kElems <= hi) {
+                __stcs(reinterpret_cast<float4*>(o + t0), make_float4(out[0], out[1], out[2], out[3]));
+                __stcs(reinterpret_cast<float4*>(o + t0 + 4), make_float4(out[4], out[5], out[6], out[7]));
+            } else {
 #pragma unroll
-            for (int e = 0; e < kElems; ++e) {
-                const int64_t t = t0 + e;
-                if (t >= lo && t < hi) o[t] = out[e];
+                for (int e = 0; e < kElems; ++e) {
+                    const int64_t t = t0 + e;
+                    if (t >= lo && t < hi) o[t] = out[e];
+                }
             }
         }
         cur = nxt;
     }
+    return carry;
+}
+
+__device__ __forceinline__ unsigned long long tagged(uint32_t epoch, float v) {
+    return (static_cast<unsigned long long>(epoch) << 32) | __float_as_uint(v);
+}
+
+template <bool GAE>
+__global__ void __launch_bounds__(kThreads) scan_kernel(const Params p) {
+    const int lane = threadIdx.x & 31;
+    // ticket -> (tape, range): position 0 is each tape's last range
+    uint32_t tk = 0;
+    if (lane == 0) tk = atomicAdd(p.hdr + 1, 1u);
+    tk = __shfl_sync(0xffffffffu, tk, 0);
+    if (static_cast<int64_t>(tk) >= p.B * p.G) return;
+    const int64_t b = tk % p.B, g = p.G - 1 - static_cast<int64_t>(tk / p.B);
+    const int64_t a = g * p.seg_len;
+    const int64_t e = min(a + p.seg_len, p.L);
+    const uint8_t* st = p.start + b * p.L;
+    const bool nf_e = e < p.L ? st[e] != 0 : true;  // begin flag of the step after the range
+    const float nv_e = (GAE && e < p.L) ? p.v[b * p.L + e] : 0.f;
+    // the first cut: the first begin flag in (a, e] (step f - 1 does not see step f)
+    const int64_t f = p.G > 1 ? find_flag(st, a + 1, min(e + 1, p.L), lane) : -1;
+    const bool cut = f >= 0;
+    if (p.G > 1) {
+        // the range's map; with a cut its steps before f are final (written now)
+        float x, A;
+        if (cut) {
+            x = walk<GAE, true>(p, b, a, f, 0.f, true, 0.f, lane);
+            A = 0.f;
+        } else {
+            x = walk<GAE, false>(p, b, a, e, 0.f, nf_e, nv_e, lane);
+            A = powf(p.c, static_cast<float>(e - a));
+        }
+        if (lane == 0) {
+            unsigned long long* m = p.maps + 2 * (b * p.G + g);
+            __stcg(m, tagged(p.epoch, A));
+            __stcg(m + 1, tagged(p.epoch, x));
+        }
+    }
+    // the value entering step e - 1 from after the range: the maps of the ranges
+    // after it composed in order, batches of 32 from the nearest, up to the first
+    // cut, applied to the value after the tape (the return's bootstrap; the
+    // advantage after the tape is 0)
+    const float after_tape = (!GAE && p.boot != nullptr) ? p.boot[b] : 0.f;
+    Aff tot{1.f, 0.f};
+    for (int64_t j0 = g + 1; j0 < p.G; j0 += 32) {
+        const int64_t j = j0 + lane;
+        Aff mj{1.f, 0.f};
+        bool ok = true;
+        if (j < p.G) {
+            // published by a warp with an earlier ticket
+            const unsigned long long* m = p.maps + 2 * (b * p.G + j);
+            uint64_t t0 = 0;
+            for (uint32_t it = 0;; ++it) {
+                const unsigned long long wa = __ldcg(m), wx = __ldcg(m + 1);
+                if (static_cast<uint32_t>(wa >> 32) == p.epoch && static_cast<uint32_t>(wx >> 32) == p.epoch) {
+                    mj = Aff{__uint_as_float(static_cast<uint32_t>(wa)), __uint_as_float(static_cast<uint32_t>(wx))};
+                    break;
+                }
+                if (it == 0) t0 = ptx::globaltimer();
+                if ((it & 15u) == 15u && ptx::globaltimer() - t0 > p.wait_ns) {
+                    ok = false;
+                    break;
+                }
+            }
+        }
+        if (!__all_sync(0xffffffffu, ok)) {
+            if (lane == 0) atomicCAS(p.hdr, 0u, static_cast<uint32_t>(DEV_LOOKBACK_TIMEOUT));
+            return;
+        }
+        const unsigned cuts = __ballot_sync(0xffffffffu, j < p.G && mj.a == 0.f);
+        // maps after the first cut do not reach this range
+        if (cuts != 0u && lane > __ffs(cuts) - 1) mj = Aff{1.f, 0.f};
+        // their composition in a fixed order (lane 0 earliest)
+        Aff suf = mj;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const float oa = __shfl_down_sync(0xffffffffu, suf.a, off);
+            const float ox = __shfl_down_sync(0xffffffffu, suf.x, off);
+            if (lane + off < 32) suf = compose(suf, Aff{oa, ox});
+        }
+        tot = compose(tot, Aff{__shfl_sync(0xffffffffu, suf.a, 0), __shfl_sync(0xffffffffu, suf.x, 0)});
+        if (cuts != 0u) break;
+    }
+    const float carry = fmaf(tot.a, after_tape, tot.x);
+    walk<GAE, true>(p, b, cut ? f : a, e, carry, nf_e, nv_e, lane);
 }
 
 memoroid_status_t launch(const float* r, const float* v, const uint8_t* start, float c, float gamma,
-                         const float* boot, float* out, int64_t B, int64_t L, void*, cudaStream_t s) {
+                         const float* boot, float* out, int64_t B, int64_t L, void* workspace, cudaStream_t s) {
     // one wave: as many warps as fit on the device at once, split evenly over the tapes
     int dev = 0, sms = 0, per_sm = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -247,9 +340,18 @@ memoroid_status_t launch(const float* r, const float* v, const uint8_t* start, f
     // every tape then starts on a 32-byte boundary of r, v and out and an 8-byte one of start
     const bool vec = (L & 7) == 0 && aligned(r, 16) && (v == nullptr || aligned(v, 16)) && aligned(start, 8) &&
                      aligned(out, 16);
-    const Params p{r, v, start, boot, out, B, L, G, seg_len, vec ? 1 : 0, c, gamma};
+    unsigned char* ws = static_cast<unsigned char*>(workspace);
     const int64_t blocks = (B * G + kWarps - 1) / kWarps;
-    if (blocks > 0x7fffffff) return MEMOROID_ERR_INVALID_ARG;
+    if (blocks > 0x7fffffff || B * G >= 0xffffffffLL) return MEMOROID_ERR_INVALID_ARG;
+    // B * G <= warps <= kMaxWarps whenever G > 1: the maps fit the workspace.  The
+    // maps' tag; their region is zeroed where an old word could carry it.
+    bool clear = false;
+    const uint32_t epoch = tagged_epoch(workspace, kHeaderBytes + kMapBytes, &clear);
+    if (cudaMemsetAsync(ws, 0, clear ? kHeaderBytes + kMapBytes : kHeaderBytes, s) != cudaSuccess)
+        return MEMOROID_ERR_CUDA;
+    const Params p{r, v, start, boot, out, reinterpret_cast<unsigned long long*>(ws + kHeaderBytes),
+                   reinterpret_cast<uint32_t*>(ws), B, L, G, seg_len, vec ? 1 : 0, c, gamma, epoch,
+                   debug_knobs().wait_ns};
     if (v != nullptr)
         scan_kernel<true><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(p);
     else

@@ -3,8 +3,8 @@ return and GAE memoroids of the appendices) against the fp64 oracle, through
 the C ABI.
 
 Bar: max |gpu - ref| / max |ref| <= 1e-4 (fp32 arithmetic).  Cases cover many
-short tapes, long and single-episode tapes (segments that cannot be cut), the
-tape bootstrap, block edges and the degenerate reset patterns.
+short tapes, long and single-episode tapes (the carry between warp ranges),
+the tape bootstrap, block edges and the degenerate reset patterns.
 """
 import numpy as np
 import pytest
@@ -78,7 +78,8 @@ def test_return_and_gae_match_oracle(B, L, mean, gamma, lam, with_boot):
 @pytest.mark.parametrize("mode", ["all", "none", "open"])
 def test_degenerate_resets(mode):
     # every step its own episode / one episode over the tape / a tape that
-    # continues an episode (no begin flag): segments cannot be cut in the last two
+    # continues an episode (no begin flag): in the last two every warp range
+    # takes its value from the ranges after it
     m = _m()
     r, v, start, boot = tape(2, 30000, 0.0, tapegen.seed_for(600), mode)
     G = m.discounted_return(dev(r), dev(start), 0.999, dev(boot))
@@ -86,6 +87,27 @@ def test_degenerate_resets(mode):
     torch.cuda.synchronize()
     assert rel_err(G.cpu().numpy(), oracle.discounted_return(r, start, 0.999, boot)) <= TOL
     assert rel_err(A.cpu().numpy(), oracle.gae(r, v, start, 0.999, 0.97, boot)) <= TOL
+
+
+@pytest.mark.parametrize("gamma,lam,flags", [(0.9999, 0.99, ()), (1.0, 1.0, (123457, 700001))])
+def test_long_tape_few_begin_flags(gamma, lam, flags):
+    # 2^20 steps with a begin flag at t = 0 only, or at two more steps: the tape
+    # is still cut into thousands of warp ranges, each of which gets the value
+    # entering it from the maps of the ranges after it
+    m = _m()
+    B, L = 1, 1 << 20
+    r, v, start, boot = tape(B, L, 0.0, tapegen.seed_for(605 + len(flags)), "none")
+    for f in flags:
+        start[0, f] = 1
+    # the call takes gamma and lambda as fp32: over a horizon of 10^4 steps the
+    # oracle must see the same values (0.9999 and its fp32 rounding differ by
+    # 1.7e-9, which moves the return by about 1e-4 of its size)
+    gamma, lam = float(np.float32(gamma)), float(np.float32(lam))
+    G = m.discounted_return(dev(r), dev(start), gamma, dev(boot))
+    A = m.gae(dev(r), dev(v), dev(start), gamma, lam, dev(boot))
+    torch.cuda.synchronize()
+    assert rel_err(G.cpu().numpy(), oracle.discounted_return(r, start, gamma, boot)) <= TOL
+    assert rel_err(A.cpu().numpy(), oracle.gae(r, v, start, gamma, lam, boot)) <= TOL
 
 
 def test_episode_heads_bitwise_independent_of_other_episodes():
