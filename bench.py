@@ -560,6 +560,11 @@ def linattn_leg(args, m, dev, stream):
     if args.la_tape_steps:
         L = args.la_tape_steps  # a shorter tape of the same workload (profiler captures)
     t = tapegen.linattn_tape_device(B, L, H, d, tapegen.seed_for(LA_CFG), c["mean"], c["gamma"], device=dev)
+    if args.la_single_gamma1:
+        # profiling mode: the timed steps run one episode per tape with gamma = 1
+        t["start"].zero_()
+        t["start"][:, 0] = 1
+        t["gamma"].fill_(1.0)
     per = 1 if t["gamma"].dim() == 3 else 0
     ws = m.linattn_workspace(B, L, H, d, dev)
     y = torch.empty((B, L, H, d), dtype=torch.float32, device=dev)
@@ -1145,6 +1150,8 @@ def main():
     ap.add_argument("--skip-linattn", action="store_true", help="omit the linear-attention leg")
     ap.add_argument("--la-steps", type=int, default=10, help="timed linattn fwd+bwd steps")
     ap.add_argument("--la-warmup", type=int, default=3, help="untimed linattn fwd+bwd steps")
+    ap.add_argument("--la-single-gamma1", action="store_true",
+                    help="profiling: the linattn leg's timed tape has one episode and gamma = 1")
     ap.add_argument("--la-tape-steps", type=int, default=0,
                     help="linattn tape length (profiler captures); 0 = the full L = 2^22 workload")
     ap.add_argument("--only-linattn", action="store_true",

@@ -234,8 +234,10 @@ __device__ __forceinline__ unsigned long long tagged(uint32_t epoch, float v) {
     return (static_cast<unsigned long long>(epoch) << 32) | __float_as_uint(v);
 }
 
+// 4 (return) or 3 (GAE) CTAs per SM: the GAE variant would otherwise take 89
+// registers and fit 2
 template <bool GAE>
-__global__ void __launch_bounds__(kThreads) scan_kernel(const Params p) {
+__global__ void __launch_bounds__(kThreads, GAE ? 3 : 4) scan_kernel(const Params p) {
     const int lane = threadIdx.x & 31;
     // ticket -> (tape, range): position 0 is each tape's last range
     uint32_t tk = 0;
