@@ -622,6 +622,27 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     constexpr int SC = D / 2;  // state and output columns per thread
     const uint32_t lane_base = tm + (static_cast<uint32_t>(32 * quarter) << 16);
 
+    // 16 values of row `row` of the bf16 state operand.  The normalised backward
+    // keeps column fold_col + 1 (a copy of column fold_col: both key channels are 1)
+    // as the bf16 rounding remainder of column fold_col instead, so the two
+    // inter-tile output columns sum to the sum channel's value to about 16 bits.
+    auto sb_store16 = [&](int row, int j0, const float* v) {
+        if (BWD && p.fold_col >= j0 && p.fold_col + 1 < j0 + 16) {
+            const int f = p.fold_col - j0;
+            float vf = 0.f;
+#pragma unroll
+            for (int x = 0; x < 16; ++x)
+                if (x == f) vf = v[x];
+            const float rem = vf - __bfloat162float(__float2bfloat16_rn(vf));
+            float w[16];
+#pragma unroll
+            for (int x = 0; x < 16; ++x) w[x] = x == f + 1 ? rem : v[x];
+            store_bf16x16(smem + S::OFF_SB, core_off(row, j0, D), core_off(row, j0 + 8, D), w);
+        } else {
+            store_bf16x16(smem + S::OFF_SB, core_off(row, j0, D), core_off(row, j0 + 8, D), v);
+        }
+    };
+
     // ---- incoming state (unless the segment's first step begins an episode) ----
     bool have_prev = false, have_state = false;
     if (s_in != nullptr && metas[0].first_start != 0) {
@@ -648,7 +669,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                         v[x + 3] = f.w;
                     }
                 }
-                store_bf16x16(smem + S::OFF_SB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
+                sb_store16(srow, j0, v);
                 if (BWD && metas[0].has_start == 0)
                     store_state_row<D>(state_image<D>(p.states, bh, p.n_tiles, tile0), srow, j0, v);
             } else {
@@ -754,6 +775,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
 #pragma unroll
             for (int cc = 0; cc < 4; ++cc) tc::ld16_nowait(lane_base + S::COL_P + half * 64 + cc * 16, raw + cc * 16);
             tc::ld_wait();
+            float rs = 0.f;  // the normalised backward: fp32 row sum of the masked scores (this half)
 #pragma unroll
             for (int cc = 0; cc < 4; ++cc) {
                 const int r0 = half * 64 + cc * 16;
@@ -763,9 +785,12 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                     const int r = r0 + x;
                     const bool in = r <= t && r >= st;
                     v[x] = in ? __uint_as_float(raw[cc * 16 + x]) * fast_exp2(lt - mc.lam2[r]) : 0.f;
+                    rs += v[x];
                 }
                 store_bf16x16(pm, core_off(t, r0, T), core_off(t, r0 + 8, T), v);
             }
+            // read at the start of the epilogue, before the z terms take the same slots
+            if (BWD && p.fold_col >= 0) reinterpret_cast<float*>(smem + S::OFF_Z)[half * T + t] = rs;
         }
         // ---- K~[r] = exp2(lam2_end - lam2_r) K[r] for rows of the last episode ----
         {
@@ -870,26 +895,33 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 if (NB) f = unpack_bf16x2(pack_bf16x2(f.x > 0.f ? 1.f + f.x : __expf(f.x), f.y > 0.f ? 1.f + f.y : __expf(f.y)));
                 return f;
             };
-            // the normalised backward: the output column of the sum channel, added to every column
+            // the normalised backward: the output column of the sum channel, added to every
+            // column.  Its intra-tile part is the row sum of the masked scores (the key
+            // operand is 1 in that channel), taken in fp32 from the unrounded scores: that
+            // sum cancels strongly, and the bf16 scores of the contraction would add their
+            // rounding to it; the inter-tile part comes from the contraction.
             float ofold = 0.f;
-            if (BWD && p.fold_col >= 0 && out_half) {
-                const int fb = p.fold_col & ~15, fx = p.fold_col & 15;
-                uint32_t fa[16], fi[16];
-                tc::ld16_nowait(lane_base + S::COL_YA + fb, fa);
-                if (have_prev) tc::ld16_nowait(lane_base + S::COL_YI + fb, fi);
-                tc::ld_wait();
-                float va = 0.f, vi = 0.f;
+            if (BWD && p.fold_col >= 0) {
+                const float* rsp = reinterpret_cast<const float*>(smem + S::OFF_Z);
+                const float rsum = rsp[t] + rsp[T + t];
+                float vi = 0.f;  // the inter-tile part: the two columns (value and remainder)
+                if (have_prev) {
+                    const int fb = p.fold_col & ~15, fx = p.fold_col & 15;
+                    float fi[16];
+                    tc::ld16(lane_base + S::COL_YI + fb, fi);
+                    float v0 = 0.f, v1 = 0.f;
 #pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    if (e == fx) {
-                        va = __uint_as_float(fa[e]);
-                        vi = __uint_as_float(fi[e]);
+                    for (int e = 0; e < 16; ++e) {
+                        if (e == fx) v0 = fi[e];
+                        if (e == fx + 1) v1 = fi[e];
                     }
+                    vi = v0 + v1;
                 }
-                ofold = have_prev ? fmaf(w_in, vi, va) : va;
+                ofold = have_prev ? fmaf(w_in, vi, rsum) : rsum;
+                __syncthreads();  // every row sum is read before the z terms overwrite the slots
             }
             // BWD: z_t = w_in_t q_t . (S_{c-1} dy_t), the inter output dotted with q
-            float zacc = 0.f;
+            float zacc = 0.f, zfold = 0.f;
 #pragma unroll
             for (int cc = 0; cc < SC / 32; ++cc) {
                 const int j0 = half * SC + cc * 32;
@@ -946,14 +978,26 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                         const float sg = ((su[0] + su[1]) + (su[2] + su[3])) + ((su[4] + su[5]) + (su[6] + su[7]));
                         const float hi = __bfloat162float(__float2bfloat16_rn(sg));
                         const float lo = __bfloat162float(__float2bfloat16_rn(sg - hi));
-                        zacc = fmaf(hi, __uint_as_float(yi[0]), zacc);
-                        zacc = fmaf(lo, __uint_as_float(yi[1]), zacc);
+                        // the sum channel pair: (sigma_hi + sigma_lo) times (value + remainder)
+                        zacc = fmaf(hi + lo, __uint_as_float(yi[0]) + __uint_as_float(yi[1]), zacc);
                     }
                 } else if (zrow) {
 #pragma unroll
                     for (int x = 0; x < 32; x += 8) {
                         const uint4 u = *reinterpret_cast<const uint4*>(qs + sw_off(t, j0 + x));
-                        const float2 q0 = qpair(u.x), q1 = qpair(u.y), q2 = qpair(u.z), q3 = qpair(u.w);
+                        float2 q0 = qpair(u.x), q1 = qpair(u.y), q2 = qpair(u.z), q3 = qpair(u.w);
+                        if (BWD && p.fold_col >= j0 + x && p.fold_col < j0 + x + 8) {
+                            // the sum channel pair (value, remainder columns) is taken below
+                            const int f = p.fold_col - (j0 + x);  // 0 or 2, 4, 6 (even)
+                            const float qs0 = f == 0 ? q0.x : (f == 2 ? q1.x : (f == 4 ? q2.x : q3.x));
+                            const float qs1 = f == 0 ? q0.y : (f == 2 ? q1.y : (f == 4 ? q2.y : q3.y));
+                            const float ys0 = __uint_as_float(yi[x + f]), ys1 = __uint_as_float(yi[x + f + 1]);
+                            zfold = fmaf(qs0 + qs1, ys0 + ys1, 0.f);
+                            if (f == 0) q0 = make_float2(0.f, 0.f);
+                            if (f == 2) q1 = make_float2(0.f, 0.f);
+                            if (f == 4) q2 = make_float2(0.f, 0.f);
+                            if (f == 6) q3 = make_float2(0.f, 0.f);
+                        }
                         zacc = fmaf(q0.x, __uint_as_float(yi[x]), zacc);
                         zacc = fmaf(q0.y, __uint_as_float(yi[x + 1]), zacc);
                         zacc = fmaf(q1.x, __uint_as_float(yi[x + 2]), zacc);
@@ -965,6 +1009,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                     }
                 }
             }
+            zacc += zfold;
             if (BWD) reinterpret_cast<float*>(smem + S::OFF_Z)[half * T + t] = w_in * zacc;
         }
         if (BWD) __syncthreads();  // every z term has read the q tile, where the state is staged next
@@ -984,8 +1029,8 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
 #pragma unroll
                 for (int x = 0; x < 32; ++x) v[x] = __uint_as_float(raw[x]);
                 if (srow >= 0) {
-                    store_bf16x16(smem + S::OFF_SB, core_off(srow, j0, D), core_off(srow, j0 + 8, D), v);
-                    store_bf16x16(smem + S::OFF_SB, core_off(srow, j0 + 16, D), core_off(srow, j0 + 24, D), v + 16);
+                    sb_store16(srow, j0, v);
+                    sb_store16(srow, j0 + 16, v + 16);
                     if (BWD && mn.has_start == 0) {
                         // staged in this stage's Q slot (the z term has read q) and
                         // bulk-stored with the output rows
