@@ -1342,9 +1342,15 @@ __global__ void __launch_bounds__(kThreads, 1) seg_state_kernel(const __grid_con
         const TileMeta& mc = metas[st];
         const int64_t t0 = tile_of(i) * T;
         if (NORM) {
-            if (REV) phiq_box<kThreads>(smem + st * S::STAGE, tid, p.L - t0);
-            else if (PSI) psi_box<kThreads>(smem + st * S::STAGE, tid, p.L - t0);
-            else phi_box<kThreads>(smem + st * S::STAGE, tid, p.L - t0);
+            if (REV) {
+                phiq_box<kThreads>(smem + st * S::STAGE, tid, p.L - t0);
+            } else if (PSI) {
+                psi_box<kThreads>(smem + st * S::STAGE, tid, p.L - t0);
+                // the constant half [1, 1, 0, ...]: this stage's last tile scaled it in place
+                const_box<kThreads>(smem + st * S::STAGE, tid, true);
+            } else {
+                phi_box<kThreads>(smem + st * S::STAGE, tid, p.L - t0);
+            }
             __syncthreads();
         }
         // X~ = w (.) X in place

@@ -114,13 +114,16 @@ def test_paper_model_gamma_one():
     check(t, False)
 
 
-@pytest.mark.parametrize("d,with_states", [(64, True), (32, False)])
-def test_one_long_episode(d, with_states):
-    # one episode over 2^15 steps with gamma = 1 (the paper's model): the
-    # normalised pair crosses every segment boundary through the carry between
-    # segments (d = 64: operands built inside the kernels; d = 32: padded)
+@pytest.mark.parametrize("d,with_states,gamma_lo", [(64, True, 1.0), (32, False, 1.0), (64, False, 0.99),
+                                                     (32, True, 0.99)])
+def test_one_long_episode(d, with_states, gamma_lo):
+    # one episode over 2^15 steps with gamma = 1 (the paper's model) or a per-step
+    # gamma in [0.99, 1): the normalised pair crosses every segment boundary
+    # through the carry between segments, whose summaries span several tiles
+    # (d = 64: operands built inside the kernels; d = 32: padded)
     t = make(1, 1 << 15, 2, d, tapegen.seed_for(817 + d), 1.0, "step", with_states, start_mode="none")
-    t["gamma"][:] = 1.0
+    rng = np.random.default_rng(tapegen.seed_for(819 + d))
+    t["gamma"][:] = 1.0 if gamma_lo == 1.0 else rng.uniform(gamma_lo, 1.0, t["gamma"].shape).astype(np.float32)
     if with_states:
         t["start"][:, 0] = 0
     check(t, with_states)
