@@ -889,6 +889,14 @@ def run_ours(args):
         # profiling mode: the Fast and Forgetful Memory leg alone
         print(json.dumps({"ffm": ffm_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
         return
+    if args.only_cfg3:
+        # profiling mode: the L=2^18, 4-head, d=64 linattn leg alone
+        print(json.dumps({"linattn_cfg3": linattn_cfg3_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
+        return
+    if args.only_cfg4:
+        # profiling mode: the 64-tape, D=128 diag leg alone
+        print(json.dumps({"diag_cfg4": diag_cfg4_leg(args, m, dev, torch.cuda.current_stream())}), flush=True)
+        return
 
     t = tapegen.diag_config(CFG)
     if args.tape_steps:
@@ -1164,6 +1172,8 @@ def main():
     ap.add_argument("--skip-tbb", action="store_true", help="omit the tape-based batching leg")
     ap.add_argument("--skip-lnorm", action="store_true", help="omit the normalised Linear Transformer leg")
     ap.add_argument("--skip-per-step", action="store_true", help="omit the per-step lambda diag leg")
+    ap.add_argument("--only-cfg3", action="store_true", help="profiling: the config-3 linattn leg alone")
+    ap.add_argument("--only-cfg4", action="store_true", help="profiling: the config-4 diag leg alone")
     ap.add_argument("--skip-cfg3", action="store_true", help="omit the L=2^18, 4-head, d=64 linattn leg")
     ap.add_argument("--cfg3-steps", type=int, default=20, help="timed config-3 linattn fwd+bwd steps")
     ap.add_argument("--skip-cfg4", action="store_true", help="omit the 64-tape, D=128 diag leg")
