@@ -297,6 +297,29 @@ def test_lookback_timeout_reported():
     assert rel_err(h.cpu().numpy(), ref) <= TOL
 
 
+@pytest.mark.parametrize("fill", [0xFF, 0x00, 0xA5])
+def test_garbage_workspace(fill):
+    # a fresh workspace full of leftover bytes: the look-back summaries' region
+    # is zeroed on the workspace's first use, so no old word is taken for a
+    # summary of this launch; forward and backward against the oracle, twice
+    m = _m()
+    B, L, D = 2, 6000, 128
+    t = tapegen.diag_tape(B, L, D, seed=tapegen.seed_for(77), mean=150.0)
+    lam, u, start, gh = dev(t["lam"]), dev(t["u"]), dev(t["start"]), dev(t["grad_h"])
+    ws = torch.full((m.memoroid_scan_diag_workspace_bytes(B, L, D),), fill, dtype=torch.uint8, device="cuda")
+    ref_h, _ = oracle.diag_fwd(t["lam"], t["u"], t["start"])
+    ref_gu, ref_gl, _ = oracle.diag_bwd(t["lam"], t["start"], ref_h, t["grad_h"])
+    for _ in range(2):
+        h = torch.empty_like(u)
+        m.memoroid_scan_diag_fwd(lam, 0, u, start, None, h, None, B, L, D, ws)
+        gu, gl = torch.empty_like(u), torch.empty_like(lam)
+        m.memoroid_scan_diag_bwd(lam, 0, start, None, h, gh, None, gu, gl, None, B, L, D, ws)
+        assert m.memoroid_get_device_error(ws) == m.MEMOROID_OK
+        assert rel_err(h.cpu().numpy(), ref_h) <= TOL
+        assert rel_err(gu.cpu().numpy(), ref_gu) <= TOL
+        assert rel_err(gl.cpu().numpy(), ref_gl) <= TOL
+
+
 def test_guard_bands_untouched():
     m = _m()
     B, L, D = 2, 1000, 70
