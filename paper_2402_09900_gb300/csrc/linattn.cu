@@ -518,8 +518,11 @@ __device__ __forceinline__ void store_bf16x16(unsigned char* base, uint32_t off0
 // (the term of dL/dlog(gamma_s) that pairs the incoming state with the tile's
 // outputs), and stores S'_{c-1} as bf16 for every tile without a begin flag,
 // for pass R.
-template <int D, bool BWD, bool NORM = false, bool HALF_OUT = false>
+template <int D, bool BWD, bool NORM = false, bool HALF_OUT = false, bool FOLD = false>
 __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant__ FwdParams p) {
+    // FOLD (pass F of the normalised backward): column p.fold_col of the output is
+    // added to every output column (see the epilogue); compiled out elsewhere
+    static_assert(!FOLD || BWD, "the fold is pass F's");
     static_assert(!NORM || (D == 128 && (!BWD || HALF_OUT)), "the normalised operands run the d = 128 kernels");
     // HALF_OUT (pass F at d = 128): only the first 64 output columns are written,
     // to a [B, L, H, 64] output (the normalised path needs no more of dq')
@@ -627,7 +630,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     // as the bf16 rounding remainder of column fold_col instead, so the two
     // inter-tile output columns sum to the sum channel's value to about 16 bits.
     auto sb_store16 = [&](int row, int j0, const float* v) {
-        if (BWD && p.fold_col >= j0 && p.fold_col + 1 < j0 + 16) {
+        if (FOLD && p.fold_col >= j0 && p.fold_col + 1 < j0 + 16) {
             const int f = p.fold_col - j0;
             float vf = 0.f;
 #pragma unroll
@@ -785,12 +788,12 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                     const int r = r0 + x;
                     const bool in = r <= t && r >= st;
                     v[x] = in ? __uint_as_float(raw[cc * 16 + x]) * fast_exp2(lt - mc.lam2[r]) : 0.f;
-                    rs += v[x];
+                    if (FOLD) rs += v[x];
                 }
                 store_bf16x16(pm, core_off(t, r0, T), core_off(t, r0 + 8, T), v);
             }
             // read at the start of the epilogue, before the z terms take the same slots
-            if (BWD && p.fold_col >= 0) reinterpret_cast<float*>(smem + S::OFF_Z)[half * T + t] = rs;
+            if (FOLD) reinterpret_cast<float*>(smem + S::OFF_Z)[half * T + t] = rs;
         }
         // ---- K~[r] = exp2(lam2_end - lam2_r) K[r] for rows of the last episode ----
         {
@@ -901,7 +904,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             // sum cancels strongly, and the bf16 scores of the contraction would add their
             // rounding to it; the inter-tile part comes from the contraction.
             float ofold = 0.f;
-            if (BWD && p.fold_col >= 0) {
+            if (FOLD) {
                 const float* rsp = reinterpret_cast<const float*>(smem + S::OFF_Z);
                 const float rsum = rsp[t] + rsp[T + t];
                 float vi = 0.f;  // the inter-tile part: the two columns (value and remainder)
@@ -946,7 +949,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                             o.z = fmaf(w_in, __uint_as_float(yi[x + 2]), o.z);
                             o.w = fmaf(w_in, __uint_as_float(yi[x + 3]), o.w);
                         }
-                        if (BWD && p.fold_col >= 0) {
+                        if (FOLD) {
                             o.x += ofold;
                             o.y += ofold;
                             o.z += ofold;
@@ -986,7 +989,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                     for (int x = 0; x < 32; x += 8) {
                         const uint4 u = *reinterpret_cast<const uint4*>(qs + sw_off(t, j0 + x));
                         float2 q0 = qpair(u.x), q1 = qpair(u.y), q2 = qpair(u.z), q3 = qpair(u.w);
-                        if (BWD && p.fold_col >= j0 + x && p.fold_col < j0 + x + 8) {
+                        if (FOLD && p.fold_col >= j0 + x && p.fold_col < j0 + x + 8) {
                             // the sum channel pair (value, remainder columns) is taken below
                             const int f = p.fold_col - (j0 + x);  // 0 or 2, 4, 6 (even)
                             const float qs0 = f == 0 ? q0.x : (f == 2 ? q1.x : (f == 4 ? q2.x : q3.x));
@@ -1009,7 +1012,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                     }
                 }
             }
-            zacc += zfold;
+            if (FOLD) zacc += zfold;
             if (BWD) reinterpret_cast<float*>(smem + S::OFF_Z)[half * T + t] = w_in * zacc;
         }
         if (BWD) __syncthreads();  // every z term has read the q tile, where the state is staged next
@@ -2404,8 +2407,20 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     f.dlam_f = dlam_f;
     f.states = states;
     f.fold_col = static_cast<int>(a.fold_col);
-    if (set_smem(fwd_kernel<D, true, NORM, HALF_OUT>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    fwd_kernel<D, true, NORM, HALF_OUT><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
+    // the normalised backward folds its sum channel (fold_col); the plain one never does
+    if constexpr (NORM) {
+        if (a.fold_col < 0) return MEMOROID_ERR_UNSUPPORTED;
+        if (set_smem(fwd_kernel<D, true, NORM, HALF_OUT, true>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+        fwd_kernel<D, true, NORM, HALF_OUT, true>
+            <<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
+    } else if (a.fold_col >= 0) {
+        if (set_smem(fwd_kernel<D, true, false, HALF_OUT, true>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+        fwd_kernel<D, true, false, HALF_OUT, true>
+            <<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
+    } else {
+        if (set_smem(fwd_kernel<D, true, false, HALF_OUT>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
+        fwd_kernel<D, true, false, HALF_OUT><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
+    }
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
 
     // pass R: dk, dv, dgamma, dS0
