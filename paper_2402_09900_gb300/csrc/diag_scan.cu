@@ -236,7 +236,7 @@ struct Cfg {
     static constexpr size_t OFF_CARRY = OFF_WX + W_ * 32 * 16;
     static constexpr size_t OFF_ACC = OFF_CARRY + 32 * 16;
     static constexpr size_t OFF_WR = OFF_ACC + ((REV_ && !PS_) ? W_ * 32 * 16 : 0);
-    static constexpr size_t OFF_MISC = (OFF_WR + W_ * 4 + 15) / 16 * 16;  // bar, ticket, abort
+    static constexpr size_t OFF_MISC = (OFF_WR + W_ * 4 + 15) / 16 * 16;  // bar, ticket, abort, h bar
     static constexpr size_t SMEM = OFF_MISC + 32;
     static_assert(R_ < 32, "R + 1 begin flags are read by one warp");
 };
@@ -459,6 +459,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
     float4* s_acc = reinterpret_cast<float4*>(smem + C::OFF_ACC);        // [W][32] grad_lambda parts
     uint32_t* s_wr = reinterpret_cast<uint32_t*>(smem + C::OFF_WR);      // [W] warp holds a reset
     uint64_t* bar = reinterpret_cast<uint64_t*>(smem + C::OFF_MISC);
+    uint64_t* bar_h = reinterpret_cast<uint64_t*>(smem + C::OFF_MISC + 24);  // h_{t-1} rows (backward)
     long long* s_tk = reinterpret_cast<long long*>(smem + C::OFF_MISC + 8);
     volatile int* s_abort = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 16);
 
@@ -467,6 +468,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
         *s_tk = static_cast<long long>(atomicAdd(p.hdr + 1, 1u));
         *s_abort = 0;
         ptx::mbar_init(bar, 1);
+        if (C::REV) ptx::mbar_init(bar_h, 1);
         ptx::fence_mbar_init();
     }
     __syncthreads();
@@ -482,7 +484,9 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
     if (warp == LB_PUBLISH) {
         // ----------------------------------------- stage the tile, publish its summary
         // one box of T rows per staged array; rows past the tape (and the row
-        // before step 0) read as zeros, and every box counts in full
+        // before step 0) read as zeros, and every box counts in full.  The
+        // backward's h_{t-1} rows complete on a barrier of their own: only the
+        // rescan reads them, so the first pass starts as soon as grad_h is in
         if (lane == 0) {
             const int x = static_cast<int>(4 * t.c2), y = static_cast<int>(t.t0), z = static_cast<int>(t.b);
             constexpr uint32_t BOX = C::T * 512u;  // a full 512-byte row per step
@@ -492,16 +496,20 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
             } else if (C::FFM) {
                 // Re halves at x = 2 c2, Im halves at x = D + 2 c2 (floats), T x 256 bytes each
                 const int re = static_cast<int>(2 * t.c2), im = static_cast<int>(2 * p.D2 + 2 * t.c2);
-                ptx::mbar_arrive_expect_tx(bar, 2 * BOX);
+                ptx::mbar_arrive_expect_tx(bar, BOX);
                 ptx::tma_load_3d(ptx::smem_addr(s_in), &p.map_in, re, y, z, bar);
                 ptx::tma_load_3d(ptx::smem_addr(s_in + C::T * 16), &p.map_in, im, y, z, bar);
-                ptx::tma_load_3d(ptx::smem_addr(s_h), &p.map_h, re, y - 1, z, bar);
-                ptx::tma_load_3d(ptx::smem_addr(s_h + C::T * 16), &p.map_h, im, y - 1, z, bar);
+                ptx::mbar_arrive_expect_tx(bar_h, BOX);
+                ptx::tma_load_3d(ptx::smem_addr(s_h), &p.map_h, re, y - 1, z, bar_h);
+                ptx::tma_load_3d(ptx::smem_addr(s_h + C::T * 16), &p.map_h, im, y - 1, z, bar_h);
             } else {
-                ptx::mbar_arrive_expect_tx(bar, BOX * C::NB);
+                ptx::mbar_arrive_expect_tx(bar, BOX * (C::NB - (C::REV ? 1 : 0)));
                 ptx::tma_load_3d(ptx::smem_addr(s_in), &p.map_in, x, y, z, bar);
-                if (C::REV) ptx::tma_load_3d(ptx::smem_addr(s_h), &p.map_h, x, y - 1, z, bar);
                 if (C::PS) ptx::tma_load_3d(ptx::smem_addr(s_l), &p.map_l, x, y + (C::REV ? 1 : 0), z, bar);
+                if (C::REV) {
+                    ptx::mbar_arrive_expect_tx(bar_h, BOX);
+                    ptx::tma_load_3d(ptx::smem_addr(s_h), &p.map_h, x, y - 1, z, bar_h);
+                }
             }
         }
         __syncwarp();
@@ -738,6 +746,16 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
     } else {
         const float4* sh = s_h + warp * R * 32 + lane;
         float4 acc = zero2();
+        // the h_{t-1} rows have their own barrier: the first pass did not wait for them
+        {
+            const uint64_t w0 = ptx::globaltimer();
+            while (!ptx::mbar_try_wait(bar_h, 0)) {
+                if (ptx::globaltimer() - w0 > p.wait_ns) {
+                    record_error(p, DEV_TMA_TIMEOUT, tk);
+                    break;
+                }
+            }
+        }
         // FFM: every lane runs the loop (grad_x~ is reduced across lanes); the
         // lanes past the slab's width touch no global memory
         if (C::FFM || lane_ok) {
