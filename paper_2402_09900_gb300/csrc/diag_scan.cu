@@ -760,6 +760,13 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
         // lanes past the slab's width touch no global memory
         if (C::FFM || lane_ok) {
             float4* dst = p.out + (t.b * p.L + ts) * p.D2 + t.c2 + lane;
+            // FFM: this lane's grad_x~ element in row ts (rows of m floats): its two
+            // channels' row i for c = 1, else the row i of its group of c / 2 lanes
+            const int lc = p.ffm_lc;
+            const int grp = lc > 0 ? 1 << (lc - 1) : 1;  // lanes per row i (c > 1)
+            const bool gx_writer = lane_ok && (lane & (grp - 1)) == 0;
+            float* gxw = C::FFM ? p.ffm_gx + (t.b * p.L + ts) * p.ffm_m + ((2 * (t.c2 + lane)) >> lc) : nullptr;
+            const int64_t gxrow = p.ffm_m;
 #pragma unroll C::UNROLL
             for (int kk = 0; kk < R; ++kk) {
                 const int k = R - 1 - kk;
@@ -768,9 +775,18 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
                 const float4 gg = C::FFM ? ffm_planar_pair<C::T>(s_in, warp * R + k, lane) : sin[k * 32];
                 const float4 m = (tt == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
                 c = ((rmask >> k) & 1u) ? gg : cfma2(m, c, gg);
-                if (C::FFM)
-                    ffm_grad_x(p, t.b * p.L + tt, t.c2 + lane, c, 0xffffffffu, lane_ok, false, true);
-                else
+                if (C::FFM) {
+                    float* g = gxw + k * gxrow;
+                    if (lc == 0) {
+                        if (lane_ok) __stcs(reinterpret_cast<float2*>(g), make_float2(c.x, c.z));
+                    } else {
+                        float v = c.x + c.z;
+                        if (grp > 1) v += __shfl_xor_sync(0xffffffffu, v, 1);
+                        if (grp > 2) v += __shfl_xor_sync(0xffffffffu, v, 2);
+                        if (grp > 4) v += __shfl_xor_sync(0xffffffffu, v, 4);
+                        if (gx_writer) __stcs(g, v);
+                    }
+                } else
                     __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
                 float4 gl = zero2();
                 if (!((bmask >> k) & 1u) && lane_ok) {
