@@ -141,8 +141,9 @@ struct Args {
     // 64-channel heads at D = 128, with q, k, v the unpadded [B, L, H, 64]
     // tensors.  Forward: y [B, L, H, 64] and den [B, L, H] (or null); S0 and
     // S_last in the padded [B, H, 128, 128] layout.  Backward: the padded bf16
-    // upstream gradient in grad_y16 and out_cols = 64 (the padded gradients'
-    // first 64 columns; the chain rule through phi is the caller's).
+    // upstream gradient in grad_y16 and out_cols = 64; dq, dk, dv [B, L, H, 64]
+    // are the gradients with respect to the raw q, k, v (the epilogues apply
+    // phi'(q) and phi'(k) to the padded gradients' first 64 columns).
     int norm = 0;
     float* den = nullptr;
     // backward only: grad_y already in bf16 [B, L, H, D] (exact values), used as

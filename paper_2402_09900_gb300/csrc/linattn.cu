@@ -286,6 +286,14 @@ __device__ __forceinline__ void scale_rows_sw(unsigned char* tile, int tid, WFn 
     }
 }
 
+// phi'(z) of the raw input (1 above 0, else e^z): the chain rule of the
+// normalised backward, applied to dq and dk in the epilogues
+__device__ __forceinline__ float phi_prime(float z) { return z > 0.f ? 1.f : expf(z); }
+__device__ __forceinline__ float4 times_phi_prime(float4 o, uint2 raw) {
+    const float2 a = unpack_bf16x2(raw.x), b = unpack_bf16x2(raw.y);
+    return make_float4(o.x * phi_prime(a.x), o.y * phi_prime(a.y), o.z * phi_prime(b.x), o.w * phi_prime(b.y));
+}
+
 // phi(z) = 1 + ELU(z) in place on the first 64-channel box of a [T x 128]
 // operand slot (bf16, round to nearest, the SFU exponential); rows at or past
 // `valid` become 0, as rows past the tape end of padded operands are.  NT
@@ -760,7 +768,9 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         // pass F: the Q slot (dy) is free once the first contractions are done; the
         // q tile of the z term goes there
         const bool zload = BWD && have_prev;
-        if (zload) {
+        // the normalised backward also reads q in the epilogue: dq = dphi(q) (.) phi'(q)
+        const bool qload = zload || NB;
+        if (qload) {
             if (tid == 0) {
                 mbar_arrive_expect_tx(qbar, T * BKV * 2);
                 tma_tile<BKV>(stage_q(s), &p.map_zq, h, (tile0 + c) * T, b, qbar);
@@ -838,7 +848,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             break;
         }
         tc::fence_after();
-        if (zload) {
+        if (qload) {
             ok = wait_mbar(qbar, q_par, p.wait_ns);
             if (__syncthreads_or(!ok)) {
                 failed = true;
@@ -956,6 +966,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                             o.w += ofold;
                         }
                         const int j = j0 + x;  // 4 channels = one 16-byte unit
+                        if (NB) o = times_phi_prime(o, *reinterpret_cast<const uint2*>(qs + sw_off(t, j)));
                         *reinterpret_cast<float4*>(yst + (j >> 5) * (T * 128) + ((((j & 31) >> 2) ^ (t & 7)) << 4)) = o;
                     }
                 }
@@ -1427,18 +1438,36 @@ __global__ void __launch_bounds__(256) seg_carry_kernel(float* __restrict__ buf,
     float* base = buf + bh * G * DD + e;
     const float2* inf = info + bh * G;
     float4 c = init != nullptr ? *reinterpret_cast<const float4*>(init + bh * DD + e) : make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 4
-    for (int k = 0; k < G - 1; ++k) {
-        const int g = REV ? G - 1 - k : k;
-        const float2 f = inf[g];
-        const float4 x = *reinterpret_cast<const float4*>(base + static_cast<int64_t>(g) * DD);
-        if (f.x != 0.f) {
-            c = x;
-        } else {
-            const float a = exp2f(f.y);
-            c = make_float4(fmaf(a, c.x, x.x), fmaf(a, c.y, x.y), fmaf(a, c.z, x.z), fmaf(a, c.w, x.w));
+    // the segments' loads go out a batch at a time (the in-place stores would
+    // otherwise hold every load back until the previous segment is folded)
+    constexpr int NB = 8;
+    for (int k0 = 0; k0 < G - 1; k0 += NB) {
+        float4 x[NB];
+        float2 f[NB];
+#pragma unroll
+        for (int j = 0; j < NB; ++j) {
+            const int k = k0 + j;
+            if (k < G - 1) {
+                const int g = REV ? G - 1 - k : k;
+                f[j] = inf[g];
+                x[j] = *reinterpret_cast<const float4*>(base + static_cast<int64_t>(g) * DD);
+            }
         }
-        *reinterpret_cast<float4*>(base + static_cast<int64_t>(g) * DD) = c;
+#pragma unroll
+        for (int j = 0; j < NB; ++j) {
+            const int k = k0 + j;
+            if (k < G - 1) {
+                const int g = REV ? G - 1 - k : k;
+                if (f[j].x != 0.f) {
+                    c = x[j];
+                } else {
+                    const float a = exp2f(f[j].y);
+                    c = make_float4(fmaf(a, c.x, x[j].x), fmaf(a, c.y, x[j].y), fmaf(a, c.z, x[j].z),
+                                    fmaf(a, c.w, x[j].w));
+                }
+                *reinterpret_cast<float4*>(base + static_cast<int64_t>(g) * DD) = c;
+            }
+        }
     }
 }
 
@@ -1586,6 +1615,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     uint64_t* full = bar1 + 3;
     uint32_t* tslot = reinterpret_cast<uint32_t*>(bar1 + 4);
     uint64_t* bar4 = bar1 + 5;  // V G^T of B1, committed apart from P and dP
+    uint64_t* kbar = bar1 + 6;  // NORM: the raw k rows for phi'(k), in V's constant half
     const TileMeta& mc = *reinterpret_cast<const TileMeta*>(smem + S::OFF_META);
     const uint32_t sbase = smem_addr(smem);
     const uint32_t sQ = sbase + S::OFF_Q, sK = sbase + S::OFF_K, sV = sbase + S::OFF_V, sDY = sbase + S::OFF_DY;
@@ -1638,6 +1668,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         mbar_init(bar3, 1);
         mbar_init(full, 1);
         mbar_init(bar4, 1);
+        if (NORM) mbar_init(kbar, 1);
         fence_mbar_init();
         prefetch_tensormap(&p.map_q);
         prefetch_tensormap(&p.map_k);
@@ -1699,6 +1730,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     uint64_t* drain = nullptr;  // a batch issued but not seen complete
     uint32_t drain_par = 0;
     uint32_t ph4 = 0;           // phase of bar4 (committed only on tiles with a reverse state)
+    bool k_pending = false;     // NORM: a raw k load not seen complete
     int it = 0;
 #pragma unroll 1
     for (int64_t tile = tile_hi - 1; tile >= tile_lo; --tile, ++it) {
@@ -1861,6 +1893,13 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
             break;
         }
         if (have_g) ph4 ^= 1;
+        if (NORM && tid == 0) {
+            // the first batch (V G^T included) is done with V: its constant half
+            // takes the raw k rows of this tile for phi'(k) in the dk epilogue
+            mbar_arrive_expect_tx(kbar, T * 64 * 2);
+            tma_tile<64>(sV + T * 128, &p.map_k, h, t0, b, kbar);
+        }
+        if (NORM) k_pending = true;
         {
             // K~ = w_out (.) K in place (K is not read unscaled after this)
             const float lend = mc.lam2[T - 1];
@@ -1961,9 +2000,20 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
                 bulk_commit();
             }
         };
+        if (NORM) {
+            ok = wait_mbar(kbar, it & 1, p.wait_ns);
+            if (__syncthreads_or(!ok)) {
+                failed = true;
+                drain = bar3;
+                drain_par = it & 1;
+                break;
+            }
+            k_pending = false;
+        }
         {
             const int r = 32 * quarter + lane;
             const float w_out = r >= mc.last_start ? fast_exp2(mc.lam2[T - 1] - mc.lam2[r]) : 0.f;
+            const unsigned char* kraw = smem + S::OFF_V + T * 128;  // NORM: row r's raw k, 64 channels
 #pragma unroll
             for (int cc = 0; cc < SC / 16; ++cc) {
                 const int j0 = cq * SC + cc * 16;
@@ -1975,6 +2025,18 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
 #pragma unroll
                 for (int x = 0; x < 16; ++x)
                     vk[x] = have_g ? fmaf(w_out, __uint_as_float(ri[x]), __uint_as_float(rk[x])) : __uint_as_float(rk[x]);
+                if (NORM && j0 < 64) {
+                    // dk = dk''[:64] (.) phi'(k) (psi' = phi')
+#pragma unroll
+                    for (int x = 0; x < 16; x += 4) {
+                        const float4 o = times_phi_prime(make_float4(vk[x], vk[x + 1], vk[x + 2], vk[x + 3]),
+                                                         *reinterpret_cast<const uint2*>(kraw + sw_off(r, j0 + x)));
+                        vk[x] = o.x;
+                        vk[x + 1] = o.y;
+                        vk[x + 2] = o.z;
+                        vk[x + 3] = o.w;
+                    }
+                }
                 stage_f32x16(smem, dk_chunk, r, j0, vk);
             }
         }
@@ -2045,7 +2107,10 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         have_g = true;
         __syncthreads();
         if (D == 64 && next && tid == 0) issue_tile_b(tile - 1);
-        if (NORM) const_box<kRThreads>(smem + S::OFF_K, tid, true);  // K's constant half held dk rows
+        if (NORM) {
+            const_box<kRThreads>(smem + S::OFF_K, tid, true);  // K's constant half held dk rows
+            const_box<kRThreads>(smem + S::OFF_V, tid, true);  // V's held the raw k rows
+        }
 
         // ---- G_{c-1} -> bf16 operand for the next tile (and dS0 at the tape start) ----
         {
@@ -2080,6 +2145,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         // let work still in flight finish before the CTA's TMEM and shared memory go away
         if (drain != nullptr) wait_mbar(drain, drain_par, kDrainNs);
         if (pending) wait_mbar(full, it & 1, kDrainNs);
+        if (NORM && k_pending) wait_mbar(kbar, it & 1, kDrainNs);
     }
     if (tid == 0) bulk_wait_all();
     if (tid == 0 && p.gpart != nullptr) p.gpart[bh * p.G + g] = gsum;

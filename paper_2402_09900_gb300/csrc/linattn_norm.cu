@@ -30,7 +30,9 @@
 // this basis the state S'' = sum decay k'' v'^T has the incoming (X, x) in its
 // first d rows and sum decay v'^T in rows d and d + 1; dphi(q)_i = dq''_i +
 // dq''_d (folded in the kernel), dq = dphi(q) (.) phi'(q), dk = dk''[:d] (.)
-// phi'(k).  Heads of width d <= 120 (a multiple of 8) are supported.
+// phi'(k): for 64-channel heads the kernels' epilogues apply phi' (from the
+// raw q and k tiles) and write the caller's gradients, otherwise a chain-rule
+// pass does.  Heads of width d <= 120 (a multiple of 8) are supported.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -301,14 +303,16 @@ int kernels_per_call(int64_t B, int64_t L, int64_t H, int64_t d, int backward, i
     if (B == 0 || L == 0 || H == 0) return 0;
     // prep, the linear-attention call, then the divide (forward) or the upstream
     // gradient and the chain rule (backward); with states: their padding and
-    // unpadding.  The forward of 64-channel heads (y 16-byte aligned) is the fused
-    // call alone; their backward builds its operands in the kernels (no prep).
+    // unpadding.  64-channel heads (in the forward with y 16-byte aligned) run the
+    // fused kernels: the forward is the linear-attention call alone, the backward
+    // the upstream gradient and that call (operands built and the chain rule
+    // applied in the kernels).
     const bool pad = debug_knobs().lnorm_padded != 0;
-    const bool fused_fwd = !backward && d == 64 && !pad, no_prep = d == 64 && !pad;
+    const bool fused = d == 64 && !pad;
     // the backward hands its bf16 upstream gradient to the linear-attention call,
     // which then skips its own bf16 copy
-    const int base = (no_prep ? 0 : 1) + (backward ? 2 : (fused_fwd ? 0 : 1)) +
-                     la::kernels_per_call(B, L, H, backward, with_dgamma_per_head) - (backward ? 1 : 0);
+    const int base = la::kernels_per_call(B, L, H, backward, with_dgamma_per_head) +
+                     (backward ? (fused ? 1 : 3) - 1 : (fused ? 0 : 2));
     return base + (with_states ? (backward ? 3 : 2) : 0);
 }
 
@@ -319,8 +323,10 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
     // inside the tensor-core kernel (la::Args::norm); everything else goes
     // through the padded operands
     // (the backward of 64-channel heads also builds its operands in the kernels)
-    const bool fused = debug_knobs().lnorm_padded == 0 &&
-                       (a.backward ? a.d == 64 : a.d == 64 && (reinterpret_cast<uintptr_t>(a.y) & 15u) == 0);  // y: TMA stores
+    // (the kernels' TMA stores write y, or dq, dk and dv, straight to the caller's
+    // arrays: y must be 16-byte aligned, as the gradients always are)
+    const bool fused = debug_knobs().lnorm_padded == 0 && a.d == 64 &&
+                       (a.backward || (reinterpret_cast<uintptr_t>(a.y) & 15u) == 0);
     if (!fused)
         prep_kernel<<<grid_for(R * 16), 256, 0, s>>>(static_cast<const uint4*>(a.q), static_cast<const uint4*>(a.k),
                                                      static_cast<const uint4*>(a.v), R, static_cast<int>(a.d),
@@ -380,25 +386,30 @@ memoroid_status_t launch(const Args& a, cudaStream_t s) {
     const int64_t wout = a.d <= 64 ? 64 : kW;
     l.out_cols = a.d <= 64 ? 64 : 0;
     l.fold_col = a.d;  // dphi(q)_i = dq''_i + dq''_d
+    l.dq = b.dq;
+    l.dk = b.dk;
+    l.dv = b.dv;
     if (fused) {
+        // the kernels build the operands from q, k, v and apply the chain rule
+        // through phi in their epilogues, writing the caller's gradients
         l.q = a.q;
         l.k = a.k;
         l.v = a.v;
         l.norm = 1;
+        l.dq = a.dq;
+        l.dk = a.dk;
+        l.dv = a.dv;
     }
-    l.dq = b.dq;
-    l.dk = b.dk;
-    l.dv = b.dv;
     l.dgamma = a.dgamma;
     l.dS0 = (a.dS0 != nullptr || a.dz0 != nullptr) ? b.S2 : nullptr;
     const memoroid_status_t st = la::launch_bwd(l, s);
     if (st != MEMOROID_OK) return st;
-    chain_kernel<<<grid_for(R * a.d / 4), 256, 0, s>>>(
-        reinterpret_cast<const float4*>(b.dq), reinterpret_cast<const float4*>(b.dk),
-        reinterpret_cast<const float4*>(b.dv), static_cast<const uint2*>(a.q), static_cast<const uint2*>(a.k),
-        static_cast<uint32_t>(R), static_cast<uint32_t>(a.d / 4), static_cast<uint32_t>(wout / 4),
-        reinterpret_cast<float4*>(a.dq),
-        reinterpret_cast<float4*>(a.dk), reinterpret_cast<float4*>(a.dv));
+    if (!fused)
+        chain_kernel<<<grid_for(R * a.d / 4), 256, 0, s>>>(
+            reinterpret_cast<const float4*>(b.dq), reinterpret_cast<const float4*>(b.dk),
+            reinterpret_cast<const float4*>(b.dv), static_cast<const uint2*>(a.q), static_cast<const uint2*>(a.k),
+            static_cast<uint32_t>(R), static_cast<uint32_t>(a.d / 4), static_cast<uint32_t>(wout / 4),
+            reinterpret_cast<float4*>(a.dq), reinterpret_cast<float4*>(a.dk), reinterpret_cast<float4*>(a.dv));
     if (l.dS0 != nullptr)
         unpad_state_kernel<<<grid_for(BH * a.d * (a.d + 1)), 256, 0, s>>>(b.S2, BH, static_cast<int>(a.d), 1, a.dS0,
                                                                            a.dz0);

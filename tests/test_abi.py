@@ -145,9 +145,10 @@ def test_linattn_norm_validation(lib):
     fwd64 = lib.memoroid_linattn_norm_kernels_per_call(1, 4096, 4, 64, 0, 0, 0)
     fwd32 = lib.memoroid_linattn_norm_kernels_per_call(1, 4096, 4, 32, 0, 0, 0)
     assert fwd32 - fwd64 == 2
-    # the backward of 64-channel heads builds its operands inside the kernels (no padding kernel)
+    # the backward of 64-channel heads builds its operands and applies the chain rule
+    # through phi inside the kernels (no padding kernel, no chain-rule kernel)
     assert lib.memoroid_linattn_norm_kernels_per_call(1, 4096, 4, 32, 1, 0, 0) - \
-        lib.memoroid_linattn_norm_kernels_per_call(1, 4096, 4, 64, 1, 0, 0) == 1
+        lib.memoroid_linattn_norm_kernels_per_call(1, 4096, 4, 64, 1, 0, 0) == 2
 
     def fwd(q=FAKE, d=64, ws=FAKE, wsb=1 << 40, gps=0):
         return lib.memoroid_linattn_norm_fwd(q, FAKE, FAKE, FAKE, gps, FAKE, None, None, FAKE + 0x1000, None, None,
