@@ -76,17 +76,34 @@ struct Aff {
 __device__ __forceinline__ Aff compose(Aff e, Aff l) { return Aff{e.a * l.a, fmaf(e.a, l.x, e.x)}; }
 
 // first nonzero flag of st in [a, e), or -1; the same value in every lane.
-// Each round trip covers 4 * 32 * 8 bytes (byte loads: no alignment needed).
-__device__ int64_t find_flag(const uint8_t* st, int64_t a, int64_t e, int lane) {
+// Each round trip covers 4 * 32 * 8 bytes.  With `vec` (st 8-byte aligned)
+// every lane loads four aligned 8-byte words from a base rounded down to 8
+// bytes, and the bytes outside [a, e) are masked; otherwise byte loads.
+__device__ int64_t find_flag(const uint8_t* st, int64_t a, int64_t e, int lane, bool vec) {
     constexpr int kSpan = 4 * 32 * 8;
-    for (int64_t base = a; base < e; base += kSpan) {
+    for (int64_t base = vec ? (a & ~int64_t{7}) : a; base < e; base += kSpan) {
         int first = kSpan;
+        if (vec) {
 #pragma unroll
-        for (int j = 4 * 8 - 1; j >= 0; --j) {
-            // lane covers bytes [q * 256 + lane * 8, + 8) of this span for q = j / 8
-            const int off = (j >> 3) * 256 + lane * 8 + (j & 7);
-            const int64_t t = base + off;
-            if (t < e && st[t] != 0) first = min(first, off);
+            for (int q = 3; q >= 0; --q) {
+                // lane covers bytes [q * 256 + lane * 8, + 8) of this span
+                const int off = q * 256 + lane * 8;
+                const int64_t t = base + off;
+                if (t < e) {
+                    unsigned long long w = *reinterpret_cast<const unsigned long long*>(st + t);
+                    // bytes before a or at / after e do not count
+                    if (t < a) w &= ~0ull << (8 * (a - t));
+                    if (t + 8 > e) w &= ~0ull >> (8 * (t + 8 - e));
+                    if (w != 0ull) first = min(first, off + (__ffsll(static_cast<long long>(w)) - 1) / 8);
+                }
+            }
+        } else {
+#pragma unroll
+            for (int j = 4 * 8 - 1; j >= 0; --j) {
+                const int off = (j >> 3) * 256 + lane * 8 + (j & 7);
+                const int64_t t = base + off;
+                if (t < e && st[t] != 0) first = min(first, off);
+            }
         }
         // smallest offset over the lanes
 #pragma unroll
@@ -251,7 +268,7 @@ __global__ void __launch_bounds__(kThreads, GAE ? 3 : 4) scan_kernel(const Param
     const bool nf_e = e < p.L ? st[e] != 0 : true;  // begin flag of the step after the range
     const float nv_e = (GAE && e < p.L) ? p.v[b * p.L + e] : 0.f;
     // the first cut: the first begin flag in (a, e] (step f - 1 does not see step f)
-    const int64_t f = p.G > 1 ? find_flag(st, a + 1, min(e + 1, p.L), lane) : -1;
+    const int64_t f = p.G > 1 ? find_flag(st, a + 1, min(e + 1, p.L), lane, p.vec != 0) : -1;
     const bool cut = f >= 0;
     if (p.G > 1) {
         // the range's map; with a cut its steps before f are final (written now)
