@@ -286,9 +286,10 @@ __device__ __forceinline__ void scale_rows_sw(unsigned char* tile, int tid, WFn 
     }
 }
 
-// phi'(z) of the raw input (1 above 0, else e^z): the chain rule of the
-// normalised backward, applied to dq and dk in the epilogues
-__device__ __forceinline__ float phi_prime(float z) { return z > 0.f ? 1.f : expf(z); }
+// phi'(z) of the raw input (1 above 0, else e^z, by the SFU exponential: a
+// few ulp of fp32): the chain rule of the normalised backward, applied to dq
+// and dk in the epilogues
+__device__ __forceinline__ float phi_prime(float z) { return z > 0.f ? 1.f : __expf(z); }
 __device__ __forceinline__ float4 times_phi_prime(float4 o, uint2 raw) {
     const float2 a = unpack_bf16x2(raw.x), b = unpack_bf16x2(raw.y);
     return make_float4(o.x * phi_prime(a.x), o.y * phi_prime(a.y), o.z * phi_prime(b.x), o.w * phi_prime(b.y));
@@ -966,7 +967,6 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                             o.w += ofold;
                         }
                         const int j = j0 + x;  // 4 channels = one 16-byte unit
-                        if (NB) o = times_phi_prime(o, *reinterpret_cast<const uint2*>(qs + sw_off(t, j)));
                         *reinterpret_cast<float4*>(yst + (j >> 5) * (T * 128) + ((((j & 31) >> 2) ^ (t & 7)) << 4)) = o;
                     }
                 }
@@ -1025,6 +1025,19 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
             }
             if (FOLD) zacc += zfold;
             if (BWD) reinterpret_cast<float*>(smem + S::OFF_Z)[half * T + t] = w_in * zacc;
+        }
+        if (NB) {
+            // dq = dphi(q) (.) phi'(q) on the staged rows, from the raw q tile: two
+            // threads per row, one 32-channel chunk each
+            __syncthreads();
+            const int r = tid >> 1, m = tid & 1;
+            unsigned char* row = smem + s * S::STAGE + Y_OFF + m * (T * 128) + r * 128;
+            const unsigned char* qs = smem + (stage_q(s) - sbase);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                float4* o = reinterpret_cast<float4*>(row + ((u ^ (r & 7)) << 4));
+                *o = times_phi_prime(*o, *reinterpret_cast<const uint2*>(qs + sw_off(r, 32 * m + 4 * u)));
+            }
         }
         if (BWD) __syncthreads();  // every z term has read the q tile, where the state is staged next
         // ---- state: bf16 copy for the next tile, decay by the next tile's a ----
@@ -2013,7 +2026,6 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
         {
             const int r = 32 * quarter + lane;
             const float w_out = r >= mc.last_start ? fast_exp2(mc.lam2[T - 1] - mc.lam2[r]) : 0.f;
-            const unsigned char* kraw = smem + S::OFF_V + T * 128;  // NORM: row r's raw k, 64 channels
 #pragma unroll
             for (int cc = 0; cc < SC / 16; ++cc) {
                 const int j0 = cq * SC + cc * 16;
@@ -2025,19 +2037,20 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
 #pragma unroll
                 for (int x = 0; x < 16; ++x)
                     vk[x] = have_g ? fmaf(w_out, __uint_as_float(ri[x]), __uint_as_float(rk[x])) : __uint_as_float(rk[x]);
-                if (NORM && j0 < 64) {
-                    // dk = dk''[:64] (.) phi'(k) (psi' = phi')
-#pragma unroll
-                    for (int x = 0; x < 16; x += 4) {
-                        const float4 o = times_phi_prime(make_float4(vk[x], vk[x + 1], vk[x + 2], vk[x + 3]),
-                                                         *reinterpret_cast<const uint2*>(kraw + sw_off(r, j0 + x)));
-                        vk[x] = o.x;
-                        vk[x + 1] = o.y;
-                        vk[x + 2] = o.z;
-                        vk[x + 3] = o.w;
-                    }
-                }
                 stage_f32x16(smem, dk_chunk, r, j0, vk);
+            }
+        }
+        if (NORM) {
+            // dk = dk''[:64] (.) phi'(k) (psi' = phi') on the staged rows, from the
+            // raw k rows: four threads per row, 16 channels each
+            __syncthreads();
+            const int r = tid >> 2, m = (tid >> 1) & 1, u0 = (tid & 1) * 4;
+            const unsigned char* kraw = smem + S::OFF_V + T * 128;
+            unsigned char* row = smem + S::dk_chunk(m) + r * 128;
+#pragma unroll
+            for (int u = u0; u < u0 + 4; ++u) {
+                float4* o = reinterpret_cast<float4*>(row + ((u ^ (r & 7)) << 4));
+                *o = times_phi_prime(*o, *reinterpret_cast<const uint2*>(kraw + sw_off(r, 32 * m + 4 * u)));
             }
         }
         tc::fence_smem_to_async();

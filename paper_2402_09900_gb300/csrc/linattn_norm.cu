@@ -52,7 +52,9 @@ constexpr int kCtas = 152 * 8;
 // (__expf, a few ulp of fp32) is exact enough; the fused forward of linattn.cu
 // computes the same expression
 __device__ __forceinline__ float phi(float z) { return z > 0.f ? 1.f + z : __expf(z); }
-__device__ __forceinline__ float dphi(float z) { return z > 0.f ? 1.f : expf(z); }
+// phi'(z), also by the SFU exponential: the fused kernels' epilogues compute the
+// same expression, so both paths give the same gradients bit for bit
+__device__ __forceinline__ float dphi(float z) { return z > 0.f ? 1.f : __expf(z); }
 
 struct Buffers {
     __nv_bfloat16 *q, *k, *v;  // [R, 128]
