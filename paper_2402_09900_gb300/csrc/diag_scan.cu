@@ -132,6 +132,7 @@ struct Params {
 };
 
 __host__ __device__ __forceinline__ int64_t lmin(int64_t a, int64_t b) { return a < b ? a : b; }
+
 __host__ __device__ __forceinline__ int64_t lmax(int64_t a, int64_t b) { return a > b ? a : b; }
 
 // ---- FFM layout: one lane's two channels (2 lane, 2 lane + 1 of the slab) ----
@@ -828,6 +829,7 @@ __global__ void __launch_bounds__(CARRY_WARPS * 32) segment_carry_kernel(const P
     __shared__ uint32_t s_b[CARRY_WARPS];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t chain = blockIdx.x;
+    ptx::grid_dependency_wait();  // the scan's summaries
     if (ptx::ld_relaxed(p.hdr) != 0u) return;  // uniform over the CTA
     const int64_t G = p.n_seg;
     const int64_t b = chain / p.n_slabs;
@@ -1015,6 +1017,7 @@ __device__ void segment_fix_tile(const Params& p, int64_t tid, int part, int npa
 
 template <class C>
 __global__ void __launch_bounds__(128) segment_fix_kernel(const Params p) {
+    ptx::grid_dependency_wait();  // the segment carries
     if (ptx::ld_relaxed(p.hdr) != 0u) return;
     const int64_t n_fix = static_cast<int64_t>(ptx::ld_relaxed(p.hdr + 4));
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1049,6 +1052,7 @@ __global__ void __launch_bounds__(256) reduce_parts_kernel(const float4* __restr
                                                            double* __restrict__ rpart, int64_t B,
                                                            int64_t n_slabs, int64_t n_tt) {
     __shared__ double s[8][32][4];
+    ptx::grid_dependency_wait();  // the tile partials, fixed up
     const int slab = blockIdx.x, part = blockIdx.y;
     const int grp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t total = B * n_tt;
@@ -1094,6 +1098,7 @@ __global__ void __launch_bounds__(256) reduce_parts_kernel(const float4* __restr
 __global__ void __launch_bounds__(RED_PARTS) reduce_final_kernel(const double* __restrict__ rpart,
                                                                  float4* __restrict__ grad_lambda, int64_t D2) {
     __shared__ double2 s[2][RED_PARTS];
+    ptx::grid_dependency_wait();  // the parts
     const int slab = blockIdx.x >> 5, lane = blockIdx.x & 31, p = threadIdx.x;
     const double2* o =
         reinterpret_cast<const double2*>(rpart + ((static_cast<int64_t>(slab) * RED_PARTS + p) * 32 + lane) * 4);
@@ -1288,11 +1293,14 @@ memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
     kernel<<<static_cast<unsigned>(n_tickets), C::THREADS, C::SMEM, s>>>(p);
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     if (sg.G > 1) {
-        segment_carry_kernel<<<static_cast<unsigned>(l.n_chains), CARRY_WARPS * 32, 0, s>>>(p, C::REV);
+        if (launch_after(segment_carry_kernel, dim3(static_cast<unsigned>(l.n_chains)), dim3(CARRY_WARPS * 32), 0, s, p,
+                         C::REV) != cudaSuccess)
+            return MEMOROID_ERR_CUDA;
         const int64_t n_tiles = l.n_chains * l.n_tt;
         // the CTAs (per-channel lambda) or warps (per-step lambda) walk the list of tiles to fix
         const int64_t fix_ctas = lmin(C::PS ? (n_tiles + 3) / 4 : n_tiles, 152 * 8);
-        segment_fix_kernel<C><<<static_cast<unsigned>(fix_ctas), 128, 0, s>>>(p);
+        if (launch_after(segment_fix_kernel<C>, dim3(static_cast<unsigned>(fix_ctas)), dim3(128), 0, s, p) != cudaSuccess)
+            return MEMOROID_ERR_CUDA;
         if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
     }
     if (out_layout) *out_layout = l;
@@ -1337,11 +1345,12 @@ memoroid_status_t launch_bwd(const Args& a, cudaStream_t s) {
         unsigned char* ws = static_cast<unsigned char*>(a.workspace);
         const float4* gpart = reinterpret_cast<const float4*>(ws + l.gpart_off);
         double* rpart = reinterpret_cast<double*>(ws + l.rpart_off);
-        reduce_parts_kernel<<<dim3(static_cast<unsigned>(l.n_slabs), RED_PARTS), 256, 0, s>>>(
-            gpart, rpart, a.B, l.n_slabs, l.n_tt);
-        reduce_final_kernel<<<static_cast<unsigned>(l.n_slabs * 32), RED_PARTS, 0, s>>>(
-            rpart, static_cast<float4*>(a.grad_lambda), a.D / 2);
-        if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+        if (launch_after(reduce_parts_kernel, dim3(static_cast<unsigned>(l.n_slabs), RED_PARTS), dim3(256), 0, s, gpart,
+                         rpart, a.B, l.n_slabs, l.n_tt) != cudaSuccess ||
+            launch_after(reduce_final_kernel, dim3(static_cast<unsigned>(l.n_slabs * 32)), dim3(RED_PARTS), 0, s,
+                         static_cast<const double*>(rpart), static_cast<float4*>(a.grad_lambda), a.D / 2) !=
+                cudaSuccess)
+            return MEMOROID_ERR_CUDA;
     }
     return MEMOROID_OK;
 }

@@ -47,6 +47,27 @@ DebugKnobs debug_knobs();
 // past generation, and the region was cleared since.
 uint32_t tagged_epoch(const void* workspace, size_t region_end, bool* clear);
 
+// Launches a kernel that follows another kernel on the stream with programmatic
+// stream serialization: it may be scheduled before that kernel completes and
+// waits for it at its first statement (ptx::grid_dependency_wait), which hides
+// the launch latency between the two.  Only for kernels whose predecessor on
+// the stream is a kernel.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_after(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                         Args... args) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // cuTensorMapEncodeTiled, taken from the driver at run time (the library does

@@ -560,6 +560,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
     constexpr int DOUT = (NORM || HALF_OUT) ? 64 : D;  // output channels written
     constexpr int Y_OFF = NF ? 0 : S::OFF_Y;  // output staging: the Q slot (NF) or the K and V slots
     extern __shared__ __align__(1024) unsigned char smem[];
+    grid_dependency_wait();  // the kernel before this one on the stream (metadata, carries)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int quarter = warp & 3, half = warp >> 2;
     const int64_t bh = blockIdx.x / p.G;
@@ -1193,6 +1194,7 @@ __global__ void __launch_bounds__(kThreads, 1) seg_state_kernel(const __grid_con
     // 1, 1, 0]; reverse X = q'' = [phi(q), sigma_hi, sigma_lo, 0]; the forward's
     // Y holds v and the columns [1, 1, 0, ...]; the reverse Y is the padded dy'
     static_assert(!NORM || D == 128, "the normalised operands run at d = 128");
+    grid_dependency_wait();  // the metadata (and, in the backward, the kernels before)
     static_assert(!REV || !NORM || PSI, "the reverse summary runs in the backward's basis");
     using S = SegSmem<D>;
     constexpr int BX = NORM ? 64 : D;
@@ -1445,6 +1447,7 @@ __global__ void __launch_bounds__(kThreads, 1) seg_state_kernel(const __grid_con
 template <bool REV>
 __global__ void __launch_bounds__(256) seg_carry_kernel(float* __restrict__ buf, const float2* __restrict__ info,
                                                        const float* __restrict__ init, int G, int DD) {
+    grid_dependency_wait();  // the segment summaries
     const int64_t bh = blockIdx.y;
     const int e = (blockIdx.x * 256 + threadIdx.x) * 4;
     if (e >= DD) return;
@@ -1609,6 +1612,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
     constexpr int DOUT = HALF_OUT ? 64 : D;
     using S = BwdSmem<D>;
     extern __shared__ __align__(1024) unsigned char smem[];
+    grid_dependency_wait();  // pass F (its tile states and dgamma terms)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int quarter = warp & 3, cq = warp >> 2;  // TMEM lane quarter, column quarter
     const int64_t bh = blockIdx.x / p.G;
@@ -2170,6 +2174,7 @@ __global__ void __launch_bounds__(kRThreads, 1) bwd_kernel(const __grid_constant
 
 // grad_y (fp32) -> bf16 operand copy (round to nearest even), 8 values per thread
 __global__ void __launch_bounds__(256) to_bf16_kernel(const float* __restrict__ x, uint16_t* __restrict__ y, int64_t n8) {
+    grid_dependency_wait();  // the kernel before it on the stream
     for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n8;
          i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const float4 a = reinterpret_cast<const float4*>(x)[2 * i];
@@ -2186,6 +2191,7 @@ __global__ void __launch_bounds__(256) to_bf16_kernel(const float* __restrict__ 
 // per-head dL/dgamma_h = (sum over tapes and segments of dL/dlog(gamma)) / gamma_h, fixed order
 __global__ void dgamma_head_kernel(const float* __restrict__ gpart, const float* __restrict__ gamma,
                                    float* __restrict__ dgamma, int64_t B, int64_t H, int G) {
+    grid_dependency_wait();  // pass R's per-segment sums
     const int64_t h = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (h >= H) return;
     double acc = 0.0;
@@ -2368,12 +2374,14 @@ memoroid_status_t launch_seg_carry(const Args& a, const Plan& pl, const TileMeta
     p.G = static_cast<int>(pl.G);
     p.wait_ns = debug_knobs().wait_ns;
     if (set_smem(seg_state_kernel<D, REV, NORM, PSI>, SegSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    seg_state_kernel<D, REV, NORM, PSI><<<static_cast<unsigned>(a.B * a.H * (pl.G - 1)), kThreads, SegSmem<D>::BYTES,
-                                     stream>>>(p);
-    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    if (launch_after(seg_state_kernel<D, REV, NORM, PSI>, dim3(static_cast<unsigned>(a.B * a.H * (pl.G - 1))),
+                     dim3(kThreads), SegSmem<D>::BYTES, stream, p) != cudaSuccess)
+        return MEMOROID_ERR_CUDA;
     const dim3 grid(static_cast<unsigned>((D * D / 4 + 255) / 256), static_cast<unsigned>(a.B * a.H));
-    seg_carry_kernel<REV><<<grid, 256, 0, stream>>>(buf, info, init, static_cast<int>(pl.G), D * D);
-    return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
+    return launch_after(seg_carry_kernel<REV>, grid, dim3(256), 0, stream, buf, static_cast<const float2*>(info), init,
+                        static_cast<int>(pl.G), D * D) == cudaSuccess
+               ? MEMOROID_OK
+               : MEMOROID_ERR_CUDA;
 }
 
 template <int D, bool NORM = false>
@@ -2416,8 +2424,9 @@ memoroid_status_t launch_fwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     p.states = nullptr;
     p.fold_col = -1;
     if (set_smem(fwd_kernel<D, false, NORM>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    fwd_kernel<D, false, NORM><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(p);
-    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    if (launch_after(fwd_kernel<D, false, NORM>, dim3(static_cast<unsigned>(a.B * a.H * pl.G)), dim3(kThreads), FwdSmem<D>::BYTES, stream, p) !=
+        cudaSuccess)
+        return MEMOROID_ERR_CUDA;
     return MEMOROID_OK;
 }
 template <int D, bool HALF_OUT = false, bool NORM = false>
@@ -2439,9 +2448,9 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     if (a.grad_y16 == nullptr) {
         const int64_t n8 = a.B * a.L * a.H * D / 8;
         const int64_t cblocks = min((n8 + 255) / 256, static_cast<int64_t>(kTargetCtas) * 16);
-        to_bf16_kernel<<<static_cast<unsigned>(cblocks), 256, 0, stream>>>(a.grad_y, reinterpret_cast<uint16_t*>(ws + ly.dy16),
-                                                                            n8);
-        if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+        if (launch_after(to_bf16_kernel, dim3(static_cast<unsigned>(cblocks)), dim3(256), 0, stream, a.grad_y,
+                         reinterpret_cast<uint16_t*>(ws + ly.dy16), n8) != cudaSuccess)
+            return MEMOROID_ERR_CUDA;
     }
 
     // the operand maps of pass R, also read by the segment summaries
@@ -2490,15 +2499,19 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     if constexpr (NORM) {
         if (a.fold_col < 0) return MEMOROID_ERR_UNSUPPORTED;
         if (set_smem(fwd_kernel<D, true, NORM, HALF_OUT, true>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-        fwd_kernel<D, true, NORM, HALF_OUT, true>
-            <<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
+        if (launch_after(fwd_kernel<D, true, NORM, HALF_OUT, true>, dim3(static_cast<unsigned>(a.B * a.H * pl.G)), dim3(kThreads), FwdSmem<D>::BYTES,
+                         stream, f) != cudaSuccess)
+            return MEMOROID_ERR_CUDA;
     } else if (a.fold_col >= 0) {
         if (set_smem(fwd_kernel<D, true, false, HALF_OUT, true>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-        fwd_kernel<D, true, false, HALF_OUT, true>
-            <<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
+        if (launch_after(fwd_kernel<D, true, false, HALF_OUT, true>, dim3(static_cast<unsigned>(a.B * a.H * pl.G)), dim3(kThreads), FwdSmem<D>::BYTES,
+                         stream, f) != cudaSuccess)
+            return MEMOROID_ERR_CUDA;
     } else {
         if (set_smem(fwd_kernel<D, true, false, HALF_OUT>, FwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-        fwd_kernel<D, true, false, HALF_OUT><<<static_cast<unsigned>(a.B * a.H * pl.G), kThreads, FwdSmem<D>::BYTES, stream>>>(f);
+        if (launch_after(fwd_kernel<D, true, false, HALF_OUT>, dim3(static_cast<unsigned>(a.B * a.H * pl.G)), dim3(kThreads), FwdSmem<D>::BYTES, stream,
+                         f) != cudaSuccess)
+            return MEMOROID_ERR_CUDA;
     }
     if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
 
@@ -2529,12 +2542,14 @@ memoroid_status_t launch_bwd_d(const Args& a, const Plan& pl, const Layout& ly, 
     r.wait_ns = debug_knobs().wait_ns;
     r.fail_cta = debug_knobs().withhold_ticket;
     if (set_smem(bwd_kernel<D, HALF_OUT, NORM>, BwdSmem<D>::BYTES) != cudaSuccess) return MEMOROID_ERR_CUDA;
-    bwd_kernel<D, HALF_OUT, NORM><<<static_cast<unsigned>(a.B * a.H * pl.G), kRThreads, BwdSmem<D>::BYTES, stream>>>(r);
-    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    if (launch_after(bwd_kernel<D, HALF_OUT, NORM>, dim3(static_cast<unsigned>(a.B * a.H * pl.G)), dim3(kRThreads), BwdSmem<D>::BYTES, stream, r) !=
+        cudaSuccess)
+        return MEMOROID_ERR_CUDA;
     if (r.gpart != nullptr) {
-        dgamma_head_kernel<<<static_cast<unsigned>((a.H + 127) / 128), 128, 0, stream>>>(gpart, a.gamma, a.dgamma,
-                                                                                          a.B, a.H, static_cast<int>(pl.G));
-        if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+        if (launch_after(dgamma_head_kernel, dim3(static_cast<unsigned>((a.H + 127) / 128)), dim3(128), 0, stream,
+                         static_cast<const float*>(gpart), a.gamma, a.dgamma, a.B, a.H, static_cast<int>(pl.G)) !=
+            cudaSuccess)
+            return MEMOROID_ERR_CUDA;
     }
     return MEMOROID_OK;
 }

@@ -131,6 +131,12 @@ __device__ __forceinline__ float fast_exp2(float x) {
     return y;
 }
 
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialization waits here until the kernel before it on the stream has
+// completed and its memory operations are visible (it may have been scheduled
+// earlier; nothing before this wait may read that kernel's results).
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ uint64_t globaltimer() {
     uint64_t t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
