@@ -1382,6 +1382,7 @@ __global__ void __launch_bounds__(256) ffm_param_grad_kernel(const float2* __res
                                                              const float* __restrict__ alpha, int64_t m, int64_t c,
                                                              float* __restrict__ grad_alpha,
                                                              float* __restrict__ grad_omega) {
+    ptx::grid_dependency_wait();  // the grad_lambda reduction
     const int64_t k = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (k < m) {
         if (grad_alpha == nullptr) return;
@@ -1460,9 +1461,11 @@ memoroid_status_t launch_ffm(const FfmArgs& f, cudaStream_t s) {
     a.grad_h0 = f.grad_S0;
     const memoroid_status_t st = launch_bwd(a, s);
     if (st != MEMOROID_OK || !param) return st;
-    ffm_param_grad_kernel<<<static_cast<unsigned>((f.m + f.c + 255) / 256), 256, 0, s>>>(
-        glam, lam, f.alpha, f.m, f.c, f.grad_alpha, f.grad_omega);
-    return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
+    return launch_after(ffm_param_grad_kernel, dim3(static_cast<unsigned>((f.m + f.c + 255) / 256)), dim3(256), 0, s,
+                        static_cast<const float2*>(glam), static_cast<const float2*>(lam), f.alpha, f.m, f.c,
+                        f.grad_alpha, f.grad_omega) == cudaSuccess
+               ? MEMOROID_OK
+               : MEMOROID_ERR_CUDA;
 }
 
 }  // namespace diag

@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 
 #include "internal.cuh"
+#include "ptx.cuh"
 
 namespace memoroid {
 namespace tape {
@@ -47,6 +48,7 @@ __global__ void __launch_bounds__(CHUNK_THREADS) count_kernel(const uint8_t* __r
 __global__ void __launch_bounds__(1024) scan_counts_kernel(int64_t* __restrict__ counts, int64_t nb,
                                                            int64_t* __restrict__ count) {
     __shared__ int64_t s[1024];
+    ptx::grid_dependency_wait();  // the chunk counts
     __shared__ int64_t s_carry;
     if (threadIdx.x == 0) s_carry = 0;
     __syncthreads();
@@ -76,6 +78,7 @@ __global__ void __launch_bounds__(CHUNK_THREADS) write_offsets_kernel(
     const uint8_t* __restrict__ start, int64_t L, const int64_t* __restrict__ base_off,
     int64_t* __restrict__ offsets) {
     __shared__ int s[CHUNK_THREADS];
+    ptx::grid_dependency_wait();  // the chunk offsets
     const int64_t base = static_cast<int64_t>(blockIdx.x) * CHUNK;
     const int64_t t0 = base + static_cast<int64_t>(threadIdx.x) * CHUNK_PER_THREAD;
     int c = 0;
@@ -128,9 +131,11 @@ memoroid_status_t launch_offsets_from_starts(const uint8_t* start, int64_t L, in
     }
     int64_t* counts = reinterpret_cast<int64_t*>(static_cast<unsigned char*>(workspace) + kHeaderBytes);
     count_kernel<<<static_cast<unsigned>(nb), CHUNK_THREADS, 0, s>>>(start, L, counts);
-    scan_counts_kernel<<<1, 1024, 0, s>>>(counts, nb, count);
-    write_offsets_kernel<<<static_cast<unsigned>(nb), CHUNK_THREADS, 0, s>>>(start, L, counts, offsets);
-    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    if (cudaGetLastError() != cudaSuccess ||
+        launch_after(scan_counts_kernel, dim3(1), dim3(1024), 0, s, counts, nb, count) != cudaSuccess ||
+        launch_after(write_offsets_kernel, dim3(static_cast<unsigned>(nb)), dim3(CHUNK_THREADS), 0, s, start, L,
+                     static_cast<const int64_t*>(counts), offsets) != cudaSuccess)
+        return MEMOROID_ERR_CUDA;
     return MEMOROID_OK;
 }
 

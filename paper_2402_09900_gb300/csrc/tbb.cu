@@ -25,6 +25,7 @@
 #include <cstdint>
 
 #include "internal.cuh"
+#include "ptx.cuh"
 
 namespace memoroid {
 namespace tbb {
@@ -128,6 +129,7 @@ __global__ void __launch_bounds__(256) fill_kernel(const int64_t* __restrict__ b
                                                    const int64_t* __restrict__ ep, int64_t B,
                                                    const int64_t* __restrict__ off, const int64_t* __restrict__ meta,
                                                    uint8_t* __restrict__ start, int64_t* __restrict__ src) {
+    ptx::grid_dependency_wait();  // the episode offsets
     const int lane = threadIdx.x & 31;
     const int64_t gw = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int64_t nw = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
@@ -206,8 +208,11 @@ memoroid_status_t launch_sample(const int64_t* begin, int64_t E, int64_t N, cons
     int64_t* meta = reinterpret_cast<int64_t*>(ws + kHeaderBytes);
     int64_t* off = meta + 2;
     offsets_kernel<<<1, kScanThreads, 0, s>>>(begin, E, N, ep, K, B, off, meta, hdr, n_used);
-    fill_kernel<<<kFillCtas, 256, 0, s>>>(begin, E, N, ep, B, off, meta, start, src);
-    return cudaGetLastError() == cudaSuccess ? MEMOROID_OK : MEMOROID_ERR_CUDA;
+    if (cudaGetLastError() != cudaSuccess) return MEMOROID_ERR_CUDA;
+    return launch_after(fill_kernel, dim3(kFillCtas), dim3(256), 0, s, begin, E, N, ep, B,
+                        static_cast<const int64_t*>(off), static_cast<const int64_t*>(meta), start, src) == cudaSuccess
+               ? MEMOROID_OK
+               : MEMOROID_ERR_CUDA;
 }
 
 memoroid_status_t launch_gather(const void* rows, int64_t N, int64_t row_bytes, const int64_t* src, int64_t B,
