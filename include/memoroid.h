@@ -392,8 +392,9 @@ memoroid_status_t memoroid_gather_rows(const void *rows, int64_t N, int64_t row_
 /* ======================================================================== */
 
 /* Workspace bytes for memoroid_discounted_return and memoroid_gae (a small
- * block: a header and one affine map per range of a tape, about 78 KB; a
- * call launches one or two kernels and keeps nothing in it afterwards). */
+ * block: a header and one affine map per range of a tape, about 152 KB; a
+ * call clears the header and launches one kernel, and keeps nothing in it
+ * afterwards). */
 size_t memoroid_returns_workspace_bytes(int64_t B, int64_t L);
 
 /*
