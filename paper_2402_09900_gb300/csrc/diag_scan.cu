@@ -954,11 +954,14 @@ __device__ void segment_fix_tile(const Params& p, int64_t tid, int part, int npa
         corr = cmul2(cpow2(C::REV ? conj2(lam) : lam, k_lo - skip), corr);
     }
     for (int k0 = k_lo; k0 < k_hi; k0 += BATCH) {
-        float4 v[BATCH], aux[BATCH];
+        // forward, per-step lambda: the batch's multipliers load with its outputs (a
+        // load behind the previous row's store would wait for it)
+        float4 v[BATCH], aux[BATCH], mul[(!C::REV && C::PS) ? BATCH : 1];
 #pragma unroll
         for (int k = 0; k < BATCH; ++k) {
             if (k0 + k < k_hi) {
                 const int64_t t = C::REV ? t0 + nrows - 1 - (k0 + k) : t0 + k0 + k;
+                if constexpr (!C::REV && C::PS) mul[k] = p.lambda[(b * p.L + t) * p.D2 + col];
                 if (!C::FFM) v[k] = p.out[(b * p.L + t) * p.D2 + col];
                 else if (!C::REV) v[k] = ffm_load_planar(p.out + (b * p.L + t) * p.D2, p.D2, col);
                 if (C::REV) {
@@ -975,7 +978,8 @@ __device__ void segment_fix_tile(const Params& p, int64_t tid, int part, int npa
             if (k0 + k >= k_hi) break;
             const int64_t t = C::REV ? t0 + nrows - 1 - (k0 + k) : t0 + k0 + k;
             if (!C::REV) {
-                const float4 l = C::PS ? p.lambda[(b * p.L + t) * p.D2 + col] : lam;
+                float4 l = lam;
+                if constexpr (C::PS) l = mul[k];
                 corr = cmul2(l, corr);
             } else {
                 const float4 m = (t == p.L - 1) ? one2()
