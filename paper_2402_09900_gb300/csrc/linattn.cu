@@ -257,8 +257,10 @@ __device__ __forceinline__ void tma_tile(uint32_t dst, const CUtensorMap* map, i
 // Scales row r of a 128-byte swizzled [T x D] bf16 tile by w[r] in place: one
 // thread per (row, 64-channel chunk) while there are enough threads, each
 // with one weight and eight 16-byte units (conflict-free: the swizzle spreads
-// the same unit of 8 consecutive rows over 8 bank groups).
-template <int D, int NT = kThreads, typename WFn>
+// the same unit of 8 consecutive rows over 8 bank groups).  SELECT: rows of
+// weight 0 become exact zeros (the forward's, so that a non-finite q or k stays
+// in its episode).
+template <int D, int NT = kThreads, bool SELECT = false, typename WFn>
 __device__ __forceinline__ void scale_rows_sw(unsigned char* tile, int tid, WFn weight) {
     constexpr int CHUNKS = D / 64;
     constexpr int UNITS = 8 * CHUNKS * T / NT;  // units per thread (NT threads)
@@ -282,6 +284,7 @@ __device__ __forceinline__ void scale_rows_sw(unsigned char* tile, int tid, WFn 
         u.z = pack_bf16x2(f.x * w, f.y * w);
         f = unpack_bf16x2(u.w);
         u.w = pack_bf16x2(f.x * w, f.y * w);
+        if (SELECT && w == 0.f) u = make_uint4(0u, 0u, 0u, 0u);
         *reinterpret_cast<uint4*>(a) = u;
     }
 }
@@ -811,7 +814,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
         {
             const float lend = mc.lam2[T - 1];
             const int ls = mc.last_start;
-            scale_rows_sw<D>(smem + (stage_k(s) - sbase), tid,
+            scale_rows_sw<D, kThreads, !BWD>(smem + (stage_k(s) - sbase), tid,
                              [&](int r) { return r >= ls ? fast_exp2(lend - mc.lam2[r]) : 0.f; });
         }
         // the previous tile's output stores, which read stage s ^ 1, have drained
@@ -879,7 +882,11 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                 tc::ld16_nowait(lane_base + S::COL_YI + j0 + 16, yi + 16);
             }
             tc::ld_wait();
-            const float dn = have_prev ? fmaf(w_in, __uint_as_float(ni[0]), __uint_as_float(na[0])) : __uint_as_float(na[0]);
+            // rows whose episode began in this tile take no inter-tile term (a select:
+            // a non-finite incoming state does not cross the begin flag)
+            const bool inter = w_in != 0.f;
+            const float dn = have_prev && inter ? fmaf(w_in, __uint_as_float(ni[0]), __uint_as_float(na[0]))
+                                                : __uint_as_float(na[0]);
             if (half == 0 && p.den != nullptr && t < r_hi) p.den[(b * p.L + t0 + t) * p.H + h] = dn;
             const float inv = 1.f / dn;
             unsigned char* yst = smem + s * S::STAGE + Y_OFF + t * 128;  // row t of chunk 0
@@ -889,7 +896,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                     o[e] = __uint_as_float(ya[x + e]);
-                    if (have_prev) o[e] = fmaf(w_in, __uint_as_float(yi[x + e]), o[e]);
+                    if (have_prev) o[e] = inter ? fmaf(w_in, __uint_as_float(yi[x + e]), o[e]) : o[e];
                     o[e] *= inv;
                 }
                 const int j = j0 + x;
@@ -932,7 +939,7 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                     }
                     vi = v0 + v1;
                 }
-                ofold = have_prev ? fmaf(w_in, vi, rsum) : rsum;
+                ofold = (have_prev && w_in != 0.f) ? fmaf(w_in, vi, rsum) : rsum;
                 __syncthreads();  // every row sum is read before the z terms overwrite the slots
             }
             // BWD: z_t = w_in_t q_t . (S_{c-1} dy_t), the inter output dotted with q
@@ -955,11 +962,12 @@ __global__ void __launch_bounds__(kThreads, 1) fwd_kernel(const __grid_constant_
                     for (int x = 0; x < 32; x += 4) {
                         float4 o = make_float4(__uint_as_float(ya[x]), __uint_as_float(ya[x + 1]),
                                                __uint_as_float(ya[x + 2]), __uint_as_float(ya[x + 3]));
-                        if (have_prev) {
-                            o.x = fmaf(w_in, __uint_as_float(yi[x]), o.x);
-                            o.y = fmaf(w_in, __uint_as_float(yi[x + 1]), o.y);
-                            o.z = fmaf(w_in, __uint_as_float(yi[x + 2]), o.z);
-                            o.w = fmaf(w_in, __uint_as_float(yi[x + 3]), o.w);
+                        if (have_prev) {  // the forward: a select where w_in = 0, as above
+                            const bool in2 = BWD || w_in != 0.f;
+                            o.x = in2 ? fmaf(w_in, __uint_as_float(yi[x]), o.x) : o.x;
+                            o.y = in2 ? fmaf(w_in, __uint_as_float(yi[x + 1]), o.y) : o.y;
+                            o.z = in2 ? fmaf(w_in, __uint_as_float(yi[x + 2]), o.z) : o.z;
+                            o.w = in2 ? fmaf(w_in, __uint_as_float(yi[x + 3]), o.w) : o.w;
                         }
                         if (FOLD) {
                             o.x += ofold;
@@ -1389,8 +1397,8 @@ __global__ void __launch_bounds__(kThreads, 1) seg_state_kernel(const __grid_con
         } else {
             const float lend = mc.lam2[T - 1];
             const int ls = mc.last_start;
-            scale_rows_sw<D>(smem + st * S::STAGE, tid,
-                             [&](int r) { return r >= ls ? fast_exp2(off + lend - mc.lam2[r]) : 0.f; });
+            scale_rows_sw<D, kThreads, true>(smem + st * S::STAGE, tid,
+                                             [&](int r) { return r >= ls ? fast_exp2(off + lend - mc.lam2[r]) : 0.f; });
         }
         off += mc.lam2[T - 1];
         tc::fence_smem_to_async();

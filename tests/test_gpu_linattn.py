@@ -171,6 +171,33 @@ def test_fwd_episode_isolation_bitwise():
     assert not np.array_equal(y0[0, s:e], y1[0, s:e])
 
 
+@pytest.mark.parametrize("d", [64, 128])
+def test_fwd_nonfinite_q_k_confined_to_their_episode(d):
+    # a NaN in q (one episode) and in k (another, ending in the middle of a tile) stays
+    # in its episode: every other episode's outputs are bit for bit those of the tape
+    # without them (the masks, the rows scaled into the state and the inter-tile term
+    # are selects, not products).  v is not covered: the tile-wide contractions
+    # multiply it by the zero weights of other episodes' rows.
+    t = tapegen.linattn_tape(1, 6000, 2, d, d, seed=tapegen.seed_for(59), mean=300.0, with_grad=False)
+    y0, s0 = run_gpu_fwd(t)
+    starts = np.flatnonzero(t["start"][0])
+    spans = [(int(starts[i]), int(starts[i + 1])) for i in (4, 9)]
+    t2 = dict(t)
+    nan = np.uint16(0x7FC0)
+    for key, (s, e) in zip(("q", "k"), spans):
+        a = t[key].copy()
+        a[0, s:e, 0, 3] = nan
+        t2[key] = a
+    y1, s1 = run_gpu_fwd(t2)
+    outside = np.ones(6000, dtype=bool)
+    for s, e in spans:
+        outside[s:e] = False
+        assert np.isnan(y1[0, s:e, 0]).any()
+    assert np.array_equal(y0[0, outside], y1[0, outside])
+    assert np.array_equal(y0[0, :, 1], y1[0, :, 1])  # the other head
+    assert np.array_equal(s0, s1)
+
+
 def test_fwd_deterministic():
     t = tapegen.linattn_tape(1, 5000, 2, 128, 128, seed=tapegen.seed_for(58), mean=500.0, gamma_mode="step",
                              with_grad=False)
