@@ -50,9 +50,17 @@ EncodeTiledFn encode_tiled() {
     return fn;
 }
 
-uint32_t tagged_epoch(const void* workspace, size_t region_end, bool* clear) {
+uint32_t tagged_epoch(const void* workspace, size_t region_end, cudaStream_t stream, bool* clear) {
     uint64_t c = 0;
     while ((c & 0x7fffffffull) == 0) c = g_epoch.fetch_add(1u);
+    // a call captured into a graph replays this tag every time: its region is
+    // cleared on every replay, and the registry, which records clears already
+    // done, is left as it is (the captured clear has not run)
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(stream, &cap) != cudaSuccess || cap != cudaStreamCaptureStatusNone) {
+        *clear = true;
+        return static_cast<uint32_t>(c & 0x7fffffffull);
+    }
     const uint64_t generation = c >> 31;
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess) dev = -1;

@@ -1290,7 +1290,7 @@ memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
     if (!make_maps(p, a, C::T, C::REV)) return MEMOROID_ERR_CUDA;
     // the summaries' tag; their region is zeroed where an old word could carry it
     bool clear = false;
-    p.epoch = tagged_epoch(a.workspace, l.gpart_off, &clear);
+    p.epoch = tagged_epoch(a.workspace, l.gpart_off, s, &clear);
     if (clear && cudaMemsetAsync(static_cast<unsigned char*>(a.workspace) + l.node_off, 0, l.gpart_off - l.node_off, s) !=
                      cudaSuccess)
         return MEMOROID_ERR_CUDA;

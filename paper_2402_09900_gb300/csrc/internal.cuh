@@ -45,7 +45,8 @@ DebugKnobs debug_knobs();
 // reaches further than the last clear.  So a summary word with this launch's
 // tag was written by this launch: every earlier write of the same tag is in a
 // past generation, and the region was cleared since.
-uint32_t tagged_epoch(const void* workspace, size_t region_end, bool* clear);
+// Under stream capture (a graph replays the tag), *clear is always true.
+uint32_t tagged_epoch(const void* workspace, size_t region_end, cudaStream_t stream, bool* clear);
 
 // Launches a kernel that follows another kernel on the stream with programmatic
 // stream serialization: it may be scheduled before that kernel completes and

@@ -365,7 +365,7 @@ memoroid_status_t launch(const float* r, const float* v, const uint8_t* start, f
     // B * G <= warps <= kMaxWarps whenever G > 1: the maps fit the workspace.  The
     // maps' tag; their region is zeroed where an old word could carry it.
     bool clear = false;
-    const uint32_t epoch = tagged_epoch(workspace, kHeaderBytes + kMapBytes, &clear);
+    const uint32_t epoch = tagged_epoch(workspace, kHeaderBytes + kMapBytes, s, &clear);
     if (cudaMemsetAsync(ws, 0, clear ? kHeaderBytes + kMapBytes : kHeaderBytes, s) != cudaSuccess)
         return MEMOROID_ERR_CUDA;
     const Params p{r, v, start, boot, out, reinterpret_cast<unsigned long long*>(ws + kHeaderBytes),
