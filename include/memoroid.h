@@ -25,6 +25,13 @@
  *     initial state, means the tape starts from the monoid identity e_I.
  *   - Gradients of complex inputs follow PyTorch's convention
  *     (grad = dL/dRe + i dL/dIm).
+ *   - Calls may be captured into a CUDA graph on a capturing stream (they
+ *     allocate nothing and make no synchronous call): a captured call clears
+ *     the part of its workspace it must read fresh on every replay, so
+ *     replays with new data in the captured buffers are correct.  Calls that
+ *     share a workspace must not overlap in time, captured or not.  (The
+ *     workspace-free memoroid_scan_diag_fwd_static must make its first call
+ *     on a device outside any capture.)
  */
 #ifndef MEMOROID_H
 #define MEMOROID_H
