@@ -136,12 +136,8 @@ __host__ __device__ __forceinline__ int64_t lmin(int64_t a, int64_t b) { return 
 __host__ __device__ __forceinline__ int64_t lmax(int64_t a, int64_t b) { return a > b ? a : b; }
 
 // ---- FFM layout: one lane's two channels (2 lane, 2 lane + 1 of the slab) ----
-// Staged forward input: x~ of the slab's rows i, repeated over the columns
-// (rows of 64 / c floats, packed).
-__device__ __forceinline__ float4 ffm_x_pair(const Params& p, const float4* buf, int r, int lane) {
-    const float* x = reinterpret_cast<const float*>(buf) + r * (64 >> p.ffm_lc);
-    return make_float4(x[(2 * lane) >> p.ffm_lc], 0.f, x[(2 * lane + 1) >> p.ffm_lc], 0.f);
-}
+// The staged forward input holds x~ of the slab's rows i (rows of 64 / c
+// floats, packed); channel 2 lane reads element (2 lane) >> log2 c of its row.
 // Staged planar rows of a T-step tile: the Re halves of all rows (64 floats
 // each), then the Im halves.
 template <int T>
@@ -217,11 +213,13 @@ __device__ __forceinline__ float4 add2(float4 a, float4 b) {
 
 // ---- tile shapes -------------------------------------------------------------
 // W warps x R steps per warp; REV = backward; PS = per-step lambda; FFM = the
-// Fast and Forgetful Memory layout (broadcast input, planar states).
-template <int W_, int R_, bool REV_, bool PS_, bool FFM_ = false>
+// Fast and Forgetful Memory layout (broadcast input, planar states); LC =
+// log2 c fixed at compile time (the FFM forward), -1 = taken from the parameters.
+template <int W_, int R_, bool REV_, bool PS_, bool FFM_ = false, int LC_ = -1>
 struct Cfg {
     static constexpr int W = W_, R = R_, T = W_ * R_;
     static constexpr bool REV = REV_, PS = PS_, FFM = FFM_;
+    static constexpr int LC = LC_;
     static_assert(!(PS_ && FFM_), "the FFM multiplier is per channel");
     static constexpr int UNROLL = REV_ ? UNROLL_BWD : (FFM_ ? UNROLL_FFM_FWD : UNROLL_FWD);
     // arrays staged per tile: input [, h (backward)] [, lambda (per step)]
@@ -632,6 +630,19 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
     }
     if (!landed && lane == 0) *s_abort = 1;
 
+    // FFM forward: this lane's two x~ values per staged row (rows of 64 / c
+    // floats); from c = 2 on, both channels of a lane belong to the same row i
+    const int lcx = C::LC >= 0 ? C::LC : p.ffm_lc;
+    const int xrow = 64 >> lcx;
+    const float* xs = reinterpret_cast<const float*>(s_in) + warp * R * xrow;
+    const int xi0 = (2 * lane) >> lcx, xi1 = lcx >= 1 ? xi0 : xi0 + 1;
+    auto xpair = [&](int k) { return make_float4(xs[k * xrow + xi0], 0.f, xs[k * xrow + xi1], 0.f); };
+    // loops without per-step tests (a per-channel lambda): a whole warp range with
+    // no begin flag; in reverse also no flag at the step after it (bits 0..R of
+    // bmask), and neither the tape's first nor its last step inside it
+    const bool plain = !C::PS && nv == R &&
+                       (C::REV ? ((bmask & ((2u << R) - 1u)) == 0u && ts > 0 && ts + R < p.L) : rmask == 0u);
+
     // phase 1: aggregate of this warp's steps, from the identity, in processing order
     float4 a = one2(), x = zero2();
     if (landed && !C::PS) {
@@ -640,18 +651,26 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
         // last step in reverse), taken once by repeated squaring
         const uint32_t rv = rmask & ((nv >= 32) ? 0xffffffffu : ((1u << nv) - 1u));
         if (!C::REV) {
-            // FFM: this lane's two x~ values per staged row (rows of 64 / c floats)
-            const int xrow = 64 >> p.ffm_lc;
-            const float* xs = reinterpret_cast<const float*>(s_in) + warp * R * xrow;
-            const int xi0 = (2 * lane) >> p.ffm_lc, xi1 = (2 * lane + 1) >> p.ffm_lc;
+            if (plain) {
 #pragma unroll C::UNROLL
-            for (int k = 0; k < R; ++k) {
-                if (k < nv) {
-                    const float4 uu = C::FFM ? make_float4(xs[k * xrow + xi0], 0.f, xs[k * xrow + xi1], 0.f) : sin[k * 32];
-                    x = ((rmask >> k) & 1u) ? uu : cfma2(lam, x, uu);
+                for (int k = 0; k < R; ++k) x = cfma2(lam, x, C::FFM ? xpair(k) : sin[k * 32]);
+            } else {
+#pragma unroll C::UNROLL
+                for (int k = 0; k < R; ++k) {
+                    if (k < nv) {
+                        const float4 uu = C::FFM ? xpair(k) : sin[k * 32];
+                        x = ((rmask >> k) & 1u) ? uu : cfma2(lam, x, uu);
+                    }
                 }
             }
             a = cpow2(lam, rv ? nv - (31 - __clz(rv)) : nv);
+        } else if (plain) {
+#pragma unroll C::UNROLL
+            for (int kk = 0; kk < R; ++kk) {
+                const int k = R - 1 - kk;
+                x = cfma2(mlam, x, C::FFM ? ffm_planar_pair<C::T>(s_in, warp * R + k, lane) : sin[k * 32]);
+            }
+            a = cpow2(mlam, nv);
         } else {
 #pragma unroll C::UNROLL
             for (int kk = 0; kk < R; ++kk) {
@@ -722,23 +741,33 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
     if (!C::REV) {
         if (lane_ok) {
             float4* dst = p.out + (t.b * p.L + ts) * p.D2 + t.c2 + lane;
-            // FFM: planar rows (Re half, then Im half, D2 float2 each) and this lane's x~
-            const int xrow = 64 >> p.ffm_lc;
-            const float* xs = reinterpret_cast<const float*>(s_in) + warp * R * xrow;
-            const int xi0 = (2 * lane) >> p.ffm_lc, xi1 = (2 * lane + 1) >> p.ffm_lc;
+            // FFM: planar rows (Re half, then Im half, D2 float2 each)
             float2* pre = reinterpret_cast<float2*>(p.out + (t.b * p.L + ts) * p.D2) + t.c2 + lane;
             const int64_t prow = 2 * p.D2;  // float2 per planar row
+            if (plain) {
 #pragma unroll C::UNROLL
-            for (int k = 0; k < R; ++k) {
-                if (k < nv) {
-                    const float4 uu = C::FFM ? make_float4(xs[k * xrow + xi0], 0.f, xs[k * xrow + xi1], 0.f) : sin[k * 32];
-                    const float4 ll = C::PS ? sl[k * 32] : lam;
-                    c = ((rmask >> k) & 1u) ? uu : cfma2(ll, c, uu);
+                for (int k = 0; k < R; ++k) {
+                    c = cfma2(lam, c, C::FFM ? xpair(k) : sin[k * 32]);
                     if (C::FFM) {
                         __stcs(pre + k * prow, make_float2(c.x, c.z));
                         __stcs(pre + k * prow + p.D2, make_float2(c.y, c.w));
                     } else {
                         __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
+                    }
+                }
+            } else {
+#pragma unroll C::UNROLL
+                for (int k = 0; k < R; ++k) {
+                    if (k < nv) {
+                        const float4 uu = C::FFM ? xpair(k) : sin[k * 32];
+                        const float4 ll = C::PS ? sl[k * 32] : lam;
+                        c = ((rmask >> k) & 1u) ? uu : cfma2(ll, c, uu);
+                        if (C::FFM) {
+                            __stcs(pre + k * prow, make_float2(c.x, c.z));
+                            __stcs(pre + k * prow + p.D2, make_float2(c.y, c.w));
+                        } else {
+                            __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
+                        }
                     }
                 }
             }
@@ -768,14 +797,8 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
             const bool gx_writer = lane_ok && (lane & (grp - 1)) == 0;
             float* gxw = C::FFM ? p.ffm_gx + (t.b * p.L + ts) * p.ffm_m + ((2 * (t.c2 + lane)) >> lc) : nullptr;
             const int64_t gxrow = p.ffm_m;
-#pragma unroll C::UNROLL
-            for (int kk = 0; kk < R; ++kk) {
-                const int k = R - 1 - kk;
-                if (k >= nv) continue;
-                const int64_t tt = ts + k;
-                const float4 gg = C::FFM ? ffm_planar_pair<C::T>(s_in, warp * R + k, lane) : sin[k * 32];
-                const float4 m = (tt == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
-                c = ((rmask >> k) & 1u) ? gg : cfma2(m, c, gg);
+            // step k's output: grad_u, or the FFM's grad_x~ (summed over the row's lanes)
+            auto emit = [&](int k) {
                 if (C::FFM) {
                     float* g = gxw + k * gxrow;
                     if (lc == 0) {
@@ -787,23 +810,47 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
                         if (grp > 4) v += __shfl_xor_sync(0xffffffffu, v, 4);
                         if (gx_writer) __stcs(g, v);
                     }
-                } else
-                    __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
-                float4 gl = zero2();
-                if (!((bmask >> k) & 1u) && lane_ok) {
-                    float4 hp;
-                    if (tt > 0) hp = C::FFM ? ffm_planar_pair<C::T>(s_h, warp * R + k, lane) : sh[k * 32];
-                    else hp = (p.h0 != nullptr) ? p.h0[t.b * p.D2 + t.c2 + lane] : zero2();
-                    gl = cmul2(c, conj2(hp));
-                }
-                if (C::PS) {
-                    if (p.grad_lambda != nullptr) __stcs(p.grad_lambda + (t.b * p.L + tt) * p.D2 + t.c2 + lane, gl);
                 } else {
-                    acc = add2(acc, gl);
+                    __stcs(dst + static_cast<int64_t>(k) * p.D2, c);
                 }
-                if (tt == 0 && p.grad_h0 != nullptr && lane_ok) {
-                    const float4 l0 = C::PS ? p.lambda[(t.b * p.L) * p.D2 + t.c2 + lane] : lam;
-                    p.grad_h0[t.b * p.D2 + t.c2 + lane] = (bmask & 1u) ? zero2() : cmul2(conj2(l0), c);
+            };
+            if (plain) {
+#pragma unroll C::UNROLL
+                for (int kk = 0; kk < R; ++kk) {
+                    const int k = R - 1 - kk;
+                    c = cfma2(mlam, c, C::FFM ? ffm_planar_pair<C::T>(s_in, warp * R + k, lane) : sin[k * 32]);
+                    emit(k);
+                    if (lane_ok) {
+                        const float4 hp = C::FFM ? ffm_planar_pair<C::T>(s_h, warp * R + k, lane) : sh[k * 32];
+                        acc = add2(acc, cmul2(c, conj2(hp)));
+                    }
+                }
+            } else {
+#pragma unroll C::UNROLL
+                for (int kk = 0; kk < R; ++kk) {
+                    const int k = R - 1 - kk;
+                    if (k >= nv) continue;
+                    const int64_t tt = ts + k;
+                    const float4 gg = C::FFM ? ffm_planar_pair<C::T>(s_in, warp * R + k, lane) : sin[k * 32];
+                    const float4 m = (tt == p.L - 1) ? one2() : (C::PS ? conj2(sl[k * 32]) : mlam);
+                    c = ((rmask >> k) & 1u) ? gg : cfma2(m, c, gg);
+                    emit(k);
+                    float4 gl = zero2();
+                    if (!((bmask >> k) & 1u) && lane_ok) {
+                        float4 hp;
+                        if (tt > 0) hp = C::FFM ? ffm_planar_pair<C::T>(s_h, warp * R + k, lane) : sh[k * 32];
+                        else hp = (p.h0 != nullptr) ? p.h0[t.b * p.D2 + t.c2 + lane] : zero2();
+                        gl = cmul2(c, conj2(hp));
+                    }
+                    if (C::PS) {
+                        if (p.grad_lambda != nullptr) __stcs(p.grad_lambda + (t.b * p.L + tt) * p.D2 + t.c2 + lane, gl);
+                    } else {
+                        acc = add2(acc, gl);
+                    }
+                    if (tt == 0 && p.grad_h0 != nullptr && lane_ok) {
+                        const float4 l0 = C::PS ? p.lambda[(t.b * p.L) * p.D2 + t.c2 + lane] : lam;
+                        p.grad_h0[t.b * p.D2 + t.c2 + lane] = (bmask & 1u) ? zero2() : cmul2(conj2(l0), c);
+                    }
                 }
             }
         }
@@ -1138,7 +1185,10 @@ using BwdC = Cfg<8, 12, true, false>;
 using BwdS = Cfg<8, 8, true, true>;
 // The FFM forward stages only x~ (a few bytes per step), so larger tiles pay:
 // 6 x 31 (186-step tiles) was the measured best on GB300.
-using FwdF = Cfg<6, 31, false, false, true>;
+// The forward is compiled for each c (log2 c = LC), so the lanes' x~ offsets
+// are constants.
+template <int LC>
+using FwdF = Cfg<6, 31, false, false, true, LC>;
 using BwdF = Cfg<8, 12, true, false, true>;
 
 // Segments per chain: enough segment chains that a tile's predecessor was
@@ -1335,7 +1385,15 @@ int kernels_per_call(int64_t B, int64_t L, int64_t D, int per_step, int backward
 }
 
 memoroid_status_t launch_fwd(const Args& a, cudaStream_t s) {
-    if (a.ffm_c > 0) return launch<FwdF>(a, s, nullptr);
+    switch (a.ffm_c) {
+        case 0: break;
+        case 1: return launch<FwdF<0>>(a, s, nullptr);
+        case 2: return launch<FwdF<1>>(a, s, nullptr);
+        case 4: return launch<FwdF<2>>(a, s, nullptr);
+        case 8: return launch<FwdF<3>>(a, s, nullptr);
+        case 16: return launch<FwdF<4>>(a, s, nullptr);
+        default: return MEMOROID_ERR_INVALID_ARG;
+    }
     return a.lambda_per_step ? launch<FwdS>(a, s, nullptr) : launch<FwdC>(a, s, nullptr);
 }
 
@@ -1425,7 +1483,7 @@ size_t ffm_workspace_bytes(int64_t B, int64_t L, int64_t m, int64_t c) {
 int ffm_kernels_per_call(int64_t B, int64_t L, int64_t m, int64_t c, int backward, int with_param_grads) {
     if (B <= 0 || L <= 0 || m <= 0 || c <= 0) return 0;
     const int64_t D = m * c;
-    const Layout l = layout(B, L, D, backward ? BwdF::T : FwdF::T, backward != 0);
+    const Layout l = layout(B, L, D, backward ? BwdF::T : FwdF<0>::T, backward != 0);
     int n = 1 + (l.sg.G > 1 ? 3 : 1);  // lambda + scan [+ segment carries + fix-up]
     if (backward && with_param_grads) n += 3;  // grad_lambda reduction + parameter gradients
     return n;
