@@ -822,7 +822,7 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
                     emit(k);
                     if (lane_ok) {
                         const float4 hp = C::FFM ? ffm_planar_pair<C::T>(s_h, warp * R + k, lane) : sh[k * 32];
-                        acc = add2(acc, cmul2(c, conj2(hp)));
+                        acc = cfma2(c, conj2(hp), acc);
                     }
                 }
             } else {
@@ -840,13 +840,11 @@ __global__ void __launch_bounds__(C::THREADS) diag_scan_kernel(const __grid_cons
                         float4 hp;
                         if (tt > 0) hp = C::FFM ? ffm_planar_pair<C::T>(s_h, warp * R + k, lane) : sh[k * 32];
                         else hp = (p.h0 != nullptr) ? p.h0[t.b * p.D2 + t.c2 + lane] : zero2();
-                        gl = cmul2(c, conj2(hp));
+                        if (C::PS) gl = cmul2(c, conj2(hp));
+                        else acc = cfma2(c, conj2(hp), acc);  // the same fused form as the loop above
                     }
-                    if (C::PS) {
-                        if (p.grad_lambda != nullptr) __stcs(p.grad_lambda + (t.b * p.L + tt) * p.D2 + t.c2 + lane, gl);
-                    } else {
-                        acc = add2(acc, gl);
-                    }
+                    if (C::PS && p.grad_lambda != nullptr)
+                        __stcs(p.grad_lambda + (t.b * p.L + tt) * p.D2 + t.c2 + lane, gl);
                     if (tt == 0 && p.grad_h0 != nullptr && lane_ok) {
                         const float4 l0 = C::PS ? p.lambda[(t.b * p.L) * p.D2 + t.c2 + lane] : lam;
                         p.grad_h0[t.b * p.D2 + t.c2 + lane] = (bmask & 1u) ? zero2() : cmul2(conj2(l0), c);
