@@ -1329,6 +1329,7 @@ memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
     const Segs sg = l.sg;
     const int64_t n_tickets = sg.Q * l.n_chains * sg.G;
     if (n_tickets >= 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;
+    if (l.total > a.workspace_bytes) return MEMOROID_ERR_WORKSPACE;  // this tile shape's layout must fit
     if (cudaMemsetAsync(a.workspace, 0, kHeaderBytes, s) != cudaSuccess) return MEMOROID_ERR_CUDA;
     auto kernel = diag_scan_kernel<C>;
     if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1504,7 +1505,7 @@ memoroid_status_t launch_ffm(const FfmArgs& f, cudaStream_t s) {
     a.L = f.L;
     a.D = D;
     a.workspace = f.workspace;
-    a.workspace_bytes = f.workspace_bytes;
+    a.workspace_bytes = ffm_lambda_off(f.B, f.L, D);  // the scan's part, before lambda and its gradient
     a.ffm_c = static_cast<int>(f.c);
     a.ffm_m = f.m;
     if (!f.backward) {
