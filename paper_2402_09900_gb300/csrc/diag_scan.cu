@@ -1176,7 +1176,12 @@ __global__ void __launch_bounds__(RED_PARTS) reduce_final_kernel(const double* _
 namespace {
 
 // Tile shapes (scan warps, steps per warp): the measured best on GB300.
-using FwdC = Cfg<4, 24, false, false>;
+// The forward (per-channel lambda) takes 5 x 20 tiles where every chain is one
+// segment and 5 x 24 where chains are cut into segments (measured: the
+// 2^20-step, 256-channel tape 0.696 ms with 4 x 24, 0.689 with 5 x 20, 0.680
+// with 5 x 24; 64 tapes x 16384 steps x 128 channels 0.349 / 0.347 / 0.364 ms).
+using FwdC = Cfg<5, 20, false, false>;
+using FwdL = Cfg<5, 24, false, false>;
 // per-step lambda (two staged arrays forward, three backward)
 using FwdS = Cfg<4, 12, false, true>;
 using BwdC = Cfg<8, 12, true, false>;
@@ -1364,9 +1369,9 @@ memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t D) {
     size_t m = 0;
-    const int Ts[4] = {FwdC::T, FwdS::T, BwdC::T, BwdS::T};
-    const bool revs[4] = {false, false, true, true};
-    for (int i = 0; i < 4; ++i) {
+    const int Ts[5] = {FwdC::T, FwdL::T, FwdS::T, BwdC::T, BwdS::T};
+    const bool revs[5] = {false, false, false, true, true};
+    for (int i = 0; i < 5; ++i) {
         const size_t t = layout(B, L, D, Ts[i], revs[i]).total;
         if (t > m) m = t;
     }
@@ -1374,9 +1379,13 @@ size_t workspace_bytes(int64_t B, int64_t L, int64_t D) {
 }
 
 
+// the forward's tiles for a per-channel lambda: the longer ones where chains are cut into segments
+static bool fwd_long_tiles(int64_t B, int64_t D) { return B * ((D + SLAB - 1) / SLAB) < CHAINS_NO_SEG; }
+
 int kernels_per_call(int64_t B, int64_t L, int64_t D, int per_step, int backward, int with_grad_lambda) {
     if (B <= 0 || L <= 0 || D <= 0) return 0;
-    const int T = backward ? (per_step ? BwdS::T : BwdC::T) : (per_step ? FwdS::T : FwdC::T);
+    const int Tf = fwd_long_tiles(B, D) ? FwdL::T : FwdC::T;
+    const int T = backward ? (per_step ? BwdS::T : BwdC::T) : (per_step ? FwdS::T : Tf);
     const Layout l = layout(B, L, D, T, backward != 0);
     int n = l.sg.G > 1 ? 3 : 1;  // scan [+ segment carries + fix-up]
     if (backward && !per_step && with_grad_lambda) n += 2;  // grad_lambda reduction
@@ -1393,7 +1402,8 @@ memoroid_status_t launch_fwd(const Args& a, cudaStream_t s) {
         case 16: return launch<FwdF<4>>(a, s, nullptr);
         default: return MEMOROID_ERR_INVALID_ARG;
     }
-    return a.lambda_per_step ? launch<FwdS>(a, s, nullptr) : launch<FwdC>(a, s, nullptr);
+    if (a.lambda_per_step) return launch<FwdS>(a, s, nullptr);
+    return fwd_long_tiles(a.B, a.D) ? launch<FwdL>(a, s, nullptr) : launch<FwdC>(a, s, nullptr);
 }
 
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t s) {
