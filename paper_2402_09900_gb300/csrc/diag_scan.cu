@@ -1184,7 +1184,11 @@ using FwdC = Cfg<5, 20, false, false>;
 using FwdL = Cfg<5, 24, false, false>;
 // per-step lambda (two staged arrays forward, three backward)
 using FwdS = Cfg<4, 12, false, true>;
+// The backward likewise: 8 x 12 where every chain is one segment, 7 x 14 where
+// chains are cut into segments (measured: 1.006 / 1.001 ms on the 2^20-step,
+// 256-channel tape; 0.559 / 0.562 ms on the 64 tapes).
 using BwdC = Cfg<8, 12, true, false>;
+using BwdL = Cfg<7, 14, true, false>;
 using BwdS = Cfg<8, 8, true, true>;
 // The FFM forward stages only x~ (a few bytes per step), so larger tiles pay:
 // 6 x 31 (186-step tiles) was the measured best on GB300.
@@ -1369,9 +1373,9 @@ memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
 
 size_t workspace_bytes(int64_t B, int64_t L, int64_t D) {
     size_t m = 0;
-    const int Ts[5] = {FwdC::T, FwdL::T, FwdS::T, BwdC::T, BwdS::T};
-    const bool revs[5] = {false, false, false, true, true};
-    for (int i = 0; i < 5; ++i) {
+    const int Ts[6] = {FwdC::T, FwdL::T, FwdS::T, BwdC::T, BwdL::T, BwdS::T};
+    const bool revs[6] = {false, false, false, true, true, true};
+    for (int i = 0; i < 6; ++i) {
         const size_t t = layout(B, L, D, Ts[i], revs[i]).total;
         if (t > m) m = t;
     }
@@ -1379,13 +1383,14 @@ size_t workspace_bytes(int64_t B, int64_t L, int64_t D) {
 }
 
 
-// the forward's tiles for a per-channel lambda: the longer ones where chains are cut into segments
-static bool fwd_long_tiles(int64_t B, int64_t D) { return B * ((D + SLAB - 1) / SLAB) < CHAINS_NO_SEG; }
+// the tiles for a per-channel lambda: the longer ones where chains are cut into segments
+static bool long_tiles(int64_t B, int64_t D) { return B * ((D + SLAB - 1) / SLAB) < CHAINS_NO_SEG; }
 
 int kernels_per_call(int64_t B, int64_t L, int64_t D, int per_step, int backward, int with_grad_lambda) {
     if (B <= 0 || L <= 0 || D <= 0) return 0;
-    const int Tf = fwd_long_tiles(B, D) ? FwdL::T : FwdC::T;
-    const int T = backward ? (per_step ? BwdS::T : BwdC::T) : (per_step ? FwdS::T : Tf);
+    const bool lt = long_tiles(B, D);
+    const int T = backward ? (per_step ? BwdS::T : (lt ? BwdL::T : BwdC::T))
+                           : (per_step ? FwdS::T : (lt ? FwdL::T : FwdC::T));
     const Layout l = layout(B, L, D, T, backward != 0);
     int n = l.sg.G > 1 ? 3 : 1;  // scan [+ segment carries + fix-up]
     if (backward && !per_step && with_grad_lambda) n += 2;  // grad_lambda reduction
@@ -1403,14 +1408,16 @@ memoroid_status_t launch_fwd(const Args& a, cudaStream_t s) {
         default: return MEMOROID_ERR_INVALID_ARG;
     }
     if (a.lambda_per_step) return launch<FwdS>(a, s, nullptr);
-    return fwd_long_tiles(a.B, a.D) ? launch<FwdL>(a, s, nullptr) : launch<FwdC>(a, s, nullptr);
+    return long_tiles(a.B, a.D) ? launch<FwdL>(a, s, nullptr) : launch<FwdC>(a, s, nullptr);
 }
 
 memoroid_status_t launch_bwd(const Args& a, cudaStream_t s) {
     const bool ps = a.lambda_per_step != 0;
     Layout l{};
     const memoroid_status_t st = a.ffm_c > 0 ? launch<BwdF>(a, s, &l)
-                                             : (ps ? launch<BwdS>(a, s, &l) : launch<BwdC>(a, s, &l));
+                                 : ps        ? launch<BwdS>(a, s, &l)
+                                 : long_tiles(a.B, a.D) ? launch<BwdL>(a, s, &l)
+                                                        : launch<BwdC>(a, s, &l);
     if (st != MEMOROID_OK) return st;
     if (!ps && a.grad_lambda != nullptr) {
         unsigned char* ws = static_cast<unsigned char*>(a.workspace);
