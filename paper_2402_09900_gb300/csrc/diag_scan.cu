@@ -1206,9 +1206,12 @@ using BwdF = Cfg<8, 12, true, false, true>;
 // 16384 steps x 128 channels, half of them one episode: fwd 0.474 -> 0.361 ms,
 // bwd 0.703 -> 0.600 ms; 4 chains keep their segments: with a quarter of the
 // target the 2^20-step, 256-channel tape took 0.733 / 1.162 instead of 0.700 /
-// 1.089 ms).
-constexpr int64_t TARGET_SC = 512;
-constexpr int64_t TARGET_SC_BWD = 256;
+// 1.089 ms).  The targets were swept again with the current tiles on that tape:
+// the times move by up to 2% between neighbouring counts (forward 384 / 416 /
+// 448 / 480 / 512 segment chains: 0.675 / 0.674 / 0.676 / 0.695 / 0.680 ms;
+// backward 208 / 224 / 228 / 240 / 256: 1.010 / 0.994 / 1.014 / 1.014 / 1.001 ms).
+constexpr int64_t TARGET_SC = 416;
+constexpr int64_t TARGET_SC_BWD = 224;
 constexpr int64_t MAX_SEG = 192;
 constexpr int64_t MIN_SEG_TILES = 8;
 constexpr int64_t CHAINS_NO_SEG = 128;
