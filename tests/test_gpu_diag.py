@@ -74,7 +74,8 @@ def check(t, h0=None, g_last=None, tol=TOL):
 # ---------------------------------------------------------------------------
 
 @pytest.mark.parametrize("per_step", [False, True])
-@pytest.mark.parametrize("B,L,D", [(1, 4096, 64), (3, 1000, 192), (2, 777, 70), (1, 333, 2)])
+@pytest.mark.parametrize("B,L,D", [(1, 4096, 64), (3, 1000, 192), (2, 777, 70), (1, 333, 2),
+                                   (130, 517, 64)])  # the last: >= 128 chains, the unsegmented tiles
 def test_parity_shapes(per_step, B, L, D):
     t = tapegen.diag_tape(B, L, D, seed=100 + L + D, mean=60.0, lambda_per_step=per_step, with_h0=True)
     t["start"][0, 0] = 0  # tape 0 continues an episode from h0
