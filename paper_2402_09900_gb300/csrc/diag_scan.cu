@@ -1210,8 +1210,12 @@ using BwdF = Cfg<8, 12, true, false, true>;
 // the times move by up to 2% between neighbouring counts (forward 384 / 416 /
 // 448 / 480 / 512 segment chains: 0.675 / 0.674 / 0.676 / 0.695 / 0.680 ms;
 // backward 208 / 224 / 228 / 240 / 256: 1.010 / 0.994 / 1.014 / 1.014 / 1.001 ms).
+// With a per-step lambda (other tiles, another CTA count per SM) the earlier
+// 512 / 256 stay: with 416 / 224 its forward took 1.114 instead of 1.036 ms.
 constexpr int64_t TARGET_SC = 416;
 constexpr int64_t TARGET_SC_BWD = 224;
+constexpr int64_t TARGET_SC_PS = 512;
+constexpr int64_t TARGET_SC_PS_BWD = 256;
 constexpr int64_t MAX_SEG = 192;
 constexpr int64_t MIN_SEG_TILES = 8;
 constexpr int64_t CHAINS_NO_SEG = 128;
@@ -1219,9 +1223,9 @@ constexpr int64_t CHAINS_NO_SEG = 128;
 struct Segs {
     int64_t G, Q;
 };
-Segs choose_segments(int64_t n_chains, int64_t n_tt, bool rev) {
+Segs choose_segments(int64_t n_chains, int64_t n_tt, bool rev, bool ps) {
     if (n_chains >= CHAINS_NO_SEG) return Segs{1, n_tt};
-    const int64_t target = rev ? TARGET_SC_BWD : TARGET_SC;
+    const int64_t target = ps ? (rev ? TARGET_SC_PS_BWD : TARGET_SC_PS) : (rev ? TARGET_SC_BWD : TARGET_SC);
     int64_t G = (target + n_chains - 1) / n_chains;
     G = lmin(G, lmin(MAX_SEG, n_tt / MIN_SEG_TILES));
     if (G < 1) G = 1;
@@ -1235,13 +1239,14 @@ struct Layout {
     size_t node_off, gpart_off, fix_off, pin_off, segc_off, sega_off, segb_off, rpart_off, total;
 };
 
-// Workspace layout for tiles of T steps (rev: the backward scan's segment target).
-Layout layout(int64_t B, int64_t L, int64_t D, int T, bool rev) {
+// Workspace layout for tiles of T steps (rev, ps: the segment target of the
+// backward scan, of a per-step lambda).
+Layout layout(int64_t B, int64_t L, int64_t D, int T, bool rev, bool ps) {
     Layout l{};
     l.n_slabs = (D + SLAB - 1) / SLAB;
     l.n_chains = B * l.n_slabs;
     l.n_tt = (L + T - 1) / T;
-    l.sg = choose_segments(l.n_chains, l.n_tt, rev);
+    l.sg = choose_segments(l.n_chains, l.n_tt, rev, ps);
     const size_t tiles = static_cast<size_t>(l.n_chains) * static_cast<size_t>(l.n_tt);
     const size_t nodes = static_cast<size_t>(l.n_chains) * static_cast<size_t>(l.sg.G * l.sg.Q);
     l.node_off = kHeaderBytes;
@@ -1337,7 +1342,7 @@ bool make_maps(Params& p, const Args& a, int T, bool backward) {
 // state entering each segment where it is missing.
 template <class C>
 memoroid_status_t launch(const Args& a, cudaStream_t s, Layout* out_layout) {
-    const Layout l = layout(a.B, a.L, a.D, C::T, C::REV);
+    const Layout l = layout(a.B, a.L, a.D, C::T, C::REV, C::PS);
     const Segs sg = l.sg;
     const int64_t n_tickets = sg.Q * l.n_chains * sg.G;
     if (n_tickets >= 0x7fffffffLL) return MEMOROID_ERR_UNSUPPORTED;
@@ -1378,8 +1383,9 @@ size_t workspace_bytes(int64_t B, int64_t L, int64_t D) {
     size_t m = 0;
     const int Ts[6] = {FwdC::T, FwdL::T, FwdS::T, BwdC::T, BwdL::T, BwdS::T};
     const bool revs[6] = {false, false, false, true, true, true};
+    const bool pss[6] = {false, false, true, false, false, true};
     for (int i = 0; i < 6; ++i) {
-        const size_t t = layout(B, L, D, Ts[i], revs[i]).total;
+        const size_t t = layout(B, L, D, Ts[i], revs[i], pss[i]).total;
         if (t > m) m = t;
     }
     return m;
@@ -1394,7 +1400,7 @@ int kernels_per_call(int64_t B, int64_t L, int64_t D, int per_step, int backward
     const bool lt = long_tiles(B, D);
     const int T = backward ? (per_step ? BwdS::T : (lt ? BwdL::T : BwdC::T))
                            : (per_step ? FwdS::T : (lt ? FwdL::T : FwdC::T));
-    const Layout l = layout(B, L, D, T, backward != 0);
+    const Layout l = layout(B, L, D, T, backward != 0, per_step != 0);
     int n = l.sg.G > 1 ? 3 : 1;  // scan [+ segment carries + fix-up]
     if (backward && !per_step && with_grad_lambda) n += 2;  // grad_lambda reduction
     return n;
@@ -1502,7 +1508,7 @@ size_t ffm_workspace_bytes(int64_t B, int64_t L, int64_t m, int64_t c) {
 int ffm_kernels_per_call(int64_t B, int64_t L, int64_t m, int64_t c, int backward, int with_param_grads) {
     if (B <= 0 || L <= 0 || m <= 0 || c <= 0) return 0;
     const int64_t D = m * c;
-    const Layout l = layout(B, L, D, backward ? BwdF::T : FwdF<0>::T, backward != 0);
+    const Layout l = layout(B, L, D, backward ? BwdF::T : FwdF<0>::T, backward != 0, false);
     int n = 1 + (l.sg.G > 1 ? 3 : 1);  // lambda + scan [+ segment carries + fix-up]
     if (backward && with_param_grads) n += 3;  // grad_lambda reduction + parameter gradients
     return n;
