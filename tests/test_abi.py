@@ -55,6 +55,19 @@ def test_workspace_queries(lib):
     assert lib.memoroid_offsets_workspace_bytes(1000) >= 256
 
 
+def test_diag_kernel_counts(lib):
+    # one tape of 256 channels is 4 chains, cut into segments: the scan, the segment
+    # carries and the fix-up; the backward adds the two grad_lambda reduction stages
+    assert lib.memoroid_scan_diag_kernels_per_call(1, 1 << 20, 256, 0, 0, 0) == 3
+    assert lib.memoroid_scan_diag_kernels_per_call(1, 1 << 20, 256, 0, 1, 1) == 5
+    assert lib.memoroid_scan_diag_kernels_per_call(1, 1 << 20, 256, 0, 1, 0) == 3
+    # 64 tapes of 128 channels are 128 chains, one segment each: the scan alone
+    assert lib.memoroid_scan_diag_kernels_per_call(64, 16384, 128, 0, 0, 0) == 1
+    assert lib.memoroid_scan_diag_kernels_per_call(64, 16384, 128, 0, 1, 1) == 3
+    # a per-step lambda has no grad_lambda reduction (its gradient is per step)
+    assert lib.memoroid_scan_diag_kernels_per_call(1, 1 << 20, 256, 1, 1, 1) == 3
+
+
 FAKE = 0x10000000  # 256-byte aligned dummy address, never dereferenced
 
 
