@@ -181,26 +181,43 @@ __device__ float walk(const Params& p, int64_t b, int64_t lo, int64_t hi, float 
         if (GAE) next_v = __shfl_sync(0xffffffffu, cur.v[0], 0);
 
         float x[kElems], m[kElems];
+        // a chunk inside [lo, hi) that ends before the tape's last step: no per-step range
+        // or tape-end tests (the same values as the general loop below)
+        const int64_t c0 = k * kChunk;
+        if (c0 >= lo && c0 + kChunk <= hi && c0 + kChunk < p.L) {
 #pragma unroll
-        for (int e = 0; e < kElems; ++e) {
-            const int64_t t = t0 + e;
-            if (t >= lo && t < hi) {
-                const bool last = t + 1 >= p.L;
-                // the successor: inside the lane's block (loaded from memory even past hi),
-                // or for the block's last step the next lane's first (hi for lane 31)
+            for (int e = 0; e < kElems; ++e) {
                 const bool sflag = e + 1 < kElems ? flag_of(cur, e + 1) : succ_flag;
-                const bool cont = !last && !sflag;  // the next step is in the same episode
-                m[e] = (last || cont) ? p.c : 0.f;
+                m[e] = sflag ? 0.f : p.c;
                 if (GAE) {
                     const float vn = e + 1 < kElems ? cur.v[e + 1] : succ_v;
-                    const float nv = last ? boot : (cont ? vn : 0.f);
-                    x[e] = fmaf(p.gamma, nv, cur.r[e]) - cur.v[e];
+                    x[e] = fmaf(p.gamma, sflag ? 0.f : vn, cur.r[e]) - cur.v[e];
                 } else {
                     x[e] = cur.r[e];
                 }
-            } else {
-                m[e] = 1.f;  // identity outside the range
-                x[e] = 0.f;
+            }
+        } else {
+#pragma unroll
+            for (int e = 0; e < kElems; ++e) {
+                const int64_t t = t0 + e;
+                if (t >= lo && t < hi) {
+                    const bool last = t + 1 >= p.L;
+                    // the successor: inside the lane's block (loaded from memory even past hi),
+                    // or for the block's last step the next lane's first (hi for lane 31)
+                    const bool sflag = e + 1 < kElems ? flag_of(cur, e + 1) : succ_flag;
+                    const bool cont = !last && !sflag;  // the next step is in the same episode
+                    m[e] = (last || cont) ? p.c : 0.f;
+                    if (GAE) {
+                        const float vn = e + 1 < kElems ? cur.v[e + 1] : succ_v;
+                        const float nv = last ? boot : (cont ? vn : 0.f);
+                        x[e] = fmaf(p.gamma, nv, cur.r[e]) - cur.v[e];
+                    } else {
+                        x[e] = cur.r[e];
+                    }
+                } else {
+                    m[e] = 1.f;  // identity outside the range
+                    x[e] = 0.f;
+                }
             }
         }
         // this lane's map: G at its first step as a function of G after its last
